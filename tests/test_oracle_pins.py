@@ -1,0 +1,413 @@
+"""Pins of the CPU oracle against what the paper and mathematics fix.
+
+None of these re-type the oracle's formulas: each compares the oracle with a
+brute-force definition on a tiny case, a library routine (torch's number
+format conversions, scipy's softmax, Triton's Philox), a closed form, an
+invariant, or a value printed in the paper (tests/golden/).
+"""
+import itertools
+import json
+import os
+import subprocess
+import sys
+import textwrap
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_13093_gb300 import workloads as wl
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def bits16(t):
+    return t.contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+def bits8(t):
+    return t.contiguous().view(torch.uint8).numpy()
+
+
+def tiny(with_bias=True, w_dtype="bf16", seed=7, V=37, d=13, d_l=5, rows=3,
+         n_keep=20, sessions=0, k=0):
+    return wl.make_workload(V=V, d=d, d_l=d_l, rows=rows, n_keep=n_keep,
+                            seed=seed, with_bias=with_bias, w_dtype=w_dtype,
+                            run_lo=2, run_hi=5, sessions=sessions, k=k)
+
+
+# ---------------------------------------------------------------------------
+# Eq. 9-13: split partial logits add up to the full head, bias once
+# ---------------------------------------------------------------------------
+
+def brute_full_head(h, W_full, bias):
+    """z[r, v] = sum_c h[r, c] W[v, c] + b[v] with explicit loops (Eq. 9)."""
+    R, d = h.shape
+    V = W_full.shape[0]
+    z = np.zeros((R, V))
+    for r in range(R):
+        for v in range(V):
+            acc = 0.0
+            for c in range(d):
+                acc += float(h[r, c]) * float(W_full[v, c])
+            z[r, v] = acc + (float(bias[v]) if bias is not None else 0.0)
+    return z
+
+
+@pytest.mark.parametrize("act_mode", ["fp32", "bf16"])
+def test_split_partials_equal_full_head(act_mode):
+    w = tiny()
+    ids = w.keep_ids.numpy()
+    h = w.h.numpy().astype(np.float64)
+    if act_mode == "bf16":
+        # the cloud half sees h rounded to bf16 (torch's conversion)
+        h[:, w.d_l:] = w.h[:, w.d_l:].to(torch.bfloat16).double().numpy()
+    W_full = torch.cat([w.W_l, w.W_h], dim=1).double().numpy()
+    z_full = brute_full_head(h, W_full, w.bias.numpy())[:, ids]
+    cloud = oracle.partial_logits(w.h_cloud.numpy(), bits16(w.W_h),
+                                  bias=w.bias.numpy(), keep_ids=ids,
+                                  clip=1e30, act_mode=act_mode)
+    local = oracle.local_partial(w.h_local.numpy(), bits16(w.W_l), ids)
+    np.testing.assert_allclose(cloud["y"] + local, z_full, rtol=1e-12, atol=1e-14)
+    # the bias enters exactly once: without it the sum drops by b[ids]
+    cloud0 = oracle.partial_logits(w.h_cloud.numpy(), bits16(w.W_h),
+                                   keep_ids=ids, clip=1e30, act_mode=act_mode)
+    np.testing.assert_allclose(cloud0["y"] + local + w.bias.numpy()[ids],
+                               z_full, rtol=1e-12, atol=1e-14)
+
+
+def test_fp8_partials_equal_full_head():
+    w = tiny(with_bias=False, w_dtype="fp8")
+    ids = w.keep_ids.numpy()
+    Wh = (w.W_h.float().double() * w.w_scale.double()[:, None]).numpy()  # torch decode
+    h = w.h.numpy().astype(np.float64)
+    z_ref = brute_full_head(h[:, w.d_l:], Wh, None)[:, ids]
+    cloud = oracle.partial_logits(w.h_cloud.numpy(), bits8(w.W_h), w_dtype="fp8",
+                                  w_scale=w.w_scale.numpy(), keep_ids=ids,
+                                  clip=1e30)
+    np.testing.assert_allclose(cloud["y"], z_ref, rtol=1e-12, atol=1e-14)
+
+
+def test_full_vocab_reduces_to_plain_matmul():
+    """keep_ids=None (mixed-language mode) is the plain GEMM over all V."""
+    w = tiny(with_bias=False, n_keep=37)
+    assert w.keep_ids is None
+    ref = w.h_cloud.double() @ w.W_h.double().T
+    out = oracle.partial_logits(w.h_cloud.numpy(), bits16(w.W_h), clip=1e30)
+    np.testing.assert_allclose(out["y"], ref.numpy(), rtol=1e-12)
+    assert out["codes"].shape == (w.rows, w.V)
+
+
+# ---------------------------------------------------------------------------
+# Eq. 18 with b = 8: quantizer invariants and closed forms
+# ---------------------------------------------------------------------------
+
+def test_quantizer_closed_form():
+    # s = 127/127 = 1 exactly; rint is half-to-even: -63.5 -> -64, 0.5 -> 0,
+    # 1.5 -> 2, 2.5 -> 2
+    y = np.array([[127.0, -63.5, 0.5, 1.5, 2.5, -127.0]])
+    codes, s = oracle.quantize_rows(y, clip=1e9)
+    assert s[0] == np.float32(1.0)
+    assert codes.tolist() == [[127, -64, 0, 2, 2, -127]]
+    # clipping happens before the row maximum: s = fl32(c/127)
+    codes, s = oracle.quantize_rows(np.array([[100.0, -5.0, 29.0]]), clip=30.0)
+    assert s[0] == np.float32(30.0 / 127.0)
+    assert codes[0, 0] == 127
+    # an all-zero row
+    codes, s = oracle.quantize_rows(np.zeros((1, 5)), clip=30.0)
+    assert s[0] == 0 and not codes.any()
+
+
+def test_quantizer_invariants():
+    rng = np.random.default_rng(3)
+    y = rng.normal(size=(64, 301)) * rng.uniform(0.01, 60, size=(64, 1))
+    y[5] = 0.0
+    clip = 30.0
+    codes, s = oracle.quantize_rows(y, clip)
+    yc = np.clip(y, -clip, clip)
+    s64 = s.astype(np.float64)
+    assert codes.dtype == np.int8
+    assert codes.min() >= -127 and codes.max() <= 127
+    err = np.abs(codes * s64[:, None] - yc)
+    assert np.all(err <= s64[:, None] / 2 * (1 + 1e-6) + 1e-300)
+    nz = np.any(yc != 0, axis=1)
+    assert np.all(np.abs(codes[nz]).max(axis=1) == 127)
+    assert s[5] == 0 and not codes[5].any()
+    # re-quantizing the dequantized payload reproduces it exactly
+    codes2, s2 = oracle.quantize_rows(codes * s64[:, None], clip)
+    assert np.array_equal(codes2, codes)
+    np.testing.assert_allclose(s2, s, rtol=1e-6)
+
+
+# ---------------------------------------------------------------------------
+# Eq. 21 payload model against the numbers the paper prints
+# ---------------------------------------------------------------------------
+
+def test_payload_matches_paper():
+    g = json.load(open(os.path.join(GOLDEN, "payload_eq21.json")))
+    V = g["V"]
+    code_bytes = oracle.payload_bytes(1, V) - 4          # minus the row scale
+    assert code_bytes == V * g["b"] // 8
+    assert round(code_bytes / 1024, 1) == g["full_logits_KB"]
+    for row in g["rows"]:
+        pct = 100 * (1 - row["downlink_KB"] / g["full_logits_KB"])
+        assert abs(pct - row["compression_pct"]) < 0.051, row
+        # the measured payload exceeds the bare clipped-logit bytes of the
+        # kept fraction (tags, metadata and padding come on top)
+        keep = g["keep_fractions"][row["mode"]]
+        bare = (oracle.payload_bytes(1, round(keep * V)) - 4) / 1024
+        assert bare < row["downlink_KB"] < bare + 10
+
+
+# ---------------------------------------------------------------------------
+# number formats against torch's conversions (exhaustive)
+# ---------------------------------------------------------------------------
+
+def test_bf16_decode_exhaustive():
+    allbits = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    ours = oracle.decode_bf16(allbits)
+    ref = torch.from_numpy(allbits.view(np.int16)).view(torch.bfloat16).double().numpy()
+    both_nan = np.isnan(ours) & np.isnan(ref)
+    assert np.all(both_nan | (ours == ref))
+
+
+def test_e4m3_decode_exhaustive():
+    allbits = np.arange(256, dtype=np.uint8)
+    ours = oracle.decode_e4m3(allbits)
+    ref = torch.from_numpy(allbits).view(torch.float8_e4m3fn).double().numpy()
+    both_nan = np.isnan(ours) & np.isnan(ref)
+    assert np.all(both_nan | (ours == ref))
+    assert np.nanmax(ours) == 448.0
+
+
+def test_bf16_rounding_matches_torch():
+    rng = np.random.default_rng(11)
+    x = rng.normal(size=200000).astype(np.float32) * 10 ** rng.uniform(-6, 6, 200000).astype(np.float32)
+    # exact ties: low 16 bits = 0x8000 with both parities of the kept lsb
+    hi = rng.integers(0, 2 ** 15, 1000, dtype=np.uint32) << np.uint32(17)
+    tb = (hi & np.uint32(0x00FE0000)) | np.uint32(0x3F000000)
+    ties = np.concatenate([tb | np.uint32(0x8000), tb | np.uint32(0x18000)]).view(np.float32)
+    x = np.concatenate([x, ties])
+    assert np.all(np.isfinite(x))
+    ours = oracle.round_fp32_to_bf16(x)
+    ref = torch.from_numpy(x).to(torch.bfloat16).double().numpy()
+    assert np.array_equal(ours, ref, equal_nan=True)
+
+
+# ---------------------------------------------------------------------------
+# Philox4x32-10 against an independent library implementation + statistics
+# ---------------------------------------------------------------------------
+
+_TRITON_PHILOX = textwrap.dedent("""
+    import os, sys, json
+    os.environ["TRITON_INTERPRET"] = "1"
+    import numpy as np, torch, triton, triton.language as tl
+
+    @triton.jit
+    def k(seed, a, b, c, d, o0, o1, o2, o3, N: tl.constexpr):
+        i = tl.arange(0, N)
+        r0, r1, r2, r3 = tl.philox(seed, tl.load(a + i), tl.load(b + i),
+                                   tl.load(c + i), tl.load(d + i), 10)
+        tl.store(o0 + i, r0); tl.store(o1 + i, r1)
+        tl.store(o2 + i, r2); tl.store(o3 + i, r3)
+
+    spec = json.loads(sys.stdin.read())
+    N = len(spec["c0"])
+    cs = [torch.from_numpy(np.array(spec[n], dtype=np.uint32)) for n in ("c0","c1","c2","c3")]
+    outs = [torch.empty(N, dtype=torch.uint32) for _ in range(4)]
+    k[(1,)](spec["seed"], *cs, *outs, N=N)
+    print(json.dumps([o.numpy().astype(np.int64).tolist() for o in outs]))
+""")
+
+
+def test_philox_matches_triton_interpreter():
+    pytest.importorskip("triton")
+    rng = np.random.default_rng(5)
+    N = 64
+    c = [rng.integers(0, 2 ** 32, N, dtype=np.uint64) for _ in range(4)]
+    c[0][:4] = [0, 1, 2, 0xFFFFFFFF]
+    c[1][:4] = 0
+    for seed in (0, 1234567, (0xDEADBEEF << 32) | 0x01234567):
+        spec = dict(seed=seed, **{f"c{i}": c[i].tolist() for i in range(4)})
+        res = subprocess.run([sys.executable, "-c", _TRITON_PHILOX],
+                             input=json.dumps(spec), capture_output=True,
+                             text=True, timeout=300)
+        if res.returncode != 0:
+            pytest.skip("triton interpreter unavailable: " + res.stderr[-300:])
+        ref = json.loads(res.stdout.strip().splitlines()[-1])
+        ours = oracle.philox4x32_10(*c, seed & 0xFFFFFFFF, seed >> 32)
+        for w in range(4):
+            assert np.array_equal(ours[w].astype(np.int64), np.array(ref[w])), (seed, w)
+
+
+def test_philox_uniform_statistics():
+    n = 1 << 20
+    u = oracle.philox_uniform(99, np.arange(n), 0, 7)
+    assert u.min() >= 0.0 and u.max() < 1.0
+    # 24-bit grid: every value is an exact multiple of 2^-24
+    assert np.all(u * 2 ** 24 == np.floor(u * 2 ** 24))
+    hist = np.bincount((u * 256).astype(np.int64), minlength=256)
+    chi2 = ((hist - n / 256) ** 2 / (n / 256)).sum()
+    assert chi2 < 255 + 6 * np.sqrt(2 * 255)
+    # neighbouring counters are uncorrelated; other purposes/offsets differ
+    assert abs(np.corrcoef(u[:-1], u[1:])[0, 1]) < 5e-3
+    u2 = oracle.philox_uniform(99, np.arange(n), 1, 7)
+    u3 = oracle.philox_uniform(99, np.arange(n), 0, 8)
+    assert abs(np.corrcoef(u, u2)[0, 1]) < 5e-3 and np.mean(u == u3) < 1e-3
+
+
+# ---------------------------------------------------------------------------
+# Eq. 14-15: masked softmax and the draw
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("tau", [0.5, 1.0, 2.0])
+def test_sampling_distribution(tau):
+    from scipy.special import softmax
+    rng = np.random.default_rng(int(tau * 10))
+    z = rng.normal(size=16) * 2
+    P = softmax(z / tau)
+    # stratified uniforms: the histogram must match P to within 1/G per bin
+    G = 1 << 16
+    u = (np.arange(G) + 0.5) / G
+    idx, _ = oracle.sample_rows(np.broadcast_to(z, (G, 16)), tau, u)
+    hist = np.bincount(idx, minlength=16) / G
+    assert np.max(np.abs(hist - P)) <= 1.0 / G + 1e-12
+    # Philox uniforms: chi-square goodness of fit
+    n = 200000
+    u = oracle.philox_uniform(3, np.arange(n), 0, int(tau * 100))
+    idx, _ = oracle.sample_rows(np.broadcast_to(z, (n, 16)), tau, u)
+    hist = np.bincount(idx, minlength=16)
+    exp = P * n
+    chi2 = ((hist - exp) ** 2 / exp).sum()
+    assert chi2 < 15 + 6 * np.sqrt(30)
+
+
+def test_small_temperature_is_argmax_and_edges():
+    z = np.array([[0.1, 3.0, 2.999, -5.0]])
+    for u in (0.0, 0.3, 0.999999):
+        j, _ = oracle.sample_rows(z, 1e-5, [u])
+        assert j[0] == 1
+    # u = 0 draws the first id with nonzero probability; margins are >= 0
+    P = np.array([0.0, 0.25, 0.75])
+    assert oracle.inverse_cdf(P, 0.0)[0] == 1
+    assert oracle.inverse_cdf(P, 0.25)[0] == 2
+    j, m = oracle.inverse_cdf(P, 0.2)
+    assert j == 1 and abs(m - 0.05) < 1e-15
+
+
+def test_masked_ids_never_sampled():
+    w = wl.make_workload(V=300, d=24, d_l=8, rows=4, n_keep=90, seed=21,
+                         run_lo=3, run_hi=9)
+    ids = w.keep_ids.numpy()
+    cloud = oracle.partial_logits(w.h_cloud.numpy(), bits16(w.W_h), keep_ids=ids,
+                                  clip=30.0)
+    seen = set()
+    for off in range(400):
+        out = oracle.fuse_sample(cloud["codes"], cloud["row_scale"],
+                                 w.h_local.numpy(), bits16(w.W_l), keep_ids=ids,
+                                 tau=3.0, seed=w.seed, offset=off)
+        seen.update(out["tokens"].tolist())
+    assert seen <= set(ids.tolist())
+    assert len(seen) > 30            # the draw does move around the subset
+
+
+# ---------------------------------------------------------------------------
+# speculative verification: exhaustive enumeration on a tiny vocabulary
+# ---------------------------------------------------------------------------
+
+def _rand_dist(rng, n, zero_some=False):
+    p = rng.uniform(0.05, 1.0, size=n)
+    if zero_some:
+        p[rng.integers(0, n)] = 0.0
+    return p / p.sum()
+
+
+@pytest.mark.parametrize("n,seed", [(4, 0), (5, 1), (6, 2)])
+def test_verify_preserves_target_k1(n, seed):
+    """Standard speculative sampling emits its first token with exactly the
+    target distribution p_0, whatever the draft distribution q_0."""
+    rng = np.random.default_rng(seed)
+    p = np.stack([_rand_dist(rng, n), _rand_dist(rng, n)])
+    q = _rand_dist(rng, n, zero_some=True)[None, :]
+    G = 1 << 10
+    grid = (np.arange(G) + 0.5) / G
+    dist = np.zeros(n)
+    for x in range(n):
+        if q[0, x] == 0:
+            continue
+        for r in grid:
+            for u in grid[::8]:
+                a, j, _, _ = oracle.verify_core(p, q, [x], [r], u)
+                first = x if a >= 1 else j
+                dist[first] += q[0, x] / (G * (G // 8))
+    assert np.max(np.abs(dist - p[0])) < 4 * n / G
+
+
+def test_verify_preserves_target_k2():
+    """k = 2: the first token follows p_0 and, once x_0 is accepted, the
+    second emitted token follows p_1."""
+    rng = np.random.default_rng(9)
+    n = 4
+    p = np.stack([_rand_dist(rng, n) for _ in range(3)])
+    q = np.stack([_rand_dist(rng, n) for _ in range(2)])
+    G = 1 << 5
+    grid = (np.arange(G) + 0.5) / G
+    first = np.zeros(n)
+    second = np.zeros(n)
+    acc0 = 0.0
+    for x0, x1 in itertools.product(range(n), range(n)):
+        wq = q[0, x0] * q[1, x1]
+        for r0, r1, u in itertools.product(grid, grid, grid):
+            a, j, _, _ = oracle.verify_core(p, q, [x0, x1], [r0, r1], u)
+            w = wq / G ** 3
+            first[x0 if a >= 1 else j] += w
+            if a >= 1:
+                acc0 += w
+                second[x1 if a >= 2 else j] += w
+    assert np.max(np.abs(first - p[0])) < 6 * n / G
+    assert np.max(np.abs(second / acc0 - p[1])) < 12 * n / G
+
+
+def test_verify_greedy_is_one_hot_q_and_identical_drafts_accept():
+    rng = np.random.default_rng(4)
+    n, k = 5, 3
+    p = np.stack([_rand_dist(rng, n) for _ in range(k + 1)])
+    x = rng.integers(0, n, size=k)
+    onehot = np.zeros((k, n))
+    onehot[np.arange(k), x] = 1.0
+    for _ in range(500):
+        r = rng.uniform(size=k)
+        u = rng.uniform()
+        a1, j1, _, _ = oracle.verify_core(p, None, x, r, u)
+        a2, j2, _, _ = oracle.verify_core(p, onehot, x, r, u)
+        assert (a1, j1) == (a2, j2)
+    # a draft that equals the target is always accepted (r < 1 = p/q)
+    for _ in range(200):
+        xs = rng.integers(0, n, size=k)
+        a, _, _, _ = oracle.verify_core(p, p[:k], xs, rng.uniform(size=k), 0.5)
+        assert a == k
+
+
+def test_verify_draft_end_to_end_tiny():
+    w = tiny(with_bias=False, V=60, d=16, d_l=4, rows=6, n_keep=25,
+             sessions=2, k=2)
+    ids = w.keep_ids.numpy()
+    cloud = oracle.partial_logits(w.h_cloud.numpy(), bits16(w.W_h), keep_ids=ids,
+                                  clip=30.0)
+    z = oracle.fuse_sample(cloud["codes"], cloud["row_scale"], w.h_local.numpy(),
+                           bits16(w.W_l), keep_ids=ids, tau=1.0,
+                           seed=w.seed)["z"]
+    out = oracle.verify_draft(z.astype(np.float32), 2, 2, keep_ids=ids, V=w.V,
+                              tau=1.0, draft_tokens=w.draft_tokens.numpy(),
+                              draft_probs=w.draft_probs.numpy(), seed=w.seed)
+    assert set(out["next_token"].tolist()) <= set(ids.tolist())
+    assert np.all((out["n_accepted"] >= 0) & (out["n_accepted"] <= 2))
+
+
+def test_compact_index_brute_force():
+    ids = np.array([2, 3, 7, 11, 12])
+    toks = np.array([0, 2, 3, 4, 7, 12, 13, 11, -1])
+    exp = [next((i for i, v in enumerate(ids) if v == t), -1) for t in toks]
+    assert oracle.compact_index(ids, 14, toks).tolist() == exp
+    assert oracle.compact_index(None, 5, np.array([0, 4, 5, -1])).tolist() == [0, 4, -1, -1]
