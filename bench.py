@@ -1,0 +1,477 @@
+#!/usr/bin/env python
+"""Split-head vocabulary projection benchmark (rows/s on GB300).
+
+A step is one pass of the whole hot path over one batch of R hidden-state
+rows: the cloud call (gathered partial logits over the kept vocabulary ids,
+clip, per-row int8) followed by the endpoint call (local partial, fuse,
+mask, softmax, sample); workloads with drafts add the speculative
+verification.  Inputs are seeded synthetic data of the paper's shapes and
+stay resident in HBM; weight copies rotate so that the bytes touched
+between two uses of the same copy exceed twice the L2 size.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload decode]
+  python bench.py --impl reference ...   # the CPU oracle, timed as it stands
+
+Under torchrun every rank runs its own batch on its own GPU (independent
+sessions, weak scaling); the only collectives are the barrier and the
+max-over-ranks of the timed region.  Rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "split-head partial-logit rows/s; % of HBM (or tensor-pipe) roofline"
+UNIT = "rows/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0,
+                  "bf16_tflops_sustained": 1700.0}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="decode",
+                    choices=["tiny", "decode", "spec", "fp8", "sweep"])
+    ap.add_argument("--rows", type=int, default=None, help="sweep: rows")
+    ap.add_argument("--keep", type=float, default=None, help="sweep: keep fraction")
+    ap.add_argument("--e2e-steps", type=int, default=300)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def describe(w):
+    s = (f"{w.name}: d={w.d} (d_l={w.d_l}, d_h={w.d_h}), V={w.V}, R={w.rows}, "
+         f"keep={w.n_keep}{' (full vocab)' if w.keep_ids is None else ''}, "
+         f"W_h {w.w_dtype}, clip={w.clip}, tau={w.tau}")
+    if w.sessions:
+        s += f", S={w.sessions} x (k={w.k}+1) drafts"
+    return s
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id=None):
+        self.samples = []
+        self.proc = None
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+               "-lms", "50"]
+        if gpu_id:
+            cmd += ["-i", str(gpu_id)]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.t = threading.Thread(target=self._read, daemon=True)
+        self.t.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        def parse(line):
+            f = [x.strip() for x in line.split(",")]
+            try:
+                return dict(sm=float(f[0]), smax=float(f[1]),
+                            active=f[3], hw=f[4], hwt=f[5], swt=f[6], pcap=f[7])
+            except Exception:
+                return None
+        inside = [parse(l) for (t, l) in self.samples if t0 <= t <= t1]
+        inside = [s for s in inside if s]
+        note = "during timed region"
+        if not inside:                       # region shorter than the period
+            near = sorted(self.samples, key=lambda s: min(abs(s[0] - t0), abs(s[0] - t1)))[:3]
+            inside = [s for s in (parse(l) for _, l in near) if s]
+            note = "nearest samples (timed region shorter than the sampling period)"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        reasons = set()
+        for s in inside:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if s[key].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(s["sm"] for s in inside),
+                "sm_max_mhz": max(s["smax"] for s in inside),
+                "reasons": sorted(reasons), "samples": len(inside), "note": note}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (the cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 0) for i in threadpool_info()]
+        if n:
+            return max(n)
+    except Exception:
+        pass
+    for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(v):
+            return int(os.environ[v])
+    return os.cpu_count()
+
+
+class OracleSample:
+    """One bounded sample of the workload for the oracle: row r of h over a
+    slice of L consecutive kept ids (cloud call, then endpoint call)."""
+
+    def __init__(self, w):
+        import numpy as np
+        import torch
+        import oracle
+        self.np, self.oracle, self.w = np, oracle, w
+
+        def bits(t):
+            t = t.detach().cpu().contiguous()
+            if t.dtype == torch.bfloat16:
+                return t.view(torch.int16).numpy().view(np.uint16)
+            return t.view(torch.uint8).numpy()
+        self.Wh = bits(w.W_h)
+        self.Wl = bits(w.W_l)
+        self.ws = None if w.w_scale is None else w.w_scale.cpu().numpy()
+        self.h = w.h.cpu().numpy()
+        ids = (np.arange(w.V, dtype=np.int64) if w.keep_ids is None
+               else w.keep_ids.cpu().numpy().astype(np.int64))
+        self.ids = ids
+        self.i = 0
+
+    def run(self, L):
+        o, w = self.oracle, self.w
+        r = self.i % w.rows
+        j0 = (self.i * 7919) % max(1, self.ids.size - L + 1)
+        self.i += 1
+        ids = self.ids[j0:j0 + L]
+        hc = self.h[r:r + 1, w.d_l:]
+        hl = self.h[r:r + 1, :w.d_l]
+        c = o.partial_logits(hc, self.Wh, w_dtype=w.w_dtype, w_scale=self.ws,
+                             keep_ids=ids, clip=w.clip)
+        o.fuse_sample(c["codes"], c["row_scale"], hl, self.Wl, keep_ids=ids,
+                      tau=w.tau, seed=w.seed, offset=self.i)
+        return L / self.ids.size                  # rows of the metric done
+
+    def calibrate(self, seconds_per_step):
+        L = min(self.ids.size, 256)
+        t = time.perf_counter()
+        self.run(L)
+        dt = max(1e-4, time.perf_counter() - t)
+        L = int(L * seconds_per_step / dt)
+        return max(min(64, self.ids.size), min(self.ids.size, L))
+
+
+def cpu_baseline(w, seconds):
+    s = OracleSample(w)
+    L = s.calibrate(min(1.0, seconds / 10))
+    done = 0.0
+    n = 0
+    t0 = time.perf_counter()
+    while time.perf_counter() - t0 < seconds:
+        done += s.run(L)
+        n += 1
+    dt = time.perf_counter() - t0
+    return {"value": done / dt, "unit": UNIT, "cores": oracle_threads(),
+            "kind": "oracle",
+            "sample": (f"{n} samples of 1 row x {L} of {s.ids.size} kept ids "
+                       f"(cloud + endpoint calls, numpy fp64), scaled to rows"),
+            "seconds": round(dt, 2)}
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def source_hash(files):
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_for(kernel_key, files):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken
+    on the current source of that kernel."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(p) as f:
+            d = json.load(f).get(kernel_key)
+        if d and d.get("source_hash") == source_hash(files):
+            return d.get("bytes_per_launch")
+    except Exception:
+        pass
+    return None
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    if rank == 0:
+        import __graft_entry__
+        __graft_entry__.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2607_13093_gb300 import sph, workloads as wl
+
+    w = wl.workload(args.workload, device=dev, rows=args.rows, keep_frac=args.keep)
+    if world > 1:                       # each rank: its own sessions
+        g = torch.Generator(device=dev)
+        g.manual_seed(10_000 + rank)
+        w.h = wl.make_hidden(w.rows, w.d, g, dev)
+    R, n = w.rows, w.n_keep
+    ctx = sph.Context(local)
+    ctx.reserve(R, n, max(w.d_h, w.d_l))
+
+    # rotation so that bytes between reuses exceed 2x L2
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    wb = 1 if w.w_dtype == "fp8" else 2
+    per_copy = n * w.d_h * wb + n * w.d_l * 2
+    ncopy = max(1, math.ceil(2 * l2 / per_copy) + 1) if per_copy < 2 * l2 else 1
+    Whs = [w.W_h] + [w.W_h.clone() for _ in range(ncopy - 1)]
+    Wls = [w.W_l] + [w.W_l.clone() for _ in range(ncopy - 1)]
+    hs = [w.h] + [w.h.roll(i + 1, dims=0).contiguous() for i in range(ncopy - 1)]
+    codes = torch.empty(R, n, dtype=torch.int8, device=dev)
+    scale = torch.empty(R, dtype=torch.float32, device=dev)
+    tokens = torch.empty(R, dtype=torch.int32, device=dev)
+    z = torch.empty(R, n, device=dev) if w.sessions else None
+    n_acc = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
+    nxt = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
+
+    def step(i, h=None):
+        c = i % ncopy
+        hh = hs[c] if h is None else h
+        ctx.partial_logits(hh[:, w.d_l:], Whs[c], keep_ids=w.keep_ids, clip=w.clip,
+                           w_row_scale=w.w_scale, bias=w.bias, codes=codes,
+                           row_scale=scale)
+        ctx.fuse_sample(codes, scale, hh[:, :w.d_l], Wls[c], keep_ids=w.keep_ids,
+                        temperature=w.tau, seed=w.seed, offset=i, tokens=tokens,
+                        fused_logits_out=z)
+        if w.sessions:
+            ctx.verify_draft(z, w.sessions, w.k, w.draft_tokens, keep_ids=w.keep_ids,
+                             draft_probs=w.draft_probs, temperature=w.tau,
+                             seed=w.seed, offset=i, n_accepted=n_acc, next_token=nxt)
+
+    for i in range(args.warmup):
+        step(i)
+    ctx.sync()
+
+    stream = torch.cuda.current_stream(dev)
+    gpu_uuid = None
+    try:
+        gpu_uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        if not gpu_uuid.startswith("GPU-"):
+            gpu_uuid = "GPU-" + gpu_uuid
+    except Exception:
+        pass
+    sampler = ClockSampler(gpu_uuid) if rank == 0 else None
+    time.sleep(0.3 if sampler else 0)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    ctx.profile_enable(True)
+    t_wall0 = time.time()
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+    if world > 1:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    clocks = None
+    if sampler:
+        time.sleep(0.2)
+        sampler.stop()
+        clocks = sampler.summary(t_wall0, t_wall1)
+
+    # ---- end to end: host buffers in, tokens out, every step -------------
+    e2e_steps = min(args.e2e_steps, args.steps)
+    h_host = [x.cpu().pin_memory() for x in hs]
+    tok_host = torch.empty(R, dtype=torch.int32).pin_memory()
+    h_dev = torch.empty_like(w.h)
+    for i in range(3):
+        h_dev.copy_(h_host[i % ncopy], non_blocking=True)
+        step(i, h_dev)
+        tok_host.copy_(tokens, non_blocking=True)
+        torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        h_dev.copy_(h_host[i % ncopy], non_blocking=True)
+        step(i, h_dev)
+        tok_host.copy_(tokens, non_blocking=True)
+        torch.cuda.synchronize(dev)
+    e2e_s = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+
+    if rank != 0:
+        if world > 1:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+
+    peaks, peaks_src = load_peaks()
+    value = R * world * args.steps / (ms / 1e3)
+    # dominant unit: the cloud call (gathered contraction + quantization)
+    cloud_ms = (prof["ms"]["cloud_gemm"] + prof["ms"]["quantize"]) / max(1, prof["calls"]["cloud_gemm"])
+    alg_bytes = wl.algorithmic_bytes_cloud(R, n, w.d_h, wb, fp8_scales=w.w_dtype == "fp8")
+    alg_flops = wl.algorithmic_flops(R, n, w.d_h)
+    ai = alg_flops / alg_bytes
+    ridge = peaks["bf16_tflops_sustained"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    files = ["paper_2607_13093_gb300/csrc/k_gemv.cu", "paper_2607_13093_gb300/csrc/k_finish.cu"]
+    if ai < ridge:
+        achieved = alg_bytes / (cloud_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
+                "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4)}
+    else:
+        achieved = alg_flops / (cloud_ms / 1e3) / 1e12
+        pk = peaks["bf16_tflops_sustained"]
+        roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": pk,
+                "unit": "TFLOP/s", "frac": round(achieved / pk, 4)}
+    roof.update({"traffic": traffic_for(f"cloud_{args.workload}", files),
+                 "kernel": "cloud call: gathered partial logits + int8 quantization",
+                 "algorithmic_bytes": alg_bytes, "algorithmic_flops": alg_flops,
+                 "avg_launch_ms": round(cloud_ms, 5),
+                 "peak_source": f"{peaks_src} (MEASURED_PEAKS.json)" if peaks_src == "measured" else "fallback"})
+    steps_ms = {k: round(v / max(1, args.steps), 5) for k, v in prof["ms"].items() if v}
+    out = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms / args.steps, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded, paper shapes; weights N(0,0.02) bf16, h RMS-normalised)",
+        "config": {"workload": describe(w), "rows_per_gpu": R, "n_keep": n,
+                   "d_h": w.d_h, "d_l": w.d_l, "V": w.V, "weights": w.w_dtype,
+                   "accumulate": "fp32",
+                   "l2": (f"inputs rotate over {ncopy} weight/h copies, "
+                          f"{ncopy * per_copy / 1e6:.0f} MB touched per cycle vs L2 "
+                          f"{l2 / 1e6:.0f} MB"),
+                   "parallelism": f"replicas x{world} (independent sessions per GPU)"},
+        "breakdown_ms_per_step": steps_ms,
+        "roofline": roof,
+        "gpu_launches": prof["launches"],
+        "e2e": {"value": round(R * world * e2e_steps / e2e_s, 1), "unit": UNIT,
+                "h2d_bytes_per_step": R * w.d * 4, "d2h_bytes_per_step": R * 4,
+                "note": "pinned host h -> device, cloud + endpoint calls, tokens -> host, sync per step"},
+        "clocks": clocks,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
+    print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the CPU oracle on the machine's host cores
+# ---------------------------------------------------------------------------
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2607_13093_gb300 import workloads as wl
+    w = wl.workload(args.workload, device="cpu", rows=args.rows, keep_frac=args.keep)
+    s = OracleSample(w)
+    budget = 150.0
+    L = s.calibrate(budget / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        s.run(L)
+    done = 0.0
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        done += s.run(L)
+    dt = time.perf_counter() - t0
+    value = done / dt
+    sample = (f"each step: 1 row x {L} of {s.ids.size} kept ids (cloud + endpoint "
+              f"calls, numpy fp64), scaled to rows")
+    out = {"impl": "reference", "metric": METRIC, "value": round(value, 3),
+           "unit": UNIT, "n_gpus": int(os.environ.get("WORLD_SIZE", "1")),
+           "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic (seeded, paper shapes)",
+           "config": {"workload": describe(w)},
+           "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "kind": "oracle",
+                            "cores": oracle_threads(), "sample": sample},
+           "e2e": {"value": round(value, 3), "unit": UNIT,
+                   "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,243 @@
+/*
+ * sph.h -- C ABI of the split-head vocabulary projection library (libsph.so)
+ *
+ * The library computes, on one GB300 GPU (sm_103a), the data-parallel hot
+ * path of the distributed vocabulary projection of "Efficient and Privacy
+ * Aware Edge Cloud Collaborative Inference for Large Language Models"
+ * (Sec. "Distributed Vocabulary Projection", Eqs. 9-15; Sec. "Transport
+ * Protection", Eq. 18; Sec. "Endpoint Speculative Decoding and Cloud
+ * Verification" with Algorithm 1):
+ *
+ *   cloud     y = h[:, d_l:] . W_h[V_l]^T (+ b[V_l])   -> clip -> per-row int8
+ *   endpoint  z = dequant(codes) + h[:, :d_l] . W_l[V_l]^T -> mask -> softmax/tau
+ *             -> sample ; speculative acceptance of k draft tokens
+ *
+ * Conventions shared by every call
+ *   - Every function returns sph_status.  Scalar arguments and pointer
+ *     presence are validated synchronously on the host; on failure nothing
+ *     is launched and sph_last_error(ctx) describes the problem.
+ *   - Compute calls are asynchronous on the context's stream.  Faults and
+ *     device-side timeouts surface at sph_sync() (or the next call).
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the
+ *     library never keeps them past the call.  Layouts are row-major with
+ *     the stated leading dimension (in elements).  The context owns only
+ *     its scratch memory (grown on demand, or pre-sized by sph_reserve()).
+ *   - keep_ids is the language subset V_l: int32 vocabulary ids, strictly
+ *     increasing, each in [0, V).  NULL means the full vocabulary
+ *     (mixed-language mode) and then n_keep must equal V.  Payloads and
+ *     logits are "compacted": column j belongs to vocabulary id keep_ids[j].
+ *   - A context is not thread-safe; use one per host thread.
+ *   - There is no CPU fallback: a shape the kernels do not support returns
+ *     SPH_ERR_UNSUPPORTED.
+ */
+#ifndef SPH_H_
+#define SPH_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum sph_status {
+  SPH_OK = 0,
+  SPH_ERR_INVALID_ARG = 1,  /* bad scalar, NULL pointer, inconsistent sizes   */
+  SPH_ERR_UNSUPPORTED = 2,  /* valid but outside what the kernels implement   */
+  SPH_ERR_CUDA = 3,         /* a CUDA runtime call or a kernel launch failed  */
+  SPH_ERR_TIMEOUT = 4,      /* a bounded device-side wait gave up             */
+  SPH_ERR_OOM = 5           /* scratch memory could not be allocated          */
+} sph_status;
+
+typedef enum sph_dtype {
+  SPH_DTYPE_BF16 = 0,       /* bfloat16 weights                                */
+  SPH_DTYPE_FP8_E4M3 = 1    /* OCP e4m3 ('fn') weights with an fp32 scale per
+                               vocabulary row: value = e4m3 * w_row_scale[v]  */
+} sph_dtype;
+
+typedef enum sph_act_mode {
+  SPH_ACT_FP32 = 0,         /* hidden states used at fp32 accuracy (default)  */
+  SPH_ACT_BF16 = 1          /* hidden states rounded to bf16 (RNE) first, as a
+                               bf16 cloud decoder would hand them over        */
+} sph_act_mode;
+
+typedef struct sph_ctx sph_ctx;
+typedef struct sph_buffer sph_buffer;
+
+/* ---- context and memory ------------------------------------------------ */
+
+/* Create a context on CUDA device `device` issuing work on `cuda_stream`
+ * (a cudaStream_t; NULL = the legacy default stream).  *out receives the
+ * handle.  Errors: INVALID_ARG (out NULL, bad device), CUDA, OOM. */
+sph_status sph_create(int device, void* cuda_stream, sph_ctx** out);
+
+/* Release the context and its scratch (waits for its stream first). */
+sph_status sph_destroy(sph_ctx* ctx);
+
+/* Issue subsequent calls on another stream of the same device. */
+sph_status sph_set_stream(sph_ctx* ctx, void* cuda_stream);
+
+/* Wait for all work of the context's stream; report device-side errors
+ * (SPH_ERR_TIMEOUT for a wait that gave up, SPH_ERR_CUDA for faults). */
+sph_status sph_sync(sph_ctx* ctx);
+
+/* Human-readable detail of the last error of `ctx` ("" if none). Owned by
+ * the context, valid until its next call. */
+const char* sph_last_error(const sph_ctx* ctx);
+
+/* Static name of a status code. */
+const char* sph_status_string(sph_status status);
+
+/* Pre-size the context's scratch for calls up to these sizes so that later
+ * calls allocate nothing (required before capturing calls into a CUDA
+ * graph).  max_d is the largest of d_h and d_l. */
+sph_status sph_reserve(sph_ctx* ctx, int64_t max_rows, int64_t max_n_keep,
+                       int64_t max_d);
+
+/* Optional device allocation helpers for callers without their own
+ * allocator.  sph_buffer_ptr returns the device address (NULL for NULL). */
+sph_status sph_buffer_alloc(sph_ctx* ctx, size_t bytes, sph_buffer** out);
+sph_status sph_buffer_free(sph_ctx* ctx, sph_buffer* buf);
+void* sph_buffer_ptr(const sph_buffer* buf);
+
+/* ---- tracing ----------------------------------------------------------- */
+
+/* Kernel classes whose device time the context can accumulate. */
+enum {
+  SPH_PROF_CLOUD_GEMM = 0,  /* gathered h_cloud . W_h contraction + epilogue */
+  SPH_PROF_QUANTIZE = 1,    /* per-row int8 quantization of the partials    */
+  SPH_PROF_LOCAL_GEMM = 2,  /* gathered h_local . W_l contraction + fuse     */
+  SPH_PROF_SAMPLE = 3,      /* softmax / inverse-CDF draw                    */
+  SPH_PROF_VERIFY = 4,      /* speculative acceptance                        */
+  SPH_PROF_PREP = 5,        /* operand preparation (hidden-state splits)     */
+  SPH_PROF_CLASSES = 8
+};
+
+typedef struct sph_profile {
+  double ms[SPH_PROF_CLASSES];       /* summed device time per class (ms)   */
+  int64_t calls[SPH_PROF_CLASSES];   /* timed launch groups per class       */
+  int64_t launches;                  /* kernels launched while enabled      */
+} sph_profile;
+
+/* Start (on != 0; resets the accumulators) or stop tracing.  While on, each
+ * kernel group is bracketed by CUDA events on the context's stream. */
+sph_status sph_profile_enable(sph_ctx* ctx, int on);
+
+/* Wait for the context's stream and return the accumulated figures. */
+sph_status sph_profile_read(sph_ctx* ctx, sph_profile* out);
+
+/* ---- host helpers (no device work) ------------------------------------- */
+
+/* Downlink payload of one cloud call (Eq. 21 with b = 8 and no tag,
+ * metadata or padding): one int8 code per kept logit plus one fp32 scale
+ * per row, i.e. rows*n_keep + 4*rows bytes.  Returns 0 for negative sizes. */
+size_t sph_payload_bytes(int64_t rows, int64_t n_keep);
+
+/* Turn the "compact subset mask" of Sec. "Distributed Vocabulary
+ * Projection" -- a HOST bitmask of ceil(V/8) bytes, bit (v & 7) of byte
+ * v >> 3 set iff id v is kept -- into the sorted HOST id list keep_ids
+ * (capacity V entries).  *n_keep receives the count.  Errors: INVALID_ARG
+ * (NULL pointers, V < 1, no id set). */
+sph_status sph_keep_ids_from_mask(const uint8_t* mask, int64_t V,
+                                  int32_t* keep_ids, int64_t* n_keep);
+
+/* ---- the hot path ------------------------------------------------------ */
+
+/* Cloud call (Eq. 12 over V_l, "after clipping, quantization" in Sec.
+ * "Distributed Vocabulary Projection", Eq. 18 with b = 8, Eq. 21):
+ *   y[r, j]      = sum_{c < d_h} h_cloud[r, c] * W_h[keep_ids[j], c]
+ *                  (+ bias[keep_ids[j]])            fp32 accumulate
+ *   yc           = min(max(y, -clip), clip)
+ *   row_scale[r] = max_j |yc[r, j]| / 127   (fp32; 0 for an all-zero row)
+ *   codes[r, j]  = round-half-even(yc / row_scale[r]) in [-127, 127]
+ * Arguments
+ *   h_cloud  fp32 [rows, d_h] with row stride ld_h (>= d_h); typically the
+ *            slice h[:, d_l:] of the full hidden state (ld_h = d).
+ *   W_h      [V, d_h] row-major, row stride ld_w (>= d_h) elements of
+ *            w_dtype; vocabulary-major, i.e. W_cloud of Eq. 10 transposed.
+ *            ld_w*element size and the base address must be multiples of 16
+ *            bytes.
+ *   w_row_scale  fp32 [V] for SPH_DTYPE_FP8_E4M3, else NULL.
+ *   bias     fp32 [V] or NULL; applied once, here (Eq. 12).
+ *   keep_ids int32 [n_keep] (see conventions) or NULL with n_keep == V.
+ *   clip     > 0 and finite.
+ *   act_mode SPH_ACT_FP32 or SPH_ACT_BF16.
+ *   codes    int8 [rows, n_keep] (out), row_scale fp32 [rows] (out).
+ *   partial_out  fp32 [rows, n_keep] unclipped y (out), or NULL.
+ *   payload_bytes  host size_t (out) = sph_payload_bytes(rows, n_keep), or
+ *            NULL.
+ * Preconditions: rows >= 1, d_h >= 1, 1 <= n_keep <= V, finite inputs.
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA, OOM. */
+sph_status sph_partial_logits(sph_ctx* ctx,
+                              const float* h_cloud, int64_t rows, int64_t ld_h,
+                              const void* W_h, sph_dtype w_dtype, int64_t V,
+                              int64_t d_h, int64_t ld_w,
+                              const float* w_row_scale, const float* bias,
+                              const int32_t* keep_ids, int64_t n_keep,
+                              float clip, sph_act_mode act_mode,
+                              int8_t* codes, float* row_scale,
+                              float* partial_out, size_t* payload_bytes);
+
+/* Endpoint call (Eq. 11, Eq. 13, Eq. 14, Eq. 15; Algorithm 1 "fuses partial
+ * logits, applies language masking, and samples"):
+ *   z[r, j]   = codes[r, j] * row_scale[r]
+ *               + sum_{c < d_l} h_local[r, c] * W_l[keep_ids[j], c]
+ *   p[r, :]   = softmax(z[r, :] / temperature) over the kept ids (ids
+ *               outside V_l have z = -inf, i.e. probability 0)
+ *   tokens[r] = keep_ids[j*], j* = the first j whose ascending-order CDF
+ *               exceeds u_r, u_r = Philox4x32-10 uniform with key = seed and
+ *               counter (r, 0, offset lo, offset hi), u = (x0 >> 8) * 2^-24
+ * Arguments
+ *   codes int8 [rows, n_keep], row_scale fp32 [rows]: the cloud payload.
+ *   h_local fp32 [rows, d_l], row stride ld_hl (the slice h[:, :d_l]).
+ *   W_l bf16 [V, d_l] row-major with row stride ld_wl (16-byte multiple).
+ *   keep_ids as for sph_partial_logits.  temperature > 0 and finite.
+ *   tokens int32 [rows] (out, vocabulary ids).
+ *   fused_logits_out fp32 [rows, n_keep] z before the division by
+ *   temperature (out), or NULL.
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA, OOM. */
+sph_status sph_fuse_sample(sph_ctx* ctx,
+                           const int8_t* codes, const float* row_scale,
+                           int64_t rows,
+                           const float* h_local, int64_t ld_hl,
+                           const void* W_l, int64_t V, int64_t d_l,
+                           int64_t ld_wl,
+                           const int32_t* keep_ids, int64_t n_keep,
+                           float temperature, uint64_t seed, uint64_t offset,
+                           int32_t* tokens, float* fused_logits_out);
+
+/* Cloud verification of speculative drafts (Sec. "Endpoint Speculative
+ * Decoding and Cloud Verification", Algorithm 1; standard speculative
+ * sampling as in the works the paper cites).  Per session s:
+ *   p_i = softmax(target_logits[s*(k+1)+i, :] / temperature), i = 0..k
+ *   for i < k: accept draft x_i iff r_i * q_i(x_i) < p_i(x_i), with
+ *     r_i = Philox uniform of counter (s, 1+i, offset lo, offset hi);
+ *   at the first rejection draw from max(0, p_i - q_i) renormalised (p_i if
+ *   that is all zero); if all k are accepted draw from p_k; the draw uses
+ *   the uniform of counter (s, 1+k, ...) and the inverse CDF in ascending
+ *   id order.
+ * Arguments
+ *   target_logits fp32 [sessions*(k+1), n_keep] compacted fused logits.
+ *   draft_tokens int32 [sessions, k] vocabulary ids (an id outside V_l has
+ *   p = q = 0 and is rejected).
+ *   draft_probs fp32 [sessions, k, n_keep] compacted q, or NULL for greedy
+ *   (one-hot) drafts, where q_i(x) = [x == x_i].
+ *   n_accepted int32 [sessions] (out) in [0, k]; next_token int32
+ *   [sessions] (out): the drawn vocabulary id.
+ * Preconditions: sessions >= 1, k >= 1, temperature > 0.
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA, OOM. */
+sph_status sph_verify_draft(sph_ctx* ctx,
+                            const float* target_logits, int64_t sessions,
+                            int64_t k,
+                            const int32_t* keep_ids, int64_t n_keep,
+                            float temperature,
+                            const int32_t* draft_tokens,
+                            const float* draft_probs,
+                            uint64_t seed, uint64_t offset,
+                            int32_t* n_accepted, int32_t* next_token);
+
+#ifdef __cplusplus
+}  /* extern "C" */
+#endif
+
+#endif  /* SPH_H_ */

@@ -1,0 +1,474 @@
+// C-ABI layer of libsph: context, scratch arena, argument validation and
+// dispatch of the split-head kernels.  Declared in include/sph.h.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "sph.h"
+#include "sph_internal.h"
+
+namespace sph {
+thread_local long long launch_count = 0;
+}
+
+struct ProfPair {
+  int cls;
+  cudaEvent_t start, stop;
+};
+
+struct sph_ctx {
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  int sm_count = 0;
+  std::string err;
+  void* scratch = nullptr;          // arena for per-call temporaries
+  size_t scratch_cap = 0;
+  unsigned* status = nullptr;       // device error word (sph::ERR_* bits)
+  // tracing
+  bool prof = false;
+  long long prof_launch0 = 0;
+  sph_profile acc{};
+  std::vector<ProfPair> pending;
+  std::vector<cudaEvent_t> pool;
+};
+
+struct sph_buffer {
+  void* ptr = nullptr;
+  size_t bytes = 0;
+};
+
+namespace {
+
+sph_status fail(sph_ctx* ctx, sph_status st, const char* fmt, ...) {
+  if (ctx) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    ctx->err = buf;
+  }
+  return st;
+}
+
+sph_status cuda_fail(sph_ctx* ctx, cudaError_t e, const char* what) {
+  return fail(ctx, SPH_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// RAII guard that makes the context's device current for one call.
+struct DeviceGuard {
+  int prev = -1;
+  bool ok = true;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev)
+      cudaSetDevice(prev);
+  }
+};
+
+// Grow the scratch arena to `bytes` (outside stream capture only).
+sph_status ensure_scratch(sph_ctx* ctx, size_t bytes) {
+  if (bytes <= ctx->scratch_cap) return SPH_OK;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(ctx->stream, &cap) == cudaSuccess &&
+      cap != cudaStreamCaptureStatusNone)
+    return fail(ctx, SPH_ERR_UNSUPPORTED,
+                "scratch must grow to %zu bytes during stream capture; call "
+                "sph_reserve() before capturing", bytes);
+  cudaError_t e = cudaStreamSynchronize(ctx->stream);   // old arena may be in use
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaStreamSynchronize");
+  if (ctx->scratch) cudaFree(ctx->scratch);
+  ctx->scratch = nullptr;
+  ctx->scratch_cap = 0;
+  const size_t want = align_up(bytes + bytes / 4, 1 << 20);
+  e = cudaMalloc(&ctx->scratch, want);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(ctx, SPH_ERR_OOM, "cudaMalloc(%zu) for scratch failed", want);
+  }
+  ctx->scratch_cap = want;
+  return SPH_OK;
+}
+
+// Bump allocator over the arena for one call.
+struct Carve {
+  char* base;
+  size_t off = 0;
+  explicit Carve(void* b) : base(static_cast<char*>(b)) {}
+  void* take(size_t bytes) {
+    void* p = base ? base + off : nullptr;
+    off = align_up(off + bytes, 256);
+    return p;
+  }
+};
+
+size_t partial_scratch_bytes(int64_t rows, int64_t n) {
+  return align_up((size_t)rows * n * 4, 256) + align_up((size_t)rows * 4, 256);
+}
+size_t fuse_scratch_bytes(int64_t rows, int64_t n) {
+  return align_up((size_t)rows * n * 4, 256);
+}
+
+bool finite_pos(float x) { return std::isfinite(x) && x > 0.f; }
+
+sph_status check_ids(sph_ctx* ctx, const int32_t* keep_ids, int64_t n_keep,
+                     int64_t V) {
+  if (V < 1 || V > INT32_MAX) return fail(ctx, SPH_ERR_INVALID_ARG, "V=%lld out of range", (long long)V);
+  if (n_keep < 1 || n_keep > V)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "n_keep=%lld must be in [1, V=%lld]",
+                (long long)n_keep, (long long)V);
+  if (!keep_ids && n_keep != V)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "keep_ids NULL requires n_keep == V");
+  return SPH_OK;
+}
+
+sph_status launch_status(sph_ctx* ctx, cudaError_t e, const char* what) {
+  if (e != cudaSuccess) return cuda_fail(ctx, e, what);
+  return SPH_OK;
+}
+
+cudaEvent_t pooled_event(sph_ctx* ctx) {
+  if (!ctx->pool.empty()) {
+    cudaEvent_t ev = ctx->pool.back();
+    ctx->pool.pop_back();
+    return ev;
+  }
+  cudaEvent_t ev = nullptr;
+  if (cudaEventCreate(&ev) != cudaSuccess) return nullptr;
+  return ev;
+}
+
+// Run one kernel group; while tracing, bracket it with events of class cls.
+template <class F>
+cudaError_t traced(sph_ctx* ctx, int cls, F&& launch) {
+  if (!ctx->prof) return launch();
+  cudaEvent_t a = pooled_event(ctx), b = pooled_event(ctx);
+  if (!a || !b) return launch();
+  cudaEventRecord(a, ctx->stream);
+  const cudaError_t e = launch();
+  cudaEventRecord(b, ctx->stream);
+  ctx->pending.push_back({cls, a, b});
+  return e;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* sph_status_string(sph_status s) {
+  switch (s) {
+    case SPH_OK: return "SPH_OK";
+    case SPH_ERR_INVALID_ARG: return "SPH_ERR_INVALID_ARG";
+    case SPH_ERR_UNSUPPORTED: return "SPH_ERR_UNSUPPORTED";
+    case SPH_ERR_CUDA: return "SPH_ERR_CUDA";
+    case SPH_ERR_TIMEOUT: return "SPH_ERR_TIMEOUT";
+    case SPH_ERR_OOM: return "SPH_ERR_OOM";
+  }
+  return "SPH_ERR_UNKNOWN";
+}
+
+const char* sph_last_error(const sph_ctx* ctx) {
+  return ctx ? ctx->err.c_str() : "null context";
+}
+
+size_t sph_payload_bytes(int64_t rows, int64_t n_keep) {
+  if (rows < 0 || n_keep < 0) return 0;
+  return (size_t)rows * (size_t)n_keep + 4 * (size_t)rows;
+}
+
+sph_status sph_keep_ids_from_mask(const uint8_t* mask, int64_t V,
+                                  int32_t* keep_ids, int64_t* n_keep) {
+  if (!mask || !keep_ids || !n_keep || V < 1 || V > INT32_MAX)
+    return SPH_ERR_INVALID_ARG;
+  int64_t n = 0;
+  for (int64_t v = 0; v < V; ++v)
+    if (mask[v >> 3] & (1u << (v & 7))) keep_ids[n++] = (int32_t)v;
+  *n_keep = n;
+  return n ? SPH_OK : SPH_ERR_INVALID_ARG;
+}
+
+sph_status sph_create(int device, void* cuda_stream, sph_ctx** out) {
+  if (!out) return SPH_ERR_INVALID_ARG;
+  *out = nullptr;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess) {
+    cudaGetLastError();
+    return SPH_ERR_CUDA;
+  }
+  if (device < 0 || device >= ndev) return SPH_ERR_INVALID_ARG;
+  sph_ctx* ctx = new (std::nothrow) sph_ctx();
+  if (!ctx) return SPH_ERR_OOM;
+  ctx->device = device;
+  ctx->stream = static_cast<cudaStream_t>(cuda_stream);
+  DeviceGuard g(device);
+  if (!g.ok) { delete ctx; return SPH_ERR_CUDA; }
+  if (cudaDeviceGetAttribute(&ctx->sm_count, cudaDevAttrMultiProcessorCount,
+                             device) != cudaSuccess) {
+    delete ctx;
+    return SPH_ERR_CUDA;
+  }
+  if (cudaMalloc(&ctx->status, sizeof(unsigned)) != cudaSuccess) {
+    cudaGetLastError();
+    delete ctx;
+    return SPH_ERR_OOM;
+  }
+  if (cudaMemset(ctx->status, 0, sizeof(unsigned)) != cudaSuccess) {
+    cudaFree(ctx->status);
+    delete ctx;
+    return SPH_ERR_CUDA;
+  }
+  *out = ctx;
+  return SPH_OK;
+}
+
+sph_status sph_destroy(sph_ctx* ctx) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  DeviceGuard g(ctx->device);
+  cudaStreamSynchronize(ctx->stream);
+  if (ctx->scratch) cudaFree(ctx->scratch);
+  if (ctx->status) cudaFree(ctx->status);
+  for (auto& p : ctx->pending) { cudaEventDestroy(p.start); cudaEventDestroy(p.stop); }
+  for (auto ev : ctx->pool) cudaEventDestroy(ev);
+  delete ctx;
+  return SPH_OK;
+}
+
+sph_status sph_profile_enable(sph_ctx* ctx, int on) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  DeviceGuard g(ctx->device);
+  if (on) {
+    for (auto& p : ctx->pending) { ctx->pool.push_back(p.start); ctx->pool.push_back(p.stop); }
+    ctx->pending.clear();
+    ctx->acc = sph_profile{};
+    ctx->prof_launch0 = sph::launch_count;
+  }
+  ctx->prof = on != 0;
+  return SPH_OK;
+}
+
+sph_status sph_profile_read(sph_ctx* ctx, sph_profile* out) {
+  if (!ctx || !out) return SPH_ERR_INVALID_ARG;
+  DeviceGuard g(ctx->device);
+  cudaError_t e = cudaStreamSynchronize(ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaStreamSynchronize");
+  for (auto& p : ctx->pending) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, p.start, p.stop) == cudaSuccess) {
+      ctx->acc.ms[p.cls] += ms;
+      ctx->acc.calls[p.cls] += 1;
+    }
+    ctx->pool.push_back(p.start);
+    ctx->pool.push_back(p.stop);
+  }
+  ctx->pending.clear();
+  ctx->acc.launches = sph::launch_count - ctx->prof_launch0;
+  *out = ctx->acc;
+  return SPH_OK;
+}
+
+sph_status sph_set_stream(sph_ctx* ctx, void* cuda_stream) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  ctx->stream = static_cast<cudaStream_t>(cuda_stream);
+  return SPH_OK;
+}
+
+sph_status sph_sync(sph_ctx* ctx) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  DeviceGuard g(ctx->device);
+  cudaError_t e = cudaStreamSynchronize(ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaStreamSynchronize");
+  unsigned st = 0;
+  e = cudaMemcpy(&st, ctx->status, sizeof st, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "reading device status");
+  if (st) {
+    cudaMemset(ctx->status, 0, sizeof(unsigned));
+    if (st & sph::ERR_TIMEOUT)
+      return fail(ctx, SPH_ERR_TIMEOUT, "a device-side wait timed out (status 0x%x)", st);
+    return fail(ctx, SPH_ERR_INVALID_ARG, "a kernel skipped out-of-range ids (status 0x%x)", st);
+  }
+  return SPH_OK;
+}
+
+sph_status sph_reserve(sph_ctx* ctx, int64_t max_rows, int64_t max_n_keep,
+                       int64_t max_d) {
+  if (!ctx || max_rows < 1 || max_n_keep < 1 || max_d < 1)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "sph_reserve: sizes must be >= 1");
+  DeviceGuard g(ctx->device);
+  size_t need = partial_scratch_bytes(max_rows, max_n_keep);
+  const size_t f = fuse_scratch_bytes(max_rows, max_n_keep);
+  if (f > need) need = f;
+  return ensure_scratch(ctx, need);
+}
+
+sph_status sph_buffer_alloc(sph_ctx* ctx, size_t bytes, sph_buffer** out) {
+  if (!ctx || !out || bytes == 0) return fail(ctx, SPH_ERR_INVALID_ARG, "sph_buffer_alloc: bad arguments");
+  DeviceGuard g(ctx->device);
+  sph_buffer* b = new (std::nothrow) sph_buffer();
+  if (!b) return SPH_ERR_OOM;
+  if (cudaMalloc(&b->ptr, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    delete b;
+    return fail(ctx, SPH_ERR_OOM, "cudaMalloc(%zu) failed", bytes);
+  }
+  b->bytes = bytes;
+  *out = b;
+  return SPH_OK;
+}
+
+sph_status sph_buffer_free(sph_ctx* ctx, sph_buffer* buf) {
+  if (!ctx || !buf) return SPH_ERR_INVALID_ARG;
+  DeviceGuard g(ctx->device);
+  cudaError_t e = cudaFree(buf->ptr);
+  delete buf;
+  return e == cudaSuccess ? SPH_OK : cuda_fail(ctx, e, "cudaFree");
+}
+
+void* sph_buffer_ptr(const sph_buffer* buf) { return buf ? buf->ptr : nullptr; }
+
+sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
+                              int64_t ld_h, const void* W_h, sph_dtype w_dtype,
+                              int64_t V, int64_t d_h, int64_t ld_w,
+                              const float* w_row_scale, const float* bias,
+                              const int32_t* keep_ids, int64_t n_keep,
+                              float clip, sph_act_mode act_mode, int8_t* codes,
+                              float* row_scale, float* partial_out,
+                              size_t* payload_bytes) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  if (!h_cloud || !W_h || !codes || !row_scale)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "h_cloud, W_h, codes and row_scale must be non-NULL");
+  if (rows < 1 || rows > (1 << 20)) return fail(ctx, SPH_ERR_INVALID_ARG, "rows=%lld out of [1, 2^20]", (long long)rows);
+  if (d_h < 1) return fail(ctx, SPH_ERR_INVALID_ARG, "d_h must be >= 1");
+  if (ld_h < d_h || ld_w < d_h) return fail(ctx, SPH_ERR_INVALID_ARG, "ld_h and ld_w must be >= d_h");
+  sph_status st = check_ids(ctx, keep_ids, n_keep, V);
+  if (st) return st;
+  if (!finite_pos(clip)) return fail(ctx, SPH_ERR_INVALID_ARG, "clip must be finite and > 0");
+  if (w_dtype != SPH_DTYPE_BF16 && w_dtype != SPH_DTYPE_FP8_E4M3)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "unknown w_dtype %d", (int)w_dtype);
+  if (act_mode != SPH_ACT_FP32 && act_mode != SPH_ACT_BF16)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "unknown act_mode %d", (int)act_mode);
+  if (w_dtype == SPH_DTYPE_FP8_E4M3 && !w_row_scale)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "fp8 weights need w_row_scale");
+  const int esz = w_dtype == SPH_DTYPE_BF16 ? 2 : 1;
+  if (((uintptr_t)W_h & 15) || ((ld_w * esz) & 15))
+    return fail(ctx, SPH_ERR_INVALID_ARG, "W_h base and row stride must be 16-byte aligned");
+  if (rows * n_keep > ((int64_t)1 << 40)) return fail(ctx, SPH_ERR_UNSUPPORTED, "rows*n_keep too large");
+  if (d_h > sph::gemv_max_k()) return fail(ctx, SPH_ERR_UNSUPPORTED, "d_h=%lld above %d", (long long)d_h, sph::gemv_max_k());
+  if (payload_bytes) *payload_bytes = sph_payload_bytes(rows, n_keep);
+
+  DeviceGuard g(ctx->device);
+  if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
+  st = ensure_scratch(ctx, partial_scratch_bytes(rows, n_keep));
+  if (st) return st;
+  Carve c(ctx->scratch);
+  float* Y = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
+  unsigned* rowmax = static_cast<unsigned*>(c.take((size_t)rows * 4));
+  cudaError_t e = cudaMemsetAsync(rowmax, 0, (size_t)rows * 4, ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMemsetAsync");
+
+  sph::GatherGemm gg{};
+  gg.h = h_cloud; gg.ld_h = ld_h; gg.rows = (int)rows;
+  gg.W = W_h; gg.ld_w = ld_w;
+  gg.w_dtype = w_dtype == SPH_DTYPE_BF16 ? sph::W_BF16 : sph::W_FP8;
+  gg.w_scale = w_row_scale; gg.K = (int)d_h;
+  gg.ids = keep_ids; gg.n = (int)n_keep;
+  gg.act_bf16 = act_mode == SPH_ACT_BF16;
+  gg.epilogue = sph::EPI_CLOUD;
+  gg.bias = bias; gg.clip = clip; gg.partial_out = partial_out;
+  gg.Y = Y; gg.rowmax = rowmax; gg.status = ctx->status;
+  st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
+                       return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
+                     }), "gemv launch");
+  if (st) return st;
+  return launch_status(ctx, traced(ctx, SPH_PROF_QUANTIZE, [&] {
+                         return sph::launch_quantize(Y, rowmax, (int)rows, (int)n_keep,
+                                                     codes, row_scale, ctx->stream);
+                       }), "quantize launch");
+}
+
+sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
+                           const float* row_scale, int64_t rows,
+                           const float* h_local, int64_t ld_hl,
+                           const void* W_l, int64_t V, int64_t d_l,
+                           int64_t ld_wl, const int32_t* keep_ids,
+                           int64_t n_keep, float temperature, uint64_t seed,
+                           uint64_t offset, int32_t* tokens,
+                           float* fused_logits_out) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  if (!codes || !row_scale || !h_local || !W_l || !tokens)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "codes, row_scale, h_local, W_l and tokens must be non-NULL");
+  if (rows < 1 || rows > (1 << 20)) return fail(ctx, SPH_ERR_INVALID_ARG, "rows=%lld out of [1, 2^20]", (long long)rows);
+  if (d_l < 1) return fail(ctx, SPH_ERR_INVALID_ARG, "d_l must be >= 1");
+  if (ld_hl < d_l || ld_wl < d_l) return fail(ctx, SPH_ERR_INVALID_ARG, "ld_hl and ld_wl must be >= d_l");
+  sph_status st = check_ids(ctx, keep_ids, n_keep, V);
+  if (st) return st;
+  if (!finite_pos(temperature)) return fail(ctx, SPH_ERR_INVALID_ARG, "temperature must be finite and > 0");
+  if (((uintptr_t)W_l & 15) || ((ld_wl * 2) & 15))
+    return fail(ctx, SPH_ERR_INVALID_ARG, "W_l base and row stride must be 16-byte aligned");
+  if (n_keep > sph::sample_max_n()) return fail(ctx, SPH_ERR_UNSUPPORTED, "n_keep above %d", sph::sample_max_n());
+  if (d_l > sph::gemv_max_k()) return fail(ctx, SPH_ERR_UNSUPPORTED, "d_l above %d", sph::gemv_max_k());
+
+  DeviceGuard g(ctx->device);
+  if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
+  float* Z = fused_logits_out;
+  if (!Z) {
+    st = ensure_scratch(ctx, fuse_scratch_bytes(rows, n_keep));
+    if (st) return st;
+    Carve c(ctx->scratch);
+    Z = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
+  }
+  sph::GatherGemm gg{};
+  gg.h = h_local; gg.ld_h = ld_hl; gg.rows = (int)rows;
+  gg.W = W_l; gg.ld_w = ld_wl; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
+  gg.ids = keep_ids; gg.n = (int)n_keep;
+  gg.epilogue = sph::EPI_ENDPOINT;
+  gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale; gg.status = ctx->status;
+  st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
+                       return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
+                     }), "gemv launch");
+  if (st) return st;
+  return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
+                         return sph::launch_sample(Z, (int)rows, (int)n_keep, keep_ids,
+                                                   1.0f / temperature, seed, offset,
+                                                   tokens, ctx->stream);
+                       }), "sample launch");
+}
+
+sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
+                            int64_t sessions, int64_t k,
+                            const int32_t* keep_ids, int64_t n_keep,
+                            float temperature, const int32_t* draft_tokens,
+                            const float* draft_probs, uint64_t seed,
+                            uint64_t offset, int32_t* n_accepted,
+                            int32_t* next_token) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  if (!target_logits || !draft_tokens || !n_accepted || !next_token)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "target_logits, draft_tokens, n_accepted and next_token must be non-NULL");
+  if (sessions < 1 || sessions > (1 << 20)) return fail(ctx, SPH_ERR_INVALID_ARG, "sessions out of [1, 2^20]");
+  if (k < 1 || k > 64) return fail(ctx, SPH_ERR_INVALID_ARG, "k must be in [1, 64]");
+  if (n_keep < 1 || n_keep > INT32_MAX) return fail(ctx, SPH_ERR_INVALID_ARG, "n_keep must be >= 1");
+  if (!finite_pos(temperature)) return fail(ctx, SPH_ERR_INVALID_ARG, "temperature must be finite and > 0");
+  if (n_keep > sph::sample_max_n()) return fail(ctx, SPH_ERR_UNSUPPORTED, "n_keep above %d", sph::sample_max_n());
+  DeviceGuard g(ctx->device);
+  if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
+  // without an id list the compact index is the vocabulary id itself
+  const int V = keep_ids ? INT32_MAX : (int)n_keep;
+  return launch_status(ctx, traced(ctx, SPH_PROF_VERIFY, [&] {
+                         return sph::launch_verify(target_logits, (int)sessions, (int)k,
+                                                   (int)n_keep, keep_ids, V,
+                                                   1.0f / temperature, draft_tokens,
+                                                   draft_probs, seed, offset,
+                                                   n_accepted, next_token, ctx->stream);
+                       }), "verify launch");
+}
+
+}  // extern "C"

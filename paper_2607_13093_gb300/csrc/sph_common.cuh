@@ -1,0 +1,103 @@
+// Device helpers shared by the split-head kernels: the counter-based
+// generator, number-format conversions, block reductions and the layout of
+// the context's scratch arena.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cuda_fp8.h>
+#include <stdint.h>
+
+namespace sph {
+
+// ---------------------------------------------------------------------------
+// Philox4x32 with 10 rounds (Salmon, Moraes, Dror, Shaw, SC'11).  A round
+// multiplies counter words 0 and 2 by the two published multipliers, then
+// mixes the high halves with the other two words and the key; the key is
+// advanced by the two Weyl constants between rounds.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 philox4x32_10(uint4 ctr, uint2 key) {
+#pragma unroll
+  for (int round = 0; round < 10; ++round) {
+    const uint32_t a = ctr.x, c = ctr.z;
+    const uint32_t hi_a = __umulhi(0xD2511F53u, a), lo_a = 0xD2511F53u * a;
+    const uint32_t hi_c = __umulhi(0xCD9E8D57u, c), lo_c = 0xCD9E8D57u * c;
+    ctr = make_uint4(hi_c ^ ctr.y ^ key.x, lo_c, hi_a ^ ctr.w ^ key.y, lo_a);
+    key.x += 0x9E3779B9u;
+    key.y += 0xBB67AE85u;
+  }
+  return ctr;
+}
+
+// Uniform in [0, 1) on the 2^-24 grid from word 0 of the Philox output for
+// counter (index, purpose, offset lo, offset hi) and key (seed lo, seed hi).
+__device__ __forceinline__ float philox_uniform(uint64_t seed, uint32_t index,
+                                                uint32_t purpose,
+                                                uint64_t offset) {
+  const uint4 r = philox4x32_10(
+      make_uint4(index, purpose, (uint32_t)offset, (uint32_t)(offset >> 32)),
+      make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
+  return (float)(r.x >> 8) * 5.9604644775390625e-08f;  // 2^-24
+}
+
+// ---------------------------------------------------------------------------
+// number formats
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float bf16_lo(uint32_t pair) {   // element 0
+  return __uint_as_float(pair << 16);
+}
+__device__ __forceinline__ float bf16_hi(uint32_t pair) {   // element 1
+  return __uint_as_float(pair & 0xFFFF0000u);
+}
+
+// two e4m3 bytes (low byte = element 0) -> two floats, exact
+__device__ __forceinline__ float2 e4m3x2_to_float2(uint16_t two) {
+  const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)two,
+                                                   __NV_E4M3);
+  return __half22float2(*reinterpret_cast<const __half2*>(&h));
+}
+
+// ---------------------------------------------------------------------------
+// reductions
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+  return v;
+}
+
+// Block-wide max / sum for blockDim.x a multiple of 32 (<= 1024).  `red`
+// is a 32-float shared array; every thread receives the result.
+__device__ __forceinline__ float block_max(float v, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = warp_max(v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  const int nw = blockDim.x >> 5;
+  v = lane < nw ? red[lane] : -INFINITY;
+  return warp_max(v);
+}
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  const int nw = blockDim.x >> 5;
+  v = lane < nw ? red[lane] : 0.f;
+  return warp_sum(v);
+}
+
+// Non-negative floats order like their bit patterns, so a row maximum of
+// |y| can be kept as an unsigned atomicMax.
+__device__ __forceinline__ void atomic_max_nonneg(unsigned int* addr, float v) {
+  atomicMax(addr, __float_as_uint(v));
+}
+
+}  // namespace sph

@@ -1,0 +1,76 @@
+// Internal interfaces between the C-ABI layer (sph_api.cu) and the kernel
+// translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace sph {
+
+enum Epilogue : int {
+  EPI_CLOUD = 0,     // +bias, optional unclipped store, clip, row |max|
+  EPI_ENDPOINT = 1,  // + code * row_scale (dequantized cloud partial)
+};
+
+enum WDtype : int { W_BF16 = 0, W_FP8 = 1 };
+
+// Device-side error bits (OR-ed into the context's status word).
+enum : unsigned int {
+  ERR_TIMEOUT = 1u,     // a bounded wait gave up
+  ERR_BAD_INDEX = 2u,   // an id or index outside its range was skipped
+};
+
+// Kernels launched by this thread (read by the tracing layer).
+extern thread_local long long launch_count;
+
+// One gathered contraction  acc[r, j] = sum_c h[r, c] * W[ids[j], c]
+// followed by an epilogue.  Pointers are device pointers.
+struct GatherGemm {
+  const float* h;          // [rows, K] fp32, row stride ld_h
+  int64_t ld_h;
+  int rows;
+  const void* W;           // [V, K] bf16 or e4m3, row stride ld_w elements
+  int64_t ld_w;
+  int w_dtype;             // WDtype
+  const float* w_scale;    // [V] (fp8 only)
+  int K;
+  const int32_t* ids;      // [n] sorted ids or nullptr (identity)
+  int n;
+  int act_bf16;            // round h to bf16 first
+  int epilogue;            // Epilogue
+  // EPI_CLOUD
+  const float* bias;       // [V] or nullptr
+  float clip;
+  float* partial_out;      // [rows, n] unclipped, or nullptr
+  float* Y;                // [rows, n] clipped (cloud) / fused z (endpoint)
+  unsigned* rowmax;        // [rows] bits of max |clipped y|, zeroed by caller
+  // EPI_ENDPOINT
+  const int8_t* codes;     // [rows, n]
+  const float* row_scale;  // [rows]
+  unsigned* status;        // device error word
+};
+
+// CUDA-core gathered GEMV (few rows); returns a cudaError_t.
+cudaError_t launch_gemv(const GatherGemm& g, int sm_count, cudaStream_t st);
+// Largest K the GEMV supports for a given row count.
+int gemv_max_k();
+
+// codes/row_scale from the clipped partials and their row maxima
+cudaError_t launch_quantize(const float* Y, const unsigned* rowmax, int rows,
+                            int n, int8_t* codes, float* row_scale,
+                            cudaStream_t st);
+
+// one inverse-CDF draw per row of Z (fp32 [rows, n])
+cudaError_t launch_sample(const float* Z, int rows, int n,
+                          const int32_t* ids, float inv_tau, uint64_t seed,
+                          uint64_t offset, int32_t* tokens, cudaStream_t st);
+int sample_max_n();
+
+// speculative verification, one CTA per session
+cudaError_t launch_verify(const float* Z, int sessions, int k, int n,
+                          const int32_t* ids, int V, float inv_tau,
+                          const int32_t* draft, const float* q,
+                          uint64_t seed, uint64_t offset, int32_t* n_acc,
+                          int32_t* next_token, cudaStream_t st);
+
+}  // namespace sph

@@ -1,0 +1,319 @@
+"""Thin Python binding of libsph (include/sph.h) over ctypes.
+
+Argument marshalling only: tensors are passed as device pointers with their
+leading dimensions, PyTorch supplies the device memory and the stream, and
+every step of the computation runs in the library's CUDA kernels.  There is
+no fallback: if the library is not built, importing this module raises.
+
+Functions carry the C names (sph_partial_logits, sph_fuse_sample,
+sph_verify_draft, ...) and take torch tensors; `Context` bundles a context
+handle with the current torch stream.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib",
+                         "libsph.so")
+
+SPH_OK = 0
+STATUS_NAMES = {0: "SPH_OK", 1: "SPH_ERR_INVALID_ARG", 2: "SPH_ERR_UNSUPPORTED",
+                3: "SPH_ERR_CUDA", 4: "SPH_ERR_TIMEOUT", 5: "SPH_ERR_OOM"}
+SPH_DTYPE_BF16, SPH_DTYPE_FP8_E4M3 = 0, 1
+SPH_ACT_FP32, SPH_ACT_BF16 = 0, 1
+
+_c_void_p = ctypes.c_void_p
+_i64 = ctypes.c_int64
+_u64 = ctypes.c_uint64
+_int = ctypes.c_int
+_f32 = ctypes.c_float
+_sz = ctypes.c_size_t
+
+PROF_CLASSES = 8
+PROF_NAMES = ("cloud_gemm", "quantize", "local_gemm", "sample", "verify",
+              "prep", "reserved6", "reserved7")
+
+
+class sph_profile(ctypes.Structure):
+    _fields_ = [("ms", ctypes.c_double * PROF_CLASSES),
+                ("calls", ctypes.c_int64 * PROF_CLASSES),
+                ("launches", ctypes.c_int64)]
+
+
+# name -> (restype, argtypes), mirroring include/sph.h
+_SIGNATURES = {
+    "sph_status_string": (ctypes.c_char_p, [_int]),
+    "sph_last_error": (ctypes.c_char_p, [_c_void_p]),
+    "sph_create": (_int, [_int, _c_void_p, ctypes.POINTER(_c_void_p)]),
+    "sph_destroy": (_int, [_c_void_p]),
+    "sph_set_stream": (_int, [_c_void_p, _c_void_p]),
+    "sph_sync": (_int, [_c_void_p]),
+    "sph_reserve": (_int, [_c_void_p, _i64, _i64, _i64]),
+    "sph_buffer_alloc": (_int, [_c_void_p, _sz, ctypes.POINTER(_c_void_p)]),
+    "sph_buffer_free": (_int, [_c_void_p, _c_void_p]),
+    "sph_buffer_ptr": (_c_void_p, [_c_void_p]),
+    "sph_profile_enable": (_int, [_c_void_p, _int]),
+    "sph_profile_read": (_int, [_c_void_p, ctypes.POINTER(sph_profile)]),
+    "sph_payload_bytes": (_sz, [_i64, _i64]),
+    "sph_keep_ids_from_mask": (_int, [_c_void_p, _i64, _c_void_p,
+                                      ctypes.POINTER(_i64)]),
+    "sph_partial_logits": (_int, [_c_void_p, _c_void_p, _i64, _i64, _c_void_p,
+                                  _int, _i64, _i64, _i64, _c_void_p, _c_void_p,
+                                  _c_void_p, _i64, _f32, _int, _c_void_p,
+                                  _c_void_p, _c_void_p, ctypes.POINTER(_sz)]),
+    "sph_fuse_sample": (_int, [_c_void_p, _c_void_p, _c_void_p, _i64, _c_void_p,
+                               _i64, _c_void_p, _i64, _i64, _i64, _c_void_p,
+                               _i64, _f32, _u64, _u64, _c_void_p, _c_void_p]),
+    "sph_verify_draft": (_int, [_c_void_p, _c_void_p, _i64, _i64, _c_void_p,
+                                _i64, _f32, _c_void_p, _c_void_p, _u64, _u64,
+                                _c_void_p, _c_void_p]),
+}
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(_LIB_PATH):
+        raise RuntimeError(
+            f"libsph.so is not built ({_LIB_PATH}); run "
+            "`python -c 'import __graft_entry__ as g; g.build()'` first")
+    lib = ctypes.CDLL(_LIB_PATH)
+    for name, (res, args) in _SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+lib = _load()
+LIB_PATH = _LIB_PATH
+
+
+class SphError(RuntimeError):
+    def __init__(self, status: int, detail: str):
+        self.status = status
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {detail}")
+
+
+def _check(ctx, status: int):
+    if status != SPH_OK:
+        detail = lib.sph_last_error(ctx).decode() if ctx else ""
+        raise SphError(status, detail)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _ld(t: torch.Tensor) -> int:
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("expected a 2-D tensor with unit inner stride")
+    return t.stride(0)
+
+
+def _need(t, dtype, name):
+    if t is None:
+        return
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+
+
+# ---------------------------------------------------------------------------
+# C functions with torch arguments
+# ---------------------------------------------------------------------------
+
+def sph_create(device: int = 0, stream: Optional[int] = None):
+    h = ctypes.c_void_p()
+    st = lib.sph_create(int(device), ctypes.c_void_p(stream or 0), ctypes.byref(h))
+    if st != SPH_OK:
+        raise SphError(st, "sph_create failed")
+    return h
+
+
+def sph_destroy(ctx):
+    _check(None, lib.sph_destroy(ctx))
+
+
+def sph_set_stream(ctx, stream: int):
+    _check(ctx, lib.sph_set_stream(ctx, ctypes.c_void_p(stream)))
+
+
+def sph_sync(ctx):
+    _check(ctx, lib.sph_sync(ctx))
+
+
+def sph_reserve(ctx, max_rows: int, max_n_keep: int, max_d: int):
+    _check(ctx, lib.sph_reserve(ctx, max_rows, max_n_keep, max_d))
+
+
+def sph_profile_enable(ctx, on: bool = True):
+    _check(ctx, lib.sph_profile_enable(ctx, 1 if on else 0))
+
+
+def sph_profile_read(ctx) -> dict:
+    """Accumulated device time (ms) and timed groups per kernel class, and
+    the number of kernels launched since tracing was enabled."""
+    p = sph_profile()
+    _check(ctx, lib.sph_profile_read(ctx, ctypes.byref(p)))
+    return dict(ms={PROF_NAMES[i]: p.ms[i] for i in range(PROF_CLASSES)},
+                calls={PROF_NAMES[i]: p.calls[i] for i in range(PROF_CLASSES)},
+                launches=int(p.launches))
+
+
+def sph_payload_bytes(rows: int, n_keep: int) -> int:
+    return int(lib.sph_payload_bytes(rows, n_keep))
+
+
+def sph_keep_ids_from_mask(mask_bits, V: int):
+    """Host helper: bitmask bytes (numpy uint8, ceil(V/8)) -> sorted ids."""
+    import numpy as np
+    mask = np.ascontiguousarray(mask_bits, dtype=np.uint8)
+    if mask.size * 8 < V:
+        raise ValueError("mask too short")
+    out = np.empty(V, dtype=np.int32)
+    n = _i64(0)
+    st = lib.sph_keep_ids_from_mask(mask.ctypes.data_as(ctypes.c_void_p), V,
+                                    out.ctypes.data_as(ctypes.c_void_p),
+                                    ctypes.byref(n))
+    if st != SPH_OK:
+        raise SphError(st, "sph_keep_ids_from_mask failed")
+    return out[: n.value].copy()
+
+
+def sph_partial_logits(ctx, h_cloud, W_h, *, keep_ids=None, clip=30.0,
+                       w_row_scale=None, bias=None, act_mode=SPH_ACT_FP32,
+                       codes=None, row_scale=None, partial_out=None):
+    """Cloud call.  Returns (codes int8 [R, n], row_scale fp32 [R],
+    payload_bytes).  h_cloud fp32 [R, d_h] (any row stride); W_h bf16 or
+    float8_e4m3fn [V, d_h]."""
+    _need(h_cloud, torch.float32, "h_cloud")
+    if W_h.dtype == torch.bfloat16:
+        wdt = SPH_DTYPE_BF16
+    elif W_h.dtype == torch.float8_e4m3fn:
+        wdt = SPH_DTYPE_FP8_E4M3
+    else:
+        raise ValueError("W_h must be bfloat16 or float8_e4m3fn")
+    _need(W_h, None, "W_h")
+    _need(keep_ids, torch.int32, "keep_ids")
+    _need(w_row_scale, torch.float32, "w_row_scale")
+    _need(bias, torch.float32, "bias")
+    R, d_h = h_cloud.shape
+    V = W_h.shape[0]
+    n = V if keep_ids is None else keep_ids.numel()
+    dev = h_cloud.device
+    if codes is None:
+        codes = torch.empty(R, n, dtype=torch.int8, device=dev)
+    if row_scale is None:
+        row_scale = torch.empty(R, dtype=torch.float32, device=dev)
+    _need(codes, torch.int8, "codes")
+    _need(row_scale, torch.float32, "row_scale")
+    _need(partial_out, torch.float32, "partial_out")
+    pb = _sz(0)
+    _check(ctx, lib.sph_partial_logits(
+        ctx, _ptr(h_cloud), R, _ld(h_cloud), _ptr(W_h), wdt, V, d_h, _ld(W_h),
+        _ptr(w_row_scale), _ptr(bias), _ptr(keep_ids), n, float(clip),
+        int(act_mode), _ptr(codes), _ptr(row_scale), _ptr(partial_out),
+        ctypes.byref(pb)))
+    return codes, row_scale, pb.value
+
+
+def sph_fuse_sample(ctx, codes, row_scale, h_local, W_l, *, keep_ids=None,
+                    temperature=1.0, seed=0, offset=0, tokens=None,
+                    fused_logits_out=None):
+    """Endpoint call.  Returns tokens int32 [R] (vocabulary ids)."""
+    _need(codes, torch.int8, "codes")
+    _need(row_scale, torch.float32, "row_scale")
+    _need(h_local, torch.float32, "h_local")
+    _need(W_l, torch.bfloat16, "W_l")
+    _need(keep_ids, torch.int32, "keep_ids")
+    _need(fused_logits_out, torch.float32, "fused_logits_out")
+    R, d_l = h_local.shape
+    V = W_l.shape[0]
+    n = V if keep_ids is None else keep_ids.numel()
+    if tokens is None:
+        tokens = torch.empty(R, dtype=torch.int32, device=h_local.device)
+    _need(tokens, torch.int32, "tokens")
+    _check(ctx, lib.sph_fuse_sample(
+        ctx, _ptr(codes), _ptr(row_scale), R, _ptr(h_local), _ld(h_local),
+        _ptr(W_l), V, d_l, _ld(W_l), _ptr(keep_ids), n, float(temperature),
+        int(seed) & 0xFFFFFFFFFFFFFFFF, int(offset) & 0xFFFFFFFFFFFFFFFF,
+        _ptr(tokens), _ptr(fused_logits_out)))
+    return tokens
+
+
+def sph_verify_draft(ctx, target_logits, sessions: int, k: int, draft_tokens,
+                     *, keep_ids=None, draft_probs=None, temperature=1.0,
+                     seed=0, offset=0, n_accepted=None, next_token=None):
+    """Speculative verification.  Returns (n_accepted, next_token)."""
+    _need(target_logits, torch.float32, "target_logits")
+    _need(draft_tokens, torch.int32, "draft_tokens")
+    _need(draft_probs, torch.float32, "draft_probs")
+    _need(keep_ids, torch.int32, "keep_ids")
+    n = target_logits.shape[-1]
+    dev = target_logits.device
+    if n_accepted is None:
+        n_accepted = torch.empty(sessions, dtype=torch.int32, device=dev)
+    if next_token is None:
+        next_token = torch.empty(sessions, dtype=torch.int32, device=dev)
+    _check(ctx, lib.sph_verify_draft(
+        ctx, _ptr(target_logits), sessions, k, _ptr(keep_ids), n,
+        float(temperature), _ptr(draft_tokens), _ptr(draft_probs),
+        int(seed) & 0xFFFFFFFFFFFFFFFF, int(offset) & 0xFFFFFFFFFFFFFFFF,
+        _ptr(n_accepted), _ptr(next_token)))
+    return n_accepted, next_token
+
+
+class Context:
+    """A library context on `device`, issuing work on torch's current
+    stream of that device (re-read at every call)."""
+
+    def __init__(self, device: int = 0):
+        self.device = int(device)
+        self._stream = torch.cuda.current_stream(self.device).cuda_stream
+        self.handle = sph_create(self.device, self._stream)
+
+    def _follow_stream(self):
+        s = torch.cuda.current_stream(self.device).cuda_stream
+        if s != self._stream:
+            sph_set_stream(self.handle, s)
+            self._stream = s
+
+    def reserve(self, max_rows, max_n_keep, max_d):
+        sph_reserve(self.handle, max_rows, max_n_keep, max_d)
+
+    def partial_logits(self, *a, **kw):
+        self._follow_stream()
+        return sph_partial_logits(self.handle, *a, **kw)
+
+    def fuse_sample(self, *a, **kw):
+        self._follow_stream()
+        return sph_fuse_sample(self.handle, *a, **kw)
+
+    def verify_draft(self, *a, **kw):
+        self._follow_stream()
+        return sph_verify_draft(self.handle, *a, **kw)
+
+    def sync(self):
+        sph_sync(self.handle)
+
+    def profile_enable(self, on: bool = True):
+        self._follow_stream()
+        sph_profile_enable(self.handle, on)
+
+    def profile_read(self) -> dict:
+        return sph_profile_read(self.handle)
+
+    def close(self):
+        if self.handle is not None:
+            sph_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

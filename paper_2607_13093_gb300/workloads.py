@@ -300,3 +300,20 @@ def algorithmic_flops(R: int, n: int, d: int) -> int:
 
 def rows_per_second(rows: int, seconds: float) -> float:
     return rows / seconds if seconds > 0 else math.inf
+
+
+def make_payload(rows: int, n: int, seed: int, device="cpu"):
+    """A synthetic cloud payload (int8 codes in [-127, 127] and positive fp32
+    row scales) for exercising the endpoint call on its own."""
+    g = _gen(device, seed)
+    codes = torch.randn(rows, n, generator=g, device=device) * 40.0
+    codes = codes.round().clamp(-127, 127).to(torch.int8)
+    scale = (torch.rand(rows, generator=g, device=device) * 0.05 + 0.01).float()
+    return codes.contiguous(), scale.contiguous()
+
+
+def make_target_logits(rows: int, n: int, seed: int, device="cpu",
+                       std: float = 1.5):
+    """Synthetic fused target logits for exercising verification alone."""
+    g = _gen(device, seed)
+    return (torch.randn(rows, n, generator=g, device=device) * std).contiguous()

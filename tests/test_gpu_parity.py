@@ -1,0 +1,187 @@
+"""GPU <-> oracle parity through the C-ABI (needs a GPU; marked gpu).
+
+Small cases span several tiles and ragged tails; the five named workloads
+run at full size in the launch configuration the benchmark times, with the
+oracle checking sampled rows."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_13093_gb300 import workloads as wl
+from _parity import (check_cloud, check_endpoint, check_verify, oracle_cloud,
+                     np_)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    from paper_2607_13093_gb300 import build_lib
+    build_lib.build()
+    from paper_2607_13093_gb300 import sph
+    c = sph.Context(0)
+    yield c
+    c.close()
+
+
+DEV = "cuda"
+
+
+def small(**kw):
+    kw.setdefault("seed", 77)
+    return wl.make_workload(device=DEV, **kw)
+
+
+# ---------------------------------------------------------------------------
+# cloud call: shapes x paths
+# ---------------------------------------------------------------------------
+
+CLOUD_CASES = [
+    # name, kwargs
+    ("tiny-full", dict(V=8192, d=512, d_l=64, rows=1, n_keep=2048)),
+    ("decode-small", dict(V=4000, d=1024, d_l=128, rows=32, n_keep=1500, tau=0.8)),
+    ("spec-small", dict(V=6000, d=640, d_l=128, rows=20, n_keep=2400, sessions=4, k=4)),
+    ("fp8-small", dict(V=3000, d=1280, d_l=256, rows=16, n_keep=3000, w_dtype="fp8", clip=40.0)),
+    ("rows3", dict(V=2000, d=300, d_l=44, rows=3, n_keep=700)),
+    ("rows17", dict(V=2000, d=300, d_l=44, rows=17, n_keep=701)),
+    ("rows64", dict(V=3000, d=520, d_l=8, rows=64, n_keep=1000)),
+    ("rows130", dict(V=1500, d=392, d_l=8, rows=130, n_keep=1300)),
+    ("keep1", dict(V=500, d=136, d_l=8, rows=2, n_keep=1, run_lo=1, run_hi=1)),
+    ("keep7", dict(V=500, d=136, d_l=8, rows=5, n_keep=7, run_lo=1, run_hi=3)),
+    ("keep127", dict(V=500, d=136, d_l=8, rows=9, n_keep=127, run_lo=2, run_hi=9)),
+    ("bias", dict(V=1000, d=264, d_l=8, rows=4, n_keep=400, with_bias=True)),
+]
+
+
+@pytest.mark.parametrize("name,kw", CLOUD_CASES, ids=[c[0] for c in CLOUD_CASES])
+def test_cloud_parity(ctx, name, kw):
+    w = small(**kw)
+    check_cloud(ctx, w)
+
+
+@pytest.mark.parametrize("rows", [1, 8, 40])
+def test_cloud_bf16_activation_mode(ctx, rows):
+    w = small(V=3000, d=776, d_l=8, rows=rows, n_keep=1200)
+    check_cloud(ctx, w, act_mode="bf16")
+
+
+def test_cloud_clipping_bites(ctx):
+    w = small(V=2000, d=1032, d_l=8, rows=6, n_keep=900, clip=0.5)
+    codes, scale, part = check_cloud(ctx, w)
+    assert (np_(part).__abs__() > 0.5).any()          # clip was exercised
+    assert np.allclose(np_(scale), np.float32(0.5 / 127))
+
+
+def test_cloud_zero_row_and_edge_ids(ctx):
+    w = small(V=1000, d=264, d_l=8, rows=5, n_keep=300)
+    w.h[2].zero_()
+    ids = w.keep_ids.clone()
+    ids[0] = 0
+    ids[-1] = w.V - 1
+    w.keep_ids = torch.unique(ids).to(torch.int32)
+    codes, scale, _ = check_cloud(ctx, w)
+    assert np_(scale)[2] == 0 and not np_(codes)[2].any()
+
+
+def test_cloud_odd_hidden_width_and_strides(ctx):
+    # d_h = 37 (not a multiple of anything) inside a padded weight stride
+    base = small(V=900, d=45, d_l=8, rows=7, n_keep=350)
+    Wpad = torch.zeros(base.V, 40, dtype=torch.bfloat16, device=DEV)
+    Wpad[:, :37] = base.W_h
+    base.W_h = Wpad[:, :37]
+    check_cloud(ctx, base)
+
+
+# ---------------------------------------------------------------------------
+# endpoint call: fuse + mask + softmax + sample on the oracle's payload
+# ---------------------------------------------------------------------------
+
+ENDPOINT_CASES = [
+    ("tiny-full", dict(V=8192, d=512, d_l=64, rows=1, n_keep=2048)),
+    ("decode-small", dict(V=4000, d=1024, d_l=256, rows=32, n_keep=1500, tau=0.8)),
+    ("rows17-keep7", dict(V=500, d=136, d_l=40, rows=17, n_keep=7, run_lo=1, run_hi=3)),
+    ("full-vocab", dict(V=3000, d=1280, d_l=264, rows=16, n_keep=3000)),
+    ("rows70", dict(V=2500, d=600, d_l=72, rows=70, n_keep=1100)),
+]
+
+
+@pytest.mark.parametrize("name,kw", ENDPOINT_CASES, ids=[c[0] for c in ENDPOINT_CASES])
+def test_endpoint_parity(ctx, name, kw):
+    w = small(**kw)
+    ref = oracle_cloud(w)
+    codes = torch.from_numpy(ref["codes"])
+    scale = torch.from_numpy(ref["row_scale"])
+    for off in (0, 1, 12345):
+        w.offset = off
+        check_endpoint(ctx, w, codes, scale)
+
+
+@pytest.mark.parametrize("tau", [0.05, 0.8, 3.0])
+def test_endpoint_temperatures(ctx, tau):
+    w = small(V=2000, d=300, d_l=64, rows=24, n_keep=800, tau=tau)
+    codes, scale = wl.make_payload(w.rows, w.n_keep, seed=5)
+    check_endpoint(ctx, w, codes, scale)
+
+
+def test_endpoint_masked_ids_never_sampled(ctx):
+    w = small(V=3000, d=200, d_l=64, rows=64, n_keep=300, tau=5.0)
+    codes, scale = wl.make_payload(w.rows, w.n_keep, seed=6)
+    ids = set(np_(w.keep_ids).tolist())
+    seen = set()
+    for off in range(50):
+        tok = ctx.fuse_sample(codes.to(DEV), scale.to(DEV), w.h_local, w.W_l,
+                              keep_ids=w.keep_ids, temperature=w.tau,
+                              seed=w.seed, offset=off)
+        seen.update(np_(tok).tolist())
+    assert seen <= ids and len(seen) > 50
+
+
+# ---------------------------------------------------------------------------
+# verification
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("S,k,n,greedy", [(4, 4, 2400, False), (9, 1, 300, False),
+                                          (5, 3, 1000, True), (64, 4, 5000, False)])
+def test_verify_parity(ctx, S, k, n, greedy):
+    w = small(V=3 * n, d=96, d_l=8, rows=S * (k + 1), n_keep=n, sessions=S, k=k)
+    if greedy:
+        w.draft_probs = None
+    for seed in (3, 4):
+        target = wl.make_target_logits(w.rows, w.n_keep, seed=seed, std=1.0)
+        w.offset = seed
+        check_verify(ctx, w, target)
+
+
+def test_verify_accepts_drafts_equal_to_target(ctx):
+    # q == p  =>  every draft accepted (r < 1 = p/q), bonus from p_k
+    S, k, n = 6, 3, 500
+    w = small(V=2 * n, d=96, d_l=8, rows=S * (k + 1), n_keep=n, sessions=S, k=k)
+    target = wl.make_target_logits(w.rows, n, seed=8, std=1.0)
+    p = torch.softmax(target.double(), dim=1).float().view(S, k + 1, n)
+    w.draft_probs = p[:, :k].contiguous().to(DEV)
+    n_acc, _, _ = check_verify(ctx, w, target)
+    assert (np_(n_acc) == k).all()
+
+
+# ---------------------------------------------------------------------------
+# full-size workloads, sampled rows
+# ---------------------------------------------------------------------------
+
+FULL = [("tiny", None, None), ("decode", None, None), ("spec", None, None),
+        ("fp8", None, None), ("sweep", 1, 0.1), ("sweep", 64, 0.5),
+        ("sweep", 1024, 1.0)]
+
+
+@pytest.mark.parametrize("name,rows,keep", FULL,
+                         ids=[f"{n}-{r}-{k}" for n, r, k in FULL])
+def test_full_size_sampled_rows(ctx, name, rows, keep):
+    w = wl.workload(name, device=DEV, rows=rows, keep_frac=keep)
+    sample = sorted({0, w.rows // 2, w.rows - 1})
+    codes, scale, _ = check_cloud(ctx, w, rows=sample)
+    # endpoint on a synthetic payload of the same shape (an input shared by
+    # both sides), full launch, sampled rows checked
+    pc, ps = wl.make_payload(w.rows, w.n_keep, seed=11, device=DEV)
+    check_endpoint(ctx, w, pc, ps, rows=sample)
+    if w.sessions:
+        target = wl.make_target_logits(w.rows, w.n_keep, seed=12, device=DEV)
+        check_verify(ctx, w, target.cpu())
