@@ -77,6 +77,23 @@ def test_split_partials_equal_full_head(act_mode):
                                z_full, rtol=1e-12, atol=1e-14)
 
 
+def test_fused_logits_within_dequantization_bound():
+    """z = code * s + z_end reproduces the full head (Eq. 13) to within half
+    a quantization step (Eq. 18) when nothing is clipped."""
+    w = tiny(with_bias=False)
+    ids = w.keep_ids.numpy()
+    h = w.h.numpy().astype(np.float64)
+    W_full = torch.cat([w.W_l, w.W_h], dim=1).double().numpy()
+    z_full = brute_full_head(h, W_full, None)[:, ids]
+    cloud = oracle.partial_logits(w.h_cloud.numpy(), bits16(w.W_h), keep_ids=ids,
+                                  clip=1e30)
+    zl = oracle.local_partial(w.h_local.numpy(), bits16(w.W_l), ids)
+    z = oracle.fuse(cloud["codes"], cloud["row_scale"], zl)
+    half = cloud["row_scale"].astype(np.float64)[:, None] / 2
+    assert np.all(np.abs(z - z_full) <= half * (1 + 1e-9))
+    assert np.any(np.abs(z - z_full) > half * 0.5)     # the bound is not slack
+
+
 def test_fp8_partials_equal_full_head():
     w = tiny(with_bias=False, w_dtype="fp8")
     ids = w.keep_ids.numpy()
