@@ -178,6 +178,46 @@ sph_status sph_partial_logits(sph_ctx* ctx,
                               int8_t* codes, float* row_scale,
                               float* partial_out, size_t* payload_bytes);
 
+/* Allocation-free cloud call.  The paper has no counterpart: this is a
+ * deployment variant of sph_partial_logits for callers that cannot allocate
+ * device memory when they run the cloud step (an allocator owned or locked
+ * by another runtime, a fixed-size memory pool, or a serving loop that must
+ * never call cudaMalloc, which can synchronise the device).  Such callers
+ * cannot create a context, so this call takes the device and stream
+ * directly and allocates nothing: no cudaMalloc, no cudaFree, no allocating
+ * library routine.  Its scratch (clipped fp32 partials and per-row maxima)
+ * lives in one fixed device array of SPH_NOALLOC_SCRATCH_BYTES inside the
+ * library, which every GPU that loads the library holds until the process
+ * exits.
+ *   - Same arguments, results and errors as sph_partial_logits, plus
+ *     `device` (made current for the call), `cuda_stream` (a cudaStream_t,
+ *     NULL = legacy default stream) and an optional host buffer err_msg of
+ *     err_msg_len bytes that receives a description of any failure.
+ *   - Size limit: round_up(rows*n_keep*4, 256) + round_up(rows*4, 256) must
+ *     not exceed SPH_NOALLOC_SCRATCH_BYTES; larger calls return
+ *     SPH_ERR_UNSUPPORTED without launching anything.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first call
+ *     before any stream capture.
+ *   - All calls share the one array and it keeps the last call's contents
+ *     (the row maxima are cleared by each call).  Calls whose kernels overlap
+ *     on the GPU -- on different streams or from different host threads --
+ *     race and corrupt each other's results; serialise them. */
+#define SPH_NOALLOC_SCRATCH_BYTES ((size_t)8 << 20)
+sph_status sph_partial_logits_noalloc(int device, void* cuda_stream,
+                                      const float* h_cloud, int64_t rows,
+                                      int64_t ld_h, const void* W_h,
+                                      sph_dtype w_dtype, int64_t V,
+                                      int64_t d_h, int64_t ld_w,
+                                      const float* w_row_scale,
+                                      const float* bias,
+                                      const int32_t* keep_ids, int64_t n_keep,
+                                      float clip, sph_act_mode act_mode,
+                                      int8_t* codes, float* row_scale,
+                                      float* partial_out,
+                                      size_t* payload_bytes, char* err_msg,
+                                      size_t err_msg_len);
+
 /* Endpoint call (Eq. 11, Eq. 13, Eq. 14, Eq. 15; Algorithm 1 "fuses partial
  * logits, applies language masking, and samples"):
  *   z[r, j]   = codes[r, j] * row_scale[r]

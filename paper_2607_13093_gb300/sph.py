@@ -65,6 +65,12 @@ _SIGNATURES = {
                                   _int, _i64, _i64, _i64, _c_void_p, _c_void_p,
                                   _c_void_p, _i64, _f32, _int, _c_void_p,
                                   _c_void_p, _c_void_p, ctypes.POINTER(_sz)]),
+    "sph_partial_logits_noalloc": (_int, [_int, _c_void_p, _c_void_p, _i64, _i64,
+                                          _c_void_p, _int, _i64, _i64, _i64,
+                                          _c_void_p, _c_void_p, _c_void_p, _i64,
+                                          _f32, _int, _c_void_p, _c_void_p,
+                                          _c_void_p, ctypes.POINTER(_sz),
+                                          ctypes.c_char_p, _sz]),
     "sph_fuse_sample": (_int, [_c_void_p, _c_void_p, _c_void_p, _i64, _c_void_p,
                                _i64, _c_void_p, _i64, _i64, _i64, _c_void_p,
                                _i64, _f32, _u64, _u64, _c_void_p, _c_void_p]),
@@ -219,6 +225,48 @@ def sph_partial_logits(ctx, h_cloud, W_h, *, keep_ids=None, clip=30.0,
         int(act_mode), _ptr(codes), _ptr(row_scale), _ptr(partial_out),
         ctypes.byref(pb)))
     return codes, row_scale, pb.value
+
+
+NOALLOC_SCRATCH_BYTES = 8 << 20
+
+
+def sph_partial_logits_noalloc(h_cloud, W_h, *, codes, row_scale,
+                               keep_ids=None, clip=30.0, w_row_scale=None,
+                               bias=None, act_mode=SPH_ACT_FP32,
+                               partial_out=None, device=None, stream=None):
+    """Allocation-free cloud call for callers that cannot allocate device
+    memory while they run (see include/sph.h): no context, caller-provided
+    outputs, scratch in the library's fixed device array.  Returns the
+    payload byte count; raises SphError with the library's message."""
+    if W_h.dtype == torch.bfloat16:
+        wdt = SPH_DTYPE_BF16
+    elif W_h.dtype == torch.float8_e4m3fn:
+        wdt = SPH_DTYPE_FP8_E4M3
+    else:
+        raise ValueError("W_h must be bfloat16 or float8_e4m3fn")
+    for t, dt, name in ((h_cloud, torch.float32, "h_cloud"), (W_h, None, "W_h"),
+                        (keep_ids, torch.int32, "keep_ids"),
+                        (w_row_scale, torch.float32, "w_row_scale"),
+                        (bias, torch.float32, "bias"), (codes, torch.int8, "codes"),
+                        (row_scale, torch.float32, "row_scale"),
+                        (partial_out, torch.float32, "partial_out")):
+        _need(t, dt, name)
+    R, d_h = h_cloud.shape
+    V = W_h.shape[0]
+    n = V if keep_ids is None else keep_ids.numel()
+    dev = h_cloud.device.index if device is None else int(device)
+    if stream is None:
+        stream = torch.cuda.current_stream(dev).cuda_stream
+    pb = _sz(0)
+    msg = ctypes.create_string_buffer(256)
+    st = lib.sph_partial_logits_noalloc(
+        dev, ctypes.c_void_p(stream), _ptr(h_cloud), R, _ld(h_cloud), _ptr(W_h),
+        wdt, V, d_h, _ld(W_h), _ptr(w_row_scale), _ptr(bias), _ptr(keep_ids), n,
+        float(clip), int(act_mode), _ptr(codes), _ptr(row_scale),
+        _ptr(partial_out), ctypes.byref(pb), msg, len(msg))
+    if st != SPH_OK:
+        raise SphError(st, msg.value.decode())
+    return pb.value
 
 
 def sph_fuse_sample(ctx, codes, row_scale, h_local, W_l, *, keep_ids=None,
