@@ -94,6 +94,20 @@ const char* sph_status_string(sph_status status);
 sph_status sph_reserve(sph_ctx* ctx, int64_t max_rows, int64_t max_n_keep,
                        int64_t max_d);
 
+/* Tunables of a context. */
+typedef enum sph_option {
+  SPH_OPT_TC_MIN_ROWS = 0,  /* row count from which the tcgen05 tensor-core
+                               kernels replace the CUDA-core GEMV (default 4;
+                               1 forces tensor cores, a huge value forces the
+                               GEMV; fp8 weights always use the GEMV path)    */
+  SPH_OPT_SPIN_LIMIT = 1    /* clock cycles a device-side wait may spin before
+                               it gives up and the call reports
+                               SPH_ERR_TIMEOUT (default 2^34, >= 1)           */
+} sph_option;
+
+/* Set a tunable (SPH_ERR_INVALID_ARG for an unknown option or a value < 1). */
+sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value);
+
 /* Optional device allocation helpers for callers without their own
  * allocator.  sph_buffer_ptr returns the device address (NULL for NULL). */
 sph_status sph_buffer_alloc(sph_ctx* ctx, size_t bytes, sph_buffer** out);

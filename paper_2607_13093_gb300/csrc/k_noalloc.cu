@@ -132,7 +132,7 @@ extern "C" sph_status sph_partial_logits_noalloc(
     if (e == cudaSuccess) {
       sph::GatherGemm gg{};
       gg.h = h_cloud; gg.ld_h = ld_h; gg.rows = (int)rows;
-      gg.W = W_h; gg.ld_w = ld_w;
+      gg.W = W_h; gg.ld_w = ld_w; gg.V = V;
       gg.w_dtype = w_dtype == SPH_DTYPE_BF16 ? sph::W_BF16 : sph::W_FP8;
       gg.w_scale = w_row_scale; gg.K = (int)d_h;
       gg.ids = keep_ids; gg.n = (int)n_keep;

@@ -28,6 +28,8 @@ struct sph_ctx {
   void* scratch = nullptr;          // arena for per-call temporaries
   size_t scratch_cap = 0;
   unsigned* status = nullptr;       // device error word (sph::ERR_* bits)
+  int64_t tc_min_rows = 4;          // SPH_OPT_TC_MIN_ROWS
+  long long spin_limit = 1ll << 34; // SPH_OPT_SPIN_LIMIT
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -112,11 +114,23 @@ struct Carve {
   }
 };
 
-size_t partial_scratch_bytes(int64_t rows, int64_t n) {
-  return align_up((size_t)rows * n * 4, 256) + align_up((size_t)rows * 4, 256);
+bool use_tc(const sph_ctx* ctx, int64_t rows, int w_dtype) {
+  return rows >= ctx->tc_min_rows && w_dtype == sph::W_BF16;
 }
-size_t fuse_scratch_bytes(int64_t rows, int64_t n) {
-  return align_up((size_t)rows * n * 4, 256);
+
+size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_bf16,
+                int w_dtype) {
+  if (!use_tc(ctx, rows, w_dtype)) return 0;
+  return sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count).scratch_bytes;
+}
+
+size_t partial_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K,
+                             int act_bf16, int w_dtype) {
+  return align_up((size_t)rows * n * 4, 256) + align_up((size_t)rows * 4, 256) +
+         tc_bytes(ctx, rows, n, K, act_bf16, w_dtype);
+}
+size_t fuse_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K) {
+  return align_up((size_t)rows * n * 4, 256) + tc_bytes(ctx, rows, n, K, 0, sph::W_BF16);
 }
 
 bool finite_pos(float x) { return std::isfinite(x) && x > 0.f; }
@@ -304,10 +318,24 @@ sph_status sph_reserve(sph_ctx* ctx, int64_t max_rows, int64_t max_n_keep,
   if (!ctx || max_rows < 1 || max_n_keep < 1 || max_d < 1)
     return fail(ctx, SPH_ERR_INVALID_ARG, "sph_reserve: sizes must be >= 1");
   DeviceGuard g(ctx->device);
-  size_t need = partial_scratch_bytes(max_rows, max_n_keep);
-  const size_t f = fuse_scratch_bytes(max_rows, max_n_keep);
+  size_t need = 0;
+  for (int act = 0; act < 2; ++act) {
+    const size_t a = partial_scratch_bytes(ctx, max_rows, max_n_keep, max_d, act, sph::W_BF16);
+    if (a > need) need = a;
+  }
+  const size_t f = fuse_scratch_bytes(ctx, max_rows, max_n_keep, max_d);
   if (f > need) need = f;
   return ensure_scratch(ctx, need);
+}
+
+sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  if (value < 1) return fail(ctx, SPH_ERR_INVALID_ARG, "option value must be >= 1");
+  switch (option) {
+    case SPH_OPT_TC_MIN_ROWS: ctx->tc_min_rows = value; return SPH_OK;
+    case SPH_OPT_SPIN_LIMIT: ctx->spin_limit = value; return SPH_OK;
+  }
+  return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
 }
 
 sph_status sph_buffer_alloc(sph_ctx* ctx, size_t bytes, sph_buffer** out) {
@@ -367,7 +395,9 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
 
   DeviceGuard g(ctx->device);
   if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
-  st = ensure_scratch(ctx, partial_scratch_bytes(rows, n_keep));
+  const int wdt = w_dtype == SPH_DTYPE_BF16 ? sph::W_BF16 : sph::W_FP8;
+  const int act_bf16 = act_mode == SPH_ACT_BF16;
+  st = ensure_scratch(ctx, partial_scratch_bytes(ctx, rows, n_keep, d_h, act_bf16, wdt));
   if (st) return st;
   Carve c(ctx->scratch);
   float* Y = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
@@ -377,17 +407,25 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
 
   sph::GatherGemm gg{};
   gg.h = h_cloud; gg.ld_h = ld_h; gg.rows = (int)rows;
-  gg.W = W_h; gg.ld_w = ld_w;
-  gg.w_dtype = w_dtype == SPH_DTYPE_BF16 ? sph::W_BF16 : sph::W_FP8;
+  gg.W = W_h; gg.ld_w = ld_w; gg.V = V;
+  gg.w_dtype = wdt;
   gg.w_scale = w_row_scale; gg.K = (int)d_h;
   gg.ids = keep_ids; gg.n = (int)n_keep;
-  gg.act_bf16 = act_mode == SPH_ACT_BF16;
+  gg.act_bf16 = act_bf16;
   gg.epilogue = sph::EPI_CLOUD;
   gg.bias = bias; gg.clip = clip; gg.partial_out = partial_out;
   gg.Y = Y; gg.rowmax = rowmax; gg.status = ctx->status;
-  st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
-                       return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
-                     }), "gemv launch");
+  if (use_tc(ctx, rows, wdt)) {
+    const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_h, act_bf16, ctx->sm_count);
+    void* tcs = c.take(pl.scratch_bytes);
+    st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
+                         return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
+                       }), "tensor-core launch");
+  } else {
+    st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
+                         return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
+                       }), "gemv launch");
+  }
   if (st) return st;
   return launch_status(ctx, traced(ctx, SPH_PROF_QUANTIZE, [&] {
                          return sph::launch_quantize(Y, rowmax, (int)rows, (int)n_keep,
@@ -419,22 +457,28 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
 
   DeviceGuard g(ctx->device);
   if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
-  float* Z = fused_logits_out;
-  if (!Z) {
-    st = ensure_scratch(ctx, fuse_scratch_bytes(rows, n_keep));
-    if (st) return st;
-    Carve c(ctx->scratch);
-    Z = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
-  }
+  st = ensure_scratch(ctx, fuse_scratch_bytes(ctx, rows, n_keep, d_l));
+  if (st) return st;
+  Carve c(ctx->scratch);
+  float* Z = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
+  if (fused_logits_out) Z = fused_logits_out;
   sph::GatherGemm gg{};
   gg.h = h_local; gg.ld_h = ld_hl; gg.rows = (int)rows;
-  gg.W = W_l; gg.ld_w = ld_wl; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
+  gg.W = W_l; gg.ld_w = ld_wl; gg.V = V; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
   gg.ids = keep_ids; gg.n = (int)n_keep;
   gg.epilogue = sph::EPI_ENDPOINT;
   gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale; gg.status = ctx->status;
-  st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
-                       return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
-                     }), "gemv launch");
+  if (use_tc(ctx, rows, sph::W_BF16)) {
+    const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0, ctx->sm_count);
+    void* tcs = c.take(pl.scratch_bytes);
+    st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
+                         return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
+                       }), "tensor-core launch");
+  } else {
+    st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
+                         return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
+                       }), "gemv launch");
+  }
   if (st) return st;
   return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                          return sph::launch_sample(Z, (int)rows, (int)n_keep, keep_ids,

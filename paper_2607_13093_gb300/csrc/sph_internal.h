@@ -34,6 +34,7 @@ struct GatherGemm {
   int w_dtype;             // WDtype
   const float* w_scale;    // [V] (fp8 only)
   int K;
+  int64_t V;               // rows of W
   const int32_t* ids;      // [n] sorted ids or nullptr (identity)
   int n;
   int act_bf16;            // round h to bf16 first
@@ -54,6 +55,19 @@ struct GatherGemm {
 cudaError_t launch_gemv(const GatherGemm& g, int sm_count, cudaStream_t st);
 // Largest K the GEMV supports for a given row count.
 int gemv_max_k();
+
+// Tensor-core path (k_tc.cu): sizes, work split and scratch of one call.
+struct TcPlan {
+  int hilo, RB, BN, Rp, KB, Kp, NT, G, stages;
+  long long T;
+  size_t hs_bytes, p_bytes, cnt_bytes, scratch_bytes, smem_bytes;
+  bool ok;
+};
+TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count);
+// Launch the operand split and the tcgen05 kernel; `scratch` holds
+// plan.scratch_bytes bytes.  bf16 weights only.
+cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,
+                      long long spin_limit, cudaStream_t st);
 
 // codes/row_scale from the clipped partials and their row maxima
 cudaError_t launch_quantize(const float* Y, const unsigned* rowmax, int rows,

@@ -25,6 +25,7 @@ STATUS_NAMES = {0: "SPH_OK", 1: "SPH_ERR_INVALID_ARG", 2: "SPH_ERR_UNSUPPORTED",
                 3: "SPH_ERR_CUDA", 4: "SPH_ERR_TIMEOUT", 5: "SPH_ERR_OOM"}
 SPH_DTYPE_BF16, SPH_DTYPE_FP8_E4M3 = 0, 1
 SPH_ACT_FP32, SPH_ACT_BF16 = 0, 1
+SPH_OPT_TC_MIN_ROWS, SPH_OPT_SPIN_LIMIT = 0, 1
 
 _c_void_p = ctypes.c_void_p
 _i64 = ctypes.c_int64
@@ -53,6 +54,7 @@ _SIGNATURES = {
     "sph_set_stream": (_int, [_c_void_p, _c_void_p]),
     "sph_sync": (_int, [_c_void_p]),
     "sph_reserve": (_int, [_c_void_p, _i64, _i64, _i64]),
+    "sph_set_option": (_int, [_c_void_p, _int, _i64]),
     "sph_buffer_alloc": (_int, [_c_void_p, _sz, ctypes.POINTER(_c_void_p)]),
     "sph_buffer_free": (_int, [_c_void_p, _c_void_p]),
     "sph_buffer_ptr": (_c_void_p, [_c_void_p]),
@@ -154,6 +156,10 @@ def sph_sync(ctx):
 
 def sph_reserve(ctx, max_rows: int, max_n_keep: int, max_d: int):
     _check(ctx, lib.sph_reserve(ctx, max_rows, max_n_keep, max_d))
+
+
+def sph_set_option(ctx, option: int, value: int):
+    _check(ctx, lib.sph_set_option(ctx, int(option), int(value)))
 
 
 def sph_profile_enable(ctx, on: bool = True):
@@ -332,6 +338,9 @@ class Context:
 
     def reserve(self, max_rows, max_n_keep, max_d):
         sph_reserve(self.handle, max_rows, max_n_keep, max_d)
+
+    def set_option(self, option: int, value: int):
+        sph_set_option(self.handle, option, value)
 
     def partial_logits(self, *a, **kw):
         self._follow_stream()

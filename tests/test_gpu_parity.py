@@ -25,6 +25,15 @@ def ctx():
 
 
 DEV = "cuda"
+PATHS = {"tc": 1, "gemv": 1 << 40}      # SPH_OPT_TC_MIN_ROWS per kernel path
+
+
+@pytest.fixture(params=sorted(PATHS))
+def path_ctx(request, ctx):
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, PATHS[request.param])
+    yield ctx
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
 
 
 def small(**kw):
@@ -54,25 +63,26 @@ CLOUD_CASES = [
 
 
 @pytest.mark.parametrize("name,kw", CLOUD_CASES, ids=[c[0] for c in CLOUD_CASES])
-def test_cloud_parity(ctx, name, kw):
+def test_cloud_parity(path_ctx, name, kw):
     w = small(**kw)
-    check_cloud(ctx, w)
+    check_cloud(path_ctx, w)
 
 
-@pytest.mark.parametrize("rows", [1, 8, 40])
-def test_cloud_bf16_activation_mode(ctx, rows):
+@pytest.mark.parametrize("rows", [1, 8, 40, 300])
+def test_cloud_bf16_activation_mode(path_ctx, rows):
     w = small(V=3000, d=776, d_l=8, rows=rows, n_keep=1200)
-    check_cloud(ctx, w, act_mode="bf16")
+    check_cloud(path_ctx, w, act_mode="bf16")
 
 
-def test_cloud_clipping_bites(ctx):
+def test_cloud_clipping_bites(path_ctx):
     w = small(V=2000, d=1032, d_l=8, rows=6, n_keep=900, clip=0.5)
-    codes, scale, part = check_cloud(ctx, w)
+    codes, scale, part = check_cloud(path_ctx, w)
     assert (np_(part).__abs__() > 0.5).any()          # clip was exercised
     assert np.allclose(np_(scale), np.float32(0.5 / 127))
 
 
-def test_cloud_zero_row_and_edge_ids(ctx):
+def test_cloud_zero_row_and_edge_ids(path_ctx):
+    ctx = path_ctx
     w = small(V=1000, d=264, d_l=8, rows=5, n_keep=300)
     w.h[2].zero_()
     ids = w.keep_ids.clone()
@@ -83,7 +93,8 @@ def test_cloud_zero_row_and_edge_ids(ctx):
     assert np_(scale)[2] == 0 and not np_(codes)[2].any()
 
 
-def test_cloud_odd_hidden_width_and_strides(ctx):
+def test_cloud_odd_hidden_width_and_strides(path_ctx):
+    ctx = path_ctx
     # d_h = 37 (not a multiple of anything) inside a padded weight stride
     base = small(V=900, d=45, d_l=8, rows=7, n_keep=350)
     Wpad = torch.zeros(base.V, 40, dtype=torch.bfloat16, device=DEV)
@@ -106,7 +117,8 @@ ENDPOINT_CASES = [
 
 
 @pytest.mark.parametrize("name,kw", ENDPOINT_CASES, ids=[c[0] for c in ENDPOINT_CASES])
-def test_endpoint_parity(ctx, name, kw):
+def test_endpoint_parity(path_ctx, name, kw):
+    ctx = path_ctx
     w = small(**kw)
     ref = oracle_cloud(w)
     codes = torch.from_numpy(ref["codes"])
