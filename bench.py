@@ -289,12 +289,16 @@ def run_ours(args):
     n_acc = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
     nxt = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
 
-    def step(i, h=None):
+    def step(i, h=None, events=None):
         c = i % ncopy
         hh = hs[c] if h is None else h
+        if events is not None:
+            events[0].record()
         ctx.partial_logits(hh[:, w.d_l:], Whs[c], keep_ids=w.keep_ids, clip=w.clip,
                            w_row_scale=w.w_scale, bias=w.bias, codes=codes,
                            row_scale=scale)
+        if events is not None:
+            events[1].record()
         ctx.fuse_sample(codes, scale, hh[:, :w.d_l], Wls[c], keep_ids=w.keep_ids,
                         temperature=w.tau, seed=w.seed, offset=i, tokens=tokens,
                         fused_logits_out=z)
@@ -306,6 +310,36 @@ def run_ours(args):
     for i in range(args.warmup):
         step(i)
     ctx.sync()
+
+    # ---- the timed loop is a CUDA graph: gsteps steps cycling the weight
+    # copies, the cloud call of each bracketed by event-record nodes
+    gsteps = ncopy * max(1, math.ceil(16 / ncopy))
+    try:
+        evs = [(torch.cuda.Event(enable_timing=True, external=True),
+                torch.cuda.Event(enable_timing=True, external=True))
+               for _ in range(gsteps)]
+    except TypeError:                       # torch without external events
+        evs = None
+
+    def capture(n_steps, with_events):
+        graph = torch.cuda.CUDAGraph()
+        cs = torch.cuda.Stream(device=dev)
+        cs.wait_stream(torch.cuda.current_stream(dev))
+        with torch.cuda.graph(graph, stream=cs):
+            for i in range(n_steps):
+                step(i, events=evs[i] if (with_events and evs) else None)
+        return graph
+
+    ctx.profile_enable(True)
+    g_main = capture(gsteps, True)
+    launches_per_step = ctx.profile_read()["launches"] / gsteps
+    ctx.profile_enable(False)
+    rem = args.steps % gsteps
+    g_rem = capture(rem, False) if rem else None
+    reps = args.steps // gsteps
+    for _ in range(2):                      # warm the graphs
+        g_main.replay()
+    torch.cuda.synchronize(dev)
 
     stream = torch.cuda.current_stream(dev)
     gpu_uuid = None
@@ -322,16 +356,15 @@ def run_ours(args):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    ctx.profile_enable(True)
     t_wall0 = time.time()
     ev0.record(stream)
-    for i in range(args.steps):
-        step(i)
+    for _ in range(reps):
+        g_main.replay()
+    if g_rem is not None:
+        g_rem.replay()
     ev1.record(stream)
     torch.cuda.synchronize(dev)
     t_wall1 = time.time()
-    prof = ctx.profile_read()
-    ctx.profile_enable(False)
     if world > 1:
         dist.barrier()
     ms = ev0.elapsed_time(ev1)
@@ -344,6 +377,37 @@ def run_ours(args):
         time.sleep(0.2)
         sampler.stop()
         clocks = sampler.summary(t_wall0, t_wall1)
+    # duration of the cloud call: its event pairs in the last replay of the
+    # timed loop (or, without external events, a graph of cloud calls alone)
+    if evs is not None and reps > 0:
+        cloud_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+        cloud_src = f"event nodes around the {gsteps} cloud calls of the last timed graph replay"
+    else:
+        gc = torch.cuda.CUDAGraph()
+        cs = torch.cuda.Stream(device=dev)
+        cs.wait_stream(torch.cuda.current_stream(dev))
+        with torch.cuda.graph(gc, stream=cs):
+            for i in range(gsteps):
+                c = i % ncopy
+                ctx.partial_logits(hs[c][:, w.d_l:], Whs[c], keep_ids=w.keep_ids,
+                                   clip=w.clip, w_row_scale=w.w_scale, bias=w.bias,
+                                   codes=codes, row_scale=scale)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        gc.replay()
+        a.record(stream)
+        for _ in range(10):
+            gc.replay()
+        b.record(stream)
+        torch.cuda.synchronize(dev)
+        cloud_ms = a.elapsed_time(b) / (10 * gsteps)
+        cloud_src = "graph of cloud calls replayed alone"
+    ctx.profile_enable(True)                 # per-class split, direct launches
+    for i in range(min(50, args.steps)):
+        step(i)
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+    nprof = max(1, min(50, args.steps))
 
     # ---- end to end: host buffers in, tokens out, every step -------------
     e2e_steps = min(args.e2e_steps, args.steps)
@@ -377,13 +441,14 @@ def run_ours(args):
 
     peaks, peaks_src = load_peaks()
     value = R * world * args.steps / (ms / 1e3)
-    # dominant unit: the cloud call (gathered contraction + quantization)
-    cloud_ms = (prof["ms"]["cloud_gemm"] + prof["ms"]["quantize"]) / max(1, prof["calls"]["cloud_gemm"])
+    # dominant unit: the cloud call (operand split + gathered contraction +
+    # quantization), timed inside the timed graph
     alg_bytes = wl.algorithmic_bytes_cloud(R, n, w.d_h, wb, fp8_scales=w.w_dtype == "fp8")
     alg_flops = wl.algorithmic_flops(R, n, w.d_h)
     ai = alg_flops / alg_bytes
     ridge = peaks["bf16_tflops_sustained"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
-    files = ["paper_2607_13093_gb300/csrc/k_gemv.cu", "paper_2607_13093_gb300/csrc/k_finish.cu"]
+    files = ["paper_2607_13093_gb300/csrc/k_tc.cu", "paper_2607_13093_gb300/csrc/k_gemv.cu",
+             "paper_2607_13093_gb300/csrc/k_finish.cu"]
     if ai < ridge:
         achieved = alg_bytes / (cloud_ms / 1e3) / 1e9
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
@@ -396,9 +461,9 @@ def run_ours(args):
     roof.update({"traffic": traffic_for(f"cloud_{args.workload}", files),
                  "kernel": "cloud call: gathered partial logits + int8 quantization",
                  "algorithmic_bytes": alg_bytes, "algorithmic_flops": alg_flops,
-                 "avg_launch_ms": round(cloud_ms, 5),
+                 "avg_launch_ms": round(cloud_ms, 5), "timing": cloud_src,
                  "peak_source": f"{peaks_src} (MEASURED_PEAKS.json)" if peaks_src == "measured" else "fallback"})
-    steps_ms = {k: round(v / max(1, args.steps), 5) for k, v in prof["ms"].items() if v}
+    steps_ms = {k: round(v / nprof, 5) for k, v in prof["ms"].items() if v}
     out = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
@@ -413,11 +478,14 @@ def run_ours(args):
                           f"{l2 / 1e6:.0f} MB"),
                    "parallelism": f"replicas x{world} (independent sessions per GPU)"},
         "breakdown_ms_per_step": steps_ms,
+        "breakdown_note": "per kernel class, direct (non-graph) launches with tracing events",
         "roofline": roof,
-        "gpu_launches": prof["launches"],
+        "gpu_launches": int(round(launches_per_step * args.steps)),
         "e2e": {"value": round(R * world * e2e_steps / e2e_s, 1), "unit": UNIT,
                 "h2d_bytes_per_step": R * w.d * 4, "d2h_bytes_per_step": R * 4,
-                "note": "pinned host h -> device, cloud + endpoint calls, tokens -> host, sync per step"},
+                "note": ("pinned host h -> device, direct C-ABI calls (no graph), "
+                         "tokens -> host, sync per step")},
+        "timed_loop": f"CUDA graph of {gsteps} steps replayed {reps}x (+{rem} steps)",
         "clocks": clocks,
     }
     if world == 1 and not args.no_cpu_baseline:

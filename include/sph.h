@@ -100,12 +100,21 @@ typedef enum sph_option {
                                kernels replace the CUDA-core GEMV (default 4;
                                1 forces tensor cores, a huge value forces the
                                GEMV; fp8 weights always use the GEMV path)    */
-  SPH_OPT_SPIN_LIMIT = 1    /* clock cycles a device-side wait may spin before
+  SPH_OPT_SPIN_LIMIT = 1,   /* clock cycles a device-side wait may spin before
                                it gives up and the call reports
                                SPH_ERR_TIMEOUT (default 2^34, >= 1)           */
+  SPH_OPT_TC_SCHEDULE = 2,  /* tensor-core work split: 0 automatic (default),
+                               1 whole vocabulary tiles per CTA, 2 contiguous
+                               k-block ranges (stream-K)                      */
+  SPH_OPT_TC_STAGES = 3,    /* tensor-core pipeline depth: 0 automatic
+                               (default), else at most this many stages (>= 2) */
+  SPH_OPT_TC_BLOCK_K = 4    /* hidden-dimension elements each pipeline stage
+                               reads per weight row: 64, 128, 256, or 0 for
+                               automatic (default)                           */
 } sph_option;
 
-/* Set a tunable (SPH_ERR_INVALID_ARG for an unknown option or a value < 1). */
+/* Set a tunable (SPH_ERR_INVALID_ARG for an unknown option or a value out of
+ * range). */
 sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value);
 
 /* Optional device allocation helpers for callers without their own
@@ -134,7 +143,9 @@ typedef struct sph_profile {
 } sph_profile;
 
 /* Start (on != 0; resets the accumulators) or stop tracing.  While on, each
- * kernel group is bracketed by CUDA events on the context's stream. */
+ * kernel group is bracketed by CUDA events on the context's stream; groups
+ * launched while the stream is being captured into a CUDA graph are not
+ * timed (but are counted in `launches`). */
 sph_status sph_profile_enable(sph_ctx* ctx, int on);
 
 /* Wait for the context's stream and return the accumulated figures. */

@@ -1,26 +1,41 @@
 // Tensor-core gathered contraction for the many-row regime (Eq. 11 / Eq. 12
-// over the kept vocabulary ids), tcgen05 + TMEM + TMA on sm_103a.
+// over the kept vocabulary ids), tcgen05 + TMEM on sm_103a.
 //
 // Swap-AB: the MMA's M dimension is a tile of 128 gathered vocabulary rows
-// (operand A, fetched from W by TMA tile::gather4, four rows per
-// instruction), its N dimension is a block of BN hidden-state rows (operand
-// B), and K runs over the hidden dimension in 64-element (128-byte) blocks,
-// 128-byte swizzled.  fp32 hidden states are split on the fly into bf16
-// hi + lo parts (h = hi + lo + O(2^-18 |h|)); both parts multiply the same
-// W tile into one fp32 TMEM accumulator, so W is read once and the result
-// keeps fp32 accuracy.  In bf16-activation mode only the hi part is used.
+// (operand A), its N dimension a block of BN hidden-state rows (operand B),
+// and K runs over the hidden dimension in 64-element (128-byte) blocks laid
+// out with the 128-byte swizzle.  fp32 hidden states are split beforehand
+// into bf16 hi + lo planes (h = hi + lo + O(2^-18 |h|)); both parts multiply
+// the same W tile into one fp32 TMEM accumulator, so W is read once and the
+// result keeps fp32 accuracy.  In bf16-activation mode only hi is used.
 //
-// Work is split stream-K style: the (row block, vocabulary tile, k-block)
-// iterations are cut into one contiguous range per CTA (one persistent CTA
-// per SM).  A tile whose k-range spans several CTAs is finished by the last
-// CTA to arrive: every contributor stores its fp32 partial tile, counts in,
-// and the last one adds the partials in a fixed order (deterministic) and
-// runs the epilogue.  Nothing waits on another CTA.
+// Operand A comes from W by TMA 2-D tile copies, one per 64-column atom:
+//   full vocabulary : one box of 128 rows per atom;
+//   kept-id subset  : the tile's 128 kept ids are cut into runs of
+//                     consecutive vocabulary ids and every run into boxes of
+//                     1, 2, 4, ..., 128 rows (one tensor map per box height),
+//                     each written at its row of the tile; language subsets
+//                     are mostly long runs, so a tile takes a few boxes, and
+//                     isolated ids still work as 1-row boxes.
+// Operand B (the h planes, L2-resident) always comes by TMA.
 //
-// Warp roles (192 threads): warp 0 issues TMA, warp 1 owns TMEM and issues
+// Work split: the (row block, vocabulary tile, k-block) iterations are cut
+// into one contiguous range per persistent CTA (one CTA per SM).  When K is
+// short, ranges cover whole tiles; otherwise they are split stream-K style
+// and a tile whose k-range spans several CTAs is finished by the last CTA to
+// arrive: contributors store fp32 partials, count in, and the last one adds
+// them in CTA order (deterministic).  No CTA ever waits on another.
+//
+// Warp roles: warp 0 issues the TMA copies, warp 1 owns TMEM and issues
 // tcgen05.mma (one thread), warps 2-5 drain the double-buffered accumulator
 // (tcgen05.ld) and run the fused epilogue.  Every wait is bounded; a wait
-// that gives up sets the context's error word and the CTA winds down.
+// that gives up sets the context's error word and the CTA winds down after
+// its copies and MMAs have landed.
+//
+// Epilogues: cloud = + bias, optional unclipped store, clip, store, row |max|
+// (atomicMax); endpoint = + code * row_scale (Eq. 13), store z, and the
+// softmax statistics (max, sum of exp((z - max)/tau)) of every 32-id segment
+// of every row, which the sampler uses instead of re-reading the row.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -33,18 +48,28 @@
 namespace sph {
 namespace {
 
-constexpr int kThreads = 192;
 constexpr int kTileM = 128;          // vocabulary rows per tile (MMA M)
-constexpr int kBlockK = 64;          // bf16 elements per 128-byte row slice
-constexpr int kATileBytes = kTileM * kBlockK * 2;
+constexpr int kAtomK = 64;           // bf16 elements per 128-byte swizzle atom
+constexpr int kAtomBytes = kTileM * kAtomK * 2;   // one A atom: 128 rows x 128 B
 constexpr int kMaxBN = 256;
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
 
+constexpr int kThreads = 192;
+constexpr int kBoxHeights = 8;       // row boxes of 1, 2, 4, ..., 128 rows
+
+// W tensor maps: box height 2^i rows for map i (64 columns each).
+struct WMaps {
+  CUtensorMap m[kBoxHeights];
+};
+
 struct TcParams {
-  int R, n, K, KB, NT, RB, BN, Rp, stages;
+  int R, n, K, KB, NT, RB, BN, Rp, stages, whole_tiles;
+  int na;                      // swizzle atoms per k-block (k-block = 64 * na)
   long long T;                 // total iterations RB * NT * KB
   const int32_t* ids;          // gather path: sorted ids
+  const int2* chunks;          // gather path: [NT][128] (first id, row | lg << 8)
+  const int2* chunk_count;     // gather path: [NT] (boxes, rows copied)
   int epilogue;
   const float* bias;
   float clip;
@@ -53,6 +78,8 @@ struct TcParams {
   unsigned* rowmax;
   const int8_t* codes;
   const float* row_scale;
+  float inv_tau;
+  float2* seg_stats;           // endpoint: [R][NT*4] (max, sum exp)
   float* P;                    // split-tile partials [2 * grid][BN][128]
   int* counters;               // [tiles][4 quadrants], zero between calls
   unsigned* status;
@@ -60,7 +87,13 @@ struct TcParams {
 };
 
 __device__ __forceinline__ long long cta_of(long long i, long long T, int G) {
-  return ((i + 1) * G + T - 1) / T - 1;    // owner of iteration i
+  return ((i + 1) * G + T - 1) / T - 1;    // owner of iteration i (split mode)
+}
+
+// First iteration of CTA c.
+__device__ __forceinline__ long long range_start(const TcParams& p, long long c, int G) {
+  if (p.whole_tiles) return (c * (long long)(p.RB * p.NT) / G) * p.KB;
+  return c * p.T / G;
 }
 
 // Walks the (tile, k-block range) segments of one CTA's iteration range.
@@ -81,14 +114,13 @@ struct Segments {
 template <int EPI>
 __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)[16],
                                              int row0, int j, bool vj, int id,
-                                             int lane) {
+                                             int lane, int seg) {
+  if constexpr (EPI == EPI_CLOUD) {
 #pragma unroll
-  for (int q = 0; q < 16; ++q) {
-    const int r = row0 + q;
-    const bool ok = vj && r < p.R;
-    if constexpr (EPI == EPI_CLOUD) {
+    for (int q = 0; q < 16; ++q) {
+      const int r = row0 + q;
       float m = 0.f;
-      if (ok) {
+      if (vj && r < p.R) {
         float y = v[q];
         if (p.bias) y += p.bias[id];
         const int64_t o = (int64_t)r * p.n + j;
@@ -99,24 +131,48 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
       }
       m = warp_max(m);
       if (lane == 0 && r < p.R && m > 0.f) atomicMax(&p.rowmax[r], __float_as_uint(m));
-    } else {
-      if (ok) {
-        const int64_t o = (int64_t)r * p.n + j;
-        p.Y[o] = v[q] + (float)p.codes[o] * p.row_scale[r];
-      }
+    }
+  } else {
+    // all payload loads first, then the stores (the stores could alias the
+    // loads as far as the compiler knows, which would serialise them)
+    float z[16];
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const int r = row0 + q;
+      z[q] = (vj && r < p.R)
+                 ? v[q] + (float)__ldg(p.codes + (int64_t)r * p.n + j) * __ldg(p.row_scale + r)
+                 : -INFINITY;
+    }
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const int r = row0 + q;
+      if (vj && r < p.R) p.Y[(int64_t)r * p.n + j] = z[q];
+    }
+    // softmax statistics of this 32-id segment for each row
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const int r = row0 + q;
+      const float m = warp_max(z[q]);
+      const float e = vj && r < p.R ? expf((z[q] - m) * p.inv_tau) : 0.f;
+      const float s = warp_sum(e);
+      if (lane == 0 && r < p.R)
+        p.seg_stats[(int64_t)r * (p.NT * 4) + seg] = make_float2(m, s);
     }
   }
 }
 
 template <int HILO, bool GATHER, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
-tc_kernel(const __grid_constant__ CUtensorMap tmW,
+tc_kernel(const __grid_constant__ WMaps wm,
           const __grid_constant__ CUtensorMap tmH, const TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* base = smem_raw + (((raw_addr + 1023) & ~1023u) - raw_addr);
   const int BN = p.BN;
-  const int stage_bytes = kATileBytes + HILO * BN * 128;
+  const int NA = p.na;
+  const int a_bytes = NA * kAtomBytes;
+  const int b_bytes = HILO * NA * BN * 128;
+  const int stage_bytes = a_bytes + b_bytes;
   const int S = p.stages;
   uint64_t* full = reinterpret_cast<uint64_t*>(base + (size_t)S * stage_bytes);
   uint64_t* empty = full + S;
@@ -132,7 +188,7 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      ptx::mbar_init(&full[s], 1);
+      ptx::mbar_init(&full[s], 1);               // the TMA thread's expect_tx
       ptx::mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -143,9 +199,9 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
     *s_abort = 0;
     ptx::fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) {
-    ptx::prefetch_tmap(&tmW);
-    ptx::prefetch_tmap(&tmH);
+  if (warp == 0 && lane < kBoxHeights) {
+    if (GATHER || lane == kBoxHeights - 1) ptx::prefetch_tmap(&wm.m[lane]);
+    if (lane == 0) ptx::prefetch_tmap(&tmH);
   }
   if (warp == 1) ptx::tmem_alloc(tmem_holder, ncols);
   ptx::tc_fence_before();
@@ -154,8 +210,8 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
   const uint32_t tmem_base = *tmem_holder;
 
   const int G = gridDim.x;
-  const long long it0 = (long long)blockIdx.x * p.T / G;
-  const long long it1 = (long long)(blockIdx.x + 1) * p.T / G;
+  const long long it0 = range_start(p, blockIdx.x, G);
+  const long long it1 = range_start(p, blockIdx.x + 1, G);
   const long long limit = p.spin_limit;
 
   auto give_up = [&]() {
@@ -164,24 +220,29 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
   };
 
   if (warp == 0) {
-    // ------------------------------------------------------------ producer
+    // ------------------------------------------------------- TMA producer
+    // lane 0 owns the ring; on the subset path every lane issues the boxes
+    // of up to four of the tile's row chunks
     Segments sg{it0, it1, p.KB};
     int stage = 0;
     uint32_t phase = 0;
     int tile, kb0, kb1;
-    const uint32_t tx = (uint32_t)stage_bytes;
     bool stop = false;
     long long issued = 0;
     while (!stop && sg.next(tile, kb0, kb1)) {
       const int rb = tile / p.NT, t = tile - rb * p.NT;
-      const int j0 = t * kTileM;
-      int y[4] = {0, 0, 0, 0};
+      int2 ch[4];
+      int nmine = 0;
+      uint32_t tx = (uint32_t)stage_bytes;
       if constexpr (GATHER) {
+        const int2 cc = p.chunk_count[t];        // (boxes, rows copied)
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          const int j = min(j0 + 4 * lane + q, p.n - 1);
-          y[q] = p.ids[j];
+          const int ci = lane + 32 * q;
+          ch[q] = ci < cc.x ? p.chunks[(int64_t)t * kTileM + ci] : make_int2(0, 0);
+          if (ci < cc.x) nmine = q + 1;
         }
+        tx = (uint32_t)(cc.y * 128 * NA + b_bytes);
       }
       for (int kb = kb0; kb < kb1; ++kb) {
         int ok = 1;
@@ -195,17 +256,27 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
         if (lane == 0) ptx::mbar_expect_tx(&full[stage], tx);
         __syncwarp();
         uint8_t* A = base + (size_t)stage * stage_bytes;
-        uint8_t* B = A + kATileBytes;
-        if constexpr (GATHER) {
-          ptx::tma_gather4(A + 512 * lane, &tmW, kb * kBlockK, y[0], y[1], y[2], y[3],
-                           &full[stage]);
-        } else {
-          if (lane == 0) ptx::tma_load_2d(A, &tmW, kb * kBlockK, j0, &full[stage]);
-        }
-        if (lane == 0) {
-          ptx::tma_load_2d(B, &tmH, kb * kBlockK, rb * BN, &full[stage]);
-          if (HILO == 2)
-            ptx::tma_load_2d(B + BN * 128, &tmH, kb * kBlockK, p.Rp + rb * BN, &full[stage]);
+        uint8_t* B = A + a_bytes;
+        for (int a = 0; a < NA; ++a) {
+          const int x = (kb * NA + a) * kAtomK;
+          if constexpr (GATHER) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              if (q < nmine) {
+                const int row = ch[q].y & 0xFF, lg = ch[q].y >> 8;
+                ptx::tma_load_2d(A + a * kAtomBytes + row * 128, &wm.m[lg], x, ch[q].x,
+                                 &full[stage]);
+              }
+            }
+          } else {
+            if (lane == 0)
+              ptx::tma_load_2d(A + a * kAtomBytes, &wm.m[kBoxHeights - 1], x, t * kTileM,
+                               &full[stage]);
+          }
+          if (lane == 0)
+            for (int h = 0; h < HILO; ++h)
+              ptx::tma_load_2d(B + (h * NA + a) * BN * 128, &tmH, x, h * p.Rp + rb * BN,
+                               &full[stage]);
         }
         ++issued;
         if (++stage == S) { stage = 0; phase ^= 1; }
@@ -242,15 +313,17 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
             break;
           }
           ptx::tc_fence_after();
-          const uint32_t a = ptx::smem_u32(base + (size_t)stage * stage_bytes);
-          const uint32_t b = a + kATileBytes;
+          const uint32_t a0 = ptx::smem_u32(base + (size_t)stage * stage_bytes);
+          const uint32_t b0 = a0 + a_bytes;
+          for (int at = 0; at < NA; ++at) {
 #pragma unroll
-          for (int h = 0; h < HILO; ++h) {
+            for (int h = 0; h < HILO; ++h) {
 #pragma unroll
-            for (int kk = 0; kk < kBlockK / 16; ++kk) {
-              ptx::umma_bf16(d, ptx::sdesc_k128(a + kk * 32),
-                             ptx::sdesc_k128(b + h * BN * 128 + kk * 32), idesc,
-                             (kb != kb0 || h != 0 || kk != 0) ? 1u : 0u);
+              for (int kk = 0; kk < kAtomK / 16; ++kk) {
+                ptx::umma_bf16(d, ptx::sdesc_k128(a0 + at * kAtomBytes + kk * 32),
+                               ptx::sdesc_k128(b0 + (h * NA + at) * BN * 128 + kk * 32),
+                               idesc, (kb != kb0 || at != 0 || h != 0 || kk != 0) ? 1u : 0u);
+              }
             }
           }
           ptx::umma_commit(&empty[stage]);
@@ -262,7 +335,7 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
       }
       // all issued MMAs complete before TMEM is released
       ptx::umma_commit(drain);
-      ptx::mbar_wait(drain, 0, limit);
+      ptx::mbar_wait(drain, 0, kDrainLimit);
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -286,6 +359,7 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
       const int j = t * kTileM + i;
       const bool vj = j < p.n;
       const int id = vj ? (GATHER ? p.ids[j] : j) : 0;
+      const int seg = t * 4 + quad;
       const bool whole = kb0 == 0 && kb1 == p.KB;
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
       // a CTA's split tiles can only be its first and its last segment:
@@ -295,7 +369,7 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
         float v[16];
         ptx::tmem_ld16(taddr + ch * 16, v);
         if (whole) {
-          finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane);
+          finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg);
         } else {
 #pragma unroll
           for (int q = 0; q < 16; ++q) Pt[(size_t)(ch * 16 + q) * kTileM + i] = v[q];
@@ -327,7 +401,7 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
 #pragma unroll
               for (int q = 0; q < 16; ++q) v[q] += __ldcg(Ps + (size_t)q * kTileM);
             }
-            finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane);
+            finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg);
           }
           if (lane == 0) p.counters[tile * 4 + quad] = 0;
         }
@@ -345,10 +419,77 @@ tc_kernel(const __grid_constant__ CUtensorMap tmW,
 // ---------------------------------------------------------------------------
 // operand preparation: fp32 h -> bf16 hi (and lo) planes, zero padded
 // ---------------------------------------------------------------------------
+// ... and, on the subset path, the row boxes of every vocabulary tile (one
+// warp per tile): the tile's kept ids are cut into runs of consecutive ids,
+// and a run of length L is covered by one box of 2^k rows if L = 2^k, else by
+// two boxes of 2^k rows (k = floor(log2 L)) placed at its start and at its
+// end, which overlap on rows they both copy identically.  Each box is stored
+// as (first id, tile row | lg << 8); per tile (box count, rows copied).
 __global__ void split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R,
                                int K, int Rp, int Kp, int hilo,
                                __nv_bfloat16* __restrict__ Hs,
-                               int* __restrict__ counters, int ncounters) {
+                               int* __restrict__ counters, int ncounters,
+                               const int32_t* __restrict__ ids, int n, int NT,
+                               int2* __restrict__ chunks, int2* __restrict__ chunk_count) {
+  if (ids) {
+    const int lane = threadIdx.x & 31;
+    const int nwarps = (gridDim.x * blockDim.x) >> 5;
+    for (int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; t < NT; t += nwarps) {
+      const int j0 = t * kTileM;
+      const int rows = min(kTileM, n - j0);
+      int idr[4];
+      unsigned smask[4];
+      int prev_last = 0;
+#pragma unroll
+      for (int g = 0; g < 4; ++g) {
+        const int r = 32 * g + lane;
+        idr[g] = r < rows ? ids[j0 + r] : 0;
+        int prev = __shfl_up_sync(0xFFFFFFFFu, idr[g], 1);
+        if (lane == 0) prev = prev_last;
+        const bool start = r < rows && (r == 0 || idr[g] != prev + 1);
+        smask[g] = __ballot_sync(0xFFFFFFFFu, start);
+        prev_last = __shfl_sync(0xFFFFFFFFu, idr[g], 31);
+      }
+      int base = 0, covered = 0;
+#pragma unroll
+      for (int g = 0; g < 4; ++g) {
+        const int r = 32 * g + lane;
+        const bool start = (smask[g] >> lane) & 1u;
+        int nbox = 0, len = 0, lg = 0;
+        if (start) {
+          // the next run start above r, or the end of the tile
+          int nxt = rows;
+          const unsigned above = lane == 31 ? 0u : (smask[g] >> (lane + 1)) << (lane + 1);
+          if (above) {
+            nxt = 32 * g + __ffs(above) - 1;
+          } else {
+            for (int g2 = g + 1; g2 < 4; ++g2)
+              if (smask[g2]) { nxt = 32 * g2 + __ffs(smask[g2]) - 1; break; }
+          }
+          len = nxt - r;
+          lg = 31 - __clz(len);
+          nbox = (len == (1 << lg)) ? 1 : 2;
+        }
+        int incl = nbox;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+          if (lane >= o) incl += v;
+        }
+        const int off = base + incl - nbox;
+        if (nbox >= 1) chunks[(int64_t)t * kTileM + off] = make_int2(idr[g], r | (lg << 8));
+        if (nbox == 2)
+          chunks[(int64_t)t * kTileM + off + 1] =
+              make_int2(idr[g] + len - (1 << lg), (r + len - (1 << lg)) | (lg << 8));
+        int rows_here = nbox * (nbox ? (1 << lg) : 0);
+#pragma unroll
+        for (int o = 16; o; o >>= 1) rows_here += __shfl_xor_sync(0xFFFFFFFFu, rows_here, o);
+        covered += rows_here;
+        base += __shfl_sync(0xFFFFFFFFu, incl, 31);
+      }
+      if (lane == 0) chunk_count[t] = make_int2(base, covered);
+    }
+  }
   const int64_t total = (int64_t)Rp * Kp;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
@@ -361,6 +502,77 @@ __global__ void split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R,
   for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < ncounters;
        t += gridDim.x * blockDim.x)
     counters[t] = 0;
+}
+
+// ---------------------------------------------------------------------------
+// sampling from the segment statistics: one warp per row
+// ---------------------------------------------------------------------------
+__global__ void sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
+                                  const float2* __restrict__ stats, int nseg,
+                                  const int32_t* __restrict__ ids, float inv_tau,
+                                  uint64_t seed, uint64_t offset,
+                                  int32_t* __restrict__ tokens) {
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (r >= rows) return;
+  const float2* st = stats + (int64_t)r * nseg;
+  float M = -INFINITY;
+  for (int s = lane; s < nseg; s += 32) M = fmaxf(M, st[s].x);
+  M = warp_max(M);
+  // segment weights in ascending order: lane owns segments [s0, s1)
+  const int per = (nseg + 31) / 32;
+  const int s0 = min(nseg, lane * per), s1 = min(nseg, s0 + per);
+  float local = 0.f;
+  for (int s = s0; s < s1; ++s) {
+    const float2 v = st[s];
+    local += v.y > 0.f ? v.y * expf((v.x - M) * inv_tau) : 0.f;
+  }
+  float incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  const float excl = incl - local;
+  const float total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+  const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
+  const float target = u * total;
+  const unsigned hit = __ballot_sync(0xFFFFFFFFu, local > 0.f && target >= excl && target < incl);
+  const unsigned nzl = __ballot_sync(0xFFFFFFFFu, local > 0.f);
+  const int owner = hit ? __ffs(hit) - 1 : (nzl ? 31 - __clz(nzl) : 0);
+  int sstar = -1;
+  float before = 0.f;
+  if (lane == owner) {
+    float run = excl, before_last = excl;
+    int last_nz = -1;
+    for (int s = s0; s < s1; ++s) {
+      const float2 v = st[s];
+      const float w = v.y > 0.f ? v.y * expf((v.x - M) * inv_tau) : 0.f;
+      if (w > 0.f) { last_nz = s; before_last = run; }
+      if (w > 0.f && target < run + w) { sstar = s; before = run; break; }
+      run += w;
+    }
+    if (sstar < 0) { sstar = last_nz >= 0 ? last_nz : s0; before = before_last; }
+  }
+  sstar = __shfl_sync(0xFFFFFFFFu, sstar, owner);
+  before = __shfl_sync(0xFFFFFFFFu, before, owner);
+  // inside the 32-id segment: one id per lane
+  const int j = sstar * 32 + lane;
+  const float w = j < n ? expf((Z[(int64_t)r * n + j] - M) * inv_tau) : 0.f;
+  float winc = w;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float t = __shfl_up_sync(0xFFFFFFFFu, winc, o);
+    if (lane >= o) winc += t;
+  }
+  const float t2 = target - before;
+  const unsigned h2 = __ballot_sync(0xFFFFFFFFu, w > 0.f && t2 < winc);
+  const unsigned nz2 = __ballot_sync(0xFFFFFFFFu, w > 0.f);
+  const int l2 = h2 ? __ffs(h2) - 1 : (nz2 ? 31 - __clz(nz2) : 0);
+  if (lane == l2) {
+    const int jj = min(sstar * 32 + l2, n - 1);
+    tokens[r] = ids ? ids[jj] : jj;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -405,7 +617,8 @@ size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
 }  // namespace
 
-TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count) {
+TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
+               int schedule, int max_stages, int block_k, int gather) {
   TcPlan pl{};
   pl.hilo = act_bf16 ? 1 : 2;
   if (rows <= kMaxBN) {
@@ -416,28 +629,47 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count) {
     pl.BN = ((rows + pl.RB - 1) / pl.RB + 15) / 16 * 16;
   }
   pl.Rp = pl.RB * pl.BN;
-  pl.KB = (K + kBlockK - 1) / kBlockK;
-  pl.Kp = pl.KB * kBlockK;
+  // k-block width: as asked (automatic: 128), narrowed until the shared
+  // memory holds at least min_stages pipeline stages
+  pl.na = block_k == 64 ? 1 : (block_k == 256 ? 4 : 2);
+  const int min_stages = block_k ? 2 : 4;
+  while (pl.na > 1 &&
+         (int)((kSmemBudget - 2048) / (pl.na * (kAtomBytes + pl.hilo * pl.BN * 128))) <
+             min_stages)
+    pl.na >>= 1;
+  const int bk = pl.na * kAtomK;
+  pl.KB = (K + bk - 1) / bk;
+  pl.Kp = pl.KB * bk;
   pl.NT = (n + kTileM - 1) / kTileM;
-  pl.T = (long long)pl.RB * pl.NT * pl.KB;
-  pl.G = (int)(pl.T < sm_count ? pl.T : sm_count);
-  const int stage_bytes = kATileBytes + pl.hilo * pl.BN * 128;
+  const int tiles = pl.RB * pl.NT;
+  pl.T = (long long)tiles * pl.KB;
+  // whole tiles per CTA unless that leaves the grid clearly unbalanced
+  const int g_whole = tiles < sm_count ? tiles : sm_count;
+  const long long whole_span = (long long)((tiles + g_whole - 1) / g_whole) * pl.KB;
+  const double split_span = (double)pl.T / (pl.T < sm_count ? pl.T : sm_count);
+  pl.whole_tiles = schedule == 1 || (schedule == 0 && whole_span <= 1.1 * split_span + 2.0);
+  pl.G = pl.whole_tiles ? g_whole : (int)(pl.T < sm_count ? pl.T : sm_count);
+  const int stage_bytes = pl.na * (kAtomBytes + pl.hilo * pl.BN * 128);
   pl.stages = (int)((kSmemBudget - 2048) / stage_bytes);
   if (pl.stages > 8) pl.stages = 8;
-  const int tiles = pl.RB * pl.NT;
+  if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
   pl.hs_bytes = align256((size_t)pl.hilo * pl.Rp * pl.Kp * 2);
   // split tiles exist only when a CTA's range does not cover whole tiles
-  const bool splits = pl.T % pl.G != 0 || (pl.T / pl.G) % pl.KB != 0;
+  const bool splits = !pl.whole_tiles && (pl.T % pl.G != 0 || (pl.T / pl.G) % pl.KB != 0);
   pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * kTileM * 4) : 0;
   pl.cnt_bytes = align256((size_t)tiles * 4 * sizeof(int));
-  pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes;
+  pl.stats_bytes = endpoint ? align256((size_t)rows * pl.NT * 4 * sizeof(float2)) : 0;
+  pl.chunk_bytes = gather ? align256((size_t)pl.NT * kTileM * sizeof(int2)) +
+                                align256((size_t)pl.NT * sizeof(int2))
+                          : 0;
+  pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes + pl.chunk_bytes;
   pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256;
   pl.ok = pl.stages >= 2;
   return pl;
 }
 
 template <int HILO, bool GATHER, int EPI>
-static cudaError_t launch_inst(const CUtensorMap& mw, const CUtensorMap& mh,
+static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
                                const TcParams& prm, const TcPlan& pl,
                                cudaStream_t st) {
   auto kern = tc_kernel<HILO, GATHER, EPI>;
@@ -456,37 +688,58 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   auto* Hs = reinterpret_cast<__nv_bfloat16*>(sc);
   float* P = pl.p_bytes ? reinterpret_cast<float*>(sc + pl.hs_bytes) : nullptr;
   int* counters = reinterpret_cast<int*>(sc + pl.hs_bytes + pl.p_bytes);
+  float2* stats = pl.stats_bytes
+                      ? reinterpret_cast<float2*>(sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes)
+                      : nullptr;
+  char* chunk_base = sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
+  const bool gather = g.ids != nullptr;
+  int2* chunks = gather ? reinterpret_cast<int2*>(chunk_base) : nullptr;
+  int2* chunk_count = gather ? reinterpret_cast<int2*>(
+                                   chunk_base + align256((size_t)pl.NT * kTileM * sizeof(int2)))
+                             : nullptr;
   const int tiles = pl.RB * pl.NT;
 
   {
     const int64_t total = (int64_t)pl.Rp * pl.Kp;
-    int blocks = (int)((total + 255) / 256);
+    int64_t work = total > (int64_t)pl.NT * 32 ? total : (int64_t)pl.NT * 32;
+    int blocks = (int)((work + 255) / 256);
     if (blocks > 4096) blocks = 4096;
     if (blocks < 1) blocks = 1;
     split_h_kernel<<<blocks, 256, 0, st>>>(g.h, g.ld_h, g.rows, g.K, pl.Rp, pl.Kp,
-                                           pl.hilo, Hs, counters, tiles * 4);
+                                           pl.hilo, Hs, counters, tiles * 4, g.ids, g.n,
+                                           pl.NT, chunks, chunk_count);
     ++launch_count;
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
 
-  alignas(64) CUtensorMap mw, mh;
-  const bool gather = g.ids != nullptr;
-  // W: [V rows, K columns], row stride ld_w; box 64 columns x (1 | 128) rows
-  if (!make_map(&mw, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K, (uint64_t)g.V,
-                (uint64_t)g.ld_w * 2, kBlockK, gather ? 1u : (uint32_t)kTileM))
-    return cudaErrorInvalidValue;
+  WMaps mw;
+  alignas(64) CUtensorMap mh;
+  // W: [V rows, K columns], row stride ld_w; map i copies boxes of 64
+  // columns x 2^i rows (the full-vocabulary path uses only the 128-row map)
+  for (int i = 0; i < kBoxHeights; ++i) {
+    if (!gather && i != kBoxHeights - 1) {
+      mw.m[i] = CUtensorMap{};
+      continue;
+    }
+    if (!make_map(&mw.m[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
+                  (uint64_t)g.V, (uint64_t)g.ld_w * 2, kAtomK, 1u << i))
+      return cudaErrorInvalidValue;
+  }
   if (!make_map(&mh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, Hs, (uint64_t)pl.Kp,
-                (uint64_t)pl.hilo * pl.Rp, (uint64_t)pl.Kp * 2, kBlockK,
+                (uint64_t)pl.hilo * pl.Rp, (uint64_t)pl.Kp * 2, kAtomK,
                 (uint32_t)pl.BN))
     return cudaErrorInvalidValue;
 
   TcParams prm{};
   prm.R = g.rows; prm.n = g.n; prm.K = g.K; prm.KB = pl.KB; prm.NT = pl.NT;
   prm.RB = pl.RB; prm.BN = pl.BN; prm.Rp = pl.Rp; prm.stages = pl.stages;
-  prm.T = pl.T; prm.ids = g.ids; prm.epilogue = g.epilogue; prm.bias = g.bias;
+  prm.whole_tiles = pl.whole_tiles; prm.T = pl.T; prm.na = pl.na;
+  prm.ids = g.ids; prm.chunks = chunks; prm.chunk_count = chunk_count;
+  prm.epilogue = g.epilogue; prm.bias = g.bias;
   prm.clip = g.clip; prm.partial_out = g.partial_out; prm.Y = g.Y;
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
+  prm.inv_tau = g.inv_tau; prm.seg_stats = stats;
   prm.P = P; prm.counters = counters;
   prm.status = g.status; prm.spin_limit = spin_limit;
 
@@ -501,6 +754,21 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                            : launch_inst<1, true, EPI_ENDPOINT>(mw, mh, prm, pl, st);
   return hilo2 ? launch_inst<2, false, EPI_ENDPOINT>(mw, mh, prm, pl, st)
                : launch_inst<1, false, EPI_ENDPOINT>(mw, mh, prm, pl, st);
+}
+
+cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPlan& pl,
+                                     const void* scratch, const int32_t* ids,
+                                     float inv_tau, uint64_t seed, uint64_t offset,
+                                     int32_t* tokens, cudaStream_t st) {
+  const char* sc = static_cast<const char*>(scratch);
+  const float2* stats =
+      reinterpret_cast<const float2*>(sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes);
+  const int warps = 8;
+  const int blocks = (rows + warps - 1) / warps;
+  sample_seg_kernel<<<blocks, warps * 32, 0, st>>>(Z, rows, n, stats, pl.NT * 4, ids,
+                                                   inv_tau, seed, offset, tokens);
+  ++launch_count;
+  return cudaGetLastError();
 }
 
 }  // namespace sph

@@ -30,6 +30,9 @@ struct sph_ctx {
   unsigned* status = nullptr;       // device error word (sph::ERR_* bits)
   int64_t tc_min_rows = 4;          // SPH_OPT_TC_MIN_ROWS
   long long spin_limit = 1ll << 34; // SPH_OPT_SPIN_LIMIT
+  int tc_schedule = 0;              // SPH_OPT_TC_SCHEDULE
+  int tc_stages = 0;                // SPH_OPT_TC_STAGES
+  int tc_block_k = 0;               // SPH_OPT_TC_BLOCK_K
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -119,18 +122,26 @@ bool use_tc(const sph_ctx* ctx, int64_t rows, int w_dtype) {
 }
 
 size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_bf16,
-                int w_dtype) {
+                int w_dtype, int endpoint) {
   if (!use_tc(ctx, rows, w_dtype)) return 0;
-  return sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count).scratch_bytes;
+  size_t b = 0;
+  for (int gather = 0; gather < 2; ++gather) {   // the larger of the two paths
+    const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count,
+                                  endpoint, ctx->tc_schedule, ctx->tc_stages,
+                                  ctx->tc_block_k, gather)
+                         .scratch_bytes;
+    if (x > b) b = x;
+  }
+  return b;
 }
 
 size_t partial_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K,
                              int act_bf16, int w_dtype) {
   return align_up((size_t)rows * n * 4, 256) + align_up((size_t)rows * 4, 256) +
-         tc_bytes(ctx, rows, n, K, act_bf16, w_dtype);
+         tc_bytes(ctx, rows, n, K, act_bf16, w_dtype, 0);
 }
 size_t fuse_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K) {
-  return align_up((size_t)rows * n * 4, 256) + tc_bytes(ctx, rows, n, K, 0, sph::W_BF16);
+  return align_up((size_t)rows * n * 4, 256) + tc_bytes(ctx, rows, n, K, 0, sph::W_BF16, 1);
 }
 
 bool finite_pos(float x) { return std::isfinite(x) && x > 0.f; }
@@ -166,6 +177,10 @@ cudaEvent_t pooled_event(sph_ctx* ctx) {
 template <class F>
 cudaError_t traced(sph_ctx* ctx, int cls, F&& launch) {
   if (!ctx->prof) return launch();
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(ctx->stream, &cap) != cudaSuccess ||
+      cap != cudaStreamCaptureStatusNone)
+    return launch();                 // events are not timed inside a graph
   cudaEvent_t a = pooled_event(ctx), b = pooled_event(ctx);
   if (!a || !b) return launch();
   cudaEventRecord(a, ctx->stream);
@@ -330,10 +345,27 @@ sph_status sph_reserve(sph_ctx* ctx, int64_t max_rows, int64_t max_n_keep,
 
 sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
   if (!ctx) return SPH_ERR_INVALID_ARG;
-  if (value < 1) return fail(ctx, SPH_ERR_INVALID_ARG, "option value must be >= 1");
   switch (option) {
-    case SPH_OPT_TC_MIN_ROWS: ctx->tc_min_rows = value; return SPH_OK;
-    case SPH_OPT_SPIN_LIMIT: ctx->spin_limit = value; return SPH_OK;
+    case SPH_OPT_TC_MIN_ROWS:
+    case SPH_OPT_SPIN_LIMIT:
+      if (value < 1) return fail(ctx, SPH_ERR_INVALID_ARG, "option value must be >= 1");
+      if (option == SPH_OPT_TC_MIN_ROWS) ctx->tc_min_rows = value;
+      else ctx->spin_limit = value;
+      return SPH_OK;
+    case SPH_OPT_TC_SCHEDULE:
+      if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "schedule must be 0, 1 or 2");
+      ctx->tc_schedule = (int)value;
+      return SPH_OK;
+    case SPH_OPT_TC_STAGES:
+      if (value != 0 && (value < 2 || value > 8))
+        return fail(ctx, SPH_ERR_INVALID_ARG, "stages must be 0 or in [2, 8]");
+      ctx->tc_stages = (int)value;
+      return SPH_OK;
+    case SPH_OPT_TC_BLOCK_K:
+      if (value != 0 && value != 64 && value != 128 && value != 256)
+        return fail(ctx, SPH_ERR_INVALID_ARG, "block_k must be 0, 64, 128 or 256");
+      ctx->tc_block_k = (int)value;
+      return SPH_OK;
   }
   return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
 }
@@ -416,7 +448,9 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
   gg.bias = bias; gg.clip = clip; gg.partial_out = partial_out;
   gg.Y = Y; gg.rowmax = rowmax; gg.status = ctx->status;
   if (use_tc(ctx, rows, wdt)) {
-    const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_h, act_bf16, ctx->sm_count);
+    const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_h, act_bf16,
+                                        ctx->sm_count, 0, ctx->tc_schedule, ctx->tc_stages,
+                                        ctx->tc_block_k, keep_ids != nullptr);
     void* tcs = c.take(pl.scratch_bytes);
     st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
@@ -468,17 +502,25 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   gg.ids = keep_ids; gg.n = (int)n_keep;
   gg.epilogue = sph::EPI_ENDPOINT;
   gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale; gg.status = ctx->status;
+  gg.inv_tau = 1.0f / temperature;
   if (use_tc(ctx, rows, sph::W_BF16)) {
-    const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0, ctx->sm_count);
+    const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0,
+                                        ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
+                                        ctx->tc_block_k, keep_ids != nullptr);
     void* tcs = c.take(pl.scratch_bytes);
     st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
                        }), "tensor-core launch");
-  } else {
-    st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
-                         return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
-                       }), "gemv launch");
+    if (st) return st;
+    return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
+                           return sph::launch_sample_from_stats(
+                               Z, (int)rows, (int)n_keep, pl, tcs, keep_ids,
+                               1.0f / temperature, seed, offset, tokens, ctx->stream);
+                         }), "sample launch");
   }
+  st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
+                       return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
+                     }), "gemv launch");
   if (st) return st;
   return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                          return sph::launch_sample(Z, (int)rows, (int)n_keep, keep_ids,

@@ -48,6 +48,7 @@ struct GatherGemm {
   // EPI_ENDPOINT
   const int8_t* codes;     // [rows, n]
   const float* row_scale;  // [rows]
+  float inv_tau;           // 1 / temperature (softmax statistics)
   unsigned* status;        // device error word
 };
 
@@ -58,16 +59,28 @@ int gemv_max_k();
 
 // Tensor-core path (k_tc.cu): sizes, work split and scratch of one call.
 struct TcPlan {
-  int hilo, RB, BN, Rp, KB, Kp, NT, G, stages;
+  int hilo, RB, BN, Rp, KB, Kp, NT, G, stages, whole_tiles, na;
   long long T;
-  size_t hs_bytes, p_bytes, cnt_bytes, scratch_bytes, smem_bytes;
+  size_t hs_bytes, p_bytes, cnt_bytes, stats_bytes, chunk_bytes, scratch_bytes, smem_bytes;
   bool ok;
 };
-TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count);
+// `endpoint` reserves the per-segment softmax statistics; schedule 0/1/2 =
+// automatic / whole tiles / stream-K; max_stages 0 = automatic; block_k =
+// hidden elements per pipeline stage (64, 128 or 256; 0 = automatic);
+// gather = the kept-id subset path (keep_ids given).
+TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
+               int schedule, int max_stages, int block_k, int gather);
 // Launch the operand split and the tcgen05 kernel; `scratch` holds
 // plan.scratch_bytes bytes.  bf16 weights only.
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,
                       long long spin_limit, cudaStream_t st);
+// One inverse-CDF draw per row from the segment statistics that an endpoint
+// launch_tc left in `scratch` (one warp per row).
+cudaError_t launch_sample_from_stats(const float* Z, int rows, int n,
+                                     const TcPlan& plan, const void* scratch,
+                                     const int32_t* ids, float inv_tau,
+                                     uint64_t seed, uint64_t offset,
+                                     int32_t* tokens, cudaStream_t st);
 
 // codes/row_scale from the clipped partials and their row maxima
 cudaError_t launch_quantize(const float* Y, const unsigned* rowmax, int rows,

@@ -197,3 +197,28 @@ def test_full_size_sampled_rows(ctx, name, rows, keep):
     if w.sessions:
         target = wl.make_target_logits(w.rows, w.n_keep, seed=12, device=DEV)
         check_verify(ctx, w, target.cpu())
+
+
+# ---------------------------------------------------------------------------
+# tensor-core kernel variants: pipeline k-block width x work schedule
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("block_k", [64, 128, 256])
+@pytest.mark.parametrize("schedule", [1, 2])
+@pytest.mark.parametrize("keep", [700, 2000])
+def test_tensor_core_variants(ctx, block_k, schedule, keep):
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    ctx.set_option(sph.SPH_OPT_TC_BLOCK_K, block_k)
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, schedule)
+    try:
+        # K = 1000 (not a multiple of any k-block), ragged vocabulary tail
+        w = small(V=2000, d=1072, d_l=72, rows=24, n_keep=keep, seed=91 + block_k)
+        check_cloud(ctx, w)
+        ref = oracle_cloud(w)
+        check_endpoint(ctx, w, torch.from_numpy(ref["codes"]),
+                       torch.from_numpy(ref["row_scale"]))
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+        ctx.set_option(sph.SPH_OPT_TC_BLOCK_K, 0)
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
