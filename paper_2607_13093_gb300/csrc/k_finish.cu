@@ -9,6 +9,7 @@
 // single warp scans the step sums in ascending id order to find the step
 // holding u * total, then scans that step lane by lane.  Everything is in
 // ascending vocabulary-id order, as the oracle's CDF.
+#include "sm100_ptx.cuh"
 #include "sph_common.cuh"
 #include "sph_internal.h"
 
@@ -29,6 +30,8 @@ __global__ void quantize_kernel(const float* __restrict__ Y,
                                 int8_t* __restrict__ codes,
                                 float* __restrict__ row_scale,
                                 int rows) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
   for (int r = blockIdx.y; r < rows; r += gridDim.y) {
     const float a = __uint_as_float(rowmax[r]);
     const float s = __fdiv_rn(a, 127.0f);
@@ -179,6 +182,8 @@ sample_kernel(const float* __restrict__ Z, int n,
               uint64_t offset, int32_t* __restrict__ tokens) {
   extern __shared__ float steps[];
   __shared__ float red[32];
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
   const int r = blockIdx.x;
   const float* z = Z + (int64_t)r * n;
   const float m = row_max(z, n, red);
@@ -214,6 +219,8 @@ verify_kernel(const float* __restrict__ Z, int k, int n,
   extern __shared__ float steps[];
   __shared__ float red[32];
   __shared__ int s_decision;            // kAccept, or the rejected draft's index
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
   const int s = blockIdx.x;
   const float u = philox_uniform(seed, (uint32_t)s, (uint32_t)(1 + k), offset);
   int i = 0;
@@ -279,9 +286,8 @@ cudaError_t launch_quantize(const float* Y, const unsigned* rowmax, int rows,
   int bx = (n + threads * 4 - 1) / (threads * 4);
   bx = bx < 1 ? 1 : (bx > 1024 ? 1024 : bx);
   dim3 grid(bx, rows < 65535 ? rows : 65535);
-  quantize_kernel<<<grid, threads, 0, st>>>(Y, rowmax, n, codes, row_scale, rows);
-  ++launch_count;
-  return cudaGetLastError();
+  return launch_pdl(quantize_kernel, grid, dim3(threads), 0, st, Y, rowmax, n, codes,
+                    row_scale, rows);
 }
 
 cudaError_t launch_sample(const float* Z, int rows, int n, const int32_t* ids,
@@ -292,10 +298,8 @@ cudaError_t launch_sample(const float* Z, int rows, int n, const int32_t* ids,
       sample_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
       (int)(kMaxSteps * sizeof(float)));
   if (e != cudaSuccess) return e;
-  sample_kernel<<<rows, kSampleThreads, smem, st>>>(Z, n, ids, inv_tau, seed,
-                                                    offset, tokens);
-  ++launch_count;
-  return cudaGetLastError();
+  return launch_pdl(sample_kernel, dim3(rows), dim3(kSampleThreads), smem, st, Z, n, ids,
+                    inv_tau, seed, offset, tokens);
 }
 
 cudaError_t launch_verify(const float* Z, int sessions, int k, int n,
@@ -308,10 +312,8 @@ cudaError_t launch_verify(const float* Z, int sessions, int k, int n,
       verify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
       (int)(kMaxSteps * sizeof(float)));
   if (e != cudaSuccess) return e;
-  verify_kernel<<<sessions, kSampleThreads, smem, st>>>(
-      Z, k, n, ids, V, inv_tau, draft, q, seed, offset, n_acc, next_token);
-  ++launch_count;
-  return cudaGetLastError();
+  return launch_pdl(verify_kernel, dim3(sessions), dim3(kSampleThreads), smem, st, Z, k, n,
+                    ids, V, inv_tau, draft, q, seed, offset, n_acc, next_token);
 }
 
 }  // namespace sph

@@ -10,6 +10,7 @@
 // HBM traffic is the kept W rows once per row tile; rows > RT are handled by
 // further row tiles (re-reading W), which is why the dispatcher routes more
 // than a couple of rows to the tensor-core kernel.
+#include "sm100_ptx.cuh"
 #include "sph_common.cuh"
 #include "sph_internal.h"
 
@@ -76,6 +77,8 @@ gemv_kernel(const GatherGemm g, const int row0) {
   const int K = g.K;
   const int KP = (K + 7) & ~7;                 // 32-byte aligned row stride
   const int rt = min(RT, g.rows - row0);
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
   for (int i = threadIdx.x; i < RT * KP; i += kThreads) {
     const int r = i / KP, c = i - r * KP;
     float v = 0.f;
@@ -193,9 +196,7 @@ cudaError_t launch_rt(const GatherGemm& g, int sm_count, cudaStream_t st) {
   blocks = blocks < sm_count * occ ? blocks : sm_count * occ;
   if (blocks < 1) blocks = 1;
   for (int row0 = 0; row0 < g.rows; row0 += RT) {
-    kern<<<blocks, kThreads, smem, st>>>(g, row0);
-    ++launch_count;
-    e = cudaGetLastError();
+    e = launch_pdl(kern, dim3(blocks), dim3(kThreads), smem, st, g, row0);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

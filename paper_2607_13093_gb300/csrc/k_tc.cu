@@ -68,8 +68,6 @@ struct TcParams {
   int na;                      // swizzle atoms per k-block (k-block = 64 * na)
   long long T;                 // total iterations RB * NT * KB
   const int32_t* ids;          // gather path: sorted ids
-  const int2* chunks;          // gather path: [NT][128] (first id, row | lg << 8)
-  const int2* chunk_count;     // gather path: [NT] (boxes, rows copied)
   int epilogue;
   const float* bias;
   float clip;
@@ -111,27 +109,67 @@ struct Segments {
   }
 };
 
+// Reduce 16 per-lane values over the 32 lanes of a warp, one result per
+// value index: a butterfly that halves the array at every exchange (16
+// shuffles in all).  Lane l ends with the reduction of index
+// (l >> 1) & 15; lanes l and l ^ 1 hold the same result.
+template <class Op>
+__device__ __forceinline__ float warp_reduce_scatter16(const float (&v)[16], Op op, int lane) {
+  float a8[8], a4[4], a2[2];
+  const bool b16 = lane & 16, b8 = lane & 8, b4 = lane & 4, b2 = lane & 2;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const float keep = b16 ? v[k + 8] : v[k], give = b16 ? v[k] : v[k + 8];
+    a8[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 16));
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float keep = b8 ? a8[k + 4] : a8[k], give = b8 ? a8[k] : a8[k + 4];
+    a4[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 8));
+  }
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const float keep = b4 ? a4[k + 2] : a4[k], give = b4 ? a4[k] : a4[k + 2];
+    a2[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 4));
+  }
+  const float keep = b2 ? a2[1] : a2[0], give = b2 ? a2[0] : a2[1];
+  float r = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 2));
+  return op(r, __shfl_xor_sync(0xFFFFFFFFu, r, 1));
+}
+
+struct MaxOp {
+  __device__ float operator()(float a, float b) const { return fmaxf(a, b); }
+};
+struct SumOp {
+  __device__ float operator()(float a, float b) const { return a + b; }
+};
+
+// Epilogue of 16 accumulator columns (hidden-state rows row0..row0+15) for
+// this lane's vocabulary column j.
 template <int EPI>
 __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)[16],
                                              int row0, int j, bool vj, int id,
                                              int lane, int seg) {
+  const int kr = (lane >> 1) & 15;               // the row this lane reduces
   if constexpr (EPI == EPI_CLOUD) {
+    const float b = (vj && p.bias) ? p.bias[id] : 0.f;
+    float m[16];
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const int r = row0 + q;
-      float m = 0.f;
+      m[q] = 0.f;
       if (vj && r < p.R) {
-        float y = v[q];
-        if (p.bias) y += p.bias[id];
+        const float y = v[q] + b;
         const int64_t o = (int64_t)r * p.n + j;
         if (p.partial_out) p.partial_out[o] = y;
         const float yc = fminf(fmaxf(y, -p.clip), p.clip);
         p.Y[o] = yc;
-        m = fabsf(yc);
+        m[q] = fabsf(yc);
       }
-      m = warp_max(m);
-      if (lane == 0 && r < p.R && m > 0.f) atomicMax(&p.rowmax[r], __float_as_uint(m));
     }
+    const float mr = warp_reduce_scatter16(m, MaxOp{}, lane);
+    if (!(lane & 1) && row0 + kr < p.R && mr > 0.f)
+      atomicMax(&p.rowmax[row0 + kr], __float_as_uint(mr));
   } else {
     // all payload loads first, then the stores (the stores could alias the
     // loads as far as the compiler knows, which would serialise them)
@@ -148,16 +186,18 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
       const int r = row0 + q;
       if (vj && r < p.R) p.Y[(int64_t)r * p.n + j] = z[q];
     }
-    // softmax statistics of this 32-id segment for each row
+    // softmax statistics of this 32-id segment for each row: the maxima,
+    // spread back to every lane, then the sums of exp((z - max) / tau)
+    const float mk = warp_reduce_scatter16(z, MaxOp{}, lane);
+    float e[16];
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
-      const int r = row0 + q;
-      const float m = warp_max(z[q]);
-      const float e = vj && r < p.R ? expf((z[q] - m) * p.inv_tau) : 0.f;
-      const float s = warp_sum(e);
-      if (lane == 0 && r < p.R)
-        p.seg_stats[(int64_t)r * (p.NT * 4) + seg] = make_float2(m, s);
+      const float mq = __shfl_sync(0xFFFFFFFFu, mk, 2 * q);
+      e[q] = (vj && row0 + q < p.R) ? expf((z[q] - mq) * p.inv_tau) : 0.f;
     }
+    const float sk = warp_reduce_scatter16(e, SumOp{}, lane);
+    if (!(lane & 1) && row0 + kr < p.R)
+      p.seg_stats[(int64_t)(row0 + kr) * (p.NT * 4) + seg] = make_float2(mk, sk);
   }
 }
 
@@ -203,6 +243,10 @@ tc_kernel(const __grid_constant__ WMaps wm,
     if (GATHER || lane == kBoxHeights - 1) ptx::prefetch_tmap(&wm.m[lane]);
     if (lane == 0) ptx::prefetch_tmap(&tmH);
   }
+  // Only the warps that touch memory written or read by the kernels before
+  // this one wait for them (griddep_wait): the producer before its first
+  // copy, the epilogue before its first store.
+  ptx::griddep_launch_dependents();
   if (warp == 1) ptx::tmem_alloc(tmem_holder, ncols);
   ptx::tc_fence_before();
   __syncthreads();
@@ -221,28 +265,68 @@ tc_kernel(const __grid_constant__ WMaps wm,
 
   if (warp == 0) {
     // ------------------------------------------------------- TMA producer
-    // lane 0 owns the ring; on the subset path every lane issues the boxes
-    // of up to four of the tile's row chunks
+    // lane 0 owns the ring.  On the subset path the warp plans each tile's
+    // row boxes itself (lane l owns tile rows l, l+32, l+64, l+96): runs of
+    // consecutive kept ids, each covered by one box of 2^k rows, or two
+    // that overlap on identically copied rows; every lane issues the boxes
+    // of the runs that start in its rows.
     Segments sg{it0, it1, p.KB};
     int stage = 0;
     uint32_t phase = 0;
     int tile, kb0, kb1;
     bool stop = false;
     long long issued = 0;
+    if (lane == 0) ptx::griddep_wait();          // h planes come from the prep kernel
+    __syncwarp();
     while (!stop && sg.next(tile, kb0, kb1)) {
       const int rb = tile / p.NT, t = tile - rb * p.NT;
-      int2 ch[4];
-      int nmine = 0;
+      int2 box[8];                               // (first id, row | lg << 8)
+      unsigned bmask = 0;                        // which of box[] are in use
       uint32_t tx = (uint32_t)stage_bytes;
       if constexpr (GATHER) {
-        const int2 cc = p.chunk_count[t];        // (boxes, rows copied)
+        const int j0 = t * kTileM;
+        const int rows = min(kTileM, p.n - j0);
+        int idr[4];
+        unsigned smask[4];
+        int prev_last = 0;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int ci = lane + 32 * q;
-          ch[q] = ci < cc.x ? p.chunks[(int64_t)t * kTileM + ci] : make_int2(0, 0);
-          if (ci < cc.x) nmine = q + 1;
+        for (int g = 0; g < 4; ++g) {
+          const int r = 32 * g + lane;
+          idr[g] = r < rows ? p.ids[j0 + r] : 0;
+          int prev = __shfl_up_sync(0xFFFFFFFFu, idr[g], 1);
+          if (lane == 0) prev = prev_last;
+          smask[g] = __ballot_sync(0xFFFFFFFFu, r < rows && (r == 0 || idr[g] != prev + 1));
+          prev_last = __shfl_sync(0xFFFFFFFFu, idr[g], 31);
         }
-        tx = (uint32_t)(cc.y * 128 * NA + b_bytes);
+        int covered = 0;
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+          const int r = 32 * g + lane;
+          if ((smask[g] >> lane) & 1u) {
+            int nxt = rows;
+            const unsigned above = lane == 31 ? 0u : (smask[g] >> (lane + 1)) << (lane + 1);
+            if (above) {
+              nxt = 32 * g + __ffs(above) - 1;
+            } else {
+              for (int g2 = g + 1; g2 < 4; ++g2)
+                if (smask[g2]) { nxt = 32 * g2 + __ffs(smask[g2]) - 1; break; }
+            }
+            const int len = nxt - r;
+            const int lg = 31 - __clz(len);
+            box[2 * g] = make_int2(idr[g], r | (lg << 8));
+            bmask |= 1u << (2 * g);
+            covered += 1 << lg;
+            if (len != (1 << lg)) {
+              box[2 * g + 1] =
+                  make_int2(idr[g] + len - (1 << lg), (r + len - (1 << lg)) | (lg << 8));
+              bmask |= 2u << (2 * g);
+              covered += 1 << lg;
+            }
+          }
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) covered += __shfl_xor_sync(0xFFFFFFFFu, covered, o);
+        tx = (uint32_t)(covered * 128 * NA + b_bytes);
       }
       for (int kb = kb0; kb < kb1; ++kb) {
         int ok = 1;
@@ -256,15 +340,14 @@ tc_kernel(const __grid_constant__ WMaps wm,
         if (lane == 0) ptx::mbar_expect_tx(&full[stage], tx);
         __syncwarp();
         uint8_t* A = base + (size_t)stage * stage_bytes;
-        uint8_t* B = A + a_bytes;
         for (int a = 0; a < NA; ++a) {
           const int x = (kb * NA + a) * kAtomK;
           if constexpr (GATHER) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              if (q < nmine) {
-                const int row = ch[q].y & 0xFF, lg = ch[q].y >> 8;
-                ptx::tma_load_2d(A + a * kAtomBytes + row * 128, &wm.m[lg], x, ch[q].x,
+            for (int q = 0; q < 8; ++q) {
+              if ((bmask >> q) & 1u) {
+                const int row = box[q].y & 0xFF, lg = box[q].y >> 8;
+                ptx::tma_load_2d(A + a * kAtomBytes + row * 128, &wm.m[lg], x, box[q].x,
                                  &full[stage]);
               }
             }
@@ -273,10 +356,13 @@ tc_kernel(const __grid_constant__ WMaps wm,
               ptx::tma_load_2d(A + a * kAtomBytes, &wm.m[kBoxHeights - 1], x, t * kTileM,
                                &full[stage]);
           }
-          if (lane == 0)
+        }
+        if (lane == 0) {
+          uint8_t* B = A + a_bytes;
+          for (int a = 0; a < NA; ++a)
             for (int h = 0; h < HILO; ++h)
-              ptx::tma_load_2d(B + (h * NA + a) * BN * 128, &tmH, x, h * p.Rp + rb * BN,
-                               &full[stage]);
+              ptx::tma_load_2d(B + (h * NA + a) * BN * 128, &tmH, (kb * NA + a) * kAtomK,
+                               h * p.Rp + rb * BN, &full[stage]);
         }
         ++issued;
         if (++stage == S) { stage = 0; phase ^= 1; }
@@ -341,6 +427,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     // ------------------------------------------------------------ epilogue
     const int quad = warp & 3;
     const int i = quad * 32 + lane;              // vocabulary row in the tile
+    ptx::griddep_wait();
     Segments sg{it0, it1, p.KB};
     uint32_t fph[2] = {0, 0};
     int si = 0, tile, kb0, kb1;
@@ -385,21 +472,40 @@ tc_kernel(const __grid_constant__ WMaps wm,
         int old = 0;
         if (lane == 0) old = atomicAdd(&p.counters[tile * 4 + quad], 1);
         old = __shfl_sync(0xFFFFFFFFu, old, 0);
-        const long long c0 = cta_of((long long)tile * p.KB, p.T, gridDim.x);
-        const long long c1 = cta_of((long long)tile * p.KB + p.KB - 1, p.T, gridDim.x);
-        if (old == (int)(c1 - c0)) {
+        const int c0 = (int)cta_of((long long)tile * p.KB, p.T, gridDim.x);
+        const int c1 = (int)cta_of((long long)tile * p.KB + p.KB - 1, p.T, gridDim.x);
+        if (old == c1 - c0) {
           __threadfence();
+          // the contributors' slots, in CTA order (a fixed summation order):
+          // every contributor after the first starts its range inside this
+          // tile, so the tile is its first segment (slot 2c); the first one
+          // holds it as its first segment only if its range starts exactly
+          // at the tile (slot 2c0), else as its last (slot 2c0 + 1)
+          constexpr int kMaxC = 8;
+          const float* ps[kMaxC];
+          const int C = c1 - c0 + 1;
+          const bool c0_first = range_start(p, c0, gridDim.x) == (long long)tile * p.KB;
+#pragma unroll
+          for (int c = 0; c < kMaxC; ++c) {
+            const int slot = c == 0 ? 2 * c0 + (c0_first ? 0 : 1) : 2 * (c0 + (c < C ? c : 0));
+            ps[c] = p.P + (size_t)slot * BN * kTileM + i;
+          }
           for (int ch = 0; ch < BN / 16; ++ch) {
             float v[16];
 #pragma unroll
-            for (int q = 0; q < 16; ++q) v[q] = 0.f;
-            // contributors in CTA order: a fixed summation order
-            for (long long c = c0; c <= c1; ++c) {
-              const long long start = c * p.T / gridDim.x;
-              const int slot = 2 * (int)c + ((start / p.KB) == tile ? 0 : 1);
-              const float* Ps = p.P + (size_t)slot * BN * kTileM + (size_t)ch * 16 * kTileM + i;
+            for (int q = 0; q < 16; ++q) v[q] = __ldcg(ps[0] + (size_t)(ch * 16 + q) * kTileM);
 #pragma unroll
-              for (int q = 0; q < 16; ++q) v[q] += __ldcg(Ps + (size_t)q * kTileM);
+            for (int c = 1; c < kMaxC; ++c) {
+              if (c < C) {
+#pragma unroll
+                for (int q = 0; q < 16; ++q)
+                  v[q] += __ldcg(ps[c] + (size_t)(ch * 16 + q) * kTileM);
+              }
+            }
+            for (int c = kMaxC; c < C; ++c) {    // rare: very many contributors
+              const float* pc = p.P + (size_t)(2 * (c0 + c)) * BN * kTileM + i;
+#pragma unroll
+              for (int q = 0; q < 16; ++q) v[q] += __ldcg(pc + (size_t)(ch * 16 + q) * kTileM);
             }
             finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg);
           }
@@ -419,77 +525,17 @@ tc_kernel(const __grid_constant__ WMaps wm,
 // ---------------------------------------------------------------------------
 // operand preparation: fp32 h -> bf16 hi (and lo) planes, zero padded
 // ---------------------------------------------------------------------------
-// ... and, on the subset path, the row boxes of every vocabulary tile (one
-// warp per tile): the tile's kept ids are cut into runs of consecutive ids,
-// and a run of length L is covered by one box of 2^k rows if L = 2^k, else by
-// two boxes of 2^k rows (k = floor(log2 L)) placed at its start and at its
-// end, which overlap on rows they both copy identically.  Each box is stored
-// as (first id, tile row | lg << 8); per tile (box count, rows copied).
+// ... and clear the split-tile counters and (cloud) the row maxima.
 __global__ void split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R,
                                int K, int Rp, int Kp, int hilo,
                                __nv_bfloat16* __restrict__ Hs,
                                int* __restrict__ counters, int ncounters,
-                               const int32_t* __restrict__ ids, int n, int NT,
-                               int2* __restrict__ chunks, int2* __restrict__ chunk_count) {
-  if (ids) {
-    const int lane = threadIdx.x & 31;
-    const int nwarps = (gridDim.x * blockDim.x) >> 5;
-    for (int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; t < NT; t += nwarps) {
-      const int j0 = t * kTileM;
-      const int rows = min(kTileM, n - j0);
-      int idr[4];
-      unsigned smask[4];
-      int prev_last = 0;
-#pragma unroll
-      for (int g = 0; g < 4; ++g) {
-        const int r = 32 * g + lane;
-        idr[g] = r < rows ? ids[j0 + r] : 0;
-        int prev = __shfl_up_sync(0xFFFFFFFFu, idr[g], 1);
-        if (lane == 0) prev = prev_last;
-        const bool start = r < rows && (r == 0 || idr[g] != prev + 1);
-        smask[g] = __ballot_sync(0xFFFFFFFFu, start);
-        prev_last = __shfl_sync(0xFFFFFFFFu, idr[g], 31);
-      }
-      int base = 0, covered = 0;
-#pragma unroll
-      for (int g = 0; g < 4; ++g) {
-        const int r = 32 * g + lane;
-        const bool start = (smask[g] >> lane) & 1u;
-        int nbox = 0, len = 0, lg = 0;
-        if (start) {
-          // the next run start above r, or the end of the tile
-          int nxt = rows;
-          const unsigned above = lane == 31 ? 0u : (smask[g] >> (lane + 1)) << (lane + 1);
-          if (above) {
-            nxt = 32 * g + __ffs(above) - 1;
-          } else {
-            for (int g2 = g + 1; g2 < 4; ++g2)
-              if (smask[g2]) { nxt = 32 * g2 + __ffs(smask[g2]) - 1; break; }
-          }
-          len = nxt - r;
-          lg = 31 - __clz(len);
-          nbox = (len == (1 << lg)) ? 1 : 2;
-        }
-        int incl = nbox;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-          if (lane >= o) incl += v;
-        }
-        const int off = base + incl - nbox;
-        if (nbox >= 1) chunks[(int64_t)t * kTileM + off] = make_int2(idr[g], r | (lg << 8));
-        if (nbox == 2)
-          chunks[(int64_t)t * kTileM + off + 1] =
-              make_int2(idr[g] + len - (1 << lg), (r + len - (1 << lg)) | (lg << 8));
-        int rows_here = nbox * (nbox ? (1 << lg) : 0);
-#pragma unroll
-        for (int o = 16; o; o >>= 1) rows_here += __shfl_xor_sync(0xFFFFFFFFu, rows_here, o);
-        covered += rows_here;
-        base += __shfl_sync(0xFFFFFFFFu, incl, 31);
-      }
-      if (lane == 0) chunk_count[t] = make_int2(base, covered);
-    }
-  }
+                               unsigned* __restrict__ rowmax) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  if (rowmax)
+    for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x)
+      rowmax[r] = 0u;
   const int64_t total = (int64_t)Rp * Kp;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
@@ -512,6 +558,8 @@ __global__ void sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
                                   const int32_t* __restrict__ ids, float inv_tau,
                                   uint64_t seed, uint64_t offset,
                                   int32_t* __restrict__ tokens) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (r >= rows) return;
@@ -659,10 +707,7 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * kTileM * 4) : 0;
   pl.cnt_bytes = align256((size_t)tiles * 4 * sizeof(int));
   pl.stats_bytes = endpoint ? align256((size_t)rows * pl.NT * 4 * sizeof(float2)) : 0;
-  pl.chunk_bytes = gather ? align256((size_t)pl.NT * kTileM * sizeof(int2)) +
-                                align256((size_t)pl.NT * sizeof(int2))
-                          : 0;
-  pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes + pl.chunk_bytes;
+  pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
   pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256;
   pl.ok = pl.stages >= 2;
   return pl;
@@ -676,9 +721,7 @@ static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)pl.smem_bytes);
   if (e != cudaSuccess) return e;
-  kern<<<pl.G, kThreads, pl.smem_bytes, st>>>(mw, mh, prm);
-  ++launch_count;
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(pl.G), dim3(kThreads), pl.smem_bytes, st, mw, mh, prm);
 }
 
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
@@ -691,25 +734,17 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   float2* stats = pl.stats_bytes
                       ? reinterpret_cast<float2*>(sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes)
                       : nullptr;
-  char* chunk_base = sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
   const bool gather = g.ids != nullptr;
-  int2* chunks = gather ? reinterpret_cast<int2*>(chunk_base) : nullptr;
-  int2* chunk_count = gather ? reinterpret_cast<int2*>(
-                                   chunk_base + align256((size_t)pl.NT * kTileM * sizeof(int2)))
-                             : nullptr;
   const int tiles = pl.RB * pl.NT;
 
   {
     const int64_t total = (int64_t)pl.Rp * pl.Kp;
-    int64_t work = total > (int64_t)pl.NT * 32 ? total : (int64_t)pl.NT * 32;
-    int blocks = (int)((work + 255) / 256);
+    int blocks = (int)((total + 255) / 256);
     if (blocks > 4096) blocks = 4096;
     if (blocks < 1) blocks = 1;
-    split_h_kernel<<<blocks, 256, 0, st>>>(g.h, g.ld_h, g.rows, g.K, pl.Rp, pl.Kp,
-                                           pl.hilo, Hs, counters, tiles * 4, g.ids, g.n,
-                                           pl.NT, chunks, chunk_count);
-    ++launch_count;
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(split_h_kernel, dim3(blocks), dim3(256), 0, st, g.h, g.ld_h,
+                               g.rows, g.K, pl.Rp, pl.Kp, pl.hilo, Hs, counters, tiles * 4,
+                               g.epilogue == EPI_CLOUD ? g.rowmax : (unsigned*)nullptr);
     if (e != cudaSuccess) return e;
   }
 
@@ -735,7 +770,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.R = g.rows; prm.n = g.n; prm.K = g.K; prm.KB = pl.KB; prm.NT = pl.NT;
   prm.RB = pl.RB; prm.BN = pl.BN; prm.Rp = pl.Rp; prm.stages = pl.stages;
   prm.whole_tiles = pl.whole_tiles; prm.T = pl.T; prm.na = pl.na;
-  prm.ids = g.ids; prm.chunks = chunks; prm.chunk_count = chunk_count;
+  prm.ids = g.ids;
   prm.epilogue = g.epilogue; prm.bias = g.bias;
   prm.clip = g.clip; prm.partial_out = g.partial_out; prm.Y = g.Y;
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
@@ -765,10 +800,8 @@ cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPl
       reinterpret_cast<const float2*>(sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes);
   const int warps = 8;
   const int blocks = (rows + warps - 1) / warps;
-  sample_seg_kernel<<<blocks, warps * 32, 0, st>>>(Z, rows, n, stats, pl.NT * 4, ids,
-                                                   inv_tau, seed, offset, tokens);
-  ++launch_count;
-  return cudaGetLastError();
+  return launch_pdl(sample_seg_kernel, dim3(blocks), dim3(warps * 32), 0, st, Z, rows, n,
+                    stats, pl.NT * 4, ids, inv_tau, seed, offset, tokens);
 }
 
 }  // namespace sph

@@ -195,3 +195,21 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 
 }  // namespace ptx
 }  // namespace sph
+
+namespace sph {
+namespace ptx {
+
+// ---- programmatic dependent launch ------------------------------------------
+// Block until the grids this one depends on have completed and their memory
+// is visible (a no-op when launched without a programmatic dependency).
+__device__ __forceinline__ void griddep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+// Let the next grid in the stream launch now; it still waits in
+// griddep_wait() for this grid to complete.
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+}  // namespace ptx
+}  // namespace sph

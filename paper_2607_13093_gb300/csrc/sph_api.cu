@@ -434,8 +434,10 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
   Carve c(ctx->scratch);
   float* Y = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
   unsigned* rowmax = static_cast<unsigned*>(c.take((size_t)rows * 4));
-  cudaError_t e = cudaMemsetAsync(rowmax, 0, (size_t)rows * 4, ctx->stream);
-  if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMemsetAsync");
+  if (!use_tc(ctx, rows, wdt)) {     // the tensor-core path clears them itself
+    cudaError_t e = cudaMemsetAsync(rowmax, 0, (size_t)rows * 4, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMemsetAsync");
+  }
 
   sph::GatherGemm gg{};
   gg.h = h_cloud; gg.ld_h = ld_h; gg.rows = (int)rows;

@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace sph {
 
 enum Epilogue : int {
@@ -22,6 +24,27 @@ enum : unsigned int {
 
 // Kernels launched by this thread (read by the tracing layer).
 extern thread_local long long launch_count;
+
+// Launch with programmatic stream serialization: the kernel may start while
+// the previous kernel of the stream is still running, and must call
+// griddepcontrol.wait (ptx::griddep_wait) before it touches memory that an
+// earlier kernel writes or reads.  Every kernel of this library does so.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  ++launch_count;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // One gathered contraction  acc[r, j] = sum_c h[r, c] * W[ids[j], c]
 // followed by an epilogue.  Pointers are device pointers.
@@ -61,7 +84,7 @@ int gemv_max_k();
 struct TcPlan {
   int hilo, RB, BN, Rp, KB, Kp, NT, G, stages, whole_tiles, na;
   long long T;
-  size_t hs_bytes, p_bytes, cnt_bytes, stats_bytes, chunk_bytes, scratch_bytes, smem_bytes;
+  size_t hs_bytes, p_bytes, cnt_bytes, stats_bytes, scratch_bytes, smem_bytes;
   bool ok;
 };
 // `endpoint` reserves the per-segment softmax statistics; schedule 0/1/2 =
