@@ -56,6 +56,8 @@ constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
 
 constexpr int kThreads = 192;
+constexpr int kThreadsFp8 = 320;     // + four converter warps (fp8 weights)
+constexpr int kMaxBNFp8 = 128;       // h rows per block with fp8 weights
 constexpr int kBoxHeights = 8;       // row boxes of 1, 2, 4, ..., 128 rows
 
 // W tensor maps: box height 2^i rows for map i (64 columns each).
@@ -68,6 +70,9 @@ struct TcParams {
   int na;                      // swizzle atoms per k-block (k-block = 64 * na)
   long long T;                 // total iterations RB * NT * KB
   const int32_t* ids;          // gather path: sorted ids
+  const uint8_t* W8;           // fp8 path: e4m3 weights, row stride ld_w bytes
+  int64_t ld_w;
+  const float* w_scale;        // fp8 path: per-vocabulary-row scale
   int epilogue;
   const float* bias;
   float clip;
@@ -153,13 +158,16 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
   const int kr = (lane >> 1) & 15;               // the row this lane reduces
   if constexpr (EPI == EPI_CLOUD) {
     const float b = (vj && p.bias) ? p.bias[id] : 0.f;
+    // fp8 weights entered the MMA as e4m3 * 2^-8 (f16); undo that and
+    // apply the row scale
+    const float ws = (vj && p.w_scale) ? 256.0f * p.w_scale[id] : 1.0f;
     float m[16];
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const int r = row0 + q;
       m[q] = 0.f;
       if (vj && r < p.R) {
-        const float y = v[q] + b;
+        const float y = v[q] * ws + b;
         const int64_t o = (int64_t)r * p.n + j;
         if (p.partial_out) p.partial_out[o] = y;
         const float yc = fminf(fmaxf(y, -p.clip), p.clip);
@@ -201,8 +209,8 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
   }
 }
 
-template <int HILO, bool GATHER, int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int HILO, bool GATHER, int EPI, bool FP8>
+__global__ void __launch_bounds__(FP8 ? kThreadsFp8 : kThreads, 1)
 tc_kernel(const __grid_constant__ WMaps wm,
           const __grid_constant__ CUtensorMap tmH, const TcParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -228,7 +236,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      ptx::mbar_init(&full[s], 1);               // the TMA thread's expect_tx
+      ptx::mbar_init(&full[s], FP8 ? 2 : 1);     // TMA thread (+ owning converter)
       ptx::mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -240,7 +248,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     ptx::fence_mbar_init();
   }
   if (warp == 0 && lane < kBoxHeights) {
-    if (GATHER || lane == kBoxHeights - 1) ptx::prefetch_tmap(&wm.m[lane]);
+    if (!FP8 && (GATHER || lane == kBoxHeights - 1)) ptx::prefetch_tmap(&wm.m[lane]);
     if (lane == 0) ptx::prefetch_tmap(&tmH);
   }
   // Only the warps that touch memory written or read by the kernels before
@@ -282,8 +290,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
       const int rb = tile / p.NT, t = tile - rb * p.NT;
       int2 box[8];                               // (first id, row | lg << 8)
       unsigned bmask = 0;                        // which of box[] are in use
-      uint32_t tx = (uint32_t)stage_bytes;
-      if constexpr (GATHER) {
+      uint32_t tx = (uint32_t)(FP8 ? b_bytes : stage_bytes);
+      if constexpr (GATHER && !FP8) {
         const int j0 = t * kTileM;
         const int rows = min(kTileM, p.n - j0);
         int idr[4];
@@ -340,7 +348,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
         if (lane == 0) ptx::mbar_expect_tx(&full[stage], tx);
         __syncwarp();
         uint8_t* A = base + (size_t)stage * stage_bytes;
-        for (int a = 0; a < NA; ++a) {
+        for (int a = 0; a < NA && !FP8; ++a) {
           const int x = (kb * NA + a) * kAtomK;
           if constexpr (GATHER) {
 #pragma unroll
@@ -381,7 +389,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
       uint32_t phase = 0;
       uint32_t tph[2] = {0, 0};
       int si = 0, tile, kb0, kb1;
-      const uint32_t idesc = ptx::idesc_bf16_f32(kTileM, BN);
+      const uint32_t idesc =
+          FP8 ? ptx::idesc_f16_f32(kTileM, BN) : ptx::idesc_bf16_f32(kTileM, BN);
       bool stop = false;
       while (!stop && sg.next(tile, kb0, kb1)) {
         const int acc = si & 1;
@@ -406,7 +415,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
             for (int h = 0; h < HILO; ++h) {
 #pragma unroll
               for (int kk = 0; kk < kAtomK / 16; ++kk) {
-                ptx::umma_bf16(d, ptx::sdesc_k128(a0 + at * kAtomBytes + kk * 32),
+                ptx::umma_f16(d, ptx::sdesc_k128(a0 + at * kAtomBytes + kk * 32),
                                ptx::sdesc_k128(b0 + (h * NA + at) * BN * 128 + kk * 32),
                                idesc, (kb != kb0 || at != 0 || h != 0 || kk != 0) ? 1u : 0u);
               }
@@ -423,7 +432,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
       ptx::umma_commit(drain);
       ptx::mbar_wait(drain, 0, kDrainLimit);
     }
-  } else {
+  } else if (warp < 6) {
     // ------------------------------------------------------------ epilogue
     const int quad = warp & 3;
     const int i = quad * 32 + lane;              // vocabulary row in the tile
@@ -514,6 +523,86 @@ tc_kernel(const __grid_constant__ WMaps wm,
       }
       ++si;
     }
+  } else if constexpr (FP8) {
+    // -------------------------------------------- converter warps (fp8 A)
+    // Stages go round-robin to the four converter warps; the ring has four
+    // or eight stages, so every slot has one owning warp.  A warp loads the
+    // 128 rows x 64 e4m3 bytes of its stage with 16-byte loads (four lanes
+    // per row), rewrites every byte as the f16 with the same sign and the
+    // magnitude bits shifted up by 7 -- exactly the e4m3 value times 2^-8,
+    // subnormals included -- stores the 128-byte-swizzled f16 rows, fences
+    // the async proxy and arrives on the stage barrier.
+    const int gw = warp - 6;
+    const int c = lane & 3;                      // 16-byte chunk of a 64-byte row slice
+    const int r0 = lane >> 2;                    // rows r0 + 8m, m = 0..15
+    ptx::griddep_wait();                         // (inputs only; keeps ordering simple)
+    Segments sg{it0, it1, p.KB};
+    long long k = 0;
+    int tile, kb0, kb1;
+    bool stop = false;
+    while (!stop && sg.next(tile, kb0, kb1)) {
+      const int t = tile % p.NT;
+      int rid[16];
+#pragma unroll
+      for (int m = 0; m < 16; ++m) {
+        const int jj = min(t * kTileM + r0 + 8 * m, p.n - 1);
+        rid[m] = GATHER ? p.ids[jj] : jj;
+      }
+      for (int kb = kb0; kb < kb1; ++kb, ++k) {
+        if ((int)(k & 3) != gw) continue;
+        const int stage = (int)(k % S);
+        const uint32_t phase = (uint32_t)((k / S) & 1);
+        int ok = 1;
+        if (lane == 0) ok = !*s_abort && ptx::mbar_wait(&empty[stage], phase ^ 1, limit);
+        ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+        if (!ok) {
+          if (lane == 0 && !*s_abort) give_up();
+          stop = true;
+          break;
+        }
+        const int e0 = kb * kAtomK + c * 16;     // first byte (= element) of my chunk
+        const int left = p.K - e0;               // valid bytes in it
+        uint4 raw[16];
+#pragma unroll
+        for (int m = 0; m < 16; ++m) {
+          raw[m] = make_uint4(0, 0, 0, 0);
+          if (left > 0)
+            raw[m] = __ldg(reinterpret_cast<const uint4*>(p.W8 + (int64_t)rid[m] * p.ld_w + e0));
+        }
+        if (left > 0 && left < 16) {             // zero the bytes past K
+#pragma unroll
+          for (int m = 0; m < 16; ++m) {
+            uint32_t w4[4] = {raw[m].x, raw[m].y, raw[m].z, raw[m].w};
+#pragma unroll
+            for (int b = 0; b < 16; ++b)
+              if (b >= left) w4[b >> 2] &= ~(0xFFu << (8 * (b & 3)));
+            raw[m] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+          }
+        }
+        uint8_t* A = base + (size_t)stage * stage_bytes;
+#pragma unroll
+        for (int m = 0; m < 16; ++m) {
+          const int row = r0 + 8 * m;
+          const uint32_t w4[4] = {raw[m].x, raw[m].y, raw[m].z, raw[m].w};
+          uint32_t h[8];                         // 16 f16 values
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t lo = __byte_perm(w4[q], 0u, 0x4140);   // bytes 0,1 -> halves
+            const uint32_t hi = __byte_perm(w4[q], 0u, 0x4342);   // bytes 2,3 -> halves
+            h[2 * q] = ((lo & 0x00800080u) << 8) | ((lo & 0x007F007Fu) << 7);
+            h[2 * q + 1] = ((hi & 0x00800080u) << 8) | ((hi & 0x007F007Fu) << 7);
+          }
+          const int c0 = 2 * c, c1 = 2 * c + 1;  // 16-byte f16 chunks of the row
+          *reinterpret_cast<uint4*>(A + row * 128 + ((c0 ^ (row & 7)) << 4)) =
+              make_uint4(h[0], h[1], h[2], h[3]);
+          *reinterpret_cast<uint4*>(A + row * 128 + ((c1 ^ (row & 7)) << 4)) =
+              make_uint4(h[4], h[5], h[6], h[7]);
+        }
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&full[stage]);
+      }
+    }
   }
 
   ptx::tc_fence_before();
@@ -526,11 +615,13 @@ tc_kernel(const __grid_constant__ WMaps wm,
 // operand preparation: fp32 h -> bf16 hi (and lo) planes, zero padded
 // ---------------------------------------------------------------------------
 // ... and clear the split-tile counters and (cloud) the row maxima.
+// (planes of f16 instead of bf16 when f16 != 0: the fp8-weight path, where
+// bf16-activation mode first rounds h to bf16 and then splits that value)
 __global__ void split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R,
                                int K, int Rp, int Kp, int hilo,
                                __nv_bfloat16* __restrict__ Hs,
                                int* __restrict__ counters, int ncounters,
-                               unsigned* __restrict__ rowmax) {
+                               unsigned* __restrict__ rowmax, int f16, int act_bf16) {
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   if (rowmax)
@@ -541,9 +632,17 @@ __global__ void split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R,
        e += (int64_t)gridDim.x * blockDim.x) {
     const int r = (int)(e / Kp), c = (int)(e - (int64_t)r * Kp);
     const float x = (r < R && c < K) ? h[(int64_t)r * ld_h + c] : 0.f;
-    const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-    Hs[e] = hi;
-    if (hilo == 2) Hs[total + e] = __float2bfloat16_rn(x - __bfloat162float(hi));
+    if (f16) {
+      __half* H = reinterpret_cast<__half*>(Hs);
+      const float xr = act_bf16 ? __bfloat162float(__float2bfloat16_rn(x)) : x;
+      const __half hi = __float2half_rn(xr);
+      H[e] = hi;
+      if (hilo == 2) H[total + e] = __float2half_rn(xr - __half2float(hi));
+    } else {
+      const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+      Hs[e] = hi;
+      if (hilo == 2) Hs[total + e] = __float2bfloat16_rn(x - __bfloat162float(hi));
+    }
   }
   for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < ncounters;
        t += gridDim.x * blockDim.x)
@@ -666,20 +765,24 @@ size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 }  // namespace
 
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
-               int schedule, int max_stages, int block_k, int gather) {
+               int schedule, int max_stages, int block_k, int gather, int fp8) {
   TcPlan pl{};
-  pl.hilo = act_bf16 ? 1 : 2;
-  if (rows <= kMaxBN) {
+  // one bf16 plane carries bf16-rounded activations exactly; f16 planes
+  // (fp8 weights) always take two
+  pl.hilo = (act_bf16 && !fp8) ? 1 : 2;
+  pl.fp8 = fp8;
+  const int max_bn = fp8 ? kMaxBNFp8 : kMaxBN;
+  if (rows <= max_bn) {
     pl.RB = 1;
     pl.BN = (rows + 15) / 16 * 16;
   } else {
-    pl.RB = (rows + kMaxBN - 1) / kMaxBN;
+    pl.RB = (rows + max_bn - 1) / max_bn;
     pl.BN = ((rows + pl.RB - 1) / pl.RB + 15) / 16 * 16;
   }
   pl.Rp = pl.RB * pl.BN;
   // k-block width: as asked (automatic: 128), narrowed until the shared
   // memory holds at least min_stages pipeline stages
-  pl.na = block_k == 64 ? 1 : (block_k == 256 ? 4 : 2);
+  pl.na = fp8 ? 1 : (block_k == 64 ? 1 : (block_k == 256 ? 4 : 2));
   const int min_stages = block_k ? 2 : 4;
   while (pl.na > 1 &&
          (int)((kSmemBudget - 2048) / (pl.na * (kAtomBytes + pl.hilo * pl.BN * 128))) <
@@ -701,6 +804,9 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.stages = (int)((kSmemBudget - 2048) / stage_bytes);
   if (pl.stages > 8) pl.stages = 8;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
+  // fp8: four converter warps own the ring slots round-robin, so the ring
+  // has four or eight stages
+  if (fp8) pl.stages = pl.stages >= 8 ? 8 : (pl.stages >= 4 ? 4 : 0);
   pl.hs_bytes = align256((size_t)pl.hilo * pl.Rp * pl.Kp * 2);
   // split tiles exist only when a CTA's range does not cover whole tiles
   const bool splits = !pl.whole_tiles && (pl.T % pl.G != 0 || (pl.T / pl.G) % pl.KB != 0);
@@ -709,24 +815,27 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.stats_bytes = endpoint ? align256((size_t)rows * pl.NT * 4 * sizeof(float2)) : 0;
   pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
   pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256;
-  pl.ok = pl.stages >= 2;
+  pl.ok = fp8 ? pl.stages >= 4 : pl.stages >= 2;
   return pl;
 }
 
-template <int HILO, bool GATHER, int EPI>
+template <int HILO, bool GATHER, int EPI, bool FP8 = false>
 static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
                                const TcParams& prm, const TcPlan& pl,
                                cudaStream_t st) {
-  auto kern = tc_kernel<HILO, GATHER, EPI>;
+  auto kern = tc_kernel<HILO, GATHER, EPI, FP8>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)pl.smem_bytes);
   if (e != cudaSuccess) return e;
-  return launch_pdl(kern, dim3(pl.G), dim3(kThreads), pl.smem_bytes, st, mw, mh, prm);
+  return launch_pdl(kern, dim3(pl.G), dim3(FP8 ? kThreadsFp8 : kThreads), pl.smem_bytes, st,
+                    mw, mh, prm);
 }
 
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                       long long spin_limit, cudaStream_t st) {
-  if (!pl.ok || g.w_dtype != W_BF16) return cudaErrorNotSupported;
+  const bool fp8 = g.w_dtype == W_FP8;
+  if (!pl.ok || (fp8 != (pl.fp8 != 0)) || (fp8 && g.epilogue != EPI_CLOUD))
+    return cudaErrorNotSupported;
   char* sc = static_cast<char*>(scratch);
   auto* Hs = reinterpret_cast<__nv_bfloat16*>(sc);
   float* P = pl.p_bytes ? reinterpret_cast<float*>(sc + pl.hs_bytes) : nullptr;
@@ -744,7 +853,8 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
     if (blocks < 1) blocks = 1;
     cudaError_t e = launch_pdl(split_h_kernel, dim3(blocks), dim3(256), 0, st, g.h, g.ld_h,
                                g.rows, g.K, pl.Rp, pl.Kp, pl.hilo, Hs, counters, tiles * 4,
-                               g.epilogue == EPI_CLOUD ? g.rowmax : (unsigned*)nullptr);
+                               g.epilogue == EPI_CLOUD ? g.rowmax : (unsigned*)nullptr,
+                               fp8 ? 1 : 0, g.act_bf16);
     if (e != cudaSuccess) return e;
   }
 
@@ -753,7 +863,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   // W: [V rows, K columns], row stride ld_w; map i copies boxes of 64
   // columns x 2^i rows (the full-vocabulary path uses only the 128-row map)
   for (int i = 0; i < kBoxHeights; ++i) {
-    if (!gather && i != kBoxHeights - 1) {
+    if (fp8 || (!gather && i != kBoxHeights - 1)) {
       mw.m[i] = CUtensorMap{};
       continue;
     }
@@ -761,7 +871,8 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                   (uint64_t)g.V, (uint64_t)g.ld_w * 2, kAtomK, 1u << i))
       return cudaErrorInvalidValue;
   }
-  if (!make_map(&mh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, Hs, (uint64_t)pl.Kp,
+  if (!make_map(&mh, fp8 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                Hs, (uint64_t)pl.Kp,
                 (uint64_t)pl.hilo * pl.Rp, (uint64_t)pl.Kp * 2, kAtomK,
                 (uint32_t)pl.BN))
     return cudaErrorInvalidValue;
@@ -771,6 +882,9 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.RB = pl.RB; prm.BN = pl.BN; prm.Rp = pl.Rp; prm.stages = pl.stages;
   prm.whole_tiles = pl.whole_tiles; prm.T = pl.T; prm.na = pl.na;
   prm.ids = g.ids;
+  prm.W8 = fp8 ? static_cast<const uint8_t*>(g.W) : nullptr;
+  prm.ld_w = g.ld_w;
+  prm.w_scale = fp8 ? g.w_scale : nullptr;
   prm.epilogue = g.epilogue; prm.bias = g.bias;
   prm.clip = g.clip; prm.partial_out = g.partial_out; prm.Y = g.Y;
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
@@ -779,6 +893,12 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.status = g.status; prm.spin_limit = spin_limit;
 
   const bool hilo2 = pl.hilo == 2;
+  if (fp8) {
+    if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, true>(mw, mh, prm, pl, st)
+                             : launch_inst<1, true, EPI_CLOUD, true>(mw, mh, prm, pl, st);
+    return hilo2 ? launch_inst<2, false, EPI_CLOUD, true>(mw, mh, prm, pl, st)
+                 : launch_inst<1, false, EPI_CLOUD, true>(mw, mh, prm, pl, st);
+  }
   if (g.epilogue == EPI_CLOUD) {
     if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD>(mw, mh, prm, pl, st)
                              : launch_inst<1, true, EPI_CLOUD>(mw, mh, prm, pl, st);

@@ -121,7 +121,13 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
          ((uint32_t)(M >> 4) << 24);
 }
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc,
+// Instruction descriptor for kind::f16 with f16 A/B, fp32 D, K-major A/B.
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
+  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+// tcgen05.mma kind::f16 (the operand types come from the instruction
+// descriptor: bf16 x bf16 or f16 x f16)
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc,
                                           uint64_t bdesc, uint32_t idesc,
                                           uint32_t accumulate) {
   asm volatile(
@@ -129,6 +135,11 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc,
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc,
+                                          uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  umma_f16(d_tmem, adesc, bdesc, idesc, accumulate);
 }
 // Arrive on `bar` once all previously issued tcgen05.mma of this thread are
 // complete.

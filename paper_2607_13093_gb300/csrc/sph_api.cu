@@ -118,7 +118,8 @@ struct Carve {
 };
 
 bool use_tc(const sph_ctx* ctx, int64_t rows, int w_dtype) {
-  return rows >= ctx->tc_min_rows && w_dtype == sph::W_BF16;
+  (void)w_dtype;
+  return rows >= ctx->tc_min_rows;
 }
 
 size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_bf16,
@@ -128,7 +129,7 @@ size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_
   for (int gather = 0; gather < 2; ++gather) {   // the larger of the two paths
     const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count,
                                   endpoint, ctx->tc_schedule, ctx->tc_stages,
-                                  ctx->tc_block_k, gather)
+                                  ctx->tc_block_k, gather, w_dtype == sph::W_FP8)
                          .scratch_bytes;
     if (x > b) b = x;
   }
@@ -452,7 +453,8 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
   if (use_tc(ctx, rows, wdt)) {
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_h, act_bf16,
                                         ctx->sm_count, 0, ctx->tc_schedule, ctx->tc_stages,
-                                        ctx->tc_block_k, keep_ids != nullptr);
+                                        ctx->tc_block_k, keep_ids != nullptr,
+                                        wdt == sph::W_FP8);
     void* tcs = c.take(pl.scratch_bytes);
     st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
@@ -508,7 +510,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   if (use_tc(ctx, rows, sph::W_BF16)) {
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0,
                                         ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
-                                        ctx->tc_block_k, keep_ids != nullptr);
+                                        ctx->tc_block_k, keep_ids != nullptr, 0);
     void* tcs = c.take(pl.scratch_bytes);
     st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);

@@ -82,7 +82,7 @@ int gemv_max_k();
 
 // Tensor-core path (k_tc.cu): sizes, work split and scratch of one call.
 struct TcPlan {
-  int hilo, RB, BN, Rp, KB, Kp, NT, G, stages, whole_tiles, na;
+  int hilo, RB, BN, Rp, KB, Kp, NT, G, stages, whole_tiles, na, fp8;
   long long T;
   size_t hs_bytes, p_bytes, cnt_bytes, stats_bytes, scratch_bytes, smem_bytes;
   bool ok;
@@ -90,9 +90,9 @@ struct TcPlan {
 // `endpoint` reserves the per-segment softmax statistics; schedule 0/1/2 =
 // automatic / whole tiles / stream-K; max_stages 0 = automatic; block_k =
 // hidden elements per pipeline stage (64, 128 or 256; 0 = automatic);
-// gather = the kept-id subset path (keep_ids given).
+// gather = the kept-id subset path (keep_ids given); fp8 = e4m3 weights.
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
-               int schedule, int max_stages, int block_k, int gather);
+               int schedule, int max_stages, int block_k, int gather, int fp8);
 // Launch the operand split and the tcgen05 kernel; `scratch` holds
 // plan.scratch_bytes bytes.  bf16 weights only.
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,

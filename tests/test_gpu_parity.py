@@ -222,3 +222,32 @@ def test_tensor_core_variants(ctx, block_k, schedule, keep):
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
         ctx.set_option(sph.SPH_OPT_TC_BLOCK_K, 0)
         ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+
+
+# ---------------------------------------------------------------------------
+# fp8 (e4m3) weights on the tensor cores
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("rows,keep,act", [(16, 3000, "fp32"), (40, 1100, "fp32"),
+                                           (200, 2000, "fp32"), (24, 900, "bf16"),
+                                           (7, 3000, "fp32")])
+def test_fp8_tensor_core(ctx, rows, keep, act):
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    try:
+        # d_h = 1008: a ragged last 64-wide k-block
+        w = small(V=3000, d=1048, d_l=40, rows=rows, n_keep=keep, w_dtype="fp8",
+                  clip=40.0, seed=321 + rows, with_bias=(rows == 40))
+        check_cloud(ctx, w, act_mode=act)
+        if rows == 7:
+            # d_h = 1000 inside a 1008-byte row stride: the last 16-byte
+            # chunk of every row is only partly valid
+            Wp = torch.zeros(w.V, 1008, dtype=torch.float8_e4m3fn, device=DEV)
+            Wp.view(torch.uint8)[:, :1000] = w.W_h.view(torch.uint8)[:, :1000]
+            Wp.view(torch.uint8)[:, 1000:] = 0x7E          # junk past the end (448)
+            w.W_h = Wp[:, :1000]
+            w.h = w.h[:, :w.d_l + 1000].contiguous()
+            w.d = w.d_l + 1000
+            check_cloud(ctx, w, act_mode=act)
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
