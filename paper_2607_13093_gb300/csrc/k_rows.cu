@@ -1,0 +1,492 @@
+// Row-wise softmax statistics, inverse-CDF draws and speculative
+// verification over fused logits z (fp32 [rows, n], ascending compact ids).
+//
+//   seg_stats : per 32-id segment of every row, (max z, sum exp((z - max)/tau))
+//   sample    : Eq. 14-15, one Philox uniform per row, inverse CDF
+//   verify    : standard speculative acceptance of k drafts per session with
+//               a residual draw at the first rejection (Sec. "Endpoint
+//               Speculative Decoding and Cloud Verification", Algorithm 1)
+//
+// Every pass is spread over the whole GPU: the statistics pass reads each
+// logit once (the only HBM-sized pass), the row reductions and draws work on
+// the 32x smaller segment statistics.  A draw is a three-level search in
+// ascending id order -- 1024-id chunks, 32-id segments, ids -- whose CDF is
+// the oracle's up to fp32 rounding.
+#include "sm100_ptx.cuh"
+#include "sph_common.cuh"
+#include "sph_internal.h"
+
+namespace sph {
+namespace {
+
+constexpr int kSeg = 32;                // ids per segment (one per lane)
+constexpr int kGroup = 16;              // segments per half chunk (one reduce-scatter)
+constexpr int kWarps = 8;               // warps per CTA
+constexpr int kMaxN = 1 << 30;          // ids per row
+constexpr int kMaxK = 64;               // drafts per session
+
+__device__ __forceinline__ float seg_weight(float2 st, float M, float inv_tau) {
+  return st.y > 0.f ? st.y * expf((st.x - M) * inv_tau) : 0.f;
+}
+
+// ---------------------------------------------------------------------------
+// statistics: a warp takes one 1024-id chunk (32 segments) of one row
+// ---------------------------------------------------------------------------
+// Lane pair (2q, 2q + 1) ends with segment h * 16 + q of the chunk for each
+// half h; the chunk statistic combines the 32 segment statistics.
+__global__ void __launch_bounds__(kWarps * 32)
+seg_stats_kernel(const float* __restrict__ Z, int rows, int n, int nseg, int nchunk,
+                 float inv_tau, float2* __restrict__ stats, float2* __restrict__ cstats) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int kr = (lane >> 1) & 15;
+  const long long total = (long long)nchunk * rows;
+  const long long nwarps = (long long)gridDim.x * kWarps;
+  for (long long g = (long long)blockIdx.x * kWarps + (threadIdx.x >> 5); g < total;
+       g += nwarps) {
+    const long long r = g / nchunk;
+    const int c = (int)(g - r * nchunk);
+    const float* z = Z + r * n;
+    float v[2][kGroup];
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int q = 0; q < kGroup; ++q) {
+        const int sg = c * kSeg + h * kGroup + q;
+        const int j = sg * kSeg + lane;
+        v[h][q] = (sg < nseg && j < n) ? __ldcs(z + j) : -INFINITY;
+      }
+    float mk[2], sk[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      mk[h] = warp_reduce_scatter16(v[h], MaxOp{}, lane);
+      float e[kGroup];
+#pragma unroll
+      for (int q = 0; q < kGroup; ++q) {
+        const float mq = __shfl_sync(0xFFFFFFFFu, mk[h], 2 * q);
+        e[q] = v[h][q] > -INFINITY ? expf((v[h][q] - mq) * inv_tau) : 0.f;
+      }
+      sk[h] = warp_reduce_scatter16(e, SumOp{}, lane);
+      const int sg = c * kSeg + h * kGroup + kr;
+      if (!(lane & 1) && sg < nseg) stats[r * nseg + sg] = make_float2(mk[h], sk[h]);
+    }
+    const float Mc = warp_max(fmaxf(mk[0], mk[1]));
+    float Sc = 0.f;
+    if (!(lane & 1))
+      Sc = seg_weight(make_float2(mk[0], sk[0]), Mc, inv_tau) +
+           seg_weight(make_float2(mk[1], sk[1]), Mc, inv_tau);
+    Sc = warp_sum(Sc);
+    if (lane == 0) cstats[r * nchunk + c] = make_float2(Mc, Sc);
+  }
+}
+
+// Chunk statistics from segment statistics (rows of `nseg` entries): a warp
+// per chunk.
+__global__ void __launch_bounds__(kWarps * 32)
+chunk_stats_kernel(const float2* __restrict__ stats, int rows, int nseg, int nchunk,
+                   float inv_tau, float2* __restrict__ cstats) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const long long total = (long long)nchunk * rows;
+  const long long nwarps = (long long)gridDim.x * kWarps;
+  for (long long g = (long long)blockIdx.x * kWarps + (threadIdx.x >> 5); g < total;
+       g += nwarps) {
+    const long long r = g / nchunk;
+    const int c = (int)(g - r * nchunk);
+    const int sg = c * kSeg + lane;
+    const float2 st = sg < nseg ? stats[r * nseg + sg] : make_float2(-INFINITY, 0.f);
+    const float Mc = warp_max(st.x);
+    const float Sc = warp_sum(seg_weight(st, Mc, inv_tau));
+    if (lane == 0) cstats[r * nchunk + c] = make_float2(Mc, Sc);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// warp-level inverse CDF over three levels: chunks, segments, ids
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float warp_incl_scan(float x, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float t = __shfl_up_sync(0xFFFFFFFFu, x, o);
+    if (lane >= o) x += t;
+  }
+  return x;
+}
+
+// Within 32 consecutive weights w (one per lane) find the first lane whose
+// running sum from `before` exceeds target; the last lane with weight if
+// rounding leaves none; lane 0 if all are zero.  Updates `before`.
+__device__ __forceinline__ int scan_pick(float w, float target, float& before, int lane) {
+  const float incl = warp_incl_scan(w, lane);
+  const unsigned hit = __ballot_sync(0xFFFFFFFFu, w > 0.f && target < before + incl);
+  const unsigned nz = __ballot_sync(0xFFFFFFFFu, w > 0.f);
+  const int l = hit ? __ffs(hit) - 1 : (nz ? 31 - __clz(nz) : 0);
+  before += __shfl_sync(0xFFFFFFFFu, incl - w, l);
+  return l;
+}
+
+// Draw with chunk weights cw(c) (c < nchunk), segment weights sw(s)
+// (s < nseg) and id weights ew(j) (j < n): the first id, in ascending order,
+// at which the running weight sum exceeds u * total.  Each lane first sums
+// a contiguous run of chunks; the warp then scans the run that holds the
+// target 32 chunks at a time, then that chunk's segments, then the
+// segment's ids.  Returns the total weight (the draw is void if it is 0);
+// all lanes receive the same j.
+template <class CW, class SW, class EW>
+__device__ __forceinline__ float warp_draw(int nchunk, int nseg, int n, const CW& cw,
+                                           const SW& sw, const EW& ew, float u, int lane,
+                                           int& j_out) {
+  const int per = (nchunk + 31) / 32;
+  const int c0 = min(nchunk, lane * per), c1 = min(nchunk, c0 + per);
+  float local = 0.f;
+  int c = c0;
+  for (; c + 4 <= c1; c += 4) {
+    const float a0 = cw(c), a1 = cw(c + 1), a2 = cw(c + 2), a3 = cw(c + 3);
+    local += a0; local += a1; local += a2; local += a3;
+  }
+  for (; c < c1; ++c) local += cw(c);
+  const float incl = warp_incl_scan(local, lane);
+  const float total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+  const float target = u * total;
+  const unsigned hit = __ballot_sync(0xFFFFFFFFu, local > 0.f && target < incl);
+  const unsigned nz = __ballot_sync(0xFFFFFFFFu, local > 0.f);
+  const int owner = hit ? __ffs(hit) - 1 : (nz ? 31 - __clz(nz) : 0);
+  float before = __shfl_sync(0xFFFFFFFFu, incl - local, owner);
+  const int o0 = __shfl_sync(0xFFFFFFFFu, c0, owner);
+  const int o1 = __shfl_sync(0xFFFFFFFFu, c1, owner);
+  int chunk = -1, last_chunk = o0;
+  float before_last = before;
+  for (int b0 = o0; b0 < o1 && chunk < 0; b0 += 32) {
+    const int cc = b0 + lane;
+    const float w = cc < o1 ? cw(cc) : 0.f;
+    const float inc = warp_incl_scan(w, lane);
+    const unsigned h2 = __ballot_sync(0xFFFFFFFFu, w > 0.f && target < before + inc);
+    const unsigned z2 = __ballot_sync(0xFFFFFFFFu, w > 0.f);
+    if (h2) {
+      const int l = __ffs(h2) - 1;
+      chunk = b0 + l;
+      before += __shfl_sync(0xFFFFFFFFu, inc - w, l);
+    } else {
+      if (z2) {
+        const int l = 31 - __clz(z2);
+        last_chunk = b0 + l;
+        before_last = before + __shfl_sync(0xFFFFFFFFu, inc - w, l);
+      }
+      before += __shfl_sync(0xFFFFFFFFu, inc, 31);
+    }
+  }
+  if (chunk < 0) { chunk = last_chunk; before = before_last; }
+  const int s = chunk * kSeg + lane;
+  const int ls = scan_pick(s < nseg ? sw(s) : 0.f, target, before, lane);
+  const int seg = chunk * kSeg + ls;
+  const int j = seg * kSeg + lane;
+  const int lj = scan_pick(j < n ? ew(j) : 0.f, target, before, lane);
+  j_out = min(seg * kSeg + lj, n - 1);
+  return total;
+}
+
+struct StatsWeight {                    // chunk or segment weight relative to M
+  const float2* st;
+  float M, inv_tau;
+  __device__ float operator()(int s) const { return seg_weight(st[s], M, inv_tau); }
+};
+struct ExpWeight {                      // exp((z_j - M) / tau)
+  const float* z;
+  float M, inv_tau;
+  __device__ float operator()(int j) const { return expf((z[j] - M) * inv_tau); }
+};
+// Residual weight of the rejected position: max(0, p_j - q_j), or with
+// greedy drafts (q == nullptr) p_j with the draft id xi removed.
+struct ResidualWeight {
+  const float* z;
+  const float* q;
+  float M, inv_tau, inv_S;
+  int xi;
+  __device__ float operator()(int j) const {
+    const float p = expf((z[j] - M) * inv_tau) * inv_S;
+    if (q) return fmaxf(0.f, p - q[j]);
+    return j == xi ? 0.f : p;
+  }
+};
+struct ArrayWeight {
+  const float* w;
+  __device__ float operator()(int s) const { return w[s]; }
+};
+
+// row maximum from the chunk statistics
+__device__ __forceinline__ float stats_max(const float2* cst, int nchunk, int lane) {
+  float M = -INFINITY;
+  int c = lane;
+  for (; c + 96 < nchunk; c += 128)
+    M = fmaxf(fmaxf(M, fmaxf(cst[c].x, cst[c + 32].x)), fmaxf(cst[c + 64].x, cst[c + 96].x));
+  for (; c < nchunk; c += 32) M = fmaxf(M, cst[c].x);
+  return warp_max(M);
+}
+
+// ---------------------------------------------------------------------------
+// sampling: one warp per row
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kWarps * 32)
+sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
+                  const float2* __restrict__ stats, int nseg,
+                  const float2* __restrict__ cstats, const int32_t* __restrict__ ids,
+                  float inv_tau, uint64_t seed, uint64_t offset,
+                  int32_t* __restrict__ tokens) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (r >= rows) return;
+  const int nchunk = (nseg + kSeg - 1) / kSeg;
+  const float2* cst = cstats + (int64_t)r * nchunk;
+  const float M = stats_max(cst, nchunk, lane);
+  const StatsWeight cw{cst, M, inv_tau};
+  const StatsWeight sw{stats + (int64_t)r * nseg, M, inv_tau};
+  const ExpWeight ew{Z + (int64_t)r * n, M, inv_tau};
+  const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
+  int j;
+  warp_draw(nchunk, nseg, n, cw, sw, ew, u, lane, j);
+  if (lane == 0) tokens[r] = ids ? ids[j] : j;
+}
+
+// ---------------------------------------------------------------------------
+// verification
+// ---------------------------------------------------------------------------
+__device__ int find_compact(const int32_t* ids, int n, int V, int x) {
+  if (!ids) return (x >= 0 && x < n && x < V) ? x : -1;
+  int lo = 0, hi = n;                   // first position with ids[pos] >= x
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (ids[mid] < x) lo = mid + 1; else hi = mid;
+  }
+  return (lo < n && ids[lo] == x) ? lo : -1;
+}
+
+// First rejected draft of session s (k if all were accepted).
+__device__ __forceinline__ int first_rejection(const int32_t* acc, int s, int k, int lane) {
+  for (int i0 = 0; i0 < k; i0 += 32) {
+    const int i = i0 + lane;
+    const unsigned rej = __ballot_sync(0xFFFFFFFFu, i < k && !acc[(int64_t)s * k + i]);
+    if (rej) return i0 + __ffs(rej) - 1;
+  }
+  return k;
+}
+
+// One warp per target row: the row's softmax maximum and normaliser and,
+// for a draft position, the acceptance test r_i * q_i(x_i) < p_i(x_i).
+__global__ void __launch_bounds__(kWarps * 32)
+verify_rows_kernel(const float* __restrict__ Z, const float2* __restrict__ cstats,
+                   int nchunk, int n, int sessions, int k, const int32_t* __restrict__ ids,
+                   int V, float inv_tau, const int32_t* __restrict__ draft,
+                   const float* __restrict__ q, uint64_t seed, uint64_t offset,
+                   float2* __restrict__ rowMS, int32_t* __restrict__ acc,
+                   int32_t* __restrict__ xis) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int64_t r = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (r >= (int64_t)sessions * (k + 1)) return;
+  const int s = (int)(r / (k + 1)), i = (int)(r - (int64_t)s * (k + 1));
+  const float2* cst = cstats + r * nchunk;
+  const float M = stats_max(cst, nchunk, lane);
+  float S = 0.f;
+  for (int t = lane; t < nchunk; t += 32) S += seg_weight(cst[t], M, inv_tau);
+  S = warp_sum(S);
+  if (lane == 0) {
+    rowMS[r] = make_float2(M, S);
+    if (i < k) {
+      const int64_t di = (int64_t)s * k + i;
+      const int xi = find_compact(ids, n, V, draft[di]);
+      const float px = xi >= 0 ? expf((Z[r * n + xi] - M) * inv_tau) / S : 0.f;
+      const float qx = xi >= 0 ? (q ? q[di * n + xi] : 1.f) : 0.f;
+      const float rr = philox_uniform(seed, (uint32_t)s, (uint32_t)(1 + i), offset);
+      acc[di] = rr * qx < px ? 1 : 0;
+      xis[di] = xi;
+    }
+  }
+}
+
+// Segment and chunk weights of the residual distribution at each session's
+// first rejection: a warp per (session, chunk).
+__global__ void __launch_bounds__(kWarps * 32)
+verify_residual_kernel(const float* __restrict__ Z, int n, int nseg, int nchunk,
+                       int sessions, int k, const float* __restrict__ q, float inv_tau,
+                       const float2* __restrict__ rowMS, const int32_t* __restrict__ acc,
+                       const int32_t* __restrict__ xis, float* __restrict__ resw,
+                       float* __restrict__ resc) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int kr = (lane >> 1) & 15;
+  const long long total = (long long)nchunk * sessions;
+  const long long nwarps = (long long)gridDim.x * kWarps;
+  for (long long g = (long long)blockIdx.x * kWarps + (threadIdx.x >> 5); g < total;
+       g += nwarps) {
+    const int s = (int)(g / nchunk);
+    const int c = (int)(g - (long long)s * nchunk);
+    const int i = first_rejection(acc, s, k, lane);
+    if (i == k) continue;               // the bonus draw uses the statistics
+    const int64_t r = (int64_t)s * (k + 1) + i;
+    const int64_t di = (int64_t)s * k + i;
+    const float2 ms = rowMS[r];
+    const ResidualWeight rw{Z + r * n, q ? q + di * n : nullptr, ms.x, inv_tau,
+                            1.f / ms.y, xis[di]};
+    float csum = 0.f;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float v[kGroup];
+#pragma unroll
+      for (int t = 0; t < kGroup; ++t) {
+        const int sg = c * kSeg + h * kGroup + t;
+        const int j = sg * kSeg + lane;
+        v[t] = (sg < nseg && j < n) ? rw(j) : 0.f;
+      }
+      const float w = warp_reduce_scatter16(v, SumOp{}, lane);
+      const int sg = c * kSeg + h * kGroup + kr;
+      if (!(lane & 1) && sg < nseg) resw[(int64_t)s * nseg + sg] = w;
+      if (!(lane & 1)) csum += w;
+    }
+    csum = warp_sum(csum);
+    if (lane == 0) resc[(int64_t)s * nchunk + c] = csum;
+  }
+}
+
+// One warp per session: the draw, from the residual (or, if that is all
+// zero, from p_i) at the first rejection, else the bonus draw from p_k.
+__global__ void __launch_bounds__(kWarps * 32)
+verify_draw_kernel(const float* __restrict__ Z, int n, const float2* __restrict__ stats,
+                   const float2* __restrict__ cstats, int nseg, int nchunk, int sessions,
+                   int k, const int32_t* __restrict__ ids, const float* __restrict__ q,
+                   float inv_tau, uint64_t seed, uint64_t offset,
+                   const float2* __restrict__ rowMS, const int32_t* __restrict__ acc,
+                   const int32_t* __restrict__ xis, const float* __restrict__ resw,
+                   const float* __restrict__ resc, int32_t* __restrict__ n_acc,
+                   int32_t* __restrict__ next_token) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int s = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (s >= sessions) return;
+  const int i = first_rejection(acc, s, k, lane);
+  const int64_t r = (int64_t)s * (k + 1) + i;
+  const float2 ms = rowMS[r];
+  const float u = philox_uniform(seed, (uint32_t)s, (uint32_t)(1 + k), offset);
+  int j = 0;
+  float tot = 0.f;
+  if (i < k) {
+    const int64_t di = (int64_t)s * k + i;
+    const ArrayWeight cw{resc + (int64_t)s * nchunk};
+    const ArrayWeight sw{resw + (int64_t)s * nseg};
+    const ResidualWeight rw{Z + r * n, q ? q + di * n : nullptr, ms.x, inv_tau,
+                            1.f / ms.y, xis[di]};
+    tot = warp_draw(nchunk, nseg, n, cw, sw, rw, u, lane, j);
+  }
+  if (!(tot > 0.f)) {
+    const StatsWeight cw{cstats + r * nchunk, ms.x, inv_tau};
+    const StatsWeight sw{stats + r * nseg, ms.x, inv_tau};
+    const ExpWeight ew{Z + r * n, ms.x, inv_tau};
+    warp_draw(nchunk, nseg, n, cw, sw, ew, u, lane, j);
+  }
+  if (lane == 0) {
+    n_acc[s] = i;
+    next_token[s] = ids ? ids[j] : j;
+  }
+}
+
+int stats_grid(long long warps_of_work, int sm_count) {
+  long long b = (warps_of_work + kWarps - 1) / kWarps;
+  const long long cap = (long long)(sm_count > 0 ? sm_count : 148) * 8;
+  if (b > cap) b = cap;
+  return (int)(b < 1 ? 1 : b);
+}
+
+size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+
+}  // namespace
+
+int sample_max_n() { return kMaxN; }
+int verify_max_k() { return kMaxK; }
+int seg_count(int n) { return (n + kSeg - 1) / kSeg; }
+int chunk_count(int nseg) { return (nseg + kSeg - 1) / kSeg; }
+
+cudaError_t launch_seg_stats(const float* Z, int rows, int n, float inv_tau,
+                             float2* stats, float2* cstats, int sm_count,
+                             cudaStream_t st) {
+  const int nseg = seg_count(n), nchunk = chunk_count(nseg);
+  return launch_pdl(seg_stats_kernel,
+                    dim3(stats_grid((long long)rows * nchunk, sm_count)),
+                    dim3(kWarps * 32), 0, st, Z, rows, n, nseg, nchunk, inv_tau, stats,
+                    cstats);
+}
+
+cudaError_t launch_chunk_stats(const float2* stats, int rows, int nseg, float inv_tau,
+                               float2* cstats, int sm_count, cudaStream_t st) {
+  const int nchunk = chunk_count(nseg);
+  return launch_pdl(chunk_stats_kernel,
+                    dim3(stats_grid((long long)rows * nchunk, sm_count)),
+                    dim3(kWarps * 32), 0, st, stats, rows, nseg, nchunk, inv_tau, cstats);
+}
+
+cudaError_t launch_sample_segments(const float* Z, int rows, int n, const float2* stats,
+                                   int nseg, const float2* cstats, const int32_t* ids,
+                                   float inv_tau, uint64_t seed, uint64_t offset,
+                                   int32_t* tokens, cudaStream_t st) {
+  return launch_pdl(sample_seg_kernel, dim3((rows + kWarps - 1) / kWarps),
+                    dim3(kWarps * 32), 0, st, Z, rows, n, stats, nseg, cstats, ids, inv_tau,
+                    seed, offset, tokens);
+}
+
+// Scratch: stats [R][nseg] float2 | chunk stats [R][nchunk] float2 | rowMS
+// [R] float2 | acc, xis [S*k] int32 | residual segment weights [S][nseg] |
+// residual chunk weights [S][nchunk], with R = S * (k + 1).
+size_t verify_scratch_bytes(int sessions, int k, int n) {
+  const size_t R = (size_t)sessions * (k + 1), nseg = (size_t)seg_count(n),
+               nchunk = (size_t)chunk_count((int)nseg);
+  return align256(R * nseg * 8) + align256(R * nchunk * 8) + align256(R * 8) +
+         2 * align256((size_t)sessions * k * 4) + align256((size_t)sessions * nseg * 4) +
+         align256((size_t)sessions * nchunk * 4);
+}
+
+cudaError_t launch_verify(const float* Z, int sessions, int k, int n, const int32_t* ids,
+                          int V, float inv_tau, const int32_t* draft, const float* q,
+                          uint64_t seed, uint64_t offset, int32_t* n_acc,
+                          int32_t* next_token, void* scratch, int sm_count,
+                          cudaStream_t st) {
+  const int R = sessions * (k + 1), nseg = seg_count(n), nchunk = chunk_count(nseg);
+  char* p = static_cast<char*>(scratch);
+  float2* stats = reinterpret_cast<float2*>(p);
+  p += align256((size_t)R * nseg * 8);
+  float2* cstats = reinterpret_cast<float2*>(p);
+  p += align256((size_t)R * nchunk * 8);
+  float2* rowMS = reinterpret_cast<float2*>(p);
+  p += align256((size_t)R * 8);
+  int32_t* acc = reinterpret_cast<int32_t*>(p);
+  p += align256((size_t)sessions * k * 4);
+  int32_t* xis = reinterpret_cast<int32_t*>(p);
+  p += align256((size_t)sessions * k * 4);
+  float* resw = reinterpret_cast<float*>(p);
+  p += align256((size_t)sessions * nseg * 4);
+  float* resc = reinterpret_cast<float*>(p);
+  cudaError_t e = launch_seg_stats(Z, R, n, inv_tau, stats, cstats, sm_count, st);
+  if (e == cudaSuccess)
+    e = launch_pdl(verify_rows_kernel, dim3((R + kWarps - 1) / kWarps), dim3(kWarps * 32), 0,
+                   st, Z, (const float2*)cstats, nchunk, n, sessions, k, ids, V, inv_tau,
+                   draft, q, seed, offset, rowMS, acc, xis);
+  if (e == cudaSuccess)
+    e = launch_pdl(verify_residual_kernel,
+                   dim3(stats_grid((long long)sessions * nchunk, sm_count)),
+                   dim3(kWarps * 32), 0, st, Z, n, nseg, nchunk, sessions, k, q, inv_tau,
+                   (const float2*)rowMS, (const int32_t*)acc, (const int32_t*)xis, resw,
+                   resc);
+  if (e == cudaSuccess)
+    e = launch_pdl(verify_draw_kernel, dim3((sessions + kWarps - 1) / kWarps),
+                   dim3(kWarps * 32), 0, st, Z, n, (const float2*)stats,
+                   (const float2*)cstats, nseg, nchunk, sessions, k, ids, q, inv_tau, seed,
+                   offset, (const float2*)rowMS, (const int32_t*)acc, (const int32_t*)xis,
+                   (const float*)resw, (const float*)resc, n_acc, next_token);
+  return e;
+}
+
+}  // namespace sph

@@ -27,10 +27,13 @@
 // them in CTA order (deterministic).  No CTA ever waits on another.
 //
 // Warp roles: warp 0 issues the TMA copies, warp 1 owns TMEM and issues
-// tcgen05.mma (one thread), warps 2-5 drain the double-buffered accumulator
-// (tcgen05.ld) and run the fused epilogue.  Every wait is bounded; a wait
-// that gives up sets the context's error word and the CTA winds down after
-// its copies and MMAs have landed.
+// tcgen05.mma (one thread), warps 2-9 drain the double-buffered accumulator
+// (tcgen05.ld) and run the fused epilogue -- two warps per TMEM lane
+// quadrant, so that the epilogue's dependent shuffle / exp chains of one
+// warp overlap with the other's; with fp8 weights warps 10-13 convert the
+// e4m3 A tiles.  Every wait is bounded; a wait that gives up sets the
+// context's error word and the CTA winds down after its copies and MMAs
+// have landed.
 //
 // Epilogues: cloud = + bias, optional unclipped store, clip, store, row |max|
 // (atomicMax); endpoint = + code * row_scale (Eq. 13), store z, and the
@@ -55,8 +58,10 @@ constexpr int kMaxBN = 256;
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
 
-constexpr int kThreads = 192;
-constexpr int kThreadsFp8 = 320;     // + four converter warps (fp8 weights)
+constexpr int kEpiWarps = 8;         // two per TMEM lane quadrant
+constexpr int kEpiGroups = kEpiWarps / 4;
+constexpr int kThreads = 64 + 32 * kEpiWarps;       // producer, MMA, epilogue
+constexpr int kThreadsFp8 = kThreads + 128;         // + four converter warps (fp8)
 constexpr int kMaxBNFp8 = 128;       // h rows per block with fp8 weights
 constexpr int kBoxHeights = 8;       // row boxes of 1, 2, 4, ..., 128 rows
 
@@ -114,47 +119,41 @@ struct Segments {
   }
 };
 
-// Reduce 16 per-lane values over the 32 lanes of a warp, one result per
-// value index: a butterfly that halves the array at every exchange (16
-// shuffles in all).  Lane l ends with the reduction of index
-// (l >> 1) & 15; lanes l and l ^ 1 hold the same result.
-template <class Op>
-__device__ __forceinline__ float warp_reduce_scatter16(const float (&v)[16], Op op, int lane) {
-  float a8[8], a4[4], a2[2];
-  const bool b16 = lane & 16, b8 = lane & 8, b4 = lane & 4, b2 = lane & 2;
+
+// Endpoint payload of one 16-row chunk at this lane's id column j: the int8
+// codes of rows row0..row0+15 and, in lane q < 16, the scale of row row0 + q.
+// Addresses are clamped into the arrays and every load is issued, so the 16
+// loads go out back to back and can be started a chunk ahead of their use.
+struct Payload {
+  int c[16];
+  float s;
+};
+__device__ __forceinline__ void load_payload(const TcParams& p, int row0, int j, int lane,
+                                             Payload& pl) {
+  const int8_t* col = p.codes + min(j, p.n - 1);
 #pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const float keep = b16 ? v[k + 8] : v[k], give = b16 ? v[k] : v[k + 8];
-    a8[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 16));
+  for (int q = 0; q < 16; ++q) pl.c[q] = __ldg(col + (int64_t)min(row0 + q, p.R - 1) * p.n);
+  pl.s = __ldg(p.row_scale + min(row0 + (lane & 15), p.R - 1));
+}
+// Warm L2 with the codes of rows row0..row0+nrows-1 at the 32 ids from j0.
+__device__ __forceinline__ void prefetch_codes(const TcParams& p, int row0, int nrows, int j0,
+                                               int lane) {
+  if (j0 >= p.n) return;
+  const int8_t* col = p.codes + j0;
+  const int last = min(31, p.n - 1 - j0);
+  for (int r = row0 + lane; r < min(row0 + nrows, p.R); r += 32) {
+    const int8_t* a = col + (int64_t)r * p.n;
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(a));
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(a + last));
   }
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const float keep = b8 ? a8[k + 4] : a8[k], give = b8 ? a8[k] : a8[k + 4];
-    a4[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 8));
-  }
-#pragma unroll
-  for (int k = 0; k < 2; ++k) {
-    const float keep = b4 ? a4[k + 2] : a4[k], give = b4 ? a4[k] : a4[k + 2];
-    a2[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 4));
-  }
-  const float keep = b2 ? a2[1] : a2[0], give = b2 ? a2[0] : a2[1];
-  float r = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 2));
-  return op(r, __shfl_xor_sync(0xFFFFFFFFu, r, 1));
 }
 
-struct MaxOp {
-  __device__ float operator()(float a, float b) const { return fmaxf(a, b); }
-};
-struct SumOp {
-  __device__ float operator()(float a, float b) const { return a + b; }
-};
-
 // Epilogue of 16 accumulator columns (hidden-state rows row0..row0+15) for
-// this lane's vocabulary column j.
+// this lane's vocabulary column j (endpoint: with the chunk's payload).
 template <int EPI>
 __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)[16],
                                              int row0, int j, bool vj, int id,
-                                             int lane, int seg) {
+                                             int lane, int seg, const Payload& pay) {
   const int kr = (lane >> 1) & 15;               // the row this lane reduces
   if constexpr (EPI == EPI_CLOUD) {
     const float b = (vj && p.bias) ? p.bias[id] : 0.f;
@@ -179,15 +178,11 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
     if (!(lane & 1) && row0 + kr < p.R && mr > 0.f)
       atomicMax(&p.rowmax[row0 + kr], __float_as_uint(mr));
   } else {
-    // all payload loads first, then the stores (the stores could alias the
-    // loads as far as the compiler knows, which would serialise them)
     float z[16];
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
-      const int r = row0 + q;
-      z[q] = (vj && r < p.R)
-                 ? v[q] + (float)__ldg(p.codes + (int64_t)r * p.n + j) * __ldg(p.row_scale + r)
-                 : -INFINITY;
+      const float sq = __shfl_sync(0xFFFFFFFFu, pay.s, q);
+      z[q] = (vj && row0 + q < p.R) ? v[q] + (float)pay.c[q] * sq : -INFINITY;
     }
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
@@ -241,7 +236,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(&tfull[a], 1);
-      ptx::mbar_init(&tempty[a], 4);
+      ptx::mbar_init(&tempty[a], kEpiWarps);
     }
     ptx::mbar_init(drain, 1);
     *s_abort = 0;
@@ -432,9 +427,12 @@ tc_kernel(const __grid_constant__ WMaps wm,
       ptx::umma_commit(drain);
       ptx::mbar_wait(drain, 0, kDrainLimit);
     }
-  } else if (warp < 6) {
+  } else if (warp < 2 + kEpiWarps) {
     // ------------------------------------------------------------ epilogue
+    // A warp may only read the TMEM lanes of its quadrant (warp index mod
+    // 4); the two warps of a quadrant take alternate 16-column chunks.
     const int quad = warp & 3;
+    const int grp = (warp - 2) >> 2;
     const int i = quad * 32 + lane;              // vocabulary row in the tile
     ptx::griddep_wait();
     Segments sg{it0, it1, p.KB};
@@ -442,6 +440,15 @@ tc_kernel(const __grid_constant__ WMaps wm,
     int si = 0, tile, kb0, kb1;
     while (sg.next(tile, kb0, kb1)) {
       const int acc = si & 1;
+      const int rb = tile / p.NT, t = tile - rb * p.NT;
+      const bool whole = kb0 == 0 && kb1 == p.KB;
+      Payload pay;
+      if constexpr (EPI == EPI_ENDPOINT) {
+        // the payload does not depend on the accumulator: start on it
+        // while the tile's MMAs run
+        prefetch_codes(p, rb * BN + grp * (BN / 2), BN / 2, t * kTileM + quad * 32, lane);
+        if (whole && grp < BN / 16) load_payload(p, rb * BN + grp * 16, t * kTileM + i, lane, pay);
+      }
       int ok = 1;
       if (lane == 0) ok = !*s_abort && ptx::mbar_wait(&tfull[acc], fph[acc], limit);
       ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
@@ -451,21 +458,23 @@ tc_kernel(const __grid_constant__ WMaps wm,
       }
       fph[acc] ^= 1;
       ptx::tc_fence_after();
-      const int rb = tile / p.NT, t = tile - rb * p.NT;
       const int j = t * kTileM + i;
       const bool vj = j < p.n;
       const int id = vj ? (GATHER ? p.ids[j] : j) : 0;
       const int seg = t * 4 + quad;
-      const bool whole = kb0 == 0 && kb1 == p.KB;
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
       // a CTA's split tiles can only be its first and its last segment:
       // slot 2c holds the first, 2c+1 the last
       float* Pt = p.P + (size_t)(2 * blockIdx.x + (si == 0 ? 0 : 1)) * BN * kTileM;
-      for (int ch = 0; ch < BN / 16; ++ch) {
+      for (int ch = grp; ch < BN / 16; ch += kEpiGroups) {
         float v[16];
         ptx::tmem_ld16(taddr + ch * 16, v);
         if (whole) {
-          finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg);
+          Payload nxt;
+          if (EPI == EPI_ENDPOINT && ch + kEpiGroups < BN / 16)
+            load_payload(p, rb * BN + (ch + kEpiGroups) * 16, j, lane, nxt);
+          finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg, pay);
+          if constexpr (EPI == EPI_ENDPOINT) pay = nxt;
         } else {
 #pragma unroll
           for (int q = 0; q < 16; ++q) Pt[(size_t)(ch * 16 + q) * kTileM + i] = v[q];
@@ -475,11 +484,13 @@ tc_kernel(const __grid_constant__ WMaps wm,
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(&tempty[acc]);
       if (!whole) {
-        // split tile: this warp's 32 vocabulary rows are finished by the
-        // last warp (over all contributing CTAs) of the same quadrant
+        // split tile: this warp's 32 vocabulary rows x its chunks are
+        // finished by the last warp (over all contributing CTAs) of the same
+        // quadrant and chunk group
         __threadfence();
         int old = 0;
-        if (lane == 0) old = atomicAdd(&p.counters[tile * 4 + quad], 1);
+        const int cnt = (tile * 4 + quad) * kEpiGroups + grp;
+        if (lane == 0) old = atomicAdd(&p.counters[cnt], 1);
         old = __shfl_sync(0xFFFFFFFFu, old, 0);
         const int c0 = (int)cta_of((long long)tile * p.KB, p.T, gridDim.x);
         const int c1 = (int)cta_of((long long)tile * p.KB + p.KB - 1, p.T, gridDim.x);
@@ -499,7 +510,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
             const int slot = c == 0 ? 2 * c0 + (c0_first ? 0 : 1) : 2 * (c0 + (c < C ? c : 0));
             ps[c] = p.P + (size_t)slot * BN * kTileM + i;
           }
-          for (int ch = 0; ch < BN / 16; ++ch) {
+          for (int ch = grp; ch < BN / 16; ch += kEpiGroups) {
+            if constexpr (EPI == EPI_ENDPOINT) load_payload(p, rb * BN + ch * 16, j, lane, pay);
             float v[16];
 #pragma unroll
             for (int q = 0; q < 16; ++q) v[q] = __ldcg(ps[0] + (size_t)(ch * 16 + q) * kTileM);
@@ -516,9 +528,9 @@ tc_kernel(const __grid_constant__ WMaps wm,
 #pragma unroll
               for (int q = 0; q < 16; ++q) v[q] += __ldcg(pc + (size_t)(ch * 16 + q) * kTileM);
             }
-            finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg);
+            finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg, pay);
           }
-          if (lane == 0) p.counters[tile * 4 + quad] = 0;
+          if (lane == 0) p.counters[cnt] = 0;
         }
       }
       ++si;
@@ -532,7 +544,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     // magnitude bits shifted up by 7 -- exactly the e4m3 value times 2^-8,
     // subnormals included -- stores the 128-byte-swizzled f16 rows, fences
     // the async proxy and arrives on the stage barrier.
-    const int gw = warp - 6;
+    const int gw = warp - (2 + kEpiWarps);
     const int c = lane & 3;                      // 16-byte chunk of a 64-byte row slice
     const int r0 = lane >> 2;                    // rows r0 + 8m, m = 0..15
     ptx::griddep_wait();                         // (inputs only; keeps ordering simple)
@@ -649,78 +661,6 @@ __global__ void split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R,
     counters[t] = 0;
 }
 
-// ---------------------------------------------------------------------------
-// sampling from the segment statistics: one warp per row
-// ---------------------------------------------------------------------------
-__global__ void sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
-                                  const float2* __restrict__ stats, int nseg,
-                                  const int32_t* __restrict__ ids, float inv_tau,
-                                  uint64_t seed, uint64_t offset,
-                                  int32_t* __restrict__ tokens) {
-  ptx::griddep_wait();
-  ptx::griddep_launch_dependents();
-  const int lane = threadIdx.x & 31;
-  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (r >= rows) return;
-  const float2* st = stats + (int64_t)r * nseg;
-  float M = -INFINITY;
-  for (int s = lane; s < nseg; s += 32) M = fmaxf(M, st[s].x);
-  M = warp_max(M);
-  // segment weights in ascending order: lane owns segments [s0, s1)
-  const int per = (nseg + 31) / 32;
-  const int s0 = min(nseg, lane * per), s1 = min(nseg, s0 + per);
-  float local = 0.f;
-  for (int s = s0; s < s1; ++s) {
-    const float2 v = st[s];
-    local += v.y > 0.f ? v.y * expf((v.x - M) * inv_tau) : 0.f;
-  }
-  float incl = local;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const float t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-    if (lane >= o) incl += t;
-  }
-  const float excl = incl - local;
-  const float total = __shfl_sync(0xFFFFFFFFu, incl, 31);
-  const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
-  const float target = u * total;
-  const unsigned hit = __ballot_sync(0xFFFFFFFFu, local > 0.f && target >= excl && target < incl);
-  const unsigned nzl = __ballot_sync(0xFFFFFFFFu, local > 0.f);
-  const int owner = hit ? __ffs(hit) - 1 : (nzl ? 31 - __clz(nzl) : 0);
-  int sstar = -1;
-  float before = 0.f;
-  if (lane == owner) {
-    float run = excl, before_last = excl;
-    int last_nz = -1;
-    for (int s = s0; s < s1; ++s) {
-      const float2 v = st[s];
-      const float w = v.y > 0.f ? v.y * expf((v.x - M) * inv_tau) : 0.f;
-      if (w > 0.f) { last_nz = s; before_last = run; }
-      if (w > 0.f && target < run + w) { sstar = s; before = run; break; }
-      run += w;
-    }
-    if (sstar < 0) { sstar = last_nz >= 0 ? last_nz : s0; before = before_last; }
-  }
-  sstar = __shfl_sync(0xFFFFFFFFu, sstar, owner);
-  before = __shfl_sync(0xFFFFFFFFu, before, owner);
-  // inside the 32-id segment: one id per lane
-  const int j = sstar * 32 + lane;
-  const float w = j < n ? expf((Z[(int64_t)r * n + j] - M) * inv_tau) : 0.f;
-  float winc = w;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const float t = __shfl_up_sync(0xFFFFFFFFu, winc, o);
-    if (lane >= o) winc += t;
-  }
-  const float t2 = target - before;
-  const unsigned h2 = __ballot_sync(0xFFFFFFFFu, w > 0.f && t2 < winc);
-  const unsigned nz2 = __ballot_sync(0xFFFFFFFFu, w > 0.f);
-  const int l2 = h2 ? __ffs(h2) - 1 : (nz2 ? 31 - __clz(nz2) : 0);
-  if (lane == l2) {
-    const int jj = min(sstar * 32 + l2, n - 1);
-    tokens[r] = ids ? ids[jj] : jj;
-  }
-}
 
 // ---------------------------------------------------------------------------
 // host side
@@ -811,7 +751,7 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   // split tiles exist only when a CTA's range does not cover whole tiles
   const bool splits = !pl.whole_tiles && (pl.T % pl.G != 0 || (pl.T / pl.G) % pl.KB != 0);
   pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * kTileM * 4) : 0;
-  pl.cnt_bytes = align256((size_t)tiles * 4 * sizeof(int));
+  pl.cnt_bytes = align256((size_t)tiles * 4 * kEpiGroups * sizeof(int));
   pl.stats_bytes = endpoint ? align256((size_t)rows * pl.NT * 4 * sizeof(float2)) : 0;
   pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
   pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256;
@@ -852,7 +792,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
     if (blocks > 4096) blocks = 4096;
     if (blocks < 1) blocks = 1;
     cudaError_t e = launch_pdl(split_h_kernel, dim3(blocks), dim3(256), 0, st, g.h, g.ld_h,
-                               g.rows, g.K, pl.Rp, pl.Kp, pl.hilo, Hs, counters, tiles * 4,
+                               g.rows, g.K, pl.Rp, pl.Kp, pl.hilo, Hs, counters, tiles * 4 * kEpiGroups,
                                g.epilogue == EPI_CLOUD ? g.rowmax : (unsigned*)nullptr,
                                fp8 ? 1 : 0, g.act_bf16);
     if (e != cudaSuccess) return e;
@@ -912,16 +852,18 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
 }
 
 cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPlan& pl,
-                                     const void* scratch, const int32_t* ids,
-                                     float inv_tau, uint64_t seed, uint64_t offset,
-                                     int32_t* tokens, cudaStream_t st) {
+                                     const void* scratch, float2* cstats,
+                                     const int32_t* ids, float inv_tau, uint64_t seed,
+                                     uint64_t offset, int sm_count, int32_t* tokens,
+                                     cudaStream_t st) {
   const char* sc = static_cast<const char*>(scratch);
   const float2* stats =
       reinterpret_cast<const float2*>(sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes);
-  const int warps = 8;
-  const int blocks = (rows + warps - 1) / warps;
-  return launch_pdl(sample_seg_kernel, dim3(blocks), dim3(warps * 32), 0, st, Z, rows, n,
-                    stats, pl.NT * 4, ids, inv_tau, seed, offset, tokens);
+  const int nseg = pl.NT * 4;
+  cudaError_t e = launch_chunk_stats(stats, rows, nseg, inv_tau, cstats, sm_count, st);
+  if (e != cudaSuccess) return e;
+  return launch_sample_segments(Z, rows, n, stats, nseg, cstats, ids, inv_tau, seed, offset,
+                                tokens, st);
 }
 
 }  // namespace sph

@@ -141,8 +141,18 @@ size_t partial_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_
   return align_up((size_t)rows * n * 4, 256) + align_up((size_t)rows * 4, 256) +
          tc_bytes(ctx, rows, n, K, act_bf16, w_dtype, 0);
 }
+// fused logits, then the tensor-core scratch (which holds the segment
+// statistics) or, on the CUDA-core path, the segment statistics alone
 size_t fuse_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K) {
-  return align_up((size_t)rows * n * 4, 256) + tc_bytes(ctx, rows, n, K, 0, sph::W_BF16, 1);
+  // chunk statistics: at most one per 1024 ids of the tensor-core tiling
+  const size_t cstats = align_up((size_t)rows * (n / 1024 + 2) * 8, 256);
+  const size_t stats = align_up((size_t)rows * sph::seg_count((int)n) * 8, 256);
+  const size_t tc = tc_bytes(ctx, rows, n, K, 0, sph::W_BF16, 1);
+  return align_up((size_t)rows * n * 4, 256) + cstats + (tc > stats ? tc : stats);
+}
+// verification over `rows` = sessions * (k + 1) target rows, for any split
+size_t verify_reserve_bytes(int64_t rows, int64_t n) {
+  return sph::verify_scratch_bytes((int)rows, 0, (int)n) + 2 * align_up((size_t)rows * 4, 256);
 }
 
 bool finite_pos(float x) { return std::isfinite(x) && x > 0.f; }
@@ -341,6 +351,8 @@ sph_status sph_reserve(sph_ctx* ctx, int64_t max_rows, int64_t max_n_keep,
   }
   const size_t f = fuse_scratch_bytes(ctx, max_rows, max_n_keep, max_d);
   if (f > need) need = f;
+  const size_t v = verify_reserve_bytes(max_rows, max_n_keep);
+  if (v > need) need = v;
   return ensure_scratch(ctx, need);
 }
 
@@ -500,6 +512,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   Carve c(ctx->scratch);
   float* Z = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
   if (fused_logits_out) Z = fused_logits_out;
+  float2* cstats = static_cast<float2*>(c.take((size_t)rows * (n_keep / 1024 + 2) * 8));
   sph::GatherGemm gg{};
   gg.h = h_local; gg.ld_h = ld_hl; gg.rows = (int)rows;
   gg.W = W_l; gg.ld_w = ld_wl; gg.V = V; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
@@ -518,18 +531,26 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
     if (st) return st;
     return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                            return sph::launch_sample_from_stats(
-                               Z, (int)rows, (int)n_keep, pl, tcs, keep_ids,
-                               1.0f / temperature, seed, offset, tokens, ctx->stream);
+                               Z, (int)rows, (int)n_keep, pl, tcs, cstats, keep_ids,
+                               1.0f / temperature, seed, offset, ctx->sm_count, tokens,
+                               ctx->stream);
                          }), "sample launch");
   }
+  float2* stats = static_cast<float2*>(c.take((size_t)rows * sph::seg_count((int)n_keep) * 8));
   st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                        return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
                      }), "gemv launch");
   if (st) return st;
   return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
-                         return sph::launch_sample(Z, (int)rows, (int)n_keep, keep_ids,
-                                                   1.0f / temperature, seed, offset,
-                                                   tokens, ctx->stream);
+                         cudaError_t e = sph::launch_seg_stats(Z, (int)rows, (int)n_keep,
+                                                               1.0f / temperature, stats,
+                                                               cstats, ctx->sm_count,
+                                                               ctx->stream);
+                         if (e != cudaSuccess) return e;
+                         return sph::launch_sample_segments(
+                             Z, (int)rows, (int)n_keep, stats, sph::seg_count((int)n_keep),
+                             cstats, keep_ids, 1.0f / temperature, seed, offset, tokens,
+                             ctx->stream);
                        }), "sample launch");
 }
 
@@ -544,12 +565,18 @@ sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
   if (!target_logits || !draft_tokens || !n_accepted || !next_token)
     return fail(ctx, SPH_ERR_INVALID_ARG, "target_logits, draft_tokens, n_accepted and next_token must be non-NULL");
   if (sessions < 1 || sessions > (1 << 20)) return fail(ctx, SPH_ERR_INVALID_ARG, "sessions out of [1, 2^20]");
-  if (k < 1 || k > 64) return fail(ctx, SPH_ERR_INVALID_ARG, "k must be in [1, 64]");
+  if (k < 1 || k > sph::verify_max_k())
+    return fail(ctx, SPH_ERR_INVALID_ARG, "k must be in [1, %d]", sph::verify_max_k());
+  if (sessions * (k + 1) > (1 << 20))
+    return fail(ctx, SPH_ERR_INVALID_ARG, "sessions * (k + 1) above 2^20 target rows");
   if (n_keep < 1 || n_keep > INT32_MAX) return fail(ctx, SPH_ERR_INVALID_ARG, "n_keep must be >= 1");
   if (!finite_pos(temperature)) return fail(ctx, SPH_ERR_INVALID_ARG, "temperature must be finite and > 0");
   if (n_keep > sph::sample_max_n()) return fail(ctx, SPH_ERR_UNSUPPORTED, "n_keep above %d", sph::sample_max_n());
   DeviceGuard g(ctx->device);
   if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
+  sph_status st = ensure_scratch(
+      ctx, sph::verify_scratch_bytes((int)sessions, (int)k, (int)n_keep));
+  if (st) return st;
   // without an id list the compact index is the vocabulary id itself
   const int V = keep_ids ? INT32_MAX : (int)n_keep;
   return launch_status(ctx, traced(ctx, SPH_PROF_VERIFY, [&] {
@@ -557,7 +584,8 @@ sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
                                                    (int)n_keep, keep_ids, V,
                                                    1.0f / temperature, draft_tokens,
                                                    draft_probs, seed, offset,
-                                                   n_accepted, next_token, ctx->stream);
+                                                   n_accepted, next_token, ctx->scratch,
+                                                   ctx->sm_count, ctx->stream);
                        }), "verify launch");
 }
 

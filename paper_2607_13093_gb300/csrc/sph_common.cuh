@@ -94,6 +94,41 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return warp_sum(v);
 }
 
+// Reduce 16 per-lane values over the 32 lanes of a warp, one result per
+// value index: a butterfly that halves the array at every exchange (16
+// shuffles in all).  Lane l ends with the reduction of index
+// (l >> 1) & 15; lanes l and l ^ 1 hold the same result.
+template <class Op>
+__device__ __forceinline__ float warp_reduce_scatter16(const float (&v)[16], Op op, int lane) {
+  float a8[8], a4[4], a2[2];
+  const bool b16 = lane & 16, b8 = lane & 8, b4 = lane & 4, b2 = lane & 2;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const float keep = b16 ? v[k + 8] : v[k], give = b16 ? v[k] : v[k + 8];
+    a8[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 16));
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float keep = b8 ? a8[k + 4] : a8[k], give = b8 ? a8[k] : a8[k + 4];
+    a4[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 8));
+  }
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const float keep = b4 ? a4[k + 2] : a4[k], give = b4 ? a4[k] : a4[k + 2];
+    a2[k] = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 4));
+  }
+  const float keep = b2 ? a2[1] : a2[0], give = b2 ? a2[0] : a2[1];
+  float r = op(keep, __shfl_xor_sync(0xFFFFFFFFu, give, 2));
+  return op(r, __shfl_xor_sync(0xFFFFFFFFu, r, 1));
+}
+
+struct MaxOp {
+  __device__ float operator()(float a, float b) const { return fmaxf(a, b); }
+};
+struct SumOp {
+  __device__ float operator()(float a, float b) const { return a + b; }
+};
+
 // Non-negative floats order like their bit patterns, so a row maximum of
 // |y| can be kept as an unsigned atomicMax.
 __device__ __forceinline__ void atomic_max_nonneg(unsigned int* addr, float v) {

@@ -98,29 +98,51 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,
                       long long spin_limit, cudaStream_t st);
 // One inverse-CDF draw per row from the segment statistics that an endpoint
-// launch_tc left in `scratch` (one warp per row).
+// launch_tc left in `scratch`; `cstats` receives rows * chunk_count(4 * NT)
+// chunk statistics on the way.
 cudaError_t launch_sample_from_stats(const float* Z, int rows, int n,
                                      const TcPlan& plan, const void* scratch,
-                                     const int32_t* ids, float inv_tau,
-                                     uint64_t seed, uint64_t offset,
-                                     int32_t* tokens, cudaStream_t st);
+                                     float2* cstats, const int32_t* ids,
+                                     float inv_tau, uint64_t seed, uint64_t offset,
+                                     int sm_count, int32_t* tokens, cudaStream_t st);
 
 // codes/row_scale from the clipped partials and their row maxima
 cudaError_t launch_quantize(const float* Y, const unsigned* rowmax, int rows,
                             int n, int8_t* codes, float* row_scale,
                             cudaStream_t st);
 
-// one inverse-CDF draw per row of Z (fp32 [rows, n])
-cudaError_t launch_sample(const float* Z, int rows, int n,
-                          const int32_t* ids, float inv_tau, uint64_t seed,
-                          uint64_t offset, int32_t* tokens, cudaStream_t st);
+// Row kernels over fused logits Z (fp32 [rows, n]), k_rows.cu.
+// Segment statistics: stats[r * nseg + s] = (max of z over the ids
+// 32s..32s+31 of row r, sum of exp((z - max) * inv_tau) over them), nseg =
+// seg_count(n); chunk statistics cstats[r * nchunk + c], nchunk =
+// chunk_count(nseg), the same pair over the 32 segments 32c..32c+31.
+int seg_count(int n);
+int chunk_count(int nseg);
+cudaError_t launch_seg_stats(const float* Z, int rows, int n, float inv_tau,
+                             float2* stats, float2* cstats, int sm_count,
+                             cudaStream_t st);
+// chunk statistics from segment statistics with nseg segments per row
+cudaError_t launch_chunk_stats(const float2* stats, int rows, int nseg,
+                               float inv_tau, float2* cstats, int sm_count,
+                               cudaStream_t st);
+// One inverse-CDF draw per row from segment and chunk statistics with nseg
+// segments per row (nseg * 32 >= n; segments past n hold zero weight).
+cudaError_t launch_sample_segments(const float* Z, int rows, int n,
+                                   const float2* stats, int nseg,
+                                   const float2* cstats, const int32_t* ids,
+                                   float inv_tau, uint64_t seed, uint64_t offset,
+                                   int32_t* tokens, cudaStream_t st);
 int sample_max_n();
+int verify_max_k();
 
-// speculative verification, one CTA per session
+// Speculative verification (four launches); `scratch` holds
+// verify_scratch_bytes(sessions, k, n) bytes.
+size_t verify_scratch_bytes(int sessions, int k, int n);
 cudaError_t launch_verify(const float* Z, int sessions, int k, int n,
                           const int32_t* ids, int V, float inv_tau,
                           const int32_t* draft, const float* q,
                           uint64_t seed, uint64_t offset, int32_t* n_acc,
-                          int32_t* next_token, cudaStream_t st);
+                          int32_t* next_token, void* scratch, int sm_count,
+                          cudaStream_t st);
 
 }  // namespace sph

@@ -164,6 +164,36 @@ def test_verify_parity(ctx, S, k, n, greedy):
         check_verify(ctx, w, target)
 
 
+@pytest.mark.parametrize("n", [1, 31, 33, 1025, 16 * 1024 + 5, 40000])
+def test_row_kernels_ragged_sizes(ctx, n):
+    # edges of the 32-id segment, the 1024-id chunk and the 16-chunk pass of
+    # the statistics and draw kernels; rows 2 and 6 take the CUDA-core and
+    # the tensor-core endpoint paths
+    for rows in (2, 6):
+        w = small(V=n + 7, d=96, d_l=16, rows=rows, n_keep=n, tau=0.7)
+        codes, scale = wl.make_payload(w.rows, w.n_keep, seed=n % 97)
+        for off in (0, 5):
+            w.offset = off
+            check_endpoint(ctx, w, codes, scale)
+    S, k = 3, 2
+    for tau, greedy in ((1.0, False), (0.1, True)):
+        w = small(V=n + 7, d=96, d_l=8, rows=S * (k + 1), n_keep=n, sessions=S, k=k,
+                  tau=tau)
+        if greedy:
+            w.draft_probs = None
+        target = wl.make_target_logits(w.rows, n, seed=n % 89, std=1.0)
+        check_verify(ctx, w, target)
+
+
+def test_verify_many_sessions(ctx):
+    S, k, n = 1000, 1, 200
+    w = small(V=3 * n, d=96, d_l=8, rows=S * (k + 1), n_keep=n, sessions=S, k=k)
+    target = wl.make_target_logits(w.rows, n, seed=21, std=2.0)
+    n_acc, _, _ = check_verify(ctx, w, target)
+    a = np_(n_acc)
+    assert 0 < (a == 0).sum() < S and 0 < (a == 1).sum() < S
+
+
 def test_verify_accepts_drafts_equal_to_target(ctx):
     # q == p  =>  every draft accepted (r < 1 = p/q), bonus from p_k
     S, k, n = 6, 3, 500
