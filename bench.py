@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--rows", type=int, default=None, help="sweep: rows")
     ap.add_argument("--keep", type=float, default=None, help="sweep: keep fraction")
     ap.add_argument("--e2e-steps", type=int, default=300)
+    ap.add_argument("--act", choices=["fp32", "bf16"], default="fp32",
+                    help="cloud activations: fp32 (exact, two bf16 planes) or bf16-rounded")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -160,11 +162,11 @@ class OracleSample:
     """One bounded sample of the workload for the oracle: row r of h over a
     slice of L consecutive kept ids (cloud call, then endpoint call)."""
 
-    def __init__(self, w):
+    def __init__(self, w, act="fp32"):
         import numpy as np
         import torch
         import oracle
-        self.np, self.oracle, self.w = np, oracle, w
+        self.np, self.oracle, self.w, self.act = np, oracle, w, act
 
         def bits(t):
             t = t.detach().cpu().contiguous()
@@ -189,7 +191,7 @@ class OracleSample:
         hc = self.h[r:r + 1, w.d_l:]
         hl = self.h[r:r + 1, :w.d_l]
         c = o.partial_logits(hc, self.Wh, w_dtype=w.w_dtype, w_scale=self.ws,
-                             keep_ids=ids, clip=w.clip)
+                             keep_ids=ids, clip=w.clip, act_mode=self.act)
         o.fuse_sample(c["codes"], c["row_scale"], hl, self.Wl, keep_ids=ids,
                       tau=w.tau, seed=w.seed, offset=self.i)
         return L / self.ids.size                  # rows of the metric done
@@ -203,8 +205,8 @@ class OracleSample:
         return max(min(64, self.ids.size), min(self.ids.size, L))
 
 
-def cpu_baseline(w, seconds):
-    s = OracleSample(w)
+def cpu_baseline(w, seconds, act="fp32"):
+    s = OracleSample(w, act)
     L = s.calibrate(min(1.0, seconds / 10))
     done = 0.0
     n = 0
@@ -272,6 +274,7 @@ def run_ours(args):
         w.h = wl.make_hidden(w.rows, w.d, g, dev)
     R, n = w.rows, w.n_keep
     ctx = sph.Context(local)
+    act_mode = sph.SPH_ACT_BF16 if args.act == "bf16" else sph.SPH_ACT_FP32
     ctx.reserve(R, n, max(w.d_h, w.d_l))
 
     # rotation so that bytes between reuses exceed 2x L2
@@ -296,7 +299,7 @@ def run_ours(args):
             events[0].record()
         ctx.partial_logits(hh[:, w.d_l:], Whs[c], keep_ids=w.keep_ids, clip=w.clip,
                            w_row_scale=w.w_scale, bias=w.bias, codes=codes,
-                           row_scale=scale)
+                           row_scale=scale, act_mode=act_mode)
         if events is not None:
             events[1].record()
         ctx.fuse_sample(codes, scale, hh[:, :w.d_l], Wls[c], keep_ids=w.keep_ids,
@@ -391,7 +394,7 @@ def run_ours(args):
                 c = i % ncopy
                 ctx.partial_logits(hs[c][:, w.d_l:], Whs[c], keep_ids=w.keep_ids,
                                    clip=w.clip, w_row_scale=w.w_scale, bias=w.bias,
-                                   codes=codes, row_scale=scale)
+                                   codes=codes, row_scale=scale, act_mode=act_mode)
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         gc.replay()
@@ -468,11 +471,14 @@ def run_ours(args):
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(ms / args.steps, 5), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32" if args.act == "fp32" else "bf16",
         "data": "synthetic (seeded, paper shapes; weights N(0,0.02) bf16, h RMS-normalised)",
         "config": {"workload": describe(w), "rows_per_gpu": R, "n_keep": n,
                    "d_h": w.d_h, "d_l": w.d_l, "V": w.V, "weights": w.w_dtype,
                    "accumulate": "fp32",
+                   "activations": ("fp32 (exact: bf16 hi + lo planes)" if args.act == "fp32"
+                                   else "bf16-rounded (one plane)"),
                    "l2": (f"inputs rotate over {ncopy} weight/h copies, "
                           f"{ncopy * per_copy / 1e6:.0f} MB touched per cycle vs L2 "
                           f"{l2 / 1e6:.0f} MB"),
@@ -489,7 +495,7 @@ def run_ours(args):
         "clocks": clocks,
     }
     if world == 1 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
+        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act)
     print(json.dumps(out), flush=True)
     if world > 1:
         dist.barrier()
@@ -506,7 +512,7 @@ def run_reference(args):
         return
     from paper_2607_13093_gb300 import workloads as wl
     w = wl.workload(args.workload, device="cpu", rows=args.rows, keep_frac=args.keep)
-    s = OracleSample(w)
+    s = OracleSample(w, args.act)
     budget = 150.0
     L = s.calibrate(budget / max(1, args.steps + args.warmup))
     for _ in range(args.warmup):

@@ -19,8 +19,10 @@
 //                     isolated ids still work as 1-row boxes.
 // Operand B (the h planes, L2-resident) always comes by TMA.
 //
-// Work split: the (row block, vocabulary tile, k-block) iterations are cut
-// into one contiguous range per persistent CTA (one CTA per SM).  When K is
+// Work split: the (vocabulary tile, row block, k-block) iterations -- row
+// blocks innermost, so that a CTA that takes a tile for several row blocks
+// reads its W rows from DRAM once and then from L2 -- are cut into one
+// contiguous range per persistent CTA (one CTA per SM).  When K is
 // short, ranges cover whole tiles; otherwise they are split stream-K style
 // and a tile whose k-range spans several CTAs is finished by the last CTA to
 // arrive: contributors store fp32 partials, count in, and the last one adds
@@ -64,6 +66,7 @@ constexpr int kThreads = 64 + 32 * kEpiWarps;       // producer, MMA, epilogue
 constexpr int kThreadsFp8 = kThreads + 128;         // + four converter warps (fp8)
 constexpr int kMaxBNFp8 = 128;       // h rows per block with fp8 weights
 constexpr int kBoxHeights = 8;       // row boxes of 1, 2, 4, ..., 128 rows
+constexpr int kMaxBoxes = 2 * 128;   // row boxes of one tile (two per run at most)
 
 // W tensor maps: box height 2^i rows for map i (64 columns each).
 struct WMaps {
@@ -204,6 +207,22 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
   }
 }
 
+// TMA copy of a box of 2^lg rows: the map is chosen by a constant index so
+// that every copy names its kernel-parameter tensor map directly.
+__device__ __forceinline__ void tma_load_box(void* dst, const WMaps& wm, int lg, int x, int y,
+                                             uint64_t* bar) {
+  switch (lg) {
+    case 0: ptx::tma_load_2d(dst, &wm.m[0], x, y, bar); break;
+    case 1: ptx::tma_load_2d(dst, &wm.m[1], x, y, bar); break;
+    case 2: ptx::tma_load_2d(dst, &wm.m[2], x, y, bar); break;
+    case 3: ptx::tma_load_2d(dst, &wm.m[3], x, y, bar); break;
+    case 4: ptx::tma_load_2d(dst, &wm.m[4], x, y, bar); break;
+    case 5: ptx::tma_load_2d(dst, &wm.m[5], x, y, bar); break;
+    case 6: ptx::tma_load_2d(dst, &wm.m[6], x, y, bar); break;
+    default: ptx::tma_load_2d(dst, &wm.m[7], x, y, bar); break;
+  }
+}
+
 template <int HILO, bool GATHER, int EPI, bool FP8>
 __global__ void __launch_bounds__(FP8 ? kThreadsFp8 : kThreads, 1)
 tc_kernel(const __grid_constant__ WMaps wm,
@@ -224,6 +243,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
   uint64_t* drain = tempty + 2;        // [1]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  // the current tile's row boxes (subset path), after the barriers
+  int2* s_box = reinterpret_cast<int2*>(base + (size_t)S * stage_bytes + 256);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint32_t ncols = 32;
@@ -281,21 +302,43 @@ tc_kernel(const __grid_constant__ WMaps wm,
     long long issued = 0;
     if (lane == 0) ptx::griddep_wait();          // h planes come from the prep kernel
     __syncwarp();
+    // subset path: the ids of a segment's tile are loaded one segment ahead,
+    // so that planning a tile never waits on memory
+    int nid[4] = {0, 0, 0, 0};
+    auto load_ids = [&](int tl, int (&dst)[4]) {
+      const int j0 = (tl / p.RB) * kTileM;
+      const int rows = min(kTileM, p.n - j0);
+#pragma unroll
+      for (int g = 0; g < 4; ++g) {
+        const int r = 32 * g + lane;
+        dst[g] = r < rows ? p.ids[j0 + r] : 0;
+      }
+    };
+    if constexpr (GATHER && !FP8) {
+      Segments pk = sg;
+      int tn, a0, a1;
+      if (pk.next(tn, a0, a1)) load_ids(tn, nid);
+    }
     while (!stop && sg.next(tile, kb0, kb1)) {
-      const int rb = tile / p.NT, t = tile - rb * p.NT;
+      const int t = tile / p.RB, rb = tile - t * p.RB;
       int2 box[8];                               // (first id, row | lg << 8)
       unsigned bmask = 0;                        // which of box[] are in use
+      int nbox = 0;
       uint32_t tx = (uint32_t)(FP8 ? b_bytes : stage_bytes);
       if constexpr (GATHER && !FP8) {
         const int j0 = t * kTileM;
         const int rows = min(kTileM, p.n - j0);
-        int idr[4];
+        int idr[4] = {nid[0], nid[1], nid[2], nid[3]};
+        {
+          Segments pk = sg;
+          int tn, a0, a1;
+          if (pk.next(tn, a0, a1)) load_ids(tn, nid);
+        }
         unsigned smask[4];
         int prev_last = 0;
 #pragma unroll
         for (int g = 0; g < 4; ++g) {
           const int r = 32 * g + lane;
-          idr[g] = r < rows ? p.ids[j0 + r] : 0;
           int prev = __shfl_up_sync(0xFFFFFFFFu, idr[g], 1);
           if (lane == 0) prev = prev_last;
           smask[g] = __ballot_sync(0xFFFFFFFFu, r < rows && (r == 0 || idr[g] != prev + 1));
@@ -330,6 +373,22 @@ tc_kernel(const __grid_constant__ WMaps wm,
 #pragma unroll
         for (int o = 16; o; o >>= 1) covered += __shfl_xor_sync(0xFFFFFFFFu, covered, o);
         tx = (uint32_t)(covered * 128 * NA + b_bytes);
+        // compact every lane's boxes into one shared list; lane b issues
+        // list entries b, b + 32, ... (measured: far faster than issuing
+        // from the planning registers under per-lane predicates)
+        const int mine = __popc(bmask);
+        int incl = mine;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+          if (lane >= o) incl += v;
+        }
+        nbox = __shfl_sync(0xFFFFFFFFu, incl, 31);
+        int slot = incl - mine;
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          if ((bmask >> q) & 1u) s_box[slot++] = box[q];
+        __syncwarp();
       }
       for (int kb = kb0; kb < kb1; ++kb) {
         int ok = 1;
@@ -346,13 +405,10 @@ tc_kernel(const __grid_constant__ WMaps wm,
         for (int a = 0; a < NA && !FP8; ++a) {
           const int x = (kb * NA + a) * kAtomK;
           if constexpr (GATHER) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              if ((bmask >> q) & 1u) {
-                const int row = box[q].y & 0xFF, lg = box[q].y >> 8;
-                ptx::tma_load_2d(A + a * kAtomBytes + row * 128, &wm.m[lg], x, box[q].x,
-                                 &full[stage]);
-              }
+            for (int b = lane; b < nbox; b += 32) {
+              const int2 bx = s_box[b];
+              tma_load_box(A + a * kAtomBytes + (bx.y & 0xFF) * 128, wm, bx.y >> 8, x, bx.x,
+                           &full[stage]);
             }
           } else {
             if (lane == 0)
@@ -440,8 +496,11 @@ tc_kernel(const __grid_constant__ WMaps wm,
     int si = 0, tile, kb0, kb1;
     while (sg.next(tile, kb0, kb1)) {
       const int acc = si & 1;
-      const int rb = tile / p.NT, t = tile - rb * p.NT;
+      const int t = tile / p.RB, rb = tile - t * p.RB;
       const bool whole = kb0 == 0 && kb1 == p.KB;
+      const int j = t * kTileM + i;
+      const bool vj = j < p.n;
+      const int id = vj ? (GATHER ? p.ids[j] : j) : 0;
       Payload pay;
       if constexpr (EPI == EPI_ENDPOINT) {
         // the payload does not depend on the accumulator: start on it
@@ -458,9 +517,6 @@ tc_kernel(const __grid_constant__ WMaps wm,
       }
       fph[acc] ^= 1;
       ptx::tc_fence_after();
-      const int j = t * kTileM + i;
-      const bool vj = j < p.n;
-      const int id = vj ? (GATHER ? p.ids[j] : j) : 0;
       const int seg = t * 4 + quad;
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
       // a CTA's split tiles can only be its first and its last segment:
@@ -553,7 +609,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     int tile, kb0, kb1;
     bool stop = false;
     while (!stop && sg.next(tile, kb0, kb1)) {
-      const int t = tile % p.NT;
+      const int t = tile / p.RB;
       int rid[16];
 #pragma unroll
       for (int m = 0; m < 16; ++m) {
@@ -754,7 +810,7 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.cnt_bytes = align256((size_t)tiles * 4 * kEpiGroups * sizeof(int));
   pl.stats_bytes = endpoint ? align256((size_t)rows * pl.NT * 4 * sizeof(float2)) : 0;
   pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
-  pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256;
+  pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256 + kMaxBoxes * sizeof(int2);
   pl.ok = fp8 ? pl.stages >= 4 : pl.stages >= 2;
   return pl;
 }
