@@ -373,9 +373,9 @@ tc_kernel(const __grid_constant__ WMaps wm,
 #pragma unroll
         for (int o = 16; o; o >>= 1) covered += __shfl_xor_sync(0xFFFFFFFFu, covered, o);
         tx = (uint32_t)(covered * 128 * NA + b_bytes);
-        // compact every lane's boxes into one shared list; lane b issues
-        // list entries b, b + 32, ... (measured: far faster than issuing
-        // from the planning registers under per-lane predicates)
+        // compact every lane's boxes into one shared list that the copy loop
+        // below hands out to lanes (measured: far faster than issuing from
+        // the planning registers under per-lane predicates)
         const int mine = __popc(bmask);
         int incl = mine;
 #pragma unroll
@@ -401,27 +401,28 @@ tc_kernel(const __grid_constant__ WMaps wm,
         }
         if (lane == 0) ptx::mbar_expect_tx(&full[stage], tx);
         __syncwarp();
+        // every copy of the stage -- NA x (row boxes) for A (fp8: none; the
+        // converter warps fill A), NA x HILO for B -- goes to its own lane,
+        // so the copies are issued side by side rather than one after another
         uint8_t* A = base + (size_t)stage * stage_bytes;
-        for (int a = 0; a < NA && !FP8; ++a) {
-          const int x = (kb * NA + a) * kAtomK;
-          if constexpr (GATHER) {
-            for (int b = lane; b < nbox; b += 32) {
-              const int2 bx = s_box[b];
+        const int nA = FP8 ? 0 : NA * (GATHER ? nbox : 1);
+        for (int op = lane; op < nA + NA * HILO; op += 32) {
+          if (op < nA) {
+            const int a = GATHER ? op / nbox : op;
+            const int x = (kb * NA + a) * kAtomK;
+            if constexpr (GATHER) {
+              const int2 bx = s_box[op - a * nbox];
               tma_load_box(A + a * kAtomBytes + (bx.y & 0xFF) * 128, wm, bx.y >> 8, x, bx.x,
                            &full[stage]);
-            }
-          } else {
-            if (lane == 0)
+            } else {
               ptx::tma_load_2d(A + a * kAtomBytes, &wm.m[kBoxHeights - 1], x, t * kTileM,
                                &full[stage]);
+            }
+          } else {
+            const int j = op - nA, a = j / HILO, h = j - a * HILO;
+            ptx::tma_load_2d(A + a_bytes + (h * NA + a) * BN * 128, &tmH,
+                             (kb * NA + a) * kAtomK, h * p.Rp + rb * BN, &full[stage]);
           }
-        }
-        if (lane == 0) {
-          uint8_t* B = A + a_bytes;
-          for (int a = 0; a < NA; ++a)
-            for (int h = 0; h < HILO; ++h)
-              ptx::tma_load_2d(B + (h * NA + a) * BN * 128, &tmH, (kb * NA + a) * kAtomK,
-                               h * p.Rp + rb * BN, &full[stage]);
         }
         ++issued;
         if (++stage == S) { stage = 0; phase ^= 1; }
