@@ -12,10 +12,10 @@
 // Operand A comes from W by TMA 2-D tile copies, one per 64-column atom:
 //   full vocabulary : one box of 128 rows per atom;
 //   kept-id subset  : the tile's 128 kept ids are cut into runs of
-//                     consecutive vocabulary ids and every run into boxes of
-//                     1, 2, 4, ..., 128 rows (one tensor map per box height),
-//                     each written at its row of the tile; language subsets
-//                     are mostly long runs, so a tile takes a few boxes, and
+//                     consecutive vocabulary ids and every run is one box of
+//                     exactly its length (one tensor map per height 1..128),
+//                     written at its row of the tile; language subsets are
+//                     mostly long runs, so a tile takes about two boxes, and
 //                     isolated ids still work as 1-row boxes.
 // Operand B (the h planes, L2-resident) always comes by TMA.
 //
@@ -65,8 +65,8 @@ constexpr int kEpiGroups = kEpiWarps / 4;
 constexpr int kThreads = 64 + 32 * kEpiWarps;       // producer, MMA, epilogue
 constexpr int kThreadsFp8 = kThreads + 128;         // + four converter warps (fp8)
 constexpr int kMaxBNFp8 = 128;       // h rows per block with fp8 weights
-constexpr int kBoxHeights = 8;       // row boxes of 1, 2, 4, ..., 128 rows
-constexpr int kMaxBoxes = 2 * 128;   // row boxes of one tile (two per run at most)
+constexpr int kBoxHeights = 128;     // row boxes of 1, 2, 3, ..., 128 rows (map h-1)
+constexpr int kMaxBoxes = 128;       // row boxes of one tile (one per run)
 
 // W tensor maps: box height 2^i rows for map i (64 columns each).
 struct WMaps {
@@ -207,22 +207,6 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
   }
 }
 
-// TMA copy of a box of 2^lg rows: the map is chosen by a constant index so
-// that every copy names its kernel-parameter tensor map directly.
-__device__ __forceinline__ void tma_load_box(void* dst, const WMaps& wm, int lg, int x, int y,
-                                             uint64_t* bar) {
-  switch (lg) {
-    case 0: ptx::tma_load_2d(dst, &wm.m[0], x, y, bar); break;
-    case 1: ptx::tma_load_2d(dst, &wm.m[1], x, y, bar); break;
-    case 2: ptx::tma_load_2d(dst, &wm.m[2], x, y, bar); break;
-    case 3: ptx::tma_load_2d(dst, &wm.m[3], x, y, bar); break;
-    case 4: ptx::tma_load_2d(dst, &wm.m[4], x, y, bar); break;
-    case 5: ptx::tma_load_2d(dst, &wm.m[5], x, y, bar); break;
-    case 6: ptx::tma_load_2d(dst, &wm.m[6], x, y, bar); break;
-    default: ptx::tma_load_2d(dst, &wm.m[7], x, y, bar); break;
-  }
-}
-
 template <int HILO, bool GATHER, int EPI, bool FP8>
 __global__ void __launch_bounds__(FP8 ? kThreadsFp8 : kThreads, 1)
 tc_kernel(const __grid_constant__ WMaps wm,
@@ -263,9 +247,10 @@ tc_kernel(const __grid_constant__ WMaps wm,
     *s_abort = 0;
     ptx::fence_mbar_init();
   }
-  if (warp == 0 && lane < kBoxHeights) {
-    if (!FP8 && (GATHER || lane == kBoxHeights - 1)) ptx::prefetch_tmap(&wm.m[lane]);
-    if (lane == 0) ptx::prefetch_tmap(&tmH);
+  if (warp == 0 && lane == 0) {
+    // (the subset path's other heights are fetched on first use)
+    if (!FP8) ptx::prefetch_tmap(&wm.m[kBoxHeights - 1]);
+    ptx::prefetch_tmap(&tmH);
   }
   // Only the warps that touch memory written or read by the kernels before
   // this one wait for them (griddep_wait): the producer before its first
@@ -291,9 +276,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     // ------------------------------------------------------- TMA producer
     // lane 0 owns the ring.  On the subset path the warp plans each tile's
     // row boxes itself (lane l owns tile rows l, l+32, l+64, l+96): runs of
-    // consecutive kept ids, each covered by one box of 2^k rows, or two
-    // that overlap on identically copied rows; every lane issues the boxes
-    // of the runs that start in its rows.
+    // consecutive kept ids, each one box of its own height.
     Segments sg{it0, it1, p.KB};
     int stage = 0;
     uint32_t phase = 0;
@@ -321,7 +304,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     }
     while (!stop && sg.next(tile, kb0, kb1)) {
       const int t = tile / p.RB, rb = tile - t * p.RB;
-      int2 box[8];                               // (first id, row | lg << 8)
+      int2 box[4];                               // (first id, row | (rows - 1) << 8)
       unsigned bmask = 0;                        // which of box[] are in use
       int nbox = 0;
       uint32_t tx = (uint32_t)(FP8 ? b_bytes : stage_bytes);
@@ -357,17 +340,10 @@ tc_kernel(const __grid_constant__ WMaps wm,
               for (int g2 = g + 1; g2 < 4; ++g2)
                 if (smask[g2]) { nxt = 32 * g2 + __ffs(smask[g2]) - 1; break; }
             }
-            const int len = nxt - r;
-            const int lg = 31 - __clz(len);
-            box[2 * g] = make_int2(idr[g], r | (lg << 8));
-            bmask |= 1u << (2 * g);
-            covered += 1 << lg;
-            if (len != (1 << lg)) {
-              box[2 * g + 1] =
-                  make_int2(idr[g] + len - (1 << lg), (r + len - (1 << lg)) | (lg << 8));
-              bmask |= 2u << (2 * g);
-              covered += 1 << lg;
-            }
+            const int len = nxt - r;               // 1..128: one box of exactly len rows
+            box[g] = make_int2(idr[g], r | ((len - 1) << 8));
+            bmask |= 1u << g;
+            covered += len;
           }
         }
 #pragma unroll
@@ -386,7 +362,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
         nbox = __shfl_sync(0xFFFFFFFFu, incl, 31);
         int slot = incl - mine;
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
+        for (int q = 0; q < 4; ++q)
           if ((bmask >> q) & 1u) s_box[slot++] = box[q];
         __syncwarp();
       }
@@ -412,8 +388,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
             const int x = (kb * NA + a) * kAtomK;
             if constexpr (GATHER) {
               const int2 bx = s_box[op - a * nbox];
-              tma_load_box(A + a * kAtomBytes + (bx.y & 0xFF) * 128, wm, bx.y >> 8, x, bx.x,
-                           &full[stage]);
+              ptx::tma_load_2d(A + a * kAtomBytes + (bx.y & 0xFF) * 128, &wm.m[bx.y >> 8], x,
+                               bx.x, &full[stage]);
             } else {
               ptx::tma_load_2d(A + a * kAtomBytes, &wm.m[kBoxHeights - 1], x, t * kTileM,
                                &full[stage]);
@@ -759,6 +735,48 @@ bool make_map(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr,
 
 size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
+// W tensor maps, encoded once per weight tensor: map i copies boxes of 64
+// columns x (i + 1) rows of W [V rows, K columns], row stride ld_w (the
+// full-vocabulary path uses only the 128-row map).  A few recently used
+// sets are kept, since encoding 128 maps costs far more than a launch.
+struct MapSet {
+  const void* W = nullptr;
+  int64_t V = 0, K = 0, ld = 0;
+  bool gather = false;
+  unsigned long long used = 0;
+  WMaps maps;
+};
+std::mutex g_map_mu;
+MapSet g_map_sets[8];
+unsigned long long g_map_tick = 0;
+
+bool w_maps(const GatherGemm& g, bool gather, WMaps& out) {
+  std::lock_guard<std::mutex> lock(g_map_mu);
+  MapSet* hit = nullptr;
+  MapSet* lru = &g_map_sets[0];
+  for (MapSet& m : g_map_sets) {
+    if (m.W == g.W && m.V == g.V && m.K == g.K && m.ld == g.ld_w && m.gather == gather) hit = &m;
+    if (m.used < lru->used) lru = &m;
+  }
+  if (!hit) {
+    hit = lru;
+    hit->W = nullptr;
+    for (int i = 0; i < kBoxHeights; ++i) {
+      if (!gather && i != kBoxHeights - 1) {
+        hit->maps.m[i] = CUtensorMap{};
+        continue;
+      }
+      if (!make_map(&hit->maps.m[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
+                    (uint64_t)g.V, (uint64_t)g.ld_w * 2, kAtomK, (uint32_t)(i + 1)))
+        return false;
+    }
+    hit->W = g.W; hit->V = g.V; hit->K = g.K; hit->ld = g.ld_w; hit->gather = gather;
+  }
+  hit->used = ++g_map_tick;
+  out = hit->maps;
+  return true;
+}
+
 }  // namespace
 
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
@@ -857,17 +875,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
 
   WMaps mw;
   alignas(64) CUtensorMap mh;
-  // W: [V rows, K columns], row stride ld_w; map i copies boxes of 64
-  // columns x 2^i rows (the full-vocabulary path uses only the 128-row map)
-  for (int i = 0; i < kBoxHeights; ++i) {
-    if (fp8 || (!gather && i != kBoxHeights - 1)) {
-      mw.m[i] = CUtensorMap{};
-      continue;
-    }
-    if (!make_map(&mw.m[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
-                  (uint64_t)g.V, (uint64_t)g.ld_w * 2, kAtomK, 1u << i))
-      return cudaErrorInvalidValue;
-  }
+  if (!fp8 && !w_maps(g, gather, mw)) return cudaErrorInvalidValue;
   if (!make_map(&mh, fp8 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
                 Hs, (uint64_t)pl.Kp,
                 (uint64_t)pl.hilo * pl.Rp, (uint64_t)pl.Kp * 2, kAtomK,
