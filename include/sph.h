@@ -99,7 +99,7 @@ typedef enum sph_option {
   SPH_OPT_TC_MIN_ROWS = 0,  /* row count from which the tcgen05 tensor-core
                                kernels replace the CUDA-core GEMV (default 4;
                                1 forces tensor cores, a huge value forces the
-                               GEMV; fp8 weights always use the GEMV path)    */
+                               GEMV)                                          */
   SPH_OPT_SPIN_LIMIT = 1,   /* clock cycles a device-side wait may spin before
                                it gives up and the call reports
                                SPH_ERR_TIMEOUT (default 2^34, >= 1)           */
@@ -108,9 +108,12 @@ typedef enum sph_option {
                                k-block ranges (stream-K)                      */
   SPH_OPT_TC_STAGES = 3,    /* tensor-core pipeline depth: 0 automatic
                                (default), else at most this many stages (>= 2) */
-  SPH_OPT_TC_BLOCK_K = 4    /* hidden-dimension elements each pipeline stage
+  SPH_OPT_TC_BLOCK_K = 4,   /* hidden-dimension elements each pipeline stage
                                reads per weight row: 64, 128, 256, or 0 for
                                automatic (default)                           */
+  SPH_OPT_TC_MAX_BN = 5     /* most hidden-state rows one tensor-core tile
+                               covers: a multiple of 16 in [16, 256], or 0
+                               for automatic (default)                       */
 } sph_option;
 
 /* Set a tunable (SPH_ERR_INVALID_ARG for an unknown option or a value out of

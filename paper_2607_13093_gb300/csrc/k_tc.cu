@@ -780,13 +780,18 @@ bool w_maps(const GatherGemm& g, bool gather, WMaps& out) {
 }  // namespace
 
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
-               int schedule, int max_stages, int block_k, int gather, int fp8) {
+               int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn_opt) {
   TcPlan pl{};
   // one bf16 plane carries bf16-rounded activations exactly; f16 planes
   // (fp8 weights) always take two
   pl.hilo = (act_bf16 && !fp8) ? 1 : 2;
   pl.fp8 = fp8;
-  const int max_bn = fp8 ? kMaxBNFp8 : kMaxBN;
+  int max_bn = fp8 ? kMaxBNFp8 : kMaxBN;
+  // two h planes: at most 224 rows, so that three stages fit (measured:
+  // 1024 rows x 256k ids x 4608 runs 21 % faster in three 224-row stages
+  // than in two 256-row ones)
+  if (!fp8 && pl.hilo == 2 && max_bn > 224) max_bn = 224;
+  if (max_bn_opt >= 16 && max_bn_opt < max_bn) max_bn = max_bn_opt;
   if (rows <= max_bn) {
     pl.RB = 1;
     pl.BN = (rows + 15) / 16 * 16;

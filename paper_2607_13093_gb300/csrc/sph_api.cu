@@ -33,6 +33,7 @@ struct sph_ctx {
   int tc_schedule = 0;              // SPH_OPT_TC_SCHEDULE
   int tc_stages = 0;                // SPH_OPT_TC_STAGES
   int tc_block_k = 0;               // SPH_OPT_TC_BLOCK_K
+  int tc_max_bn = 0;                // SPH_OPT_TC_MAX_BN
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -129,7 +130,8 @@ size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_
   for (int gather = 0; gather < 2; ++gather) {   // the larger of the two paths
     const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count,
                                   endpoint, ctx->tc_schedule, ctx->tc_stages,
-                                  ctx->tc_block_k, gather, w_dtype == sph::W_FP8)
+                                  ctx->tc_block_k, gather, w_dtype == sph::W_FP8,
+                                  ctx->tc_max_bn)
                          .scratch_bytes;
     if (x > b) b = x;
   }
@@ -379,6 +381,11 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
         return fail(ctx, SPH_ERR_INVALID_ARG, "block_k must be 0, 64, 128 or 256");
       ctx->tc_block_k = (int)value;
       return SPH_OK;
+    case SPH_OPT_TC_MAX_BN:
+      if (value != 0 && (value < 16 || value > 256 || value % 16))
+        return fail(ctx, SPH_ERR_INVALID_ARG, "max_bn must be 0 or a multiple of 16 in [16, 256]");
+      ctx->tc_max_bn = (int)value;
+      return SPH_OK;
   }
   return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
 }
@@ -466,7 +473,7 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_h, act_bf16,
                                         ctx->sm_count, 0, ctx->tc_schedule, ctx->tc_stages,
                                         ctx->tc_block_k, keep_ids != nullptr,
-                                        wdt == sph::W_FP8);
+                                        wdt == sph::W_FP8, ctx->tc_max_bn);
     void* tcs = c.take(pl.scratch_bytes);
     st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
@@ -523,7 +530,8 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   if (use_tc(ctx, rows, sph::W_BF16)) {
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0,
                                         ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
-                                        ctx->tc_block_k, keep_ids != nullptr, 0);
+                                        ctx->tc_block_k, keep_ids != nullptr, 0,
+                                        ctx->tc_max_bn);
     void* tcs = c.take(pl.scratch_bytes);
     st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);

@@ -90,9 +90,10 @@ struct TcPlan {
 // `endpoint` reserves the per-segment softmax statistics; schedule 0/1/2 =
 // automatic / whole tiles / stream-K; max_stages 0 = automatic; block_k =
 // hidden elements per pipeline stage (64, 128 or 256; 0 = automatic);
-// gather = the kept-id subset path (keep_ids given); fp8 = e4m3 weights.
+// gather = the kept-id subset path (keep_ids given); fp8 = e4m3 weights;
+// max_bn = most hidden-state rows per tile (0 = automatic).
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
-               int schedule, int max_stages, int block_k, int gather, int fp8);
+               int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn);
 // Launch the operand split and the tcgen05 kernel; `scratch` holds
 // plan.scratch_bytes bytes.  bf16 weights only.
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,
