@@ -71,6 +71,7 @@ constexpr int kMaxBoxes = 128;       // row boxes of one tile (one per run)
 // W tensor maps: box height 2^i rows for map i (64 columns each).
 struct WMaps {
   CUtensorMap m[kBoxHeights];
+  CUtensorMap a3;              // full vocabulary: (element, row, atom) view, all atoms of a stage
 };
 
 struct TcParams {
@@ -90,7 +91,8 @@ struct TcParams {
   const int8_t* codes;
   const float* row_scale;
   float inv_tau;
-  float2* seg_stats;           // endpoint: [R][NT*4] (max, sum exp)
+  float2* seg_stats;
+  int a3d;                     // full vocabulary: A by one 3-D copy per stage           // endpoint: [R][NT*4] (max, sum exp)
   float* P;                    // split-tile partials [2 * grid][BN][128]
   int* counters;               // [tiles][4 quadrants], zero between calls
   unsigned* status;
@@ -377,27 +379,30 @@ tc_kernel(const __grid_constant__ WMaps wm,
         }
         if (lane == 0) ptx::mbar_expect_tx(&full[stage], tx);
         __syncwarp();
-        // every copy of the stage -- NA x (row boxes) for A (fp8: none; the
-        // converter warps fill A), NA x HILO for B -- goes to its own lane,
-        // so the copies are issued side by side rather than one after another
+        // every copy of the stage goes to its own lane, so the copies are
+        // issued side by side rather than one after another: A as NA x (row
+        // boxes), or over the full vocabulary (when its width allows) one 3-D
+        // copy of all NA atoms (fp8: none; the converter warps fill A); B as
+        // one 3-D copy of all NA atoms per plane
         uint8_t* A = base + (size_t)stage * stage_bytes;
-        const int nA = FP8 ? 0 : NA * (GATHER ? nbox : 1);
-        for (int op = lane; op < nA + NA * HILO; op += 32) {
+        const int nA = FP8 ? 0 : (GATHER ? NA * nbox : (p.a3d ? 1 : NA));
+        for (int op = lane; op < nA + HILO; op += 32) {
           if (op < nA) {
-            const int a = GATHER ? op / nbox : op;
-            const int x = (kb * NA + a) * kAtomK;
             if constexpr (GATHER) {
+              const int a = op / nbox;
               const int2 bx = s_box[op - a * nbox];
-              ptx::tma_load_2d(A + a * kAtomBytes + (bx.y & 0xFF) * 128, &wm.m[bx.y >> 8], x,
-                               bx.x, &full[stage]);
+              ptx::tma_load_2d(A + a * kAtomBytes + (bx.y & 0xFF) * 128, &wm.m[bx.y >> 8],
+                               (kb * NA + a) * kAtomK, bx.x, &full[stage]);
+            } else if (p.a3d) {
+              ptx::tma_load_3d(A, &wm.a3, 0, t * kTileM, kb * NA, &full[stage]);
             } else {
-              ptx::tma_load_2d(A + a * kAtomBytes, &wm.m[kBoxHeights - 1], x, t * kTileM,
-                               &full[stage]);
+              ptx::tma_load_2d(A + op * kAtomBytes, &wm.m[kBoxHeights - 1],
+                               (kb * NA + op) * kAtomK, t * kTileM, &full[stage]);
             }
           } else {
-            const int j = op - nA, a = j / HILO, h = j - a * HILO;
-            ptx::tma_load_2d(A + a_bytes + (h * NA + a) * BN * 128, &tmH,
-                             (kb * NA + a) * kAtomK, h * p.Rp + rb * BN, &full[stage]);
+            const int h = op - nA;
+            ptx::tma_load_3d(A + a_bytes + h * NA * BN * 128, &tmH, 0, h * p.Rp + rb * BN,
+                             kb * NA, &full[stage]);
           }
         }
         ++issued;
@@ -733,6 +738,25 @@ bool make_map(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D view (element, row, 64-element atom) of a row-major [rows, cols]
+// matrix: strides row_bytes and 128 bytes; a box of (64, box_rows,
+// box_atoms) lands as box_atoms consecutive 128-byte-swizzled atom tiles
+// of box_rows rows.  cols must be a multiple of 64 (the view cannot mark
+// the end of a row).
+bool make_map3(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64_t cols,
+               uint64_t rows, uint64_t row_bytes, uint32_t box_rows, uint32_t box_atoms) {
+  EncodeFn fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)kAtomK, rows, cols / kAtomK};
+  const cuuint64_t strides[2] = {row_bytes, 128};
+  const cuuint32_t box[3] = {(cuuint32_t)kAtomK, box_rows, box_atoms};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, dt, 3, const_cast<void*>(ptr), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
 // W tensor maps, encoded once per weight tensor: map i copies boxes of 64
@@ -881,10 +905,17 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   WMaps mw;
   alignas(64) CUtensorMap mh;
   if (!fp8 && !w_maps(g, gather, mw)) return cudaErrorInvalidValue;
-  if (!make_map(&mh, fp8 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
-                Hs, (uint64_t)pl.Kp,
-                (uint64_t)pl.hilo * pl.Rp, (uint64_t)pl.Kp * 2, kAtomK,
-                (uint32_t)pl.BN))
+  // h planes [hilo * Rp rows, Kp columns], zero padded: all atoms of a
+  // stage in one copy per plane
+  if (!make_map3(&mh, fp8 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                 Hs, (uint64_t)pl.Kp, (uint64_t)pl.hilo * pl.Rp, (uint64_t)pl.Kp * 2,
+                 (uint32_t)pl.BN, (uint32_t)pl.na))
+    return cudaErrorInvalidValue;
+  // full vocabulary with a width that is a multiple of 64: A likewise
+  const int a3d = (!fp8 && !gather && g.K % kAtomK == 0 && g.K >= pl.na * kAtomK) ? 1 : 0;
+  mw.a3 = CUtensorMap{};
+  if (a3d && !make_map3(&mw.a3, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
+                        (uint64_t)g.V, (uint64_t)g.ld_w * 2, kTileM, (uint32_t)pl.na))
     return cudaErrorInvalidValue;
 
   TcParams prm{};
@@ -898,7 +929,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.epilogue = g.epilogue; prm.bias = g.bias;
   prm.clip = g.clip; prm.partial_out = g.partial_out; prm.Y = g.Y;
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
-  prm.inv_tau = g.inv_tau; prm.seg_stats = stats;
+  prm.inv_tau = g.inv_tau; prm.seg_stats = stats; prm.a3d = a3d;
   prm.P = P; prm.counters = counters;
   prm.status = g.status; prm.spin_limit = spin_limit;
 

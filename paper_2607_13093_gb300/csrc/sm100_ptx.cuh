@@ -64,6 +64,16 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map,
       "l"(map), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
 }
+// 3-D box at (x, y, z) -- here (element, row, 64-element atom) views whose
+// boxes land as consecutive 128-byte-row atom tiles.
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y,
+                                            int z, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
+      "l"(map), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
 // Four rows y0..y3 (each one box row of the map) at column x, written as
 // four consecutive box rows at dst.
 __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map,
