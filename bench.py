@@ -38,6 +38,37 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0,
                   "bf16_tflops_sustained": 1700.0}
 
 
+# ---------------------------------------------------------------------------
+# multi-rank host logic (replicas: every rank runs its own sessions)
+# ---------------------------------------------------------------------------
+def rank_env():
+    """(world, rank, local rank) from the torchrun environment."""
+    return (int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def rank_seed(rank):
+    """Seed of a rank's own hidden states; weights and kept ids stay the
+    workload's (every rank holds the same replicated head)."""
+    return 10_000 + rank
+
+
+def max_over_ranks(x, device=None):
+    """The largest x over all ranks (x itself without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rows_per_s(rows_per_rank, world, steps, ms):
+    """Whole-job throughput: every rank's rows over the slowest rank's time."""
+    return rows_per_rank * world * steps / (ms / 1e3)
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -252,9 +283,7 @@ def run_ours(args):
     import torch
     import torch.distributed as dist
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local = rank_env()
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     torch.cuda.set_device(local)
@@ -270,7 +299,7 @@ def run_ours(args):
     w = wl.workload(args.workload, device=dev, rows=args.rows, keep_frac=args.keep)
     if world > 1:                       # each rank: its own sessions
         g = torch.Generator(device=dev)
-        g.manual_seed(10_000 + rank)
+        g.manual_seed(rank_seed(rank))
         w.h = wl.make_hidden(w.rows, w.d, g, dev)
     R, n = w.rows, w.n_keep
     ctx = sph.Context(local)
@@ -370,11 +399,7 @@ def run_ours(args):
     t_wall1 = time.time()
     if world > 1:
         dist.barrier()
-    ms = ev0.elapsed_time(ev1)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ev0.elapsed_time(ev1), dev)
     clocks = None
     if sampler:
         time.sleep(0.2)
@@ -430,11 +455,7 @@ def run_ours(args):
         step(i, h_dev)
         tok_host.copy_(tokens, non_blocking=True)
         torch.cuda.synchronize(dev)
-    e2e_s = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
 
     if rank != 0:
         if world > 1:
@@ -443,7 +464,7 @@ def run_ours(args):
         return
 
     peaks, peaks_src = load_peaks()
-    value = R * world * args.steps / (ms / 1e3)
+    value = job_rows_per_s(R, world, args.steps, ms)
     # dominant unit: the cloud call (operand split + gathered contraction +
     # quantization), timed inside the timed graph
     alg_bytes = wl.algorithmic_bytes_cloud(R, n, w.d_h, wb, fp8_scales=w.w_dtype == "fp8")

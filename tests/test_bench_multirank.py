@@ -1,0 +1,61 @@
+"""The benchmark's multi-rank host logic (replicas: each rank its own
+sessions, max-over-ranks timing) run as two gloo ranks on the CPU."""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), WORLD_SIZE=str(world),
+                      RANK=str(rank), LOCAL_RANK=str(rank))
+    import bench
+    from paper_2607_13093_gb300 import workloads as wl
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        w_, r_, l_ = bench.rank_env()
+        assert (w_, r_, l_) == (world, rank, rank)
+        # a timed region of a different length on every rank: all ranks
+        # report the slowest
+        ms = bench.max_over_ranks(10.0 + 5.0 * rank)
+        # replicated head, own sessions
+        w = wl.workload("tiny", device="cpu")
+        g = torch.Generator().manual_seed(bench.rank_seed(rank))
+        h = wl.make_hidden(w.rows, w.d, g, "cpu")
+        W = w.W_h.float()
+        hs = [torch.empty_like(h) for _ in range(world)]
+        Ws = [torch.empty_like(W[:64]) for _ in range(world)]
+        dist.all_gather(hs, h)
+        dist.all_gather(Ws, W[:64].contiguous())
+        out[rank] = (ms, bool(torch.equal(Ws[0], Ws[1])), bool(torch.equal(hs[0], hs[1])))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_replicas_and_max_timing():
+    world, port = 2, _free_port()
+    mgr = mp.get_context("spawn").Manager()
+    out = mgr.dict()
+    mp.start_processes(_rank_main, args=(world, port, out), nprocs=world, join=True,
+                       start_method="spawn")
+    assert sorted(out.keys()) == [0, 1]
+    for rank in range(world):
+        ms, same_w, same_h = out[rank]
+        assert ms == 15.0                  # the slower rank's time everywhere
+        assert same_w                      # every rank holds the same head
+        assert not same_h                  # but its own sessions
+
+
+def test_job_throughput_counts_every_rank():
+    import bench
+    assert bench.job_rows_per_s(32, 4, 100, 1000.0) == 32 * 4 * 100 / 1.0
+    assert bench.max_over_ranks(3.5) == 3.5          # no process group: identity
