@@ -194,6 +194,7 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
       const int r = row0 + q;
       if (vj && r < p.R) p.Y[(int64_t)r * p.n + j] = z[q];
     }
+    if (!p.seg_stats) return;          // statistics come from a pass over z
     // softmax statistics of this 32-id segment for each row: the maxima,
     // spread back to every lane, then the sums of exp((z - max) / tau)
     const float mk = warp_reduce_scatter16(z, MaxOp{}, lane);
@@ -857,6 +858,12 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * kTileM * 4) : 0;
   pl.cnt_bytes = align256((size_t)tiles * 4 * kEpiGroups * sizeof(int));
   pl.stats_bytes = endpoint ? align256((size_t)rows * pl.NT * 4 * sizeof(float2)) : 0;
+  // the epilogue's statistics are latency-bound chains of shuffles and
+  // exponentials per 16 rows, hidden behind the next tile's MMAs only when
+  // the hidden dimension is long enough; otherwise a separate pass over z at
+  // memory speed is cheaper (measured: 320 rows x 51302 ids x 512 and
+  // 1024 rows x 256000 ids x 512 gain; 256 rows x 152064 ids x 1024 loses)
+  pl.epi_stats = endpoint && (pl.BN < 128 || 4 * pl.BN <= K);
   pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
   pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256 + kMaxBoxes * sizeof(int2);
   pl.ok = fp8 ? pl.stages >= 4 : pl.stages >= 2;
@@ -929,7 +936,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.epilogue = g.epilogue; prm.bias = g.bias;
   prm.clip = g.clip; prm.partial_out = g.partial_out; prm.Y = g.Y;
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
-  prm.inv_tau = g.inv_tau; prm.seg_stats = stats; prm.a3d = a3d;
+  prm.inv_tau = g.inv_tau; prm.seg_stats = pl.epi_stats ? stats : nullptr; prm.a3d = a3d;
   prm.P = P; prm.counters = counters;
   prm.status = g.status; prm.spin_limit = spin_limit;
 
@@ -960,6 +967,13 @@ cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPl
   const char* sc = static_cast<const char*>(scratch);
   const float2* stats =
       reinterpret_cast<const float2*>(sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes);
+  if (!pl.epi_stats) {
+    float2* sst = const_cast<float2*>(stats);
+    cudaError_t e = launch_seg_stats(Z, rows, n, inv_tau, sst, cstats, sm_count, st);
+    if (e != cudaSuccess) return e;
+    return launch_sample_segments(Z, rows, n, sst, seg_count(n), cstats, ids, inv_tau, seed,
+                                  offset, tokens, st);
+  }
   const int nseg = pl.NT * 4;
   cudaError_t e = launch_chunk_stats(stats, rows, nseg, inv_tau, cstats, sm_count, st);
   if (e != cudaSuccess) return e;

@@ -83,6 +83,7 @@ int gemv_max_k();
 // Tensor-core path (k_tc.cu): sizes, work split and scratch of one call.
 struct TcPlan {
   int hilo, RB, BN, Rp, KB, Kp, NT, G, stages, whole_tiles, na, fp8;
+  int epi_stats;   // endpoint: softmax statistics in the epilogue (else a pass over z)
   long long T;
   size_t hs_bytes, p_bytes, cnt_bytes, stats_bytes, scratch_bytes, smem_bytes;
   bool ok;
@@ -98,9 +99,10 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
 // plan.scratch_bytes bytes.  bf16 weights only.
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,
                       long long spin_limit, cudaStream_t st);
-// One inverse-CDF draw per row from the segment statistics that an endpoint
-// launch_tc left in `scratch`; `cstats` receives rows * chunk_count(4 * NT)
-// chunk statistics on the way.
+// One inverse-CDF draw per row after an endpoint launch_tc: from the segment
+// statistics its epilogue left in `scratch` (plan.epi_stats), else from a
+// statistics pass over Z into the same area; `cstats` receives the chunk
+// statistics on the way (at most rows * (n / 1024 + 2)).
 cudaError_t launch_sample_from_stats(const float* Z, int rows, int n,
                                      const TcPlan& plan, const void* scratch,
                                      float2* cstats, const int32_t* ids,
