@@ -255,11 +255,14 @@ sph_status sph_partial_logits_noalloc(int device, void* cuda_stream,
  *   tokens[r] = keep_ids[j*], j* = the first j whose ascending-order CDF
  *               exceeds u_r, u_r = Philox4x32-10 uniform with key = seed and
  *               counter (r, 0, offset lo, offset hi), u = (x0 >> 8) * 2^-24
+ *   temperature 0 is greedy decoding (the argmax decoding of Eq. 17):
+ *   tokens[r] = keep_ids[j*], j* = the first j with the largest z[r, j]
+ *   (the lowest kept id on ties); no uniform is drawn.
  * Arguments
  *   codes int8 [rows, n_keep], row_scale fp32 [rows]: the cloud payload.
  *   h_local fp32 [rows, d_l], row stride ld_hl (the slice h[:, :d_l]).
  *   W_l bf16 [V, d_l] row-major with row stride ld_wl (16-byte multiple).
- *   keep_ids as for sph_partial_logits.  temperature > 0 and finite.
+ *   keep_ids as for sph_partial_logits.  temperature >= 0 and finite.
  *   tokens int32 [rows] (out, vocabulary ids).
  *   fused_logits_out fp32 [rows, n_keep] z before the division by
  *   temperature (out), or NULL.
@@ -284,6 +287,10 @@ sph_status sph_fuse_sample(sph_ctx* ctx,
  *   that is all zero); if all k are accepted draw from p_k; the draw uses
  *   the uniform of counter (s, 1+k, ...) and the inverse CDF in ascending
  *   id order.
+ *   temperature 0 is greedy verification (the limit of the rule above with
+ *   ties to the lowest id): with a_i the first argmax of row i, drafts are
+ *   accepted while x_i == a_i and the next token is a_i at the first
+ *   mismatch, or a_k; draft_probs is not read and no uniform is drawn.
  * Arguments
  *   target_logits fp32 [sessions*(k+1), n_keep] compacted fused logits.
  *   draft_tokens int32 [sessions, k] vocabulary ids (an id outside V_l has
@@ -292,7 +299,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx,
  *   (one-hot) drafts, where q_i(x) = [x == x_i].
  *   n_accepted int32 [sessions] (out) in [0, k]; next_token int32
  *   [sessions] (out): the drawn vocabulary id.
- * Preconditions: sessions >= 1, k >= 1, temperature > 0.
+ * Preconditions: sessions >= 1, k >= 1, temperature >= 0 and finite.
  * Errors: INVALID_ARG, UNSUPPORTED, CUDA, OOM. */
 sph_status sph_verify_draft(sph_ctx* ctx,
                             const float* target_logits, int64_t sessions,

@@ -260,18 +260,36 @@ def sample_rows(z, tau: float, u):
     return out, margin
 
 
+def greedy_rows(z):
+    """Greedy decoding (temperature 0; the argmax decoding the paper's draft
+    model uses, Eq. 17): per row the first index of the maximum, that is the
+    lowest kept id on ties.  Returns (index, margin) with margin = the gap
+    between the largest and the second-largest value (0 on a tie)."""
+    z = np.asarray(z, dtype=np.float64)
+    j = np.argmax(z, axis=-1)
+    if z.shape[-1] < 2:
+        return j, np.full(z.shape[0], np.inf)
+    top2 = np.sort(z, axis=-1)[:, -2:]
+    return j, top2[:, 1] - top2[:, 0]
+
+
 def fuse_sample(codes, row_scale, h_local, W_l_bits, *, keep_ids=None,
                 tau=1.0, seed=0, offset=0):
     """Endpoint call: local partial, fuse, mask, softmax(./tau), one Philox
-    uniform per row (purpose 0), inverse-CDF draw.  Returns vocabulary-id
-    `tokens`, the CDF `margin` of each draw and the fused logits `z`."""
+    uniform per row (purpose 0), inverse-CDF draw; tau = 0 is greedy
+    decoding (no uniform).  Returns vocabulary-id `tokens`, the `margin` of
+    each draw (CDF distance, or for greedy the top-two gap) and the fused
+    logits `z`."""
     V = W_l_bits.shape[0]
     ids = _ids(keep_ids, V)
     zl = local_partial(h_local, W_l_bits, ids)
     z = fuse(codes, row_scale, zl)
     R = z.shape[0]
     u = philox_uniform(seed, np.arange(R), 0, offset)
-    j, margin = sample_rows(z, tau, u)
+    if tau == 0:
+        j, margin = greedy_rows(z)
+    else:
+        j, margin = sample_rows(z, tau, u)
     return dict(tokens=ids[j].astype(np.int32), margin=margin, z=z, u=u,
                 index=j)
 
@@ -335,8 +353,9 @@ def verify_draft(target_logits, sessions: int, k: int, *, keep_ids=None,
                  offset=0):
     """Cloud verification of k drafts per session.  target_logits
     [S*(k+1), n] are fused logits (row s*(k+1)+i is the target at draft
-    position i, row s*(k+1)+k the bonus position); p_i = softmax(. / tau).
-    Uniforms: r_i = Philox(session, 1+i), u = Philox(session, 1+k)."""
+    position i, row s*(k+1)+k the bonus position); p_i = softmax(. / tau),
+    tau = 0 greedy.  Uniforms: r_i = Philox(session, 1+i),
+    u = Philox(session, 1+k)."""
     Z = np.asarray(target_logits, dtype=np.float32).astype(np.float64)
     n = Z.shape[1]
     if V is None:
@@ -347,6 +366,23 @@ def verify_draft(target_logits, sessions: int, k: int, *, keep_ids=None,
     am = np.empty(sessions)
     dm = np.empty(sessions)
     xs = compact_index(keep_ids, V, np.asarray(draft_tokens).reshape(sessions, k))
+    if tau == 0:
+        # greedy verification, the tau -> 0 limit of the rule in verify_core
+        # with ties resolved to the lowest id: p_i is one-hot at a_i =
+        # argmax z_i, so x_i is accepted iff x_i == a_i (r_i q_i(x_i) < 1
+        # always holds), the residual at the first rejection is one-hot at
+        # a_i (or, all zero, falls back to p_i), and the bonus token is a_k.
+        for s in range(sessions):
+            a, gap = greedy_rows(Z[s * (k + 1):(s + 1) * (k + 1)])
+            i = 0
+            while i < k and xs[s][i] == a[i]:
+                i += 1
+            n_acc[s] = i
+            nxt[s] = ids[a[i]]
+            am[s] = np.min(gap[:i + 1])
+            dm[s] = gap[i]
+        return dict(n_accepted=n_acc, next_token=nxt, accept_margin=am,
+                    draw_margin=dm)
     for s in range(sessions):
         P = softmax_rows(Z[s * (k + 1):(s + 1) * (k + 1)], tau)
         r = philox_uniform(seed, np.full(k, s), 1 + np.arange(k), offset)

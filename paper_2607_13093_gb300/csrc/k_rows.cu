@@ -252,6 +252,50 @@ sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
 }
 
 // ---------------------------------------------------------------------------
+// greedy decoding (temperature 0): the first id of the row maximum
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int warp_min_int(int v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v = min(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+  return v;
+}
+
+// The lowest segment holding the row maximum (from its statistics), then the
+// lowest id in it whose z equals that maximum; all lanes return it.
+__device__ __forceinline__ int warp_argmax(const float* z, int n, const float2* st, int nseg,
+                                           int lane) {
+  float M = -INFINITY;
+  int sb = nseg;
+  for (int s = lane; s < nseg; s += 32) {
+    const float m = st[s].x;
+    if (m > M) { M = m; sb = s; }
+  }
+  const float Mw = warp_max(M);
+  if (!(Mw > -INFINITY)) return 0;
+  const int seg = warp_min_int(M == Mw ? sb : nseg);
+  const int j = seg * kSeg + lane;
+  const unsigned hit = __ballot_sync(0xFFFFFFFFu, j < n && z[j] == Mw);
+  return hit ? seg * kSeg + __ffs(hit) - 1 : min(seg * kSeg, n - 1);
+}
+
+// One warp per row: vocabulary ids into tokens and/or compact indices.
+__global__ void __launch_bounds__(kWarps * 32)
+greedy_kernel(const float* __restrict__ Z, int rows, int n, const float2* __restrict__ stats,
+              int nseg, const int32_t* __restrict__ ids, int32_t* __restrict__ tokens,
+              int32_t* __restrict__ compact) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (r >= rows) return;
+  const int j = warp_argmax(Z + (int64_t)r * n, n, stats + (int64_t)r * nseg, nseg, lane);
+  if (lane == 0) {
+    if (tokens) tokens[r] = ids ? ids[j] : j;
+    if (compact) compact[r] = j;
+  }
+}
+
+// ---------------------------------------------------------------------------
 // verification
 // ---------------------------------------------------------------------------
 __device__ int find_compact(const int32_t* ids, int n, int V, int x) {
@@ -353,6 +397,25 @@ verify_residual_kernel(const float* __restrict__ Z, int n, int nseg, int nchunk,
   }
 }
 
+// Greedy verification, one thread per session: accept while the draft is
+// the target's argmax; the next token is the argmax at the first mismatch,
+// or at the bonus position.
+__global__ void greedy_verify_kernel(const int32_t* __restrict__ amax, int sessions, int k,
+                                     int n, const int32_t* __restrict__ ids, int V,
+                                     const int32_t* __restrict__ draft,
+                                     int32_t* __restrict__ n_acc,
+                                     int32_t* __restrict__ next_token) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int s = blockIdx.x * blockDim.x + threadIdx.x;
+  if (s >= sessions) return;
+  const int32_t* a = amax + (int64_t)s * (k + 1);
+  int i = 0;
+  while (i < k && find_compact(ids, n, V, draft[(int64_t)s * k + i]) == a[i]) ++i;
+  n_acc[s] = i;
+  next_token[s] = ids ? ids[a[i]] : a[i];
+}
+
 // One warp per session: the draw, from the residual (or, if that is all
 // zero, from p_i) at the first rejection, else the bonus draw from p_k.
 __global__ void __launch_bounds__(kWarps * 32)
@@ -432,7 +495,10 @@ cudaError_t launch_chunk_stats(const float2* stats, int rows, int nseg, float in
 cudaError_t launch_sample_segments(const float* Z, int rows, int n, const float2* stats,
                                    int nseg, const float2* cstats, const int32_t* ids,
                                    float inv_tau, uint64_t seed, uint64_t offset,
-                                   int32_t* tokens, cudaStream_t st) {
+                                   int32_t* tokens, cudaStream_t st, int greedy) {
+  if (greedy)
+    return launch_pdl(greedy_kernel, dim3((rows + kWarps - 1) / kWarps), dim3(kWarps * 32), 0,
+                      st, Z, rows, n, stats, nseg, ids, tokens, (int32_t*)nullptr);
   return launch_pdl(sample_seg_kernel, dim3((rows + kWarps - 1) / kWarps),
                     dim3(kWarps * 32), 0, st, Z, rows, n, stats, nseg, cstats, ids, inv_tau,
                     seed, offset, tokens);
@@ -453,7 +519,7 @@ cudaError_t launch_verify(const float* Z, int sessions, int k, int n, const int3
                           int V, float inv_tau, const int32_t* draft, const float* q,
                           uint64_t seed, uint64_t offset, int32_t* n_acc,
                           int32_t* next_token, void* scratch, int sm_count,
-                          cudaStream_t st) {
+                          cudaStream_t st, int greedy) {
   const int R = sessions * (k + 1), nseg = seg_count(n), nchunk = chunk_count(nseg);
   char* p = static_cast<char*>(scratch);
   float2* stats = reinterpret_cast<float2*>(p);
@@ -470,6 +536,18 @@ cudaError_t launch_verify(const float* Z, int sessions, int k, int n, const int3
   p += align256((size_t)sessions * nseg * 4);
   float* resc = reinterpret_cast<float*>(p);
   cudaError_t e = launch_seg_stats(Z, R, n, inv_tau, stats, cstats, sm_count, st);
+  if (greedy) {
+    // the row maxima only: argmax per target row (into the normaliser
+    // area), then one thread per session
+    int32_t* amax = reinterpret_cast<int32_t*>(rowMS);
+    if (e == cudaSuccess)
+      e = launch_pdl(greedy_kernel, dim3((R + kWarps - 1) / kWarps), dim3(kWarps * 32), 0, st,
+                     Z, R, n, (const float2*)stats, nseg, ids, (int32_t*)nullptr, amax);
+    if (e == cudaSuccess)
+      e = launch_pdl(greedy_verify_kernel, dim3((sessions + 127) / 128), dim3(128), 0, st,
+                     (const int32_t*)amax, sessions, k, n, ids, V, draft, n_acc, next_token);
+    return e;
+  }
   if (e == cudaSuccess)
     e = launch_pdl(verify_rows_kernel, dim3((R + kWarps - 1) / kWarps), dim3(kWarps * 32), 0,
                    st, Z, (const float2*)cstats, nchunk, n, sessions, k, ids, V, inv_tau,

@@ -963,7 +963,7 @@ cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPl
                                      const void* scratch, float2* cstats,
                                      const int32_t* ids, float inv_tau, uint64_t seed,
                                      uint64_t offset, int sm_count, int32_t* tokens,
-                                     cudaStream_t st) {
+                                     cudaStream_t st, int greedy) {
   const char* sc = static_cast<const char*>(scratch);
   const float2* stats =
       reinterpret_cast<const float2*>(sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes);
@@ -972,9 +972,12 @@ cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPl
     cudaError_t e = launch_seg_stats(Z, rows, n, inv_tau, sst, cstats, sm_count, st);
     if (e != cudaSuccess) return e;
     return launch_sample_segments(Z, rows, n, sst, seg_count(n), cstats, ids, inv_tau, seed,
-                                  offset, tokens, st);
+                                  offset, tokens, st, greedy);
   }
   const int nseg = pl.NT * 4;
+  if (greedy)   // the segment maxima are all greedy decoding needs
+    return launch_sample_segments(Z, rows, n, stats, nseg, nullptr, ids, inv_tau, seed, offset,
+                                  tokens, st, 1);
   cudaError_t e = launch_chunk_stats(stats, rows, nseg, inv_tau, cstats, sm_count, st);
   if (e != cudaSuccess) return e;
   return launch_sample_segments(Z, rows, n, stats, nseg, cstats, ids, inv_tau, seed, offset,

@@ -158,6 +158,9 @@ size_t verify_reserve_bytes(int64_t rows, int64_t n) {
 }
 
 bool finite_pos(float x) { return std::isfinite(x) && x > 0.f; }
+// temperature: > 0 samples from softmax(z / t); 0 is greedy decoding
+bool valid_temperature(float t) { return std::isfinite(t) && t >= 0.f; }
+float stats_inv_tau(float t) { return t > 0.f ? 1.0f / t : 1.0f; }
 
 sph_status check_ids(sph_ctx* ctx, const int32_t* keep_ids, int64_t n_keep,
                      int64_t V) {
@@ -506,7 +509,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   if (ld_hl < d_l || ld_wl < d_l) return fail(ctx, SPH_ERR_INVALID_ARG, "ld_hl and ld_wl must be >= d_l");
   sph_status st = check_ids(ctx, keep_ids, n_keep, V);
   if (st) return st;
-  if (!finite_pos(temperature)) return fail(ctx, SPH_ERR_INVALID_ARG, "temperature must be finite and > 0");
+  if (!valid_temperature(temperature)) return fail(ctx, SPH_ERR_INVALID_ARG, "temperature must be finite and >= 0");
   if (((uintptr_t)W_l & 15) || ((ld_wl * 2) & 15))
     return fail(ctx, SPH_ERR_INVALID_ARG, "W_l base and row stride must be 16-byte aligned");
   if (n_keep > sph::sample_max_n()) return fail(ctx, SPH_ERR_UNSUPPORTED, "n_keep above %d", sph::sample_max_n());
@@ -526,7 +529,8 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   gg.ids = keep_ids; gg.n = (int)n_keep;
   gg.epilogue = sph::EPI_ENDPOINT;
   gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale; gg.status = ctx->status;
-  gg.inv_tau = 1.0f / temperature;
+  gg.inv_tau = stats_inv_tau(temperature);
+  const int greedy = temperature == 0.f;
   if (use_tc(ctx, rows, sph::W_BF16)) {
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0,
                                         ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
@@ -540,8 +544,8 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
     return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                            return sph::launch_sample_from_stats(
                                Z, (int)rows, (int)n_keep, pl, tcs, cstats, keep_ids,
-                               1.0f / temperature, seed, offset, ctx->sm_count, tokens,
-                               ctx->stream);
+                               gg.inv_tau, seed, offset, ctx->sm_count, tokens,
+                               ctx->stream, greedy);
                          }), "sample launch");
   }
   float2* stats = static_cast<float2*>(c.take((size_t)rows * sph::seg_count((int)n_keep) * 8));
@@ -551,14 +555,14 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   if (st) return st;
   return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                          cudaError_t e = sph::launch_seg_stats(Z, (int)rows, (int)n_keep,
-                                                               1.0f / temperature, stats,
+                                                               gg.inv_tau, stats,
                                                                cstats, ctx->sm_count,
                                                                ctx->stream);
                          if (e != cudaSuccess) return e;
                          return sph::launch_sample_segments(
                              Z, (int)rows, (int)n_keep, stats, sph::seg_count((int)n_keep),
-                             cstats, keep_ids, 1.0f / temperature, seed, offset, tokens,
-                             ctx->stream);
+                             cstats, keep_ids, gg.inv_tau, seed, offset, tokens,
+                             ctx->stream, greedy);
                        }), "sample launch");
 }
 
@@ -578,7 +582,7 @@ sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
   if (sessions * (k + 1) > (1 << 20))
     return fail(ctx, SPH_ERR_INVALID_ARG, "sessions * (k + 1) above 2^20 target rows");
   if (n_keep < 1 || n_keep > INT32_MAX) return fail(ctx, SPH_ERR_INVALID_ARG, "n_keep must be >= 1");
-  if (!finite_pos(temperature)) return fail(ctx, SPH_ERR_INVALID_ARG, "temperature must be finite and > 0");
+  if (!valid_temperature(temperature)) return fail(ctx, SPH_ERR_INVALID_ARG, "temperature must be finite and >= 0");
   if (n_keep > sph::sample_max_n()) return fail(ctx, SPH_ERR_UNSUPPORTED, "n_keep above %d", sph::sample_max_n());
   DeviceGuard g(ctx->device);
   if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
@@ -590,10 +594,11 @@ sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
   return launch_status(ctx, traced(ctx, SPH_PROF_VERIFY, [&] {
                          return sph::launch_verify(target_logits, (int)sessions, (int)k,
                                                    (int)n_keep, keep_ids, V,
-                                                   1.0f / temperature, draft_tokens,
+                                                   stats_inv_tau(temperature), draft_tokens,
                                                    draft_probs, seed, offset,
                                                    n_accepted, next_token, ctx->scratch,
-                                                   ctx->sm_count, ctx->stream);
+                                                   ctx->sm_count, ctx->stream,
+                                                   temperature == 0.f);
                        }), "verify launch");
 }
 

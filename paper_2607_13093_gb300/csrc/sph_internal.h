@@ -107,7 +107,8 @@ cudaError_t launch_sample_from_stats(const float* Z, int rows, int n,
                                      const TcPlan& plan, const void* scratch,
                                      float2* cstats, const int32_t* ids,
                                      float inv_tau, uint64_t seed, uint64_t offset,
-                                     int sm_count, int32_t* tokens, cudaStream_t st);
+                                     int sm_count, int32_t* tokens, cudaStream_t st,
+                                     int greedy = 0);
 
 // codes/row_scale from the clipped partials and their row maxima
 cudaError_t launch_quantize(const float* Y, const unsigned* rowmax, int rows,
@@ -134,11 +135,11 @@ cudaError_t launch_sample_segments(const float* Z, int rows, int n,
                                    const float2* stats, int nseg,
                                    const float2* cstats, const int32_t* ids,
                                    float inv_tau, uint64_t seed, uint64_t offset,
-                                   int32_t* tokens, cudaStream_t st);
+                                   int32_t* tokens, cudaStream_t st, int greedy = 0);
 int sample_max_n();
 int verify_max_k();
 
-// Speculative verification (four launches); `scratch` holds
+// Speculative verification (four launches; greedy: three); `scratch` holds
 // verify_scratch_bytes(sessions, k, n) bytes.
 size_t verify_scratch_bytes(int sessions, int k, int n);
 cudaError_t launch_verify(const float* Z, int sessions, int k, int n,
@@ -146,6 +147,6 @@ cudaError_t launch_verify(const float* Z, int sessions, int k, int n,
                           const int32_t* draft, const float* q,
                           uint64_t seed, uint64_t offset, int32_t* n_acc,
                           int32_t* next_token, void* scratch, int sm_count,
-                          cudaStream_t st);
+                          cudaStream_t st, int greedy = 0);
 
 }  // namespace sph

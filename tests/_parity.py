@@ -12,6 +12,7 @@ RTOL = 1e-3
 ATOL = 1e-3
 CODE_FRAC = 1e-3
 MARGIN = 1e-5
+GREEDY_GAP = 1e-4      # greedy decoding: top-two gap of the fp64 logits
 
 
 def bits(t: torch.Tensor) -> np.ndarray:
@@ -93,12 +94,19 @@ def check_endpoint(ctx, w, codes, scale, rows=None):
     zl = oracle.local_partial(hl[sel], bits(w.W_l), ids)
     zref = oracle.fuse(c[sel], s[sel], zl)
     assert_close(np_(z)[sel], zref, "fused logits")
-    u = oracle.philox_uniform(w.seed, sel, 0, w.offset)
-    j, margin = oracle.sample_rows(zref, w.tau, u)
+    if w.tau == 0:
+        # greedy: identical unless the top-two gap of the exact logits is
+        # within the fused logits' own rounding (GREEDY_GAP)
+        j, gap = oracle.greedy_rows(zref)
+        ok = gap >= GREEDY_GAP
+    else:
+        u = oracle.philox_uniform(w.seed, sel, 0, w.offset)
+        j, margin = oracle.sample_rows(zref, w.tau, u)
+        ok = margin >= MARGIN
     vocab = np.arange(w.V) if ids is None else ids
     want = vocab[j]
     got = np_(tok)[sel]
-    bad = (got != want) & (margin >= MARGIN)
+    bad = (got != want) & ok
     assert not bad.any(), f"tokens differ at rows {sel[bad]}: {got[bad]} vs {want[bad]}"
     assert np.isin(np_(tok), vocab).all(), "a masked id was sampled"
     return tok, z

@@ -194,6 +194,45 @@ def test_verify_many_sessions(ctx):
     assert 0 < (a == 0).sum() < S and 0 < (a == 1).sum() < S
 
 
+GREEDY_ENDPOINT = [
+    ("decode-like", dict(V=4000, d=1024, d_l=256, rows=32, n_keep=1500)),
+    ("gemv-rows", dict(V=3000, d=600, d_l=72, rows=3, n_keep=3000)),
+    ("stats-pass", dict(V=60000, d=640, d_l=128, rows=160, n_keep=40000)),
+]
+
+
+@pytest.mark.parametrize("name,kw", GREEDY_ENDPOINT, ids=[c[0] for c in GREEDY_ENDPOINT])
+def test_endpoint_greedy(path_ctx, name, kw):
+    # temperature 0: the first argmax of the fused logits
+    w = small(tau=0.0, **kw)
+    ref = oracle_cloud(w)
+    codes = torch.from_numpy(ref["codes"])
+    scale = torch.from_numpy(ref["row_scale"])
+    check_endpoint(path_ctx, w, codes, scale)
+
+
+@pytest.mark.parametrize("S,k,n", [(16, 4, 3000), (64, 2, 51302), (5, 1, 40)])
+def test_verify_greedy(ctx, S, k, n):
+    # temperature 0: drafts that follow the target's argmax for a random
+    # number of positions, then deviate
+    w = small(V=2 * n, d=96, d_l=8, rows=S * (k + 1), n_keep=n, sessions=S, k=k, tau=0.0)
+    target = wl.make_target_logits(w.rows, n, seed=S + k, std=2.0)
+    a = np.argmax(np_(target).astype(np.float64), axis=1).reshape(S, k + 1)
+    rng = np.random.default_rng(S)
+    ids = np_(w.keep_ids)
+    vocab = np.arange(w.V) if ids is None else ids
+    drafts = np.empty((S, k), dtype=np.int32)
+    for s in range(S):
+        cut = rng.integers(0, k + 1)
+        for i in range(k):
+            j = a[s, i] if i < cut else (a[s, i] + 1 + rng.integers(0, n - 1)) % n
+            drafts[s, i] = vocab[j]
+    w.draft_tokens = torch.from_numpy(drafts).to(DEV)
+    w.draft_probs = None
+    n_acc, _, ref = check_verify(ctx, w, target)
+    assert 0 < (np_(n_acc) > 0).sum() or S < 8
+
+
 def test_verify_accepts_drafts_equal_to_target(ctx):
     # q == p  =>  every draft accepted (r < 1 = p/q), bonus from p_k
     S, k, n = 6, 3, 500

@@ -428,3 +428,73 @@ def test_compact_index_brute_force():
     exp = [next((i for i, v in enumerate(ids) if v == t), -1) for t in toks]
     assert oracle.compact_index(ids, 14, toks).tolist() == exp
     assert oracle.compact_index(None, 5, np.array([0, 4, 5, -1])).tolist() == [0, 4, -1, -1]
+
+
+# ---------------------------------------------------------------------------
+# greedy decoding (temperature 0)
+# ---------------------------------------------------------------------------
+
+def test_greedy_rows_first_maximum_by_brute_force():
+    rng = np.random.default_rng(41)
+    z = rng.integers(-3, 4, size=(200, 9)).astype(np.float64)   # many ties
+    j, gap = oracle.greedy_rows(z)
+    for r in range(z.shape[0]):
+        m = max(z[r])
+        first = min(i for i in range(z.shape[1]) if z[r, i] == m)
+        assert j[r] == first
+        rest = sorted(z[r])[-2]
+        assert gap[r] == m - rest
+    assert (gap[np.array([np.sum(z[r] == z[r].max()) > 1 for r in range(200)])] == 0).all()
+
+
+def test_greedy_is_the_small_temperature_limit_of_sampling():
+    # well separated maxima: softmax(z / tau) puts all mass on the argmax for
+    # tiny tau, so every uniform draws it
+    rng = np.random.default_rng(42)
+    z = rng.normal(size=(50, 300)) * 3
+    j, gap = oracle.greedy_rows(z)
+    keep = gap > 0.05
+    u = rng.random(50)
+    js, _ = oracle.sample_rows(z, 1e-4, u)
+    assert (js[keep] == j[keep]).all()
+
+
+def test_fuse_sample_tau_zero_is_argmax_of_fused_logits():
+    rng = np.random.default_rng(43)
+    V, dl, R, n = 300, 12, 5, 120
+    ids = np.sort(rng.choice(V, n, replace=False))
+    W = rng.normal(size=(V, dl)) * 0.02
+    Wb = (np.asarray(W, dtype=np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    codes = rng.integers(-127, 128, size=(R, n)).astype(np.int8)
+    scale = (rng.random(R) * 0.2 + 0.01).astype(np.float32)
+    h = rng.normal(size=(R, dl)).astype(np.float32)
+    out = oracle.fuse_sample(codes, scale, h, Wb, keep_ids=ids, tau=0)
+    z = oracle.fuse(codes, scale, oracle.local_partial(h, Wb, ids))
+    assert (out["tokens"] == ids[np.argmax(z, axis=1)]).all()
+
+
+def test_greedy_verify_matches_its_closed_form_and_the_small_tau_limit():
+    rng = np.random.default_rng(44)
+    S, k, n = 40, 3, 50
+    Z = (rng.normal(size=(S * (k + 1), n)) * 4).astype(np.float32)
+    a = np.argmax(Z.astype(np.float64), axis=1).reshape(S, k + 1)
+    # drafts: the argmax for a random prefix, then something else
+    drafts = np.empty((S, k), dtype=np.int64)
+    for s in range(S):
+        cut = rng.integers(0, k + 1)
+        for i in range(k):
+            drafts[s, i] = a[s, i] if i < cut else (a[s, i] + 1 + rng.integers(0, n - 1)) % n
+    out = oracle.verify_draft(Z, S, k, tau=0, draft_tokens=drafts, draft_probs=None)
+    for s in range(S):
+        i = 0
+        while i < k and drafts[s, i] == a[s, i]:
+            i += 1
+        assert out["n_accepted"][s] == i
+        assert out["next_token"][s] == a[s, i]
+        # the stochastic rule at a tiny temperature reaches the same result
+        # (greedy one-hot drafts; p is one-hot up to exp(-gap / tau))
+        P = oracle.softmax_rows(Z[s * (k + 1):(s + 1) * (k + 1)].astype(np.float64), 1e-3)
+        acc, j, _, _ = oracle.verify_core(P, None, drafts[s], np.full(k, 0.5), 0.5)
+        gaps = oracle.greedy_rows(Z[s * (k + 1):(s + 1) * (k + 1)])[1]
+        if gaps.min() > 0.05:
+            assert acc == i and j == a[s, i]
