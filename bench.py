@@ -76,9 +76,10 @@ def parse():
     ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="decode",
-                    choices=["tiny", "decode", "spec", "fp8", "sweep"])
-    ap.add_argument("--rows", type=int, default=None, help="sweep: rows")
-    ap.add_argument("--keep", type=float, default=None, help="sweep: keep fraction")
+                    choices=["tiny", "decode", "spec", "fp8", "sweep", "dend"])
+    ap.add_argument("--rows", type=int, default=None, help="sweep / dend: rows")
+    ap.add_argument("--keep", type=float, default=None, help="sweep / dend: keep fraction")
+    ap.add_argument("--d-l", type=int, default=None, help="dend: split dimension d_l")
     ap.add_argument("--e2e-steps", type=int, default=300)
     ap.add_argument("--act", choices=["fp32", "bf16"], default="fp32",
                     help="cloud activations: fp32 (exact, two bf16 planes) or bf16-rounded")
@@ -296,7 +297,8 @@ def run_ours(args):
         dist.barrier()
     from paper_2607_13093_gb300 import sph, workloads as wl
 
-    w = wl.workload(args.workload, device=dev, rows=args.rows, keep_frac=args.keep)
+    w = wl.workload(args.workload, device=dev, rows=args.rows, keep_frac=args.keep,
+                    d_l=args.d_l)
     if world > 1:                       # each rank: its own sessions
         g = torch.Generator(device=dev)
         g.manual_seed(rank_seed(rank))
@@ -532,7 +534,8 @@ def run_reference(args):
     if rank != 0:
         return
     from paper_2607_13093_gb300 import workloads as wl
-    w = wl.workload(args.workload, device="cpu", rows=args.rows, keep_frac=args.keep)
+    w = wl.workload(args.workload, device="cpu", rows=args.rows, keep_frac=args.keep,
+                    d_l=args.d_l)
     s = OracleSample(w, args.act)
     budget = 150.0
     L = s.calibrate(budget / max(1, args.steps + args.warmup))

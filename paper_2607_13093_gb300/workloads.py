@@ -16,6 +16,8 @@ the vocabulary) and the five workloads used throughout this package:
   fp8       d=8192 (d_l=1024, d_h=7168), V=152064, R=256, full vocab, W_h e4m3
   sweep     d=5120 (d_l=512,  d_h=4608), V=256000, R in {1,8,64,256,1024},
             keep in {10 %, 50 %, 100 %}
+  dend      d=4096 (d_l in {48, 96, 128, 256, 512}), V=150000, R=32,
+            keep 40 % or 30 % (the paper's split-dimension study)
 
 Input recipe (every workload):
   * W_lm is stored vocab-major, W[V, d] ~ N(0, 0.02) rounded to bf16 (RNE);
@@ -57,6 +59,8 @@ WORKLOADS = {
                 clip=40.0, tau=1.0, w_dtype="fp8"),
     "sweep": dict(num=5, d=5120, d_l=512, V=256000, rows=64, n_keep=256000,
                   clip=30.0, tau=1.0, w_dtype="bf16"),
+    "dend": dict(num=6, d=4096, d_l=96, V=150000, rows=32, n_keep=round(0.4 * 150000),
+                 clip=30.0, tau=1.0, w_dtype="bf16"),
 }
 SWEEP_ROWS = (1, 8, 64, 256, 1024)
 SWEEP_KEEP = (0.10, 0.50, 1.00)
@@ -257,18 +261,22 @@ def make_workload(name: str = "custom", *, V: int, d: int, d_l: int, rows: int,
 
 
 def workload(name: str, device="cpu", rows: Optional[int] = None,
-             keep_frac: Optional[float] = None) -> Workload:
-    """One of the five named workloads at full size.  For "sweep", `rows`
-    and `keep_frac` pick the grid point (defaults 64 rows, 100 %)."""
+             keep_frac: Optional[float] = None, d_l: Optional[int] = None) -> Workload:
+    """One of the named workloads at full size.  For "sweep" and "dend",
+    `rows` and `keep_frac` pick the grid point (defaults: sweep 64 rows,
+    100 %; dend 32 rows, 40 %), and for "dend" `d_l` the split dimension
+    (default 96, the paper's D_end)."""
     cfg = dict(WORKLOADS[name])
     num = cfg.pop("num")
     sessions = cfg.pop("sessions", 0)
     k = cfg.pop("k", 0)
-    if name == "sweep":
+    if name in ("sweep", "dend"):
         if rows is not None:
             cfg["rows"] = rows
         if keep_frac is not None:
             cfg["n_keep"] = round(keep_frac * cfg["V"])
+    if name == "dend" and d_l is not None:
+        cfg["d_l"] = d_l
     return make_workload(name, seed=1000 + num, device=device,
                          sessions=sessions, k=k, **cfg)
 
