@@ -516,6 +516,14 @@ def run_ours(args):
                          "tokens -> host, sync per step")},
         "timed_loop": f"CUDA graph of {gsteps} steps replayed {reps}x (+{rem} steps)",
         "clocks": clocks,
+        # downlink of one step (Eq. 21 with b = 8, no tag/metadata/padding):
+        # int8 codes of the kept ids + an fp32 scale per row, against the full
+        # vocabulary as int8 and as fp32 logits
+        "payload": {"bytes_per_step": sph.sph_payload_bytes(R, n),
+                    "full_vocab_int8_bytes": sph.sph_payload_bytes(R, w.V),
+                    "full_vocab_fp32_bytes": 4 * R * w.V,
+                    "reduction_vs_full_int8": round(
+                        1 - sph.sph_payload_bytes(R, n) / sph.sph_payload_bytes(R, w.V), 4)},
     }
     if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act)

@@ -320,3 +320,48 @@ def test_fp8_tensor_core(ctx, rows, keep, act):
             check_cloud(ctx, w, act_mode=act)
     finally:
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+
+
+# ---------------------------------------------------------------------------
+# CUDA-graph capture (as the benchmark times the step) = direct calls
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("rows_kw", [dict(rows=20, sessions=4, k=4), dict(rows=3, sessions=1, k=2)])
+def test_graph_capture_matches_direct_calls(ctx, rows_kw):
+    w = small(V=6000, d=640, d_l=128, n_keep=2400, **rows_kw)
+    ctx.reserve(w.rows, w.n_keep, max(w.d_h, w.d_l))
+    target = wl.make_target_logits(w.rows, w.n_keep, seed=31, std=1.0).to(DEV)
+    R, n, S = w.rows, w.n_keep, w.sessions
+    codes = torch.empty(R, n, dtype=torch.int8, device=DEV)
+    scale = torch.empty(R, device=DEV)
+    tokens = torch.empty(R, dtype=torch.int32, device=DEV)
+    z = torch.empty(R, n, device=DEV)
+    n_acc = torch.empty(S, dtype=torch.int32, device=DEV)
+    nxt = torch.empty(S, dtype=torch.int32, device=DEV)
+
+    def step():
+        ctx.partial_logits(w.h_cloud, w.W_h, keep_ids=w.keep_ids, clip=w.clip, codes=codes,
+                           row_scale=scale)
+        ctx.fuse_sample(codes, scale, w.h_local, w.W_l, keep_ids=w.keep_ids, temperature=w.tau,
+                        seed=w.seed, offset=7, tokens=tokens, fused_logits_out=z)
+        ctx.verify_draft(target, S, w.k, w.draft_tokens, keep_ids=w.keep_ids,
+                         draft_probs=w.draft_probs, temperature=w.tau, seed=w.seed, offset=9,
+                         n_accepted=n_acc, next_token=nxt)
+
+    step()
+    ctx.sync()
+    ref = [t.clone() for t in (codes, scale, tokens, z, n_acc, nxt)]
+    for t in (codes, scale, tokens, z, n_acc, nxt):
+        t.zero_()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    cs = torch.cuda.Stream(device=DEV)
+    cs.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.graph(g, stream=cs):
+        step()
+    g.replay()
+    g.replay()
+    torch.cuda.synchronize()
+    ctx.sync()
+    for a, b in zip(ref, (codes, scale, tokens, z, n_acc, nxt)):
+        assert torch.equal(a, b)
