@@ -57,6 +57,7 @@ constexpr int kTileM = 128;          // vocabulary rows per tile (MMA M)
 constexpr int kAtomK = 64;           // bf16 elements per 128-byte swizzle atom
 constexpr int kAtomBytes = kTileM * kAtomK * 2;   // one A atom: 128 rows x 128 B
 constexpr int kMaxBN = 256;
+constexpr int kMaxStages = 12;       // (the barrier area holds (3 * 12 + 5) words)
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
 
@@ -66,7 +67,8 @@ constexpr int kThreads = 64 + 32 * kEpiWarps;       // producer, MMA, epilogue
 constexpr int kThreadsFp8 = kThreads + 128;         // + four converter warps (fp8)
 constexpr int kMaxBNFp8 = 128;       // h rows per block with fp8 weights
 constexpr int kBoxHeights = 128;     // row boxes of 1, 2, 3, ..., 128 rows (map h-1)
-constexpr int kMaxBoxes = 128;       // row boxes of one tile (one per run)
+constexpr int kMaxBoxes = 260;       // row boxes of one tile (one per run, two per
+                                     // run longer than 128 rows in a 256-row tile)
 
 // W tensor maps: box height 2^i rows for map i (64 columns each).
 struct WMaps {
@@ -76,6 +78,7 @@ struct WMaps {
 
 struct TcParams {
   int R, n, K, KB, NT, RB, BN, Rp, stages, whole_tiles;
+  int nseg;                    // endpoint statistics: 32-id segments per row (NT * TM / 32)
   int na;                      // swizzle atoms per k-block (k-block = 64 * na)
   long long T;                 // total iterations RB * NT * KB
   const int32_t* ids;          // gather path: sorted ids
@@ -91,10 +94,10 @@ struct TcParams {
   const int8_t* codes;
   const float* row_scale;
   float inv_tau;
-  float2* seg_stats;
-  int a3d;                     // full vocabulary: A by one 3-D copy per stage           // endpoint: [R][NT*4] (max, sum exp)
-  float* P;                    // split-tile partials [2 * grid][BN][128]
-  int* counters;               // [tiles][4 quadrants], zero between calls
+  float2* seg_stats;           // endpoint: [R][nseg] (max, sum exp)
+  int a3d;                     // full vocabulary: A by one 3-D copy per stage
+  float* P;                    // split-tile partials [2 * grid][BN][TM]
+  int* counters;               // [tiles][4 quadrants][epilogue groups], zero between calls
   unsigned* status;
   long long spin_limit;
 };
@@ -206,20 +209,28 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
     }
     const float sk = warp_reduce_scatter16(e, SumOp{}, lane);
     if (!(lane & 1) && row0 + kr < p.R)
-      p.seg_stats[(int64_t)(row0 + kr) * (p.NT * 4) + seg] = make_float2(mk, sk);
+      p.seg_stats[(int64_t)(row0 + kr) * p.nseg + seg] = make_float2(mk, sk);
   }
 }
 
-template <int HILO, bool GATHER, int EPI, bool FP8>
+// TM = vocabulary rows per tile: 128, or 256 as two M = 128 MMAs that share
+// each B stage (half the B bytes per A byte; TMEM holds 2 x 2 x BN columns)
+template <int HILO, bool GATHER, int EPI, bool FP8, int TM>
 __global__ void __launch_bounds__(FP8 ? kThreadsFp8 : kThreads, 1)
 tc_kernel(const __grid_constant__ WMaps wm,
           const __grid_constant__ CUtensorMap tmH, const TcParams p) {
+  static_assert(TM == 128 || TM == 256, "tile height");
+  static_assert(!FP8 || TM == 128, "fp8 converter warps fill 128-row tiles");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* base = smem_raw + (((raw_addr + 1023) & ~1023u) - raw_addr);
+  constexpr int kHalves = TM / 128;     // M = 128 halves of a tile
+  constexpr int kGroups = TM / 32;      // 32-row lane groups of a tile
   const int BN = p.BN;
   const int NA = p.na;
-  const int a_bytes = NA * kAtomBytes;
+  // A: per atom the TM tile rows at 128-byte stride (half h at h * 16 KB)
+  const int atom_bytes = kHalves * kAtomBytes;
+  const int a_bytes = NA * atom_bytes;
   const int b_bytes = HILO * NA * BN * 128;
   const int stage_bytes = a_bytes + b_bytes;
   const int S = p.stages;
@@ -234,8 +245,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
   int2* s_box = reinterpret_cast<int2*>(base + (size_t)S * stage_bytes + 256);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  uint32_t ncols = 32;
-  while (ncols < (uint32_t)(2 * BN)) ncols <<= 1;
+  uint32_t ncols = 32;                 // two accumulators of kHalves x BN columns
+  while (ncols < (uint32_t)(2 * kHalves * BN)) ncols <<= 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -290,12 +301,14 @@ tc_kernel(const __grid_constant__ WMaps wm,
     __syncwarp();
     // subset path: the ids of a segment's tile are loaded one segment ahead,
     // so that planning a tile never waits on memory
-    int nid[4] = {0, 0, 0, 0};
-    auto load_ids = [&](int tl, int (&dst)[4]) {
-      const int j0 = (tl / p.RB) * kTileM;
-      const int rows = min(kTileM, p.n - j0);
+    int nid[kGroups];
 #pragma unroll
-      for (int g = 0; g < 4; ++g) {
+    for (int g = 0; g < kGroups; ++g) nid[g] = 0;
+    auto load_ids = [&](int tl, int (&dst)[kGroups]) {
+      const int j0 = (tl / p.RB) * TM;
+      const int rows = min(TM, p.n - j0);
+#pragma unroll
+      for (int g = 0; g < kGroups; ++g) {
         const int r = 32 * g + lane;
         dst[g] = r < rows ? p.ids[j0 + r] : 0;
       }
@@ -307,23 +320,25 @@ tc_kernel(const __grid_constant__ WMaps wm,
     }
     while (!stop && sg.next(tile, kb0, kb1)) {
       const int t = tile / p.RB, rb = tile - t * p.RB;
-      int2 box[4];                               // (first id, row | (rows - 1) << 8)
+      int2 box[2 * kGroups];                     // (first id, row | (rows - 1) << 8)
       unsigned bmask = 0;                        // which of box[] are in use
       int nbox = 0;
       uint32_t tx = (uint32_t)(FP8 ? b_bytes : stage_bytes);
       if constexpr (GATHER && !FP8) {
-        const int j0 = t * kTileM;
-        const int rows = min(kTileM, p.n - j0);
-        int idr[4] = {nid[0], nid[1], nid[2], nid[3]};
+        const int j0 = t * TM;
+        const int rows = min(TM, p.n - j0);
+        int idr[kGroups];
+#pragma unroll
+        for (int g = 0; g < kGroups; ++g) idr[g] = nid[g];
         {
           Segments pk = sg;
           int tn, a0, a1;
           if (pk.next(tn, a0, a1)) load_ids(tn, nid);
         }
-        unsigned smask[4];
+        unsigned smask[kGroups];
         int prev_last = 0;
 #pragma unroll
-        for (int g = 0; g < 4; ++g) {
+        for (int g = 0; g < kGroups; ++g) {
           const int r = 32 * g + lane;
           int prev = __shfl_up_sync(0xFFFFFFFFu, idr[g], 1);
           if (lane == 0) prev = prev_last;
@@ -332,7 +347,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
         }
         int covered = 0;
 #pragma unroll
-        for (int g = 0; g < 4; ++g) {
+        for (int g = 0; g < kGroups; ++g) {
           const int r = 32 * g + lane;
           if ((smask[g] >> lane) & 1u) {
             int nxt = rows;
@@ -340,12 +355,18 @@ tc_kernel(const __grid_constant__ WMaps wm,
             if (above) {
               nxt = 32 * g + __ffs(above) - 1;
             } else {
-              for (int g2 = g + 1; g2 < 4; ++g2)
+              for (int g2 = g + 1; g2 < kGroups; ++g2)
                 if (smask[g2]) { nxt = 32 * g2 + __ffs(smask[g2]) - 1; break; }
             }
-            const int len = nxt - r;               // 1..128: one box of exactly len rows
-            box[g] = make_int2(idr[g], r | ((len - 1) << 8));
-            bmask |= 1u << g;
+            // one box of exactly len rows (two, 128 + rest, past 128 rows)
+            const int len = nxt - r;
+            const int l0 = min(len, 128);
+            box[2 * g] = make_int2(idr[g], r | ((l0 - 1) << 8));
+            bmask |= 1u << (2 * g);
+            if (len > 128) {
+              box[2 * g + 1] = make_int2(idr[g] + 128, (r + 128) | ((len - 129) << 8));
+              bmask |= 2u << (2 * g);
+            }
             covered += len;
           }
         }
@@ -365,7 +386,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
         nbox = __shfl_sync(0xFFFFFFFFu, incl, 31);
         int slot = incl - mine;
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
+        for (int q = 0; q < 2 * kGroups; ++q)
           if ((bmask >> q) & 1u) s_box[slot++] = box[q];
         __syncwarp();
       }
@@ -386,19 +407,20 @@ tc_kernel(const __grid_constant__ WMaps wm,
         // copy of all NA atoms (fp8: none; the converter warps fill A); B as
         // one 3-D copy of all NA atoms per plane
         uint8_t* A = base + (size_t)stage * stage_bytes;
-        const int nA = FP8 ? 0 : (GATHER ? NA * nbox : (p.a3d ? 1 : NA));
+        const int nA = FP8 ? 0 : (GATHER ? NA * nbox : (p.a3d ? 1 : NA * kHalves));
         for (int op = lane; op < nA + HILO; op += 32) {
           if (op < nA) {
             if constexpr (GATHER) {
               const int a = op / nbox;
               const int2 bx = s_box[op - a * nbox];
-              ptx::tma_load_2d(A + a * kAtomBytes + (bx.y & 0xFF) * 128, &wm.m[bx.y >> 8],
+              ptx::tma_load_2d(A + a * atom_bytes + (bx.y & 0xFF) * 128, &wm.m[bx.y >> 8],
                                (kb * NA + a) * kAtomK, bx.x, &full[stage]);
             } else if (p.a3d) {
-              ptx::tma_load_3d(A, &wm.a3, 0, t * kTileM, kb * NA, &full[stage]);
+              ptx::tma_load_3d(A, &wm.a3, 0, t * TM, kb * NA, &full[stage]);
             } else {
-              ptx::tma_load_2d(A + op * kAtomBytes, &wm.m[kBoxHeights - 1],
-                               (kb * NA + op) * kAtomK, t * kTileM, &full[stage]);
+              const int a = op / kHalves, hf = op - a * kHalves;
+              ptx::tma_load_2d(A + a * atom_bytes + hf * kAtomBytes, &wm.m[kBoxHeights - 1],
+                               (kb * NA + a) * kAtomK, t * TM + hf * 128, &full[stage]);
             }
           } else {
             const int h = op - nA;
@@ -425,6 +447,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
       int si = 0, tile, kb0, kb1;
       const uint32_t idesc =
           FP8 ? ptx::idesc_f16_f32(kTileM, BN) : ptx::idesc_bf16_f32(kTileM, BN);
+      // accumulator `acc`, tile half hf: TMEM columns (acc * kHalves + hf) * BN
       bool stop = false;
       while (!stop && sg.next(tile, kb0, kb1)) {
         const int acc = si & 1;
@@ -434,7 +457,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
         }
         tph[acc] ^= 1;
         ptx::tc_fence_after();
-        const uint32_t d = tmem_base + (uint32_t)(acc * BN);
+        const uint32_t d = tmem_base + (uint32_t)(acc * kHalves * BN);
         for (int kb = kb0; kb < kb1; ++kb) {
           if (*s_abort || !ptx::mbar_wait(&full[stage], phase, limit)) {
             if (!*s_abort) give_up();
@@ -449,9 +472,12 @@ tc_kernel(const __grid_constant__ WMaps wm,
             for (int h = 0; h < HILO; ++h) {
 #pragma unroll
               for (int kk = 0; kk < kAtomK / 16; ++kk) {
-                ptx::umma_f16(d, ptx::sdesc_k128(a0 + at * kAtomBytes + kk * 32),
-                               ptx::sdesc_k128(b0 + (h * NA + at) * BN * 128 + kk * 32),
-                               idesc, (kb != kb0 || at != 0 || h != 0 || kk != 0) ? 1u : 0u);
+#pragma unroll
+                for (int hf = 0; hf < kHalves; ++hf)
+                  ptx::umma_f16(d + (uint32_t)(hf * BN),
+                                ptx::sdesc_k128(a0 + at * atom_bytes + hf * kAtomBytes + kk * 32),
+                                ptx::sdesc_k128(b0 + (h * NA + at) * BN * 128 + kk * 32), idesc,
+                                (kb != kb0 || at != 0 || h != 0 || kk != 0) ? 1u : 0u);
               }
             }
           }
@@ -472,7 +498,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
     // 4); the two warps of a quadrant take alternate 16-column chunks.
     const int quad = warp & 3;
     const int grp = (warp - 2) >> 2;
-    const int i = quad * 32 + lane;              // vocabulary row in the tile
+    const int nch = BN / 16;                     // 16-column chunks per tile half
+    const int nhc = kHalves * nch;               // (half, chunk) pairs, hc = hf * nch + ch
     ptx::griddep_wait();
     Segments sg{it0, it1, p.KB};
     uint32_t fph[2] = {0, 0};
@@ -481,15 +508,28 @@ tc_kernel(const __grid_constant__ WMaps wm,
       const int acc = si & 1;
       const int t = tile / p.RB, rb = tile - t * p.RB;
       const bool whole = kb0 == 0 && kb1 == p.KB;
-      const int j = t * kTileM + i;
-      const bool vj = j < p.n;
-      const int id = vj ? (GATHER ? p.ids[j] : j) : 0;
+      // this lane's vocabulary row in each half: i = hf * 128 + quad * 32 + lane
+      int jh[kHalves], idh[kHalves];
+      bool vjh[kHalves];
+#pragma unroll
+      for (int hf = 0; hf < kHalves; ++hf) {
+        jh[hf] = t * TM + hf * 128 + quad * 32 + lane;
+        vjh[hf] = jh[hf] < p.n;
+        idh[hf] = vjh[hf] ? (GATHER ? p.ids[jh[hf]] : jh[hf]) : 0;
+      }
+      // (selects, not a runtime-indexed array, for the loops' half index)
+      auto J = [&](int hf) { return (kHalves > 1 && hf) ? jh[kHalves - 1] : jh[0]; };
+      auto VJ = [&](int hf) { return (kHalves > 1 && hf) ? vjh[kHalves - 1] : vjh[0]; };
+      auto ID = [&](int hf) { return (kHalves > 1 && hf) ? idh[kHalves - 1] : idh[0]; };
       Payload pay;
       if constexpr (EPI == EPI_ENDPOINT) {
         // the payload does not depend on the accumulator: start on it
         // while the tile's MMAs run
-        prefetch_codes(p, rb * BN + grp * (BN / 2), BN / 2, t * kTileM + quad * 32, lane);
-        if (whole && grp < BN / 16) load_payload(p, rb * BN + grp * 16, t * kTileM + i, lane, pay);
+#pragma unroll
+        for (int hf = 0; hf < kHalves; ++hf)
+          prefetch_codes(p, rb * BN + grp * (BN / 2), BN / 2, t * TM + hf * 128 + quad * 32, lane);
+        if (whole && grp < nhc)
+          load_payload(p, rb * BN + (grp % nch) * 16, J(grp / nch), lane, pay);
       }
       int ok = 1;
       if (lane == 0) ok = !*s_abort && ptx::mbar_wait(&tfull[acc], fph[acc], limit);
@@ -500,32 +540,36 @@ tc_kernel(const __grid_constant__ WMaps wm,
       }
       fph[acc] ^= 1;
       ptx::tc_fence_after();
-      const int seg = t * 4 + quad;
-      const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * BN);
+      const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) +
+                             (uint32_t)(acc * kHalves * BN);
       // a CTA's split tiles can only be its first and its last segment:
-      // slot 2c holds the first, 2c+1 the last
-      float* Pt = p.P + (size_t)(2 * blockIdx.x + (si == 0 ? 0 : 1)) * BN * kTileM;
-      for (int ch = grp; ch < BN / 16; ch += kEpiGroups) {
+      // slot 2c holds the first, 2c+1 the last ([BN][TM] each)
+      float* Pt = p.P + (size_t)(2 * blockIdx.x + (si == 0 ? 0 : 1)) * BN * TM;
+      for (int hc = grp; hc < nhc; hc += kEpiGroups) {
+        const int hf = hc / nch, ch = hc - hf * nch;
+        const int i = hf * 128 + quad * 32 + lane;
         float v[16];
-        ptx::tmem_ld16(taddr + ch * 16, v);
+        ptx::tmem_ld16(taddr + hf * BN + ch * 16, v);
         if (whole) {
           Payload nxt;
-          if (EPI == EPI_ENDPOINT && ch + kEpiGroups < BN / 16)
-            load_payload(p, rb * BN + (ch + kEpiGroups) * 16, j, lane, nxt);
-          finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg, pay);
+          const int hn = hc + kEpiGroups;
+          if (EPI == EPI_ENDPOINT && hn < nhc)
+            load_payload(p, rb * BN + (hn % nch) * 16, J(hn / nch), lane, nxt);
+          finish_chunk<EPI>(p, v, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
+                            t * kGroups + hf * 4 + quad, pay);
           if constexpr (EPI == EPI_ENDPOINT) pay = nxt;
         } else {
 #pragma unroll
-          for (int q = 0; q < 16; ++q) Pt[(size_t)(ch * 16 + q) * kTileM + i] = v[q];
+          for (int q = 0; q < 16; ++q) Pt[(size_t)(ch * 16 + q) * TM + i] = v[q];
         }
       }
       ptx::tc_fence_before();
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(&tempty[acc]);
       if (!whole) {
-        // split tile: this warp's 32 vocabulary rows x its chunks are
-        // finished by the last warp (over all contributing CTAs) of the same
-        // quadrant and chunk group
+        // split tile: this warp's rows x its chunks are finished by the last
+        // warp (over all contributing CTAs) of the same quadrant and chunk
+        // group
         __threadfence();
         int old = 0;
         const int cnt = (tile * 4 + quad) * kEpiGroups + grp;
@@ -547,27 +591,29 @@ tc_kernel(const __grid_constant__ WMaps wm,
 #pragma unroll
           for (int c = 0; c < kMaxC; ++c) {
             const int slot = c == 0 ? 2 * c0 + (c0_first ? 0 : 1) : 2 * (c0 + (c < C ? c : 0));
-            ps[c] = p.P + (size_t)slot * BN * kTileM + i;
+            ps[c] = p.P + (size_t)slot * BN * TM + quad * 32 + lane;
           }
-          for (int ch = grp; ch < BN / 16; ch += kEpiGroups) {
-            if constexpr (EPI == EPI_ENDPOINT) load_payload(p, rb * BN + ch * 16, j, lane, pay);
+          for (int hc = grp; hc < nhc; hc += kEpiGroups) {
+            const int hf = hc / nch, ch = hc - hf * nch;
+            if constexpr (EPI == EPI_ENDPOINT) load_payload(p, rb * BN + ch * 16, J(hf), lane, pay);
+            const size_t o = (size_t)ch * 16 * TM + hf * 128;
             float v[16];
 #pragma unroll
-            for (int q = 0; q < 16; ++q) v[q] = __ldcg(ps[0] + (size_t)(ch * 16 + q) * kTileM);
+            for (int q = 0; q < 16; ++q) v[q] = __ldcg(ps[0] + o + (size_t)q * TM);
 #pragma unroll
             for (int c = 1; c < kMaxC; ++c) {
               if (c < C) {
 #pragma unroll
-                for (int q = 0; q < 16; ++q)
-                  v[q] += __ldcg(ps[c] + (size_t)(ch * 16 + q) * kTileM);
+                for (int q = 0; q < 16; ++q) v[q] += __ldcg(ps[c] + o + (size_t)q * TM);
               }
             }
             for (int c = kMaxC; c < C; ++c) {    // rare: very many contributors
-              const float* pc = p.P + (size_t)(2 * (c0 + c)) * BN * kTileM + i;
+              const float* pc = p.P + (size_t)(2 * (c0 + c)) * BN * TM + quad * 32 + lane;
 #pragma unroll
-              for (int q = 0; q < 16; ++q) v[q] += __ldcg(pc + (size_t)(ch * 16 + q) * kTileM);
+              for (int q = 0; q < 16; ++q) v[q] += __ldcg(pc + o + (size_t)q * TM);
             }
-            finish_chunk<EPI>(p, v, rb * BN + ch * 16, j, vj, id, lane, seg, pay);
+            finish_chunk<EPI>(p, v, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
+                              t * kGroups + hf * 4 + quad, pay);
           }
           if (lane == 0) p.counters[cnt] = 0;
         }
@@ -805,7 +851,8 @@ bool w_maps(const GatherGemm& g, bool gather, WMaps& out) {
 }  // namespace
 
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
-               int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn_opt) {
+               int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn_opt,
+               int tile_m) {
   TcPlan pl{};
   // one bf16 plane carries bf16-rounded activations exactly; f16 planes
   // (fp8 weights) always take two
@@ -817,26 +864,41 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   // than in two 256-row ones)
   if (!fp8 && pl.hilo == 2 && max_bn > 224) max_bn = 224;
   if (max_bn_opt >= 16 && max_bn_opt < max_bn) max_bn = max_bn_opt;
-  if (rows <= max_bn) {
-    pl.RB = 1;
-    pl.BN = (rows + 15) / 16 * 16;
-  } else {
-    pl.RB = (rows + max_bn - 1) / max_bn;
-    pl.BN = ((rows + pl.RB - 1) / pl.RB + 15) / 16 * 16;
-  }
+  auto row_blocks = [&](int cap) {
+    if (rows <= cap) {
+      pl.RB = 1;
+      pl.BN = (rows + 15) / 16 * 16;
+    } else {
+      pl.RB = (rows + cap - 1) / cap;
+      pl.BN = ((rows + pl.RB - 1) / pl.RB + 15) / 16 * 16;
+    }
+  };
+  row_blocks(max_bn);
+  // 256-id tiles: two M = 128 MMAs share every B stage, which halves the
+  // B bytes per A byte, but their two double-buffered accumulators hold at
+  // most 128 hidden-state rows per row block and the tiles are half as
+  // many.  Automatic: only where the row blocks already have <= 128 rows,
+  // the hidden dimension is long and every SM gets >= 4 tiles (measured,
+  // fp32 h: 64 rows x 256000 ids x 4608 is 29 % and 256 rows 19 % faster;
+  // 32 rows x 60000 ids, 320 rows x 51302 ids and 208-row blocks slower).
+  const bool tm256_auto = tile_m == 0 && pl.BN <= 128 && K >= 2048 &&
+                          (long long)pl.RB * ((n + 255) / 256) >= 4ll * sm_count;
+  pl.tm = (!fp8 && (tile_m == 256 || tm256_auto)) ? 256 : 128;
+  const int halves = pl.tm / 128;
+  if (pl.tm == 256 && pl.BN > 128) row_blocks(max_bn < 128 ? max_bn : 128);
   pl.Rp = pl.RB * pl.BN;
   // k-block width: as asked (automatic: 128), narrowed until the shared
   // memory holds at least min_stages pipeline stages
   pl.na = fp8 ? 1 : (block_k == 64 ? 1 : (block_k == 256 ? 4 : 2));
   const int min_stages = block_k ? 2 : 4;
   while (pl.na > 1 &&
-         (int)((kSmemBudget - 2048) / (pl.na * (kAtomBytes + pl.hilo * pl.BN * 128))) <
+         (int)((kSmemBudget - 2048) / (pl.na * (halves * kAtomBytes + pl.hilo * pl.BN * 128))) <
              min_stages)
     pl.na >>= 1;
   const int bk = pl.na * kAtomK;
   pl.KB = (K + bk - 1) / bk;
   pl.Kp = pl.KB * bk;
-  pl.NT = (n + kTileM - 1) / kTileM;
+  pl.NT = (n + pl.tm - 1) / pl.tm;
   const int tiles = pl.RB * pl.NT;
   pl.T = (long long)tiles * pl.KB;
   // whole tiles per CTA unless that leaves the grid clearly unbalanced
@@ -845,9 +907,9 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   const double split_span = (double)pl.T / (pl.T < sm_count ? pl.T : sm_count);
   pl.whole_tiles = schedule == 1 || (schedule == 0 && whole_span <= 1.1 * split_span + 2.0);
   pl.G = pl.whole_tiles ? g_whole : (int)(pl.T < sm_count ? pl.T : sm_count);
-  const int stage_bytes = pl.na * (kAtomBytes + pl.hilo * pl.BN * 128);
+  const int stage_bytes = pl.na * (halves * kAtomBytes + pl.hilo * pl.BN * 128);
   pl.stages = (int)((kSmemBudget - 2048) / stage_bytes);
-  if (pl.stages > 8) pl.stages = 8;
+  if (pl.stages > kMaxStages) pl.stages = kMaxStages;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
   // fp8: four converter warps own the ring slots round-robin, so the ring
   // has four or eight stages
@@ -855,9 +917,10 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.hs_bytes = align256((size_t)pl.hilo * pl.Rp * pl.Kp * 2);
   // split tiles exist only when a CTA's range does not cover whole tiles
   const bool splits = !pl.whole_tiles && (pl.T % pl.G != 0 || (pl.T / pl.G) % pl.KB != 0);
-  pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * kTileM * 4) : 0;
+  pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * pl.tm * 4) : 0;
   pl.cnt_bytes = align256((size_t)tiles * 4 * kEpiGroups * sizeof(int));
-  pl.stats_bytes = endpoint ? align256((size_t)rows * pl.NT * 4 * sizeof(float2)) : 0;
+  pl.nseg = pl.NT * (pl.tm / 32);
+  pl.stats_bytes = endpoint ? align256((size_t)rows * pl.nseg * sizeof(float2)) : 0;
   // the epilogue's statistics are latency-bound chains of shuffles and
   // exponentials per 16 rows, hidden behind the next tile's MMAs only when
   // the hidden dimension is long enough; otherwise a separate pass over z at
@@ -870,11 +933,11 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   return pl;
 }
 
-template <int HILO, bool GATHER, int EPI, bool FP8 = false>
+template <int HILO, bool GATHER, int EPI, bool FP8 = false, int TM = 128>
 static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
                                const TcParams& prm, const TcPlan& pl,
                                cudaStream_t st) {
-  auto kern = tc_kernel<HILO, GATHER, EPI, FP8>;
+  auto kern = tc_kernel<HILO, GATHER, EPI, FP8, TM>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)pl.smem_bytes);
   if (e != cudaSuccess) return e;
@@ -922,13 +985,13 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   const int a3d = (!fp8 && !gather && g.K % kAtomK == 0 && g.K >= pl.na * kAtomK) ? 1 : 0;
   mw.a3 = CUtensorMap{};
   if (a3d && !make_map3(&mw.a3, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
-                        (uint64_t)g.V, (uint64_t)g.ld_w * 2, kTileM, (uint32_t)pl.na))
+                        (uint64_t)g.V, (uint64_t)g.ld_w * 2, (uint32_t)pl.tm, (uint32_t)pl.na))
     return cudaErrorInvalidValue;
 
   TcParams prm{};
   prm.R = g.rows; prm.n = g.n; prm.K = g.K; prm.KB = pl.KB; prm.NT = pl.NT;
   prm.RB = pl.RB; prm.BN = pl.BN; prm.Rp = pl.Rp; prm.stages = pl.stages;
-  prm.whole_tiles = pl.whole_tiles; prm.T = pl.T; prm.na = pl.na;
+  prm.whole_tiles = pl.whole_tiles; prm.T = pl.T; prm.na = pl.na; prm.nseg = pl.nseg;
   prm.ids = g.ids;
   prm.W8 = fp8 ? static_cast<const uint8_t*>(g.W) : nullptr;
   prm.ld_w = g.ld_w;
@@ -941,6 +1004,19 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.status = g.status; prm.spin_limit = spin_limit;
 
   const bool hilo2 = pl.hilo == 2;
+  if (pl.tm == 256) {
+    if (fp8) return cudaErrorNotSupported;
+    if (g.epilogue == EPI_CLOUD) {
+      if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, false, 256>(mw, mh, prm, pl, st)
+                               : launch_inst<1, true, EPI_CLOUD, false, 256>(mw, mh, prm, pl, st);
+      return hilo2 ? launch_inst<2, false, EPI_CLOUD, false, 256>(mw, mh, prm, pl, st)
+                   : launch_inst<1, false, EPI_CLOUD, false, 256>(mw, mh, prm, pl, st);
+    }
+    if (gather) return hilo2 ? launch_inst<2, true, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st)
+                             : launch_inst<1, true, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st);
+    return hilo2 ? launch_inst<2, false, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st)
+                 : launch_inst<1, false, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st);
+  }
   if (fp8) {
     if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, true>(mw, mh, prm, pl, st)
                              : launch_inst<1, true, EPI_CLOUD, true>(mw, mh, prm, pl, st);
@@ -974,7 +1050,7 @@ cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPl
     return launch_sample_segments(Z, rows, n, sst, seg_count(n), cstats, ids, inv_tau, seed,
                                   offset, tokens, st, greedy);
   }
-  const int nseg = pl.NT * 4;
+  const int nseg = pl.nseg;
   if (greedy)   // the segment maxima are all greedy decoding needs
     return launch_sample_segments(Z, rows, n, stats, nseg, nullptr, ids, inv_tau, seed, offset,
                                   tokens, st, 1);

@@ -34,6 +34,7 @@ struct sph_ctx {
   int tc_stages = 0;                // SPH_OPT_TC_STAGES
   int tc_block_k = 0;               // SPH_OPT_TC_BLOCK_K
   int tc_max_bn = 0;                // SPH_OPT_TC_MAX_BN
+  int tc_tile_m = 0;                // SPH_OPT_TC_TILE_M
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -127,14 +128,18 @@ size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_
                 int w_dtype, int endpoint) {
   if (!use_tc(ctx, rows, w_dtype)) return 0;
   size_t b = 0;
-  for (int gather = 0; gather < 2; ++gather) {   // the larger of the two paths
-    const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count,
-                                  endpoint, ctx->tc_schedule, ctx->tc_stages,
-                                  ctx->tc_block_k, gather, w_dtype == sph::W_FP8,
-                                  ctx->tc_max_bn)
-                         .scratch_bytes;
-    if (x > b) b = x;
-  }
+  // the larger of the two paths and (automatic tile height, which smaller
+  // calls may choose differently) of the two tile heights
+  for (int gather = 0; gather < 2; ++gather)
+    for (int tm = 128; tm <= 256; tm += 128) {
+      if (ctx->tc_tile_m && tm != ctx->tc_tile_m) continue;
+      const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count,
+                                    endpoint, ctx->tc_schedule, ctx->tc_stages,
+                                    ctx->tc_block_k, gather, w_dtype == sph::W_FP8,
+                                    ctx->tc_max_bn, tm)
+                           .scratch_bytes;
+      if (x > b) b = x;
+    }
   return b;
 }
 
@@ -375,8 +380,8 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       ctx->tc_schedule = (int)value;
       return SPH_OK;
     case SPH_OPT_TC_STAGES:
-      if (value != 0 && (value < 2 || value > 8))
-        return fail(ctx, SPH_ERR_INVALID_ARG, "stages must be 0 or in [2, 8]");
+      if (value != 0 && (value < 2 || value > 12))
+        return fail(ctx, SPH_ERR_INVALID_ARG, "stages must be 0 or in [2, 12]");
       ctx->tc_stages = (int)value;
       return SPH_OK;
     case SPH_OPT_TC_BLOCK_K:
@@ -388,6 +393,11 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       if (value != 0 && (value < 16 || value > 256 || value % 16))
         return fail(ctx, SPH_ERR_INVALID_ARG, "max_bn must be 0 or a multiple of 16 in [16, 256]");
       ctx->tc_max_bn = (int)value;
+      return SPH_OK;
+    case SPH_OPT_TC_TILE_M:
+      if (value != 0 && value != 128 && value != 256)
+        return fail(ctx, SPH_ERR_INVALID_ARG, "tile_m must be 0, 128 or 256");
+      ctx->tc_tile_m = (int)value;
       return SPH_OK;
   }
   return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
@@ -476,7 +486,7 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_h, act_bf16,
                                         ctx->sm_count, 0, ctx->tc_schedule, ctx->tc_stages,
                                         ctx->tc_block_k, keep_ids != nullptr,
-                                        wdt == sph::W_FP8, ctx->tc_max_bn);
+                                        wdt == sph::W_FP8, ctx->tc_max_bn, ctx->tc_tile_m);
     void* tcs = c.take(pl.scratch_bytes);
     st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
@@ -535,7 +545,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0,
                                         ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
                                         ctx->tc_block_k, keep_ids != nullptr, 0,
-                                        ctx->tc_max_bn);
+                                        ctx->tc_max_bn, ctx->tc_tile_m);
     void* tcs = c.take(pl.scratch_bytes);
     st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);

@@ -83,6 +83,8 @@ int gemv_max_k();
 // Tensor-core path (k_tc.cu): sizes, work split and scratch of one call.
 struct TcPlan {
   int hilo, RB, BN, Rp, KB, Kp, NT, G, stages, whole_tiles, na, fp8;
+  int tm;          // vocabulary rows per tile: 128 or 256
+  int nseg;        // endpoint statistics: 32-id segments per row, NT * tm / 32
   int epi_stats;   // endpoint: softmax statistics in the epilogue (else a pass over z)
   long long T;
   size_t hs_bytes, p_bytes, cnt_bytes, stats_bytes, scratch_bytes, smem_bytes;
@@ -92,9 +94,11 @@ struct TcPlan {
 // automatic / whole tiles / stream-K; max_stages 0 = automatic; block_k =
 // hidden elements per pipeline stage (64, 128 or 256; 0 = automatic);
 // gather = the kept-id subset path (keep_ids given); fp8 = e4m3 weights;
-// max_bn = most hidden-state rows per tile (0 = automatic).
+// max_bn = most hidden-state rows per tile (0 = automatic); tile_m =
+// vocabulary rows per tile (128, 256 = two M = 128 halves, 0 = automatic).
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
-               int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn);
+               int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn,
+               int tile_m);
 // Launch the operand split and the tcgen05 kernel; `scratch` holds
 // plan.scratch_bytes bytes.  bf16 weights only.
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,

@@ -250,7 +250,7 @@ def test_verify_accepts_drafts_equal_to_target(ctx):
 
 FULL = [("tiny", None, None), ("decode", None, None), ("spec", None, None),
         ("fp8", None, None), ("sweep", 1, 0.1), ("sweep", 64, 0.5),
-        ("sweep", 1024, 1.0)]
+        ("sweep", 256, 1.0), ("sweep", 1024, 1.0)]
 
 
 @pytest.mark.parametrize("name,rows,keep", FULL,
@@ -290,6 +290,43 @@ def test_tensor_core_variants(ctx, block_k, schedule, keep):
     finally:
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
         ctx.set_option(sph.SPH_OPT_TC_BLOCK_K, 0)
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+
+
+# ---------------------------------------------------------------------------
+# 256-id tensor-core tiles (two M = 128 MMAs per hidden-state stage)
+# ---------------------------------------------------------------------------
+
+TILE256_CASES = [
+    # full vocabulary, K = 1000: one 2-D copy per (atom, tile half), ragged tail
+    ("full-k1000", dict(V=3000, d=1072, d_l=72, rows=24, n_keep=3000)),
+    # full vocabulary, K = 1024: one 3-D copy of all atoms per stage
+    ("full-k1024", dict(V=3000, d=1096, d_l=72, rows=40, n_keep=3000)),
+    # kept runs longer than 128 ids: two row boxes per run
+    ("long-runs", dict(V=4000, d=1072, d_l=72, rows=24, n_keep=2000, run_lo=150, run_hi=400)),
+    # isolated ids (one-row boxes) and two row blocks of 80 rows
+    ("isolated", dict(V=2000, d=1072, d_l=72, rows=130, n_keep=700, run_lo=1, run_hi=3)),
+]
+
+
+@pytest.mark.parametrize("name,kw", TILE256_CASES, ids=[c[0] for c in TILE256_CASES])
+@pytest.mark.parametrize("schedule", [1, 2])
+@pytest.mark.parametrize("act", ["fp32", "bf16"])
+def test_tensor_core_256_tiles(ctx, name, kw, schedule, act):
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    ctx.set_option(sph.SPH_OPT_TC_TILE_M, 256)
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, schedule)
+    try:
+        w = small(seed=400 + len(name) + schedule, **kw)
+        check_cloud(ctx, w, act_mode=act)
+        if act == "fp32":
+            ref = oracle_cloud(w)
+            check_endpoint(ctx, w, torch.from_numpy(ref["codes"]),
+                           torch.from_numpy(ref["row_scale"]))
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+        ctx.set_option(sph.SPH_OPT_TC_TILE_M, 0)
         ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
 
 
