@@ -251,6 +251,55 @@ sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
   if (lane == 0) tokens[r] = ids ? ids[j] : j;
 }
 
+// Sampling with the chunk statistics made in the same block (one block per
+// row, 4..32 warps as the chunk count asks): the warps reduce the row's
+// segment statistics to chunk statistics in shared memory -- the same
+// reductions, and so the same values, as the chunk-statistics kernel --
+// then warp 0 draws.  Saves that kernel's launch on the step's critical
+// path.
+constexpr int kMaxFusedChunks = 4096;   // shared memory: 8 bytes per chunk
+constexpr int kFusedU = 4;              // chunks in flight per warp
+__global__ void __launch_bounds__(1024)
+sample_rows_kernel(const float* __restrict__ Z, int n, const float2* __restrict__ stats,
+                   int nseg, const int32_t* __restrict__ ids, float inv_tau, uint64_t seed,
+                   uint64_t offset, int32_t* __restrict__ tokens) {
+  extern __shared__ float2 s_cst[];
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const int r = blockIdx.x;
+  const int nchunk = (nseg + kSeg - 1) / kSeg;
+  const float2* srow = stats + (int64_t)r * nseg;
+  constexpr int kU = kFusedU;
+  for (int cb = warp; cb < nchunk; cb += nw * kU) {
+    float2 st[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int c = cb + u * nw, sg = c * kSeg + lane;
+      st[u] = (c < nchunk && sg < nseg) ? srow[sg] : make_float2(-INFINITY, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int c = cb + u * nw;
+      if (c < nchunk) {
+        const float Mc = warp_max(st[u].x);
+        const float Sc = warp_sum(seg_weight(st[u], Mc, inv_tau));
+        if (lane == 0) s_cst[c] = make_float2(Mc, Sc);
+      }
+    }
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  const float M = stats_max(s_cst, nchunk, lane);
+  const StatsWeight cw{s_cst, M, inv_tau};
+  const StatsWeight sw{srow, M, inv_tau};
+  const ExpWeight ew{Z + (int64_t)r * n, M, inv_tau};
+  const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
+  int j;
+  warp_draw(nchunk, nseg, n, cw, sw, ew, u, lane, j);
+  if (lane == 0) tokens[r] = ids ? ids[j] : j;
+}
+
 // ---------------------------------------------------------------------------
 // greedy decoding (temperature 0): the first id of the row maximum
 // ---------------------------------------------------------------------------
@@ -502,6 +551,18 @@ cudaError_t launch_sample_segments(const float* Z, int rows, int n, const float2
   return launch_pdl(sample_seg_kernel, dim3((rows + kWarps - 1) / kWarps),
                     dim3(kWarps * 32), 0, st, Z, rows, n, stats, nseg, cstats, ids, inv_tau,
                     seed, offset, tokens);
+}
+
+cudaError_t launch_sample_rows(const float* Z, int rows, int n, const float2* stats,
+                               int nseg, const int32_t* ids, float inv_tau, uint64_t seed,
+                               uint64_t offset, int32_t* tokens, cudaStream_t st) {
+  const int nchunk = chunk_count(nseg);
+  if (rows < 1 || nchunk > kMaxFusedChunks) return cudaErrorNotSupported;
+  int warps = (nchunk + kFusedU - 1) / kFusedU;
+  warps = warps < 4 ? 4 : (warps > 32 ? 32 : warps);
+  return launch_pdl(sample_rows_kernel, dim3(rows), dim3(warps * 32),
+                    (size_t)nchunk * sizeof(float2), st, Z, n, stats, nseg, ids, inv_tau, seed,
+                    offset, tokens);
 }
 
 // Scratch: stats [R][nseg] float2 | chunk stats [R][nchunk] float2 | rowMS

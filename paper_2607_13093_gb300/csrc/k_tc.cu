@@ -60,6 +60,7 @@ constexpr int kMaxBN = 256;
 constexpr int kMaxStages = 12;       // (the barrier area holds (3 * 12 + 5) words)
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
+constexpr long long kFinisherWait = 1ll << 15; // cycles a split tile's finisher polls
 
 constexpr int kEpiWarps = 8;         // two per TMEM lane quadrant
 constexpr int kEpiGroups = kEpiWarps / 4;
@@ -245,6 +246,97 @@ tc_kernel(const __grid_constant__ WMaps wm,
   int2* s_box = reinterpret_cast<int2*>(base + (size_t)S * stage_bytes + 256);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = gridDim.x;
+  const long long it0 = range_start(p, blockIdx.x, G);
+  const long long it1 = range_start(p, blockIdx.x + 1, G);
+  // producer, subset path: the ids of a segment's tile are loaded one
+  // segment ahead, so that planning a tile never waits on memory; the first
+  // tile's load goes out before the CTA's setup
+  int nid[kGroups];
+#pragma unroll
+  for (int g = 0; g < kGroups; ++g) nid[g] = 0;
+  auto load_ids = [&](int tl, int (&dst)[kGroups]) {
+    const int j0 = (tl / p.RB) * TM;
+    const int rows = min(TM, p.n - j0);
+#pragma unroll
+    for (int g = 0; g < kGroups; ++g) {
+      const int r = 32 * g + lane;
+      dst[g] = r < rows ? p.ids[j0 + r] : 0;
+    }
+  };
+  // Subset path: plan tile t's row boxes (runs of consecutive kept ids,
+  // each one box of its own height; lane l owns tile rows l, l + 32, ...)
+  // into s_box, from the ids in nid, and start loading the ids of segment
+  // tile next_tile (-1: none) into nid.  Returns the box count and the
+  // stage's transaction bytes.  Warp-collective (producer warp).
+  auto plan_tile = [&](int t, int next_tile, int& nbox, uint32_t& tx) {
+    int2 box[2 * kGroups];                       // (first id, row | (rows - 1) << 8)
+    unsigned bmask = 0;                          // which of box[] are in use
+    const int j0 = t * TM;
+    const int rows = min(TM, p.n - j0);
+    int idr[kGroups];
+#pragma unroll
+    for (int g = 0; g < kGroups; ++g) idr[g] = nid[g];
+    if (next_tile >= 0) load_ids(next_tile, nid);
+    unsigned smask[kGroups];
+    int prev_last = 0;
+#pragma unroll
+    for (int g = 0; g < kGroups; ++g) {
+      const int r = 32 * g + lane;
+      int prev = __shfl_up_sync(0xFFFFFFFFu, idr[g], 1);
+      if (lane == 0) prev = prev_last;
+      smask[g] = __ballot_sync(0xFFFFFFFFu, r < rows && (r == 0 || idr[g] != prev + 1));
+      prev_last = __shfl_sync(0xFFFFFFFFu, idr[g], 31);
+    }
+    int covered = 0;
+#pragma unroll
+    for (int g = 0; g < kGroups; ++g) {
+      const int r = 32 * g + lane;
+      if ((smask[g] >> lane) & 1u) {
+        int nxt = rows;
+        const unsigned above = lane == 31 ? 0u : (smask[g] >> (lane + 1)) << (lane + 1);
+        if (above) {
+          nxt = 32 * g + __ffs(above) - 1;
+        } else {
+          for (int g2 = g + 1; g2 < kGroups; ++g2)
+            if (smask[g2]) { nxt = 32 * g2 + __ffs(smask[g2]) - 1; break; }
+        }
+        // one box of exactly len rows (two, 128 + rest, past 128 rows)
+        const int len = nxt - r;
+        const int l0 = min(len, 128);
+        box[2 * g] = make_int2(idr[g], r | ((l0 - 1) << 8));
+        bmask |= 1u << (2 * g);
+        if (len > 128) {
+          box[2 * g + 1] = make_int2(idr[g] + 128, (r + 128) | ((len - 129) << 8));
+          bmask |= 2u << (2 * g);
+        }
+        covered += len;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) covered += __shfl_xor_sync(0xFFFFFFFFu, covered, o);
+    tx = (uint32_t)(covered * 128 * NA + b_bytes);
+    // compact every lane's boxes into one shared list that the copy loop
+    // below hands out to lanes (measured: far faster than issuing from
+    // the planning registers under per-lane predicates)
+    const int mine = __popc(bmask);
+    int incl = mine;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    nbox = __shfl_sync(0xFFFFFFFFu, incl, 31);
+    int slot = incl - mine;
+#pragma unroll
+    for (int q = 0; q < 2 * kGroups; ++q)
+      if ((bmask >> q) & 1u) s_box[slot++] = box[q];
+    __syncwarp();
+  };
+  // the first tile's ids load while the CTA sets up
+  if constexpr (GATHER && !FP8) {
+    if (warp == 0 && it0 < it1) load_ids((int)(it0 / p.KB), nid);
+  }
   uint32_t ncols = 32;                 // two accumulators of kHalves x BN columns
   while (ncols < (uint32_t)(2 * kHalves * BN)) ncols <<= 1;
 
@@ -270,15 +362,18 @@ tc_kernel(const __grid_constant__ WMaps wm,
   // this one wait for them (griddep_wait): the producer before its first
   // copy, the epilogue before its first store.
   ptx::griddep_launch_dependents();
-  if (warp == 1) ptx::tmem_alloc(tmem_holder, ncols);
-  ptx::tc_fence_before();
-  __syncthreads();
-  ptx::tc_fence_after();
-  const uint32_t tmem_base = *tmem_holder;
+  __syncthreads();                     // barriers initialised
+  // the producer needs no tensor memory: it starts now, while warp 1
+  // allocates the accumulators for itself and the other warps
+  uint32_t tmem_base = 0;
+  if (warp != 0) {
+    if (warp == 1) ptx::tmem_alloc(tmem_holder, ncols);
+    ptx::tc_fence_before();
+    ptx::named_bar_sync(1, (int)blockDim.x - 32);
+    ptx::tc_fence_after();
+    tmem_base = *tmem_holder;
+  }
 
-  const int G = gridDim.x;
-  const long long it0 = range_start(p, blockIdx.x, G);
-  const long long it1 = range_start(p, blockIdx.x + 1, G);
   const long long limit = p.spin_limit;
 
   auto give_up = [&]() {
@@ -297,98 +392,40 @@ tc_kernel(const __grid_constant__ WMaps wm,
     int tile, kb0, kb1;
     bool stop = false;
     long long issued = 0;
-    if (lane == 0) ptx::griddep_wait();          // h planes come from the prep kernel
-    __syncwarp();
-    // subset path: the ids of a segment's tile are loaded one segment ahead,
-    // so that planning a tile never waits on memory
-    int nid[kGroups];
-#pragma unroll
-    for (int g = 0; g < kGroups; ++g) nid[g] = 0;
-    auto load_ids = [&](int tl, int (&dst)[kGroups]) {
-      const int j0 = (tl / p.RB) * TM;
-      const int rows = min(TM, p.n - j0);
-#pragma unroll
-      for (int g = 0; g < kGroups; ++g) {
-        const int r = 32 * g + lane;
-        dst[g] = r < rows ? p.ids[j0 + r] : 0;
-      }
-    };
-    if constexpr (GATHER && !FP8) {
-      Segments pk = sg;
-      int tn, a0, a1;
-      if (pk.next(tn, a0, a1)) load_ids(tn, nid);
+    // The h planes come from the operand-split kernel, the weights and ids
+    // from the caller: the first segment's plan and the A copies of its
+    // first stage go out before the wait for that kernel, the stage's B
+    // copies right after it (fp8: the converter warps fill A, so wait up
+    // front).
+    bool waited = FP8;
+    int rb_first = 0, kb_first = 0;
+    if (FP8) {
+      if (lane == 0) ptx::griddep_wait();
+      __syncwarp();
     }
+    // the B copy of plane l of stage st (k-block kb, row block rb)
+    auto issue_b = [&](int st, int kb, int rb, int l) {
+      if (l >= 0 && l < HILO)
+        ptx::tma_load_3d(base + (size_t)st * stage_bytes + a_bytes + l * NA * BN * 128, &tmH, 0,
+                         l * p.Rp + rb * BN, kb * NA, &full[st]);
+    };
+    auto finish_wait = [&]() {
+      if (lane == 0) ptx::griddep_wait();
+      __syncwarp();
+      // the stages issued so far (0 or 1) are the first of the ring
+      for (int q = lane; q < issued * HILO; q += 32)
+        issue_b(q / HILO, kb_first + q / HILO, rb_first, q % HILO);
+      waited = true;
+    };
     while (!stop && sg.next(tile, kb0, kb1)) {
       const int t = tile / p.RB, rb = tile - t * p.RB;
-      int2 box[2 * kGroups];                     // (first id, row | (rows - 1) << 8)
-      unsigned bmask = 0;                        // which of box[] are in use
       int nbox = 0;
       uint32_t tx = (uint32_t)(FP8 ? b_bytes : stage_bytes);
       if constexpr (GATHER && !FP8) {
-        const int j0 = t * TM;
-        const int rows = min(TM, p.n - j0);
-        int idr[kGroups];
-#pragma unroll
-        for (int g = 0; g < kGroups; ++g) idr[g] = nid[g];
-        {
-          Segments pk = sg;
-          int tn, a0, a1;
-          if (pk.next(tn, a0, a1)) load_ids(tn, nid);
-        }
-        unsigned smask[kGroups];
-        int prev_last = 0;
-#pragma unroll
-        for (int g = 0; g < kGroups; ++g) {
-          const int r = 32 * g + lane;
-          int prev = __shfl_up_sync(0xFFFFFFFFu, idr[g], 1);
-          if (lane == 0) prev = prev_last;
-          smask[g] = __ballot_sync(0xFFFFFFFFu, r < rows && (r == 0 || idr[g] != prev + 1));
-          prev_last = __shfl_sync(0xFFFFFFFFu, idr[g], 31);
-        }
-        int covered = 0;
-#pragma unroll
-        for (int g = 0; g < kGroups; ++g) {
-          const int r = 32 * g + lane;
-          if ((smask[g] >> lane) & 1u) {
-            int nxt = rows;
-            const unsigned above = lane == 31 ? 0u : (smask[g] >> (lane + 1)) << (lane + 1);
-            if (above) {
-              nxt = 32 * g + __ffs(above) - 1;
-            } else {
-              for (int g2 = g + 1; g2 < kGroups; ++g2)
-                if (smask[g2]) { nxt = 32 * g2 + __ffs(smask[g2]) - 1; break; }
-            }
-            // one box of exactly len rows (two, 128 + rest, past 128 rows)
-            const int len = nxt - r;
-            const int l0 = min(len, 128);
-            box[2 * g] = make_int2(idr[g], r | ((l0 - 1) << 8));
-            bmask |= 1u << (2 * g);
-            if (len > 128) {
-              box[2 * g + 1] = make_int2(idr[g] + 128, (r + 128) | ((len - 129) << 8));
-              bmask |= 2u << (2 * g);
-            }
-            covered += len;
-          }
-        }
-#pragma unroll
-        for (int o = 16; o; o >>= 1) covered += __shfl_xor_sync(0xFFFFFFFFu, covered, o);
-        tx = (uint32_t)(covered * 128 * NA + b_bytes);
-        // compact every lane's boxes into one shared list that the copy loop
-        // below hands out to lanes (measured: far faster than issuing from
-        // the planning registers under per-lane predicates)
-        const int mine = __popc(bmask);
-        int incl = mine;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-          if (lane >= o) incl += v;
-        }
-        nbox = __shfl_sync(0xFFFFFFFFu, incl, 31);
-        int slot = incl - mine;
-#pragma unroll
-        for (int q = 0; q < 2 * kGroups; ++q)
-          if ((bmask >> q) & 1u) s_box[slot++] = box[q];
-        __syncwarp();
+        Segments pk = sg;
+        int tn = -1, a0, a1;
+        if (!pk.next(tn, a0, a1)) tn = -1;
+        plan_tile(t, tn, nbox, tx);
       }
       for (int kb = kb0; kb < kb1; ++kb) {
         int ok = 1;
@@ -408,7 +445,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
         // one 3-D copy of all NA atoms per plane
         uint8_t* A = base + (size_t)stage * stage_bytes;
         const int nA = FP8 ? 0 : (GATHER ? NA * nbox : (p.a3d ? 1 : NA * kHalves));
-        for (int op = lane; op < nA + HILO; op += 32) {
+        if (!waited && issued == 0) { rb_first = rb; kb_first = kb; }
+        for (int op = lane; op < nA + (waited ? HILO : 0); op += 32) {
           if (op < nA) {
             if constexpr (GATHER) {
               const int a = op / nbox;
@@ -423,15 +461,18 @@ tc_kernel(const __grid_constant__ WMaps wm,
                                (kb * NA + a) * kAtomK, t * TM + hf * 128, &full[stage]);
             }
           } else {
-            const int h = op - nA;
-            ptx::tma_load_3d(A + a_bytes + h * NA * BN * 128, &tmH, 0, h * p.Rp + rb * BN,
-                             kb * NA, &full[stage]);
+            issue_b(stage, kb, rb, op - nA);
           }
         }
         ++issued;
         if (++stage == S) { stage = 0; phase ^= 1; }
+        if (!waited) finish_wait();
       }
     }
+    // (a CTA without work, or one that stopped before its first segment's
+    // stages were all issued, still sends their B copies, so that every
+    // issued stage completes)
+    if (!waited) finish_wait();
     if (stop && lane == 0) {
       // let the copies already issued land before the CTA winds down
       for (long long k = issued > S ? issued - S : 0; k < issued; ++k)
@@ -531,6 +572,51 @@ tc_kernel(const __grid_constant__ WMaps wm,
         if (whole && grp < nhc)
           load_payload(p, rb * BN + (grp % nch) * 16, J(grp / nch), lane, pay);
       }
+      // Split tile: contributors c0 .. c0 + C - 1 (CTA order).  All but the
+      // last end their ranges inside the tile, so they reach it at the end
+      // of their work; the last one reaches it first thing (its range starts
+      // inside the tile).  Contributor c0 + C - 2 is the tile's finisher: it
+      // waits (briefly, bounded) until every other contributor's warp of
+      // this quadrant and chunk group has stored its partial and counted
+      // in, then finishes the tile from its own accumulator and their
+      // partials.  The others store and count in; if the finisher gave up
+      // waiting it counts in like them, and whoever counts in last finishes
+      // the tile from the stored partials.
+      constexpr int kMaxC = 8;
+      int c0 = 0, C = 1, cnt = 0;
+      bool fin = false, known_last = false, pre_ok = false;
+      float pre[16];                   // two contributors: the other's first chunk
+      if (!whole) {
+        cnt = (tile * 4 + quad) * kEpiGroups + grp;
+        c0 = (int)cta_of((long long)tile * p.KB, p.T, gridDim.x);
+        C = (int)cta_of((long long)tile * p.KB + p.KB - 1, p.T, gridDim.x) - c0 + 1;
+        fin = C >= 2 && C <= kMaxC && (int)blockIdx.x == c0 + C - 2;
+      }
+      // the contributors' partial slots: every contributor after the first
+      // starts its range inside this tile, so the tile is its first segment
+      // (slot 2c); the first one holds it as its first segment only if its
+      // range starts exactly at the tile (slot 2c0), else as its last
+      // (slot 2c0 + 1)
+      const bool c0_first = !whole && range_start(p, c0, gridDim.x) == (long long)tile * p.KB;
+      auto slot_of = [&](int c) { return c == 0 ? 2 * c0 + (c0_first ? 0 : 1) : 2 * (c0 + c); };
+      if (fin) {
+        // the early contributor (the tile's last) has usually arrived
+        // already: then fetch its partial while the MMAs finish
+        int arrived = 0;
+        if (lane == 0) arrived = ptx::ld_acquire_gpu(&p.counters[cnt]);
+        known_last = __shfl_sync(0xFFFFFFFFu, arrived, 0) == C - 1;
+        __syncwarp();
+        // (cloud only: the endpoint epilogue's payload registers leave no
+        // room, and its short hidden dimension mostly gives whole tiles)
+        if (EPI == EPI_CLOUD && known_last && C == 2 && grp < nhc) {
+          const int hf = grp / nch, ch = grp - hf * nch;
+          const float* pc = p.P + (size_t)slot_of(1) * BN * TM + (size_t)ch * 16 * TM +
+                            hf * 128 + quad * 32 + lane;
+#pragma unroll
+          for (int q = 0; q < 16; ++q) pre[q] = __ldcg(pc + (size_t)q * TM);
+          pre_ok = true;
+        }
+      }
       int ok = 1;
       if (lane == 0) ok = !*s_abort && ptx::mbar_wait(&tfull[acc], fph[acc], limit);
       ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
@@ -539,6 +625,21 @@ tc_kernel(const __grid_constant__ WMaps wm,
         break;
       }
       fph[acc] ^= 1;
+      if (fin && !known_last) {
+        // the other contributors that end with this tile finish at about
+        // the same time: poll for them, bounded (giving up only costs the
+        // round trip through the partial buffer)
+        int arrived = 0;
+        if (lane == 0) {
+          const long long t0 = clock64();
+          const long long bound = limit < kFinisherWait ? limit : kFinisherWait;
+          while ((arrived = ptx::ld_acquire_gpu(&p.counters[cnt])) != C - 1 &&
+                 clock64() - t0 < bound)
+            __nanosleep(64);
+        }
+        known_last = __shfl_sync(0xFFFFFFFFu, arrived, 0) == C - 1;
+        __syncwarp();
+      }
       ptx::tc_fence_after();
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) +
                              (uint32_t)(acc * kHalves * BN);
@@ -558,6 +659,31 @@ tc_kernel(const __grid_constant__ WMaps wm,
           finish_chunk<EPI>(p, v, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
                             t * kGroups + hf * 4 + quad, pay);
           if constexpr (EPI == EPI_ENDPOINT) pay = nxt;
+        } else if (known_last) {
+          // the partials in CTA order (the same order, and so the same
+          // result, as the fix-up below), this CTA's own from registers
+          if constexpr (EPI == EPI_ENDPOINT) load_payload(p, rb * BN + ch * 16, J(hf), lane, pay);
+          const int me = (int)blockIdx.x - c0;
+          const size_t o = (size_t)ch * 16 * TM + i;
+          float s[16];
+          if (pre_ok && hc == grp) {       // two contributors, the other's part prefetched
+#pragma unroll
+            for (int q = 0; q < 16; ++q) s[q] = v[q] + pre[q];   // (me == 0)
+          } else {
+#pragma unroll
+            for (int c = 0; c < kMaxC; ++c) {
+              if (c < C) {
+                const float* pc = p.P + (size_t)slot_of(c) * BN * TM + o;
+#pragma unroll
+                for (int q = 0; q < 16; ++q) {
+                  const float x = c == me ? v[q] : __ldcg(pc + (size_t)q * TM);
+                  s[q] = c == 0 ? x : s[q] + x;
+                }
+              }
+            }
+          }
+          finish_chunk<EPI>(p, s, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
+                            t * kGroups + hf * 4 + quad, pay);
         } else {
 #pragma unroll
           for (int q = 0; q < 16; ++q) Pt[(size_t)(ch * 16 + q) * TM + i] = v[q];
@@ -566,33 +692,23 @@ tc_kernel(const __grid_constant__ WMaps wm,
       ptx::tc_fence_before();
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(&tempty[acc]);
-      if (!whole) {
+      if (known_last) {
+        if (lane == 0) p.counters[cnt] = 0;
+      } else if (!whole) {
         // split tile: this warp's rows x its chunks are finished by the last
         // warp (over all contributing CTAs) of the same quadrant and chunk
         // group
         __threadfence();
         int old = 0;
-        const int cnt = (tile * 4 + quad) * kEpiGroups + grp;
         if (lane == 0) old = atomicAdd(&p.counters[cnt], 1);
         old = __shfl_sync(0xFFFFFFFFu, old, 0);
-        const int c0 = (int)cta_of((long long)tile * p.KB, p.T, gridDim.x);
-        const int c1 = (int)cta_of((long long)tile * p.KB + p.KB - 1, p.T, gridDim.x);
-        if (old == c1 - c0) {
+        if (old == C - 1) {
           __threadfence();
-          // the contributors' slots, in CTA order (a fixed summation order):
-          // every contributor after the first starts its range inside this
-          // tile, so the tile is its first segment (slot 2c); the first one
-          // holds it as its first segment only if its range starts exactly
-          // at the tile (slot 2c0), else as its last (slot 2c0 + 1)
-          constexpr int kMaxC = 8;
+          // the contributors' partials in CTA order (a fixed summation order)
           const float* ps[kMaxC];
-          const int C = c1 - c0 + 1;
-          const bool c0_first = range_start(p, c0, gridDim.x) == (long long)tile * p.KB;
 #pragma unroll
-          for (int c = 0; c < kMaxC; ++c) {
-            const int slot = c == 0 ? 2 * c0 + (c0_first ? 0 : 1) : 2 * (c0 + (c < C ? c : 0));
-            ps[c] = p.P + (size_t)slot * BN * TM + quad * 32 + lane;
-          }
+          for (int c = 0; c < kMaxC; ++c)
+            ps[c] = p.P + (size_t)slot_of(c < C ? c : 0) * BN * TM + quad * 32 + lane;
           for (int hc = grp; hc < nhc; hc += kEpiGroups) {
             const int hf = hc / nch, ch = hc - hf * nch;
             if constexpr (EPI == EPI_ENDPOINT) load_payload(p, rb * BN + ch * 16, J(hf), lane, pay);
@@ -714,36 +830,90 @@ tc_kernel(const __grid_constant__ WMaps wm,
 // ... and clear the split-tile counters and (cloud) the row maxima.
 // (planes of f16 instead of bf16 when f16 != 0: the fp8-weight path, where
 // bf16-activation mode first rounds h to bf16 and then splits that value)
-__global__ void split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R,
-                               int K, int Rp, int Kp, int hilo,
-                               __nv_bfloat16* __restrict__ Hs,
-                               int* __restrict__ counters, int ncounters,
-                               unsigned* __restrict__ rowmax, int f16, int act_bf16) {
+// One thread converts 8 consecutive columns of one row (Kp is a multiple of
+// 64, so a group never crosses a row) and stores 16 bytes per plane.  Small
+// 128-thread blocks with at most 32 registers fit beside a tensor-core CTA
+// on the same SM, so that kernel starts (and issues its first weight copies)
+// while this one runs.
+template <typename T>
+__device__ __forceinline__ uint32_t pack2(float a, float b);
+template <>
+__device__ __forceinline__ uint32_t pack2<__nv_bfloat16>(float a, float b) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+template <>
+__device__ __forceinline__ uint32_t pack2<__half>(float a, float b) {
+  const __half2 v = __floats2half2_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+template <typename T>
+__device__ __forceinline__ float round_to(float x);
+template <>
+__device__ __forceinline__ float round_to<__nv_bfloat16>(float x) {
+  return __bfloat162float(__float2bfloat16_rn(x));
+}
+template <>
+__device__ __forceinline__ float round_to<__half>(float x) {
+  return __half2float(__float2half_rn(x));
+}
+
+template <typename T>
+__device__ __forceinline__ void split_group(const float (&x)[8], int hilo, uint4* hi, uint4* lo) {
+  float r[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) r[i] = round_to<T>(x[i]);
+  *hi = make_uint4(pack2<T>(r[0], r[1]), pack2<T>(r[2], r[3]), pack2<T>(r[4], r[5]),
+                   pack2<T>(r[6], r[7]));
+  if (hilo == 2)
+    *lo = make_uint4(pack2<T>(x[0] - r[0], x[1] - r[1]), pack2<T>(x[2] - r[2], x[3] - r[3]),
+                     pack2<T>(x[4] - r[4], x[5] - r[5]), pack2<T>(x[6] - r[6], x[7] - r[7]));
+}
+
+constexpr int kSplitThreads = 128;
+__global__ void __launch_bounds__(kSplitThreads, 16)
+split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R, int K, int Rp, int Kp,
+               int hilo, __nv_bfloat16* __restrict__ Hs, int* __restrict__ counters,
+               int ncounters, unsigned* __restrict__ rowmax, int f16, int act_bf16) {
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int nth = gridDim.x * blockDim.x;
   if (rowmax)
-    for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x)
-      rowmax[r] = 0u;
+    for (int r = tid; r < R; r += nth) rowmax[r] = 0u;
+  for (int t = tid; t < ncounters; t += nth) counters[t] = 0;
+  const int gpr = Kp / 8;                          // groups per row
+  const int64_t groups = (int64_t)Rp * gpr;
   const int64_t total = (int64_t)Rp * Kp;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    const int r = (int)(e / Kp), c = (int)(e - (int64_t)r * Kp);
-    const float x = (r < R && c < K) ? h[(int64_t)r * ld_h + c] : 0.f;
-    if (f16) {
-      __half* H = reinterpret_cast<__half*>(Hs);
-      const float xr = act_bf16 ? __bfloat162float(__float2bfloat16_rn(x)) : x;
-      const __half hi = __float2half_rn(xr);
-      H[e] = hi;
-      if (hilo == 2) H[total + e] = __float2half_rn(xr - __half2float(hi));
+  const bool vec = (((uintptr_t)h | (uintptr_t)(ld_h * 4)) & 15) == 0;
+  for (int64_t g = tid; g < groups; g += nth) {
+    const int r = (int)(g / gpr), c0 = (int)(g - (int64_t)r * gpr) * 8;
+    float x[8];
+    const float* src = h + (int64_t)r * ld_h + c0;
+    if (r < R && vec && c0 + 8 <= K) {
+      const float4 a = __ldg(reinterpret_cast<const float4*>(src));
+      const float4 b = __ldg(reinterpret_cast<const float4*>(src) + 1);
+      x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+      x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
     } else {
-      const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-      Hs[e] = hi;
-      if (hilo == 2) Hs[total + e] = __float2bfloat16_rn(x - __bfloat162float(hi));
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] = (r < R && c0 + i < K) ? __ldg(src + i) : 0.f;
     }
+    uint4 hi, lo;
+    if (f16) {
+      // fp8 weights: f16 planes of h, or of h rounded to bf16 first
+      if (act_bf16) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] = round_to<__nv_bfloat16>(x[i]);
+      }
+      split_group<__half>(x, hilo, &hi, &lo);
+    } else {
+      split_group<__nv_bfloat16>(x, hilo, &hi, &lo);
+    }
+    uint4* dst = reinterpret_cast<uint4*>(Hs + g * 8);
+    dst[0] = hi;
+    if (hilo == 2) *reinterpret_cast<uint4*>(Hs + total + g * 8) = lo;
   }
-  for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < ncounters;
-       t += gridDim.x * blockDim.x)
-    counters[t] = 0;
 }
 
 
@@ -961,11 +1131,11 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   const int tiles = pl.RB * pl.NT;
 
   {
-    const int64_t total = (int64_t)pl.Rp * pl.Kp;
-    int blocks = (int)((total + 255) / 256);
+    const int64_t groups = (int64_t)pl.Rp * pl.Kp / 8;
+    int blocks = (int)((groups + kSplitThreads - 1) / kSplitThreads);
     if (blocks > 4096) blocks = 4096;
     if (blocks < 1) blocks = 1;
-    cudaError_t e = launch_pdl(split_h_kernel, dim3(blocks), dim3(256), 0, st, g.h, g.ld_h,
+    cudaError_t e = launch_pdl(split_h_kernel, dim3(blocks), dim3(kSplitThreads), 0, st, g.h, g.ld_h,
                                g.rows, g.K, pl.Rp, pl.Kp, pl.hilo, Hs, counters, tiles * 4 * kEpiGroups,
                                g.epilogue == EPI_CLOUD ? g.rowmax : (unsigned*)nullptr,
                                fp8 ? 1 : 0, g.act_bf16);
@@ -1054,6 +1224,8 @@ cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPl
   if (greedy)   // the segment maxima are all greedy decoding needs
     return launch_sample_segments(Z, rows, n, stats, nseg, nullptr, ids, inv_tau, seed, offset,
                                   tokens, st, 1);
+  if (chunk_count(nseg) <= 4096)
+    return launch_sample_rows(Z, rows, n, stats, nseg, ids, inv_tau, seed, offset, tokens, st);
   cudaError_t e = launch_chunk_stats(stats, rows, nseg, inv_tau, cstats, sm_count, st);
   if (e != cudaSuccess) return e;
   return launch_sample_segments(Z, rows, n, stats, nseg, cstats, ids, inv_tau, seed, offset,

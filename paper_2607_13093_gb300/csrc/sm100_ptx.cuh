@@ -208,6 +208,13 @@ __device__ __forceinline__ void cp_async_wait(int n) {
     default: asm volatile("cp.async.wait_group 7;" ::: "memory"); break;
   }
 }
+// Load with acquire semantics at GPU scope (pairs with a fence before
+// another CTA's atomic update of the same word).
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
 // Make this thread's generic-proxy shared-memory writes visible to later
 // async-proxy reads (tcgen05.mma operands).
 __device__ __forceinline__ void fence_proxy_async_smem() {

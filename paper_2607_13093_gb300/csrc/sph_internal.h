@@ -133,6 +133,12 @@ cudaError_t launch_seg_stats(const float* Z, int rows, int n, float inv_tau,
 cudaError_t launch_chunk_stats(const float2* stats, int rows, int nseg,
                                float inv_tau, float2* cstats, int sm_count,
                                cudaStream_t st);
+// One inverse-CDF draw per row from segment statistics alone (nseg per row):
+// a block per row makes the chunk statistics in shared memory first.
+// cudaErrorNotSupported (nothing launched) past 4096 chunks per row.
+cudaError_t launch_sample_rows(const float* Z, int rows, int n, const float2* stats,
+                               int nseg, const int32_t* ids, float inv_tau, uint64_t seed,
+                               uint64_t offset, int32_t* tokens, cudaStream_t st);
 // One inverse-CDF draw per row from segment and chunk statistics with nseg
 // segments per row (nseg * 32 >= n; segments past n hold zero weight).
 cudaError_t launch_sample_segments(const float* Z, int rows, int n,
