@@ -10,6 +10,9 @@
 // HBM traffic is the kept W rows once per row tile; rows > RT are handled by
 // further row tiles (re-reading W), which is why the dispatcher routes more
 // than a couple of rows to the tensor-core kernel.
+#include <atomic>
+#include <mutex>
+
 #include "sm100_ptx.cuh"
 #include "sph_common.cuh"
 #include "sph_internal.h"
@@ -184,13 +187,36 @@ template <int RT, int WDT, int EPI>
 cudaError_t launch_rt(const GatherGemm& g, int sm_count, cudaStream_t st) {
   const size_t smem = (size_t)RT * ((g.K + 7) & ~7) * sizeof(float);
   auto kern = gemv_kernel<RT, WDT, EPI>;
-  cudaError_t e = cudaFuncSetAttribute(
-      kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemLimit);
+  // the shared-memory opt-in and the occupancy are host calls: made once per
+  // device (and shared-memory size) and remembered
+  constexpr int kMaxDev = 64, kOccSlots = 8;
+  static std::atomic<bool> opted[kMaxDev];
+  static std::mutex occ_mu;
+  static struct { int dev; size_t smem; int occ; } occ_cache[kOccSlots];
+  static int occ_next = 0;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  int occ = 1;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kThreads, smem);
-  if (e != cudaSuccess) return e;
-  if (occ < 1) occ = 1;
+  const bool cacheable = dev >= 0 && dev < kMaxDev;
+  if (!cacheable || !opted[dev].load()) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemLimit);
+    if (e != cudaSuccess) return e;
+    if (cacheable) opted[dev].store(true);
+  }
+  int occ = 0;
+  {
+    std::lock_guard<std::mutex> lock(occ_mu);
+    for (const auto& c : occ_cache)
+      if (c.occ > 0 && c.dev == dev && c.smem == smem) occ = c.occ;
+  }
+  if (occ == 0) {
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kThreads, smem);
+    if (e != cudaSuccess) return e;
+    if (occ < 1) occ = 1;
+    std::lock_guard<std::mutex> lock(occ_mu);
+    occ_cache[occ_next] = {dev, smem, occ};
+    occ_next = (occ_next + 1) % kOccSlots;
+  }
   const int work = (g.n + vpw<RT>() - 1) / vpw<RT>();       // warp tasks
   int blocks = (work + kWarps - 1) / kWarps;
   blocks = blocks < sm_count * occ ? blocks : sm_count * occ;

@@ -44,6 +44,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "sm100_ptx.cuh"
@@ -61,6 +62,7 @@ constexpr int kMaxStages = 12;       // (the barrier area holds (3 * 12 + 5) wor
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
 constexpr long long kFinisherWait = 1ll << 15; // cycles a split tile's finisher polls
+constexpr int kMaxDevices = 64;      // per-device launch attribute cache
 
 constexpr int kEpiWarps = 8;         // two per TMEM lane quadrant
 constexpr int kEpiGroups = kEpiWarps / 4;
@@ -976,6 +978,53 @@ bool make_map3(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64_t
 
 size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
+// make_map3 with a small cache: the h-plane and full-vocabulary maps of a
+// call usually repeat the previous calls' (the scratch arena and the weights
+// stay put), and encoding costs more host time than the launch itself.
+struct Map3Key {
+  int dt;
+  const void* ptr;
+  uint64_t cols, rows, row_bytes;
+  uint32_t box_rows, box_atoms;
+  bool operator==(const Map3Key& o) const {
+    return dt == o.dt && ptr == o.ptr && cols == o.cols && rows == o.rows &&
+           row_bytes == o.row_bytes && box_rows == o.box_rows && box_atoms == o.box_atoms;
+  }
+};
+struct Map3Entry {
+  Map3Key key{};
+  bool valid = false;
+  unsigned long long used = 0;
+  CUtensorMap map;
+};
+std::mutex g_map3_mu;
+Map3Entry g_map3[16];
+unsigned long long g_map3_tick = 0;
+
+bool cached_map3(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64_t cols,
+                 uint64_t rows, uint64_t row_bytes, uint32_t box_rows, uint32_t box_atoms) {
+  const Map3Key key{(int)dt, ptr, cols, rows, row_bytes, box_rows, box_atoms};
+  std::lock_guard<std::mutex> lock(g_map3_mu);
+  Map3Entry* lru = &g_map3[0];
+  for (Map3Entry& e : g_map3) {
+    if (e.valid && e.key == key) {
+      e.used = ++g_map3_tick;
+      *m = e.map;
+      return true;
+    }
+    if (!e.valid || e.used < lru->used) lru = &e;
+  }
+  if (!make_map3(&lru->map, dt, ptr, cols, rows, row_bytes, box_rows, box_atoms)) {
+    lru->valid = false;
+    return false;
+  }
+  lru->key = key;
+  lru->valid = true;
+  lru->used = ++g_map3_tick;
+  *m = lru->map;
+  return true;
+}
+
 // W tensor maps, encoded once per weight tensor: map i copies boxes of 64
 // columns x (i + 1) rows of W [V rows, K columns], row stride ld_w (the
 // full-vocabulary path uses only the 128-row map).  A few recently used
@@ -1108,9 +1157,23 @@ static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
                                const TcParams& prm, const TcPlan& pl,
                                cudaStream_t st) {
   auto kern = tc_kernel<HILO, GATHER, EPI, FP8, TM>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)pl.smem_bytes);
+  // the shared-memory opt-in, raised only when a launch needs more than any
+  // earlier one on this device (a host call per launch otherwise)
+  static std::atomic<int> configured[kMaxDevices];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
+  std::atomic<int>* cfg = dev >= 0 && dev < kMaxDevices ? &configured[dev] : nullptr;
+  if (!cfg || cfg->load() < (int)pl.smem_bytes) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)pl.smem_bytes);
+    if (e != cudaSuccess) return e;
+    if (cfg) {
+      int cur = cfg->load();
+      while (cur < (int)pl.smem_bytes && !cfg->compare_exchange_weak(cur, (int)pl.smem_bytes)) {
+      }
+    }
+  }
   return launch_pdl(kern, dim3(pl.G), dim3(FP8 ? kThreadsFp8 : kThreads), pl.smem_bytes, st,
                     mw, mh, prm);
 }
@@ -1147,14 +1210,14 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   if (!fp8 && !w_maps(g, gather, mw)) return cudaErrorInvalidValue;
   // h planes [hilo * Rp rows, Kp columns], zero padded: all atoms of a
   // stage in one copy per plane
-  if (!make_map3(&mh, fp8 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+  if (!cached_map3(&mh, fp8 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
                  Hs, (uint64_t)pl.Kp, (uint64_t)pl.hilo * pl.Rp, (uint64_t)pl.Kp * 2,
                  (uint32_t)pl.BN, (uint32_t)pl.na))
     return cudaErrorInvalidValue;
   // full vocabulary with a width that is a multiple of 64: A likewise
   const int a3d = (!fp8 && !gather && g.K % kAtomK == 0 && g.K >= pl.na * kAtomK) ? 1 : 0;
   mw.a3 = CUtensorMap{};
-  if (a3d && !make_map3(&mw.a3, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
+  if (a3d && !cached_map3(&mw.a3, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
                         (uint64_t)g.V, (uint64_t)g.ld_w * 2, (uint32_t)pl.tm, (uint32_t)pl.na))
     return cudaErrorInvalidValue;
 

@@ -114,7 +114,7 @@ def _check(ctx, status: int):
 
 
 def _ptr(t: Optional[torch.Tensor]):
-    return None if t is None else ctypes.c_void_p(t.data_ptr())
+    return None if t is None else t.data_ptr()
 
 
 def _ld(t: torch.Tensor) -> int:
