@@ -19,10 +19,10 @@
 //                     isolated ids still work as 1-row boxes.
 // Operand B (the h planes, L2-resident) always comes by TMA.
 //
-// Work split: the (vocabulary tile, row block, k-block) iterations -- row
-// blocks innermost, so that a CTA that takes a tile for several row blocks
-// reads its W rows from DRAM once and then from L2 -- are cut into one
-// contiguous range per persistent CTA (one CTA per SM).  When K is
+// Work split: the (row block, vocabulary tile, k-block) iterations -- row
+// blocks outermost, so that CTA c and CTA c + G/RB work on the same W rows
+// at the same time and one of the two reads them from L2 -- are cut into
+// one contiguous range per persistent CTA (one CTA per SM).  When K is
 // short, ranges cover whole tiles; otherwise they are split stream-K style
 // and a tile whose k-range spans several CTAs is finished by the last CTA to
 // arrive: contributors store fp32 partials, count in, and the last one adds
@@ -258,7 +258,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
 #pragma unroll
   for (int g = 0; g < kGroups; ++g) nid[g] = 0;
   auto load_ids = [&](int tl, int (&dst)[kGroups]) {
-    const int j0 = (tl / p.RB) * TM;
+    const int j0 = (tl % p.NT) * TM;
     const int rows = min(TM, p.n - j0);
 #pragma unroll
     for (int g = 0; g < kGroups; ++g) {
@@ -420,7 +420,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
       waited = true;
     };
     while (!stop && sg.next(tile, kb0, kb1)) {
-      const int t = tile / p.RB, rb = tile - t * p.RB;
+      const int rb = tile / p.NT, t = tile - rb * p.NT;
       int nbox = 0;
       uint32_t tx = (uint32_t)(FP8 ? b_bytes : stage_bytes);
       if constexpr (GATHER && !FP8) {
@@ -549,7 +549,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     int si = 0, tile, kb0, kb1;
     while (sg.next(tile, kb0, kb1)) {
       const int acc = si & 1;
-      const int t = tile / p.RB, rb = tile - t * p.RB;
+      const int rb = tile / p.NT, t = tile - rb * p.NT;
       const bool whole = kb0 == 0 && kb1 == p.KB;
       // this lane's vocabulary row in each half: i = hf * 128 + quad * 32 + lane
       int jh[kHalves], idh[kHalves];
@@ -756,7 +756,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     int tile, kb0, kb1;
     bool stop = false;
     while (!stop && sg.next(tile, kb0, kb1)) {
-      const int t = tile / p.RB;
+      const int t = tile % p.NT;
       int rid[16];
 #pragma unroll
       for (int m = 0; m < 16; ++m) {
