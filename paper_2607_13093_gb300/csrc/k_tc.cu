@@ -1094,14 +1094,16 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   };
   row_blocks(max_bn);
   // 256-id tiles: two M = 128 MMAs share every B stage, which halves the
-  // B bytes per A byte, but their two double-buffered accumulators hold at
-  // most 128 hidden-state rows per row block and the tiles are half as
-  // many.  Automatic: only where the row blocks already have <= 128 rows,
-  // the hidden dimension is long and every SM gets >= 4 tiles (measured,
-  // fp32 h: 64 rows x 256000 ids x 4608 is 29 % and 256 rows 19 % faster;
-  // 32 rows x 60000 ids, 320 rows x 51302 ids and 208-row blocks slower).
+  // B bytes per A byte (more of the shared memory holds weights), but their
+  // two double-buffered accumulators hold at most 128 hidden-state rows per
+  // row block and the tiles are half as many.  Automatic: only where the
+  // row blocks already have <= 128 rows, the hidden dimension is long and
+  // there are >= 3/4 tiles per SM (measured over 8..256 rows, 30000..256000
+  // ids, K 2048..8192: 4..44 % faster; decode's 47 tiles on 152 SMs, every
+  // one split three or four ways, 10 % slower; the endpoint's short K and
+  // 160..208-row blocks slower).
   const bool tm256_auto = tile_m == 0 && pl.BN <= 128 && K >= 2048 &&
-                          (long long)pl.RB * ((n + 255) / 256) >= 4ll * sm_count;
+                          4ll * pl.RB * ((n + 255) / 256) >= 3ll * sm_count;
   pl.tm = (!fp8 && (tile_m == 256 || tm256_auto)) ? 256 : 128;
   const int halves = pl.tm / 128;
   if (pl.tm == 256 && pl.BN > 128) row_blocks(max_bn < 128 ? max_bn : 128);
