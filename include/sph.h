@@ -114,11 +114,17 @@ typedef enum sph_option {
   SPH_OPT_TC_MAX_BN = 5,    /* most hidden-state rows one tensor-core tile
                                covers: a multiple of 16 in [16, 256], or 0
                                for automatic (default)                       */
-  SPH_OPT_TC_TILE_M = 6     /* kept vocabulary ids one tensor-core tile
+  SPH_OPT_TC_TILE_M = 6,    /* kept vocabulary ids one tensor-core tile
                                covers: 128, 256 (two 128-row MMAs sharing each
                                hidden-state stage; at most 128 hidden-state
                                rows per tile; bf16 weights only), or 0 for
                                automatic (default)                           */
+  SPH_OPT_TC_FINISH_WAIT = 7 /* clock cycles the designated finisher of a
+                               tensor-core tile split across CTAs polls for
+                               the other contributors' partials (default
+                               2^15, >= 0; 0: no finisher, the last
+                               contributor to count in finishes the tile).
+                               Results are bit-identical for every value.   */
 } sph_option;
 
 /* Set a tunable (SPH_ERR_INVALID_ARG for an unknown option or a value out of

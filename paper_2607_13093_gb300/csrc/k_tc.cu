@@ -61,7 +61,6 @@ constexpr int kMaxBN = 256;
 constexpr int kMaxStages = 12;       // (the barrier area holds (3 * 12 + 5) words)
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
-constexpr long long kFinisherWait = 1ll << 15; // cycles a split tile's finisher polls
 constexpr int kMaxDevices = 64;      // per-device launch attribute cache
 
 constexpr int kEpiWarps = 8;         // two per TMEM lane quadrant
@@ -103,6 +102,7 @@ struct TcParams {
   int* counters;               // [tiles][4 quadrants][epilogue groups], zero between calls
   unsigned* status;
   long long spin_limit;
+  long long finish_wait;       // split-tile finisher poll bound (cycles); 0: no finisher
 };
 
 __device__ __forceinline__ long long cta_of(long long i, long long T, int G) {
@@ -592,7 +592,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
         cnt = (tile * 4 + quad) * kEpiGroups + grp;
         c0 = (int)cta_of((long long)tile * p.KB, p.T, gridDim.x);
         C = (int)cta_of((long long)tile * p.KB + p.KB - 1, p.T, gridDim.x) - c0 + 1;
-        fin = C >= 2 && C <= kMaxC && (int)blockIdx.x == c0 + C - 2;
+        fin = p.finish_wait > 0 && C >= 2 && C <= kMaxC && (int)blockIdx.x == c0 + C - 2;
       }
       // the contributors' partial slots: every contributor after the first
       // starts its range inside this tile, so the tile is its first segment
@@ -634,7 +634,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
         int arrived = 0;
         if (lane == 0) {
           const long long t0 = clock64();
-          const long long bound = limit < kFinisherWait ? limit : kFinisherWait;
+          const long long bound = limit < p.finish_wait ? limit : p.finish_wait;
           while ((arrived = ptx::ld_acquire_gpu(&p.counters[cnt])) != C - 1 &&
                  clock64() - t0 < bound)
             __nanosleep(64);
@@ -1236,7 +1236,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
   prm.inv_tau = g.inv_tau; prm.seg_stats = pl.epi_stats ? stats : nullptr; prm.a3d = a3d;
   prm.P = P; prm.counters = counters;
-  prm.status = g.status; prm.spin_limit = spin_limit;
+  prm.status = g.status; prm.spin_limit = spin_limit; prm.finish_wait = g.finish_wait;
 
   const bool hilo2 = pl.hilo == 2;
   if (pl.tm == 256) {

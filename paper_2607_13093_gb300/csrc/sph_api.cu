@@ -35,6 +35,7 @@ struct sph_ctx {
   int tc_block_k = 0;               // SPH_OPT_TC_BLOCK_K
   int tc_max_bn = 0;                // SPH_OPT_TC_MAX_BN
   int tc_tile_m = 0;                // SPH_OPT_TC_TILE_M
+  long long tc_finish_wait = 1ll << 15;   // SPH_OPT_TC_FINISH_WAIT
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -399,6 +400,10 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
         return fail(ctx, SPH_ERR_INVALID_ARG, "tile_m must be 0, 128 or 256");
       ctx->tc_tile_m = (int)value;
       return SPH_OK;
+    case SPH_OPT_TC_FINISH_WAIT:
+      if (value < 0) return fail(ctx, SPH_ERR_INVALID_ARG, "finish_wait must be >= 0");
+      ctx->tc_finish_wait = value;
+      return SPH_OK;
   }
   return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
 }
@@ -481,7 +486,7 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
   gg.act_bf16 = act_bf16;
   gg.epilogue = sph::EPI_CLOUD;
   gg.bias = bias; gg.clip = clip; gg.partial_out = partial_out;
-  gg.Y = Y; gg.rowmax = rowmax; gg.status = ctx->status;
+  gg.Y = Y; gg.rowmax = rowmax; gg.status = ctx->status; gg.finish_wait = ctx->tc_finish_wait;
   if (use_tc(ctx, rows, wdt)) {
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_h, act_bf16,
                                         ctx->sm_count, 0, ctx->tc_schedule, ctx->tc_stages,
@@ -538,7 +543,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   gg.W = W_l; gg.ld_w = ld_wl; gg.V = V; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
   gg.ids = keep_ids; gg.n = (int)n_keep;
   gg.epilogue = sph::EPI_ENDPOINT;
-  gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale; gg.status = ctx->status;
+  gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale; gg.status = ctx->status; gg.finish_wait = ctx->tc_finish_wait;
   gg.inv_tau = stats_inv_tau(temperature);
   const int greedy = temperature == 0.f;
   if (use_tc(ctx, rows, sph::W_BF16)) {

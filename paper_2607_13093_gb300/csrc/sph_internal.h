@@ -73,6 +73,7 @@ struct GatherGemm {
   const float* row_scale;  // [rows]
   float inv_tau;           // 1 / temperature (softmax statistics)
   unsigned* status;        // device error word
+  long long finish_wait = 1ll << 15;   // split-tile finisher poll (cycles; 0: none)
 };
 
 // CUDA-core gathered GEMV (few rows); returns a cudaError_t.

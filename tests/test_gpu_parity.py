@@ -294,6 +294,43 @@ def test_tensor_core_variants(ctx, block_k, schedule, keep):
 
 
 # ---------------------------------------------------------------------------
+# split tiles: the designated finisher and the count-in fallback agree bit
+# for bit (the partials are added in the same CTA order on both paths)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n_keep", [3000, 6000, 20000])
+@pytest.mark.parametrize("rows", [24, 130])
+def test_split_tile_finisher_matches_count_in(ctx, n_keep, rows):
+    from paper_2607_13093_gb300 import sph
+    w = small(V=24000, d=2000, d_l=1000, rows=rows, n_keep=n_keep, seed=500 + rows)
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 2)
+    ctx.set_option(sph.SPH_OPT_TC_BLOCK_K, 64)
+    outs = []
+    try:
+        for wait in (1 << 15, 0):
+            ctx.set_option(sph.SPH_OPT_TC_FINISH_WAIT, wait)
+            part = torch.empty(w.rows, w.n_keep, dtype=torch.float32, device=DEV)
+            codes, scale, _ = ctx.partial_logits(w.h_cloud, w.W_h, keep_ids=w.keep_ids,
+                                                 clip=w.clip, partial_out=part)
+            z = torch.empty(w.rows, w.n_keep, dtype=torch.float32, device=DEV)
+            tok = ctx.fuse_sample(codes, scale, w.h_local, w.W_l, keep_ids=w.keep_ids,
+                                  temperature=w.tau, seed=w.seed, fused_logits_out=z)
+            ctx.sync()
+            outs.append((part, codes, scale, z, tok))
+        for a, b in zip(*outs):
+            assert torch.equal(a, b)
+        # and the finisher's results are the oracle's
+        ctx.set_option(sph.SPH_OPT_TC_FINISH_WAIT, 1 << 15)
+        check_cloud(ctx, w, rows=sorted({0, rows // 2, rows - 1}))
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_FINISH_WAIT, 1 << 15)
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+        ctx.set_option(sph.SPH_OPT_TC_BLOCK_K, 0)
+
+
+# ---------------------------------------------------------------------------
 # 256-id tensor-core tiles (two M = 128 MMAs per hidden-state stage)
 # ---------------------------------------------------------------------------
 
