@@ -83,6 +83,10 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=300)
     ap.add_argument("--act", choices=["fp32", "bf16"], default="fp32",
                     help="cloud activations: fp32 (exact, two bf16 planes) or bf16-rounded")
+    ap.add_argument("--nosplit", action="store_true",
+                    help="time the unsplit head in place of the split step: the whole hidden "
+                         "state times the whole head over the kept ids, then the sample (one "
+                         "endpoint call without payload; the paper's no-split ablation)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -194,11 +198,11 @@ class OracleSample:
     """One bounded sample of the workload for the oracle: row r of h over a
     slice of L consecutive kept ids (cloud call, then endpoint call)."""
 
-    def __init__(self, w, act="fp32"):
+    def __init__(self, w, act="fp32", nosplit=False):
         import numpy as np
         import torch
         import oracle
-        self.np, self.oracle, self.w, self.act = np, oracle, w, act
+        self.np, self.oracle, self.w, self.act, self.nosplit = np, oracle, w, act, nosplit
 
         def bits(t):
             t = t.detach().cpu().contiguous()
@@ -207,6 +211,7 @@ class OracleSample:
             return t.view(torch.uint8).numpy()
         self.Wh = bits(w.W_h)
         self.Wl = bits(w.W_l)
+        self.Wf = np.concatenate([self.Wl, self.Wh], axis=1) if nosplit else None
         self.ws = None if w.w_scale is None else w.w_scale.cpu().numpy()
         self.h = w.h.cpu().numpy()
         ids = (np.arange(w.V, dtype=np.int64) if w.keep_ids is None
@@ -220,6 +225,10 @@ class OracleSample:
         j0 = (self.i * 7919) % max(1, self.ids.size - L + 1)
         self.i += 1
         ids = self.ids[j0:j0 + L]
+        if self.nosplit:                          # the unsplit head, no payload
+            o.fuse_sample(None, None, self.h[r:r + 1], self.Wf, keep_ids=ids, tau=w.tau,
+                          seed=w.seed, offset=self.i)
+            return L / self.ids.size
         hc = self.h[r:r + 1, w.d_l:]
         hl = self.h[r:r + 1, :w.d_l]
         c = o.partial_logits(hc, self.Wh, w_dtype=w.w_dtype, w_scale=self.ws,
@@ -237,8 +246,8 @@ class OracleSample:
         return max(min(64, self.ids.size), min(self.ids.size, L))
 
 
-def cpu_baseline(w, seconds, act="fp32"):
-    s = OracleSample(w, act)
+def cpu_baseline(w, seconds, act="fp32", nosplit=False):
+    s = OracleSample(w, act, nosplit)
     L = s.calibrate(min(1.0, seconds / 10))
     done = 0.0
     n = 0
@@ -250,7 +259,8 @@ def cpu_baseline(w, seconds, act="fp32"):
     return {"value": done / dt, "unit": UNIT, "cores": oracle_threads(),
             "kind": "oracle",
             "sample": (f"{n} samples of 1 row x {L} of {s.ids.size} kept ids "
-                       f"(cloud + endpoint calls, numpy fp64), scaled to rows"),
+                       + ("(unsplit head + sample" if nosplit else "(cloud + endpoint calls")
+                       + ", numpy fp64), scaled to rows"),
             "seconds": round(dt, 2)}
 
 
@@ -306,15 +316,24 @@ def run_ours(args):
     R, n = w.rows, w.n_keep
     ctx = sph.Context(local)
     act_mode = sph.SPH_ACT_BF16 if args.act == "bf16" else sph.SPH_ACT_FP32
-    ctx.reserve(R, n, max(w.d_h, w.d_l))
+    nosplit = args.nosplit
+    if nosplit and w.w_dtype != "bf16":
+        raise SystemExit("--nosplit needs bf16 weights (the endpoint head is bf16)")
+    ctx.reserve(R, n, w.d if nosplit else max(w.d_h, w.d_l))
 
     # rotation so that bytes between reuses exceed 2x L2
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     wb = 1 if w.w_dtype == "fp8" else 2
     per_copy = n * w.d_h * wb + n * w.d_l * 2
     ncopy = max(1, math.ceil(2 * l2 / per_copy) + 1) if per_copy < 2 * l2 else 1
-    Whs = [w.W_h] + [w.W_h.clone() for _ in range(ncopy - 1)]
-    Wls = [w.W_l] + [w.W_l.clone() for _ in range(ncopy - 1)]
+    if nosplit:
+        # the whole head [V, d] in one tensor (the no-split ablation)
+        Wfs = [torch.cat([w.W_l, w.W_h], dim=1).contiguous()]
+        Wfs += [Wfs[0].clone() for _ in range(ncopy - 1)]
+        Whs = Wls = [None] * ncopy
+    else:
+        Whs = [w.W_h] + [w.W_h.clone() for _ in range(ncopy - 1)]
+        Wls = [w.W_l] + [w.W_l.clone() for _ in range(ncopy - 1)]
     hs = [w.h] + [w.h.roll(i + 1, dims=0).contiguous() for i in range(ncopy - 1)]
     codes = torch.empty(R, n, dtype=torch.int8, device=dev)
     scale = torch.empty(R, dtype=torch.float32, device=dev)
@@ -326,6 +345,19 @@ def run_ours(args):
     def step(i, h=None, events=None):
         c = i % ncopy
         hh = hs[c] if h is None else h
+        if nosplit:                     # one endpoint call over the whole head
+            if events is not None:
+                events[0].record()
+            ctx.fuse_sample(None, None, hh, Wfs[c], keep_ids=w.keep_ids,
+                            temperature=w.tau, seed=w.seed, offset=i, tokens=tokens,
+                            fused_logits_out=z)
+            if events is not None:
+                events[1].record()
+            if w.sessions:
+                ctx.verify_draft(z, w.sessions, w.k, w.draft_tokens, keep_ids=w.keep_ids,
+                                 draft_probs=w.draft_probs, temperature=w.tau,
+                                 seed=w.seed, offset=i, n_accepted=n_acc, next_token=nxt)
+            return
         if events is not None:
             events[0].record()
         ctx.partial_logits(hh[:, w.d_l:], Whs[c], keep_ids=w.keep_ids, clip=w.clip,
@@ -423,6 +455,10 @@ def run_ours(args):
         with torch.cuda.graph(gc, stream=cs):
             for i in range(gsteps):
                 c = i % ncopy
+                if nosplit:
+                    ctx.fuse_sample(None, None, hs[c], Wfs[c], keep_ids=w.keep_ids,
+                                    temperature=w.tau, seed=w.seed, offset=i, tokens=tokens)
+                    continue
                 ctx.partial_logits(hs[c][:, w.d_l:], Whs[c], keep_ids=w.keep_ids,
                                    clip=w.clip, w_row_scale=w.w_scale, bias=w.bias,
                                    codes=codes, row_scale=scale, act_mode=act_mode)
@@ -473,8 +509,13 @@ def run_ours(args):
     value = job_rows_per_s(R, world, args.steps, ms)
     # dominant unit: the cloud call (operand split + gathered contraction +
     # quantization), timed inside the timed graph
-    alg_bytes = wl.algorithmic_bytes_cloud(R, n, w.d_h, wb, fp8_scales=w.w_dtype == "fp8")
-    alg_flops = wl.algorithmic_flops(R, n, w.d_h)
+    if nosplit:
+        # the whole head's kept rows, the whole h, the ids and the tokens
+        alg_bytes = n * w.d * 2 + 4 * R * w.d + 4 * n + 4 * R
+        alg_flops = wl.algorithmic_flops(R, n, w.d)
+    else:
+        alg_bytes = wl.algorithmic_bytes_cloud(R, n, w.d_h, wb, fp8_scales=w.w_dtype == "fp8")
+        alg_flops = wl.algorithmic_flops(R, n, w.d_h)
     ai = alg_flops / alg_bytes
     ridge = peaks["bf16_tflops_sustained"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
     files = ["paper_2607_13093_gb300/csrc/k_tc.cu", "paper_2607_13093_gb300/csrc/k_gemv.cu",
@@ -488,8 +529,10 @@ def run_ours(args):
         pk = peaks["bf16_tflops_sustained"]
         roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": pk,
                 "unit": "TFLOP/s", "frac": round(achieved / pk, 4)}
-    roof.update({"traffic": traffic_for(f"cloud_{args.workload}", files),
-                 "kernel": "cloud call: gathered partial logits + int8 quantization",
+    roof.update({"traffic": None if nosplit else traffic_for(f"cloud_{args.workload}", files),
+                 "kernel": ("unsplit head: gathered whole-d contraction + sample (one endpoint "
+                            "call without payload)" if nosplit else
+                            "cloud call: gathered partial logits + int8 quantization"),
                  "algorithmic_bytes": alg_bytes, "algorithmic_flops": alg_flops,
                  "avg_launch_ms": round(cloud_ms, 5), "timing": cloud_src,
                  "peak_source": f"{peaks_src} (MEASURED_PEAKS.json)" if peaks_src == "measured" else "fallback"})
@@ -501,7 +544,8 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None,
         "dtype": "f32" if args.act == "fp32" else "bf16",
         "data": "synthetic (seeded, paper shapes; weights N(0,0.02) bf16, h RMS-normalised)",
-        "config": {"workload": describe(w), "rows_per_gpu": R, "n_keep": n,
+        "config": {"workload": describe(w) + (", unsplit head (no-split ablation)" if nosplit else ""),
+                   "rows_per_gpu": R, "n_keep": n,
                    "d_h": w.d_h, "d_l": w.d_l, "V": w.V, "weights": w.w_dtype,
                    "accumulate": "fp32",
                    "activations": ("fp32 (exact: bf16 hi + lo planes)" if args.act == "fp32"
@@ -523,14 +567,16 @@ def run_ours(args):
         # downlink of one step (Eq. 21 with b = 8, no tag/metadata/padding):
         # int8 codes of the kept ids + an fp32 scale per row, against the full
         # vocabulary as int8 and as fp32 logits
-        "payload": {"bytes_per_step": sph.sph_payload_bytes(R, n),
+        "payload": {"bytes_per_step": (4 * R * n if nosplit else sph.sph_payload_bytes(R, n)),
+                    "what": ("fp32 logits of the kept ids, which an unsplit cloud head would send"
+                             if nosplit else "int8 codes of the kept ids + an fp32 scale per row"),
                     "full_vocab_int8_bytes": sph.sph_payload_bytes(R, w.V),
                     "full_vocab_fp32_bytes": 4 * R * w.V,
                     "reduction_vs_full_int8": round(
                         1 - sph.sph_payload_bytes(R, n) / sph.sph_payload_bytes(R, w.V), 4)},
     }
     if world == 1 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act)
+        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act, args.nosplit)
     print(json.dumps(out), flush=True)
     if world > 1:
         dist.barrier()
@@ -548,7 +594,7 @@ def run_reference(args):
     from paper_2607_13093_gb300 import workloads as wl
     w = wl.workload(args.workload, device="cpu", rows=args.rows, keep_frac=args.keep,
                     d_l=args.d_l)
-    s = OracleSample(w, args.act)
+    s = OracleSample(w, args.act, args.nosplit)
     budget = 150.0
     L = s.calibrate(budget / max(1, args.steps + args.warmup))
     for _ in range(args.warmup):
@@ -559,15 +605,17 @@ def run_reference(args):
         done += s.run(L)
     dt = time.perf_counter() - t0
     value = done / dt
-    sample = (f"each step: 1 row x {L} of {s.ids.size} kept ids (cloud + endpoint "
-              f"calls, numpy fp64), scaled to rows")
+    sample = (f"each step: 1 row x {L} of {s.ids.size} kept ids "
+              + ("(unsplit head + sample" if args.nosplit else "(cloud + endpoint calls")
+              + ", numpy fp64), scaled to rows")
     out = {"impl": "reference", "metric": METRIC, "value": round(value, 3),
            "unit": UNIT, "n_gpus": int(os.environ.get("WORLD_SIZE", "1")),
            "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic (seeded, paper shapes)",
-           "config": {"workload": describe(w)},
+           "config": {"workload": describe(w) + (", unsplit head (no-split ablation)"
+                                                 if args.nosplit else "")},
            "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "kind": "oracle",
                             "cores": oracle_threads(), "sample": sample},
            "e2e": {"value": round(value, 3), "unit": UNIT,

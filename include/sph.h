@@ -270,7 +270,11 @@ sph_status sph_partial_logits_noalloc(int device, void* cuda_stream,
  *   tokens[r] = keep_ids[j*], j* = the first j with the largest z[r, j]
  *   (the lowest kept id on ties); no uniform is drawn.
  * Arguments
- *   codes int8 [rows, n_keep], row_scale fp32 [rows]: the cloud payload.
+ *   codes int8 [rows, n_keep], row_scale fp32 [rows]: the cloud payload;
+ *   both NULL for no payload (z is the local partial alone: with the whole
+ *   hidden state and head, d_l = d, this is the unsplit head of Eq. 9, the
+ *   comparator of the paper's "no split projection" ablation).  Exactly one
+ *   of them NULL is INVALID_ARG.
  *   h_local fp32 [rows, d_l], row stride ld_hl (the slice h[:, :d_l]).
  *   W_l bf16 [V, d_l] row-major with row stride ld_wl (16-byte multiple).
  *   keep_ids as for sph_partial_logits.  temperature >= 0 and finite.

@@ -223,7 +223,11 @@ def local_partial(h_local, W_l_bits, keep_ids=None) -> np.ndarray:
 
 
 def fuse(codes, row_scale, z_local) -> np.ndarray:
-    """z = dequant(z_cloud) + z_end (Eq. 13); dequant(code) = code * s_r."""
+    """z = dequant(z_cloud) + z_end (Eq. 13); dequant(code) = code * s_r.
+    Without a payload (codes and row_scale None) z is z_end alone: given
+    the whole hidden state and head, the unsplit head of Eq. 9."""
+    if codes is None and row_scale is None:
+        return np.asarray(z_local, dtype=np.float64)
     s = np.asarray(row_scale, dtype=np.float32).astype(np.float64)
     return np.asarray(codes).astype(np.float64) * s[:, None] + z_local
 

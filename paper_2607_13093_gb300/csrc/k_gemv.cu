@@ -170,7 +170,7 @@ gemv_kernel(const GatherGemm g, const int row0) {
           g.Y[o] = yc;
           lmax = fmaxf(lmax, fabsf(yc));
         } else {
-          g.Y[o] = y + (float)g.codes[o] * g.row_scale[row0 + r];
+          g.Y[o] = g.codes ? y + (float)g.codes[o] * g.row_scale[row0 + r] : y;
         }
       }
     }

@@ -141,6 +141,12 @@ struct Payload {
 };
 __device__ __forceinline__ void load_payload(const TcParams& p, int row0, int j, int lane,
                                              Payload& pl) {
+  if (!p.codes) {                      // no payload: z is the local partial alone
+#pragma unroll
+    for (int q = 0; q < 16; ++q) pl.c[q] = 0;
+    pl.s = 0.f;
+    return;
+  }
   const int8_t* col = p.codes + min(j, p.n - 1);
 #pragma unroll
   for (int q = 0; q < 16; ++q) pl.c[q] = __ldg(col + (int64_t)min(row0 + q, p.R - 1) * p.n);
@@ -149,7 +155,7 @@ __device__ __forceinline__ void load_payload(const TcParams& p, int row0, int j,
 // Warm L2 with the codes of rows row0..row0+nrows-1 at the 32 ids from j0.
 __device__ __forceinline__ void prefetch_codes(const TcParams& p, int row0, int nrows, int j0,
                                                int lane) {
-  if (j0 >= p.n) return;
+  if (j0 >= p.n || !p.codes) return;
   const int8_t* col = p.codes + j0;
   const int last = min(31, p.n - 1 - j0);
   for (int r = row0 + lane; r < min(row0 + nrows, p.R); r += 32) {

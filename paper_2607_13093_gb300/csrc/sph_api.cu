@@ -517,8 +517,10 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
                            uint64_t offset, int32_t* tokens,
                            float* fused_logits_out) {
   if (!ctx) return SPH_ERR_INVALID_ARG;
-  if (!codes || !row_scale || !h_local || !W_l || !tokens)
-    return fail(ctx, SPH_ERR_INVALID_ARG, "codes, row_scale, h_local, W_l and tokens must be non-NULL");
+  if (!h_local || !W_l || !tokens)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "h_local, W_l and tokens must be non-NULL");
+  if (!codes != !row_scale)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "codes and row_scale must both be given or both be NULL");
   if (rows < 1 || rows > (1 << 20)) return fail(ctx, SPH_ERR_INVALID_ARG, "rows=%lld out of [1, 2^20]", (long long)rows);
   if (d_l < 1) return fail(ctx, SPH_ERR_INVALID_ARG, "d_l must be >= 1");
   if (ld_hl < d_l || ld_wl < d_l) return fail(ctx, SPH_ERR_INVALID_ARG, "ld_hl and ld_wl must be >= d_l");

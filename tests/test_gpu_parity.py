@@ -8,8 +8,9 @@ import pytest
 import torch
 
 from paper_2607_13093_gb300 import workloads as wl
-from _parity import (check_cloud, check_endpoint, check_verify, oracle_cloud,
-                     np_)
+import oracle
+from _parity import (GREEDY_GAP, MARGIN, assert_close, bits, check_cloud, check_endpoint,
+                     check_verify, np_, oracle_cloud)
 
 pytestmark = pytest.mark.gpu
 
@@ -291,6 +292,43 @@ def test_tensor_core_variants(ctx, block_k, schedule, keep):
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
         ctx.set_option(sph.SPH_OPT_TC_BLOCK_K, 0)
         ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+
+
+# ---------------------------------------------------------------------------
+# the unsplit head (no payload, whole hidden state and head): the comparator
+# of the paper's "no split projection" ablation
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("kw", [dict(V=4000, d=1024, d_l=128, rows=32, n_keep=1500, tau=0.8),
+                                dict(V=3000, d=600, d_l=40, rows=3, n_keep=3000),
+                                dict(V=6000, d=1088, d_l=64, rows=20, n_keep=2400, tau=0.0)])
+def test_unsplit_head(path_ctx, kw):
+    w = small(seed=611, **kw)
+    W_full = torch.cat([w.W_l, w.W_h], dim=1).contiguous()
+    z = torch.empty(w.rows, w.n_keep, device=DEV)
+    tok = path_ctx.fuse_sample(None, None, w.h, W_full, keep_ids=w.keep_ids,
+                               temperature=w.tau, seed=w.seed, offset=3, fused_logits_out=z)
+    path_ctx.sync()
+    ids = np_(w.keep_ids)
+    ids = np.arange(w.V) if ids is None else ids
+    zref = oracle.fuse(None, None, oracle.local_partial(np_(w.h), bits(W_full), ids))
+    assert_close(np_(z), zref, "unsplit logits")
+    if w.tau == 0:
+        j, gap = oracle.greedy_rows(zref)
+        ok = gap >= GREEDY_GAP
+    else:
+        j, margin = oracle.sample_rows(zref, w.tau, oracle.philox_uniform(w.seed, np.arange(w.rows), 0, 3))
+        ok = margin >= MARGIN
+    got = np_(tok)
+    assert not ((got != ids[j]) & ok).any()
+
+
+def test_payload_arguments_together(ctx):
+    from paper_2607_13093_gb300 import sph
+    w = small(V=2000, d=512, d_l=64, rows=4, n_keep=800)
+    with pytest.raises(sph.SphError):
+        ctx.fuse_sample(None, torch.ones(w.rows, device=DEV), w.h_local, w.W_l,
+                        keep_ids=w.keep_ids)
 
 
 # ---------------------------------------------------------------------------

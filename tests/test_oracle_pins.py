@@ -77,6 +77,23 @@ def test_split_partials_equal_full_head(act_mode):
                                z_full, rtol=1e-12, atol=1e-14)
 
 
+def test_unsplit_endpoint_call_is_full_head():
+    """Without a payload the endpoint call over the whole hidden state and
+    head computes the unsplit head (Eq. 9) -- the comparator of the paper's
+    "no split projection" ablation -- and samples from it."""
+    w = tiny(with_bias=False)
+    ids = w.keep_ids.numpy()
+    h = w.h.numpy().astype(np.float64)
+    W_full = torch.cat([w.W_l, w.W_h], dim=1)
+    z_full = brute_full_head(h, W_full.double().numpy(), None)[:, ids]
+    out = oracle.fuse_sample(None, None, w.h.numpy(), bits16(W_full.contiguous()),
+                             keep_ids=ids, tau=1.0, seed=5, offset=2)
+    np.testing.assert_allclose(out["z"], z_full, rtol=1e-12, atol=1e-14)
+    u = oracle.philox_uniform(5, np.arange(w.rows), 0, 2)
+    j, _ = oracle.sample_rows(z_full, 1.0, u)
+    assert (out["tokens"] == ids[j]).all()
+
+
 def test_fused_logits_within_dequantization_bound():
     """z = code * s + z_end reproduces the full head (Eq. 13) to within half
     a quantization step (Eq. 18) when nothing is clipped."""
