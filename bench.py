@@ -87,6 +87,8 @@ def parse():
                     help="time the unsplit head in place of the split step: the whole hidden "
                          "state times the whole head over the kept ids, then the sample (one "
                          "endpoint call without payload; the paper's no-split ablation)")
+    ap.add_argument("--sampler", choices=["cdf", "gumbel"], default="cdf",
+                    help="endpoint draw: inverse CDF (default) or Gumbel-max")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -198,11 +200,12 @@ class OracleSample:
     """One bounded sample of the workload for the oracle: row r of h over a
     slice of L consecutive kept ids (cloud call, then endpoint call)."""
 
-    def __init__(self, w, act="fp32", nosplit=False):
+    def __init__(self, w, act="fp32", nosplit=False, sampler="cdf"):
         import numpy as np
         import torch
         import oracle
         self.np, self.oracle, self.w, self.act, self.nosplit = np, oracle, w, act, nosplit
+        self.sampler = sampler
 
         def bits(t):
             t = t.detach().cpu().contiguous()
@@ -227,14 +230,14 @@ class OracleSample:
         ids = self.ids[j0:j0 + L]
         if self.nosplit:                          # the unsplit head, no payload
             o.fuse_sample(None, None, self.h[r:r + 1], self.Wf, keep_ids=ids, tau=w.tau,
-                          seed=w.seed, offset=self.i)
+                          seed=w.seed, offset=self.i, sampler=self.sampler)
             return L / self.ids.size
         hc = self.h[r:r + 1, w.d_l:]
         hl = self.h[r:r + 1, :w.d_l]
         c = o.partial_logits(hc, self.Wh, w_dtype=w.w_dtype, w_scale=self.ws,
                              keep_ids=ids, clip=w.clip, act_mode=self.act)
         o.fuse_sample(c["codes"], c["row_scale"], hl, self.Wl, keep_ids=ids,
-                      tau=w.tau, seed=w.seed, offset=self.i)
+                      tau=w.tau, seed=w.seed, offset=self.i, sampler=self.sampler)
         return L / self.ids.size                  # rows of the metric done
 
     def calibrate(self, seconds_per_step):
@@ -246,8 +249,8 @@ class OracleSample:
         return max(min(64, self.ids.size), min(self.ids.size, L))
 
 
-def cpu_baseline(w, seconds, act="fp32", nosplit=False):
-    s = OracleSample(w, act, nosplit)
+def cpu_baseline(w, seconds, act="fp32", nosplit=False, sampler="cdf"):
+    s = OracleSample(w, act, nosplit, sampler)
     L = s.calibrate(min(1.0, seconds / 10))
     done = 0.0
     n = 0
@@ -316,6 +319,8 @@ def run_ours(args):
     R, n = w.rows, w.n_keep
     ctx = sph.Context(local)
     act_mode = sph.SPH_ACT_BF16 if args.act == "bf16" else sph.SPH_ACT_FP32
+    if args.sampler == "gumbel":
+        ctx.set_option(sph.SPH_OPT_SAMPLER, sph.SPH_SAMPLER_GUMBEL)
     nosplit = args.nosplit
     if nosplit and w.w_dtype != "bf16":
         raise SystemExit("--nosplit needs bf16 weights (the endpoint head is bf16)")
@@ -548,6 +553,7 @@ def run_ours(args):
                    "rows_per_gpu": R, "n_keep": n,
                    "d_h": w.d_h, "d_l": w.d_l, "V": w.V, "weights": w.w_dtype,
                    "accumulate": "fp32",
+                   "sampler": "Gumbel-max" if args.sampler == "gumbel" else "inverse CDF",
                    "activations": ("fp32 (exact: bf16 hi + lo planes)" if args.act == "fp32"
                                    else "bf16-rounded (one plane)"),
                    "l2": (f"inputs rotate over {ncopy} weight/h copies, "
@@ -576,7 +582,8 @@ def run_ours(args):
                         1 - sph.sph_payload_bytes(R, n) / sph.sph_payload_bytes(R, w.V), 4)},
     }
     if world == 1 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act, args.nosplit)
+        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act, args.nosplit,
+                                           args.sampler)
     print(json.dumps(out), flush=True)
     if world > 1:
         dist.barrier()
@@ -594,7 +601,7 @@ def run_reference(args):
     from paper_2607_13093_gb300 import workloads as wl
     w = wl.workload(args.workload, device="cpu", rows=args.rows, keep_frac=args.keep,
                     d_l=args.d_l)
-    s = OracleSample(w, args.act, args.nosplit)
+    s = OracleSample(w, args.act, args.nosplit, args.sampler)
     budget = 150.0
     L = s.calibrate(budget / max(1, args.steps + args.warmup))
     for _ in range(args.warmup):

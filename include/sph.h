@@ -119,12 +119,20 @@ typedef enum sph_option {
                                hidden-state stage; at most 128 hidden-state
                                rows per tile; bf16 weights only), or 0 for
                                automatic (default)                           */
-  SPH_OPT_TC_FINISH_WAIT = 7 /* clock cycles the designated finisher of a
+  SPH_OPT_TC_FINISH_WAIT = 7, /* clock cycles the designated finisher of a
                                tensor-core tile split across CTAs polls for
                                the other contributors' partials (default
                                2^15, >= 0; 0: no finisher, the last
                                contributor to count in finishes the tile).
                                Results are bit-identical for every value.   */
+  SPH_OPT_SAMPLER = 8       /* the draw of sph_fuse_sample at temperature > 0:
+                               0 inverse CDF (default), 1 Gumbel-max: the
+                               first index j of the largest
+                               z_j / temperature - log(-log u_j), u_j = word
+                               j mod 4 of the Philox output for counter
+                               (r, 2^31 + j / 4, offset lo, offset hi),
+                               ((x >> 9) + 1/2) * 2^-23 (a draw from the same
+                               softmax, with other random numbers)         */
 } sph_option;
 
 /* Set a tunable (SPH_ERR_INVALID_ARG for an unknown option or a value out of

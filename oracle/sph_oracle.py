@@ -277,13 +277,43 @@ def greedy_rows(z):
     return j, top2[:, 1] - top2[:, 0]
 
 
+# Gumbel-max sampling: an alternative single-pass sampler (reading listed
+# in the design notes).  Index j of row r gets its own uniform: word j mod 4
+# of the Philox output for counter (r, 2^31 + j div 4, offset lo, offset hi)
+# under key (seed lo, seed hi), u = ((x >> 9) + 1/2) * 2^-23, which lies in
+# (0, 1) and is exact in fp32 and fp64.
+GUMBEL_TAG = 0x80000000
+
+
+def gumbel_uniforms(seed: int, rows: int, n: int, offset: int) -> np.ndarray:
+    """The [rows, n] uniforms of Gumbel-max sampling (see GUMBEL_TAG)."""
+    g = (n + 3) // 4
+    r = np.repeat(np.arange(rows, dtype=np.uint64), g)
+    q = np.tile(np.arange(g, dtype=np.uint64), rows) | np.uint64(GUMBEL_TAG)
+    off = int(offset)
+    words = philox4x32_10(r, q, np.full(r.shape, off & _MASK32, np.uint64),
+                          np.full(r.shape, (off >> 32) & _MASK32, np.uint64),
+                          int(seed) & _MASK32, (int(seed) >> 32) & _MASK32)
+    x = np.stack(words, axis=-1).reshape(rows, 4 * g)[:, :n]
+    return ((x >> np.uint32(9)).astype(np.float64) + 0.5) * 2.0 ** -23
+
+
+def gumbel_rows(z, tau: float, u):
+    """Gumbel-max draw: per row the first index of the largest
+    z_j / tau - log(-log u_j), a sample from softmax(z / tau) (the Gumbel-max
+    property).  Returns (index, margin = top-two key gap)."""
+    key = np.asarray(z, dtype=np.float64) / tau - np.log(-np.log(u))
+    return greedy_rows(key)
+
+
 def fuse_sample(codes, row_scale, h_local, W_l_bits, *, keep_ids=None,
-                tau=1.0, seed=0, offset=0):
+                tau=1.0, seed=0, offset=0, sampler="cdf"):
     """Endpoint call: local partial, fuse, mask, softmax(./tau), one Philox
     uniform per row (purpose 0), inverse-CDF draw; tau = 0 is greedy
-    decoding (no uniform).  Returns vocabulary-id `tokens`, the `margin` of
-    each draw (CDF distance, or for greedy the top-two gap) and the fused
-    logits `z`."""
+    decoding (no uniform); sampler="gumbel" draws by Gumbel-max instead
+    (gumbel_rows).  Returns vocabulary-id `tokens`, the `margin` of each
+    draw (CDF distance, or for greedy and Gumbel-max the top-two gap) and
+    the fused logits `z`."""
     V = W_l_bits.shape[0]
     ids = _ids(keep_ids, V)
     zl = local_partial(h_local, W_l_bits, ids)
@@ -292,6 +322,9 @@ def fuse_sample(codes, row_scale, h_local, W_l_bits, *, keep_ids=None,
     u = philox_uniform(seed, np.arange(R), 0, offset)
     if tau == 0:
         j, margin = greedy_rows(z)
+    elif sampler == "gumbel":
+        u = gumbel_uniforms(seed, R, z.shape[1], offset)
+        j, margin = gumbel_rows(z, tau, u)
     else:
         j, margin = sample_rows(z, tau, u)
     return dict(tokens=ids[j].astype(np.int32), margin=margin, z=z, u=u,

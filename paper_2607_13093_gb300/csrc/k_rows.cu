@@ -12,6 +12,8 @@
 // the 32x smaller segment statistics.  A draw is a three-level search in
 // ascending id order -- 1024-id chunks, 32-id segments, ids -- whose CDF is
 // the oracle's up to fp32 rounding.
+#include <climits>
+
 #include "sm100_ptx.cuh"
 #include "sph_common.cuh"
 #include "sph_internal.h"
@@ -301,6 +303,70 @@ sample_rows_kernel(const float* __restrict__ Z, int n, const float2* __restrict_
 }
 
 // ---------------------------------------------------------------------------
+// Gumbel-max sampling (the alternative single-pass sampler): the first index
+// of the largest z_j / tau - log(-log u_j) is a draw from softmax(z / tau).
+// Index j of row r takes word j mod 4 of the Philox output for counter
+// (r, 2^31 + j / 4, offset lo, offset hi), u = ((x >> 9) + 1/2) * 2^-23,
+// strictly inside (0, 1).  A block per row; no softmax statistics needed.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kGumbelTag = 0x80000000u;
+constexpr int kGumbelThreads = 256;
+__global__ void __launch_bounds__(kGumbelThreads)
+gumbel_rows_kernel(const float* __restrict__ Z, int n, const int32_t* __restrict__ ids,
+                   float inv_tau, uint64_t seed, uint64_t offset,
+                   int32_t* __restrict__ tokens) {
+  __shared__ float s_key[kGumbelThreads / 32];
+  __shared__ int s_idx[kGumbelThreads / 32];
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int r = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const float* z = Z + (int64_t)r * n;
+  const uint2 key = make_uint2((uint32_t)seed, (uint32_t)(seed >> 32));
+  float best = -INFINITY;
+  int bj = INT_MAX;
+  const int groups = (n + 3) >> 2;
+  for (int q = threadIdx.x; q < groups; q += blockDim.x) {
+    const uint4 x = philox4x32_10(
+        make_uint4((uint32_t)r, kGumbelTag | (uint32_t)q, (uint32_t)offset,
+                   (uint32_t)(offset >> 32)), key);
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int j = 4 * q + t;
+      if (j < n) {
+        const float u = ((float)(w[t] >> 9) + 0.5f) * 1.1920928955078125e-07f;  // 2^-23
+        const float k = z[j] * inv_tau - logf(-logf(u));
+        if (k > best) { best = k; bj = j; }    // a thread's j ascend: ties keep the first
+      }
+    }
+  }
+  // the largest key, the lowest index among equal keys
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const float ob = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+    const int oj = __shfl_xor_sync(0xFFFFFFFFu, bj, o);
+    if (ob > best || (ob == best && oj < bj)) { best = ob; bj = oj; }
+  }
+  if (lane == 0) { s_key[warp] = best; s_idx[warp] = bj; }
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+    best = lane < nw ? s_key[lane] : -INFINITY;
+    bj = lane < nw ? s_idx[lane] : INT_MAX;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      const float ob = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+      const int oj = __shfl_xor_sync(0xFFFFFFFFu, bj, o);
+      if (ob > best || (ob == best && oj < bj)) { best = ob; bj = oj; }
+    }
+    if (lane == 0) {
+      const int j = bj < n ? bj : 0;
+      tokens[r] = ids ? ids[j] : j;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // greedy decoding (temperature 0): the first id of the row maximum
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int warp_min_int(int v) {
@@ -551,6 +617,13 @@ cudaError_t launch_sample_segments(const float* Z, int rows, int n, const float2
   return launch_pdl(sample_seg_kernel, dim3((rows + kWarps - 1) / kWarps),
                     dim3(kWarps * 32), 0, st, Z, rows, n, stats, nseg, cstats, ids, inv_tau,
                     seed, offset, tokens);
+}
+
+cudaError_t launch_gumbel(const float* Z, int rows, int n, const int32_t* ids, float inv_tau,
+                          uint64_t seed, uint64_t offset, int32_t* tokens, cudaStream_t st) {
+  if (rows < 1) return cudaErrorInvalidValue;
+  return launch_pdl(gumbel_rows_kernel, dim3(rows), dim3(kGumbelThreads), 0, st, Z, n, ids,
+                    inv_tau, seed, offset, tokens);
 }
 
 cudaError_t launch_sample_rows(const float* Z, int rows, int n, const float2* stats,

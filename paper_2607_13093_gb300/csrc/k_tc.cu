@@ -1240,7 +1240,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.epilogue = g.epilogue; prm.bias = g.bias;
   prm.clip = g.clip; prm.partial_out = g.partial_out; prm.Y = g.Y;
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
-  prm.inv_tau = g.inv_tau; prm.seg_stats = pl.epi_stats ? stats : nullptr; prm.a3d = a3d;
+  prm.inv_tau = g.inv_tau; prm.seg_stats = (pl.epi_stats && !g.no_stats) ? stats : nullptr; prm.a3d = a3d;
   prm.P = P; prm.counters = counters;
   prm.status = g.status; prm.spin_limit = spin_limit; prm.finish_wait = g.finish_wait;
 

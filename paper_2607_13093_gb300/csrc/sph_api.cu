@@ -36,6 +36,7 @@ struct sph_ctx {
   int tc_max_bn = 0;                // SPH_OPT_TC_MAX_BN
   int tc_tile_m = 0;                // SPH_OPT_TC_TILE_M
   long long tc_finish_wait = 1ll << 15;   // SPH_OPT_TC_FINISH_WAIT
+  int sampler = 0;                  // SPH_OPT_SAMPLER
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -404,6 +405,10 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       if (value < 0) return fail(ctx, SPH_ERR_INVALID_ARG, "finish_wait must be >= 0");
       ctx->tc_finish_wait = value;
       return SPH_OK;
+    case SPH_OPT_SAMPLER:
+      if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "sampler must be 0 or 1");
+      ctx->sampler = (int)value;
+      return SPH_OK;
   }
   return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
 }
@@ -548,6 +553,16 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale; gg.status = ctx->status; gg.finish_wait = ctx->tc_finish_wait;
   gg.inv_tau = stats_inv_tau(temperature);
   const int greedy = temperature == 0.f;
+  // Gumbel-max draws need no softmax statistics: the epilogue skips them
+  const bool gumbel = ctx->sampler == 1 && !greedy;
+  gg.no_stats = gumbel;
+  auto draw_gumbel = [&] {
+    return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
+                           return sph::launch_gumbel(Z, (int)rows, (int)n_keep, keep_ids,
+                                                     gg.inv_tau, seed, offset, tokens,
+                                                     ctx->stream);
+                         }), "sample launch");
+  };
   if (use_tc(ctx, rows, sph::W_BF16)) {
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0,
                                         ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
@@ -558,6 +573,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
                        }), "tensor-core launch");
     if (st) return st;
+    if (gumbel) return draw_gumbel();
     return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                            return sph::launch_sample_from_stats(
                                Z, (int)rows, (int)n_keep, pl, tcs, cstats, keep_ids,
@@ -570,6 +586,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
                        return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
                      }), "gemv launch");
   if (st) return st;
+  if (gumbel) return draw_gumbel();
   return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                          cudaError_t e = sph::launch_seg_stats(Z, (int)rows, (int)n_keep,
                                                                gg.inv_tau, stats,

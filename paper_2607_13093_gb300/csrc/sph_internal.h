@@ -74,6 +74,7 @@ struct GatherGemm {
   float inv_tau;           // 1 / temperature (softmax statistics)
   unsigned* status;        // device error word
   long long finish_wait = 1ll << 15;   // split-tile finisher poll (cycles; 0: none)
+  bool no_stats = false;   // endpoint: skip the softmax statistics (Gumbel-max draw)
 };
 
 // CUDA-core gathered GEMV (few rows); returns a cudaError_t.
@@ -134,6 +135,10 @@ cudaError_t launch_seg_stats(const float* Z, int rows, int n, float inv_tau,
 cudaError_t launch_chunk_stats(const float2* stats, int rows, int nseg,
                                float inv_tau, float2* cstats, int sm_count,
                                cudaStream_t st);
+// Gumbel-max draw per row over Z (fp32 [rows, n]): the first index of the
+// largest z * inv_tau - log(-log u) with per-(row, index) Philox uniforms.
+cudaError_t launch_gumbel(const float* Z, int rows, int n, const int32_t* ids, float inv_tau,
+                          uint64_t seed, uint64_t offset, int32_t* tokens, cudaStream_t st);
 // One inverse-CDF draw per row from segment statistics alone (nseg per row):
 // a block per row makes the chunk statistics in shared memory first.
 // cudaErrorNotSupported (nothing launched) past 4096 chunks per row.

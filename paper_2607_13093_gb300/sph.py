@@ -29,6 +29,8 @@ SPH_OPT_TC_MIN_ROWS, SPH_OPT_SPIN_LIMIT = 0, 1
 SPH_OPT_TC_SCHEDULE, SPH_OPT_TC_STAGES, SPH_OPT_TC_BLOCK_K, SPH_OPT_TC_MAX_BN = 2, 3, 4, 5
 SPH_OPT_TC_TILE_M = 6
 SPH_OPT_TC_FINISH_WAIT = 7
+SPH_OPT_SAMPLER = 8
+SPH_SAMPLER_CDF, SPH_SAMPLER_GUMBEL = 0, 1
 
 _c_void_p = ctypes.c_void_p
 _i64 = ctypes.c_int64

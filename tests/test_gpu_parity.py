@@ -323,6 +323,35 @@ def test_unsplit_head(path_ctx, kw):
     assert not ((got != ids[j]) & ok).any()
 
 
+GUMBEL_GAP = 2e-4     # Gumbel-max: top-two key gap of the fp64 keys
+
+
+@pytest.mark.parametrize("kw", [dict(V=4000, d=1024, d_l=128, rows=32, n_keep=1500, tau=0.8),
+                                dict(V=3000, d=600, d_l=40, rows=3, n_keep=3000, tau=1.3),
+                                dict(V=9000, d=900, d_l=96, rows=40, n_keep=4001, tau=0.5)])
+def test_gumbel_sampler(path_ctx, kw):
+    from paper_2607_13093_gb300 import sph
+    w = small(seed=733, **kw)
+    pc, ps = wl.make_payload(w.rows, w.n_keep, seed=9, device=DEV)
+    z = torch.empty(w.rows, w.n_keep, device=DEV)
+    path_ctx.set_option(sph.SPH_OPT_SAMPLER, sph.SPH_SAMPLER_GUMBEL)
+    try:
+        tok = path_ctx.fuse_sample(pc, ps, w.h_local, w.W_l, keep_ids=w.keep_ids,
+                                   temperature=w.tau, seed=w.seed, offset=11, fused_logits_out=z)
+        path_ctx.sync()
+    finally:
+        path_ctx.set_option(sph.SPH_OPT_SAMPLER, sph.SPH_SAMPLER_CDF)
+    ids = np_(w.keep_ids)
+    ids = np.arange(w.V) if ids is None else ids
+    zref = oracle.fuse(np_(pc), np_(ps), oracle.local_partial(np_(w.h_local), bits(w.W_l), ids))
+    assert_close(np_(z), zref, "fused logits")
+    u = oracle.gumbel_uniforms(w.seed, w.rows, w.n_keep, 11)
+    j, gap = oracle.gumbel_rows(zref, w.tau, u)
+    got = np_(tok)
+    bad = (got != ids[j]) & (gap >= GUMBEL_GAP)
+    assert not bad.any(), f"rows {np.nonzero(bad)[0]}: {got[bad]} vs {ids[j][bad]}"
+
+
 def test_payload_arguments_together(ctx):
     from paper_2607_13093_gb300 import sph
     w = small(V=2000, d=512, d_l=64, rows=4, n_keep=800)

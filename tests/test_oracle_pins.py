@@ -515,3 +515,42 @@ def test_greedy_verify_matches_its_closed_form_and_the_small_tau_limit():
         gaps = oracle.greedy_rows(Z[s * (k + 1):(s + 1) * (k + 1)])[1]
         if gaps.min() > 0.05:
             assert acc == i and j == a[s, i]
+
+
+# ---------------------------------------------------------------------------
+# Gumbel-max sampling (the alternative single-pass sampler)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("tau", [0.7, 1.0, 2.0])
+def test_gumbel_max_draws_follow_softmax(tau):
+    """argmax(z/tau + Gumbel noise) is a draw from softmax(z/tau): a chi-square
+    test over 60000 independent rows of the same logits."""
+    z0 = np.array([0.3, -1.2, 2.0, 0.0, 1.1, -0.4])
+    N, n = 60000, z0.size
+    u = oracle.gumbel_uniforms(seed=77, rows=N, n=n, offset=5)
+    j, _ = oracle.gumbel_rows(np.tile(z0, (N, 1)), tau, u)
+    counts = np.bincount(j, minlength=n)
+    p = np.exp(z0 / tau) / np.exp(z0 / tau).sum()
+    chi2 = ((counts - N * p) ** 2 / (N * p)).sum()
+    assert chi2 < 25.7          # df = 5, upper tail 1e-4
+
+
+def test_gumbel_uniforms_are_strictly_inside_the_unit_interval():
+    u = oracle.gumbel_uniforms(seed=3, rows=64, n=4099, offset=2 ** 40 + 7)
+    assert u.min() > 0.0 and u.max() < 1.0
+    # 23 random bits per value, on the grid (k + 1/2) 2^-23
+    k = u * 2.0 ** 23 - 0.5
+    assert np.all(k == np.round(k))
+    # indices 4q .. 4q+3 use the four words of one Philox block
+    w = oracle.philox4x32_10(np.uint64(5), np.uint64(oracle.GUMBEL_TAG | 1), np.uint64(2 ** 40 + 7 & 0xFFFFFFFF),
+                             np.uint64((2 ** 40 + 7) >> 32), 3, 0)
+    assert [int(x) >> 9 for x in w] == [int(v) for v in k[5, 4:8]]
+
+
+def test_gumbel_max_small_temperature_is_greedy():
+    rng = np.random.default_rng(4)
+    z = rng.normal(size=(16, 300))
+    u = oracle.gumbel_uniforms(seed=1, rows=16, n=300, offset=0)
+    j, _ = oracle.gumbel_rows(z, 1e-9, u)
+    g, gap = oracle.greedy_rows(z)
+    assert (gap > 1e-6).all() and (j == g).all()
