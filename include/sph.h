@@ -117,8 +117,7 @@ typedef enum sph_option {
   SPH_OPT_TC_TILE_M = 6,    /* kept vocabulary ids one tensor-core tile
                                covers: 128, 256 (two 128-row MMAs sharing each
                                hidden-state stage; at most 128 hidden-state
-                               rows per tile; bf16 weights only), or 0 for
-                               automatic (default)                           */
+                               rows per tile), or 0 for automatic (default)  */
   SPH_OPT_TC_FINISH_WAIT = 7, /* clock cycles the designated finisher of a
                                tensor-core tile split across CTAs polls for
                                the other contributors' partials (default

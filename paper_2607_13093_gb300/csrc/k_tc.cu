@@ -32,16 +32,23 @@
 // tcgen05.mma (one thread), warps 2-9 drain the double-buffered accumulator
 // (tcgen05.ld) and run the fused epilogue -- two warps per TMEM lane
 // quadrant, so that the epilogue's dependent shuffle / exp chains of one
-// warp overlap with the other's; with fp8 weights warps 10-13 convert the
-// e4m3 A tiles.  Every wait is bounded; a wait that gives up sets the
+// warp overlap with the other's.  Every wait is bounded; a wait that gives up sets the
 // context's error word and the CTA winds down after its copies and MMAs
 // have landed.
+//
+// fp8 (e4m3) weights: the raw e4m3 rows are the A operand of
+// tcgen05.mma kind::f8f6f4 (a 128-byte atom is 128 elements); h is split
+// into e4m3 planes under a per-row power-of-two scale (4 planes: 2^-13 of
+// |h|; 2 planes reproduce bf16-rounded h) that all add into one fp32
+// accumulator; the epilogue multiplies by the row's scale and the weight
+// row's scale.
 //
 // Epilogues: cloud = + bias, optional unclipped store, clip, store, row |max|
 // (atomicMax); endpoint = + code * row_scale (Eq. 13), store z, and the
 // softmax statistics (max, sum of exp((z - max)/tau)) of every 32-id segment
 // of every row, which the sampler uses instead of re-reading the row.
 #include <cuda.h>
+#include <cuda_fp8.h>
 #include <cuda_runtime.h>
 
 #include <atomic>
@@ -66,8 +73,7 @@ constexpr int kMaxDevices = 64;      // per-device launch attribute cache
 constexpr int kEpiWarps = 8;         // two per TMEM lane quadrant
 constexpr int kEpiGroups = kEpiWarps / 4;
 constexpr int kThreads = 64 + 32 * kEpiWarps;       // producer, MMA, epilogue
-constexpr int kThreadsFp8 = kThreads + 128;         // + four converter warps (fp8)
-constexpr int kMaxBNFp8 = 128;       // h rows per block with fp8 weights
+constexpr int kAtomE8 = 128;         // e4m3 elements per 128-byte atom
 constexpr int kBoxHeights = 128;     // row boxes of 1, 2, 3, ..., 128 rows (map h-1)
 constexpr int kMaxBoxes = 260;       // row boxes of one tile (one per run, two per
                                      // run longer than 128 rows in a 256-row tile)
@@ -84,7 +90,7 @@ struct TcParams {
   int na;                      // swizzle atoms per k-block (k-block = 64 * na)
   long long T;                 // total iterations RB * NT * KB
   const int32_t* ids;          // gather path: sorted ids
-  const uint8_t* W8;           // fp8 path: e4m3 weights, row stride ld_w bytes
+  const float* h_scale;        // fp8 path: per h-row power-of-two scale of the planes
   int64_t ld_w;
   const float* w_scale;        // fp8 path: per-vocabulary-row scale
   int epilogue;
@@ -174,16 +180,16 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
   const int kr = (lane >> 1) & 15;               // the row this lane reduces
   if constexpr (EPI == EPI_CLOUD) {
     const float b = (vj && p.bias) ? p.bias[id] : 0.f;
-    // fp8 weights entered the MMA as e4m3 * 2^-8 (f16); undo that and
-    // apply the row scale
-    const float ws = (vj && p.w_scale) ? 256.0f * p.w_scale[id] : 1.0f;
+    // fp8 weights: the product of raw e4m3 codes and h's scaled planes,
+    // times the weight row's scale and (below) the h row's scale
+    const float ws = (vj && p.w_scale) ? p.w_scale[id] : 1.0f;
     float m[16];
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const int r = row0 + q;
       m[q] = 0.f;
       if (vj && r < p.R) {
-        const float y = v[q] * ws + b;
+        const float y = (p.h_scale ? v[q] * __ldg(p.h_scale + r) : v[q]) * ws + b;
         const int64_t o = (int64_t)r * p.n + j;
         if (p.partial_out) p.partial_out[o] = y;
         const float yc = fminf(fmaxf(y, -p.clip), p.clip);
@@ -225,11 +231,11 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
 // TM = vocabulary rows per tile: 128, or 256 as two M = 128 MMAs that share
 // each B stage (half the B bytes per A byte; TMEM holds 2 x 2 x BN columns)
 template <int HILO, bool GATHER, int EPI, bool FP8, int TM>
-__global__ void __launch_bounds__(FP8 ? kThreadsFp8 : kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 1)
 tc_kernel(const __grid_constant__ WMaps wm,
           const __grid_constant__ CUtensorMap tmH, const TcParams p) {
   static_assert(TM == 128 || TM == 256, "tile height");
-  static_assert(!FP8 || TM == 128, "fp8 converter warps fill 128-row tiles");
+  constexpr int kAtomE = FP8 ? kAtomE8 : kAtomK;   // elements per 128-byte atom
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* base = smem_raw + (((raw_addr + 1023) & ~1023u) - raw_addr);
@@ -342,7 +348,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     __syncwarp();
   };
   // the first tile's ids load while the CTA sets up
-  if constexpr (GATHER && !FP8) {
+  if constexpr (GATHER) {
     if (warp == 0 && it0 < it1) load_ids((int)(it0 / p.KB), nid);
   }
   uint32_t ncols = 32;                 // two accumulators of kHalves x BN columns
@@ -350,7 +356,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      ptx::mbar_init(&full[s], FP8 ? 2 : 1);     // TMA thread (+ owning converter)
+      ptx::mbar_init(&full[s], 1);               // the TMA thread
       ptx::mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -363,7 +369,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
   }
   if (warp == 0 && lane == 0) {
     // (the subset path's other heights are fetched on first use)
-    if (!FP8) ptx::prefetch_tmap(&wm.m[kBoxHeights - 1]);
+    ptx::prefetch_tmap(&wm.m[kBoxHeights - 1]);
     ptx::prefetch_tmap(&tmH);
   }
   // Only the warps that touch memory written or read by the kernels before
@@ -403,14 +409,9 @@ tc_kernel(const __grid_constant__ WMaps wm,
     // The h planes come from the operand-split kernel, the weights and ids
     // from the caller: the first segment's plan and the A copies of its
     // first stage go out before the wait for that kernel, the stage's B
-    // copies right after it (fp8: the converter warps fill A, so wait up
-    // front).
-    bool waited = FP8;
+    // copies right after it.
+    bool waited = false;
     int rb_first = 0, kb_first = 0;
-    if (FP8) {
-      if (lane == 0) ptx::griddep_wait();
-      __syncwarp();
-    }
     // the B copy of plane l of stage st (k-block kb, row block rb)
     auto issue_b = [&](int st, int kb, int rb, int l) {
       if (l >= 0 && l < HILO)
@@ -428,8 +429,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
     while (!stop && sg.next(tile, kb0, kb1)) {
       const int rb = tile / p.NT, t = tile - rb * p.NT;
       int nbox = 0;
-      uint32_t tx = (uint32_t)(FP8 ? b_bytes : stage_bytes);
-      if constexpr (GATHER && !FP8) {
+      uint32_t tx = (uint32_t)stage_bytes;
+      if constexpr (GATHER) {
         Segments pk = sg;
         int tn = -1, a0, a1;
         if (!pk.next(tn, a0, a1)) tn = -1;
@@ -449,10 +450,9 @@ tc_kernel(const __grid_constant__ WMaps wm,
         // every copy of the stage goes to its own lane, so the copies are
         // issued side by side rather than one after another: A as NA x (row
         // boxes), or over the full vocabulary (when its width allows) one 3-D
-        // copy of all NA atoms (fp8: none; the converter warps fill A); B as
-        // one 3-D copy of all NA atoms per plane
+        // copy of all NA atoms; B as one 3-D copy of all NA atoms per plane
         uint8_t* A = base + (size_t)stage * stage_bytes;
-        const int nA = FP8 ? 0 : (GATHER ? NA * nbox : (p.a3d ? 1 : NA * kHalves));
+        const int nA = GATHER ? NA * nbox : (p.a3d ? 1 : NA * kHalves);
         if (!waited && issued == 0) { rb_first = rb; kb_first = kb; }
         for (int op = lane; op < nA + (waited ? HILO : 0); op += 32) {
           if (op < nA) {
@@ -460,13 +460,13 @@ tc_kernel(const __grid_constant__ WMaps wm,
               const int a = op / nbox;
               const int2 bx = s_box[op - a * nbox];
               ptx::tma_load_2d(A + a * atom_bytes + (bx.y & 0xFF) * 128, &wm.m[bx.y >> 8],
-                               (kb * NA + a) * kAtomK, bx.x, &full[stage]);
+                               (kb * NA + a) * kAtomE, bx.x, &full[stage]);
             } else if (p.a3d) {
               ptx::tma_load_3d(A, &wm.a3, 0, t * TM, kb * NA, &full[stage]);
             } else {
               const int a = op / kHalves, hf = op - a * kHalves;
               ptx::tma_load_2d(A + a * atom_bytes + hf * kAtomBytes, &wm.m[kBoxHeights - 1],
-                               (kb * NA + a) * kAtomK, t * TM + hf * 128, &full[stage]);
+                               (kb * NA + a) * kAtomE, t * TM + hf * 128, &full[stage]);
             }
           } else {
             issue_b(stage, kb, rb, op - nA);
@@ -495,7 +495,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
       uint32_t tph[2] = {0, 0};
       int si = 0, tile, kb0, kb1;
       const uint32_t idesc =
-          FP8 ? ptx::idesc_f16_f32(kTileM, BN) : ptx::idesc_bf16_f32(kTileM, BN);
+          FP8 ? ptx::idesc_e4m3_f32(kTileM, BN) : ptx::idesc_bf16_f32(kTileM, BN);
       // accumulator `acc`, tile half hf: TMEM columns (acc * kHalves + hf) * BN
       bool stop = false;
       while (!stop && sg.next(tile, kb0, kb1)) {
@@ -523,10 +523,17 @@ tc_kernel(const __grid_constant__ WMaps wm,
               for (int kk = 0; kk < kAtomK / 16; ++kk) {
 #pragma unroll
                 for (int hf = 0; hf < kHalves; ++hf)
-                  ptx::umma_f16(d + (uint32_t)(hf * BN),
-                                ptx::sdesc_k128(a0 + at * atom_bytes + hf * kAtomBytes + kk * 32),
-                                ptx::sdesc_k128(b0 + (h * NA + at) * BN * 128 + kk * 32), idesc,
-                                (kb != kb0 || at != 0 || h != 0 || kk != 0) ? 1u : 0u);
+                {
+                  // 32 bytes of K per MMA: 16 bf16 or 32 e4m3 elements
+                  const uint64_t ad =
+                      ptx::sdesc_k128(a0 + at * atom_bytes + hf * kAtomBytes + kk * 32);
+                  const uint64_t bd = ptx::sdesc_k128(b0 + (h * NA + at) * BN * 128 + kk * 32);
+                  const uint32_t accum = (kb != kb0 || at != 0 || h != 0 || kk != 0) ? 1u : 0u;
+                  if constexpr (FP8)
+                    ptx::umma_f8(d + (uint32_t)(hf * BN), ad, bd, idesc, accum);
+                  else
+                    ptx::umma_f16(d + (uint32_t)(hf * BN), ad, bd, idesc, accum);
+                }
               }
             }
           }
@@ -744,86 +751,6 @@ tc_kernel(const __grid_constant__ WMaps wm,
       }
       ++si;
     }
-  } else if constexpr (FP8) {
-    // -------------------------------------------- converter warps (fp8 A)
-    // Stages go round-robin to the four converter warps; the ring has four
-    // or eight stages, so every slot has one owning warp.  A warp loads the
-    // 128 rows x 64 e4m3 bytes of its stage with 16-byte loads (four lanes
-    // per row), rewrites every byte as the f16 with the same sign and the
-    // magnitude bits shifted up by 7 -- exactly the e4m3 value times 2^-8,
-    // subnormals included -- stores the 128-byte-swizzled f16 rows, fences
-    // the async proxy and arrives on the stage barrier.
-    const int gw = warp - (2 + kEpiWarps);
-    const int c = lane & 3;                      // 16-byte chunk of a 64-byte row slice
-    const int r0 = lane >> 2;                    // rows r0 + 8m, m = 0..15
-    ptx::griddep_wait();                         // (inputs only; keeps ordering simple)
-    Segments sg{it0, it1, p.KB};
-    long long k = 0;
-    int tile, kb0, kb1;
-    bool stop = false;
-    while (!stop && sg.next(tile, kb0, kb1)) {
-      const int t = tile % p.NT;
-      int rid[16];
-#pragma unroll
-      for (int m = 0; m < 16; ++m) {
-        const int jj = min(t * kTileM + r0 + 8 * m, p.n - 1);
-        rid[m] = GATHER ? p.ids[jj] : jj;
-      }
-      for (int kb = kb0; kb < kb1; ++kb, ++k) {
-        if ((int)(k & 3) != gw) continue;
-        const int stage = (int)(k % S);
-        const uint32_t phase = (uint32_t)((k / S) & 1);
-        int ok = 1;
-        if (lane == 0) ok = !*s_abort && ptx::mbar_wait(&empty[stage], phase ^ 1, limit);
-        ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
-        if (!ok) {
-          if (lane == 0 && !*s_abort) give_up();
-          stop = true;
-          break;
-        }
-        const int e0 = kb * kAtomK + c * 16;     // first byte (= element) of my chunk
-        const int left = p.K - e0;               // valid bytes in it
-        uint4 raw[16];
-#pragma unroll
-        for (int m = 0; m < 16; ++m) {
-          raw[m] = make_uint4(0, 0, 0, 0);
-          if (left > 0)
-            raw[m] = __ldg(reinterpret_cast<const uint4*>(p.W8 + (int64_t)rid[m] * p.ld_w + e0));
-        }
-        if (left > 0 && left < 16) {             // zero the bytes past K
-#pragma unroll
-          for (int m = 0; m < 16; ++m) {
-            uint32_t w4[4] = {raw[m].x, raw[m].y, raw[m].z, raw[m].w};
-#pragma unroll
-            for (int b = 0; b < 16; ++b)
-              if (b >= left) w4[b >> 2] &= ~(0xFFu << (8 * (b & 3)));
-            raw[m] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
-          }
-        }
-        uint8_t* A = base + (size_t)stage * stage_bytes;
-#pragma unroll
-        for (int m = 0; m < 16; ++m) {
-          const int row = r0 + 8 * m;
-          const uint32_t w4[4] = {raw[m].x, raw[m].y, raw[m].z, raw[m].w};
-          uint32_t h[8];                         // 16 f16 values
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const uint32_t lo = __byte_perm(w4[q], 0u, 0x4140);   // bytes 0,1 -> halves
-            const uint32_t hi = __byte_perm(w4[q], 0u, 0x4342);   // bytes 2,3 -> halves
-            h[2 * q] = ((lo & 0x00800080u) << 8) | ((lo & 0x007F007Fu) << 7);
-            h[2 * q + 1] = ((hi & 0x00800080u) << 8) | ((hi & 0x007F007Fu) << 7);
-          }
-          const int c0 = 2 * c, c1 = 2 * c + 1;  // 16-byte f16 chunks of the row
-          *reinterpret_cast<uint4*>(A + row * 128 + ((c0 ^ (row & 7)) << 4)) =
-              make_uint4(h[0], h[1], h[2], h[3]);
-          *reinterpret_cast<uint4*>(A + row * 128 + ((c1 ^ (row & 7)) << 4)) =
-              make_uint4(h[4], h[5], h[6], h[7]);
-        }
-        ptx::fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(&full[stage]);
-      }
-    }
   }
 
   ptx::tc_fence_before();
@@ -836,53 +763,33 @@ tc_kernel(const __grid_constant__ WMaps wm,
 // operand preparation: fp32 h -> bf16 hi (and lo) planes, zero padded
 // ---------------------------------------------------------------------------
 // ... and clear the split-tile counters and (cloud) the row maxima.
-// (planes of f16 instead of bf16 when f16 != 0: the fp8-weight path, where
-// bf16-activation mode first rounds h to bf16 and then splits that value)
 // One thread converts 8 consecutive columns of one row (Kp is a multiple of
 // 64, so a group never crosses a row) and stores 16 bytes per plane.  Small
 // 128-thread blocks with at most 32 registers fit beside a tensor-core CTA
 // on the same SM, so that kernel starts (and issues its first weight copies)
 // while this one runs.
-template <typename T>
-__device__ __forceinline__ uint32_t pack2(float a, float b);
-template <>
-__device__ __forceinline__ uint32_t pack2<__nv_bfloat16>(float a, float b) {
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<const uint32_t*>(&v);
 }
-template <>
-__device__ __forceinline__ uint32_t pack2<__half>(float a, float b) {
-  const __half2 v = __floats2half2_rn(a, b);
-  return *reinterpret_cast<const uint32_t*>(&v);
-}
-template <typename T>
-__device__ __forceinline__ float round_to(float x);
-template <>
-__device__ __forceinline__ float round_to<__nv_bfloat16>(float x) {
-  return __bfloat162float(__float2bfloat16_rn(x));
-}
-template <>
-__device__ __forceinline__ float round_to<__half>(float x) {
-  return __half2float(__float2half_rn(x));
-}
 
-template <typename T>
+// hi = bf16(x), lo = bf16(x - hi) of 8 values
 __device__ __forceinline__ void split_group(const float (&x)[8], int hilo, uint4* hi, uint4* lo) {
   float r[8];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) r[i] = round_to<T>(x[i]);
-  *hi = make_uint4(pack2<T>(r[0], r[1]), pack2<T>(r[2], r[3]), pack2<T>(r[4], r[5]),
-                   pack2<T>(r[6], r[7]));
+  for (int i = 0; i < 8; ++i) r[i] = __bfloat162float(__float2bfloat16_rn(x[i]));
+  *hi = make_uint4(pack_bf16x2(r[0], r[1]), pack_bf16x2(r[2], r[3]), pack_bf16x2(r[4], r[5]),
+                   pack_bf16x2(r[6], r[7]));
   if (hilo == 2)
-    *lo = make_uint4(pack2<T>(x[0] - r[0], x[1] - r[1]), pack2<T>(x[2] - r[2], x[3] - r[3]),
-                     pack2<T>(x[4] - r[4], x[5] - r[5]), pack2<T>(x[6] - r[6], x[7] - r[7]));
+    *lo = make_uint4(pack_bf16x2(x[0] - r[0], x[1] - r[1]), pack_bf16x2(x[2] - r[2], x[3] - r[3]),
+                     pack_bf16x2(x[4] - r[4], x[5] - r[5]), pack_bf16x2(x[6] - r[6], x[7] - r[7]));
 }
 
 constexpr int kSplitThreads = 128;
 __global__ void __launch_bounds__(kSplitThreads, 16)
 split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R, int K, int Rp, int Kp,
                int hilo, __nv_bfloat16* __restrict__ Hs, int* __restrict__ counters,
-               int ncounters, unsigned* __restrict__ rowmax, int f16, int act_bf16) {
+               int ncounters, unsigned* __restrict__ rowmax) {
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   const int tid = blockIdx.x * blockDim.x + threadIdx.x;
@@ -908,19 +815,66 @@ split_h_kernel(const float* __restrict__ h, int64_t ld_h, int R, int K, int Rp, 
       for (int i = 0; i < 8; ++i) x[i] = (r < R && c0 + i < K) ? __ldg(src + i) : 0.f;
     }
     uint4 hi, lo;
-    if (f16) {
-      // fp8 weights: f16 planes of h, or of h rounded to bf16 first
-      if (act_bf16) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) x[i] = round_to<__nv_bfloat16>(x[i]);
-      }
-      split_group<__half>(x, hilo, &hi, &lo);
-    } else {
-      split_group<__nv_bfloat16>(x, hilo, &hi, &lo);
-    }
+    split_group(x, hilo, &hi, &lo);
     uint4* dst = reinterpret_cast<uint4*>(Hs + g * 8);
     dst[0] = hi;
     if (hilo == 2) *reinterpret_cast<uint4*>(Hs + total + g * 8) = lo;
+  }
+}
+
+
+// fp8 weights: h -> e4m3 planes under a per-row power-of-two scale.  One
+// block per padded row: the row's max |h| fixes the scale 2^e with
+// max |h| / 2^e in [128, 256) (e4m3 holds up to 448).  Plane q is the e4m3
+// rounding (to nearest) of what planes 0..q-1 left of h / 2^e, so h equals
+// 2^e times the sum of the planes up to the last one's rounding: 4 planes
+// leave 2^-13 |h| (or 2^-10 2^e where the planes reach e4m3's subnormal
+// range); 2 planes reproduce bf16-rounded h, whose 8 significant bits are
+// two 4-bit halves.  Also clears the split-tile counters and row maxima.
+constexpr int kSplit8Threads = 256;
+__global__ void __launch_bounds__(kSplit8Threads)
+split_h_e4m3_kernel(const float* __restrict__ h, int64_t ld_h, int R, int K, int Rp, int Kp,
+                    int planes, uint8_t* __restrict__ Hs, float* __restrict__ h_scale,
+                    int* __restrict__ counters, int ncounters, unsigned* __restrict__ rowmax,
+                    int act_bf16) {
+  __shared__ float s_max[kSplit8Threads / 32];
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int nth = gridDim.x * blockDim.x;
+  if (rowmax)
+    for (int i = tid; i < R; i += nth) rowmax[i] = 0u;
+  for (int i = tid; i < ncounters; i += nth) counters[i] = 0;
+  const int r = blockIdx.x;
+  const float* hr = h + (int64_t)r * ld_h;
+  auto value = [&](int c) {
+    float x = (r < R && c < K) ? __ldg(hr + c) : 0.f;
+    if (act_bf16) x = __bfloat162float(__float2bfloat16_rn(x));
+    return x;
+  };
+  float m = 0.f;
+  for (int c = threadIdx.x; c < K; c += blockDim.x) m = fmaxf(m, fabsf(value(c)));
+#pragma unroll
+  for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+  if ((threadIdx.x & 31) == 0) s_max[threadIdx.x >> 5] = m;
+  __syncthreads();
+  m = 0.f;
+#pragma unroll
+  for (int w = 0; w < kSplit8Threads / 32; ++w) m = fmaxf(m, s_max[w]);
+  // 2^e with m / 2^e in [128, 256): the exponent field of m less 7
+  const int eb = (int)((__float_as_uint(m) >> 23) & 0xFF);
+  const float scale = eb > 7 ? __uint_as_float((uint32_t)(eb - 7) << 23) : 1.0f;
+  const float inv = eb > 7 && eb - 7 < 254 ? __uint_as_float((uint32_t)(254 - (eb - 7)) << 23)
+                                           : 1.0f;
+  if (threadIdx.x == 0) h_scale[r] = scale;
+  const int64_t plane = (int64_t)Rp * Kp;
+  for (int c = threadIdx.x; c < Kp; c += blockDim.x) {
+    float x = value(c) * inv;            // exact: a power of two
+    for (int q = 0; q < planes; ++q) {
+      const __nv_fp8_e4m3 e(x);          // round to nearest, saturating
+      Hs[q * plane + (int64_t)r * Kp + c] = e.__x;
+      x -= static_cast<float>(e);
+    }
   }
 }
 
@@ -963,18 +917,19 @@ bool make_map(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// 3-D view (element, row, 64-element atom) of a row-major [rows, cols]
-// matrix: strides row_bytes and 128 bytes; a box of (64, box_rows,
-// box_atoms) lands as box_atoms consecutive 128-byte-swizzled atom tiles
-// of box_rows rows.  cols must be a multiple of 64 (the view cannot mark
-// the end of a row).
+// 3-D view (element, row, atom) of a row-major [rows, cols] matrix, an atom
+// being the `atom` elements of 128 bytes (64 bf16, 128 e4m3): strides
+// row_bytes and 128 bytes; a box of (atom, box_rows, box_atoms) lands as
+// box_atoms consecutive 128-byte-swizzled atom tiles of box_rows rows.  cols
+// must be a multiple of atom (the view cannot mark the end of a row).
 bool make_map3(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64_t cols,
-               uint64_t rows, uint64_t row_bytes, uint32_t box_rows, uint32_t box_atoms) {
+               uint64_t rows, uint64_t row_bytes, uint32_t box_rows, uint32_t box_atoms,
+               int atom) {
   EncodeFn fn = encode_fn();
   if (!fn) return false;
-  const cuuint64_t dims[3] = {(cuuint64_t)kAtomK, rows, cols / kAtomK};
+  const cuuint64_t dims[3] = {(cuuint64_t)atom, rows, cols / atom};
   const cuuint64_t strides[2] = {row_bytes, 128};
-  const cuuint32_t box[3] = {(cuuint32_t)kAtomK, box_rows, box_atoms};
+  const cuuint32_t box[3] = {(cuuint32_t)atom, box_rows, box_atoms};
   const cuuint32_t es[3] = {1, 1, 1};
   return fn(m, dt, 3, const_cast<void*>(ptr), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -992,9 +947,11 @@ struct Map3Key {
   const void* ptr;
   uint64_t cols, rows, row_bytes;
   uint32_t box_rows, box_atoms;
+  int atom;
   bool operator==(const Map3Key& o) const {
     return dt == o.dt && ptr == o.ptr && cols == o.cols && rows == o.rows &&
-           row_bytes == o.row_bytes && box_rows == o.box_rows && box_atoms == o.box_atoms;
+           row_bytes == o.row_bytes && box_rows == o.box_rows && box_atoms == o.box_atoms &&
+           atom == o.atom;
   }
 };
 struct Map3Entry {
@@ -1008,8 +965,9 @@ Map3Entry g_map3[16];
 unsigned long long g_map3_tick = 0;
 
 bool cached_map3(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64_t cols,
-                 uint64_t rows, uint64_t row_bytes, uint32_t box_rows, uint32_t box_atoms) {
-  const Map3Key key{(int)dt, ptr, cols, rows, row_bytes, box_rows, box_atoms};
+                 uint64_t rows, uint64_t row_bytes, uint32_t box_rows, uint32_t box_atoms,
+                 int atom) {
+  const Map3Key key{(int)dt, ptr, cols, rows, row_bytes, box_rows, box_atoms, atom};
   std::lock_guard<std::mutex> lock(g_map3_mu);
   Map3Entry* lru = &g_map3[0];
   for (Map3Entry& e : g_map3) {
@@ -1020,7 +978,7 @@ bool cached_map3(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64
     }
     if (!e.valid || e.used < lru->used) lru = &e;
   }
-  if (!make_map3(&lru->map, dt, ptr, cols, rows, row_bytes, box_rows, box_atoms)) {
+  if (!make_map3(&lru->map, dt, ptr, cols, rows, row_bytes, box_rows, box_atoms, atom)) {
     lru->valid = false;
     return false;
   }
@@ -1031,13 +989,15 @@ bool cached_map3(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64
   return true;
 }
 
-// W tensor maps, encoded once per weight tensor: map i copies boxes of 64
-// columns x (i + 1) rows of W [V rows, K columns], row stride ld_w (the
-// full-vocabulary path uses only the 128-row map).  A few recently used
+// W tensor maps, encoded once per weight tensor: map i copies boxes of one
+// 128-byte atom (64 bf16 or 128 e4m3 columns) x (i + 1) rows of W [V rows,
+// K columns], row stride ld_w (the full-vocabulary path uses only the
+// 128-row map).  A few recently used
 // sets are kept, since encoding 128 maps costs far more than a launch.
 struct MapSet {
   const void* W = nullptr;
   int64_t V = 0, K = 0, ld = 0;
+  int w_dtype = 0;
   bool gather = false;
   unsigned long long used = 0;
   WMaps maps;
@@ -1051,7 +1011,9 @@ bool w_maps(const GatherGemm& g, bool gather, WMaps& out) {
   MapSet* hit = nullptr;
   MapSet* lru = &g_map_sets[0];
   for (MapSet& m : g_map_sets) {
-    if (m.W == g.W && m.V == g.V && m.K == g.K && m.ld == g.ld_w && m.gather == gather) hit = &m;
+    if (m.W == g.W && m.V == g.V && m.K == g.K && m.ld == g.ld_w && m.gather == gather &&
+        m.w_dtype == g.w_dtype)
+      hit = &m;
     if (m.used < lru->used) lru = &m;
   }
   if (!hit) {
@@ -1062,11 +1024,15 @@ bool w_maps(const GatherGemm& g, bool gather, WMaps& out) {
         hit->maps.m[i] = CUtensorMap{};
         continue;
       }
-      if (!make_map(&hit->maps.m[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
-                    (uint64_t)g.V, (uint64_t)g.ld_w * 2, kAtomK, (uint32_t)(i + 1)))
+      const bool e4m3 = g.w_dtype == W_FP8;
+      if (!make_map(&hit->maps.m[i],
+                    e4m3 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W,
+                    (uint64_t)g.K, (uint64_t)g.V, (uint64_t)g.ld_w * (e4m3 ? 1 : 2),
+                    e4m3 ? kAtomE8 : kAtomK, (uint32_t)(i + 1)))
         return false;
     }
     hit->W = g.W; hit->V = g.V; hit->K = g.K; hit->ld = g.ld_w; hit->gather = gather;
+    hit->w_dtype = g.w_dtype;
   }
   hit->used = ++g_map_tick;
   out = hit->maps;
@@ -1079,11 +1045,17 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
                int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn_opt,
                int tile_m) {
   TcPlan pl{};
-  // one bf16 plane carries bf16-rounded activations exactly; f16 planes
-  // (fp8 weights) always take two
-  pl.hilo = (act_bf16 && !fp8) ? 1 : 2;
+  // h planes: bf16 weights take one bf16 plane for bf16-rounded
+  // activations (exact) and two (hi + lo) for fp32; e4m3 weights take two
+  // e4m3 planes for bf16-rounded activations (exact) and four for fp32
+  pl.hilo = fp8 ? (act_bf16 ? 2 : 4) : (act_bf16 ? 1 : 2);
   pl.fp8 = fp8;
-  int max_bn = fp8 ? kMaxBNFp8 : kMaxBN;
+  const int atom = fp8 ? kAtomE8 : kAtomK;   // elements per 128-byte atom
+  // e4m3: row blocks of up to 128 rows (measured on 256 rows x 152064 ids
+  // x 7168, 256-id tiles: four planes 1229 / 996 / 743 us and two planes
+  // 784 / 661 / 474 us at 64 / 96 / 128 rows -- fewer weight re-reads beat
+  // deeper pipelines; 128-row blocks leave two 96 KB stages)
+  int max_bn = fp8 ? 128 : kMaxBN;
   // two h planes: at most 224 rows, so that three stages fit (measured:
   // 1024 rows x 256k ids x 4608 runs 21 % faster in three 224-row stages
   // than in two 256-row ones)
@@ -1110,7 +1082,7 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   // 160..208-row blocks slower).
   const bool tm256_auto = tile_m == 0 && pl.BN <= 128 && K >= 2048 &&
                           4ll * pl.RB * ((n + 255) / 256) >= 3ll * sm_count;
-  pl.tm = (!fp8 && (tile_m == 256 || tm256_auto)) ? 256 : 128;
+  pl.tm = (tile_m == 256 || tm256_auto) ? 256 : 128;
   const int halves = pl.tm / 128;
   if (pl.tm == 256 && pl.BN > 128) row_blocks(max_bn < 128 ? max_bn : 128);
   pl.Rp = pl.RB * pl.BN;
@@ -1122,7 +1094,7 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
          (int)((kSmemBudget - 2048) / (pl.na * (halves * kAtomBytes + pl.hilo * pl.BN * 128))) <
              min_stages)
     pl.na >>= 1;
-  const int bk = pl.na * kAtomK;
+  const int bk = pl.na * atom;
   pl.KB = (K + bk - 1) / bk;
   pl.Kp = pl.KB * bk;
   pl.NT = (n + pl.tm - 1) / pl.tm;
@@ -1138,10 +1110,9 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.stages = (int)((kSmemBudget - 2048) / stage_bytes);
   if (pl.stages > kMaxStages) pl.stages = kMaxStages;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
-  // fp8: four converter warps own the ring slots round-robin, so the ring
-  // has four or eight stages
-  if (fp8) pl.stages = pl.stages >= 8 ? 8 : (pl.stages >= 4 ? 4 : 0);
-  pl.hs_bytes = align256((size_t)pl.hilo * pl.Rp * pl.Kp * 2);
+  // h planes (bf16 or e4m3), and with e4m3 the per-row scales after them
+  pl.hs_bytes = fp8 ? align256((size_t)pl.hilo * pl.Rp * pl.Kp) + align256((size_t)pl.Rp * 4)
+                    : align256((size_t)pl.hilo * pl.Rp * pl.Kp * 2);
   // split tiles exist only when a CTA's range does not cover whole tiles
   const bool splits = !pl.whole_tiles && (pl.T % pl.G != 0 || (pl.T / pl.G) % pl.KB != 0);
   pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * pl.tm * 4) : 0;
@@ -1156,7 +1127,7 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.epi_stats = endpoint && (pl.BN < 128 || 4 * pl.BN <= K);
   pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
   pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256 + kMaxBoxes * sizeof(int2);
-  pl.ok = fp8 ? pl.stages >= 4 : pl.stages >= 2;
+  pl.ok = pl.stages >= 2;
   return pl;
 }
 
@@ -1182,7 +1153,7 @@ static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
       }
     }
   }
-  return launch_pdl(kern, dim3(pl.G), dim3(FP8 ? kThreadsFp8 : kThreads), pl.smem_bytes, st,
+  return launch_pdl(kern, dim3(pl.G), dim3(kThreads), pl.smem_bytes, st,
                     mw, mh, prm);
 }
 
@@ -1201,32 +1172,44 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   const bool gather = g.ids != nullptr;
   const int tiles = pl.RB * pl.NT;
 
-  {
+  // e4m3 planes of h (1 byte per element) and, after them, the rows' scales
+  float* h_scale = fp8 ? reinterpret_cast<float*>(
+                             sc + align256((size_t)pl.hilo * pl.Rp * pl.Kp))
+                       : nullptr;
+  if (fp8) {
+    cudaError_t e = launch_pdl(split_h_e4m3_kernel, dim3(pl.Rp), dim3(kSplit8Threads), 0, st,
+                               g.h, g.ld_h, g.rows, g.K, pl.Rp, pl.Kp, pl.hilo,
+                               reinterpret_cast<uint8_t*>(sc), h_scale, counters,
+                               tiles * 4 * kEpiGroups, g.rowmax, g.act_bf16);
+    if (e != cudaSuccess) return e;
+  } else {
     const int64_t groups = (int64_t)pl.Rp * pl.Kp / 8;
     int blocks = (int)((groups + kSplitThreads - 1) / kSplitThreads);
     if (blocks > 4096) blocks = 4096;
     if (blocks < 1) blocks = 1;
     cudaError_t e = launch_pdl(split_h_kernel, dim3(blocks), dim3(kSplitThreads), 0, st, g.h, g.ld_h,
                                g.rows, g.K, pl.Rp, pl.Kp, pl.hilo, Hs, counters, tiles * 4 * kEpiGroups,
-                               g.epilogue == EPI_CLOUD ? g.rowmax : (unsigned*)nullptr,
-                               fp8 ? 1 : 0, g.act_bf16);
+                               g.epilogue == EPI_CLOUD ? g.rowmax : (unsigned*)nullptr);
     if (e != cudaSuccess) return e;
   }
 
   WMaps mw;
   alignas(64) CUtensorMap mh;
-  if (!fp8 && !w_maps(g, gather, mw)) return cudaErrorInvalidValue;
+  if (!w_maps(g, gather, mw)) return cudaErrorInvalidValue;
+  const CUtensorMapDataType dt =
+      fp8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  const int atom = fp8 ? kAtomE8 : kAtomK;
+  const int esz = fp8 ? 1 : 2;
   // h planes [hilo * Rp rows, Kp columns], zero padded: all atoms of a
   // stage in one copy per plane
-  if (!cached_map3(&mh, fp8 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
-                 Hs, (uint64_t)pl.Kp, (uint64_t)pl.hilo * pl.Rp, (uint64_t)pl.Kp * 2,
-                 (uint32_t)pl.BN, (uint32_t)pl.na))
+  if (!cached_map3(&mh, dt, sc, (uint64_t)pl.Kp, (uint64_t)pl.hilo * pl.Rp,
+                   (uint64_t)pl.Kp * esz, (uint32_t)pl.BN, (uint32_t)pl.na, atom))
     return cudaErrorInvalidValue;
-  // full vocabulary with a width that is a multiple of 64: A likewise
-  const int a3d = (!fp8 && !gather && g.K % kAtomK == 0 && g.K >= pl.na * kAtomK) ? 1 : 0;
+  // full vocabulary with a width that is a multiple of the atom: A likewise
+  const int a3d = (!gather && g.K % atom == 0 && g.K >= pl.na * atom) ? 1 : 0;
   mw.a3 = CUtensorMap{};
-  if (a3d && !cached_map3(&mw.a3, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.W, (uint64_t)g.K,
-                        (uint64_t)g.V, (uint64_t)g.ld_w * 2, (uint32_t)pl.tm, (uint32_t)pl.na))
+  if (a3d && !cached_map3(&mw.a3, dt, g.W, (uint64_t)g.K, (uint64_t)g.V,
+                          (uint64_t)g.ld_w * esz, (uint32_t)pl.tm, (uint32_t)pl.na, atom))
     return cudaErrorInvalidValue;
 
   TcParams prm{};
@@ -1234,7 +1217,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.RB = pl.RB; prm.BN = pl.BN; prm.Rp = pl.Rp; prm.stages = pl.stages;
   prm.whole_tiles = pl.whole_tiles; prm.T = pl.T; prm.na = pl.na; prm.nseg = pl.nseg;
   prm.ids = g.ids;
-  prm.W8 = fp8 ? static_cast<const uint8_t*>(g.W) : nullptr;
+  prm.h_scale = h_scale;
   prm.ld_w = g.ld_w;
   prm.w_scale = fp8 ? g.w_scale : nullptr;
   prm.epilogue = g.epilogue; prm.bias = g.bias;
@@ -1246,7 +1229,12 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
 
   const bool hilo2 = pl.hilo == 2;
   if (pl.tm == 256) {
-    if (fp8) return cudaErrorNotSupported;
+    if (fp8) {
+      if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, true, 256>(mw, mh, prm, pl, st)
+                               : launch_inst<4, true, EPI_CLOUD, true, 256>(mw, mh, prm, pl, st);
+      return hilo2 ? launch_inst<2, false, EPI_CLOUD, true, 256>(mw, mh, prm, pl, st)
+                   : launch_inst<4, false, EPI_CLOUD, true, 256>(mw, mh, prm, pl, st);
+    }
     if (g.epilogue == EPI_CLOUD) {
       if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, false, 256>(mw, mh, prm, pl, st)
                                : launch_inst<1, true, EPI_CLOUD, false, 256>(mw, mh, prm, pl, st);
@@ -1258,11 +1246,11 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
     return hilo2 ? launch_inst<2, false, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st)
                  : launch_inst<1, false, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st);
   }
-  if (fp8) {
+  if (fp8) {                // four e4m3 planes of h, or two for bf16-rounded h
     if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, true>(mw, mh, prm, pl, st)
-                             : launch_inst<1, true, EPI_CLOUD, true>(mw, mh, prm, pl, st);
+                             : launch_inst<4, true, EPI_CLOUD, true>(mw, mh, prm, pl, st);
     return hilo2 ? launch_inst<2, false, EPI_CLOUD, true>(mw, mh, prm, pl, st)
-                 : launch_inst<1, false, EPI_CLOUD, true>(mw, mh, prm, pl, st);
+                 : launch_inst<4, false, EPI_CLOUD, true>(mw, mh, prm, pl, st);
   }
   if (g.epilogue == EPI_CLOUD) {
     if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD>(mw, mh, prm, pl, st)

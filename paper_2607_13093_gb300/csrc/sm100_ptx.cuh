@@ -135,6 +135,20 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
 __host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
   return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
+// Instruction descriptor for kind::f8f6f4 with e4m3 A/B (format code 0 in
+// both operand fields), fp32 D, K-major A/B.
+__host__ __device__ constexpr uint32_t idesc_e4m3_f32(int M, int N) {
+  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+// tcgen05.mma kind::f8f6f4 (8-bit operands; 32 elements of K per MMA)
+__device__ __forceinline__ void umma_f8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                        uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 // tcgen05.mma kind::f16 (the operand types come from the instruction
 // descriptor: bf16 x bf16 or f16 x f16)
 __device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc,

@@ -463,6 +463,24 @@ def test_fp8_tensor_core(ctx, rows, keep, act):
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
 
 
+@pytest.mark.parametrize("tile_m", [128, 256])
+@pytest.mark.parametrize("act", ["fp32", "bf16"])
+def test_fp8_tile_heights(ctx, tile_m, act):
+    """e4m3 weights with both tile heights, gathered and full vocabulary,
+    K = 2048 (16 e4m3 atoms), ragged vocabulary tails."""
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    ctx.set_option(sph.SPH_OPT_TC_TILE_M, tile_m)
+    try:
+        for keep in (2900, 3000):
+            w = small(V=3000, d=2304, d_l=256, rows=150, n_keep=keep, w_dtype="fp8",
+                      clip=40.0, seed=808 + keep)
+            check_cloud(ctx, w, act_mode=act)
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+        ctx.set_option(sph.SPH_OPT_TC_TILE_M, 0)
+
+
 # ---------------------------------------------------------------------------
 # CUDA-graph capture (as the benchmark times the step) = direct calls
 # ---------------------------------------------------------------------------
