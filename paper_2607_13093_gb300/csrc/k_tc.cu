@@ -104,6 +104,7 @@ struct TcParams {
   float inv_tau;
   float2* seg_stats;           // endpoint: [R][nseg] (max, sum exp)
   int a3d;                     // full vocabulary: A by one 3-D copy per stage
+  int single_acc;              // one accumulator (no epilogue overlap): 256-id tiles of > 128 rows
   float* P;                    // split-tile partials [2 * grid][BN][TM]
   int* counters;               // [tiles][4 quadrants][epilogue groups], zero between calls
   unsigned* status;
@@ -352,7 +353,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     if (warp == 0 && it0 < it1) load_ids((int)(it0 / p.KB), nid);
   }
   uint32_t ncols = 32;                 // two accumulators of kHalves x BN columns
-  while (ncols < (uint32_t)(2 * kHalves * BN)) ncols <<= 1;
+  while (ncols < (uint32_t)((p.single_acc ? 1 : 2) * kHalves * BN)) ncols <<= 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -499,7 +500,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
       // accumulator `acc`, tile half hf: TMEM columns (acc * kHalves + hf) * BN
       bool stop = false;
       while (!stop && sg.next(tile, kb0, kb1)) {
-        const int acc = si & 1;
+        const int acc = p.single_acc ? 0 : (si & 1);
         if (*s_abort || !ptx::mbar_wait(&tempty[acc], tph[acc] ^ 1, limit)) {
           if (!*s_abort) give_up();
           break;
@@ -561,7 +562,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     uint32_t fph[2] = {0, 0};
     int si = 0, tile, kb0, kb1;
     while (sg.next(tile, kb0, kb1)) {
-      const int acc = si & 1;
+      const int acc = p.single_acc ? 0 : (si & 1);
       const int rb = tile / p.NT, t = tile - rb * p.NT;
       const bool whole = kb0 == 0 && kb1 == p.KB;
       // this lane's vocabulary row in each half: i = hf * 128 + quad * 32 + lane
@@ -1080,11 +1081,23 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   // ids, K 2048..8192: 4..44 % faster; decode's 47 tiles on 152 SMs, every
   // one split three or four ways, 10 % slower; the endpoint's short K and
   // 160..208-row blocks slower).
-  const bool tm256_auto = tile_m == 0 && pl.BN <= 128 && K >= 2048 &&
+  // Row blocks of 129..192 rows also take 256-id tiles, with one
+  // accumulator (three stages still fit; measured on 320 rows x 51302 ids x
+  // 3584: 245 -> 227 us fp32 h, 233 -> 200 us bf16 h; 208-row blocks of
+  // R = 1024 with two stages are slower).
+  const bool wide_auto = !fp8 && pl.BN > 128 && pl.BN <= 192;
+  const bool tm256_auto = tile_m == 0 && (pl.BN <= 128 || wide_auto) && K >= 2048 &&
                           4ll * pl.RB * ((n + 255) / 256) >= 3ll * sm_count;
   pl.tm = (tile_m == 256 || tm256_auto) ? 256 : 128;
   const int halves = pl.tm / 128;
-  if (pl.tm == 256 && pl.BN > 128) row_blocks(max_bn < 128 ? max_bn : 128);
+  // 256-id tiles: row blocks of <= 128 rows keep two accumulators; asked
+  // for with larger blocks (max_bn above 128), one accumulator holds up to
+  // 256 rows and the epilogue no longer overlaps the next tile's MMAs
+  pl.single_acc = 0;
+  if (pl.tm == 256 && pl.BN > 128) {
+    if ((tile_m == 256 && max_bn_opt > 128) || (tile_m == 0 && wide_auto)) pl.single_acc = 1;
+    else row_blocks(max_bn < 128 ? max_bn : 128);
+  }
   pl.Rp = pl.RB * pl.BN;
   // k-block width: as asked (automatic: 128), narrowed until the shared
   // memory holds at least min_stages pipeline stages
@@ -1223,6 +1236,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.epilogue = g.epilogue; prm.bias = g.bias;
   prm.clip = g.clip; prm.partial_out = g.partial_out; prm.Y = g.Y;
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
+  prm.single_acc = pl.single_acc;
   prm.inv_tau = g.inv_tau; prm.seg_stats = (pl.epi_stats && !g.no_stats) ? stats : nullptr; prm.a3d = a3d;
   prm.P = P; prm.counters = counters;
   prm.status = g.status; prm.spin_limit = spin_limit; prm.finish_wait = g.finish_wait;

@@ -109,16 +109,21 @@ sph_status ensure_scratch(sph_ctx* ctx, size_t bytes) {
   return SPH_OK;
 }
 
-// Bump allocator over the arena for one call.
+// Bump allocator over the arena for one call.  fits() says whether every
+// piece taken so far lies inside the arena; calls check it before their
+// first launch, so that a scratch plan that outgrew the arena is an error,
+// never an out-of-bounds write.
 struct Carve {
   char* base;
+  size_t cap;
   size_t off = 0;
-  explicit Carve(void* b) : base(static_cast<char*>(b)) {}
+  Carve(void* b, size_t c) : base(static_cast<char*>(b)), cap(c) {}
   void* take(size_t bytes) {
     void* p = base ? base + off : nullptr;
     off = align_up(off + bytes, 256);
     return p;
   }
+  bool fits() const { return off <= cap; }
 };
 
 bool use_tc(const sph_ctx* ctx, int64_t rows, int w_dtype) {
@@ -130,10 +135,11 @@ size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_
                 int w_dtype, int endpoint) {
   if (!use_tc(ctx, rows, w_dtype)) return 0;
   size_t b = 0;
-  // the larger of the two paths and (automatic tile height, which smaller
-  // calls may choose differently) of the two tile heights
+  // the larger of the two paths, for the plan the call makes (tile height
+  // as set, 0 automatic) and, with the automatic height, for both heights
+  // (which smaller calls may choose)
   for (int gather = 0; gather < 2; ++gather)
-    for (int tm = 128; tm <= 256; tm += 128) {
+    for (int tm = 0; tm <= 256; tm += 128) {
       if (ctx->tc_tile_m && tm != ctx->tc_tile_m) continue;
       const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count,
                                     endpoint, ctx->tc_schedule, ctx->tc_stages,
@@ -474,7 +480,7 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
   const int act_bf16 = act_mode == SPH_ACT_BF16;
   st = ensure_scratch(ctx, partial_scratch_bytes(ctx, rows, n_keep, d_h, act_bf16, wdt));
   if (st) return st;
-  Carve c(ctx->scratch);
+  Carve c(ctx->scratch, ctx->scratch_cap);
   float* Y = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
   unsigned* rowmax = static_cast<unsigned*>(c.take((size_t)rows * 4));
   if (!use_tc(ctx, rows, wdt)) {     // the tensor-core path clears them itself
@@ -498,6 +504,9 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
                                         ctx->tc_block_k, keep_ids != nullptr,
                                         wdt == sph::W_FP8, ctx->tc_max_bn, ctx->tc_tile_m);
     void* tcs = c.take(pl.scratch_bytes);
+    if (!c.fits())
+      return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
+                  c.off, ctx->scratch_cap);
     st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
                        }), "tensor-core launch");
@@ -541,7 +550,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
   st = ensure_scratch(ctx, fuse_scratch_bytes(ctx, rows, n_keep, d_l));
   if (st) return st;
-  Carve c(ctx->scratch);
+  Carve c(ctx->scratch, ctx->scratch_cap);
   float* Z = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
   if (fused_logits_out) Z = fused_logits_out;
   float2* cstats = static_cast<float2*>(c.take((size_t)rows * (n_keep / 1024 + 2) * 8));
@@ -569,6 +578,9 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
                                         ctx->tc_block_k, keep_ids != nullptr, 0,
                                         ctx->tc_max_bn, ctx->tc_tile_m);
     void* tcs = c.take(pl.scratch_bytes);
+    if (!c.fits())
+      return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
+                  c.off, ctx->scratch_cap);
     st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
                        }), "tensor-core launch");
@@ -582,6 +594,9 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
                          }), "sample launch");
   }
   float2* stats = static_cast<float2*>(c.take((size_t)rows * sph::seg_count((int)n_keep) * 8));
+  if (!c.fits())
+    return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
+                c.off, ctx->scratch_cap);
   st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                        return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
                      }), "gemv launch");

@@ -86,6 +86,7 @@ int gemv_max_k();
 struct TcPlan {
   int hilo, RB, BN, Rp, KB, Kp, NT, G, stages, whole_tiles, na, fp8;
   int tm;          // vocabulary rows per tile: 128 or 256
+  int single_acc;  // one TMEM accumulator (256-id tiles over > 128 rows)
   int nseg;        // endpoint statistics: 32-id segments per row, NT * tm / 32
   int epi_stats;   // endpoint: softmax statistics in the epilogue (else a pass over z)
   long long T;

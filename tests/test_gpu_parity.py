@@ -360,6 +360,27 @@ def test_payload_arguments_together(ctx):
                         keep_ids=w.keep_ids)
 
 
+@pytest.mark.parametrize("schedule", [1, 2])
+def test_tensor_core_256_tiles_one_accumulator(ctx, schedule):
+    """256-id tiles over row blocks of more than 128 rows: one accumulator."""
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    ctx.set_option(sph.SPH_OPT_TC_TILE_M, 256)
+    ctx.set_option(sph.SPH_OPT_TC_MAX_BN, 192)
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, schedule)
+    try:
+        w = small(V=5000, d=1096, d_l=72, rows=300, n_keep=3100, seed=950 + schedule)
+        check_cloud(ctx, w, rows=[0, 150, 299])
+        ref = oracle_cloud(w)
+        check_endpoint(ctx, w, torch.from_numpy(ref["codes"]),
+                       torch.from_numpy(ref["row_scale"]), rows=[0, 150, 299])
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+        ctx.set_option(sph.SPH_OPT_TC_TILE_M, 0)
+        ctx.set_option(sph.SPH_OPT_TC_MAX_BN, 0)
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+
+
 # ---------------------------------------------------------------------------
 # split tiles: the designated finisher and the count-in fallback agree bit
 # for bit (the partials are added in the same CTA order on both paths)
