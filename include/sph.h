@@ -113,7 +113,9 @@ typedef enum sph_option {
                                automatic (default)                           */
   SPH_OPT_TC_MAX_BN = 5,    /* most hidden-state rows one tensor-core tile
                                covers: a multiple of 16 in [16, 256], or 0
-                               for automatic (default)                       */
+                               for automatic (default); with
+                               SPH_OPT_TC_TILE_M = 256, above 128 selects
+                               256-id tiles with one accumulator            */
   SPH_OPT_TC_TILE_M = 6,    /* kept vocabulary ids one tensor-core tile
                                covers: 128, 256 (two 128-row MMAs sharing each
                                hidden-state stage; at most 128 hidden-state

@@ -1,47 +1,49 @@
 // Tensor-core gathered contraction for the many-row regime (Eq. 11 / Eq. 12
 // over the kept vocabulary ids), tcgen05 + TMEM on sm_103a.
 //
-// Swap-AB: the MMA's M dimension is a tile of 128 gathered vocabulary rows
+// Swap-AB: the MMA's M dimension is a block of 128 gathered vocabulary rows
 // (operand A), its N dimension a block of BN hidden-state rows (operand B),
-// and K runs over the hidden dimension in 64-element (128-byte) blocks laid
-// out with the 128-byte swizzle.  fp32 hidden states are split beforehand
-// into bf16 hi + lo planes (h = hi + lo + O(2^-18 |h|)); both parts multiply
-// the same W tile into one fp32 TMEM accumulator, so W is read once and the
-// result keeps fp32 accuracy.  In bf16-activation mode only hi is used.
+// and K runs over the hidden dimension in 128-byte atoms (64 bf16 or 128
+// e4m3 elements) laid out with the 128-byte swizzle.  A tile is 128 or 256
+// vocabulary rows; a 256-row tile is two M = 128 MMAs sharing every B stage.
 //
-// Operand A comes from W by TMA 2-D tile copies, one per 64-column atom:
-//   full vocabulary : one box of 128 rows per atom;
-//   kept-id subset  : the tile's 128 kept ids are cut into runs of
-//                     consecutive vocabulary ids and every run is one box of
-//                     exactly its length (one tensor map per height 1..128),
-//                     written at its row of the tile; language subsets are
-//                     mostly long runs, so a tile takes about two boxes, and
-//                     isolated ids still work as 1-row boxes.
-// Operand B (the h planes, L2-resident) always comes by TMA.
+// Hidden states: fp32 h is split beforehand into bf16 hi + lo planes
+// (h = hi + lo + O(2^-18 |h|)) that multiply the same W tile into one fp32
+// TMEM accumulator, so W is read once and the result keeps fp32 accuracy;
+// bf16-activation mode uses hi alone.  With fp8 (e4m3) weights the raw e4m3
+// rows are the A operand of kind::f8f6f4 MMAs against e4m3 planes of h
+// under a per-row power-of-two scale (four planes: 2^-13 of |h|; two
+// reproduce bf16-rounded h), all into one accumulator; the epilogue applies
+// the row's scale and the weight row's scale.
+//
+// Operand A comes from W by TMA 2-D tile copies, one per atom:
+//   full vocabulary : one box of 128 rows per atom (or one 3-D copy of all
+//                     the stage's atoms when the width allows);
+//   kept-id subset  : the tile's kept ids are cut into runs of consecutive
+//                     vocabulary ids and every run is one box of exactly its
+//                     length (one tensor map per height 1..128), written at
+//                     its row of the tile; language subsets are mostly long
+//                     runs, so a 128-id tile takes about two boxes.
+// Operand B (the h planes, L2-resident) comes by one 3-D TMA copy per plane.
 //
 // Work split: the (row block, vocabulary tile, k-block) iterations -- row
 // blocks outermost, so that CTA c and CTA c + G/RB work on the same W rows
 // at the same time and one of the two reads them from L2 -- are cut into
-// one contiguous range per persistent CTA (one CTA per SM).  When K is
-// short, ranges cover whole tiles; otherwise they are split stream-K style
-// and a tile whose k-range spans several CTAs is finished by the last CTA to
-// arrive: contributors store fp32 partials, count in, and the last one adds
-// them in CTA order (deterministic).  No CTA ever waits on another.
+// one contiguous range per persistent CTA (one CTA per SM): whole tiles, or
+// stream-K ranges when that balances better.  A tile whose k-range spans
+// CTAs is finished by a designated contributor (the last to reach it in
+// time), which adds the others' stored fp32 partials in CTA order after a
+// bounded poll for them; if the poll runs out it counts in like the others
+// and the last to count in finishes the tile.  The order of the sum is fixed
+// either way, so results are deterministic.
 //
 // Warp roles: warp 0 issues the TMA copies, warp 1 owns TMEM and issues
-// tcgen05.mma (one thread), warps 2-9 drain the double-buffered accumulator
-// (tcgen05.ld) and run the fused epilogue -- two warps per TMEM lane
-// quadrant, so that the epilogue's dependent shuffle / exp chains of one
-// warp overlap with the other's.  Every wait is bounded; a wait that gives up sets the
-// context's error word and the CTA winds down after its copies and MMAs
-// have landed.
-//
-// fp8 (e4m3) weights: the raw e4m3 rows are the A operand of
-// tcgen05.mma kind::f8f6f4 (a 128-byte atom is 128 elements); h is split
-// into e4m3 planes under a per-row power-of-two scale (4 planes: 2^-13 of
-// |h|; 2 planes reproduce bf16-rounded h) that all add into one fp32
-// accumulator; the epilogue multiplies by the row's scale and the weight
-// row's scale.
+// tcgen05.mma (one thread), warps 2-9 drain the accumulator (double-buffered,
+// or single for 256-row tiles over more than 128 rows) with tcgen05.ld and
+// run the fused epilogue -- two warps per TMEM lane quadrant, so that the
+// epilogue's dependent shuffle / exp chains of one warp overlap with the
+// other's.  Every wait is bounded; a wait that gives up sets the context's
+// error word and the CTA winds down after its copies and MMAs have landed.
 //
 // Epilogues: cloud = + bias, optional unclipped store, clip, store, row |max|
 // (atomicMax); endpoint = + code * row_scale (Eq. 13), store z, and the
@@ -61,11 +63,11 @@
 namespace sph {
 namespace {
 
-constexpr int kTileM = 128;          // vocabulary rows per tile (MMA M)
+constexpr int kTileM = 128;          // vocabulary rows per MMA (M); a tile is 1 or 2 of them
 constexpr int kAtomK = 64;           // bf16 elements per 128-byte swizzle atom
 constexpr int kAtomBytes = kTileM * kAtomK * 2;   // one A atom: 128 rows x 128 B
 constexpr int kMaxBN = 256;
-constexpr int kMaxStages = 12;       // (the barrier area holds (3 * 12 + 5) words)
+constexpr int kMaxStages = 12;       // (the barriers, 2 * 12 + 5 words, fit the 256-byte area)
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
 constexpr int kMaxDevices = 64;      // per-device launch attribute cache
