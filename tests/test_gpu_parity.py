@@ -270,6 +270,27 @@ def test_full_size_sampled_rows(ctx, name, rows, keep):
 
 
 # ---------------------------------------------------------------------------
+# maximum sizes: the API's 2^20 rows, and a kept set past the fused
+# sampler's 4096 chunks (4.19M ids), where the chunk statistics take their
+# own pass
+# ---------------------------------------------------------------------------
+
+def test_max_rows(ctx):
+    w = small(V=600, d=128, d_l=64, rows=1 << 20, n_keep=40, run_lo=4, run_hi=12, seed=1201)
+    sample = [0, 1, 777_777, (1 << 20) - 1]
+    codes, scale, _ = check_cloud(ctx, w, rows=sample)
+    check_endpoint(ctx, w, codes.cpu(), scale.cpu(), rows=sample)
+
+
+def test_kept_set_past_the_fused_sampler(ctx):
+    n = 4096 * 1024 + 5000
+    w = small(V=n + 7000, d=96, d_l=32, rows=4, n_keep=n, run_lo=200, run_hi=4000,
+              seed=1202)
+    codes, scale, _ = check_cloud(ctx, w, rows=[0, 3])
+    check_endpoint(ctx, w, codes.cpu(), scale.cpu())
+
+
+# ---------------------------------------------------------------------------
 # tensor-core kernel variants: pipeline k-block width x work schedule
 # ---------------------------------------------------------------------------
 
