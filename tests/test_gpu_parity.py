@@ -505,14 +505,17 @@ def test_fp8_tensor_core(ctx, rows, keep, act):
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
 
 
+@pytest.mark.parametrize("schedule", [1, 2])
 @pytest.mark.parametrize("tile_m", [128, 256])
 @pytest.mark.parametrize("act", ["fp32", "bf16"])
-def test_fp8_tile_heights(ctx, tile_m, act):
-    """e4m3 weights with both tile heights, gathered and full vocabulary,
-    K = 2048 (16 e4m3 atoms), ragged vocabulary tails."""
+def test_fp8_tile_heights(ctx, tile_m, act, schedule):
+    """e4m3 weights with both tile heights and both schedules (whole tiles;
+    stream-K split tiles), gathered and full vocabulary, K = 2048 (16 e4m3
+    atoms), ragged vocabulary tails."""
     from paper_2607_13093_gb300 import sph
     ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
     ctx.set_option(sph.SPH_OPT_TC_TILE_M, tile_m)
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, schedule)
     try:
         for keep in (2900, 3000):
             w = small(V=3000, d=2304, d_l=256, rows=150, n_keep=keep, w_dtype="fp8",
@@ -521,6 +524,7 @@ def test_fp8_tile_heights(ctx, tile_m, act):
     finally:
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
         ctx.set_option(sph.SPH_OPT_TC_TILE_M, 0)
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
 
 
 # ---------------------------------------------------------------------------
