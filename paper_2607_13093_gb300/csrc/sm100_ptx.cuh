@@ -74,18 +74,6 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, i
       "l"(map), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
 }
-// Four rows y0..y3 (each one box row of the map) at column x, written as
-// four consecutive box rows at dst.
-__device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map,
-                                            int x, int y0, int y1, int y2,
-                                            int y3, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(smem_u32(dst)),
-      "l"(map), "r"(x), "r"(y0), "r"(y1), "r"(y2), "r"(y3),
-      "r"(smem_u32(bar))
-      : "memory");
-}
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }
@@ -131,10 +119,6 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
          ((uint32_t)(M >> 4) << 24);
 }
-// Instruction descriptor for kind::f16 with f16 A/B, fp32 D, K-major A/B.
-__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
-  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
 // Instruction descriptor for kind::f8f6f4 with e4m3 A/B (format code 0 in
 // both operand fields), fp32 D, K-major A/B.
 __host__ __device__ constexpr uint32_t idesc_e4m3_f32(int M, int N) {
@@ -150,7 +134,7 @@ __device__ __forceinline__ void umma_f8(uint32_t d_tmem, uint64_t adesc, uint64_
       : "memory");
 }
 // tcgen05.mma kind::f16 (the operand types come from the instruction
-// descriptor: bf16 x bf16 or f16 x f16)
+// descriptor: bf16 x bf16 here)
 __device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc,
                                           uint64_t bdesc, uint32_t idesc,
                                           uint32_t accumulate) {
@@ -159,11 +143,6 @@ __device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc,
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
-}
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc,
-                                          uint64_t bdesc, uint32_t idesc,
-                                          uint32_t accumulate) {
-  umma_f16(d_tmem, adesc, bdesc, idesc, accumulate);
 }
 // Arrive on `bar` once all previously issued tcgen05.mma of this thread are
 // complete.
@@ -192,36 +171,6 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
-
-}  // namespace ptx
-}  // namespace sph
-
-namespace sph {
-namespace ptx {
-
-// ---- cp.async (16 bytes, L2 only); bytes beyond src_bytes are zero-filled --
-__device__ __forceinline__ void cp_async_16(void* dst, const void* src,
-                                            uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)),
-               "l"(src), "r"(src_bytes)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-// Wait until at most n (0..7) of this thread's most recent groups are pending.
-__device__ __forceinline__ void cp_async_wait(int n) {
-  switch (n) {
-    case 0: asm volatile("cp.async.wait_group 0;" ::: "memory"); break;
-    case 1: asm volatile("cp.async.wait_group 1;" ::: "memory"); break;
-    case 2: asm volatile("cp.async.wait_group 2;" ::: "memory"); break;
-    case 3: asm volatile("cp.async.wait_group 3;" ::: "memory"); break;
-    case 4: asm volatile("cp.async.wait_group 4;" ::: "memory"); break;
-    case 5: asm volatile("cp.async.wait_group 5;" ::: "memory"); break;
-    case 6: asm volatile("cp.async.wait_group 6;" ::: "memory"); break;
-    default: asm volatile("cp.async.wait_group 7;" ::: "memory"); break;
-  }
-}
 // Load with acquire semantics at GPU scope (pairs with a fence before
 // another CTA's atomic update of the same word).
 __device__ __forceinline__ int ld_acquire_gpu(const int* p) {
@@ -229,11 +178,13 @@ __device__ __forceinline__ int ld_acquire_gpu(const int* p) {
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
-// Make this thread's generic-proxy shared-memory writes visible to later
-// async-proxy reads (tcgen05.mma operands).
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
+
+}  // namespace ptx
+}  // namespace sph
+
+namespace sph {
+namespace ptx {
+
 
 }  // namespace ptx
 }  // namespace sph
