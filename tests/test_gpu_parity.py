@@ -94,6 +94,20 @@ def test_cloud_zero_row_and_edge_ids(path_ctx):
     assert np_(scale)[2] == 0 and not np_(codes)[2].any()
 
 
+def test_cloud_tiny_row_scales(path_ctx):
+    # row scales below 2^-64 quantize like ordinary rows
+    w = small(V=3000, d=264, d_l=8, rows=4, n_keep=2500)
+    w.h[1] *= 1e-21
+    w.h[3] *= 1e-24
+    codes, scale, _ = check_cloud(path_ctx, w)
+    ref = oracle_cloud(w, "fp32", None)
+    s = np_(scale).astype(np.float64)
+    for r in (1, 3):
+        assert 0 < s[r] < 2.0 ** -64
+        assert abs(s[r] - ref["row_scale"][r]) <= 1e-3 * ref["row_scale"][r]
+        assert np.abs(np_(codes)[r]).max() == 127
+
+
 def test_cloud_odd_hidden_width_and_strides(path_ctx):
     ctx = path_ctx
     # d_h = 37 (not a multiple of anything) inside a padded weight stride
