@@ -17,9 +17,10 @@ namespace {
 // quantize: s_r = fl32(max_r / 127); code = rint_even(yc * fl32(1 / s_r)), |code|<=127
 // ---------------------------------------------------------------------------
 // A work item is one row and a span of 2048 of its entries: the row's scale
-// is found once per item, and each thread takes eight consecutive entries
-// (two 16-byte loads and one 8-byte store of the codes where alignment
-// allows, else element by element).
+// is found once per item.  Where rows start 16-byte aligned each thread takes
+// eight consecutive entries (two 16-byte loads, one 8-byte store of the
+// codes); otherwise it takes every 256th entry of the span, so that a warp's
+// loads and stores stay contiguous.
 constexpr int kQVec = 8;
 constexpr int kQThreads = 256;
 constexpr int kQSpan = kQThreads * kQVec;
@@ -60,12 +61,31 @@ quantize_kernel(const float* __restrict__ Y, const unsigned* __restrict__ rowmax
     // factor 2^64 on both sides so that its reciprocal stays finite
     const float k = s < 0x1p-64f ? 0x1p64f : 1.f;
     const float inv_s = s > 0.f ? __frcp_rn(s * k) : 0.f;  // an all-zero row: codes 0
+    const int64_t row0 = (int64_t)r * n;
+    if (!vec_load) {
+      // rows not 16-byte aligned: entry i of the thread is column
+      // span + i * 256 + thread, so each warp instruction reads 32 adjacent
+      // partials and writes 32 adjacent codes
+      const int cb = sp * kQSpan + threadIdx.x;
+      float y[kQVec];
+#pragma unroll
+      for (int i = 0; i < kQVec; ++i) {
+        const int c = cb + i * kQThreads;
+        y[i] = c < n ? __ldcs(Y + row0 + c) : 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < kQVec; ++i) {
+        const int c = cb + i * kQThreads;
+        if (c < n) codes[row0 + c] = (int8_t)quantize_one(y[i], k, inv_s);
+      }
+      continue;
+    }
     const int c0 = sp * kQSpan + threadIdx.x * kQVec;
     if (c0 >= n) continue;
-    const int64_t e0 = (int64_t)r * n + c0;
+    const int64_t e0 = row0 + c0;
     const bool full = c0 + kQVec <= n;
     float y[kQVec];
-    if (full && vec_load) {
+    if (full) {
       const float4 u = __ldcs(reinterpret_cast<const float4*>(Y + e0));
       const float4 v = __ldcs(reinterpret_cast<const float4*>(Y + e0) + 1);
       y[0] = u.x; y[1] = u.y; y[2] = u.z; y[3] = u.w;
