@@ -27,6 +27,15 @@ constexpr int kWarps = 8;               // warps per CTA
 constexpr int kMaxN = 1 << 30;          // ids per row
 constexpr int kMaxK = 64;               // drafts per session
 
+// exp(d / tau) for the per-logit passes, as 2^(d * (log2(e) / tau)): the
+// scale is one fp32 rounding of log2(e) / tau (relative 2^-24, so an error of
+// at most |d / tau| * 6e-8 in the exponent) and exp2f then needs no range
+// reduction of its own.
+constexpr float kLog2e = 1.4426950408889634f;
+__device__ __forceinline__ float exp_tau(float d, float log2e_inv_tau) {
+  return exp2f(d * log2e_inv_tau);
+}
+
 __device__ __forceinline__ float seg_weight(float2 st, float M, float inv_tau) {
   return st.y > 0.f ? st.y * expf((st.x - M) * inv_tau) : 0.f;
 }
@@ -43,12 +52,22 @@ seg_stats_kernel(const float* __restrict__ Z, int rows, int n, int nseg, int nch
   ptx::griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
   const int kr = (lane >> 1) & 15;
+  const float l2t = inv_tau * kLog2e;
   const long long total = (long long)nchunk * rows;
   const long long nwarps = (long long)gridDim.x * kWarps;
+  const bool narrow = total <= INT_MAX;
   for (long long g = (long long)blockIdx.x * kWarps + (threadIdx.x >> 5); g < total;
        g += nwarps) {
-    const long long r = g / nchunk;
-    const int c = (int)(g - r * nchunk);
+    long long r;
+    int c;
+    if (narrow) {
+      const unsigned rr = (unsigned)g / (unsigned)nchunk;
+      r = rr;
+      c = (int)((unsigned)g - rr * (unsigned)nchunk);
+    } else {
+      r = g / nchunk;
+      c = (int)(g - r * nchunk);
+    }
     const float* z = Z + r * n;
     float v[2][kGroup];
 #pragma unroll
@@ -67,7 +86,7 @@ seg_stats_kernel(const float* __restrict__ Z, int rows, int n, int nseg, int nch
 #pragma unroll
       for (int q = 0; q < kGroup; ++q) {
         const float mq = __shfl_sync(0xFFFFFFFFu, mk[h], 2 * q);
-        e[q] = v[h][q] > -INFINITY ? expf((v[h][q] - mq) * inv_tau) : 0.f;
+        e[q] = v[h][q] > -INFINITY ? exp_tau(v[h][q] - mq, l2t) : 0.f;
       }
       sk[h] = warp_reduce_scatter16(e, SumOp{}, lane);
       const int sg = c * kSeg + h * kGroup + kr;
@@ -204,10 +223,10 @@ struct ExpWeight {                      // exp((z_j - M) / tau)
 struct ResidualWeight {
   const float* z;
   const float* q;
-  float M, inv_tau, inv_S;
+  float M, l2t, inv_S;                  // l2t = log2(e) / tau
   int xi;
   __device__ float operator()(int j) const {
-    const float p = expf((z[j] - M) * inv_tau) * inv_S;
+    const float p = exp_tau(z[j] - M, l2t) * inv_S;
     if (q) return fmaxf(0.f, p - q[j]);
     return j == xi ? 0.f : p;
   }
@@ -490,7 +509,7 @@ verify_residual_kernel(const float* __restrict__ Z, int n, int nseg, int nchunk,
     const int64_t r = (int64_t)s * (k + 1) + i;
     const int64_t di = (int64_t)s * k + i;
     const float2 ms = rowMS[r];
-    const ResidualWeight rw{Z + r * n, q ? q + di * n : nullptr, ms.x, inv_tau,
+    const ResidualWeight rw{Z + r * n, q ? q + di * n : nullptr, ms.x, inv_tau * kLog2e,
                             1.f / ms.y, xis[di]};
     float csum = 0.f;
 #pragma unroll
@@ -557,7 +576,7 @@ verify_draw_kernel(const float* __restrict__ Z, int n, const float2* __restrict_
     const int64_t di = (int64_t)s * k + i;
     const ArrayWeight cw{resc + (int64_t)s * nchunk};
     const ArrayWeight sw{resw + (int64_t)s * nseg};
-    const ResidualWeight rw{Z + r * n, q ? q + di * n : nullptr, ms.x, inv_tau,
+    const ResidualWeight rw{Z + r * n, q ? q + di * n : nullptr, ms.x, inv_tau * kLog2e,
                             1.f / ms.y, xis[di]};
     tot = warp_draw(nchunk, nseg, n, cw, sw, rw, u, lane, j);
   }
