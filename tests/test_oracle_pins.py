@@ -439,6 +439,46 @@ def test_verify_draft_end_to_end_tiny():
     assert np.all((out["n_accepted"] >= 0) & (out["n_accepted"] <= 2))
 
 
+def test_verify_draft_preserves_each_sessions_target_distribution():
+    # End to end through verify_draft's own row, draft and uniform wiring:
+    # drafts drawn from q (numpy's generator, independent of Philox), then
+    # over many offsets the first emitted token of session s follows
+    # softmax(z_{s,0} / tau), and after an accepted first draft the second
+    # follows softmax(z_{s,1} / tau) -- the defining property of
+    # speculative sampling.  Rows differ per session and position, ids are
+    # a masked subset of V, so a wrong row, draft-probability or id mapping
+    # shows up as a distribution mismatch.
+    from scipy.stats import chisquare
+    S, k, n, tau = 2, 2, 5, 0.7
+    V = 9
+    keep = np.array([0, 2, 3, 6, 8])
+    g = np.random.default_rng(2024)
+    Z = g.normal(0.0, 1.2, size=(S * (k + 1), n)).astype(np.float32)
+    q = g.dirichlet(np.ones(n), size=(S, k))
+    P = np.exp(Z.astype(np.float64) / tau)
+    P /= P.sum(axis=1, keepdims=True)
+    trials = 3000
+    first = np.zeros((S, n))
+    second = np.zeros((S, n))
+    pos = {int(v): i for i, v in enumerate(keep)}
+    for t in range(trials):
+        x = np.array([[g.choice(n, p=q[s, i]) for i in range(k)] for s in range(S)])
+        out = oracle.verify_draft(Z, S, k, keep_ids=keep, V=V, tau=tau,
+                                  draft_tokens=keep[x], draft_probs=q, seed=11,
+                                  offset=t)
+        for s in range(S):
+            a = int(out["n_accepted"][s])
+            nxt = pos[int(out["next_token"][s])]
+            first[s, x[s, 0] if a >= 1 else nxt] += 1
+            if a >= 1:
+                second[s, x[s, 1] if a >= 2 else nxt] += 1
+    for s in range(S):
+        assert chisquare(first[s], P[s * (k + 1)] * trials).pvalue > 1e-3
+        m = second[s].sum()
+        assert m > trials / 10
+        assert chisquare(second[s], P[s * (k + 1) + 1] * m).pvalue > 1e-3
+
+
 def test_compact_index_brute_force():
     ids = np.array([2, 3, 7, 11, 12])
     toks = np.array([0, 2, 3, 4, 7, 12, 13, 11, -1])
