@@ -118,8 +118,13 @@ typedef enum sph_option {
                                256-id tiles with one accumulator            */
   SPH_OPT_TC_TILE_M = 6,    /* kept vocabulary ids one tensor-core tile
                                covers: 128, 256 (two 128-row MMAs sharing each
-                               hidden-state stage; at most 128 hidden-state
-                               rows per tile), or 0 for automatic (default)  */
+                               hidden-state stage), or 0 for automatic
+                               (default).  A 256-id tile keeps two
+                               accumulators for up to 128 hidden-state rows;
+                               with SPH_OPT_TC_MAX_BN above 128 (and in the
+                               automatic plan for row blocks of 129-192 rows)
+                               it keeps one, for up to 256 rows (224 with fp32
+                               activations)                                  */
   SPH_OPT_TC_FINISH_WAIT = 7, /* clock cycles the designated finisher of a
                                tensor-core tile split across CTAs polls for
                                the other contributors' partials (default
