@@ -90,6 +90,8 @@ def parse():
     ap.add_argument("--sampler", choices=["cdf", "gumbel"], default="cdf",
                     help="endpoint draw: inverse CDF (default) or Gumbel-max")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--ref-seconds", type=float, default=150.0,
+                    help="--impl reference: host seconds of oracle work over all steps")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
 
@@ -602,7 +604,7 @@ def run_reference(args):
     w = wl.workload(args.workload, device="cpu", rows=args.rows, keep_frac=args.keep,
                     d_l=args.d_l)
     s = OracleSample(w, args.act, args.nosplit, args.sampler)
-    budget = 150.0
+    budget = args.ref_seconds
     L = s.calibrate(budget / max(1, args.steps + args.warmup))
     for _ in range(args.warmup):
         s.run(L)

@@ -59,3 +59,28 @@ def test_job_throughput_counts_every_rank():
     import bench
     assert bench.job_rows_per_s(32, 4, 100, 1000.0) == 32 * 4 * 100 / 1.0
     assert bench.max_over_ranks(3.5) == 3.5          # no process group: identity
+
+
+def test_reference_arm_under_torchrun_prints_once_from_rank_zero():
+    # two ranks launched as the driver launches them; rank 0 alone times the
+    # oracle and prints the one JSON line, rank 1 exits 0 without work
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(_free_port()),
+           "bench.py", "--impl", "reference", "--gpus", "2", "--steps", "2", "--warmup", "1",
+           "--workload", "tiny", "--ref-seconds", "2"]
+    env = dict(os.environ, OMP_NUM_THREADS="1")
+    p = subprocess.run(cmd, cwd=root, env=env, capture_output=True, text=True, timeout=600)
+    assert p.returncode == 0, p.stderr[-2000:]
+    lines = [l for l in p.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    out = json.loads(lines[0])
+    assert out["impl"] == "reference" and out["n_gpus"] == 2
+    assert out["value"] > 0 and out["e2e"]["value"] == out["value"]
+    assert out["cpu_baseline"]["kind"] == "oracle"
+    for key in ("metric", "unit", "steps", "warmup", "ms_per_step", "higher_is_better",
+                "config", "dtype"):
+        assert key in out
