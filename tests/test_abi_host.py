@@ -75,3 +75,47 @@ def test_create_without_device_fails_cleanly(sph):
         pytest.skip("a GPU is present")
     with pytest.raises(sph.SphError):
         sph.sph_create(0, None)
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path):
+    # a copy of the binding beside no built library: importing it raises
+    # instead of falling back to anything else
+    import importlib.util
+    import shutil
+    src = os.path.join(ROOT, "paper_2607_13093_gb300", "sph.py")
+    dst = tmp_path / "sph_copy.py"
+    shutil.copy(src, dst)
+    spec = importlib.util.spec_from_file_location("sph_copy", dst)
+    mod = importlib.util.module_from_spec(spec)
+    with pytest.raises(RuntimeError, match="not built"):
+        spec.loader.exec_module(mod)
+
+
+def test_product_package_never_imports_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2607_13093_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp", ".c")):
+                text = open(os.path.join(dirpath, f), errors="replace").read()
+                assert not re.search(r"^\s*(import|from)\s+oracle\b", text, flags=re.M), f
+                assert "sph_oracle" not in text, f
+
+
+def test_oracle_imports_nothing_of_the_product():
+    # the oracle depends on numpy alone (and on its own modules)
+    import ast
+    odir = os.path.join(ROOT, "oracle")
+    for f in os.listdir(odir):
+        if f.endswith(".py"):
+            tree = ast.parse(open(os.path.join(odir, f)).read())
+            for node in ast.walk(tree):
+                if isinstance(node, ast.Import):
+                    mods = [a.name for a in node.names]
+                elif isinstance(node, ast.ImportFrom):
+                    if node.level > 0:
+                        continue
+                    mods = [node.module]
+                else:
+                    continue
+                for m in mods:
+                    assert m.split(".")[0] in ("numpy", "__future__"), (f, m)
