@@ -32,7 +32,7 @@ Input recipe (every workload):
   * speculative drafts: per session and draft position, logits ~ N(0, std 2)
     over the kept ids, q = softmax(logits) stored fp32, draft token drawn from
     q; target rows are the fused logits of the S*(k+1) verification rows.
-  * seeds: workload seed = 1000 + workload number (tiny=1 ... sweep=5).
+  * seeds: workload seed = 1000 + workload number (tiny=1 ... dend=6).
 """
 from __future__ import annotations
 
