@@ -28,7 +28,8 @@
  *     logits are "compacted": column j belongs to vocabulary id keep_ids[j].
  *   - A context is not thread-safe; use one per host thread.
  *   - There is no CPU fallback: a shape the kernels do not support returns
- *     SPH_ERR_UNSUPPORTED.
+ *     SPH_ERR_UNSUPPORTED.  The hot-path calls take at most 2^20 rows (or
+ *     sessions*(k+1) target rows) and at most 2^30 kept ids per row.
  */
 #ifndef SPH_H_
 #define SPH_H_

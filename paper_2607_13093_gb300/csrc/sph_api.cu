@@ -471,6 +471,9 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
   if (((uintptr_t)W_h & 15) || ((ld_w * esz) & 15))
     return fail(ctx, SPH_ERR_INVALID_ARG, "W_h base and row stride must be 16-byte aligned");
   if (rows * n_keep > ((int64_t)1 << 40)) return fail(ctx, SPH_ERR_UNSUPPORTED, "rows*n_keep too large");
+  // the payload's consumer takes at most this many ids, and the kernels
+  // index columns in 32 bits
+  if (n_keep > sph::sample_max_n()) return fail(ctx, SPH_ERR_UNSUPPORTED, "n_keep above %d", sph::sample_max_n());
   if (d_h > sph::gemv_max_k()) return fail(ctx, SPH_ERR_UNSUPPORTED, "d_h=%lld above %d", (long long)d_h, sph::gemv_max_k());
   if (payload_bytes) *payload_bytes = sph_payload_bytes(rows, n_keep);
 
