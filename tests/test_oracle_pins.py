@@ -255,6 +255,19 @@ _TRITON_PHILOX = textwrap.dedent("""
 """)
 
 
+def test_philox_known_answers():
+    # the published known-answer outputs of Philox4x32-10
+    # (tests/golden/philox4x32_10_kat.json)
+    with open(os.path.join(GOLDEN, "philox4x32_10_kat.json")) as f:
+        kat = json.load(f)
+    for v in kat["vectors"]:
+        c = [np.array([int(x, 16)], dtype=np.uint64) for x in v["counter"]]
+        k0, k1 = (int(x, 16) for x in v["key"])
+        out = oracle.philox4x32_10(*c, k0, k1)
+        got = [int(np.asarray(o).ravel()[0]) for o in out]
+        assert got == [int(x, 16) for x in v["output"]]
+
+
 def test_philox_matches_triton_interpreter():
     pytest.importorskip("triton")
     rng = np.random.default_rng(5)
