@@ -108,6 +108,62 @@ def test_cloud_tiny_row_scales(path_ctx):
         assert np.abs(np_(codes)[r]).max() == 127
 
 
+GUARD_BYTES = 256              # keeps every output view 256-byte aligned
+SENTINEL = 0xA5
+
+
+def guarded(shape, dtype):
+    """An output tensor inside a larger buffer whose GUARD_BYTES margins on
+    each side hold a sentinel byte."""
+    n = int(np.prod(shape))
+    g = GUARD_BYTES // torch.empty((), dtype=dtype).element_size()
+    buf = torch.empty(n + 2 * g, dtype=dtype, device=DEV)
+    buf.view(torch.uint8).fill_(SENTINEL)
+    return buf, buf[g:g + n].view(shape)
+
+
+def guards_intact(buf):
+    b = buf.view(torch.uint8)
+    return bool((b[:GUARD_BYTES] == SENTINEL).all()) and bool((b[-GUARD_BYTES:] == SENTINEL).all())
+
+
+@pytest.mark.parametrize("w_dtype", ["bf16", "fp8"])
+@pytest.mark.parametrize("n_keep", [1301, 1304])
+def test_outputs_stay_inside_their_buffers(path_ctx, w_dtype, n_keep):
+    # every output of the three calls sits between sentinel margins; a write
+    # past either end of any output (a vector store rounded up to a tile, a
+    # ragged tail) shows up as a changed margin byte
+    ctx = path_ctx
+    S, k = 6, 2
+    w = small(V=3000, d=1048, d_l=40, rows=S * (k + 1), n_keep=n_keep, w_dtype=w_dtype,
+              clip=40.0 if w_dtype == "fp8" else 30.0, sessions=S, k=k, tau=0.9)
+    R, n = w.rows, w.n_keep
+    outs = {}
+    outs["codes"], codes = guarded((R, n), torch.int8)
+    outs["row_scale"], scale = guarded((R,), torch.float32)
+    outs["partial_out"], part = guarded((R, n), torch.float32)
+    ctx.partial_logits(w.h_cloud, w.W_h, keep_ids=w.keep_ids, clip=w.clip,
+                       w_row_scale=w.w_scale, codes=codes, row_scale=scale,
+                       partial_out=part)
+    for tau in (w.tau, 0.0):
+        outs[f"tokens {tau}"], tok = guarded((R,), torch.int32)
+        outs[f"z {tau}"], z = guarded((R, n), torch.float32)
+        ctx.fuse_sample(codes, scale, w.h_local, w.W_l, keep_ids=w.keep_ids,
+                        temperature=tau, seed=w.seed, tokens=tok, fused_logits_out=z)
+        outs[f"n_accepted {tau}"], acc = guarded((S,), torch.int32)
+        outs[f"next_token {tau}"], nxt = guarded((S,), torch.int32)
+        ctx.verify_draft(z, S, k, w.draft_tokens, keep_ids=w.keep_ids,
+                         draft_probs=w.draft_probs if tau > 0 else None, temperature=tau,
+                         seed=w.seed, n_accepted=acc, next_token=nxt)
+        ctx.sync()
+        assert set(np_(tok).tolist()) <= set(np_(w.keep_ids).tolist())
+        assert ((np_(acc) >= 0) & (np_(acc) <= k)).all()
+    ctx.sync()
+    assert np.abs(np_(codes).astype(int)).max() == 127 and (np_(scale) > 0).all()
+    for name, buf in outs.items():
+        assert guards_intact(buf), name
+
+
 def test_cloud_odd_hidden_width_and_strides(path_ctx):
     ctx = path_ctx
     # d_h = 37 (not a multiple of anything) inside a padded weight stride
