@@ -640,3 +640,26 @@ def test_graph_capture_matches_direct_calls(ctx, rows_kw):
     ctx.sync()
     for a, b in zip(ref, (codes, scale, tokens, z, n_acc, nxt)):
         assert torch.equal(a, b)
+
+
+def test_tracing_times_each_call_class_once(ctx):
+    # one cloud, one endpoint and one verification call under tracing: one
+    # timed group per class with positive device time, and every kernel
+    # counted; enabling again starts from zero
+    S, k = 6, 2
+    w = small(V=3000, d=1048, d_l=40, rows=S * (k + 1), n_keep=1301, sessions=S, k=k, tau=0.9)
+    z = torch.empty(w.rows, w.n_keep, device=DEV)
+    ctx.profile_enable(True)
+    codes, scale, _ = ctx.partial_logits(w.h_cloud, w.W_h, keep_ids=w.keep_ids, clip=w.clip)
+    ctx.fuse_sample(codes, scale, w.h_local, w.W_l, keep_ids=w.keep_ids, temperature=w.tau,
+                    seed=w.seed, fused_logits_out=z)
+    ctx.verify_draft(z, S, k, w.draft_tokens, keep_ids=w.keep_ids, draft_probs=w.draft_probs,
+                     temperature=w.tau, seed=w.seed)
+    p = ctx.profile_read()
+    ctx.profile_enable(True)
+    fresh = ctx.profile_read()
+    ctx.profile_enable(False)
+    for c in ("cloud_gemm", "quantize", "local_gemm", "sample", "verify"):
+        assert p["calls"][c] == 1 and p["ms"][c] > 0, (c, p)
+    assert p["launches"] >= 7          # split + contraction, quantize, endpoint, draw, verification
+    assert fresh["launches"] == 0 and not any(fresh["calls"].values())
