@@ -23,7 +23,9 @@
  *     the stated leading dimension (in elements).  The context owns only
  *     its scratch memory (grown on demand, or pre-sized by sph_reserve()).
  *   - keep_ids is the language subset V_l: int32 vocabulary ids, strictly
- *     increasing, each in [0, V).  NULL means the full vocabulary
+ *     increasing, each in [0, V).  This is a precondition the kernels do
+ *     not check: an id outside [0, V) makes them read outside W (and
+ *     w_row_scale, bias).  NULL means the full vocabulary
  *     (mixed-language mode) and then n_keep must equal V.  Payloads and
  *     logits are "compacted": column j belongs to vocabulary id keep_ids[j].
  *   - A context is not thread-safe; use one per host thread.

@@ -19,7 +19,7 @@ enum WDtype : int { W_BF16 = 0, W_FP8 = 1 };
 // Device-side error bits (OR-ed into the context's status word).
 enum : unsigned int {
   ERR_TIMEOUT = 1u,     // a bounded wait gave up
-  ERR_BAD_INDEX = 2u,   // an id or index outside its range was skipped
+  ERR_BAD_INDEX = 2u,   // reserved for an id outside its range (no kernel checks ids yet)
 };
 
 // Kernels launched by this thread (read by the tracing layer).
