@@ -206,6 +206,10 @@ sph_status sph_keep_ids_from_mask(const uint8_t* mask, int64_t V,
  *   yc           = min(max(y, -clip), clip)
  *   row_scale[r] = max_j |yc[r, j]| / 127   (fp32; 0 for an all-zero row)
  *   codes[r, j]  = round-half-even(yc / row_scale[r]) in [-127, 127]
+ *                  (the kernels multiply yc by the correctly rounded fp32
+ *                  reciprocal of row_scale[r], so a code can differ by one
+ *                  from the exact quotient's rounding only where that
+ *                  quotient lies within about 1.5e-5 of a half-integer)
  * Arguments
  *   h_cloud  fp32 [rows, d_h] with row stride ld_h (>= d_h); typically the
  *            slice h[:, d_l:] of the full hidden state (ld_h = d).
@@ -293,7 +297,8 @@ sph_status sph_partial_logits_noalloc(int device, void* cuda_stream,
  *   comparator of the paper's "no split projection" ablation).  Exactly one
  *   of them NULL is INVALID_ARG.
  *   h_local fp32 [rows, d_l], row stride ld_hl (the slice h[:, :d_l]).
- *   W_l bf16 [V, d_l] row-major with row stride ld_wl (16-byte multiple).
+ *   W_l bf16 [V, d_l] row-major with row stride ld_wl; the base address
+ *   and ld_wl*2 must be multiples of 16 bytes.
  *   keep_ids as for sph_partial_logits.  temperature >= 0 and finite.
  *   tokens int32 [rows] (out, vocabulary ids).
  *   fused_logits_out fp32 [rows, n_keep] z before the division by
