@@ -72,11 +72,13 @@ def job_rows_per_s(rows_per_rank, world, steps, ms):
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="decode",
-                    choices=["tiny", "decode", "spec", "fp8", "sweep", "dend"])
+    ap.add_argument("--workload", default="sweep",
+                    choices=["tiny", "decode", "spec", "fp8", "sweep", "dend"],
+                    help="headline workload (default: the largest, the sweep at 1024 rows "
+                         "over the full 256000-id vocabulary)")
     ap.add_argument("--rows", type=int, default=None, help="sweep / dend: rows")
     ap.add_argument("--keep", type=float, default=None, help="sweep / dend: keep fraction")
     ap.add_argument("--d-l", type=int, default=None, help="dend: split dimension d_l")
@@ -90,6 +92,12 @@ def parse():
     ap.add_argument("--sampler", choices=["cdf", "gumbel"], default="cdf",
                     help="endpoint draw: inverse CDF (default) or Gumbel-max")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--config-cpu-seconds", type=float, default=3.0,
+                    help="oracle seconds per entry of the per-configuration block")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the per-configuration block")
+    ap.add_argument("--dend-grid", action="store_true",
+                    help="add the split-dimension study's grid (d_l x keep) to the block")
     ap.add_argument("--ref-seconds", type=float, default=150.0,
                     help="--impl reference: host seconds of oracle work over all steps")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -281,7 +289,11 @@ def source_hash(files):
     return h.hexdigest()[:16]
 
 
-def traffic_for(kernel_key, files):
+KERNEL_FILES = ["paper_2607_13093_gb300/csrc/k_tc.cu", "paper_2607_13093_gb300/csrc/k_gemv.cu",
+                "paper_2607_13093_gb300/csrc/k_finish.cu"]
+
+
+def traffic_for(kernel_key, files=KERNEL_FILES):
     """DRAM bytes per launch from a committed ncu summary, if it was taken
     on the current source of that kernel."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
@@ -293,6 +305,307 @@ def traffic_for(kernel_key, files):
     except Exception:
         pass
     return None
+
+
+def operand_planes(w, act):
+    """MMA passes the tensor-core kernel issues per algorithmic one: fp32
+    activations take bf16 hi + lo planes (e4m3 heads: four e4m3 planes),
+    bf16-rounded activations one plane (e4m3 heads: two)."""
+    if w.w_dtype == "fp8":
+        return 4 if act == "fp32" else 2
+    return 2 if act == "fp32" else 1
+
+
+def roofline(w, act, unit_ms, peaks, nosplit=False):
+    """Roofline of the dominant unit (the cloud call; the unsplit head with
+    nosplit) from its mean event-timed duration.  Only algorithmic bytes and
+    flops are credited.  The bound is whichever roof takes longer at its
+    peak: HBM (the measured copy bandwidth) or the tensor pipe (the measured
+    bf16 burst rate; for e4m3 weights on the f8f6f4 pipe twice that, the
+    nominal fp8:bf16 ratio)."""
+    from paper_2607_13093_gb300 import workloads as wl
+    R, n = w.rows, w.n_keep
+    fp8 = w.w_dtype == "fp8"
+    if nosplit:
+        alg_bytes = n * w.d * 2 + 4 * R * w.d + 4 * n + 4 * R
+        alg_flops = wl.algorithmic_flops(R, n, w.d)
+    else:
+        alg_bytes = wl.algorithmic_bytes_cloud(R, n, w.d_h, 1 if fp8 else 2, fp8_scales=fp8)
+        alg_flops = wl.algorithmic_flops(R, n, w.d_h)
+    hbm = peaks["hbm_gbs"]
+    tc = peaks["bf16_tflops"] * (2 if fp8 and not nosplit else 1)
+    s = unit_ms / 1e3
+    bw = alg_bytes / s / 1e9
+    fl = alg_flops / s / 1e12
+    t_hbm = alg_bytes / (hbm * 1e9)
+    t_tc = alg_flops / (tc * 1e12)
+    planes = 1 if nosplit else operand_planes(w, act)
+    tensor = {"achieved": round(fl, 2), "peak": tc, "unit": "TFLOP/s",
+              "frac": round(fl / tc, 4),
+              "issued_frac": round(planes * fl / tc, 4) if not nosplit else None,
+              "planes": planes,
+              "peak_note": ("e4m3 x e4m3 (kind::f8f6f4): 2 x the measured bf16 burst"
+                            if fp8 and not nosplit else "measured bf16 burst")}
+    mem = {"achieved": round(bw, 1), "peak": hbm, "unit": "GB/s", "frac": round(bw / hbm, 4)}
+    bound = "tensor" if t_tc > t_hbm else "hbm"
+    main = tensor if bound == "tensor" else mem
+    out = {"bound": bound, "achieved": main["achieved"], "peak": main["peak"],
+           "unit": main["unit"], "frac": main["frac"],
+           "algorithmic_bytes": alg_bytes, "algorithmic_flops": alg_flops,
+           "hbm": mem, "tensor": tensor,
+           "avg_launch_ms": round(unit_ms, 5)}
+    if bound == "tensor":
+        out["issued_frac"] = tensor["issued_frac"]
+    return out
+
+
+class Runner:
+    """One workload's buffers and its step: the cloud call then the endpoint
+    call (+ verification for drafted workloads); `nosplit` replaces both
+    with one endpoint call over the whole head (the no-split ablation)."""
+
+    def __init__(self, sph, wl, w, dev, act="fp32", nosplit=False, sampler="cdf"):
+        import torch
+        self.sph, self.w, self.dev, self.act, self.nosplit = sph, w, dev, act, nosplit
+        R, n = w.rows, w.n_keep
+        self.ctx = ctx = sph.Context(dev.index or 0)
+        self.act_mode = sph.SPH_ACT_BF16 if act == "bf16" else sph.SPH_ACT_FP32
+        if sampler == "gumbel":
+            ctx.set_option(sph.SPH_OPT_SAMPLER, sph.SPH_SAMPLER_GUMBEL)
+        if nosplit and w.w_dtype != "bf16":
+            raise SystemExit("--nosplit needs bf16 weights (the endpoint head is bf16)")
+        ctx.reserve(R, n, w.d if nosplit else max(w.d_h, w.d_l))
+        # weight and h copies rotate so that the bytes touched between two
+        # uses of the same copy exceed twice the L2
+        self.l2 = l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+        wb = 1 if w.w_dtype == "fp8" else 2
+        self.per_copy = per_copy = n * w.d_h * wb + n * w.d_l * 2
+        self.ncopy = ncopy = (max(1, math.ceil(2 * l2 / per_copy) + 1)
+                              if per_copy < 2 * l2 else 1)
+        if nosplit:
+            self.Wfs = [torch.cat([w.W_l, w.W_h], dim=1).contiguous()]
+            self.Wfs += [self.Wfs[0].clone() for _ in range(ncopy - 1)]
+            self.Whs = self.Wls = [None] * ncopy
+        else:
+            self.Whs = [w.W_h] + [w.W_h.clone() for _ in range(ncopy - 1)]
+            self.Wls = [w.W_l] + [w.W_l.clone() for _ in range(ncopy - 1)]
+        self.hs = [w.h] + [w.h.roll(i + 1, dims=0).contiguous() for i in range(ncopy - 1)]
+        self.codes = torch.empty(R, n, dtype=torch.int8, device=dev)
+        self.scale = torch.empty(R, dtype=torch.float32, device=dev)
+        self.tokens = torch.empty(R, dtype=torch.int32, device=dev)
+        self.z = torch.empty(R, n, device=dev) if w.sessions else None
+        self.n_acc = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
+        self.nxt = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
+        self.gsteps = ncopy * max(1, math.ceil(16 / ncopy))
+
+    def step(self, i, h=None, events=None):
+        w, ctx = self.w, self.ctx
+        c = i % self.ncopy
+        hh = self.hs[c] if h is None else h
+        if events is not None:
+            events[0].record()
+        if self.nosplit:                 # one endpoint call over the whole head
+            ctx.fuse_sample(None, None, hh, self.Wfs[c], keep_ids=w.keep_ids,
+                            temperature=w.tau, seed=w.seed, offset=i, tokens=self.tokens,
+                            fused_logits_out=self.z)
+        else:
+            ctx.partial_logits(hh[:, w.d_l:], self.Whs[c], keep_ids=w.keep_ids, clip=w.clip,
+                               w_row_scale=w.w_scale, bias=w.bias, codes=self.codes,
+                               row_scale=self.scale, act_mode=self.act_mode)
+        if events is not None:
+            events[1].record()
+        if not self.nosplit:
+            ctx.fuse_sample(self.codes, self.scale, hh[:, :w.d_l], self.Wls[c],
+                            keep_ids=w.keep_ids, temperature=w.tau, seed=w.seed, offset=i,
+                            tokens=self.tokens, fused_logits_out=self.z)
+        if w.sessions:
+            ctx.verify_draft(self.z, w.sessions, w.k, w.draft_tokens, keep_ids=w.keep_ids,
+                             draft_probs=w.draft_probs, temperature=w.tau,
+                             seed=w.seed, offset=i, n_accepted=self.n_acc, next_token=self.nxt)
+
+    def capture(self, first, n_steps, events=None):
+        """A CUDA graph of steps first .. first + n_steps - 1; events[i]
+        (a pair) brackets the dominant call of step first + i."""
+        import torch
+        graph = torch.cuda.CUDAGraph()
+        cs = torch.cuda.Stream(device=self.dev)
+        cs.wait_stream(torch.cuda.current_stream(self.dev))
+        with torch.cuda.graph(graph, stream=cs):
+            for i in range(n_steps):
+                self.step(first + i, events=None if events is None else events[i])
+        return graph
+
+    def close(self):
+        self.ctx.close()
+
+
+def event_pairs(n):
+    import torch
+    return [(torch.cuda.Event(enable_timing=True, external=True),
+             torch.cuda.Event(enable_timing=True, external=True)) for _ in range(n)]
+
+
+def timed_run(r, steps, warmup, *, bracket, min_pairs=64, world=1, rank=0, sampler=None):
+    """Warm up, then time exactly `steps` steps as CUDA-graph replays between
+    two events on the launching stream (barrier + synchronize on both sides).
+    With `bracket`, every step's dominant call in the timed graphs is
+    bracketed by its own event pair; otherwise (and to reach `min_pairs`
+    pairs) a separate pass of bracketed replays follows the timed region.
+    Returns the step time, the per-call durations and how they were taken."""
+    import torch
+    import torch.distributed as dist
+    dev = r.dev
+    for i in range(warmup):
+        r.step(i)
+    r.ctx.sync()
+    G = r.gsteps
+    n_graphs = 4 if bracket else 1
+    # the timed graphs: n_graphs instances of G steps (cycled), and the rest
+    ev_main = [event_pairs(G) if bracket else None for _ in range(n_graphs)]
+    r.ctx.profile_enable(True)
+    graphs = [r.capture(0, G, ev_main[0])]
+    launches_per_step = r.ctx.profile_read()["launches"] / G
+    r.ctx.profile_enable(False)
+    graphs += [r.capture(0, G, ev_main[g]) for g in range(1, n_graphs)]
+    reps, rem = divmod(steps, G)
+    ev_rem = event_pairs(rem) if (bracket and rem) else None
+    g_rem = r.capture(0, rem, ev_rem) if rem else None
+    for g in graphs:                       # warm the graphs
+        g.replay()
+    torch.cuda.synchronize(dev)
+    stream = torch.cuda.current_stream(dev)
+    if sampler is not None:
+        time.sleep(0.3)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t_wall0 = time.time()
+    e0.record(stream)
+    for k in range(reps):
+        graphs[k % n_graphs].replay()
+    if g_rem is not None:
+        g_rem.replay()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    if world > 1:
+        dist.barrier()
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    unit = []
+    if bracket:
+        for g in range(min(n_graphs, reps)):         # each graph's last replay
+            unit += [a.elapsed_time(b) for a, b in ev_main[g]]
+        if ev_rem:
+            unit += [a.elapsed_time(b) for a, b in ev_rem]
+    n_in = len(unit)
+    extra_reps = 0
+    if len(unit) < min_pairs:
+        # a pass of bracketed replays right after the timed region
+        evx = event_pairs(G)
+        gx = r.capture(0, G, evx)
+        gx.replay()
+        while len(unit) < min_pairs:
+            gx.replay()
+            torch.cuda.synchronize(dev)
+            unit += [a.elapsed_time(b) for a, b in evx]
+            extra_reps += 1
+    how = (f"event pairs around the dominant call of every step of the timed graphs: "
+           f"the last replay of each of {min(n_graphs, reps) + (1 if ev_rem else 0)} "
+           f"graph(s), {n_in} calls" if n_in else "")
+    if extra_reps:
+        how += ((" + " if n_in else "") + f"{len(unit) - n_in} calls in {extra_reps} "
+                f"bracketed replays of a {G}-step graph right after the timed region")
+    return dict(ms=ms, unit=unit, timing=how, launches_per_step=launches_per_step,
+                t_wall=(t_wall0, t_wall1), reps=reps, rem=rem, G=G, n_graphs=n_graphs)
+
+
+def e2e_run(r, steps, world=1):
+    """The step through the public API with host buffers: pinned h in,
+    tokens out, synchronised every step."""
+    import torch
+    import torch.distributed as dist
+    dev, w = r.dev, r.w
+    h_host = [x.cpu().pin_memory() for x in r.hs]
+    tok_host = torch.empty(w.rows, dtype=torch.int32).pin_memory()
+    h_dev = torch.empty_like(w.h)
+    for i in range(3):
+        h_dev.copy_(h_host[i % r.ncopy], non_blocking=True)
+        r.step(i, h_dev)
+        tok_host.copy_(r.tokens, non_blocking=True)
+        torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for i in range(steps):
+        h_dev.copy_(h_host[i % r.ncopy], non_blocking=True)
+        r.step(i, h_dev)
+        tok_host.copy_(r.tokens, non_blocking=True)
+        torch.cuda.synchronize(dev)
+    dt = max_over_ranks(time.perf_counter() - t0, dev)
+    return {"value": round(w.rows * world * steps / dt, 1), "unit": UNIT,
+            "h2d_bytes_per_step": w.rows * w.d * 4, "d2h_bytes_per_step": w.rows * 4,
+            "steps": steps,
+            "note": ("pinned host h -> device, direct C-ABI calls (no graph), "
+                     "tokens -> host, sync per step")}
+
+
+def unit_stats(unit):
+    return {"mean_ms": round(statistics.mean(unit), 5), "min_ms": round(min(unit), 5),
+            "max_ms": round(max(unit), 5), "pairs": len(unit)}
+
+
+# sub-configurations timed beside the headline (name, rows, keep, d_l, act)
+CONFIG_BLOCK = [("tiny", None, None, None, "fp32"),
+                ("decode", None, None, None, "fp32"), ("decode", None, None, None, "bf16"),
+                ("spec", None, None, None, "fp32"), ("spec", None, None, None, "bf16"),
+                ("fp8", None, None, None, "fp32"), ("fp8", None, None, None, "bf16"),
+                ("sweep", 1, 1.0, None, "fp32"), ("sweep", 8, 1.0, None, "fp32"),
+                ("sweep", 64, 1.0, None, "fp32"), ("sweep", 256, 1.0, None, "fp32"),
+                ("sweep", 1024, 1.0, None, "bf16"),
+                ("dend", None, 0.4, 96, "fp32")]
+DEND_GRID = [(k, d) for k in (0.4, 0.3) for d in (48, 96, 128, 256, 512)]
+
+
+def config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks, cpu_seconds,
+                 target_s=0.3, e2e_steps=50, with_cpu=True):
+    """One line of the per-configuration block: its own step rate, cloud-call
+    time and roofline, end-to-end rate and oracle baseline."""
+    import torch
+    w = wl.workload(name, device=dev, rows=rows, keep_frac=keep, d_l=d_l)
+    r = Runner(sph, wl, w, dev, act)
+    try:
+        # steps for about target_s of timed work, from one timed warm-up graph
+        for i in range(3):
+            r.step(i)
+        torch.cuda.synchronize(dev)
+        t = time.perf_counter()
+        for i in range(r.gsteps):
+            r.step(i)
+        torch.cuda.synchronize(dev)
+        est = (time.perf_counter() - t) / r.gsteps
+        steps = int(min(20000, max(2 * r.gsteps, target_s / max(est, 1e-6))))
+        steps = steps // r.gsteps * r.gsteps
+        res = timed_run(r, steps, 3, bracket=False, min_pairs=64)
+        unit = unit_stats(res["unit"])
+        roof = roofline(w, act, unit["mean_ms"], peaks)
+        roof["timing"] = res["timing"]
+        roof["spread"] = unit
+        entry = {"workload": describe(w), "activations": act,
+                 "rows_per_s": round(job_rows_per_s(w.rows, 1, steps, res["ms"]), 1),
+                 "ms_per_step": round(res["ms"] / steps, 5), "steps": steps,
+                 "cloud_us": round(unit["mean_ms"] * 1e3, 2),
+                 "roofline": roof,
+                 "e2e_rows_per_s": e2e_run(r, e2e_steps)["value"],
+                 "payload_bytes_per_step": sph.sph_payload_bytes(w.rows, w.n_keep),
+                 "gpu_launches_per_step": round(res["launches_per_step"], 2)}
+        if with_cpu:
+            entry["cpu_baseline"] = cpu_baseline(w, cpu_seconds, act)
+        return entry
+    finally:
+        r.close()
+        del r, w
+        torch.cuda.empty_cache()
 
 
 def run_ours(args):
@@ -319,105 +632,8 @@ def run_ours(args):
         g.manual_seed(rank_seed(rank))
         w.h = wl.make_hidden(w.rows, w.d, g, dev)
     R, n = w.rows, w.n_keep
-    ctx = sph.Context(local)
-    act_mode = sph.SPH_ACT_BF16 if args.act == "bf16" else sph.SPH_ACT_FP32
-    if args.sampler == "gumbel":
-        ctx.set_option(sph.SPH_OPT_SAMPLER, sph.SPH_SAMPLER_GUMBEL)
-    nosplit = args.nosplit
-    if nosplit and w.w_dtype != "bf16":
-        raise SystemExit("--nosplit needs bf16 weights (the endpoint head is bf16)")
-    ctx.reserve(R, n, w.d if nosplit else max(w.d_h, w.d_l))
+    r = Runner(sph, wl, w, dev, args.act, args.nosplit, args.sampler)
 
-    # rotation so that bytes between reuses exceed 2x L2
-    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    wb = 1 if w.w_dtype == "fp8" else 2
-    per_copy = n * w.d_h * wb + n * w.d_l * 2
-    ncopy = max(1, math.ceil(2 * l2 / per_copy) + 1) if per_copy < 2 * l2 else 1
-    if nosplit:
-        # the whole head [V, d] in one tensor (the no-split ablation)
-        Wfs = [torch.cat([w.W_l, w.W_h], dim=1).contiguous()]
-        Wfs += [Wfs[0].clone() for _ in range(ncopy - 1)]
-        Whs = Wls = [None] * ncopy
-    else:
-        Whs = [w.W_h] + [w.W_h.clone() for _ in range(ncopy - 1)]
-        Wls = [w.W_l] + [w.W_l.clone() for _ in range(ncopy - 1)]
-    hs = [w.h] + [w.h.roll(i + 1, dims=0).contiguous() for i in range(ncopy - 1)]
-    codes = torch.empty(R, n, dtype=torch.int8, device=dev)
-    scale = torch.empty(R, dtype=torch.float32, device=dev)
-    tokens = torch.empty(R, dtype=torch.int32, device=dev)
-    z = torch.empty(R, n, device=dev) if w.sessions else None
-    n_acc = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
-    nxt = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
-
-    def step(i, h=None, events=None):
-        c = i % ncopy
-        hh = hs[c] if h is None else h
-        if nosplit:                     # one endpoint call over the whole head
-            if events is not None:
-                events[0].record()
-            ctx.fuse_sample(None, None, hh, Wfs[c], keep_ids=w.keep_ids,
-                            temperature=w.tau, seed=w.seed, offset=i, tokens=tokens,
-                            fused_logits_out=z)
-            if events is not None:
-                events[1].record()
-            if w.sessions:
-                ctx.verify_draft(z, w.sessions, w.k, w.draft_tokens, keep_ids=w.keep_ids,
-                                 draft_probs=w.draft_probs, temperature=w.tau,
-                                 seed=w.seed, offset=i, n_accepted=n_acc, next_token=nxt)
-            return
-        if events is not None:
-            events[0].record()
-        ctx.partial_logits(hh[:, w.d_l:], Whs[c], keep_ids=w.keep_ids, clip=w.clip,
-                           w_row_scale=w.w_scale, bias=w.bias, codes=codes,
-                           row_scale=scale, act_mode=act_mode)
-        if events is not None:
-            events[1].record()
-        ctx.fuse_sample(codes, scale, hh[:, :w.d_l], Wls[c], keep_ids=w.keep_ids,
-                        temperature=w.tau, seed=w.seed, offset=i, tokens=tokens,
-                        fused_logits_out=z)
-        if w.sessions:
-            ctx.verify_draft(z, w.sessions, w.k, w.draft_tokens, keep_ids=w.keep_ids,
-                             draft_probs=w.draft_probs, temperature=w.tau,
-                             seed=w.seed, offset=i, n_accepted=n_acc, next_token=nxt)
-
-    for i in range(args.warmup):
-        step(i)
-    ctx.sync()
-
-    # ---- the timed loop is a CUDA graph: gsteps steps cycling the weight
-    # copies.  Two of its cloud calls are bracketed by event-record nodes
-    # (an event node between two kernels cuts their programmatic-launch
-    # overlap, so bracketing every call would slow the step it times)
-    gsteps = ncopy * max(1, math.ceil(16 / ncopy))
-    ev_steps = sorted({0, gsteps // 2})
-    try:
-        evs = {i: (torch.cuda.Event(enable_timing=True, external=True),
-                   torch.cuda.Event(enable_timing=True, external=True))
-               for i in ev_steps}
-    except TypeError:                       # torch without external events
-        evs = None
-
-    def capture(n_steps, with_events):
-        graph = torch.cuda.CUDAGraph()
-        cs = torch.cuda.Stream(device=dev)
-        cs.wait_stream(torch.cuda.current_stream(dev))
-        with torch.cuda.graph(graph, stream=cs):
-            for i in range(n_steps):
-                step(i, events=evs.get(i) if (with_events and evs) else None)
-        return graph
-
-    ctx.profile_enable(True)
-    g_main = capture(gsteps, True)
-    launches_per_step = ctx.profile_read()["launches"] / gsteps
-    ctx.profile_enable(False)
-    rem = args.steps % gsteps
-    g_rem = capture(rem, False) if rem else None
-    reps = args.steps // gsteps
-    for _ in range(2):                      # warm the graphs
-        g_main.replay()
-    torch.cuda.synchronize(dev)
-
-    stream = torch.cuda.current_stream(dev)
     gpu_uuid = None
     try:
         gpu_uuid = str(torch.cuda.get_device_properties(dev).uuid)
@@ -425,88 +641,37 @@ def run_ours(args):
             gpu_uuid = "GPU-" + gpu_uuid
     except Exception:
         pass
-    sampler = ClockSampler(gpu_uuid) if rank == 0 else None
-    time.sleep(0.3 if sampler else 0)
-    ev0 = torch.cuda.Event(enable_timing=True)
-    ev1 = torch.cuda.Event(enable_timing=True)
-    if world > 1:
-        dist.barrier()
+    clock = ClockSampler(gpu_uuid) if rank == 0 else None
+    # every dominant call of the timed region is bracketed by events when
+    # it is long enough that the event nodes cost nothing measurable; short
+    # calls are timed in a bracketed pass right after the timed region
+    for i in range(2):
+        r.step(i)
     torch.cuda.synchronize(dev)
-    t_wall0 = time.time()
-    ev0.record(stream)
-    for _ in range(reps):
-        g_main.replay()
-    if g_rem is not None:
-        g_rem.replay()
-    ev1.record(stream)
+    t = time.perf_counter()
+    for i in range(4):
+        r.step(i)
     torch.cuda.synchronize(dev)
-    t_wall1 = time.time()
-    if world > 1:
-        dist.barrier()
-    ms = max_over_ranks(ev0.elapsed_time(ev1), dev)
+    bracket = (time.perf_counter() - t) / 4 > 1e-3
+    res = timed_run(r, args.steps, args.warmup, bracket=bracket, min_pairs=64,
+                    world=world, rank=rank, sampler=clock)
+    ms = res["ms"]
     clocks = None
-    if sampler:
+    if clock:
         time.sleep(0.2)
-        sampler.stop()
-        clocks = sampler.summary(t_wall0, t_wall1)
-    # duration of the cloud call: its event pairs in the last replay of the
-    # timed loop (or, without external events, a graph of cloud calls alone)
-    if evs is not None and reps > 0:
-        cloud_ms = statistics.mean(a.elapsed_time(b) for a, b in evs.values())
-        cloud_src = (f"event nodes around cloud calls {ev_steps} of the {gsteps}-step graph, "
-                     "last timed replay")
-    else:
-        gc = torch.cuda.CUDAGraph()
-        cs = torch.cuda.Stream(device=dev)
-        cs.wait_stream(torch.cuda.current_stream(dev))
-        with torch.cuda.graph(gc, stream=cs):
-            for i in range(gsteps):
-                c = i % ncopy
-                if nosplit:
-                    ctx.fuse_sample(None, None, hs[c], Wfs[c], keep_ids=w.keep_ids,
-                                    temperature=w.tau, seed=w.seed, offset=i, tokens=tokens)
-                    continue
-                ctx.partial_logits(hs[c][:, w.d_l:], Whs[c], keep_ids=w.keep_ids,
-                                   clip=w.clip, w_row_scale=w.w_scale, bias=w.bias,
-                                   codes=codes, row_scale=scale, act_mode=act_mode)
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        gc.replay()
-        a.record(stream)
-        for _ in range(10):
-            gc.replay()
-        b.record(stream)
-        torch.cuda.synchronize(dev)
-        cloud_ms = a.elapsed_time(b) / (10 * gsteps)
-        cloud_src = "graph of cloud calls replayed alone"
-    ctx.profile_enable(True)                 # per-class split, direct launches
-    for i in range(min(50, args.steps)):
-        step(i)
-    prof = ctx.profile_read()
-    ctx.profile_enable(False)
+        clock.stop()
+        clocks = clock.summary(*res["t_wall"])
+    # per-class split, direct launches with tracing events
+    r.ctx.profile_enable(True)
     nprof = max(1, min(50, args.steps))
-
-    # ---- end to end: host buffers in, tokens out, every step -------------
-    e2e_steps = min(args.e2e_steps, args.steps)
-    h_host = [x.cpu().pin_memory() for x in hs]
-    tok_host = torch.empty(R, dtype=torch.int32).pin_memory()
-    h_dev = torch.empty_like(w.h)
-    for i in range(3):
-        h_dev.copy_(h_host[i % ncopy], non_blocking=True)
-        step(i, h_dev)
-        tok_host.copy_(tokens, non_blocking=True)
-        torch.cuda.synchronize(dev)
-    if world > 1:
-        dist.barrier()
-    t0 = time.perf_counter()
-    for i in range(e2e_steps):
-        h_dev.copy_(h_host[i % ncopy], non_blocking=True)
-        step(i, h_dev)
-        tok_host.copy_(tokens, non_blocking=True)
-        torch.cuda.synchronize(dev)
-    e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
+    for i in range(nprof):
+        r.step(i)
+    prof = r.ctx.profile_read()
+    r.ctx.profile_enable(False)
+    e2e = e2e_run(r, min(args.e2e_steps, max(args.steps, 20)), world)
 
     if rank != 0:
+        r.close()
         if world > 1:
             dist.barrier()
             dist.destroy_process_group()
@@ -514,35 +679,17 @@ def run_ours(args):
 
     peaks, peaks_src = load_peaks()
     value = job_rows_per_s(R, world, args.steps, ms)
-    # dominant unit: the cloud call (operand split + gathered contraction +
-    # quantization), timed inside the timed graph
-    if nosplit:
-        # the whole head's kept rows, the whole h, the ids and the tokens
-        alg_bytes = n * w.d * 2 + 4 * R * w.d + 4 * n + 4 * R
-        alg_flops = wl.algorithmic_flops(R, n, w.d)
-    else:
-        alg_bytes = wl.algorithmic_bytes_cloud(R, n, w.d_h, wb, fp8_scales=w.w_dtype == "fp8")
-        alg_flops = wl.algorithmic_flops(R, n, w.d_h)
-    ai = alg_flops / alg_bytes
-    ridge = peaks["bf16_tflops_sustained"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
-    files = ["paper_2607_13093_gb300/csrc/k_tc.cu", "paper_2607_13093_gb300/csrc/k_gemv.cu",
-             "paper_2607_13093_gb300/csrc/k_finish.cu"]
-    if ai < ridge:
-        achieved = alg_bytes / (cloud_ms / 1e3) / 1e9
-        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
-                "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4)}
-    else:
-        achieved = alg_flops / (cloud_ms / 1e3) / 1e12
-        pk = peaks["bf16_tflops_sustained"]
-        roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": pk,
-                "unit": "TFLOP/s", "frac": round(achieved / pk, 4)}
-    roof.update({"traffic": None if nosplit else traffic_for(f"cloud_{args.workload}", files),
+    unit = unit_stats(res["unit"])
+    roof = roofline(w, args.act, unit["mean_ms"], peaks, args.nosplit)
+    roof.update({"traffic": None if args.nosplit else traffic_for(
+                     f"cloud_{args.workload}_{R}_{n}_{args.act}"),
                  "kernel": ("unsplit head: gathered whole-d contraction + sample (one endpoint "
-                            "call without payload)" if nosplit else
-                            "cloud call: gathered partial logits + int8 quantization"),
-                 "algorithmic_bytes": alg_bytes, "algorithmic_flops": alg_flops,
-                 "avg_launch_ms": round(cloud_ms, 5), "timing": cloud_src,
-                 "peak_source": f"{peaks_src} (MEASURED_PEAKS.json)" if peaks_src == "measured" else "fallback"})
+                            "call without payload)" if args.nosplit else
+                            "cloud call: operand split + gathered tcgen05 contraction + int8 "
+                            "quantization"),
+                 "timing": res["timing"], "spread": unit,
+                 "peak_source": ("measured (MEASURED_PEAKS.json)" if peaks_src == "measured"
+                                 else "fallback")})
     steps_ms = {k: round(v / nprof, 5) for k, v in prof["ms"].items() if v}
     out = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
@@ -551,41 +698,57 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None,
         "dtype": "f32" if args.act == "fp32" else "bf16",
         "data": "synthetic (seeded, paper shapes; weights N(0,0.02) bf16, h RMS-normalised)",
-        "config": {"workload": describe(w) + (", unsplit head (no-split ablation)" if nosplit else ""),
+        "config": {"workload": describe(w) + (", unsplit head (no-split ablation)"
+                                              if args.nosplit else ""),
                    "rows_per_gpu": R, "n_keep": n,
                    "d_h": w.d_h, "d_l": w.d_l, "V": w.V, "weights": w.w_dtype,
                    "accumulate": "fp32",
                    "sampler": "Gumbel-max" if args.sampler == "gumbel" else "inverse CDF",
                    "activations": ("fp32 (exact: bf16 hi + lo planes)" if args.act == "fp32"
                                    else "bf16-rounded (one plane)"),
-                   "l2": (f"inputs rotate over {ncopy} weight/h copies, "
-                          f"{ncopy * per_copy / 1e6:.0f} MB touched per cycle vs L2 "
-                          f"{l2 / 1e6:.0f} MB"),
+                   "l2": (f"inputs rotate over {r.ncopy} weight/h copies, "
+                          f"{r.ncopy * r.per_copy / 1e6:.0f} MB touched per cycle vs L2 "
+                          f"{r.l2 / 1e6:.0f} MB (inputs larger than L2, no flush)"),
                    "parallelism": f"replicas x{world} (independent sessions per GPU)"},
         "breakdown_ms_per_step": steps_ms,
         "breakdown_note": "per kernel class, direct (non-graph) launches with tracing events",
         "roofline": roof,
-        "gpu_launches": int(round(launches_per_step * args.steps)),
-        "e2e": {"value": round(R * world * e2e_steps / e2e_s, 1), "unit": UNIT,
-                "h2d_bytes_per_step": R * w.d * 4, "d2h_bytes_per_step": R * 4,
-                "note": ("pinned host h -> device, direct C-ABI calls (no graph), "
-                         "tokens -> host, sync per step")},
-        "timed_loop": f"CUDA graph of {gsteps} steps replayed {reps}x (+{rem} steps)",
+        "gpu_launches": int(round(res["launches_per_step"] * args.steps)),
+        "e2e": e2e,
+        "timed_loop": (f"{res['n_graphs']} CUDA graph(s) of {res['G']} steps replayed "
+                       f"{res['reps']}x in turn (+{res['rem']} steps)"),
         "clocks": clocks,
         # downlink of one step (Eq. 21 with b = 8, no tag/metadata/padding):
         # int8 codes of the kept ids + an fp32 scale per row, against the full
         # vocabulary as int8 and as fp32 logits
-        "payload": {"bytes_per_step": (4 * R * n if nosplit else sph.sph_payload_bytes(R, n)),
+        "payload": {"bytes_per_step": (4 * R * n if args.nosplit else sph.sph_payload_bytes(R, n)),
                     "what": ("fp32 logits of the kept ids, which an unsplit cloud head would send"
-                             if nosplit else "int8 codes of the kept ids + an fp32 scale per row"),
+                             if args.nosplit else "int8 codes of the kept ids + an fp32 scale per row"),
                     "full_vocab_int8_bytes": sph.sph_payload_bytes(R, w.V),
                     "full_vocab_fp32_bytes": 4 * R * w.V,
                     "reduction_vs_full_int8": round(
                         1 - sph.sph_payload_bytes(R, n) / sph.sph_payload_bytes(R, w.V), 4)},
     }
+    r.close()
+    del r
+    torch.cuda.empty_cache()
     if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act, args.nosplit,
                                            args.sampler)
+    del w
+    torch.cuda.empty_cache()
+    if world == 1 and not args.no_configs and not args.nosplit:
+        block = list(CONFIG_BLOCK) + ([("dend", None, k, d, "fp32") for k, d in DEND_GRID]
+                                      if args.dend_grid else [])
+        entries = []
+        for (name, rows, keep, d_l, act) in block:
+            if (name, rows, keep, d_l, act) == (args.workload, args.rows, args.keep,
+                                                args.d_l, args.act):
+                continue
+            with_cpu = not args.no_cpu_baseline and (name != "dend" or (keep, d_l) == (0.4, 96))
+            entries.append(config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks,
+                                        args.config_cpu_seconds, with_cpu=with_cpu))
+        out["configs"] = entries
     print(json.dumps(out), flush=True)
     if world > 1:
         dist.barrier()
@@ -634,6 +797,8 @@ def run_reference(args):
 
 def main():
     args = parse()
+    if args.workload == "sweep" and args.rows is None and args.keep is None:
+        args.rows, args.keep = 1024, 1.0       # the headline: the largest workload
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -134,6 +134,14 @@ typedef enum sph_option {
                                2^15, >= 0; 0: no finisher, the last
                                contributor to count in finishes the tile).
                                Results are bit-identical for every value.   */
+  SPH_OPT_CHECK_IDS = 9,    /* 1: before launching anything, every hot-path
+                               call copies keep_ids to the host (a
+                               synchronous copy on the context's stream; not
+                               allowed while the stream is being captured)
+                               and checks them with sph_check_keep_ids,
+                               returning SPH_ERR_INVALID_ARG for unsorted,
+                               repeated or out-of-range ids.  0 (default):
+                               the ids are a precondition, not checked.    */
   SPH_OPT_SAMPLER = 8       /* the draw of sph_fuse_sample at temperature > 0:
                                0 inverse CDF (default), 1 Gumbel-max: the
                                first index j of the largest
@@ -197,6 +205,35 @@ size_t sph_payload_bytes(int64_t rows, int64_t n_keep);
 sph_status sph_keep_ids_from_mask(const uint8_t* mask, int64_t V,
                                   int32_t* keep_ids, int64_t* n_keep);
 
+/* Check a HOST copy of a kept-id list against the conventions above:
+ * strictly increasing, each in [0, V).  Returns SPH_OK, or
+ * SPH_ERR_INVALID_ARG (NULL with n_keep > 0, n_keep < 1, V < 1, or a bad
+ * id); *bad_index (if not NULL) receives the first offending position, or
+ * -1.  The same check SPH_OPT_CHECK_IDS applies to device lists. */
+sph_status sph_check_keep_ids(const int32_t* keep_ids, int64_t n_keep,
+                              int64_t V, int64_t* bad_index);
+
+/* The work split a context would choose for one call, without launching
+ * anything (for tests and tuning).  `call`: 0 cloud (sph_partial_logits,
+ * K = d_h), 1 endpoint (sph_fuse_sample, K = d_l).  gather: 1 for a kept-id
+ * subset, 0 for the full vocabulary. */
+typedef struct sph_plan {
+  int32_t tensor_core;      /* 1: tcgen05 kernel; 0: CUDA-core GEMV        */
+  int32_t row_blocks;       /* hidden-state row blocks (tensor core)       */
+  int32_t block_rows;       /* rows per row block (a multiple of 16)       */
+  int32_t tile_ids;         /* kept ids per vocabulary tile: 128 or 256    */
+  int32_t tiles;            /* row blocks x vocabulary tiles               */
+  int32_t k_blocks;         /* pipeline stages per tile (hidden dimension) */
+  int32_t stages;           /* shared-memory pipeline depth                */
+  int32_t grid;             /* persistent CTAs                             */
+  int32_t whole_tiles;      /* 1: whole tiles per CTA; 0: stream-K ranges  */
+  int32_t planes;           /* hidden-state operand planes (bf16 or e4m3)  */
+  int32_t gemv_rows;        /* GEMV: rows per launch (1, 2, 4 or 8)        */
+} sph_plan;
+sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep,
+                          int64_t K, sph_dtype w_dtype, sph_act_mode act_mode,
+                          int gather, sph_plan* out);
+
 /* ---- the hot path ------------------------------------------------------ */
 
 /* Cloud call (Eq. 12 over V_l, "after clipping, quantization" in Sec.
@@ -244,11 +281,12 @@ sph_status sph_partial_logits(sph_ctx* ctx,
  * by another runtime, a fixed-size memory pool, or a serving loop that must
  * never call cudaMalloc, which can synchronise the device).  Such callers
  * cannot create a context, so this call takes the device and stream
- * directly and allocates nothing: no cudaMalloc, no cudaFree, no allocating
- * library routine.  Its scratch (clipped fp32 partials and per-row maxima)
- * lives in one fixed device array of SPH_NOALLOC_SCRATCH_BYTES inside the
- * library, which every GPU that loads the library holds until the process
- * exits.
+ * directly and, once set up on a device (see the first call below),
+ * allocates nothing: no cudaMalloc, no cudaFree, no allocating library
+ * routine.  Its scratch (clipped fp32 partials and per-row maxima) lives in
+ * one fixed device array of SPH_NOALLOC_SCRATCH_BYTES inside the library,
+ * which every GPU that has loaded the library's modules holds until the
+ * process exits.
  *   - Same arguments, results and errors as sph_partial_logits, plus
  *     `device` (made current for the call), `cuda_stream` (a cudaStream_t,
  *     NULL = legacy default stream) and an optional host buffer err_msg of
@@ -256,9 +294,17 @@ sph_status sph_partial_logits(sph_ctx* ctx,
  *   - Size limit: round_up(rows*n_keep*4, 256) + round_up(rows*4, 256) must
  *     not exceed SPH_NOALLOC_SCRATCH_BYTES; larger calls return
  *     SPH_ERR_UNSUPPORTED without launching anything.
- *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress, with that device current); make that first call
- *     before any stream capture.
+ *   - rows is at most 2^20 (INVALID_ARG beyond), as for sph_partial_logits.
+ *   - The call always runs the CUDA-core GEMV, which re-reads the kept W
+ *     rows once per 8 hidden-state rows: it is meant for few rows.
+ *   - The first call on a device is a set-up call: it looks up the array's
+ *     device address (cudaGetSymbolAddress, with that device current), and
+ *     under CUDA's lazy module loading (the default) it is also the moment
+ *     the library's modules -- the array among them -- are loaded onto that
+ *     device, which allocates device memory and may synchronise.  Make one
+ *     warm-up call per device before entering the region where nothing may
+ *     allocate, and before any stream capture.  Later calls allocate
+ *     nothing.
  *   - All calls share the one array and it keeps the last call's contents
  *     (the row maxima are cleared by each call).  Calls whose kernels overlap
  *     on the GPU -- on different streams or from different host threads --

@@ -228,18 +228,29 @@ cudaError_t launch_rt(const GatherGemm& g, int sm_count, cudaStream_t st) {
   return cudaSuccess;
 }
 
+// hidden-state rows one launch covers: as many of 8, 4, 2 as the rows and
+// the shared-memory tile allow
+int rows_per_launch(int rows, int K) {
+  const size_t per_row = (size_t)((K + 7) & ~7) * sizeof(float);
+  for (int rt = 8; rt > 1; rt >>= 1)
+    if (rows >= rt && rt * per_row <= kSmemLimit) return rt;
+  return 1;
+}
+
 template <int WDT, int EPI>
 cudaError_t launch_wdt(const GatherGemm& g, int sm_count, cudaStream_t st) {
-  const size_t per_row = (size_t)((g.K + 7) & ~7) * sizeof(float);
-  if (g.rows >= 8 && 8 * per_row <= kSmemLimit) return launch_rt<8, WDT, EPI>(g, sm_count, st);
-  if (g.rows >= 4 && 4 * per_row <= kSmemLimit) return launch_rt<4, WDT, EPI>(g, sm_count, st);
-  if (g.rows >= 2 && 2 * per_row <= kSmemLimit) return launch_rt<2, WDT, EPI>(g, sm_count, st);
+  switch (rows_per_launch(g.rows, g.K)) {
+    case 8: return launch_rt<8, WDT, EPI>(g, sm_count, st);
+    case 4: return launch_rt<4, WDT, EPI>(g, sm_count, st);
+    case 2: return launch_rt<2, WDT, EPI>(g, sm_count, st);
+  }
   return launch_rt<1, WDT, EPI>(g, sm_count, st);
 }
 
 }  // namespace
 
 int gemv_max_k() { return (int)(kSmemLimit / sizeof(float)) & ~7; }
+int gemv_rows_per_launch(int rows, int K) { return rows_per_launch(rows, K); }
 
 cudaError_t launch_gemv(const GatherGemm& g, int sm_count, cudaStream_t st) {
   if (g.w_dtype == W_BF16)

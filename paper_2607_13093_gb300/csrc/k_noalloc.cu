@@ -12,9 +12,18 @@
 // every input and output buffer.
 //
 // The array costs kNoallocBytes of device memory on every GPU that loads
-// the library, until the process exits.  All calls share it: two calls
-// whose kernels overlap on the GPU (different streams, or different host
-// threads) corrupt each other's results, so such callers must serialise.
+// the library's module, until the process exits.  With CUDA's lazy module
+// loading (the default), a module -- this array included -- is loaded onto a
+// device the first time one of its kernels or symbols is used there, so the
+// FIRST call on each device does allocate device memory (and may
+// synchronise): callers make one warm-up call before they enter the region
+// where nothing may allocate.  Every later call allocates nothing.  All
+// calls share the array: two calls whose kernels overlap on the GPU
+// (different streams, or different host threads) corrupt each other's
+// results, so such callers must serialise.
+//
+// The call always takes the CUDA-core GEMV path, which re-reads the kept W
+// rows once per 8 hidden-state rows: it is meant for few rows.
 #include <cmath>
 #include <cstdio>
 #include <mutex>
@@ -58,7 +67,11 @@ extern "C" sph_status sph_partial_logits_noalloc(
     put(err_msg, err_msg_len, "h_cloud, W_h, codes and row_scale must be non-NULL");
     return SPH_ERR_INVALID_ARG;
   }
-  if (rows < 1 || d_h < 1 || V < 1 || V > INT32_MAX || n_keep < 1 || n_keep > V ||
+  if (rows < 1 || rows > (1 << 20)) {
+    put(err_msg, err_msg_len, "rows out of [1, 2^20]");
+    return SPH_ERR_INVALID_ARG;
+  }
+  if (d_h < 1 || V < 1 || V > INT32_MAX || n_keep < 1 || n_keep > V ||
       ld_h < d_h || ld_w < d_h || (!keep_ids && n_keep != V)) {
     put(err_msg, err_msg_len, "inconsistent sizes (rows, d_h, V, n_keep, ld_h, ld_w)");
     return SPH_ERR_INVALID_ARG;
@@ -96,7 +109,11 @@ extern "C" sph_status sph_partial_logits_noalloc(
   if (payload_bytes) *payload_bytes = sph_payload_bytes(rows, n_keep);
 
   int prev = -1;
-  if (cudaGetDevice(&prev) != cudaSuccess) return SPH_ERR_CUDA;
+  const cudaError_t ge = cudaGetDevice(&prev);
+  if (ge != cudaSuccess) {
+    put(err_msg, err_msg_len, cudaGetErrorString(ge));
+    return SPH_ERR_CUDA;
+  }
   if (prev != device && cudaSetDevice(device) != cudaSuccess) {
     put(err_msg, err_msg_len, "cudaSetDevice failed");
     return SPH_ERR_CUDA;

@@ -185,13 +185,6 @@ __device__ __forceinline__ int ld_acquire_gpu(const int* p) {
 namespace sph {
 namespace ptx {
 
-
-}  // namespace ptx
-}  // namespace sph
-
-namespace sph {
-namespace ptx {
-
 // ---- programmatic dependent launch ------------------------------------------
 // Block until the grids this one depends on have completed and their memory
 // is visible (a no-op when launched without a programmatic dependency).

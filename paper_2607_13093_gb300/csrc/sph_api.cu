@@ -37,6 +37,7 @@ struct sph_ctx {
   int tc_tile_m = 0;                // SPH_OPT_TC_TILE_M
   long long tc_finish_wait = 1ll << 15;   // SPH_OPT_TC_FINISH_WAIT
   int sampler = 0;                  // SPH_OPT_SAMPLER
+  int check_ids = 0;                // SPH_OPT_CHECK_IDS
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -186,6 +187,29 @@ sph_status check_ids(sph_ctx* ctx, const int32_t* keep_ids, int64_t n_keep,
   return SPH_OK;
 }
 
+// SPH_OPT_CHECK_IDS: copy the device id list to the host and check it
+// before anything is launched.  V < 0: the upper bound is not known (the
+// verification call), only order and sign are checked.
+sph_status host_check_ids(sph_ctx* ctx, const int32_t* keep_ids, int64_t n_keep, int64_t V) {
+  if (!ctx->check_ids || !keep_ids) return SPH_OK;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(ctx->stream, &cap) == cudaSuccess &&
+      cap != cudaStreamCaptureStatusNone)
+    return fail(ctx, SPH_ERR_UNSUPPORTED,
+                "SPH_OPT_CHECK_IDS copies the ids to the host: not allowed during stream capture");
+  std::vector<int32_t> ids((size_t)n_keep);
+  cudaError_t e = cudaMemcpyAsync(ids.data(), keep_ids, (size_t)n_keep * 4,
+                                  cudaMemcpyDeviceToHost, ctx->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "copying keep_ids to the host");
+  int64_t bad = -1;
+  if (sph_check_keep_ids(ids.data(), n_keep, V < 0 ? (int64_t)INT32_MAX + 1 : V, &bad) != SPH_OK)
+    return fail(ctx, SPH_ERR_INVALID_ARG,
+                "keep_ids[%lld] = %d breaks the id conventions (strictly increasing, in [0, V))",
+                (long long)bad, bad >= 0 ? ids[(size_t)bad] : 0);
+  return SPH_OK;
+}
+
 sph_status launch_status(sph_ctx* ctx, cudaError_t e, const char* what) {
   if (e != cudaSuccess) return cuda_fail(ctx, e, what);
   return SPH_OK;
@@ -253,6 +277,56 @@ sph_status sph_keep_ids_from_mask(const uint8_t* mask, int64_t V,
     if (mask[v >> 3] & (1u << (v & 7))) keep_ids[n++] = (int32_t)v;
   *n_keep = n;
   return n ? SPH_OK : SPH_ERR_INVALID_ARG;
+}
+
+sph_status sph_check_keep_ids(const int32_t* keep_ids, int64_t n_keep, int64_t V,
+                              int64_t* bad_index) {
+  if (bad_index) *bad_index = -1;
+  if (!keep_ids || n_keep < 1 || V < 1) return SPH_ERR_INVALID_ARG;
+  int64_t prev = -1;
+  for (int64_t j = 0; j < n_keep; ++j) {
+    const int64_t id = keep_ids[j];
+    if (id <= prev || id >= V) {
+      if (bad_index) *bad_index = j;
+      return SPH_ERR_INVALID_ARG;
+    }
+    prev = id;
+  }
+  return SPH_OK;
+}
+
+sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep, int64_t K,
+                          sph_dtype w_dtype, sph_act_mode act_mode, int gather,
+                          sph_plan* out) {
+  if (!ctx || !out) return SPH_ERR_INVALID_ARG;
+  if ((call != 0 && call != 1) || rows < 1 || rows > (1 << 20) || n_keep < 1 ||
+      n_keep > INT32_MAX || K < 1 || K > sph::gemv_max_k() ||
+      (w_dtype != SPH_DTYPE_BF16 && w_dtype != SPH_DTYPE_FP8_E4M3) ||
+      (act_mode != SPH_ACT_FP32 && act_mode != SPH_ACT_BF16) ||
+      (call == 1 && w_dtype != SPH_DTYPE_BF16))
+    return fail(ctx, SPH_ERR_INVALID_ARG, "sph_plan_query: bad arguments");
+  *out = sph_plan{};
+  const int wdt = w_dtype == SPH_DTYPE_BF16 ? sph::W_BF16 : sph::W_FP8;
+  if (!use_tc(ctx, rows, wdt)) {
+    out->gemv_rows = sph::gemv_rows_per_launch((int)rows, (int)K);
+    return SPH_OK;
+  }
+  const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)K,
+                                      call == 0 && act_mode == SPH_ACT_BF16, ctx->sm_count,
+                                      call, ctx->tc_schedule, ctx->tc_stages, ctx->tc_block_k,
+                                      gather != 0, wdt == sph::W_FP8, ctx->tc_max_bn,
+                                      ctx->tc_tile_m);
+  out->tensor_core = 1;
+  out->row_blocks = pl.RB;
+  out->block_rows = pl.BN;
+  out->tile_ids = pl.tm;
+  out->tiles = pl.RB * pl.NT;
+  out->k_blocks = pl.KB;
+  out->stages = pl.stages;
+  out->grid = pl.G;
+  out->whole_tiles = pl.whole_tiles;
+  out->planes = pl.hilo;
+  return SPH_OK;
 }
 
 sph_status sph_create(int device, void* cuda_stream, sph_ctx** out) {
@@ -415,6 +489,10 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "sampler must be 0 or 1");
       ctx->sampler = (int)value;
       return SPH_OK;
+    case SPH_OPT_CHECK_IDS:
+      if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "check_ids must be 0 or 1");
+      ctx->check_ids = (int)value;
+      return SPH_OK;
   }
   return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
 }
@@ -479,6 +557,8 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
 
   DeviceGuard g(ctx->device);
   if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
+  st = host_check_ids(ctx, keep_ids, n_keep, V);
+  if (st) return st;
   const int wdt = w_dtype == SPH_DTYPE_BF16 ? sph::W_BF16 : sph::W_FP8;
   const int act_bf16 = act_mode == SPH_ACT_BF16;
   st = ensure_scratch(ctx, partial_scratch_bytes(ctx, rows, n_keep, d_h, act_bf16, wdt));
@@ -551,6 +631,8 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
 
   DeviceGuard g(ctx->device);
   if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
+  st = host_check_ids(ctx, keep_ids, n_keep, V);
+  if (st) return st;
   st = ensure_scratch(ctx, fuse_scratch_bytes(ctx, rows, n_keep, d_l));
   if (st) return st;
   Carve c(ctx->scratch, ctx->scratch_cap);
@@ -638,7 +720,9 @@ sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
   if (n_keep > sph::sample_max_n()) return fail(ctx, SPH_ERR_UNSUPPORTED, "n_keep above %d", sph::sample_max_n());
   DeviceGuard g(ctx->device);
   if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
-  sph_status st = ensure_scratch(
+  sph_status st = host_check_ids(ctx, keep_ids, n_keep, -1);
+  if (st) return st;
+  st = ensure_scratch(
       ctx, sph::verify_scratch_bytes((int)sessions, (int)k, (int)n_keep));
   if (st) return st;
   // without an id list the compact index is the vocabulary id itself

@@ -81,6 +81,8 @@ struct GatherGemm {
 cudaError_t launch_gemv(const GatherGemm& g, int sm_count, cudaStream_t st);
 // Largest K the GEMV supports for a given row count.
 int gemv_max_k();
+// Hidden-state rows one GEMV launch covers (1, 2, 4 or 8).
+int gemv_rows_per_launch(int rows, int K);
 
 // Tensor-core path (k_tc.cu): sizes, work split and scratch of one call.
 struct TcPlan {

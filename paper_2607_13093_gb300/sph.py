@@ -30,6 +30,7 @@ SPH_OPT_TC_SCHEDULE, SPH_OPT_TC_STAGES, SPH_OPT_TC_BLOCK_K, SPH_OPT_TC_MAX_BN = 
 SPH_OPT_TC_TILE_M = 6
 SPH_OPT_TC_FINISH_WAIT = 7
 SPH_OPT_SAMPLER = 8
+SPH_OPT_CHECK_IDS = 9
 SPH_SAMPLER_CDF, SPH_SAMPLER_GUMBEL = 0, 1
 
 _c_void_p = ctypes.c_void_p
@@ -50,6 +51,14 @@ class sph_profile(ctypes.Structure):
                 ("launches", ctypes.c_int64)]
 
 
+PLAN_FIELDS = ("tensor_core", "row_blocks", "block_rows", "tile_ids", "tiles",
+               "k_blocks", "stages", "grid", "whole_tiles", "planes", "gemv_rows")
+
+
+class sph_plan(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int32) for f in PLAN_FIELDS]
+
+
 # name -> (restype, argtypes), mirroring include/sph.h
 _SIGNATURES = {
     "sph_status_string": (ctypes.c_char_p, [_int]),
@@ -68,6 +77,9 @@ _SIGNATURES = {
     "sph_payload_bytes": (_sz, [_i64, _i64]),
     "sph_keep_ids_from_mask": (_int, [_c_void_p, _i64, _c_void_p,
                                       ctypes.POINTER(_i64)]),
+    "sph_check_keep_ids": (_int, [_c_void_p, _i64, _i64, ctypes.POINTER(_i64)]),
+    "sph_plan_query": (_int, [_c_void_p, _int, _i64, _i64, _i64, _int, _int, _int,
+                              ctypes.POINTER(sph_plan)]),
     "sph_partial_logits": (_int, [_c_void_p, _c_void_p, _i64, _i64, _c_void_p,
                                   _int, _i64, _i64, _i64, _c_void_p, _c_void_p,
                                   _c_void_p, _i64, _f32, _int, _c_void_p,
@@ -201,6 +213,28 @@ def sph_keep_ids_from_mask(mask_bits, V: int):
     return out[: n.value].copy()
 
 
+def sph_check_keep_ids(keep_ids, V: int):
+    """Host helper: check a host id list (numpy int32) against the id
+    conventions; returns (ok, first bad position or -1)."""
+    import numpy as np
+    ids = np.ascontiguousarray(keep_ids, dtype=np.int32)
+    bad = _i64(-1)
+    st = lib.sph_check_keep_ids(ids.ctypes.data_as(ctypes.c_void_p), ids.size, int(V),
+                                ctypes.byref(bad))
+    return st == SPH_OK, int(bad.value)
+
+
+def sph_plan_query(ctx, call: int, rows: int, n_keep: int, K: int, *,
+                   w_dtype=SPH_DTYPE_BF16, act_mode=SPH_ACT_FP32, gather=True) -> dict:
+    """The work split the context would choose for one call (call 0: cloud,
+    1: endpoint), without launching anything."""
+    p = sph_plan()
+    _check(ctx, lib.sph_plan_query(ctx, int(call), int(rows), int(n_keep), int(K),
+                                   int(w_dtype), int(act_mode), 1 if gather else 0,
+                                   ctypes.byref(p)))
+    return {f: int(getattr(p, f)) for f in PLAN_FIELDS}
+
+
 def sph_partial_logits(ctx, h_cloud, W_h, *, keep_ids=None, clip=30.0,
                        w_row_scale=None, bias=None, act_mode=SPH_ACT_FP32,
                        codes=None, row_scale=None, partial_out=None):
@@ -266,6 +300,22 @@ def sph_partial_logits_noalloc(h_cloud, W_h, *, codes, row_scale,
     V = W_h.shape[0]
     n = V if keep_ids is None else keep_ids.numel()
     dev = h_cloud.device.index if device is None else int(device)
+    # the kernels write codes[r * n + j], partial_out[r * n + j] and
+    # row_scale[r] densely, on `dev`: every tensor must live there and the
+    # outputs must be contiguous and of exactly these shapes
+    for t, name, shape in ((h_cloud, "h_cloud", None), (W_h, "W_h", None),
+                           (keep_ids, "keep_ids", (n,)), (w_row_scale, "w_row_scale", (V,)),
+                           (bias, "bias", (V,)), (codes, "codes", (R, n)),
+                           (row_scale, "row_scale", (R,)), (partial_out, "partial_out", (R, n))):
+        if t is None:
+            continue
+        if t.device.index != dev:
+            raise ValueError(f"{name} is on {t.device}, not on cuda:{dev}")
+        if shape is not None:
+            if tuple(t.shape) != shape:
+                raise ValueError(f"{name} must have shape {shape}, got {tuple(t.shape)}")
+            if not t.is_contiguous():
+                raise ValueError(f"{name} must be contiguous")
     if stream is None:
         stream = torch.cuda.current_stream(dev).cuda_stream
     pb = _sz(0)
@@ -346,6 +396,9 @@ class Context:
 
     def set_option(self, option: int, value: int):
         sph_set_option(self.handle, option, value)
+
+    def plan(self, call: int, rows: int, n_keep: int, K: int, **kw) -> dict:
+        return sph_plan_query(self.handle, call, rows, n_keep, K, **kw)
 
     def partial_logits(self, *a, **kw):
         self._follow_stream()

@@ -119,3 +119,26 @@ def test_oracle_imports_nothing_of_the_product():
                     continue
                 for m in mods:
                     assert m.split(".")[0] in ("numpy", "__future__"), (f, m)
+
+
+def test_check_keep_ids_against_the_conventions(sph):
+    # strictly increasing ids in [0, V): the first offending position is
+    # reported (host lists only; nothing here reaches a kernel)
+    ok = np.array([0, 3, 4, 9], np.int32)
+    assert sph.sph_check_keep_ids(ok, 10) == (True, -1)
+    assert sph.sph_check_keep_ids(ok, 9) == (False, 3)            # id == V
+    assert sph.sph_check_keep_ids([0, 3, 3, 9], 10) == (False, 2)  # repeated
+    assert sph.sph_check_keep_ids([0, 5, 4, 9], 10) == (False, 2)  # unsorted
+    assert sph.sph_check_keep_ids([-1, 5], 10) == (False, 0)       # negative
+    assert sph.sph_check_keep_ids([7], 8) == (True, -1)
+    assert not sph.sph_check_keep_ids(np.zeros(0, np.int32), 8)[0]
+    rng = np.random.default_rng(3)
+    for _ in range(20):
+        V = int(rng.integers(2, 500))
+        ids = np.sort(rng.choice(V, size=int(rng.integers(1, V)), replace=False))
+        assert sph.sph_check_keep_ids(ids, V) == (True, -1)
+        bad = ids.copy()
+        j = int(rng.integers(0, ids.size))
+        bad[j] = V + int(rng.integers(0, 3))
+        good, at = sph.sph_check_keep_ids(bad, V)
+        assert not good and at <= j

@@ -319,17 +319,53 @@ def test_verify_accepts_drafts_equal_to_target(ctx):
 # full-size workloads, sampled rows
 # ---------------------------------------------------------------------------
 
-FULL = [("tiny", None, None), ("decode", None, None), ("spec", None, None),
-        ("fp8", None, None), ("sweep", 1, 0.1), ("sweep", 64, 0.5),
-        ("sweep", 256, 1.0), ("sweep", 1024, 1.0)]
+FULL = [("tiny", None, None, "fp32"), ("decode", None, None, "fp32"),
+        ("decode", None, None, "bf16"), ("spec", None, None, "fp32"),
+        ("spec", None, None, "bf16"), ("fp8", None, None, "fp32"),
+        ("fp8", None, None, "bf16"), ("sweep", 1, 0.1, "fp32"),
+        ("sweep", 8, 1.0, "fp32"), ("sweep", 64, 0.5, "fp32"),
+        ("sweep", 256, 1.0, "fp32"), ("sweep", 1024, 1.0, "fp32"),
+        ("sweep", 1024, 1.0, "bf16")]
 
 
-@pytest.mark.parametrize("name,rows,keep", FULL,
-                         ids=[f"{n}-{r}-{k}" for n, r, k in FULL])
-def test_full_size_sampled_rows(ctx, name, rows, keep):
+def rows_to_check(ctx, w, act, want=16):
+    """Rows of a full-size launch to compare with the oracle: every row when
+    there are at most 32, else at least `want`, with at least two from every
+    row block of the cloud and the endpoint plans (the block's last row and
+    one at an offset that moves with the block, so that different 16-row
+    epilogue chunks and lanes are hit), plus rows spread evenly."""
+    from paper_2607_13093_gb300 import sph
+    R = w.rows
+    if R <= 32:
+        return list(range(R))
+    gather = w.keep_ids is not None
+    wdt = sph.SPH_DTYPE_FP8_E4M3 if w.w_dtype == "fp8" else sph.SPH_DTYPE_BF16
+    plans = [ctx.plan(0, R, w.n_keep, w.d_h, w_dtype=wdt, gather=gather,
+                      act_mode=sph.SPH_ACT_BF16 if act == "bf16" else sph.SPH_ACT_FP32),
+             ctx.plan(1, R, w.n_keep, w.d_l, gather=gather)]
+    sel = {0, R - 1}
+    for p in plans:
+        if not p["tensor_core"]:
+            continue
+        BN = p["block_rows"]
+        for b in range(p["row_blocks"]):
+            lo, hi = b * BN, min(R, (b + 1) * BN)
+            if lo >= R:
+                continue
+            sel.add(lo + (23 * b + 7) % (hi - lo))
+            sel.add(hi - 1)
+    for r in np.linspace(0, R - 1, want).round().astype(int):
+        sel.add(int(r))
+    return sorted(sel)
+
+
+@pytest.mark.parametrize("name,rows,keep,act", FULL,
+                         ids=[f"{n}-{r}-{k}-{a}" for n, r, k, a in FULL])
+def test_full_size_sampled_rows(ctx, name, rows, keep, act):
     w = wl.workload(name, device=DEV, rows=rows, keep_frac=keep)
-    sample = sorted({0, w.rows // 2, w.rows - 1})
-    codes, scale, _ = check_cloud(ctx, w, rows=sample)
+    sample = rows_to_check(ctx, w, act)
+    assert len(sample) >= min(16, w.rows)
+    codes, scale, _ = check_cloud(ctx, w, act_mode=act, rows=sample)
     # endpoint on a synthetic payload of the same shape (an input shared by
     # both sides), full launch, sampled rows checked
     pc, ps = wl.make_payload(w.rows, w.n_keep, seed=11, device=DEV)
@@ -337,6 +373,36 @@ def test_full_size_sampled_rows(ctx, name, rows, keep):
     if w.sessions:
         target = wl.make_target_logits(w.rows, w.n_keep, seed=12, device=DEV)
         check_verify(ctx, w, target.cpu())
+
+
+def test_full_size_plans_are_covered(ctx):
+    # the C5 1024-row plan has several row blocks, and the sampled rows hit
+    # every one of them
+    from paper_2607_13093_gb300 import sph
+    w = wl.workload("sweep", device=DEV, rows=1024, keep_frac=1.0)
+    p = ctx.plan(0, 1024, w.n_keep, w.d_h, gather=False)
+    assert p["tensor_core"] and p["row_blocks"] >= 4
+    sample = rows_to_check(ctx, w, "fp32")
+    hit = {r // p["block_rows"] for r in sample}
+    assert hit == set(range(p["row_blocks"]))
+    assert len({(r % p["block_rows"]) // 16 for r in sample}) >= 4
+
+
+# ---------------------------------------------------------------------------
+# the paper's split-dimension study (Sec. "Sensitivity to Split Dimension"):
+# D = 4096, V = 150000, 32 rows, language subsets of 40 % and 30 %, every
+# d_l of its table; all rows compared
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("keep", [0.4, 0.3])
+@pytest.mark.parametrize("d_l", [48, 96, 128, 256, 512])
+def test_split_dimension_study_shapes(ctx, d_l, keep):
+    w = wl.workload("dend", device=DEV, keep_frac=keep, d_l=d_l)
+    assert (w.d, w.V, w.rows, w.n_keep) == (4096, 150000, 32, round(keep * 150000))
+    check_cloud(ctx, w)
+    # the endpoint on the oracle's own payload (an input both sides share)
+    ref = oracle_cloud(w)
+    check_endpoint(ctx, w, torch.from_numpy(ref["codes"]), torch.from_numpy(ref["row_scale"]))
 
 
 # ---------------------------------------------------------------------------
@@ -348,16 +414,18 @@ def test_full_size_sampled_rows(ctx, name, rows, keep):
 def test_max_rows(ctx):
     w = small(V=600, d=128, d_l=64, rows=1 << 20, n_keep=40, run_lo=4, run_hi=12, seed=1201)
     sample = [0, 1, 777_777, (1 << 20) - 1]
-    codes, scale, _ = check_cloud(ctx, w, rows=sample)
-    check_endpoint(ctx, w, codes.cpu(), scale.cpu(), rows=sample)
+    check_cloud(ctx, w, rows=sample)
+    pc, ps = wl.make_payload(w.rows, w.n_keep, seed=13, device=DEV)
+    check_endpoint(ctx, w, pc, ps, rows=sample)
 
 
 def test_kept_set_past_the_fused_sampler(ctx):
     n = 4096 * 1024 + 5000
     w = small(V=n + 7000, d=96, d_l=32, rows=4, n_keep=n, run_lo=200, run_hi=4000,
               seed=1202)
-    codes, scale, _ = check_cloud(ctx, w, rows=[0, 3])
-    check_endpoint(ctx, w, codes.cpu(), scale.cpu())
+    check_cloud(ctx, w, rows=[0, 3])
+    pc, ps = wl.make_payload(w.rows, w.n_keep, seed=14, device=DEV)
+    check_endpoint(ctx, w, pc, ps)
 
 
 # ---------------------------------------------------------------------------
