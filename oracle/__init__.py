@@ -9,4 +9,6 @@ from .sph_oracle import (decode_bf16, decode_e4m3, round_fp32_to_bf16,  # noqa: 
                          quantize_rows, payload_bytes, partial_logits,
                          local_partial, fuse, softmax_rows, inverse_cdf,
                          sample_rows, fuse_sample, verify_core,
-                         compact_index, verify_draft, E4M3_VALUES)
+                         compact_index, verify_draft, E4M3_VALUES, draw,
+                         chunk_bounds, quantize_chunks, payload_bytes_chunked,
+                         fuse_chunks, split_step)

@@ -306,18 +306,12 @@ def gumbel_rows(z, tau: float, u):
     return greedy_rows(key)
 
 
-def fuse_sample(codes, row_scale, h_local, W_l_bits, *, keep_ids=None,
-                tau=1.0, seed=0, offset=0, sampler="cdf"):
-    """Endpoint call: local partial, fuse, mask, softmax(./tau), one Philox
-    uniform per row (purpose 0), inverse-CDF draw; tau = 0 is greedy
-    decoding (no uniform); sampler="gumbel" draws by Gumbel-max instead
-    (gumbel_rows).  Returns vocabulary-id `tokens`, the `margin` of each
-    draw (CDF distance, or for greedy and Gumbel-max the top-two gap) and
-    the fused logits `z`."""
-    V = W_l_bits.shape[0]
-    ids = _ids(keep_ids, V)
-    zl = local_partial(h_local, W_l_bits, ids)
-    z = fuse(codes, row_scale, zl)
+def draw(z, ids, *, tau=1.0, seed=0, offset=0, sampler="cdf"):
+    """The endpoint's draw from fused logits z (Eq. 15): one Philox uniform
+    per row (purpose 0) and the inverse CDF; tau = 0 is greedy decoding (no
+    uniform); sampler="gumbel" draws by Gumbel-max instead (gumbel_rows).
+    Returns vocabulary-id `tokens`, the `margin` of each draw (CDF distance,
+    or for greedy and Gumbel-max the top-two gap) and `z` itself."""
     R = z.shape[0]
     u = philox_uniform(seed, np.arange(R), 0, offset)
     if tau == 0:
@@ -329,6 +323,86 @@ def fuse_sample(codes, row_scale, h_local, W_l_bits, *, keep_ids=None,
         j, margin = sample_rows(z, tau, u)
     return dict(tokens=ids[j].astype(np.int32), margin=margin, z=z, u=u,
                 index=j)
+
+
+def fuse_sample(codes, row_scale, h_local, W_l_bits, *, keep_ids=None,
+                tau=1.0, seed=0, offset=0, sampler="cdf"):
+    """Endpoint call: local partial, fuse, mask, softmax(./tau), draw (see
+    `draw`)."""
+    V = W_l_bits.shape[0]
+    ids = _ids(keep_ids, V)
+    zl = local_partial(h_local, W_l_bits, ids)
+    z = fuse(codes, row_scale, zl)
+    return draw(z, ids, tau=tau, seed=seed, offset=offset, sampler=sampler)
+
+
+# ---------------------------------------------------------------------------
+# block streaming of the payload (Sec. "Device-Adaptive Feature
+# Preparation", Eq. 3: a tensor cut by columns into blocks that travel, and
+# are processed, one after another; Eq. 18 quantizes each transmitted
+# tensor; Eq. 21 counts its bytes).  Reading: the compacted logits are cut
+# into chunks of L consecutive kept ids, chunk q = ids q*L .. (q+1)*L - 1
+# (the last one shorter), and each chunk is quantized as a tensor of its
+# own, with one scale per row and chunk.
+# ---------------------------------------------------------------------------
+
+def chunk_bounds(n: int, chunk: int):
+    """[(j0, j1)] of the chunks of `chunk` kept ids (one chunk for chunk = 0
+    or chunk >= n)."""
+    L = n if (chunk <= 0 or chunk >= n) else int(chunk)
+    return [(j0, min(n, j0 + L)) for j0 in range(0, n, L)]
+
+
+def quantize_chunks(y: np.ndarray, clip: float, chunk: int):
+    """Q_8 of Eq. 18 applied to every chunk as its own tensor: codes [R, n]
+    (compacted id order) and scales [nchunk, R]."""
+    R, n = y.shape
+    b = chunk_bounds(n, chunk)
+    codes = np.zeros((R, n), dtype=np.int8)
+    scales = np.zeros((len(b), R), dtype=np.float32)
+    for q, (j0, j1) in enumerate(b):
+        codes[:, j0:j1], scales[q] = quantize_rows(y[:, j0:j1], clip)
+    return codes, scales
+
+
+def payload_bytes_chunked(rows: int, n_keep: int, chunk: int) -> int:
+    """Eq. 21 with b = 8 for a chunked payload: every kept logit's byte plus
+    one fp32 scale per row and chunk (the chunks' metadata B_meta); tag and
+    padding 0."""
+    return int(rows) * int(n_keep) + 4 * int(rows) * len(chunk_bounds(int(n_keep), chunk))
+
+
+def fuse_chunks(codes, scales, z_local, chunk: int) -> np.ndarray:
+    """Eq. 13 on a chunked payload: each chunk dequantized with its own
+    scales, plus the local partial."""
+    codes = np.asarray(codes)
+    z = np.array(z_local, dtype=np.float64)
+    for q, (j0, j1) in enumerate(chunk_bounds(codes.shape[1], chunk)):
+        s = np.asarray(scales[q], dtype=np.float32).astype(np.float64)
+        z[:, j0:j1] += codes[:, j0:j1].astype(np.float64) * s[:, None]
+    return z
+
+
+def split_step(h, d_l: int, W_h_bits, W_l_bits, *, w_dtype="bf16", w_scale=None,
+               bias=None, keep_ids=None, clip=30.0, act_mode="fp32", tau=1.0,
+               seed=0, offset=0, chunk=0, sampler="cdf"):
+    """The whole split step from the full hidden state (Algorithm 1's cloud
+    projection, then the endpoint's fusion and sampling): the cloud partial
+    of h[:, d_l:] (Eq. 12) clipped and quantized per chunk (Eq. 18; one
+    chunk = the whole row), the payload that would cross (Eq. 21), then the
+    local partial of h[:, :d_l] (Eq. 11), the fusion (Eq. 13) and the draw
+    (Eqs. 14-15).  Returns the cloud dict of `partial_logits` with the
+    chunked `codes`/`scales`, and the draw's dict under "draw"."""
+    h = np.asarray(h, dtype=np.float32)
+    c = partial_logits(h[:, d_l:], W_h_bits, w_dtype=w_dtype, w_scale=w_scale, bias=bias,
+                       keep_ids=keep_ids, clip=clip, act_mode=act_mode)
+    codes, scales = quantize_chunks(c["y"], clip, chunk)
+    ids = _ids(keep_ids, W_h_bits.shape[0])
+    zl = local_partial(h[:, :d_l], W_l_bits, ids)
+    z = fuse_chunks(codes, scales, zl, chunk)
+    return dict(y=c["y"], codes=codes, scales=scales,
+                payload_bytes=payload_bytes_chunked(h.shape[0], ids.size, chunk),
+                draw=draw(z, ids, tau=tau, seed=seed, offset=offset, sampler=sampler))
 
 
 # ---------------------------------------------------------------------------

@@ -607,3 +607,127 @@ def test_gumbel_max_small_temperature_is_greedy():
     j, _ = oracle.gumbel_rows(z, 1e-9, u)
     g, gap = oracle.greedy_rows(z)
     assert (gap > 1e-6).all() and (j == g).all()
+
+
+# ---------------------------------------------------------------------------
+# block streaming of the payload (Eq. 3 blocks, Eq. 18 per block, Eq. 21):
+# a chunked quantizer, its payload count, fusion, and the whole split step
+# ---------------------------------------------------------------------------
+
+def test_one_chunk_is_the_row_quantizer():
+    rng = np.random.default_rng(11)
+    y = rng.normal(size=(7, 533)) * 20.0
+    codes, s = oracle.quantize_rows(y, 30.0)
+    for chunk in (0, 533, 534, 10 ** 6):
+        c2, s2 = oracle.quantize_chunks(y, 30.0, chunk)
+        assert np.array_equal(c2, codes) and s2.shape == (1, 7)
+        assert np.array_equal(s2[0], s)
+        assert oracle.payload_bytes_chunked(7, 533, chunk) == oracle.payload_bytes(7, 533)
+
+
+def test_chunk_bounds_cover_the_ids_in_order():
+    assert oracle.chunk_bounds(10, 4) == [(0, 4), (4, 8), (8, 10)]
+    assert oracle.chunk_bounds(8, 4) == [(0, 4), (4, 8)]
+    assert oracle.chunk_bounds(5, 0) == [(0, 5)]
+    for n, L in ((1, 1), (1000, 7), (1024, 256), (150000, 37500)):
+        b = oracle.chunk_bounds(n, L)
+        assert b[0][0] == 0 and b[-1][1] == n
+        assert all(b[i][1] == b[i + 1][0] for i in range(len(b) - 1))
+        assert all(j1 - j0 == L for j0, j1 in b[:-1]) and 0 < b[-1][1] - b[-1][0] <= L
+
+
+def test_chunked_quantizer_closed_form():
+    # chunk q's largest |entry| is 127 * 2^-q exactly, so its scale is 2^-q
+    # and every entry of the form m * 2^-q quantizes to m; the all-zero
+    # chunk has scale 0 and codes 0
+    L = 5
+    y = np.zeros((1, 4 * L))
+    ms = np.array([127, -3, 64, 0, 5])
+    for q in range(3):
+        y[0, q * L:(q + 1) * L] = ms * 2.0 ** -q
+    codes, s = oracle.quantize_chunks(y, 1e9, L)
+    assert s[:, 0].tolist() == [1.0, 0.5, 0.25, 0.0]
+    for q in range(3):
+        assert codes[0, q * L:(q + 1) * L].tolist() == ms.tolist()
+    assert not codes[0, 3 * L:].any()
+    assert oracle.payload_bytes_chunked(1, 4 * L, L) == 4 * L + 16
+
+
+def test_chunked_quantizer_invariants():
+    # every chunk obeys the row quantizer's invariants with its own scale;
+    # the chunk scales never exceed the row scale and their maximum is it,
+    # so the chunked payload is never coarser than one scale per row
+    rng = np.random.default_rng(12)
+    R, n, L, clip = 9, 1000, 128, 30.0
+    y = rng.normal(size=(R, n)) * rng.uniform(0.01, 60, size=(1, n))
+    y[2, 256:384] = 0.0
+    codes, s = oracle.quantize_chunks(y, clip, L)
+    _, s_row = oracle.quantize_rows(y, clip)
+    yc = np.clip(y, -clip, clip)
+    b = oracle.chunk_bounds(n, L)
+    assert s.shape == (len(b), R) and len(b) == 8
+    for q, (j0, j1) in enumerate(b):
+        sq = s[q].astype(np.float64)[:, None]
+        err = np.abs(codes[:, j0:j1] * sq - yc[:, j0:j1])
+        assert np.all(err <= sq / 2 * (1 + 1e-6) + 1e-300)
+        nz = np.any(yc[:, j0:j1] != 0, axis=1)
+        assert np.all(np.abs(codes[nz, j0:j1]).max(axis=1) == 127)
+        assert np.all(s[q] <= s_row)
+    assert s[2, 2] == 0 and not codes[2, 256:384].any()
+    assert np.array_equal(s.max(axis=0), s_row)
+    assert oracle.payload_bytes_chunked(R, n, L) == R * n + 4 * R * 8
+    # the paper's CPU endpoint streams N_b = 4 blocks: 16 bytes of scales
+    # per row on top of Eq. 21's one byte per kept logit
+    assert oracle.payload_bytes_chunked(1, 150000, 37500) == 150000 + 16
+
+
+def test_chunked_fusion_within_each_chunks_bound():
+    """z from a chunked payload reproduces the full head (Eq. 13) to within
+    half of each chunk's own quantization step, and that bound is tighter
+    than one scale per row gives."""
+    w = tiny(with_bias=False, V=60, n_keep=40, rows=4)
+    ids = w.keep_ids.numpy()
+    h = w.h.numpy().astype(np.float64)
+    W_full = torch.cat([w.W_l, w.W_h], dim=1).double().numpy()
+    z_full = brute_full_head(h, W_full, None)[:, ids]
+    y = oracle.partial_logits(w.h_cloud.numpy(), bits16(w.W_h), keep_ids=ids, clip=1e30)["y"]
+    L = 8
+    codes, s = oracle.quantize_chunks(y, 1e30, L)
+    zl = oracle.local_partial(w.h_local.numpy(), bits16(w.W_l), ids)
+    z = oracle.fuse_chunks(codes, s, zl, L)
+    for q, (j0, j1) in enumerate(oracle.chunk_bounds(40, L)):
+        half = s[q].astype(np.float64)[:, None] / 2
+        assert np.all(np.abs(z[:, j0:j1] - z_full[:, j0:j1]) <= half * (1 + 1e-9))
+    _, s_row = oracle.quantize_rows(y, 1e30)
+    assert np.any(s < s_row[None, :])
+
+
+@pytest.mark.parametrize("chunk", [0, 8])
+def test_split_step_chains_cloud_and_endpoint(chunk):
+    # one chunk: exactly the cloud call followed by the endpoint call on its
+    # payload; chunks: the fused logits stay within each chunk's bound of
+    # the brute-force full head (Eq. 9) and the draw comes from them
+    w = tiny(with_bias=True, V=60, n_keep=40, rows=5)
+    ids = w.keep_ids.numpy()
+    out = oracle.split_step(w.h.numpy(), w.d_l, bits16(w.W_h), bits16(w.W_l),
+                            bias=w.bias.numpy(), keep_ids=ids, clip=1e30, tau=0.9,
+                            seed=5, offset=3, chunk=chunk)
+    if chunk == 0:
+        c = oracle.partial_logits(w.h_cloud.numpy(), bits16(w.W_h), bias=w.bias.numpy(),
+                                  keep_ids=ids, clip=1e30)
+        e = oracle.fuse_sample(c["codes"], c["row_scale"], w.h_local.numpy(), bits16(w.W_l),
+                               keep_ids=ids, tau=0.9, seed=5, offset=3)
+        assert np.array_equal(out["codes"], c["codes"])
+        assert np.array_equal(out["scales"][0], c["row_scale"])
+        assert np.array_equal(out["draw"]["z"], e["z"])
+        assert np.array_equal(out["draw"]["tokens"], e["tokens"])
+        assert out["payload_bytes"] == c["payload_bytes"]
+    h = w.h.numpy().astype(np.float64)
+    W_full = torch.cat([w.W_l, w.W_h], dim=1).double().numpy()
+    z_full = brute_full_head(h, W_full, w.bias.numpy())[:, ids]
+    b = oracle.chunk_bounds(40, chunk)
+    for q, (j0, j1) in enumerate(b):
+        half = out["scales"][q].astype(np.float64)[:, None] / 2
+        assert np.all(np.abs(out["draw"]["z"][:, j0:j1] - z_full[:, j0:j1]) <= half * (1 + 1e-9))
+    assert out["payload_bytes"] == 5 * 40 + 4 * 5 * len(b)
+    assert np.isin(out["draw"]["tokens"], ids).all()
