@@ -88,7 +88,18 @@ def parse():
     ap.add_argument("--nosplit", action="store_true",
                     help="time the unsplit head in place of the split step: the whole hidden "
                          "state times the whole head over the kept ids, then the sample (one "
-                         "endpoint call without payload; the paper's no-split ablation)")
+                         "endpoint call without payload; the paper's no-split ablation); "
+                         "the same as --step nosplit")
+    ap.add_argument("--step", choices=STEP_MODES, default="split",
+                    help="split: cloud call + endpoint call; fused: one sph_split_step call "
+                         "(one payload chunk); chunked: sph_split_step with --chunk-id "
+                         "payload blocks on two streams; nosplit: the unsplit head")
+    ap.add_argument("--chunk", type=int, default=4096, help="--step chunked: ids per block")
+    ap.add_argument("--vocab", type=int, default=None,
+                    help="sweep / dend: a smaller vocabulary (same kept fraction), for small "
+                         "profiling captures of the same kernel plan")
+    ap.add_argument("--opt", action="append", default=[],
+                    help="context option NAME=VALUE (" + ", ".join(OPTION_NAMES) + ")")
     ap.add_argument("--sampler", choices=["cdf", "gumbel"], default="cdf",
                     help="endpoint draw: inverse CDF (default) or Gumbel-max")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -316,16 +327,19 @@ def operand_planes(w, act):
     return 2 if act == "fp32" else 1
 
 
-def roofline(w, act, unit_ms, peaks, nosplit=False):
-    """Roofline of the dominant unit (the cloud call; the unsplit head with
-    nosplit) from its mean event-timed duration.  Only algorithmic bytes and
-    flops are credited.  The bound is whichever roof takes longer at its
-    peak: HBM (the measured copy bandwidth) or the tensor pipe (the measured
-    bf16 burst rate; for e4m3 weights on the f8f6f4 pipe twice that, the
-    nominal fp8:bf16 ratio)."""
+def roofline(w, act, unit_ms, peaks, mode="split"):
+    """Roofline of the dominant unit from its mean event-timed duration: the
+    cloud call (mode "split"), the unsplit head ("nosplit"), or the whole
+    one-call step ("fused", "chunked": both halves' bytes and flops).  Only
+    algorithmic bytes and flops are credited.  The bound is whichever roof
+    takes longer at its peak: HBM (the measured copy bandwidth) or the
+    tensor pipe (the measured bf16 burst rate; for e4m3 weights on the
+    f8f6f4 pipe twice that, the nominal fp8:bf16 ratio)."""
     from paper_2607_13093_gb300 import workloads as wl
     R, n = w.rows, w.n_keep
     fp8 = w.w_dtype == "fp8"
+    nosplit = mode == "nosplit"
+    whole = mode in ("fused", "chunked")
     if nosplit:
         alg_bytes = n * w.d * 2 + 4 * R * w.d + 4 * n + 4 * R
         alg_flops = wl.algorithmic_flops(R, n, w.d)
@@ -334,18 +348,26 @@ def roofline(w, act, unit_ms, peaks, nosplit=False):
         alg_flops = wl.algorithmic_flops(R, n, w.d_h)
     hbm = peaks["hbm_gbs"]
     tc = peaks["bf16_tflops"] * (2 if fp8 and not nosplit else 1)
+    if whole:
+        # + the endpoint half (bf16 W_l at the bf16 rate)
+        t_peak = alg_flops / tc + wl.algorithmic_flops(R, n, w.d_l) / peaks["bf16_tflops"]
+        alg_bytes += wl.algorithmic_bytes_endpoint(R, n, w.d_l)
+        alg_flops += wl.algorithmic_flops(R, n, w.d_l)
+        tc = alg_flops / t_peak
     s = unit_ms / 1e3
     bw = alg_bytes / s / 1e9
     fl = alg_flops / s / 1e12
     t_hbm = alg_bytes / (hbm * 1e9)
     t_tc = alg_flops / (tc * 1e12)
     planes = 1 if nosplit else operand_planes(w, act)
-    tensor = {"achieved": round(fl, 2), "peak": tc, "unit": "TFLOP/s",
+    tensor = {"achieved": round(fl, 2), "peak": round(tc, 1), "unit": "TFLOP/s",
               "frac": round(fl / tc, 4),
-              "issued_frac": round(planes * fl / tc, 4) if not nosplit else None,
+              "issued_frac": round(planes * fl / tc, 4) if not (nosplit or whole) else None,
               "planes": planes,
               "peak_note": ("e4m3 x e4m3 (kind::f8f6f4): 2 x the measured bf16 burst"
-                            if fp8 and not nosplit else "measured bf16 burst")}
+                            if fp8 and not nosplit else "measured bf16 burst")
+                           + (" (cloud half; the endpoint half at the bf16 rate)"
+                              if whole else "")}
     mem = {"achieved": round(bw, 1), "peak": hbm, "unit": "GB/s", "frac": round(bw / hbm, 4)}
     bound = "tensor" if t_tc > t_hbm else "hbm"
     main = tensor if bound == "tensor" else mem
@@ -359,16 +381,33 @@ def roofline(w, act, unit_ms, peaks, nosplit=False):
     return out
 
 
-class Runner:
-    """One workload's buffers and its step: the cloud call then the endpoint
-    call (+ verification for drafted workloads); `nosplit` replaces both
-    with one endpoint call over the whole head (the no-split ablation)."""
+STEP_MODES = ("split", "fused", "chunked", "nosplit")
 
-    def __init__(self, sph, wl, w, dev, act="fp32", nosplit=False, sampler="cdf"):
+OPTION_NAMES = {"tc_min_rows": "SPH_OPT_TC_MIN_ROWS", "schedule": "SPH_OPT_TC_SCHEDULE",
+                "stages": "SPH_OPT_TC_STAGES", "block_k": "SPH_OPT_TC_BLOCK_K",
+                "max_bn": "SPH_OPT_TC_MAX_BN", "tile_m": "SPH_OPT_TC_TILE_M",
+                "finish_wait": "SPH_OPT_TC_FINISH_WAIT"}
+
+
+class Runner:
+    """One workload's buffers and its step.  mode "split": the cloud call
+    then the endpoint call (+ verification for drafted workloads); "fused":
+    the same step as one sph_split_step call (one payload chunk, quantized
+    in the endpoint's epilogue); "chunked": sph_split_step with a payload
+    of `chunk`-id blocks, the endpoint fusing block q - 1 on its own stream
+    while the cloud computes block q; "nosplit": one endpoint call over the
+    whole head (the no-split ablation)."""
+
+    def __init__(self, sph, wl, w, dev, act="fp32", mode="split", sampler="cdf", chunk=0,
+                 options=()):
         import torch
+        nosplit = mode == "nosplit"
         self.sph, self.w, self.dev, self.act, self.nosplit = sph, w, dev, act, nosplit
+        self.mode, self.chunk = mode, chunk
         R, n = w.rows, w.n_keep
         self.ctx = ctx = sph.Context(dev.index or 0)
+        for name, value in options:
+            ctx.set_option(getattr(sph, OPTION_NAMES[name]), int(value))
         self.act_mode = sph.SPH_ACT_BF16 if act == "bf16" else sph.SPH_ACT_FP32
         if sampler == "gumbel":
             ctx.set_option(sph.SPH_OPT_SAMPLER, sph.SPH_SAMPLER_GUMBEL)
@@ -392,6 +431,9 @@ class Runner:
         self.hs = [w.h] + [w.h.roll(i + 1, dims=0).contiguous() for i in range(ncopy - 1)]
         self.codes = torch.empty(R, n, dtype=torch.int8, device=dev)
         self.scale = torch.empty(R, dtype=torch.float32, device=dev)
+        L = n if (chunk <= 0 or chunk >= n) else chunk
+        self.nchunk = (n + L - 1) // L
+        self.scales = torch.empty(self.nchunk * R, dtype=torch.float32, device=dev)
         self.tokens = torch.empty(R, dtype=torch.int32, device=dev)
         self.z = torch.empty(R, n, device=dev) if w.sessions else None
         self.n_acc = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
@@ -404,7 +446,16 @@ class Runner:
         hh = self.hs[c] if h is None else h
         if events is not None:
             events[0].record()
-        if self.nosplit:                 # one endpoint call over the whole head
+        if self.mode in ("fused", "chunked"):
+            ctx.split_step(hh, w.d_l, self.Whs[c], self.Wls[c], keep_ids=w.keep_ids, clip=w.clip,
+                           w_row_scale=w.w_scale, bias=w.bias, act_mode=self.act_mode,
+                           temperature=w.tau, seed=w.seed, offset=i,
+                           chunk=self.chunk if self.mode == "chunked" else 0,
+                           codes=self.codes.view(-1), scales=self.scales, tokens=self.tokens,
+                           fused_logits_out=self.z)
+            if events is not None:
+                events[1].record()
+        elif self.nosplit:               # one endpoint call over the whole head
             ctx.fuse_sample(None, None, hh, self.Wfs[c], keep_ids=w.keep_ids,
                             temperature=w.tau, seed=w.seed, offset=i, tokens=self.tokens,
                             fused_logits_out=self.z)
@@ -412,9 +463,9 @@ class Runner:
             ctx.partial_logits(hh[:, w.d_l:], self.Whs[c], keep_ids=w.keep_ids, clip=w.clip,
                                w_row_scale=w.w_scale, bias=w.bias, codes=self.codes,
                                row_scale=self.scale, act_mode=self.act_mode)
-        if events is not None:
+        if events is not None and self.mode in ("split", "nosplit"):
             events[1].record()
-        if not self.nosplit:
+        if self.mode == "split":
             ctx.fuse_sample(self.codes, self.scale, hh[:, :w.d_l], self.Wls[c],
                             keep_ids=w.keep_ids, temperature=w.tau, seed=w.seed, offset=i,
                             tokens=self.tokens, fused_logits_out=self.z)
@@ -555,25 +606,42 @@ def unit_stats(unit):
             "max_ms": round(max(unit), 5), "pairs": len(unit)}
 
 
-# sub-configurations timed beside the headline (name, rows, keep, d_l, act)
-CONFIG_BLOCK = [("tiny", None, None, None, "fp32"),
-                ("decode", None, None, None, "fp32"), ("decode", None, None, None, "bf16"),
-                ("spec", None, None, None, "fp32"), ("spec", None, None, None, "bf16"),
-                ("fp8", None, None, None, "fp32"), ("fp8", None, None, None, "bf16"),
-                ("sweep", 1, 1.0, None, "fp32"), ("sweep", 8, 1.0, None, "fp32"),
-                ("sweep", 64, 1.0, None, "fp32"), ("sweep", 256, 1.0, None, "fp32"),
-                ("sweep", 1024, 1.0, None, "bf16"),
-                ("dend", None, 0.4, 96, "fp32")]
+# sub-configurations timed beside the headline
+# (name, rows, keep, d_l, act, step mode, chunk)
+CONFIG_BLOCK = [("tiny", None, None, None, "fp32", "split", 0),
+                ("decode", None, None, None, "fp32", "split", 0),
+                ("decode", None, None, None, "bf16", "split", 0),
+                ("spec", None, None, None, "fp32", "split", 0),
+                ("spec", None, None, None, "bf16", "split", 0),
+                ("fp8", None, None, None, "fp32", "split", 0),
+                ("fp8", None, None, None, "bf16", "split", 0),
+                ("sweep", 1, 1.0, None, "fp32", "split", 0),
+                ("sweep", 8, 1.0, None, "fp32", "split", 0),
+                ("sweep", 64, 1.0, None, "fp32", "split", 0),
+                ("sweep", 256, 1.0, None, "fp32", "split", 0),
+                ("sweep", 1024, 1.0, None, "bf16", "split", 0),
+                ("dend", None, 0.4, 96, "fp32", "split", 0),
+                # the one-call step (one chunk, quantized in the endpoint's
+                # epilogue) and the block-streamed payload beside the two calls
+                ("decode", None, None, None, "fp32", "fused", 0),
+                ("decode", None, None, None, "fp32", "chunked", 4096),
+                ("dend", None, 0.4, 96, "fp32", "fused", 0),
+                ("dend", None, 0.4, 96, "fp32", "chunked", 15000),
+                ("sweep", 1024, 1.0, None, "fp32", "fused", 0),
+                ("sweep", 1024, 1.0, None, "fp32", "chunked", 64000),
+                # the unsplit head (the no-split ablation)
+                ("decode", None, None, None, "fp32", "nosplit", 0)]
 DEND_GRID = [(k, d) for k in (0.4, 0.3) for d in (48, 96, 128, 256, 512)]
 
 
 def config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks, cpu_seconds,
-                 target_s=0.3, e2e_steps=50, with_cpu=True):
-    """One line of the per-configuration block: its own step rate, cloud-call
-    time and roofline, end-to-end rate and oracle baseline."""
+                 target_s=0.3, e2e_steps=50, with_cpu=True, mode="split", chunk=0):
+    """One line of the per-configuration block: its own step rate, time and
+    roofline of the dominant call (the cloud call; the whole step for the
+    one-call modes), end-to-end rate and oracle baseline."""
     import torch
     w = wl.workload(name, device=dev, rows=rows, keep_frac=keep, d_l=d_l)
-    r = Runner(sph, wl, w, dev, act)
+    r = Runner(sph, wl, w, dev, act, mode=mode, chunk=chunk)
     try:
         # steps for about target_s of timed work, from one timed warm-up graph
         for i in range(3):
@@ -588,19 +656,21 @@ def config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks, cpu_seconds,
         steps = steps // r.gsteps * r.gsteps
         res = timed_run(r, steps, 3, bracket=False, min_pairs=64)
         unit = unit_stats(res["unit"])
-        roof = roofline(w, act, unit["mean_ms"], peaks)
+        roof = roofline(w, act, unit["mean_ms"], peaks, mode)
         roof["timing"] = res["timing"]
         roof["spread"] = unit
+        one_call = mode in ("fused", "chunked")
         entry = {"workload": describe(w), "activations": act,
+                 "step": mode + (f" ({r.nchunk} chunks of {chunk} ids)" if mode == "chunked" else ""),
                  "rows_per_s": round(job_rows_per_s(w.rows, 1, steps, res["ms"]), 1),
                  "ms_per_step": round(res["ms"] / steps, 5), "steps": steps,
-                 "cloud_us": round(unit["mean_ms"] * 1e3, 2),
+                 ("step_call_us" if one_call else "cloud_us"): round(unit["mean_ms"] * 1e3, 2),
                  "roofline": roof,
                  "e2e_rows_per_s": e2e_run(r, e2e_steps)["value"],
-                 "payload_bytes_per_step": sph.sph_payload_bytes(w.rows, w.n_keep),
+                 "payload_bytes_per_step": (w.rows * w.n_keep + 4 * w.rows * r.nchunk),
                  "gpu_launches_per_step": round(res["launches_per_step"], 2)}
         if with_cpu:
-            entry["cpu_baseline"] = cpu_baseline(w, cpu_seconds, act)
+            entry["cpu_baseline"] = cpu_baseline(w, cpu_seconds, act, mode == "nosplit")
         return entry
     finally:
         r.close()
@@ -626,13 +696,14 @@ def run_ours(args):
     from paper_2607_13093_gb300 import sph, workloads as wl
 
     w = wl.workload(args.workload, device=dev, rows=args.rows, keep_frac=args.keep,
-                    d_l=args.d_l)
+                    d_l=args.d_l, V=args.vocab)
     if world > 1:                       # each rank: its own sessions
         g = torch.Generator(device=dev)
         g.manual_seed(rank_seed(rank))
         w.h = wl.make_hidden(w.rows, w.d, g, dev)
     R, n = w.rows, w.n_keep
-    r = Runner(sph, wl, w, dev, args.act, args.nosplit, args.sampler)
+    options = [tuple(o.split("=", 1)) for o in args.opt]
+    r = Runner(sph, wl, w, dev, args.act, args.step, args.sampler, args.chunk, options)
 
     gpu_uuid = None
     try:
@@ -680,13 +751,16 @@ def run_ours(args):
     peaks, peaks_src = load_peaks()
     value = job_rows_per_s(R, world, args.steps, ms)
     unit = unit_stats(res["unit"])
-    roof = roofline(w, args.act, unit["mean_ms"], peaks, args.nosplit)
-    roof.update({"traffic": None if args.nosplit else traffic_for(
-                     f"cloud_{args.workload}_{R}_{n}_{args.act}"),
-                 "kernel": ("unsplit head: gathered whole-d contraction + sample (one endpoint "
-                            "call without payload)" if args.nosplit else
-                            "cloud call: operand split + gathered tcgen05 contraction + int8 "
-                            "quantization"),
+    roof = roofline(w, args.act, unit["mean_ms"], peaks, args.step)
+    kernel = {"nosplit": ("unsplit head: gathered whole-d contraction + sample (one endpoint "
+                          "call without payload)"),
+              "split": ("cloud call: operand split + gathered tcgen05 contraction + int8 "
+                        "quantization"),
+              "fused": "the one-call split step (cloud + endpoint, one payload chunk)",
+              "chunked": f"the one-call split step, {r.nchunk} payload chunks on two streams"}
+    roof.update({"traffic": traffic_for(f"cloud_{args.workload}_{R}_{n}_{args.act}")
+                 if args.step == "split" else None,
+                 "kernel": kernel[args.step],
                  "timing": res["timing"], "spread": unit,
                  "peak_source": ("measured (MEASURED_PEAKS.json)" if peaks_src == "measured"
                                  else "fallback")})
@@ -698,8 +772,10 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None,
         "dtype": "f32" if args.act == "fp32" else "bf16",
         "data": "synthetic (seeded, paper shapes; weights N(0,0.02) bf16, h RMS-normalised)",
-        "config": {"workload": describe(w) + (", unsplit head (no-split ablation)"
-                                              if args.nosplit else ""),
+        "config": {"workload": describe(w) + {
+                       "split": "", "nosplit": ", unsplit head (no-split ablation)",
+                       "fused": ", one-call split step",
+                       "chunked": f", one-call split step, {r.nchunk} payload chunks"}[args.step],
                    "rows_per_gpu": R, "n_keep": n,
                    "d_h": w.d_h, "d_l": w.d_l, "V": w.V, "weights": w.w_dtype,
                    "accumulate": "fp32",
@@ -721,9 +797,10 @@ def run_ours(args):
         # downlink of one step (Eq. 21 with b = 8, no tag/metadata/padding):
         # int8 codes of the kept ids + an fp32 scale per row, against the full
         # vocabulary as int8 and as fp32 logits
-        "payload": {"bytes_per_step": (4 * R * n if args.nosplit else sph.sph_payload_bytes(R, n)),
+        "payload": {"bytes_per_step": (4 * R * n if args.nosplit else R * n + 4 * R * r.nchunk),
                     "what": ("fp32 logits of the kept ids, which an unsplit cloud head would send"
-                             if args.nosplit else "int8 codes of the kept ids + an fp32 scale per row"),
+                             if args.nosplit else "int8 codes of the kept ids + an fp32 scale per "
+                             "row and payload chunk"),
                     "full_vocab_int8_bytes": sph.sph_payload_bytes(R, w.V),
                     "full_vocab_fp32_bytes": 4 * R * w.V,
                     "reduction_vs_full_int8": round(
@@ -733,21 +810,28 @@ def run_ours(args):
     del r
     torch.cuda.empty_cache()
     if world == 1 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act, args.nosplit,
+        out["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, args.act, args.step == "nosplit",
                                            args.sampler)
     del w
     torch.cuda.empty_cache()
-    if world == 1 and not args.no_configs and not args.nosplit:
-        block = list(CONFIG_BLOCK) + ([("dend", None, k, d, "fp32") for k, d in DEND_GRID]
-                                      if args.dend_grid else [])
+    if world == 1 and not args.no_configs and args.step == "split" and not args.opt and \
+            args.vocab is None:
+        block = list(CONFIG_BLOCK) + ([("dend", None, k, d, "fp32", "split", 0)
+                                       for k, d in DEND_GRID] if args.dend_grid else [])
         entries = []
-        for (name, rows, keep, d_l, act) in block:
-            if (name, rows, keep, d_l, act) == (args.workload, args.rows, args.keep,
-                                                args.d_l, args.act):
+        seen_cpu = set()
+        for (name, rows, keep, d_l, act, mode, chunk) in block:
+            if (name, rows, keep, d_l, act, mode) == (args.workload, args.rows, args.keep,
+                                                      args.d_l, args.act, args.step):
                 continue
-            with_cpu = not args.no_cpu_baseline and (name != "dend" or (keep, d_l) == (0.4, 96))
+            # one oracle baseline per workload and activation mode
+            key = (name, rows, keep, d_l, act, mode == "nosplit")
+            with_cpu = not args.no_cpu_baseline and key not in seen_cpu and (
+                name != "dend" or (keep, d_l) == (0.4, 96))
+            seen_cpu.add(key)
             entries.append(config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks,
-                                        args.config_cpu_seconds, with_cpu=with_cpu))
+                                        args.config_cpu_seconds, with_cpu=with_cpu,
+                                        mode=mode, chunk=chunk))
         out["configs"] = entries
     print(json.dumps(out), flush=True)
     if world > 1:
@@ -765,7 +849,7 @@ def run_reference(args):
         return
     from paper_2607_13093_gb300 import workloads as wl
     w = wl.workload(args.workload, device="cpu", rows=args.rows, keep_frac=args.keep,
-                    d_l=args.d_l)
+                    d_l=args.d_l, V=args.vocab)
     s = OracleSample(w, args.act, args.nosplit, args.sampler)
     budget = args.ref_seconds
     L = s.calibrate(budget / max(1, args.steps + args.warmup))
@@ -797,6 +881,12 @@ def run_reference(args):
 
 def main():
     args = parse()
+    if args.nosplit:
+        args.step = "nosplit"
+    args.nosplit = args.step == "nosplit"
+    for o in args.opt:
+        if "=" not in o or o.split("=", 1)[0] not in OPTION_NAMES:
+            raise SystemExit(f"--opt {o}: expected NAME=VALUE with NAME in {sorted(OPTION_NAMES)}")
     if args.workload == "sweep" and args.rows is None and args.keep is None:
         args.rows, args.keep = 1024, 1.0       # the headline: the largest workload
     if args.impl == "reference":

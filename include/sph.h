@@ -244,9 +244,10 @@ sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep,
  *   row_scale[r] = max_j |yc[r, j]| / 127   (fp32; 0 for an all-zero row)
  *   codes[r, j]  = round-half-even(yc / row_scale[r]) in [-127, 127]
  *                  (the kernels multiply yc by the correctly rounded fp32
- *                  reciprocal of row_scale[r], so a code can differ by one
- *                  from the exact quotient's rounding only where that
- *                  quotient lies within about 1.5e-5 of a half-integer)
+ *                  reciprocal of row_scale[r] and round that product once,
+ *                  so a code can differ by one from the exact quotient's
+ *                  rounding only where that quotient lies within about
+ *                  1e-5 of a half-integer)
  * Arguments
  *   h_cloud  fp32 [rows, d_h] with row stride ld_h (>= d_h); typically the
  *            slice h[:, d_l:] of the full hidden state (ld_h = d).
@@ -359,6 +360,56 @@ sph_status sph_fuse_sample(sph_ctx* ctx,
                            const int32_t* keep_ids, int64_t n_keep,
                            float temperature, uint64_t seed, uint64_t offset,
                            int32_t* tokens, float* fused_logits_out);
+
+/* The whole split step in one call, from the full hidden state to tokens:
+ * the cloud call followed by the endpoint call (Eqs. 11-15, Eq. 18;
+ * Algorithm 1, the cloud's partial projection and the endpoint's fusion and
+ * sampling), on one GPU, with the payload that would cross between them
+ * (Eq. 21) written out.  It is the single-GPU form of the paper's split
+ * projection, the counterpart of the unsplit head that sph_fuse_sample
+ * computes without a payload (Sec. "Ablation Study").
+ *   h        fp32 [rows, d_l + d_h], row stride ld_h: h[:, :d_l] is the
+ *            endpoint's part, h[:, d_l:] the cloud's (Eq. 10).
+ *   W_h, w_dtype, w_row_scale, ld_wh, bias, keep_ids, n_keep, clip,
+ *   act_mode  as for sph_partial_logits;  W_l, ld_wl  as for
+ *            sph_fuse_sample;  temperature, seed, offset  as there too (the
+ *            draw is the same: purpose 0 of row r).
+ *   chunk    kept ids per payload chunk.  0 (or >= n_keep): one chunk, the
+ *            payload of sph_partial_logits (one scale per row); the
+ *            endpoint's contraction then quantizes the cloud's clipped
+ *            partials in its own epilogue, so no separate quantization pass
+ *            runs.  1 <= chunk < n_keep: block streaming (the GPU form of
+ *            the paper's block-wise streaming in Sec. "Device-Adaptive
+ *            Feature Preparation"): chunk q holds the ids
+ *            q*chunk .. min(n_keep, (q+1)*chunk) - 1 and carries its own
+ *            row scales, scale[q][r] = max over the chunk of |clipped y| /
+ *            127 (Eq. 18 applied per chunk); the cloud emits chunk q on the
+ *            context's stream while the endpoint fuses chunk q - 1 on
+ *            endpoint_stream (the SMs are divided between the two in
+ *            proportion to d_l : d_h).
+ *   endpoint_stream  a cudaStream_t other than the context's, or NULL for
+ *            one the context creates on first use and owns; used only when
+ *            there is more than one chunk.  The call's work is complete, on
+ *            the context's stream, when the endpoint's is.
+ *   codes    int8, rows * n_keep bytes (out), chunk-major: chunk q is the
+ *            row-major [rows][its ids] block starting at byte
+ *            q * chunk * rows.  One chunk: [rows, n_keep].
+ *   scales   fp32 [nchunk][rows] (out), nchunk = ceil(n_keep / chunk).
+ *   tokens   int32 [rows] (out) vocabulary ids;  fused_logits_out fp32
+ *            [rows, n_keep] z (out), or NULL.
+ *   payload_bytes  host (out), or NULL: rows * n_keep + 4 * rows * nchunk.
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA, OOM. */
+sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows,
+                          int64_t ld_h, int64_t d_l, int64_t d_h,
+                          const void* W_h, sph_dtype w_dtype,
+                          const float* w_row_scale, int64_t ld_wh,
+                          const void* W_l, int64_t ld_wl, int64_t V,
+                          const float* bias, const int32_t* keep_ids,
+                          int64_t n_keep, float clip, sph_act_mode act_mode,
+                          float temperature, uint64_t seed, uint64_t offset,
+                          int64_t chunk, void* endpoint_stream,
+                          int8_t* codes, float* scales, int32_t* tokens,
+                          float* fused_logits_out, size_t* payload_bytes);
 
 /* Cloud verification of speculative drafts (Sec. "Endpoint Speculative
  * Decoding and Cloud Verification", Algorithm 1; standard speculative

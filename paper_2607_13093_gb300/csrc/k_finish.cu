@@ -1,9 +1,9 @@
 // Quantisation of the clipped cloud partials (Eq. 18 with b = 8): one
 // symmetric fp32 scale per row, round to nearest even.  The quotient is the
-// partial times the correctly rounded fp32 reciprocal of the scale (at most
-// 1.5 fp32 roundings from the exact quotient); the oracle divides in fp64,
-// so a code can differ by one only where the quotient lies within about two
-// fp32 roundings (2e-5 at 127) of a half-integer.
+// partial times the correctly rounded fp32 reciprocal of the scale, rounded
+// once to an integer (quantize_one); the oracle divides in fp64, so a code
+// can differ by one only where the quotient lies within one rounding of the
+// reciprocal (about 8e-6 at 127) of a half-integer.
 #include <climits>
 
 #include "sm100_ptx.cuh"
@@ -24,15 +24,6 @@ namespace {
 constexpr int kQVec = 8;
 constexpr int kQThreads = 256;
 constexpr int kQSpan = kQThreads * kQVec;
-
-__device__ __forceinline__ float row_scale_of(const unsigned* rowmax, int r) {
-  return __fdiv_rn(__uint_as_float(rowmax[r]), 127.0f);
-}
-
-__device__ __forceinline__ int quantize_one(float y, float k, float inv_s) {
-  const int q = __float2int_rn((y * k) * inv_s);
-  return q > 127 ? 127 : (q < -127 ? -127 : q);
-}
 
 __global__ void __launch_bounds__(kQThreads)
 quantize_kernel(const float* __restrict__ Y, const unsigned* __restrict__ rowmax, int rows,
@@ -55,12 +46,9 @@ quantize_kernel(const float* __restrict__ Y, const unsigned* __restrict__ rowmax
       r = (int)(it / spans);
       sp = (int)(it - (int64_t)r * spans);
     }
-    const float s = row_scale_of(rowmax, r);
-    if (sp == 0 && threadIdx.x == 0) row_scale[r] = s;
-    // a scale below 2^-64 (partials below about 1e-17) is lifted by the exact
-    // factor 2^64 on both sides so that its reciprocal stays finite
-    const float k = s < 0x1p-64f ? 0x1p64f : 1.f;
-    const float inv_s = s > 0.f ? __frcp_rn(s * k) : 0.f;  // an all-zero row: codes 0
+    const RowQuant rq = row_quant(rowmax[r]);
+    const float k = rq.k, inv_s = rq.inv;
+    if (sp == 0 && threadIdx.x == 0) row_scale[r] = rq.s;
     const int64_t row0 = (int64_t)r * n;
     if (!vec_load) {
       // rows not 16-byte aligned: entry i of the thread is column

@@ -169,8 +169,17 @@ gemv_kernel(const GatherGemm g, const int row0) {
           const float yc = fminf(fmaxf(y, -g.clip), g.clip);
           g.Y[o] = yc;
           lmax = fmaxf(lmax, fabsf(yc));
+        } else if constexpr (EPI == EPI_FUSED) {
+          // quantize the cloud's clipped partial (Eq. 18), emit the code
+          // (and, at the first id, the row scale), dequantize it (Eq. 13)
+          const RowQuant rq = row_quant(__ldcg(g.rowmax_in + row0 + r));
+          const int code = quantize_one(__ldcg(g.yc + o), rq.k, rq.inv);
+          g.codes_out[o] = (int8_t)code;
+          if (j == 0) g.scale_out[row0 + r] = rq.s;
+          g.Y[(int64_t)(row0 + r) * g.ldy + j] = y + (float)code * rq.s;
         } else {
-          g.Y[o] = g.codes ? y + (float)g.codes[o] * g.row_scale[row0 + r] : y;
+          g.Y[(int64_t)(row0 + r) * g.ldy + j] =
+              g.codes ? y + (float)g.codes[o] * g.row_scale[row0 + r] : y;
         }
       }
     }
@@ -252,7 +261,14 @@ cudaError_t launch_wdt(const GatherGemm& g, int sm_count, cudaStream_t st) {
 int gemv_max_k() { return (int)(kSmemLimit / sizeof(float)) & ~7; }
 int gemv_rows_per_launch(int rows, int K) { return rows_per_launch(rows, K); }
 
-cudaError_t launch_gemv(const GatherGemm& g, int sm_count, cudaStream_t st) {
+cudaError_t launch_gemv(const GatherGemm& g_in, int sm_count, cudaStream_t st) {
+  GatherGemm g = g_in;
+  if (!g.ldy) g.ldy = g.n;
+  if (g.epilogue == EPI_FUSED) {
+    if (g.w_dtype != W_BF16 || !g.yc || !g.rowmax_in || !g.codes_out || !g.scale_out)
+      return cudaErrorNotSupported;
+    return launch_wdt<W_BF16, EPI_FUSED>(g, sm_count, st);
+  }
   if (g.w_dtype == W_BF16)
     return g.epilogue == EPI_CLOUD ? launch_wdt<W_BF16, EPI_CLOUD>(g, sm_count, st)
                                    : launch_wdt<W_BF16, EPI_ENDPOINT>(g, sm_count, st);

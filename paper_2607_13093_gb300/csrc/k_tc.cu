@@ -104,6 +104,11 @@ struct TcParams {
   const int8_t* codes;
   const float* row_scale;
   float inv_tau;
+  int64_t ldy;                 // row stride of Y (endpoint: z) in elements
+  const float* yc;             // fused endpoint: the cloud's clipped partials [R][n]
+  const unsigned* rowmax_in;   // fused endpoint: their row |max| bits [R]
+  int8_t* codes_out;           // fused endpoint: the payload codes [R][n] (out)
+  float* scale_out;            // fused endpoint: the row scales [R] (out)
   float2* seg_stats;           // endpoint: [R][nseg] (max, sum exp)
   int a3d;                     // full vocabulary: A by one 3-D copy per stage
   int single_acc;              // one accumulator (no epilogue overlap): 256-id tiles of > 128 rows
@@ -141,34 +146,52 @@ struct Segments {
 
 
 // Endpoint payload of one 16-row chunk at this lane's id column j: the int8
-// codes of rows row0..row0+15 and, in lane q < 16, the scale of row row0 + q.
+// codes of rows row0..row0+15 (as floats) and, in lane q < 16, the scale of
+// row row0 + q.  The fused endpoint loads the cloud's clipped fp32 partials
+// instead, and the quantizer's lift and reciprocal of the row scale.
 // Addresses are clamped into the arrays and every load is issued, so the 16
 // loads go out back to back and can be started a chunk ahead of their use.
 struct Payload {
-  int c[16];
+  float c[16];
   float s;
+  float k, inv;                        // fused endpoint only
 };
+template <int EPI>
 __device__ __forceinline__ void load_payload(const TcParams& p, int row0, int j, int lane,
                                              Payload& pl) {
+  if constexpr (EPI == EPI_FUSED) {
+    const float* col = p.yc + min(j, p.n - 1);
+#pragma unroll
+    for (int q = 0; q < 16; ++q) pl.c[q] = __ldcg(col + (int64_t)min(row0 + q, p.R - 1) * p.n);
+    const RowQuant rq = row_quant(__ldcg(p.rowmax_in + min(row0 + (lane & 15), p.R - 1)));
+    pl.s = rq.s;
+    pl.k = rq.k;
+    pl.inv = rq.inv;
+    return;
+  }
   if (!p.codes) {                      // no payload: z is the local partial alone
 #pragma unroll
-    for (int q = 0; q < 16; ++q) pl.c[q] = 0;
+    for (int q = 0; q < 16; ++q) pl.c[q] = 0.f;
     pl.s = 0.f;
     return;
   }
   const int8_t* col = p.codes + min(j, p.n - 1);
 #pragma unroll
-  for (int q = 0; q < 16; ++q) pl.c[q] = __ldg(col + (int64_t)min(row0 + q, p.R - 1) * p.n);
+  for (int q = 0; q < 16; ++q) pl.c[q] = (float)__ldg(col + (int64_t)min(row0 + q, p.R - 1) * p.n);
   pl.s = __ldg(p.row_scale + min(row0 + (lane & 15), p.R - 1));
 }
-// Warm L2 with the codes of rows row0..row0+nrows-1 at the 32 ids from j0.
-__device__ __forceinline__ void prefetch_codes(const TcParams& p, int row0, int nrows, int j0,
-                                               int lane) {
-  if (j0 >= p.n || !p.codes) return;
-  const int8_t* col = p.codes + j0;
-  const int last = min(31, p.n - 1 - j0);
+// Warm L2 with the payload of rows row0..row0+nrows-1 at the 32 ids from j0
+// (the codes, or for the fused endpoint the clipped partials).
+template <int EPI>
+__device__ __forceinline__ void prefetch_payload(const TcParams& p, int row0, int nrows, int j0,
+                                                 int lane) {
+  const int esz = EPI == EPI_FUSED ? 4 : 1;
+  const char* base = EPI == EPI_FUSED ? reinterpret_cast<const char*>(p.yc)
+                                      : reinterpret_cast<const char*>(p.codes);
+  if (j0 >= p.n || !base) return;
+  const int last = min(31, p.n - 1 - j0) * esz;
   for (int r = row0 + lane; r < min(row0 + nrows, p.R); r += 32) {
-    const int8_t* a = col + (int64_t)r * p.n;
+    const char* a = base + ((int64_t)r * p.n + j0) * esz;
     asm volatile("prefetch.global.L2 [%0];" ::"l"(a));
     asm volatile("prefetch.global.L2 [%0];" ::"l"(a + last));
   }
@@ -208,12 +231,26 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const float sq = __shfl_sync(0xFFFFFFFFu, pay.s, q);
-      z[q] = (vj && row0 + q < p.R) ? v[q] + (float)pay.c[q] * sq : -INFINITY;
+      float cq = pay.c[q];
+      if constexpr (EPI == EPI_FUSED) {
+        // quantize the cloud's clipped partial (Eq. 18) exactly as the
+        // quantize kernel does, emit the code, and dequantize it (Eq. 13)
+        const float kq = __shfl_sync(0xFFFFFFFFu, pay.k, q);
+        const float iq = __shfl_sync(0xFFFFFFFFu, pay.inv, q);
+        const int code = quantize_one(cq, kq, iq);
+        if (vj && row0 + q < p.R) p.codes_out[(int64_t)(row0 + q) * p.n + j] = (int8_t)code;
+        cq = (float)code;
+      }
+      z[q] = (vj && row0 + q < p.R) ? v[q] + cq * sq : -INFINITY;
+    }
+    if constexpr (EPI == EPI_FUSED) {
+      // the warp holding the first 32 ids emits the 16 rows' scales
+      if (j == lane && lane < 16 && row0 + lane < p.R) p.scale_out[row0 + lane] = pay.s;
     }
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const int r = row0 + q;
-      if (vj && r < p.R) p.Y[(int64_t)r * p.n + j] = z[q];
+      if (vj && r < p.R) p.Y[(int64_t)r * p.ldy + j] = z[q];
     }
     if (!p.seg_stats) return;          // statistics come from a pass over z
     // softmax statistics of this 32-id segment for each row: the maxima,
@@ -581,14 +618,15 @@ tc_kernel(const __grid_constant__ WMaps wm,
       auto VJ = [&](int hf) { return (kHalves > 1 && hf) ? vjh[kHalves - 1] : vjh[0]; };
       auto ID = [&](int hf) { return (kHalves > 1 && hf) ? idh[kHalves - 1] : idh[0]; };
       Payload pay;
-      if constexpr (EPI == EPI_ENDPOINT) {
+      if constexpr (EPI != EPI_CLOUD) {
         // the payload does not depend on the accumulator: start on it
         // while the tile's MMAs run
 #pragma unroll
         for (int hf = 0; hf < kHalves; ++hf)
-          prefetch_codes(p, rb * BN + grp * (BN / 2), BN / 2, t * TM + hf * 128 + quad * 32, lane);
+          prefetch_payload<EPI>(p, rb * BN + grp * (BN / 2), BN / 2,
+                                t * TM + hf * 128 + quad * 32, lane);
         if (whole && grp < nhc)
-          load_payload(p, rb * BN + (grp % nch) * 16, J(grp / nch), lane, pay);
+          load_payload<EPI>(p, rb * BN + (grp % nch) * 16, J(grp / nch), lane, pay);
       }
       // Split tile: contributors c0 .. c0 + C - 1 (CTA order).  All but the
       // last end their ranges inside the tile, so they reach it at the end
@@ -672,15 +710,15 @@ tc_kernel(const __grid_constant__ WMaps wm,
         if (whole) {
           Payload nxt;
           const int hn = hc + kEpiGroups;
-          if (EPI == EPI_ENDPOINT && hn < nhc)
-            load_payload(p, rb * BN + (hn % nch) * 16, J(hn / nch), lane, nxt);
+          if (EPI != EPI_CLOUD && hn < nhc)
+            load_payload<EPI>(p, rb * BN + (hn % nch) * 16, J(hn / nch), lane, nxt);
           finish_chunk<EPI>(p, v, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
                             t * kGroups + hf * 4 + quad, pay);
-          if constexpr (EPI == EPI_ENDPOINT) pay = nxt;
+          if constexpr (EPI != EPI_CLOUD) pay = nxt;
         } else if (known_last) {
           // the partials in CTA order (the same order, and so the same
           // result, as the fix-up below), this CTA's own from registers
-          if constexpr (EPI == EPI_ENDPOINT) load_payload(p, rb * BN + ch * 16, J(hf), lane, pay);
+          if constexpr (EPI != EPI_CLOUD) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
           const int me = (int)blockIdx.x - c0;
           const size_t o = (size_t)ch * 16 * TM + i;
           float s[16];
@@ -729,7 +767,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
             ps[c] = p.P + (size_t)slot_of(c < C ? c : 0) * BN * TM + quad * 32 + lane;
           for (int hc = grp; hc < nhc; hc += kEpiGroups) {
             const int hf = hc / nch, ch = hc - hf * nch;
-            if constexpr (EPI == EPI_ENDPOINT) load_payload(p, rb * BN + ch * 16, J(hf), lane, pay);
+            if constexpr (EPI != EPI_CLOUD) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
             const size_t o = (size_t)ch * 16 * TM + hf * 128;
             float v[16];
 #pragma unroll
@@ -1115,12 +1153,20 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.NT = (n + pl.tm - 1) / pl.tm;
   const int tiles = pl.RB * pl.NT;
   pl.T = (long long)tiles * pl.KB;
+  // CTAs: with several row blocks, a multiple of the row-block count, so
+  // that every row block's iterations split at the same offsets and the
+  // CTAs that stream the same weight tile for different row blocks run in
+  // step (one reads it from DRAM, the others from L2).  Measured on 1024
+  // rows x 25600 ids x 4608 in five row blocks: 152 CTAs (ranges offset by
+  // 2.6 tiles between row blocks) read 5.6x the kept weights from DRAM.
+  int sm_use = sm_count;
+  if (pl.RB > 1 && pl.RB <= sm_count) sm_use = sm_count / pl.RB * pl.RB;
   // whole tiles per CTA unless that leaves the grid clearly unbalanced
-  const int g_whole = tiles < sm_count ? tiles : sm_count;
+  const int g_whole = tiles < sm_use ? tiles : sm_use;
   const long long whole_span = (long long)((tiles + g_whole - 1) / g_whole) * pl.KB;
-  const double split_span = (double)pl.T / (pl.T < sm_count ? pl.T : sm_count);
+  const double split_span = (double)pl.T / (pl.T < sm_use ? pl.T : sm_use);
   pl.whole_tiles = schedule == 1 || (schedule == 0 && whole_span <= 1.1 * split_span + 2.0);
-  pl.G = pl.whole_tiles ? g_whole : (int)(pl.T < sm_count ? pl.T : sm_count);
+  pl.G = pl.whole_tiles ? g_whole : (int)(pl.T < sm_use ? pl.T : sm_use);
   const int stage_bytes = pl.na * (halves * kAtomBytes + pl.hilo * pl.BN * 128);
   pl.stages = (int)((kSmemBudget - 2048) / stage_bytes);
   if (pl.stages > kMaxStages) pl.stages = kMaxStages;
@@ -1175,7 +1221,9 @@ static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                       long long spin_limit, cudaStream_t st) {
   const bool fp8 = g.w_dtype == W_FP8;
-  if (!pl.ok || (fp8 != (pl.fp8 != 0)) || (fp8 && g.epilogue != EPI_CLOUD))
+  if (!pl.ok || (fp8 != (pl.fp8 != 0)) || (fp8 && g.epilogue != EPI_CLOUD) ||
+      (g.epilogue != EPI_CLOUD && pl.hilo != 2) ||
+      (g.epilogue == EPI_FUSED && (!g.yc || !g.rowmax_in || !g.codes_out || !g.scale_out)))
     return cudaErrorNotSupported;
   char* sc = static_cast<char*>(scratch);
   auto* Hs = reinterpret_cast<__nv_bfloat16*>(sc);
@@ -1236,6 +1284,9 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.ld_w = g.ld_w;
   prm.w_scale = fp8 ? g.w_scale : nullptr;
   prm.epilogue = g.epilogue; prm.bias = g.bias;
+  prm.ldy = g.ldy ? g.ldy : g.n;
+  prm.yc = g.yc; prm.rowmax_in = g.rowmax_in; prm.codes_out = g.codes_out;
+  prm.scale_out = g.scale_out;
   prm.clip = g.clip; prm.partial_out = g.partial_out; prm.Y = g.Y;
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
   prm.single_acc = pl.single_acc;
@@ -1257,10 +1308,12 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
       return hilo2 ? launch_inst<2, false, EPI_CLOUD, false, 256>(mw, mh, prm, pl, st)
                    : launch_inst<1, false, EPI_CLOUD, false, 256>(mw, mh, prm, pl, st);
     }
-    if (gather) return hilo2 ? launch_inst<2, true, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st)
-                             : launch_inst<1, true, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st);
-    return hilo2 ? launch_inst<2, false, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st)
-                 : launch_inst<1, false, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st);
+    // (the endpoint's activations are always fp32-exact: two planes)
+    if (g.epilogue == EPI_FUSED)
+      return gather ? launch_inst<2, true, EPI_FUSED, false, 256>(mw, mh, prm, pl, st)
+                    : launch_inst<2, false, EPI_FUSED, false, 256>(mw, mh, prm, pl, st);
+    return gather ? launch_inst<2, true, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st)
+                  : launch_inst<2, false, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st);
   }
   if (fp8) {                // four e4m3 planes of h, or two for bf16-rounded h
     if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, true>(mw, mh, prm, pl, st)
@@ -1274,10 +1327,11 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
     return hilo2 ? launch_inst<2, false, EPI_CLOUD>(mw, mh, prm, pl, st)
                  : launch_inst<1, false, EPI_CLOUD>(mw, mh, prm, pl, st);
   }
-  if (gather) return hilo2 ? launch_inst<2, true, EPI_ENDPOINT>(mw, mh, prm, pl, st)
-                           : launch_inst<1, true, EPI_ENDPOINT>(mw, mh, prm, pl, st);
-  return hilo2 ? launch_inst<2, false, EPI_ENDPOINT>(mw, mh, prm, pl, st)
-               : launch_inst<1, false, EPI_ENDPOINT>(mw, mh, prm, pl, st);
+  if (g.epilogue == EPI_FUSED)
+    return gather ? launch_inst<2, true, EPI_FUSED>(mw, mh, prm, pl, st)
+                  : launch_inst<2, false, EPI_FUSED>(mw, mh, prm, pl, st);
+  return gather ? launch_inst<2, true, EPI_ENDPOINT>(mw, mh, prm, pl, st)
+                : launch_inst<2, false, EPI_ENDPOINT>(mw, mh, prm, pl, st);
 }
 
 cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPlan& pl,

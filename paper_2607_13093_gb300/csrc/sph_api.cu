@@ -38,6 +38,10 @@ struct sph_ctx {
   long long tc_finish_wait = 1ll << 15;   // SPH_OPT_TC_FINISH_WAIT
   int sampler = 0;                  // SPH_OPT_SAMPLER
   int check_ids = 0;                // SPH_OPT_CHECK_IDS
+  // chunked split steps: the endpoint's own stream (created on first use
+  // when the caller passes none) and the events that order the two streams
+  cudaStream_t aux_stream = nullptr;
+  std::vector<cudaEvent_t> step_events;
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -133,8 +137,9 @@ bool use_tc(const sph_ctx* ctx, int64_t rows, int w_dtype) {
 }
 
 size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_bf16,
-                int w_dtype, int endpoint) {
+                int w_dtype, int endpoint, int sm_count = 0) {
   if (!use_tc(ctx, rows, w_dtype)) return 0;
+  if (sm_count <= 0) sm_count = ctx->sm_count;
   size_t b = 0;
   // the larger of the two paths, for the plan the call makes (tile height
   // as set, 0 automatic) and, with the automatic height, for both heights
@@ -142,7 +147,7 @@ size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_
   for (int gather = 0; gather < 2; ++gather)
     for (int tm = 0; tm <= 256; tm += 128) {
       if (ctx->tc_tile_m && tm != ctx->tc_tile_m) continue;
-      const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, ctx->sm_count,
+      const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, sm_count,
                                     endpoint, ctx->tc_schedule, ctx->tc_stages,
                                     ctx->tc_block_k, gather, w_dtype == sph::W_FP8,
                                     ctx->tc_max_bn, tm)
@@ -169,6 +174,43 @@ size_t fuse_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K
 // verification over `rows` = sessions * (k + 1) target rows, for any split
 size_t verify_reserve_bytes(int64_t rows, int64_t n) {
   return sph::verify_scratch_bytes((int)rows, 0, (int)n) + 2 * align_up((size_t)rows * 4, 256);
+}
+
+// SMs of the two halves of a chunked split step: the endpoint's share is its
+// share of the hidden dimension (at least 4 SMs, at most half)
+void split_sms(const sph_ctx* ctx, int64_t d_l, int64_t d_h, int* sm_cloud, int* sm_end) {
+  int e = (int)((double)ctx->sm_count * (double)d_l / (double)(d_l + d_h) + 0.5);
+  if (e < 4) e = 4;
+  if (e > ctx->sm_count / 2) e = ctx->sm_count / 2;
+  if (e < 1) e = 1;
+  *sm_end = e;
+  *sm_cloud = ctx->sm_count - e > 0 ? ctx->sm_count - e : 1;
+}
+// Scratch of sph_split_step with chunks of L ids (L = n for one chunk), in
+// the order the call carves it.
+size_t split_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t L, int64_t d_h,
+                           int64_t d_l, int act_bf16, int w_dtype) {
+  const bool chunked = L < n;
+  int smc = ctx->sm_count, sme = ctx->sm_count;
+  if (chunked) split_sms(ctx, d_l, d_h, &smc, &sme);
+  const int64_t last = n - (n - 1) / L * L;
+  size_t b = align_up((size_t)rows * L * 4, 256) + align_up((size_t)rows * 4, 256);
+  size_t tcc = tc_bytes(ctx, rows, L, d_h, act_bf16, w_dtype, 0, smc);
+  const size_t tcc2 = tc_bytes(ctx, rows, last, d_h, act_bf16, w_dtype, 0, smc);
+  b += align_up(tcc > tcc2 ? tcc : tcc2, 256);
+  b += align_up((size_t)rows * n * 4, 256);                          // z
+  b += align_up((size_t)rows * (n / 1024 + 2) * 8, 256);             // chunk statistics
+  if (chunked) {
+    size_t tce = tc_bytes(ctx, rows, L, d_l, 0, sph::W_BF16, 1, sme);
+    const size_t tce2 = tc_bytes(ctx, rows, last, d_l, 0, sph::W_BF16, 1, sme);
+    b += align_up(tce > tce2 ? tce : tce2, 256);
+    b += align_up((size_t)rows * sph::seg_count((int)n) * 8, 256);   // segment statistics
+  } else {
+    const size_t tce = tc_bytes(ctx, rows, n, d_l, 0, sph::W_BF16, 1);
+    const size_t st = (size_t)rows * sph::seg_count((int)n) * 8;
+    b += align_up(tce > st ? tce : st, 256);
+  }
+  return b + 4096;
 }
 
 bool finite_pos(float x) { return std::isfinite(x) && x > 0.f; }
@@ -241,6 +283,84 @@ cudaError_t traced(sph_ctx* ctx, int cls, F&& launch) {
   cudaEventRecord(b, ctx->stream);
   ctx->pending.push_back({cls, a, b});
   return e;
+}
+
+// traced() for a launch group that reports an sph_status
+template <class F>
+sph_status traced_status(sph_ctx* ctx, int cls, F&& launch) {
+  sph_status st = SPH_OK;
+  traced(ctx, cls, [&] {
+    st = launch();
+    return cudaSuccess;
+  });
+  return st;
+}
+
+// The endpoint half of a step on a prepared GatherGemm (EPI_ENDPOINT or
+// EPI_FUSED, gg.Y = z): the local contraction with its fused epilogue, then
+// the draw (S7-S11), on the context's stream.  `c` carves the rest of the
+// scratch arena.
+sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temperature,
+                         uint64_t seed, uint64_t offset, int32_t* tokens) {
+  const int rows = gg.rows, n_keep = gg.n;
+  const int32_t* keep_ids = gg.ids;
+  float* Z = gg.Y;
+  float2* cstats = static_cast<float2*>(c.take((size_t)rows * (n_keep / 1024 + 2) * 8));
+  gg.status = ctx->status; gg.finish_wait = ctx->tc_finish_wait;
+  gg.inv_tau = stats_inv_tau(temperature);
+  const int greedy = temperature == 0.f;
+  // Gumbel-max draws need no softmax statistics: the epilogue skips them
+  const bool gumbel = ctx->sampler == 1 && !greedy;
+  gg.no_stats = gumbel;
+  sph_status st;
+  auto draw_gumbel = [&] {
+    return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
+                           return sph::launch_gumbel(Z, rows, n_keep, keep_ids,
+                                                     gg.inv_tau, seed, offset, tokens,
+                                                     ctx->stream);
+                         }), "sample launch");
+  };
+  if (use_tc(ctx, rows, sph::W_BF16)) {
+    const sph::TcPlan pl = sph::tc_plan(rows, n_keep, gg.K, 0,
+                                        ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
+                                        ctx->tc_block_k, keep_ids != nullptr, 0,
+                                        ctx->tc_max_bn, ctx->tc_tile_m);
+    void* tcs = c.take(pl.scratch_bytes);
+    if (!c.fits())
+      return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
+                  c.off, ctx->scratch_cap);
+    st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
+                         return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
+                       }), "tensor-core launch");
+    if (st) return st;
+    if (gumbel) return draw_gumbel();
+    return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
+                           return sph::launch_sample_from_stats(
+                               Z, rows, n_keep, pl, tcs, cstats, keep_ids,
+                               gg.inv_tau, seed, offset, ctx->sm_count, tokens,
+                               ctx->stream, greedy);
+                         }), "sample launch");
+  }
+  float2* stats = static_cast<float2*>(c.take((size_t)rows * sph::seg_count(n_keep) * 8));
+  if (!c.fits())
+    return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
+                c.off, ctx->scratch_cap);
+  st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
+                       return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
+                     }), "gemv launch");
+  if (st) return st;
+  if (gumbel) return draw_gumbel();
+  return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
+                         cudaError_t e = sph::launch_seg_stats(Z, rows, n_keep,
+                                                               gg.inv_tau, stats,
+                                                               cstats, ctx->sm_count,
+                                                               ctx->stream);
+                         if (e != cudaSuccess) return e;
+                         return sph::launch_sample_segments(
+                             Z, rows, n_keep, stats, sph::seg_count(n_keep),
+                             cstats, keep_ids, gg.inv_tau, seed, offset, tokens,
+                             ctx->stream, greedy);
+                       }), "sample launch");
 }
 
 }  // namespace
@@ -369,6 +489,8 @@ sph_status sph_destroy(sph_ctx* ctx) {
   cudaStreamSynchronize(ctx->stream);
   if (ctx->scratch) cudaFree(ctx->scratch);
   if (ctx->status) cudaFree(ctx->status);
+  if (ctx->aux_stream) cudaStreamDestroy(ctx->aux_stream);
+  for (auto ev : ctx->step_events) cudaEventDestroy(ev);
   for (auto& p : ctx->pending) { cudaEventDestroy(p.start); cudaEventDestroy(p.stop); }
   for (auto ev : ctx->pool) cudaEventDestroy(ev);
   delete ctx;
@@ -445,6 +567,11 @@ sph_status sph_reserve(sph_ctx* ctx, int64_t max_rows, int64_t max_n_keep,
   if (f > need) need = f;
   const size_t v = verify_reserve_bytes(max_rows, max_n_keep);
   if (v > need) need = v;
+  for (int act = 0; act < 2; ++act) {      // a one-chunk split step
+    const size_t a = split_scratch_bytes(ctx, max_rows, max_n_keep, max_n_keep, max_d, max_d,
+                                         act, sph::W_BF16);
+    if (a > need) need = a;
+  }
   return ensure_scratch(ctx, need);
 }
 
@@ -638,66 +765,13 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   Carve c(ctx->scratch, ctx->scratch_cap);
   float* Z = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
   if (fused_logits_out) Z = fused_logits_out;
-  float2* cstats = static_cast<float2*>(c.take((size_t)rows * (n_keep / 1024 + 2) * 8));
   sph::GatherGemm gg{};
   gg.h = h_local; gg.ld_h = ld_hl; gg.rows = (int)rows;
   gg.W = W_l; gg.ld_w = ld_wl; gg.V = V; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
   gg.ids = keep_ids; gg.n = (int)n_keep;
   gg.epilogue = sph::EPI_ENDPOINT;
-  gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale; gg.status = ctx->status; gg.finish_wait = ctx->tc_finish_wait;
-  gg.inv_tau = stats_inv_tau(temperature);
-  const int greedy = temperature == 0.f;
-  // Gumbel-max draws need no softmax statistics: the epilogue skips them
-  const bool gumbel = ctx->sampler == 1 && !greedy;
-  gg.no_stats = gumbel;
-  auto draw_gumbel = [&] {
-    return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
-                           return sph::launch_gumbel(Z, (int)rows, (int)n_keep, keep_ids,
-                                                     gg.inv_tau, seed, offset, tokens,
-                                                     ctx->stream);
-                         }), "sample launch");
-  };
-  if (use_tc(ctx, rows, sph::W_BF16)) {
-    const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_l, 0,
-                                        ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
-                                        ctx->tc_block_k, keep_ids != nullptr, 0,
-                                        ctx->tc_max_bn, ctx->tc_tile_m);
-    void* tcs = c.take(pl.scratch_bytes);
-    if (!c.fits())
-      return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
-                  c.off, ctx->scratch_cap);
-    st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
-                         return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
-                       }), "tensor-core launch");
-    if (st) return st;
-    if (gumbel) return draw_gumbel();
-    return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
-                           return sph::launch_sample_from_stats(
-                               Z, (int)rows, (int)n_keep, pl, tcs, cstats, keep_ids,
-                               gg.inv_tau, seed, offset, ctx->sm_count, tokens,
-                               ctx->stream, greedy);
-                         }), "sample launch");
-  }
-  float2* stats = static_cast<float2*>(c.take((size_t)rows * sph::seg_count((int)n_keep) * 8));
-  if (!c.fits())
-    return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
-                c.off, ctx->scratch_cap);
-  st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
-                       return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
-                     }), "gemv launch");
-  if (st) return st;
-  if (gumbel) return draw_gumbel();
-  return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
-                         cudaError_t e = sph::launch_seg_stats(Z, (int)rows, (int)n_keep,
-                                                               gg.inv_tau, stats,
-                                                               cstats, ctx->sm_count,
-                                                               ctx->stream);
-                         if (e != cudaSuccess) return e;
-                         return sph::launch_sample_segments(
-                             Z, (int)rows, (int)n_keep, stats, sph::seg_count((int)n_keep),
-                             cstats, keep_ids, gg.inv_tau, seed, offset, tokens,
-                             ctx->stream, greedy);
-                       }), "sample launch");
+  gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale;
+  return endpoint_draw(ctx, gg, c, temperature, seed, offset, tokens);
 }
 
 sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
@@ -736,6 +810,204 @@ sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
                                                    ctx->sm_count, ctx->stream,
                                                    temperature == 0.f);
                        }), "verify launch");
+}
+
+sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld_h,
+                          int64_t d_l, int64_t d_h, const void* W_h, sph_dtype w_dtype,
+                          const float* w_row_scale, int64_t ld_wh, const void* W_l,
+                          int64_t ld_wl, int64_t V, const float* bias,
+                          const int32_t* keep_ids, int64_t n_keep, float clip,
+                          sph_act_mode act_mode, float temperature, uint64_t seed,
+                          uint64_t offset, int64_t chunk, void* endpoint_stream,
+                          int8_t* codes, float* scales, int32_t* tokens,
+                          float* fused_logits_out, size_t* payload_bytes) {
+  if (!ctx) return SPH_ERR_INVALID_ARG;
+  if (!h || !W_h || !W_l || !codes || !scales || !tokens)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "h, W_h, W_l, codes, scales and tokens must be non-NULL");
+  if (rows < 1 || rows > (1 << 20)) return fail(ctx, SPH_ERR_INVALID_ARG, "rows=%lld out of [1, 2^20]", (long long)rows);
+  if (d_l < 1 || d_h < 1) return fail(ctx, SPH_ERR_INVALID_ARG, "d_l and d_h must be >= 1");
+  if (ld_h < d_l + d_h || ld_wh < d_h || ld_wl < d_l)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "ld_h >= d_l + d_h, ld_wh >= d_h and ld_wl >= d_l are required");
+  sph_status st = check_ids(ctx, keep_ids, n_keep, V);
+  if (st) return st;
+  if (!finite_pos(clip)) return fail(ctx, SPH_ERR_INVALID_ARG, "clip must be finite and > 0");
+  if (!valid_temperature(temperature)) return fail(ctx, SPH_ERR_INVALID_ARG, "temperature must be finite and >= 0");
+  if (w_dtype != SPH_DTYPE_BF16 && w_dtype != SPH_DTYPE_FP8_E4M3)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "unknown w_dtype %d", (int)w_dtype);
+  if (act_mode != SPH_ACT_FP32 && act_mode != SPH_ACT_BF16)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "unknown act_mode %d", (int)act_mode);
+  if (w_dtype == SPH_DTYPE_FP8_E4M3 && !w_row_scale)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "fp8 weights need w_row_scale");
+  const int esz = w_dtype == SPH_DTYPE_BF16 ? 2 : 1;
+  if (((uintptr_t)W_h & 15) || ((ld_wh * esz) & 15) || ((uintptr_t)W_l & 15) || ((ld_wl * 2) & 15))
+    return fail(ctx, SPH_ERR_INVALID_ARG, "W_h and W_l base addresses and row strides must be 16-byte aligned");
+  if (chunk < 0) return fail(ctx, SPH_ERR_INVALID_ARG, "chunk must be >= 0");
+  if (n_keep > sph::sample_max_n()) return fail(ctx, SPH_ERR_UNSUPPORTED, "n_keep above %d", sph::sample_max_n());
+  if (d_h > sph::gemv_max_k() || d_l > sph::gemv_max_k())
+    return fail(ctx, SPH_ERR_UNSUPPORTED, "d_h or d_l above %d", sph::gemv_max_k());
+  const int64_t L = (chunk == 0 || chunk >= n_keep) ? n_keep : chunk;
+  const int64_t nchunk = (n_keep + L - 1) / L;
+  if (payload_bytes) *payload_bytes = (size_t)rows * (size_t)n_keep + 4 * (size_t)rows * (size_t)nchunk;
+
+  DeviceGuard g(ctx->device);
+  if (!g.ok) return fail(ctx, SPH_ERR_CUDA, "cudaSetDevice(%d) failed", ctx->device);
+  st = host_check_ids(ctx, keep_ids, n_keep, V);
+  if (st) return st;
+  const int wdt = w_dtype == SPH_DTYPE_BF16 ? sph::W_BF16 : sph::W_FP8;
+  const int act_bf16 = act_mode == SPH_ACT_BF16;
+  st = ensure_scratch(ctx, split_scratch_bytes(ctx, rows, n_keep, L, d_h, d_l, act_bf16, wdt));
+  if (st) return st;
+  const bool chunked = nchunk > 1;
+  int sm_cloud = ctx->sm_count, sm_end = ctx->sm_count;
+  if (chunked) split_sms(ctx, d_l, d_h, &sm_cloud, &sm_end);
+
+  Carve c(ctx->scratch, ctx->scratch_cap);
+  float* Y = static_cast<float*>(c.take((size_t)rows * L * 4));
+  unsigned* rowmax = static_cast<unsigned*>(c.take((size_t)rows * 4));
+  const int64_t last = n_keep - (nchunk - 1) * L;
+  size_t tcc = tc_bytes(ctx, rows, L, d_h, act_bf16, wdt, 0, sm_cloud);
+  const size_t tcc2 = tc_bytes(ctx, rows, last, d_h, act_bf16, wdt, 0, sm_cloud);
+  void* cloud_tc = c.take(tcc > tcc2 ? tcc : tcc2);
+  float* Z = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
+  if (fused_logits_out) Z = fused_logits_out;
+
+  // the cloud half of chunk q (S1-S4; the quantization is the caller's)
+  auto cloud = [&](int64_t q, int64_t n_q, cudaStream_t s) -> sph_status {
+    const int64_t j0 = q * L;
+    sph::GatherGemm gg{};
+    gg.h = h + d_l; gg.ld_h = ld_h; gg.rows = (int)rows;
+    // the full vocabulary is cut by moving the weights' base to the chunk's
+    // first row (its ids are then 0 .. n_q - 1 again); a kept-id list by
+    // moving the list
+    gg.W = keep_ids ? W_h : static_cast<const char*>(W_h) + j0 * ld_wh * esz;
+    gg.ld_w = ld_wh; gg.V = keep_ids ? V : V - j0;
+    gg.w_dtype = wdt;
+    gg.w_scale = (w_row_scale && !keep_ids) ? w_row_scale + j0 : w_row_scale;
+    gg.K = (int)d_h;
+    gg.ids = keep_ids ? keep_ids + j0 : nullptr; gg.n = (int)n_q;
+    gg.act_bf16 = act_bf16;
+    gg.epilogue = sph::EPI_CLOUD;
+    gg.bias = (bias && !keep_ids) ? bias + j0 : bias; gg.clip = clip;
+    gg.Y = Y; gg.rowmax = rowmax; gg.status = ctx->status; gg.finish_wait = ctx->tc_finish_wait;
+    if (use_tc(ctx, rows, wdt)) {
+      const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_q, (int)d_h, act_bf16, sm_cloud, 0,
+                                          ctx->tc_schedule, ctx->tc_stages, ctx->tc_block_k,
+                                          keep_ids != nullptr, wdt == sph::W_FP8,
+                                          ctx->tc_max_bn, ctx->tc_tile_m);
+      if (pl.scratch_bytes > (tcc > tcc2 ? tcc : tcc2))
+        return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: cloud plan outgrew its scratch");
+      return launch_status(ctx, sph::launch_tc(gg, pl, cloud_tc, ctx->spin_limit, s),
+                           "tensor-core launch");
+    }
+    cudaError_t e = cudaMemsetAsync(rowmax, 0, (size_t)rows * 4, s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMemsetAsync");
+    return launch_status(ctx, sph::launch_gemv(gg, ctx->sm_count, s), "gemv launch");
+  };
+
+  if (!chunked) {
+    // one chunk: the cloud contraction, then the endpoint contraction whose
+    // epilogue quantizes the cloud's clipped partials itself (no separate
+    // quantize pass) and fuses them (S5-S10), then the draw
+    if (!c.fits())
+      return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
+                  c.off, ctx->scratch_cap);
+    st = traced_status(ctx, SPH_PROF_CLOUD_GEMM, [&] { return cloud(0, n_keep, ctx->stream); });
+    if (st) return st;
+    sph::GatherGemm gg{};
+    gg.h = h; gg.ld_h = ld_h; gg.rows = (int)rows;
+    gg.W = W_l; gg.ld_w = ld_wl; gg.V = V; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
+    gg.ids = keep_ids; gg.n = (int)n_keep;
+    gg.epilogue = sph::EPI_FUSED;
+    gg.yc = Y; gg.rowmax_in = rowmax; gg.codes_out = codes; gg.scale_out = scales;
+    gg.Y = Z;
+    return endpoint_draw(ctx, gg, c, temperature, seed, offset, tokens);
+  }
+
+  // chunks: the cloud emits chunk q (codes + a scale per row) on the
+  // context's stream while the endpoint fuses chunk q - 1 on its own stream
+  void* ecarve_tc;
+  size_t tce = tc_bytes(ctx, rows, L, d_l, 0, sph::W_BF16, 1, sm_end);
+  const size_t tce2 = tc_bytes(ctx, rows, last, d_l, 0, sph::W_BF16, 1, sm_end);
+  ecarve_tc = c.take(tce > tce2 ? tce : tce2);
+  float2* cstats = static_cast<float2*>(c.take((size_t)rows * (n_keep / 1024 + 2) * 8));
+  float2* stats = static_cast<float2*>(c.take((size_t)rows * sph::seg_count((int)n_keep) * 8));
+  if (!c.fits())
+    return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
+                c.off, ctx->scratch_cap);
+  cudaStream_t es = static_cast<cudaStream_t>(endpoint_stream);
+  if (!es) {
+    if (!ctx->aux_stream) {
+      cudaError_t e = cudaStreamCreateWithFlags(&ctx->aux_stream, cudaStreamNonBlocking);
+      if (e != cudaSuccess) { ctx->aux_stream = nullptr; return cuda_fail(ctx, e, "cudaStreamCreate"); }
+    }
+    es = ctx->aux_stream;
+  }
+  if (es == ctx->stream) return fail(ctx, SPH_ERR_INVALID_ARG, "endpoint_stream must differ from the context's stream");
+  while (ctx->step_events.size() < (size_t)nchunk + 2) {
+    cudaEvent_t ev = nullptr;
+    cudaError_t e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaEventCreate");
+    ctx->step_events.push_back(ev);
+  }
+  cudaEvent_t* ev = ctx->step_events.data();
+  cudaError_t e = cudaEventRecord(ev[0], ctx->stream);   // the endpoint follows earlier work
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(es, ev[0], 0);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "ordering the endpoint stream");
+  const float inv_tau = stats_inv_tau(temperature);
+  for (int64_t q = 0; q < nchunk; ++q) {
+    const int64_t j0 = q * L, n_q = q + 1 < nchunk ? L : last;
+    int8_t* codes_q = codes + j0 * rows;         // chunk-major payload
+    float* scales_q = scales + q * rows;
+    st = cloud(q, n_q, ctx->stream);
+    if (st) return st;
+    st = launch_status(ctx, sph::launch_quantize(Y, rowmax, (int)rows, (int)n_q, codes_q,
+                                                 scales_q, ctx->stream), "quantize launch");
+    if (st) return st;
+    e = cudaEventRecord(ev[q + 1], ctx->stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(es, ev[q + 1], 0);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "ordering the endpoint stream");
+    // the endpoint half of chunk q: z[:, j0 : j0 + n_q] (S7-S8); the
+    // statistics come from one pass over all of z after the last chunk
+    sph::GatherGemm gg{};
+    gg.h = h; gg.ld_h = ld_h; gg.rows = (int)rows;
+    gg.W = keep_ids ? W_l : static_cast<const char*>(W_l) + j0 * ld_wl * 2;
+    gg.ld_w = ld_wl; gg.V = keep_ids ? V : V - j0; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
+    gg.ids = keep_ids ? keep_ids + j0 : nullptr; gg.n = (int)n_q;
+    gg.epilogue = sph::EPI_ENDPOINT;
+    gg.codes = codes_q; gg.row_scale = scales_q;
+    gg.Y = Z + j0; gg.ldy = n_keep;
+    gg.status = ctx->status; gg.finish_wait = ctx->tc_finish_wait;
+    gg.inv_tau = inv_tau; gg.no_stats = true;
+    if (use_tc(ctx, rows, sph::W_BF16)) {
+      const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_q, (int)d_l, 0, sm_end, 1,
+                                          ctx->tc_schedule, ctx->tc_stages, ctx->tc_block_k,
+                                          keep_ids != nullptr, 0, ctx->tc_max_bn, ctx->tc_tile_m);
+      if (pl.scratch_bytes > (tce > tce2 ? tce : tce2))
+        return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: endpoint plan outgrew its scratch");
+      st = launch_status(ctx, sph::launch_tc(gg, pl, ecarve_tc, ctx->spin_limit, es),
+                         "tensor-core launch");
+    } else {
+      st = launch_status(ctx, sph::launch_gemv(gg, ctx->sm_count, es), "gemv launch");
+    }
+    if (st) return st;
+  }
+  // the draw over the whole fused row (S9-S11), on the endpoint's stream
+  const int greedy = temperature == 0.f;
+  if (ctx->sampler == 1 && !greedy) {
+    e = sph::launch_gumbel(Z, (int)rows, (int)n_keep, keep_ids, inv_tau, seed, offset, tokens, es);
+  } else {
+    e = sph::launch_seg_stats(Z, (int)rows, (int)n_keep, inv_tau, stats, cstats, ctx->sm_count, es);
+    if (e == cudaSuccess)
+      e = sph::launch_sample_segments(Z, (int)rows, (int)n_keep, stats,
+                                      sph::seg_count((int)n_keep), cstats, keep_ids, inv_tau,
+                                      seed, offset, tokens, es, greedy);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "sample launch");
+  // the call ends, on the context's stream, when the endpoint's work has
+  e = cudaEventRecord(ev[nchunk + 1], es);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->stream, ev[nchunk + 1], 0);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "joining the endpoint stream");
+  return SPH_OK;
 }
 
 }  // extern "C"

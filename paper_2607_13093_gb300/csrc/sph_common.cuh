@@ -129,6 +129,37 @@ struct SumOp {
   __device__ float operator()(float a, float b) const { return a + b; }
 };
 
+// ---------------------------------------------------------------------------
+// the int8 quantizer (Eq. 18 with b = 8), shared by the quantize kernel and
+// the fused endpoint epilogue so that both round identically
+// ---------------------------------------------------------------------------
+struct RowQuant {
+  float s;     // row scale fl32(max / 127)
+  float k;     // exact lift 2^64 for scales below 2^-64, else 1
+  float inv;   // fl32(1 / (s * k)); 0 for an all-zero row (codes 0)
+};
+// From the bit pattern of the row's clipped |max|.  A scale below 2^-64
+// (partials below about 1e-17) is lifted by the exact factor 2^64 on both
+// sides so that its reciprocal stays finite.
+__device__ __forceinline__ RowQuant row_quant(unsigned max_bits) {
+  RowQuant q;
+  q.s = __fdiv_rn(__uint_as_float(max_bits), 127.0f);
+  q.k = q.s < 0x1p-64f ? 0x1p64f : 1.f;
+  q.inv = q.s > 0.f ? __frcp_rn(q.s * q.k) : 0.f;
+  return q;
+}
+// code = round-half-even(y / s) in [-127, 127], as the exact product
+// (y k) * fl32(1 / (s k)) rounded once to an integer: one fused multiply-add
+// of 1.5 * 2^23, whose sum lies in [2^23, 2^24) where the fp32 grid is the
+// integers (|quotient| <= 127 here), so the FMA's round-to-nearest-even is
+// the integer rounding and the low bits are the code.  (y k is exact: k is a
+// power of two.)  This keeps the conversion on the FMA pipe.
+__device__ __forceinline__ int quantize_one(float y, float k, float inv_s) {
+  const float t = __fmaf_rn(y * k, inv_s, 12582912.0f);    // 1.5 * 2^23
+  const int q = __float_as_int(t) - 0x4B400000;            // bits of 1.5 * 2^23
+  return max(-127, min(127, q));
+}
+
 // Non-negative floats order like their bit patterns, so a row maximum of
 // |y| can be kept as an unsigned atomicMax.
 __device__ __forceinline__ void atomic_max_nonneg(unsigned int* addr, float v) {

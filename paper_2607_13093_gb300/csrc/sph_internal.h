@@ -12,6 +12,9 @@ namespace sph {
 enum Epilogue : int {
   EPI_CLOUD = 0,     // +bias, optional unclipped store, clip, row |max|
   EPI_ENDPOINT = 1,  // + code * row_scale (dequantized cloud partial)
+  EPI_FUSED = 2,     // endpoint that quantizes the cloud's clipped partials
+                     // itself: code = Q(yc), written out as the payload,
+                     // then + code * row_scale as EPI_ENDPOINT
 };
 
 enum WDtype : int { W_BF16 = 0, W_FP8 = 1 };
@@ -72,6 +75,12 @@ struct GatherGemm {
   const int8_t* codes;     // [rows, n]
   const float* row_scale;  // [rows]
   float inv_tau;           // 1 / temperature (softmax statistics)
+  int64_t ldy = 0;         // row stride of Y (z) in elements; 0: n
+  // EPI_FUSED: the cloud's clipped partials and row maxima in, the payload out
+  const float* yc = nullptr;            // [rows, n] clipped cloud partials
+  const unsigned* rowmax_in = nullptr;  // [rows] bits of their row |max|
+  int8_t* codes_out = nullptr;          // [rows, n] int8 codes (Eq. 18)
+  float* scale_out = nullptr;           // [rows] row scales
   unsigned* status;        // device error word
   long long finish_wait = 1ll << 15;   // split-tile finisher poll (cycles; 0: none)
   bool no_stats = false;   // endpoint: skip the softmax statistics (Gumbel-max draw)

@@ -93,6 +93,11 @@ _SIGNATURES = {
     "sph_fuse_sample": (_int, [_c_void_p, _c_void_p, _c_void_p, _i64, _c_void_p,
                                _i64, _c_void_p, _i64, _i64, _i64, _c_void_p,
                                _i64, _f32, _u64, _u64, _c_void_p, _c_void_p]),
+    "sph_split_step": (_int, [_c_void_p, _c_void_p, _i64, _i64, _i64, _i64, _c_void_p, _int,
+                              _c_void_p, _i64, _c_void_p, _i64, _i64, _c_void_p, _c_void_p,
+                              _i64, _f32, _int, _f32, _u64, _u64, _i64, _c_void_p,
+                              _c_void_p, _c_void_p, _c_void_p, _c_void_p,
+                              ctypes.POINTER(_sz)]),
     "sph_verify_draft": (_int, [_c_void_p, _c_void_p, _i64, _i64, _c_void_p,
                                 _i64, _f32, _c_void_p, _c_void_p, _u64, _u64,
                                 _c_void_p, _c_void_p]),
@@ -354,6 +359,58 @@ def sph_fuse_sample(ctx, codes, row_scale, h_local, W_l, *, keep_ids=None,
     return tokens
 
 
+def sph_split_step(ctx, h, d_l: int, W_h, W_l, *, keep_ids=None, clip=30.0,
+                   w_row_scale=None, bias=None, act_mode=SPH_ACT_FP32, temperature=1.0,
+                   seed=0, offset=0, chunk=0, endpoint_stream=None, codes=None,
+                   scales=None, tokens=None, fused_logits_out=None):
+    """The whole split step from the full hidden state h [R, d] (h[:, :d_l]
+    the endpoint's part, h[:, d_l:] the cloud's) to tokens.  Returns
+    (codes, scales, tokens, payload_bytes): the payload that would cross,
+    chunk-major (int8 [R * n] flat, fp32 [nchunk * R])."""
+    _need(h, torch.float32, "h")
+    if W_h.dtype == torch.bfloat16:
+        wdt = SPH_DTYPE_BF16
+    elif W_h.dtype == torch.float8_e4m3fn:
+        wdt = SPH_DTYPE_FP8_E4M3
+    else:
+        raise ValueError("W_h must be bfloat16 or float8_e4m3fn")
+    _need(W_h, None, "W_h")
+    _need(W_l, torch.bfloat16, "W_l")
+    _need(keep_ids, torch.int32, "keep_ids")
+    _need(w_row_scale, torch.float32, "w_row_scale")
+    _need(bias, torch.float32, "bias")
+    R = h.shape[0]
+    V, d_h = W_h.shape
+    n = V if keep_ids is None else keep_ids.numel()
+    L = n if (chunk == 0 or chunk >= n) else int(chunk)
+    nchunk = (n + L - 1) // L
+    dev = h.device
+    if codes is None:
+        codes = torch.empty(R * n, dtype=torch.int8, device=dev)
+    if scales is None:
+        scales = torch.empty(nchunk * R, dtype=torch.float32, device=dev)
+    if tokens is None:
+        tokens = torch.empty(R, dtype=torch.int32, device=dev)
+    _need(codes, torch.int8, "codes")
+    _need(scales, torch.float32, "scales")
+    _need(tokens, torch.int32, "tokens")
+    _need(fused_logits_out, torch.float32, "fused_logits_out")
+    if codes.numel() < R * n or scales.numel() < nchunk * R or tokens.numel() < R:
+        raise ValueError("codes, scales or tokens too small")
+    if fused_logits_out is not None and (tuple(fused_logits_out.shape) != (R, n)
+                                         or not fused_logits_out.is_contiguous()):
+        raise ValueError("fused_logits_out must be a contiguous (R, n) tensor")
+    pb = _sz(0)
+    _check(ctx, lib.sph_split_step(
+        ctx, _ptr(h), R, _ld(h), int(d_l), d_h, _ptr(W_h), wdt, _ptr(w_row_scale),
+        _ld(W_h), _ptr(W_l), _ld(W_l), V, _ptr(bias), _ptr(keep_ids), n, float(clip),
+        int(act_mode), float(temperature), int(seed) & 0xFFFFFFFFFFFFFFFF,
+        int(offset) & 0xFFFFFFFFFFFFFFFF, int(chunk),
+        ctypes.c_void_p(endpoint_stream or 0), _ptr(codes), _ptr(scales), _ptr(tokens),
+        _ptr(fused_logits_out), ctypes.byref(pb)))
+    return codes, scales, tokens, pb.value
+
+
 def sph_verify_draft(ctx, target_logits, sessions: int, k: int, draft_tokens,
                      *, keep_ids=None, draft_probs=None, temperature=1.0,
                      seed=0, offset=0, n_accepted=None, next_token=None):
@@ -411,6 +468,10 @@ class Context:
     def verify_draft(self, *a, **kw):
         self._follow_stream()
         return sph_verify_draft(self.handle, *a, **kw)
+
+    def split_step(self, *a, **kw):
+        self._follow_stream()
+        return sph_split_step(self.handle, *a, **kw)
 
     def sync(self):
         sph_sync(self.handle)

@@ -261,16 +261,23 @@ def make_workload(name: str = "custom", *, V: int, d: int, d_l: int, rows: int,
 
 
 def workload(name: str, device="cpu", rows: Optional[int] = None,
-             keep_frac: Optional[float] = None, d_l: Optional[int] = None) -> Workload:
+             keep_frac: Optional[float] = None, d_l: Optional[int] = None,
+             V: Optional[int] = None) -> Workload:
     """One of the named workloads at full size.  For "sweep" and "dend",
     `rows` and `keep_frac` pick the grid point (defaults: sweep 64 rows,
     100 %; dend 32 rows, 40 %), and for "dend" `d_l` the split dimension
-    (default 96, the paper's D_end)."""
+    (default 96, the paper's D_end).  `V` shrinks the vocabulary of "sweep"
+    or "dend" (the kept fraction stays), for small profiling captures of the
+    same kernel plan."""
     cfg = dict(WORKLOADS[name])
     num = cfg.pop("num")
     sessions = cfg.pop("sessions", 0)
     k = cfg.pop("k", 0)
     if name in ("sweep", "dend"):
+        if V is not None:
+            frac = cfg["n_keep"] / cfg["V"]
+            cfg["V"] = int(V)
+            cfg["n_keep"] = round(frac * cfg["V"])
         if rows is not None:
             cfg["rows"] = rows
         if keep_frac is not None:
