@@ -339,7 +339,7 @@ def roofline(w, act, unit_ms, peaks, mode="split"):
     R, n = w.rows, w.n_keep
     fp8 = w.w_dtype == "fp8"
     nosplit = mode == "nosplit"
-    whole = mode in ("fused", "chunked")
+    whole = mode in ("fused", "chunked", "chunked_serial")
     if nosplit:
         alg_bytes = n * w.d * 2 + 4 * R * w.d + 4 * n + 4 * R
         alg_flops = wl.algorithmic_flops(R, n, w.d)
@@ -381,7 +381,7 @@ def roofline(w, act, unit_ms, peaks, mode="split"):
     return out
 
 
-STEP_MODES = ("split", "fused", "chunked", "nosplit")
+STEP_MODES = ("split", "fused", "chunked", "chunked_serial", "nosplit")
 
 OPTION_NAMES = {"tc_min_rows": "SPH_OPT_TC_MIN_ROWS", "schedule": "SPH_OPT_TC_SCHEDULE",
                 "stages": "SPH_OPT_TC_STAGES", "block_k": "SPH_OPT_TC_BLOCK_K",
@@ -446,11 +446,15 @@ class Runner:
         hh = self.hs[c] if h is None else h
         if events is not None:
             events[0].record()
-        if self.mode in ("fused", "chunked"):
+        if self.mode in ("fused", "chunked", "chunked_serial"):
+            import torch
+            serial = self.mode == "chunked_serial"
             ctx.split_step(hh, w.d_l, self.Whs[c], self.Wls[c], keep_ids=w.keep_ids, clip=w.clip,
                            w_row_scale=w.w_scale, bias=w.bias, act_mode=self.act_mode,
                            temperature=w.tau, seed=w.seed, offset=i,
-                           chunk=self.chunk if self.mode == "chunked" else 0,
+                           chunk=0 if self.mode == "fused" else self.chunk,
+                           endpoint_stream=(torch.cuda.current_stream(self.dev).cuda_stream
+                                            if serial else None),
                            codes=self.codes.view(-1), scales=self.scales, tokens=self.tokens,
                            fused_logits_out=self.z)
             if events is not None:
@@ -625,10 +629,13 @@ CONFIG_BLOCK = [("tiny", None, None, None, "fp32", "split", 0),
                 # epilogue) and the block-streamed payload beside the two calls
                 ("decode", None, None, None, "fp32", "fused", 0),
                 ("decode", None, None, None, "fp32", "chunked", 4096),
+                ("decode", None, None, None, "fp32", "chunked_serial", 4096),
                 ("dend", None, 0.4, 96, "fp32", "fused", 0),
                 ("dend", None, 0.4, 96, "fp32", "chunked", 15000),
+                ("dend", None, 0.4, 96, "fp32", "chunked_serial", 15000),
                 ("sweep", 1024, 1.0, None, "fp32", "fused", 0),
                 ("sweep", 1024, 1.0, None, "fp32", "chunked", 64000),
+                ("sweep", 1024, 1.0, None, "fp32", "chunked_serial", 64000),
                 # the unsplit head (the no-split ablation)
                 ("decode", None, None, None, "fp32", "nosplit", 0)]
 DEND_GRID = [(k, d) for k in (0.4, 0.3) for d in (48, 96, 128, 256, 512)]
@@ -659,9 +666,10 @@ def config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks, cpu_seconds,
         roof = roofline(w, act, unit["mean_ms"], peaks, mode)
         roof["timing"] = res["timing"]
         roof["spread"] = unit
-        one_call = mode in ("fused", "chunked")
+        one_call = mode in ("fused", "chunked", "chunked_serial")
         entry = {"workload": describe(w), "activations": act,
-                 "step": mode + (f" ({r.nchunk} chunks of {chunk} ids)" if mode == "chunked" else ""),
+                 "step": mode + (f" ({r.nchunk} chunks of {chunk} ids)"
+                                 if mode.startswith("chunked") else ""),
                  "rows_per_s": round(job_rows_per_s(w.rows, 1, steps, res["ms"]), 1),
                  "ms_per_step": round(res["ms"] / steps, 5), "steps": steps,
                  ("step_call_us" if one_call else "cloud_us"): round(unit["mean_ms"] * 1e3, 2),
@@ -757,7 +765,9 @@ def run_ours(args):
               "split": ("cloud call: operand split + gathered tcgen05 contraction + int8 "
                         "quantization"),
               "fused": "the one-call split step (cloud + endpoint, one payload chunk)",
-              "chunked": f"the one-call split step, {r.nchunk} payload chunks on two streams"}
+              "chunked": f"the one-call split step, {r.nchunk} payload chunks on two streams",
+              "chunked_serial": (f"the one-call split step, {r.nchunk} payload chunks one "
+                                 "after another on one stream")}
     roof.update({"traffic": traffic_for(f"cloud_{args.workload}_{R}_{n}_{args.act}")
                  if args.step == "split" else None,
                  "kernel": kernel[args.step],
@@ -775,7 +785,9 @@ def run_ours(args):
         "config": {"workload": describe(w) + {
                        "split": "", "nosplit": ", unsplit head (no-split ablation)",
                        "fused": ", one-call split step",
-                       "chunked": f", one-call split step, {r.nchunk} payload chunks"}[args.step],
+                       "chunked": f", one-call split step, {r.nchunk} payload chunks",
+                       "chunked_serial": f", one-call split step, {r.nchunk} payload chunks "
+                                         "(serial)"}[args.step],
                    "rows_per_gpu": R, "n_keep": n,
                    "d_h": w.d_h, "d_l": w.d_l, "V": w.V, "weights": w.w_dtype,
                    "accumulate": "fp32",

@@ -390,7 +390,9 @@ sph_status sph_fuse_sample(sph_ctx* ctx,
  *   endpoint_stream  a cudaStream_t other than the context's, or NULL for
  *            one the context creates on first use and owns; used only when
  *            there is more than one chunk.  The call's work is complete, on
- *            the context's stream, when the endpoint's is.
+ *            the context's stream, when the endpoint's is.  The context's
+ *            own stream runs the chunks one after another instead, each
+ *            kernel with every SM (the same results, without the overlap).
  *   codes    int8, rows * n_keep bytes (out), chunk-major: chunk q is the
  *            row-major [rows][its ids] block starting at byte
  *            q * chunk * rows.  One chunk: [rows, n_keep].

@@ -176,10 +176,16 @@ size_t verify_reserve_bytes(int64_t rows, int64_t n) {
   return sph::verify_scratch_bytes((int)rows, 0, (int)n) + 2 * align_up((size_t)rows * 4, 256);
 }
 
-// SMs of the two halves of a chunked split step: the endpoint's share is its
-// share of the hidden dimension (at least 4 SMs, at most half)
-void split_sms(const sph_ctx* ctx, int64_t d_l, int64_t d_h, int* sm_cloud, int* sm_end) {
-  int e = (int)((double)ctx->sm_count * (double)d_l / (double)(d_l + d_h) + 0.5);
+// SMs of the two halves of a chunked split step, in proportion to their
+// cost per (row, id): the cloud's contraction over d_h in its operand
+// planes (two for fp32 activations), the endpoint's over d_l in two planes
+// plus its epilogue, which costs about as much as 1400 more columns
+// (measured: 1024 rows x 256000 ids, cloud 3.17 ms over 4608 x 2, endpoint
+// 0.82 ms over 512 x 2).  At least 4 SMs, at most half.
+void split_sms(const sph_ctx* ctx, int64_t d_l, int64_t d_h, int act_bf16, int* sm_cloud,
+               int* sm_end) {
+  const double cloud = (double)d_h * (act_bf16 ? 1 : 2), end = 2.0 * (double)d_l + 1400.0;
+  int e = (int)((double)ctx->sm_count * end / (cloud + end) + 0.5);
   if (e < 4) e = 4;
   if (e > ctx->sm_count / 2) e = ctx->sm_count / 2;
   if (e < 1) e = 1;
@@ -192,18 +198,25 @@ size_t split_scratch_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t 
                            int64_t d_l, int act_bf16, int w_dtype) {
   const bool chunked = L < n;
   int smc = ctx->sm_count, sme = ctx->sm_count;
-  if (chunked) split_sms(ctx, d_l, d_h, &smc, &sme);
+  if (chunked) split_sms(ctx, d_l, d_h, act_bf16, &smc, &sme);
   const int64_t last = n - (n - 1) / L * L;
+  // the larger of a chunk's plans, with the split SMs or (chunks one after
+  // another on one stream) all of them
+  auto plan_bytes = [&](int64_t K, int act, int wdt, int endpoint, int sm) {
+    size_t x = 0;
+    for (int64_t nq : {L, last})
+      for (int s2 : {sm, ctx->sm_count}) {
+        const size_t y = tc_bytes(ctx, rows, nq, K, act, wdt, endpoint, s2);
+        if (y > x) x = y;
+      }
+    return x;
+  };
   size_t b = align_up((size_t)rows * L * 4, 256) + align_up((size_t)rows * 4, 256);
-  size_t tcc = tc_bytes(ctx, rows, L, d_h, act_bf16, w_dtype, 0, smc);
-  const size_t tcc2 = tc_bytes(ctx, rows, last, d_h, act_bf16, w_dtype, 0, smc);
-  b += align_up(tcc > tcc2 ? tcc : tcc2, 256);
+  b += align_up(plan_bytes(d_h, act_bf16, w_dtype, 0, smc), 256);
   b += align_up((size_t)rows * n * 4, 256);                          // z
   b += align_up((size_t)rows * (n / 1024 + 2) * 8, 256);             // chunk statistics
   if (chunked) {
-    size_t tce = tc_bytes(ctx, rows, L, d_l, 0, sph::W_BF16, 1, sme);
-    const size_t tce2 = tc_bytes(ctx, rows, last, d_l, 0, sph::W_BF16, 1, sme);
-    b += align_up(tce > tce2 ? tce : tce2, 256);
+    b += align_up(plan_bytes(d_l, 0, sph::W_BF16, 1, sme), 256);
     b += align_up((size_t)rows * sph::seg_count((int)n) * 8, 256);   // segment statistics
   } else {
     const size_t tce = tc_bytes(ctx, rows, n, d_l, 0, sph::W_BF16, 1);
@@ -858,8 +871,11 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
   st = ensure_scratch(ctx, split_scratch_bytes(ctx, rows, n_keep, L, d_h, d_l, act_bf16, wdt));
   if (st) return st;
   const bool chunked = nchunk > 1;
+  // the endpoint's chunks on the context's own stream: one after another,
+  // each with every SM
+  const bool serial = chunked && endpoint_stream == static_cast<void*>(ctx->stream);
   int sm_cloud = ctx->sm_count, sm_end = ctx->sm_count;
-  if (chunked) split_sms(ctx, d_l, d_h, &sm_cloud, &sm_end);
+  if (chunked && !serial) split_sms(ctx, d_l, d_h, act_bf16, &sm_cloud, &sm_end);
 
   Carve c(ctx->scratch, ctx->scratch_cap);
   float* Y = static_cast<float*>(c.take((size_t)rows * L * 4));
@@ -867,7 +883,8 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
   const int64_t last = n_keep - (nchunk - 1) * L;
   size_t tcc = tc_bytes(ctx, rows, L, d_h, act_bf16, wdt, 0, sm_cloud);
   const size_t tcc2 = tc_bytes(ctx, rows, last, d_h, act_bf16, wdt, 0, sm_cloud);
-  void* cloud_tc = c.take(tcc > tcc2 ? tcc : tcc2);
+  if (tcc2 > tcc) tcc = tcc2;
+  void* cloud_tc = c.take(tcc);
   float* Z = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
   if (fused_logits_out) Z = fused_logits_out;
 
@@ -894,7 +911,7 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
                                           ctx->tc_schedule, ctx->tc_stages, ctx->tc_block_k,
                                           keep_ids != nullptr, wdt == sph::W_FP8,
                                           ctx->tc_max_bn, ctx->tc_tile_m);
-      if (pl.scratch_bytes > (tcc > tcc2 ? tcc : tcc2))
+      if (pl.scratch_bytes > tcc)
         return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: cloud plan outgrew its scratch");
       return launch_status(ctx, sph::launch_tc(gg, pl, cloud_tc, ctx->spin_limit, s),
                            "tensor-core launch");
@@ -928,31 +945,35 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
   void* ecarve_tc;
   size_t tce = tc_bytes(ctx, rows, L, d_l, 0, sph::W_BF16, 1, sm_end);
   const size_t tce2 = tc_bytes(ctx, rows, last, d_l, 0, sph::W_BF16, 1, sm_end);
-  ecarve_tc = c.take(tce > tce2 ? tce : tce2);
+  if (tce2 > tce) tce = tce2;
+  ecarve_tc = c.take(tce);
   float2* cstats = static_cast<float2*>(c.take((size_t)rows * (n_keep / 1024 + 2) * 8));
   float2* stats = static_cast<float2*>(c.take((size_t)rows * sph::seg_count((int)n_keep) * 8));
   if (!c.fits())
     return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
                 c.off, ctx->scratch_cap);
   cudaStream_t es = static_cast<cudaStream_t>(endpoint_stream);
-  if (!es) {
+  if (!es && !serial) {
     if (!ctx->aux_stream) {
       cudaError_t e = cudaStreamCreateWithFlags(&ctx->aux_stream, cudaStreamNonBlocking);
       if (e != cudaSuccess) { ctx->aux_stream = nullptr; return cuda_fail(ctx, e, "cudaStreamCreate"); }
     }
     es = ctx->aux_stream;
   }
-  if (es == ctx->stream) return fail(ctx, SPH_ERR_INVALID_ARG, "endpoint_stream must differ from the context's stream");
-  while (ctx->step_events.size() < (size_t)nchunk + 2) {
+  if (serial) es = ctx->stream;
+  while (!serial && ctx->step_events.size() < (size_t)nchunk + 2) {
     cudaEvent_t ev = nullptr;
     cudaError_t e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaEventCreate");
     ctx->step_events.push_back(ev);
   }
   cudaEvent_t* ev = ctx->step_events.data();
-  cudaError_t e = cudaEventRecord(ev[0], ctx->stream);   // the endpoint follows earlier work
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(es, ev[0], 0);
-  if (e != cudaSuccess) return cuda_fail(ctx, e, "ordering the endpoint stream");
+  cudaError_t e = cudaSuccess;
+  if (!serial) {
+    e = cudaEventRecord(ev[0], ctx->stream);   // the endpoint follows earlier work
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(es, ev[0], 0);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "ordering the endpoint stream");
+  }
   const float inv_tau = stats_inv_tau(temperature);
   for (int64_t q = 0; q < nchunk; ++q) {
     const int64_t j0 = q * L, n_q = q + 1 < nchunk ? L : last;
@@ -963,9 +984,11 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
     st = launch_status(ctx, sph::launch_quantize(Y, rowmax, (int)rows, (int)n_q, codes_q,
                                                  scales_q, ctx->stream), "quantize launch");
     if (st) return st;
-    e = cudaEventRecord(ev[q + 1], ctx->stream);
-    if (e == cudaSuccess) e = cudaStreamWaitEvent(es, ev[q + 1], 0);
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "ordering the endpoint stream");
+    if (!serial) {
+      e = cudaEventRecord(ev[q + 1], ctx->stream);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(es, ev[q + 1], 0);
+      if (e != cudaSuccess) return cuda_fail(ctx, e, "ordering the endpoint stream");
+    }
     // the endpoint half of chunk q: z[:, j0 : j0 + n_q] (S7-S8); the
     // statistics come from one pass over all of z after the last chunk
     sph::GatherGemm gg{};
@@ -982,7 +1005,7 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
       const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_q, (int)d_l, 0, sm_end, 1,
                                           ctx->tc_schedule, ctx->tc_stages, ctx->tc_block_k,
                                           keep_ids != nullptr, 0, ctx->tc_max_bn, ctx->tc_tile_m);
-      if (pl.scratch_bytes > (tce > tce2 ? tce : tce2))
+      if (pl.scratch_bytes > tce)
         return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: endpoint plan outgrew its scratch");
       st = launch_status(ctx, sph::launch_tc(gg, pl, ecarve_tc, ctx->spin_limit, es),
                          "tensor-core launch");
@@ -1003,6 +1026,7 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
                                       seed, offset, tokens, es, greedy);
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "sample launch");
+  if (serial) return SPH_OK;
   // the call ends, on the context's stream, when the endpoint's work has
   e = cudaEventRecord(ev[nchunk + 1], es);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->stream, ev[nchunk + 1], 0);
