@@ -142,6 +142,13 @@ typedef enum sph_option {
                                returning SPH_ERR_INVALID_ARG for unsorted,
                                repeated or out-of-range ids.  0 (default):
                                the ids are a precondition, not checked.    */
+  SPH_OPT_SPLIT_QUANTIZE = 10, /* sph_split_step with one payload chunk: 0
+                               automatic (default: in the endpoint's epilogue
+                               for at most 2^20 rows x ids, else a separate
+                               pass), 1 always in the endpoint contraction's
+                               epilogue, 2 always a separate quantize pass.
+                               The payload, z and tokens are bit-identical
+                               either way.                                  */
   SPH_OPT_SAMPLER = 8       /* the draw of sph_fuse_sample at temperature > 0:
                                0 inverse CDF (default), 1 Gumbel-max: the
                                first index j of the largest
@@ -375,10 +382,11 @@ sph_status sph_fuse_sample(sph_ctx* ctx,
  *            sph_fuse_sample;  temperature, seed, offset  as there too (the
  *            draw is the same: purpose 0 of row r).
  *   chunk    kept ids per payload chunk.  0 (or >= n_keep): one chunk, the
- *            payload of sph_partial_logits (one scale per row); the
- *            endpoint's contraction then quantizes the cloud's clipped
- *            partials in its own epilogue, so no separate quantization pass
- *            runs.  1 <= chunk < n_keep: block streaming (the GPU form of
+ *            payload of sph_partial_logits (one scale per row); for small
+ *            payloads the endpoint's contraction then quantizes the cloud's
+ *            clipped partials in its own epilogue, so no separate
+ *            quantization pass runs (SPH_OPT_SPLIT_QUANTIZE).
+ *            1 <= chunk < n_keep: block streaming (the GPU form of
  *            the paper's block-wise streaming in Sec. "Device-Adaptive
  *            Feature Preparation"): chunk q holds the ids
  *            q*chunk .. min(n_keep, (q+1)*chunk) - 1 and carries its own

@@ -38,6 +38,7 @@ struct sph_ctx {
   long long tc_finish_wait = 1ll << 15;   // SPH_OPT_TC_FINISH_WAIT
   int sampler = 0;                  // SPH_OPT_SAMPLER
   int check_ids = 0;                // SPH_OPT_CHECK_IDS
+  int split_quantize = 0;           // SPH_OPT_SPLIT_QUANTIZE
   // chunked split steps: the endpoint's own stream (created on first use
   // when the caller passes none) and the events that order the two streams
   cudaStream_t aux_stream = nullptr;
@@ -629,6 +630,10 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "sampler must be 0 or 1");
       ctx->sampler = (int)value;
       return SPH_OK;
+    case SPH_OPT_SPLIT_QUANTIZE:
+      if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "split_quantize must be 0, 1 or 2");
+      ctx->split_quantize = (int)value;
+      return SPH_OK;
     case SPH_OPT_CHECK_IDS:
       if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "check_ids must be 0 or 1");
       ctx->check_ids = (int)value;
@@ -922,21 +927,39 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
   };
 
   if (!chunked) {
-    // one chunk: the cloud contraction, then the endpoint contraction whose
-    // epilogue quantizes the cloud's clipped partials itself (no separate
-    // quantize pass) and fuses them (S5-S10), then the draw
+    // one chunk: the cloud contraction, then either the endpoint
+    // contraction whose epilogue quantizes the cloud's clipped partials
+    // itself and fuses them (no separate quantize launch: faster where the
+    // payload is small and the launch's fixed cost weighs most), or the
+    // quantize pass and the ordinary endpoint epilogue (faster for large
+    // payloads, where the fused epilogue's fp32 reads are not hidden behind
+    // the short endpoint contraction); then the draw.  Measured: decode (32
+    // x 12000 ids) 47.4 vs 48.6 us a step fused; 32 x 60000 ids and 1024 x
+    // 256000 ids slower fused.
     if (!c.fits())
       return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
                   c.off, ctx->scratch_cap);
     st = traced_status(ctx, SPH_PROF_CLOUD_GEMM, [&] { return cloud(0, n_keep, ctx->stream); });
     if (st) return st;
+    const bool fuse_q = ctx->split_quantize == 1 ||
+                        (ctx->split_quantize == 0 && rows * n_keep <= ((int64_t)1 << 20));
     sph::GatherGemm gg{};
     gg.h = h; gg.ld_h = ld_h; gg.rows = (int)rows;
     gg.W = W_l; gg.ld_w = ld_wl; gg.V = V; gg.w_dtype = sph::W_BF16; gg.K = (int)d_l;
     gg.ids = keep_ids; gg.n = (int)n_keep;
-    gg.epilogue = sph::EPI_FUSED;
-    gg.yc = Y; gg.rowmax_in = rowmax; gg.codes_out = codes; gg.scale_out = scales;
     gg.Y = Z;
+    if (fuse_q) {
+      gg.epilogue = sph::EPI_FUSED;
+      gg.yc = Y; gg.rowmax_in = rowmax; gg.codes_out = codes; gg.scale_out = scales;
+    } else {
+      st = launch_status(ctx, traced(ctx, SPH_PROF_QUANTIZE, [&] {
+                           return sph::launch_quantize(Y, rowmax, (int)rows, (int)n_keep, codes,
+                                                       scales, ctx->stream);
+                         }), "quantize launch");
+      if (st) return st;
+      gg.epilogue = sph::EPI_ENDPOINT;
+      gg.codes = codes; gg.row_scale = scales;
+    }
     return endpoint_draw(ctx, gg, c, temperature, seed, offset, tokens);
   }
 

@@ -31,6 +31,7 @@ SPH_OPT_TC_TILE_M = 6
 SPH_OPT_TC_FINISH_WAIT = 7
 SPH_OPT_SAMPLER = 8
 SPH_OPT_CHECK_IDS = 9
+SPH_OPT_SPLIT_QUANTIZE = 10
 SPH_SAMPLER_CDF, SPH_SAMPLER_GUMBEL = 0, 1
 
 _c_void_p = ctypes.c_void_p

@@ -144,15 +144,22 @@ def test_split_step_bf16_activations(path_ctx, rows):
     check_split(path_ctx, small(V=3000, d=776, d_l=64, rows=rows, n_keep=1200), 0, act="bf16")
 
 
-def test_split_step_equals_the_two_calls(ctx):
+@pytest.mark.parametrize("where", [1, 2], ids=["epilogue", "pass"])
+def test_split_step_equals_the_two_calls(ctx, where):
     # one chunk: the fused epilogue rounds exactly as the quantize kernel,
     # and the endpoint's contraction is the same, so the payload, the fused
-    # logits and the tokens are bit-identical to the two calls'
+    # logits and the tokens are bit-identical to the two calls', whether the
+    # quantization runs in the endpoint's epilogue or as its own pass
+    from paper_2607_13093_gb300 import sph
     for kw in (dict(V=4000, d=1024, d_l=128, rows=32, n_keep=1500, tau=0.8),
                dict(V=2000, d=312, d_l=40, rows=3, n_keep=700),
                dict(V=6000, d=2112, d_l=64, rows=160, n_keep=5000)):
         w = small(**kw)
-        c, s, tok, z, _ = run_gpu(ctx, w, 0)
+        ctx.set_option(sph.SPH_OPT_SPLIT_QUANTIZE, where)
+        try:
+            c, s, tok, z, _ = run_gpu(ctx, w, 0)
+        finally:
+            ctx.set_option(sph.SPH_OPT_SPLIT_QUANTIZE, 0)
         codes2, scale2, _ = ctx.partial_logits(w.h_cloud, w.W_h, keep_ids=w.keep_ids,
                                                clip=w.clip)
         z2 = torch.empty(w.rows, w.n_keep, device=DEV)
