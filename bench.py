@@ -386,7 +386,8 @@ STEP_MODES = ("split", "fused", "chunked", "chunked_serial", "nosplit")
 OPTION_NAMES = {"tc_min_rows": "SPH_OPT_TC_MIN_ROWS", "schedule": "SPH_OPT_TC_SCHEDULE",
                 "stages": "SPH_OPT_TC_STAGES", "block_k": "SPH_OPT_TC_BLOCK_K",
                 "max_bn": "SPH_OPT_TC_MAX_BN", "tile_m": "SPH_OPT_TC_TILE_M",
-                "finish_wait": "SPH_OPT_TC_FINISH_WAIT", "split_quantize": "SPH_OPT_SPLIT_QUANTIZE"}
+                "finish_wait": "SPH_OPT_TC_FINISH_WAIT", "split_quantize": "SPH_OPT_SPLIT_QUANTIZE",
+                "pair": "SPH_OPT_TC_PAIR"}
 
 
 class Runner:

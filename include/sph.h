@@ -142,6 +142,17 @@ typedef enum sph_option {
                                returning SPH_ERR_INVALID_ARG for unsorted,
                                repeated or out-of-range ids.  0 (default):
                                the ids are a precondition, not checked.    */
+  SPH_OPT_TC_PAIR = 11,     /* CTA pairs for the cloud contraction with bf16
+                               weights (clusters of two CTAs, tcgen05
+                               .cta_group::2): each 256-id tile is one M = 256
+                               MMA over both CTAs' shared memory, each CTA
+                               loading 128 ids of the weights and half of the
+                               hidden-state rows.  0 (default): where the row
+                               blocks are long (>= 192 rows, or >= 128 with
+                               bf16 activations); 1: always (SPH_ERR_
+                               UNSUPPORTED where pairs cannot be scheduled);
+                               2: never.  The results are the fp32 sums of
+                               the same products either way.               */
   SPH_OPT_SPLIT_QUANTIZE = 10, /* sph_split_step with one payload chunk: 0
                                automatic (default: in the endpoint's epilogue
                                for at most 2^20 rows x ids, else a separate
@@ -236,6 +247,8 @@ typedef struct sph_plan {
   int32_t whole_tiles;      /* 1: whole tiles per CTA; 0: stream-K ranges  */
   int32_t planes;           /* hidden-state operand planes (bf16 or e4m3)  */
   int32_t gemv_rows;        /* GEMV: rows per launch (1, 2, 4 or 8)        */
+  int32_t pair;             /* 1: CTA pairs (SPH_OPT_TC_PAIR); grid counts
+                               CTAs, tile_ids is per CTA (a tile is 256)   */
 } sph_plan;
 sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep,
                           int64_t K, sph_dtype w_dtype, sph_act_mode act_mode,

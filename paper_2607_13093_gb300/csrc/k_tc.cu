@@ -67,7 +67,9 @@ constexpr int kTileM = 128;          // vocabulary rows per MMA (M); a tile is 1
 constexpr int kAtomK = 64;           // bf16 elements per 128-byte swizzle atom
 constexpr int kAtomBytes = kTileM * kAtomK * 2;   // one A atom: 128 rows x 128 B
 constexpr int kMaxBN = 256;
-constexpr int kMaxStages = 12;       // (the barriers, 2 * 12 + 5 words, fit the 256-byte area)
+constexpr int kMaxStages = 12;       // (the barriers, 2 * 12 + 5 words and two more, fit
+                                     // the 512-byte area)
+constexpr int kBarrierArea = 512;
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
 constexpr int kMaxDevices = 64;      // per-device launch attribute cache
@@ -269,24 +271,35 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
 }
 
 // TM = vocabulary rows per tile: 128, or 256 as two M = 128 MMAs that share
-// each B stage (half the B bytes per A byte; TMEM holds 2 x 2 x BN columns)
-template <int HILO, bool GATHER, int EPI, bool FP8, int TM>
+// each B stage (half the B bytes per A byte; TMEM holds 2 x 2 x BN columns).
+// PAIR: a cluster of two CTAs computes each 256-id tile as one M = 256
+// tcgen05 MMA (.cta_group::2) issued by the even CTA: each CTA loads its own
+// 128 ids of A and half (BN / 2) of the tile's hidden-state rows of B, and
+// holds the accumulator of its 128 ids for all BN rows, so each SM takes in
+// half the B bytes.  Both CTAs' copies of a stage complete on the even
+// CTA's stage barrier (which expects both CTAs' bytes); the even CTA's
+// commits arrive on both CTAs' barriers; both epilogues report to the even
+// CTA.  Work is split over pairs.
+template <int HILO, bool GATHER, int EPI, bool FP8, int TM, bool PAIR = false>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_kernel(const __grid_constant__ WMaps wm,
           const __grid_constant__ CUtensorMap tmH, const TcParams p) {
   static_assert(TM == 128 || TM == 256, "tile height");
+  static_assert(!PAIR || TM == 128, "a pair tile is two CTAs of 128 ids");
   constexpr int kAtomE = FP8 ? kAtomE8 : kAtomK;   // elements per 128-byte atom
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* base = smem_raw + (((raw_addr + 1023) & ~1023u) - raw_addr);
   constexpr int kHalves = TM / 128;     // M = 128 halves of a tile
   constexpr int kGroups = TM / 32;      // 32-row lane groups of a tile
+  constexpr int kTileStride = PAIR ? 256 : TM;      // ids between tiles
   const int BN = p.BN;
+  const int BNc = PAIR ? BN / 2 : BN;   // hidden-state rows of B in this CTA
   const int NA = p.na;
   // A: per atom the TM tile rows at 128-byte stride (half h at h * 16 KB)
   const int atom_bytes = kHalves * kAtomBytes;
   const int a_bytes = NA * atom_bytes;
-  const int b_bytes = HILO * NA * BN * 128;
+  const int b_bytes = HILO * NA * BNc * 128;
   const int stage_bytes = a_bytes + b_bytes;
   const int S = p.stages;
   uint64_t* full = reinterpret_cast<uint64_t*>(base + (size_t)S * stage_bytes);
@@ -297,12 +310,16 @@ tc_kernel(const __grid_constant__ WMaps wm,
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
   // the current tile's row boxes (subset path), after the barriers
-  int2* s_box = reinterpret_cast<int2*>(base + (size_t)S * stage_bytes + 256);
+  int2* s_box = reinterpret_cast<int2*>(base + (size_t)S * stage_bytes + kBarrierArea);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int G = gridDim.x;
-  const long long it0 = range_start(p, blockIdx.x, G);
-  const long long it1 = range_start(p, blockIdx.x + 1, G);
+  // pair: `half` = the CTA's rank in its cluster (0 issues the MMAs), the
+  // work unit is the pair
+  const int half = PAIR ? (int)ptx::cluster_ctarank() : 0;
+  const int unit = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int G = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  const long long it0 = range_start(p, unit, G);
+  const long long it1 = range_start(p, unit + 1, G);
   // producer, subset path: the ids of a segment's tile are loaded one
   // segment ahead, so that planning a tile never waits on memory; the first
   // tile's load goes out before the CTA's setup
@@ -310,7 +327,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
 #pragma unroll
   for (int g = 0; g < kGroups; ++g) nid[g] = 0;
   auto load_ids = [&](int tl, int (&dst)[kGroups]) {
-    const int j0 = (tl % p.NT) * TM;
+    const int j0 = (tl % p.NT) * kTileStride + half * 128;
     const int rows = min(TM, p.n - j0);
 #pragma unroll
     for (int g = 0; g < kGroups; ++g) {
@@ -326,7 +343,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
   auto plan_tile = [&](int t, int next_tile, int& nbox, uint32_t& tx) {
     int2 box[2 * kGroups];                       // (first id, row | (rows - 1) << 8)
     unsigned bmask = 0;                          // which of box[] are in use
-    const int j0 = t * TM;
+    const int j0 = t * kTileStride + half * 128;
     const int rows = min(TM, p.n - j0);
     int idr[kGroups];
 #pragma unroll
@@ -401,7 +418,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(&tfull[a], 1);
-      ptx::mbar_init(&tempty[a], kEpiWarps);
+      ptx::mbar_init(&tempty[a], kEpiWarps * (PAIR ? 2 : 1));   // (pair: both epilogues)
     }
     ptx::mbar_init(drain, 1);
     *s_abort = 0;
@@ -416,12 +433,19 @@ tc_kernel(const __grid_constant__ WMaps wm,
   // this one wait for them (griddep_wait): the producer before its first
   // copy, the epilogue before its first store.
   ptx::griddep_launch_dependents();
-  __syncthreads();                     // barriers initialised
+  // barriers initialised (pair: in both CTAs, before either signals the
+  // other's)
+  if constexpr (PAIR) ptx::cluster_sync();
+  else __syncthreads();
   // the producer needs no tensor memory: it starts now, while warp 1
   // allocates the accumulators for itself and the other warps
   uint32_t tmem_base = 0;
   if (warp != 0) {
-    if (warp == 1) ptx::tmem_alloc(tmem_holder, ncols);
+    if (warp == 1) {
+      __syncwarp();
+      if constexpr (PAIR) ptx::tmem_alloc_pair(tmem_holder, ncols);
+      else ptx::tmem_alloc(tmem_holder, ncols);
+    }
     ptx::tc_fence_before();
     ptx::named_bar_sync(1, (int)blockDim.x - 32);
     ptx::tc_fence_after();
@@ -452,11 +476,22 @@ tc_kernel(const __grid_constant__ WMaps wm,
     // copies right after it.
     bool waited = false;
     int rb_first = 0, kb_first = 0;
+    // pair: the odd CTA's copies complete on the even CTA's stage barrier
+    // (whose MMAs read both CTAs' stages)
+    const uint32_t lead_full = PAIR ? ptx::mapa(ptx::smem_u32(full), 0) : 0u;
+    auto load2 = [&](void* dst, const CUtensorMap* map, int x, int y, int st) {
+      if (PAIR && half) ptx::tma_load_2d_pair(dst, map, x, y, lead_full + (uint32_t)(st * 8));
+      else ptx::tma_load_2d(dst, map, x, y, &full[st]);
+    };
+    auto load3 = [&](void* dst, const CUtensorMap* map, int x, int y, int z, int st) {
+      if (PAIR && half) ptx::tma_load_3d_pair(dst, map, x, y, z, lead_full + (uint32_t)(st * 8));
+      else ptx::tma_load_3d(dst, map, x, y, z, &full[st]);
+    };
     // the B copy of plane l of stage st (k-block kb, row block rb)
     auto issue_b = [&](int st, int kb, int rb, int l) {
       if (l >= 0 && l < HILO)
-        ptx::tma_load_3d(base + (size_t)st * stage_bytes + a_bytes + l * NA * BN * 128, &tmH, 0,
-                         l * p.Rp + rb * BN, kb * NA, &full[st]);
+        load3(base + (size_t)st * stage_bytes + a_bytes + l * NA * BNc * 128, &tmH, 0,
+              l * p.Rp + rb * BN + half * BNc, kb * NA, st);
     };
     auto finish_wait = [&]() {
       if (lane == 0) ptx::griddep_wait();
@@ -476,16 +511,31 @@ tc_kernel(const __grid_constant__ WMaps wm,
         if (!pk.next(tn, a0, a1)) tn = -1;
         plan_tile(t, tn, nbox, tx);
       }
+      // pair: the odd CTA's bytes of each stage of this tile -- its B part,
+      // and its A boxes, which cover each of its tile rows below n once (the
+      // full-vocabulary path copies whole 128-row boxes)
+      uint32_t tx_peer = 0;
+      if constexpr (PAIR) {
+        if constexpr (GATHER) {
+          const int prow = max(0, min(128, p.n - (t * kTileStride + 128)));
+          tx_peer = (uint32_t)(prow * 128 * NA + b_bytes);
+        } else {
+          tx_peer = (uint32_t)stage_bytes;
+        }
+      }
       for (int kb = kb0; kb < kb1; ++kb) {
         int ok = 1;
-        if (lane == 0) ok = !*s_abort && ptx::mbar_wait(&empty[stage], phase ^ 1, limit);
+        if (lane == 0)
+          ok = !*s_abort && ptx::mbar_wait(&empty[stage], phase ^ 1, limit);
         ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
         if (!ok) {
           if (lane == 0 && !*s_abort) give_up();
           stop = true;
           break;
         }
-        if (lane == 0) ptx::mbar_expect_tx(&full[stage], tx);
+        // (pair: the even CTA expects both CTAs' bytes; the odd CTA's copies
+        // complete on that barrier without an arrival of their own)
+        if (lane == 0 && !(PAIR && half)) ptx::mbar_expect_tx(&full[stage], tx + tx_peer);
         __syncwarp();
         // every copy of the stage goes to its own lane, so the copies are
         // issued side by side rather than one after another: A as NA x (row
@@ -499,14 +549,14 @@ tc_kernel(const __grid_constant__ WMaps wm,
             if constexpr (GATHER) {
               const int a = op / nbox;
               const int2 bx = s_box[op - a * nbox];
-              ptx::tma_load_2d(A + a * atom_bytes + (bx.y & 0xFF) * 128, &wm.m[bx.y >> 8],
-                               (kb * NA + a) * kAtomE, bx.x, &full[stage]);
+              load2(A + a * atom_bytes + (bx.y & 0xFF) * 128, &wm.m[bx.y >> 8],
+                    (kb * NA + a) * kAtomE, bx.x, stage);
             } else if (p.a3d) {
-              ptx::tma_load_3d(A, &wm.a3, 0, t * TM, kb * NA, &full[stage]);
+              load3(A, &wm.a3, 0, t * kTileStride + half * 128, kb * NA, stage);
             } else {
               const int a = op / kHalves, hf = op - a * kHalves;
-              ptx::tma_load_2d(A + a * atom_bytes + hf * kAtomBytes, &wm.m[kBoxHeights - 1],
-                               (kb * NA + a) * kAtomE, t * TM + hf * 128, &full[stage]);
+              load2(A + a * atom_bytes + hf * kAtomBytes, &wm.m[kBoxHeights - 1],
+                    (kb * NA + a) * kAtomE, t * kTileStride + half * 128 + hf * 128, stage);
             }
           } else {
             issue_b(stage, kb, rb, op - nA);
@@ -522,10 +572,19 @@ tc_kernel(const __grid_constant__ WMaps wm,
     // issued stage completes)
     if (!waited) finish_wait();
     if (stop && lane == 0) {
-      // let the copies already issued land before the CTA winds down
-      for (long long k = issued > S ? issued - S : 0; k < issued; ++k)
-        ptx::mbar_wait(&full[k % S], (uint32_t)((k / S) & 1), kDrainLimit);
+      // let the copies already issued land before the CTA winds down (the
+      // odd CTA of a pair cannot wait on the even CTA's barriers: it waits
+      // about 100 us, far longer than a copy takes)
+      if (PAIR && half) {
+        const long long t0 = clock64();
+        while (clock64() - t0 < (200000ll)) __nanosleep(1000);
+      } else {
+        for (long long k = issued > S ? issued - S : 0; k < issued; ++k)
+          ptx::mbar_wait(&full[k % S], (uint32_t)((k / S) & 1), kDrainLimit);
+      }
     }
+  } else if (warp == 1 && PAIR && half == 1) {
+    // pair, odd CTA: the even CTA issues the MMAs for both
   } else if (warp == 1) {
     // ---------------------------------------------------------- MMA issuer
     if (lane == 0) {
@@ -534,13 +593,17 @@ tc_kernel(const __grid_constant__ WMaps wm,
       uint32_t phase = 0;
       uint32_t tph[2] = {0, 0};
       int si = 0, tile, kb0, kb1;
+      constexpr int kMmaM = PAIR ? 2 * kTileM : kTileM;
       const uint32_t idesc =
-          FP8 ? ptx::idesc_e4m3_f32(kTileM, BN) : ptx::idesc_bf16_f32(kTileM, BN);
+          FP8 ? ptx::idesc_e4m3_f32(kMmaM, BN) : ptx::idesc_bf16_f32(kMmaM, BN);
+      auto wait_x = [&](uint64_t* bar, uint32_t parity) {
+        return ptx::mbar_wait(bar, parity, limit);
+      };
       // accumulator `acc`, tile half hf: TMEM columns (acc * kHalves + hf) * BN
       bool stop = false;
       while (!stop && sg.next(tile, kb0, kb1)) {
         const int acc = p.single_acc ? 0 : (si & 1);
-        if (*s_abort || !ptx::mbar_wait(&tempty[acc], tph[acc] ^ 1, limit)) {
+        if (*s_abort || !wait_x(&tempty[acc], tph[acc] ^ 1)) {
           if (!*s_abort) give_up();
           break;
         }
@@ -548,7 +611,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
         ptx::tc_fence_after();
         const uint32_t d = tmem_base + (uint32_t)(acc * kHalves * BN);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (*s_abort || !ptx::mbar_wait(&full[stage], phase, limit)) {
+          if (*s_abort || !wait_x(&full[stage], phase)) {
             if (!*s_abort) give_up();
             stop = true;
             break;
@@ -567,9 +630,13 @@ tc_kernel(const __grid_constant__ WMaps wm,
                   // 32 bytes of K per MMA: 16 bf16 or 32 e4m3 elements
                   const uint64_t ad =
                       ptx::sdesc_k128(a0 + at * atom_bytes + hf * kAtomBytes + kk * 32);
-                  const uint64_t bd = ptx::sdesc_k128(b0 + (h * NA + at) * BN * 128 + kk * 32);
+                  const uint64_t bd = ptx::sdesc_k128(b0 + (h * NA + at) * BNc * 128 + kk * 32);
                   const uint32_t accum = (kb != kb0 || at != 0 || h != 0 || kk != 0) ? 1u : 0u;
-                  if constexpr (FP8)
+                  if constexpr (PAIR && FP8)
+                    ptx::umma_f8_pair(d, ad, bd, idesc, accum);
+                  else if constexpr (PAIR)
+                    ptx::umma_f16_pair(d, ad, bd, idesc, accum);
+                  else if constexpr (FP8)
                     ptx::umma_f8(d + (uint32_t)(hf * BN), ad, bd, idesc, accum);
                   else
                     ptx::umma_f16(d + (uint32_t)(hf * BN), ad, bd, idesc, accum);
@@ -577,16 +644,23 @@ tc_kernel(const __grid_constant__ WMaps wm,
               }
             }
           }
-          ptx::umma_commit(&empty[stage]);
+          if constexpr (PAIR) ptx::umma_commit_pair(&empty[stage]);
+          else ptx::umma_commit(&empty[stage]);
           if (++stage == S) { stage = 0; phase ^= 1; }
         }
         if (stop) break;
-        ptx::umma_commit(&tfull[acc]);
+        if constexpr (PAIR) ptx::umma_commit_pair(&tfull[acc]);
+        else ptx::umma_commit(&tfull[acc]);
         ++si;
       }
       // all issued MMAs complete before TMEM is released
-      ptx::umma_commit(drain);
-      ptx::mbar_wait(drain, 0, kDrainLimit);
+      if constexpr (PAIR) {
+        ptx::umma_commit_pair(drain);
+        ptx::mbar_wait(drain, 0, kDrainLimit);
+      } else {
+        ptx::umma_commit(drain);
+        ptx::mbar_wait(drain, 0, kDrainLimit);
+      }
     }
   } else if (warp < 2 + kEpiWarps) {
     // ------------------------------------------------------------ epilogue
@@ -604,12 +678,13 @@ tc_kernel(const __grid_constant__ WMaps wm,
       const int acc = p.single_acc ? 0 : (si & 1);
       const int rb = tile / p.NT, t = tile - rb * p.NT;
       const bool whole = kb0 == 0 && kb1 == p.KB;
+      const int segb = (t * kTileStride + half * 128) / 32;   // first 32-id segment
       // this lane's vocabulary row in each half: i = hf * 128 + quad * 32 + lane
       int jh[kHalves], idh[kHalves];
       bool vjh[kHalves];
 #pragma unroll
       for (int hf = 0; hf < kHalves; ++hf) {
-        jh[hf] = t * TM + hf * 128 + quad * 32 + lane;
+        jh[hf] = t * kTileStride + half * 128 + hf * 128 + quad * 32 + lane;
         vjh[hf] = jh[hf] < p.n;
         idh[hf] = vjh[hf] ? (GATHER ? p.ids[jh[hf]] : jh[hf]) : 0;
       }
@@ -624,7 +699,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
 #pragma unroll
         for (int hf = 0; hf < kHalves; ++hf)
           prefetch_payload<EPI>(p, rb * BN + grp * (BN / 2), BN / 2,
-                                t * TM + hf * 128 + quad * 32, lane);
+                                t * kTileStride + half * 128 + hf * 128 + quad * 32, lane);
         if (whole && grp < nhc)
           load_payload<EPI>(p, rb * BN + (grp % nch) * 16, J(grp / nch), lane, pay);
       }
@@ -643,18 +718,22 @@ tc_kernel(const __grid_constant__ WMaps wm,
       bool fin = false, known_last = false, pre_ok = false;
       float pre[16];                   // two contributors: the other's first chunk
       if (!whole) {
-        cnt = (tile * 4 + quad) * kEpiGroups + grp;
-        c0 = (int)cta_of((long long)tile * p.KB, p.T, gridDim.x);
-        C = (int)cta_of((long long)tile * p.KB + p.KB - 1, p.T, gridDim.x) - c0 + 1;
-        fin = p.finish_wait > 0 && C >= 2 && C <= kMaxC && (int)blockIdx.x == c0 + C - 2;
+        cnt = ((tile * 4 + quad) * kEpiGroups + grp) * (PAIR ? 2 : 1) + half;
+        c0 = (int)cta_of((long long)tile * p.KB, p.T, G);
+        C = (int)cta_of((long long)tile * p.KB + p.KB - 1, p.T, G) - c0 + 1;
+        fin = p.finish_wait > 0 && C >= 2 && C <= kMaxC && unit == c0 + C - 2;
       }
       // the contributors' partial slots: every contributor after the first
       // starts its range inside this tile, so the tile is its first segment
       // (slot 2c); the first one holds it as its first segment only if its
       // range starts exactly at the tile (slot 2c0), else as its last
       // (slot 2c0 + 1)
-      const bool c0_first = !whole && range_start(p, c0, gridDim.x) == (long long)tile * p.KB;
-      auto slot_of = [&](int c) { return c == 0 ? 2 * c0 + (c0_first ? 0 : 1) : 2 * (c0 + c); };
+      const bool c0_first = !whole && range_start(p, c0, G) == (long long)tile * p.KB;
+      // (pair: each CTA of a unit keeps its own half of the partial)
+      auto pslot = [&](int u) { return PAIR ? 2 * u + half : u; };
+      auto slot_of = [&](int c) {
+        return pslot(c == 0 ? 2 * c0 + (c0_first ? 0 : 1) : 2 * (c0 + c));
+      };
       if (fin) {
         // the early contributor (the tile's last) has usually arrived
         // already: then fetch its partial while the MMAs finish
@@ -674,7 +753,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
         }
       }
       int ok = 1;
-      if (lane == 0) ok = !*s_abort && ptx::mbar_wait(&tfull[acc], fph[acc], limit);
+      if (lane == 0)
+        ok = !*s_abort && ptx::mbar_wait(&tfull[acc], fph[acc], limit);
       ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
       if (!ok) {
         if (lane == 0 && !*s_abort) give_up();
@@ -701,7 +781,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
                              (uint32_t)(acc * kHalves * BN);
       // a CTA's split tiles can only be its first and its last segment:
       // slot 2c holds the first, 2c+1 the last ([BN][TM] each)
-      float* Pt = p.P + (size_t)(2 * blockIdx.x + (si == 0 ? 0 : 1)) * BN * TM;
+      float* Pt = p.P + (size_t)pslot(2 * unit + (si == 0 ? 0 : 1)) * BN * TM;
       for (int hc = grp; hc < nhc; hc += kEpiGroups) {
         const int hf = hc / nch, ch = hc - hf * nch;
         const int i = hf * 128 + quad * 32 + lane;
@@ -713,13 +793,13 @@ tc_kernel(const __grid_constant__ WMaps wm,
           if (EPI != EPI_CLOUD && hn < nhc)
             load_payload<EPI>(p, rb * BN + (hn % nch) * 16, J(hn / nch), lane, nxt);
           finish_chunk<EPI>(p, v, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
-                            t * kGroups + hf * 4 + quad, pay);
+                            segb + hf * 4 + quad, pay);
           if constexpr (EPI != EPI_CLOUD) pay = nxt;
         } else if (known_last) {
           // the partials in CTA order (the same order, and so the same
           // result, as the fix-up below), this CTA's own from registers
           if constexpr (EPI != EPI_CLOUD) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
-          const int me = (int)blockIdx.x - c0;
+          const int me = unit - c0;
           const size_t o = (size_t)ch * 16 * TM + i;
           float s[16];
           if (pre_ok && hc == grp) {       // two contributors, the other's part prefetched
@@ -739,7 +819,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
             }
           }
           finish_chunk<EPI>(p, s, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
-                            t * kGroups + hf * 4 + quad, pay);
+                            segb + hf * 4 + quad, pay);
         } else {
 #pragma unroll
           for (int q = 0; q < 16; ++q) Pt[(size_t)(ch * 16 + q) * TM + i] = v[q];
@@ -747,7 +827,10 @@ tc_kernel(const __grid_constant__ WMaps wm,
       }
       ptx::tc_fence_before();
       __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(&tempty[acc]);
+      if (lane == 0) {
+        if (PAIR && half) ptx::mbar_arrive_remote(ptx::mapa(ptx::smem_u32(&tempty[acc]), 0));
+        else ptx::mbar_arrive(&tempty[acc]);
+      }
       if (known_last) {
         if (lane == 0) p.counters[cnt] = 0;
       } else if (!whole) {
@@ -780,12 +863,12 @@ tc_kernel(const __grid_constant__ WMaps wm,
               }
             }
             for (int c = kMaxC; c < C; ++c) {    // rare: very many contributors
-              const float* pc = p.P + (size_t)(2 * (c0 + c)) * BN * TM + quad * 32 + lane;
+              const float* pc = p.P + (size_t)pslot(2 * (c0 + c)) * BN * TM + quad * 32 + lane;
 #pragma unroll
               for (int q = 0; q < 16; ++q) v[q] += __ldcg(pc + o + (size_t)q * TM);
             }
             finish_chunk<EPI>(p, v, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
-                              t * kGroups + hf * 4 + quad, pay);
+                              segb + hf * 4 + quad, pay);
           }
           if (lane == 0) p.counters[cnt] = 0;
         }
@@ -795,9 +878,16 @@ tc_kernel(const __grid_constant__ WMaps wm,
   }
 
   ptx::tc_fence_before();
-  __syncthreads();
+  // pair: neither CTA leaves (or frees its tensor memory) before the other
+  // is done with its arrivals and the even CTA's MMAs have completed
+  if constexpr (PAIR) ptx::cluster_sync();
+  else __syncthreads();
   ptx::tc_fence_after();
-  if (warp == 1) ptx::tmem_dealloc(tmem_base, ncols);
+  if (warp == 1) {
+    __syncwarp();
+    if constexpr (PAIR) ptx::tmem_dealloc_pair(tmem_base, ncols);
+    else ptx::tmem_dealloc(tmem_base, ncols);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1082,15 +1172,87 @@ bool w_maps(const GatherGemm& g, bool gather, WMaps& out) {
 
 }  // namespace
 
+namespace {
+// The plan of a CTA-pair launch: 256-id tiles, each CTA of a pair with 128
+// ids of A and half of B's rows, row blocks of up to 256 rows (a multiple of
+// 32, so that each CTA's half is whole 16-row groups), work split over the
+// pairs (a multiple of the row-block count, as below).
+TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pairs,
+                    int schedule, int max_stages, int block_k, int max_bn_opt) {
+  int cap = 256;
+  if (max_bn_opt >= 32 && max_bn_opt < cap) cap = max_bn_opt / 32 * 32;
+  pl.RB = (rows + cap - 1) / cap;
+  pl.BN = ((rows + pl.RB - 1) / pl.RB + 31) / 32 * 32;
+  pl.tm = 128;
+  pl.single_acc = 0;
+  pl.Rp = pl.RB * pl.BN;
+  auto stage_of = [&](int na) { return na * (kAtomBytes + pl.hilo * (pl.BN / 2) * 128); };
+  // (a pair pays a cross-CTA hand-off per stage, so it prefers fewer,
+  // larger stages: measured on 1024 rows x 256000 ids x 4608 with bf16
+  // activations, three 128-column stages 1746 us, six 64-column 2005 us)
+  pl.na = block_k == 64 ? 1 : (block_k == 256 ? 4 : 2);
+  const int min_stages = block_k ? 2 : 3;
+  while (pl.na > 1 && (int)((kSmemBudget - 2048) / stage_of(pl.na)) < min_stages) pl.na >>= 1;
+  const int bk = pl.na * kAtomK;
+  pl.KB = (K + bk - 1) / bk;
+  pl.Kp = pl.KB * bk;
+  pl.NT = (n + 255) / 256;
+  const int tiles = pl.RB * pl.NT;
+  pl.T = (long long)tiles * pl.KB;
+  // pairs: as many as fit at once (the SMs of a GPU section pair up)
+  int units = sm_count / 2;
+  if (max_pairs > 0 && max_pairs < units) units = max_pairs;
+  if (pl.RB > 1 && pl.RB <= units) units = units / pl.RB * pl.RB;
+  const int g_whole = tiles < units ? tiles : units;
+  const long long whole_span = (long long)((tiles + g_whole - 1) / g_whole) * pl.KB;
+  const double split_span = (double)pl.T / (pl.T < units ? pl.T : units);
+  pl.whole_tiles = schedule == 1 || (schedule == 0 && whole_span <= 1.1 * split_span + 2.0);
+  units = pl.whole_tiles ? g_whole : (int)(pl.T < units ? pl.T : units);
+  pl.G = 2 * units;
+  pl.stages = (int)((kSmemBudget - 2048) / stage_of(pl.na));
+  if (pl.stages > kMaxStages) pl.stages = kMaxStages;
+  if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
+  pl.hs_bytes = align256((size_t)pl.hilo * pl.Rp * pl.Kp * 2);
+  const bool splits = !pl.whole_tiles && (pl.T % units != 0 || (pl.T / units) % pl.KB != 0);
+  pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * 128 * 4) : 0;
+  pl.cnt_bytes = align256((size_t)tiles * 4 * kEpiGroups * 2 * sizeof(int));
+  pl.nseg = pl.NT * 8;
+  pl.stats_bytes = 0;
+  pl.epi_stats = 0;
+  pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes;
+  pl.smem_bytes = 1024 + (size_t)pl.stages * stage_of(pl.na) + kBarrierArea +
+                  kMaxBoxes * sizeof(int2);
+  pl.ok = pl.stages >= 2;
+  return pl;
+}
+}  // namespace
+
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
                int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn_opt,
-               int tile_m) {
+               int tile_m, int pair_mode, int max_pairs) {
   TcPlan pl{};
   // h planes: bf16 weights take one bf16 plane for bf16-rounded
   // activations (exact) and two (hi + lo) for fp32; e4m3 weights take two
   // e4m3 planes for bf16-rounded activations (exact) and four for fp32
   pl.hilo = fp8 ? (act_bf16 ? 2 : 4) : (act_bf16 ? 1 : 2);
   pl.fp8 = fp8;
+  (void)gather;
+  // CTA pairs: forced (pair_mode 2), or chosen (1) where their row blocks
+  // are long enough that halving each SM's B bytes pays for the pair's
+  // hand-offs: >= 192 rows, or >= 128 with one plane.  Measured pair vs
+  // single: 1024 rows x 256000 ids x 4608 fp32 2654 vs 3191 us, bf16 (three
+  // stages) 1746 vs 2005; 256 rows x 256000 fp32 737 vs 897; 320 rows x
+  // 51302 x 3584 bf16 161 vs 195, fp32 (160-row blocks) 242 vs 223; 32
+  // rows x 12000 x 3840 38.9 vs 37.2; 64 rows x 256000 x 4608 471 vs 433.
+  // (an explicitly set tile height keeps single-CTA tiles unless pairs are
+  // forced)
+  if (pair_mode > 0 && !fp8 && !endpoint && sm_count >= 2 && (tile_m == 0 || pair_mode == 2)) {
+    pl.pair = 1;
+    const TcPlan pp = tc_plan_pair(pl, rows, n, K, sm_count, max_pairs, schedule, max_stages,
+                                   block_k, max_bn_opt);
+    if (pair_mode == 2 || pp.BN >= 192 || (pl.hilo == 1 && pp.BN >= 128)) return pp;
+    pl.pair = 0;
+  }
   const int atom = fp8 ? kAtomE8 : kAtomK;   // elements per 128-byte atom
   // e4m3: row blocks of up to 128 rows (measured on 256 rows x 152064 ids
   // x 7168, 256-id tiles: four planes 1229 / 996 / 743 us and two planes
@@ -1187,16 +1349,16 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   // 1024 rows x 256000 ids x 512 gain; 256 rows x 152064 ids x 1024 loses)
   pl.epi_stats = endpoint && (pl.BN < 128 || 4 * pl.BN <= K);
   pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
-  pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + 256 + kMaxBoxes * sizeof(int2);
+  pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + kBarrierArea + kMaxBoxes * sizeof(int2);
   pl.ok = pl.stages >= 2;
   return pl;
 }
 
-template <int HILO, bool GATHER, int EPI, bool FP8 = false, int TM = 128>
+template <int HILO, bool GATHER, int EPI, bool FP8 = false, int TM = 128, bool PAIR = false>
 static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
                                const TcParams& prm, const TcPlan& pl,
                                cudaStream_t st) {
-  auto kern = tc_kernel<HILO, GATHER, EPI, FP8, TM>;
+  auto kern = tc_kernel<HILO, GATHER, EPI, FP8, TM, PAIR>;
   // the shared-memory opt-in, raised only when a launch needs more than any
   // earlier one on this device (a host call per launch otherwise)
   static std::atomic<int> configured[kMaxDevices];
@@ -1214,14 +1376,51 @@ static cudaError_t launch_inst(const WMaps& mw, const CUtensorMap& mh,
       }
     }
   }
+  if constexpr (PAIR)
+    return launch_pdl_cluster(kern, dim3(pl.G), dim3(kThreads), pl.smem_bytes, st, 2,
+                              mw, mh, prm);
   return launch_pdl(kern, dim3(pl.G), dim3(kThreads), pl.smem_bytes, st,
                     mw, mh, prm);
+}
+
+int tc_pair_max_units(int device) {
+  static std::atomic<int> cache[kMaxDevices];
+  if (device < 0 || device >= kMaxDevices) return 0;
+  const int c = cache[device].load();
+  if (c) return c;
+  // the largest shared memory a pair launch asks for
+  auto kern = tc_kernel<2, false, EPI_CLOUD, false, 128, true>;
+  const int smem = (int)(kSmemBudget + 1024 + kBarrierArea + kMaxBoxes * sizeof(int2));
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(2);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) {
+    cudaGetLastError();
+    return 0;
+  }
+  cache[device].store(n);
+  return n;
 }
 
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                       long long spin_limit, cudaStream_t st) {
   const bool fp8 = g.w_dtype == W_FP8;
   if (!pl.ok || (fp8 != (pl.fp8 != 0)) || (fp8 && g.epilogue != EPI_CLOUD) ||
+      (pl.pair && (fp8 || g.epilogue != EPI_CLOUD || pl.G % 2 || pl.BN % 32)) ||
       (g.epilogue != EPI_CLOUD && pl.hilo != 2) ||
       (g.epilogue == EPI_FUSED && (!g.yc || !g.rowmax_in || !g.codes_out || !g.scale_out)))
     return cudaErrorNotSupported;
@@ -1243,7 +1442,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
     cudaError_t e = launch_pdl(split_h_e4m3_kernel, dim3(pl.Rp), dim3(kSplit8Threads), 0, st,
                                g.h, g.ld_h, g.rows, g.K, pl.Rp, pl.Kp, pl.hilo,
                                reinterpret_cast<uint8_t*>(sc), h_scale, counters,
-                               tiles * 4 * kEpiGroups, g.rowmax, g.act_bf16);
+                               tiles * 4 * kEpiGroups * (pl.pair ? 2 : 1), g.rowmax, g.act_bf16);
     if (e != cudaSuccess) return e;
   } else {
     const int64_t groups = (int64_t)pl.Rp * pl.Kp / 8;
@@ -1251,7 +1450,8 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
     if (blocks > 4096) blocks = 4096;
     if (blocks < 1) blocks = 1;
     cudaError_t e = launch_pdl(split_h_kernel, dim3(blocks), dim3(kSplitThreads), 0, st, g.h, g.ld_h,
-                               g.rows, g.K, pl.Rp, pl.Kp, pl.hilo, Hs, counters, tiles * 4 * kEpiGroups,
+                               g.rows, g.K, pl.Rp, pl.Kp, pl.hilo, Hs, counters,
+                               tiles * 4 * kEpiGroups * (pl.pair ? 2 : 1),
                                g.epilogue == EPI_CLOUD ? g.rowmax : (unsigned*)nullptr);
     if (e != cudaSuccess) return e;
   }
@@ -1265,8 +1465,10 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   const int esz = fp8 ? 1 : 2;
   // h planes [hilo * Rp rows, Kp columns], zero padded: all atoms of a
   // stage in one copy per plane
+  // (a pair's CTAs each take half of the block's rows)
   if (!cached_map3(&mh, dt, sc, (uint64_t)pl.Kp, (uint64_t)pl.hilo * pl.Rp,
-                   (uint64_t)pl.Kp * esz, (uint32_t)pl.BN, (uint32_t)pl.na, atom))
+                   (uint64_t)pl.Kp * esz, (uint32_t)(pl.pair ? pl.BN / 2 : pl.BN),
+                   (uint32_t)pl.na, atom))
     return cudaErrorInvalidValue;
   // full vocabulary with a width that is a multiple of the atom: A likewise
   const int a3d = (!gather && g.K % atom == 0 && g.K >= pl.na * atom) ? 1 : 0;
@@ -1295,6 +1497,12 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.status = g.status; prm.spin_limit = spin_limit; prm.finish_wait = g.finish_wait;
 
   const bool hilo2 = pl.hilo == 2;
+  if (pl.pair) {
+    if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st)
+                             : launch_inst<1, true, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st);
+    return hilo2 ? launch_inst<2, false, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st)
+                 : launch_inst<1, false, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st);
+  }
   if (pl.tm == 256) {
     if (fp8) {
       if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, true, 256>(mw, mh, prm, pl, st)

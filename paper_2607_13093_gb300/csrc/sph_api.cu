@@ -39,6 +39,8 @@ struct sph_ctx {
   int sampler = 0;                  // SPH_OPT_SAMPLER
   int check_ids = 0;                // SPH_OPT_CHECK_IDS
   int split_quantize = 0;           // SPH_OPT_SPLIT_QUANTIZE
+  int tc_pair = 0;                  // SPH_OPT_TC_PAIR: 0 automatic, 1 always, 2 never
+  int pair_units = 0;               // CTA pairs that fit at once (0: pairs unavailable)
   // chunked split steps: the endpoint's own stream (created on first use
   // when the caller passes none) and the events that order the two streams
   cudaStream_t aux_stream = nullptr;
@@ -137,6 +139,12 @@ bool use_tc(const sph_ctx* ctx, int64_t rows, int w_dtype) {
   return rows >= ctx->tc_min_rows;
 }
 
+// tc_plan's pair mode: 0 never, 1 where it pays, 2 always
+int pair_mode(const sph_ctx* ctx) {
+  if (ctx->pair_units < 1 || ctx->tc_pair == 2) return 0;
+  return ctx->tc_pair == 1 ? 2 : 1;
+}
+
 size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_bf16,
                 int w_dtype, int endpoint, int sm_count = 0) {
   if (!use_tc(ctx, rows, w_dtype)) return 0;
@@ -151,7 +159,7 @@ size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_
       const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, sm_count,
                                     endpoint, ctx->tc_schedule, ctx->tc_stages,
                                     ctx->tc_block_k, gather, w_dtype == sph::W_FP8,
-                                    ctx->tc_max_bn, tm)
+                                    ctx->tc_max_bn, tm, pair_mode(ctx), ctx->pair_units)
                            .scratch_bytes;
       if (x > b) b = x;
     }
@@ -449,7 +457,7 @@ sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep, 
                                       call == 0 && act_mode == SPH_ACT_BF16, ctx->sm_count,
                                       call, ctx->tc_schedule, ctx->tc_stages, ctx->tc_block_k,
                                       gather != 0, wdt == sph::W_FP8, ctx->tc_max_bn,
-                                      ctx->tc_tile_m);
+                                      ctx->tc_tile_m, pair_mode(ctx), ctx->pair_units);
   out->tensor_core = 1;
   out->row_blocks = pl.RB;
   out->block_rows = pl.BN;
@@ -460,6 +468,7 @@ sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep, 
   out->grid = pl.G;
   out->whole_tiles = pl.whole_tiles;
   out->planes = pl.hilo;
+  out->pair = pl.pair;
   return SPH_OK;
 }
 
@@ -483,6 +492,8 @@ sph_status sph_create(int device, void* cuda_stream, sph_ctx** out) {
     delete ctx;
     return SPH_ERR_CUDA;
   }
+  // how many CTA pairs of the pair kernel fit at once (0: none)
+  ctx->pair_units = sph::tc_pair_max_units(device);
   if (cudaMalloc(&ctx->status, sizeof(unsigned)) != cudaSuccess) {
     cudaGetLastError();
     delete ctx;
@@ -630,6 +641,12 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "sampler must be 0 or 1");
       ctx->sampler = (int)value;
       return SPH_OK;
+    case SPH_OPT_TC_PAIR:
+      if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "tc_pair must be 0, 1 or 2");
+      if (value == 1 && ctx->pair_units < 1)
+        return fail(ctx, SPH_ERR_UNSUPPORTED, "CTA pairs cannot be scheduled on this device");
+      ctx->tc_pair = (int)value;
+      return SPH_OK;
     case SPH_OPT_SPLIT_QUANTIZE:
       if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "split_quantize must be 0, 1 or 2");
       ctx->split_quantize = (int)value;
@@ -730,7 +747,8 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
     const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_keep, (int)d_h, act_bf16,
                                         ctx->sm_count, 0, ctx->tc_schedule, ctx->tc_stages,
                                         ctx->tc_block_k, keep_ids != nullptr,
-                                        wdt == sph::W_FP8, ctx->tc_max_bn, ctx->tc_tile_m);
+                                        wdt == sph::W_FP8, ctx->tc_max_bn, ctx->tc_tile_m,
+                                        pair_mode(ctx), ctx->pair_units);
     void* tcs = c.take(pl.scratch_bytes);
     if (!c.fits())
       return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
@@ -915,7 +933,8 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
       const sph::TcPlan pl = sph::tc_plan((int)rows, (int)n_q, (int)d_h, act_bf16, sm_cloud, 0,
                                           ctx->tc_schedule, ctx->tc_stages, ctx->tc_block_k,
                                           keep_ids != nullptr, wdt == sph::W_FP8,
-                                          ctx->tc_max_bn, ctx->tc_tile_m);
+                                          ctx->tc_max_bn, ctx->tc_tile_m, pair_mode(ctx),
+                                          ctx->pair_units);
       if (pl.scratch_bytes > tcc)
         return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: cloud plan outgrew its scratch");
       return launch_status(ctx, sph::launch_tc(gg, pl, cloud_tc, ctx->spin_limit, s),

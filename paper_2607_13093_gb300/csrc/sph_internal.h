@@ -48,6 +48,27 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   ++launch_count;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
+// launch_pdl with thread-block clusters of `cluster_x` CTAs along x
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                               cudaStream_t st, int cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)cluster_x;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++launch_count;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // One gathered contraction  acc[r, j] = sum_c h[r, c] * W[ids[j], c]
 // followed by an epilogue.  Pointers are device pointers.
@@ -96,6 +117,7 @@ int gemv_rows_per_launch(int rows, int K);
 // Tensor-core path (k_tc.cu): sizes, work split and scratch of one call.
 struct TcPlan {
   int hilo, RB, BN, Rp, KB, Kp, NT, G, stages, whole_tiles, na, fp8;
+  int pair;        // CTA pairs (clusters of two) share each 256-id tile; G counts CTAs
   int tm;          // vocabulary rows per tile: 128 or 256
   int single_acc;  // one TMEM accumulator (256-id tiles over > 128 rows)
   int nseg;        // endpoint statistics: 32-id segments per row, NT * tm / 32
@@ -109,10 +131,16 @@ struct TcPlan {
 // hidden elements per pipeline stage (64, 128 or 256; 0 = automatic);
 // gather = the kept-id subset path (keep_ids given); fp8 = e4m3 weights;
 // max_bn = most hidden-state rows per tile (0 = automatic); tile_m =
-// vocabulary rows per tile (128, 256 = two M = 128 halves, 0 = automatic).
+// vocabulary rows per tile (128, 256 = two M = 128 halves, 0 = automatic);
+// pair_mode = CTA pairs on 256-id tiles (cloud epilogue with bf16 weights
+// only; ignored elsewhere): 0 never, 1 where the row blocks are long enough,
+// 2 always; max_pairs caps the pairs (0: no cap).
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
                int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn,
-               int tile_m);
+               int tile_m, int pair_mode = 0, int max_pairs = 0);
+// CTA pairs of the pair kernel that can run at once on `device` (0 when the
+// query fails): tc_plan's max_pairs.
+int tc_pair_max_units(int device);
 // Launch the operand split and the tcgen05 kernel; `scratch` holds
 // plan.scratch_bytes bytes.  bf16 weights only.
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,

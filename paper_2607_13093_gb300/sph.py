@@ -32,6 +32,7 @@ SPH_OPT_TC_FINISH_WAIT = 7
 SPH_OPT_SAMPLER = 8
 SPH_OPT_CHECK_IDS = 9
 SPH_OPT_SPLIT_QUANTIZE = 10
+SPH_OPT_TC_PAIR = 11
 SPH_SAMPLER_CDF, SPH_SAMPLER_GUMBEL = 0, 1
 
 _c_void_p = ctypes.c_void_p
@@ -53,7 +54,7 @@ class sph_profile(ctypes.Structure):
 
 
 PLAN_FIELDS = ("tensor_core", "row_blocks", "block_rows", "tile_ids", "tiles",
-               "k_blocks", "stages", "grid", "whole_tiles", "planes", "gemv_rows")
+               "k_blocks", "stages", "grid", "whole_tiles", "planes", "gemv_rows", "pair")
 
 
 class sph_plan(ctypes.Structure):

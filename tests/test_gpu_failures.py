@@ -47,6 +47,24 @@ def test_cloud_wait_timeout_is_reported_and_context_recovers(ctx):
     check_cloud(ctx, w)
 
 
+@pytest.mark.parametrize("gather", [True, False])
+def test_pair_wait_timeout_is_reported_and_context_recovers(ctx, gather):
+    # CTA pairs: a wait that gives up in either CTA winds both down (every
+    # wait bounded, the odd CTA's in-flight copies given time to land, both
+    # CTAs meet at the end before freeing tensor memory)
+    from paper_2607_13093_gb300 import sph
+    w = wl.make_workload(V=6000, d=1024, d_l=128, rows=200, n_keep=3000 if gather else 6000,
+                         device=DEV, seed=94)
+    ctx.set_option(sph.SPH_OPT_TC_PAIR, 1)
+    try:
+        assert ctx.plan(0, w.rows, w.n_keep, w.d_h, gather=gather)["pair"] == 1
+        _expect_timeout(ctx, lambda: ctx.partial_logits(w.h_cloud, w.W_h, keep_ids=w.keep_ids,
+                                                        clip=w.clip))
+        check_cloud(ctx, w)
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
+
+
 def test_endpoint_wait_timeout_is_reported_and_context_recovers(ctx):
     import torch
     w = wl.make_workload(V=6000, d=1024, d_l=128, rows=48, n_keep=3000, device=DEV, seed=92)

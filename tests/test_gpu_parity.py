@@ -731,3 +731,71 @@ def test_tracing_times_each_call_class_once(ctx):
         assert p["calls"][c] == 1 and p["ms"][c] > 0, (c, p)
     assert p["launches"] >= 7          # split + contraction, quantize, endpoint, draw, verification
     assert fresh["launches"] == 0 and not any(fresh["calls"].values())
+
+
+# ---------------------------------------------------------------------------
+# CTA pairs (SPH_OPT_TC_PAIR): each 256-id tile one M = 256 MMA over two
+# CTAs, each holding 128 ids and half of the hidden-state rows
+# ---------------------------------------------------------------------------
+
+PAIR_CASES = [
+    ("decode-like", dict(V=4000, d=1024, d_l=128, rows=32, n_keep=1500)),
+    ("full-vocab", dict(V=3000, d=1280, d_l=256, rows=48, n_keep=3000)),
+    ("ragged-K", dict(V=2000, d=1072, d_l=72, rows=24, n_keep=700)),
+    ("rows300", dict(V=3000, d=776, d_l=8, rows=300, n_keep=2000)),
+    ("rows1000-bias", dict(V=6000, d=2112, d_l=64, rows=1000, n_keep=5000, with_bias=True)),
+]
+
+
+@pytest.mark.parametrize("name,kw", PAIR_CASES, ids=[c[0] for c in PAIR_CASES])
+@pytest.mark.parametrize("schedule", [1, 2])
+@pytest.mark.parametrize("act", ["fp32", "bf16"])
+def test_tensor_core_pairs(ctx, name, kw, schedule, act):
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    ctx.set_option(sph.SPH_OPT_TC_PAIR, 1)
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, schedule)
+    try:
+        w = small(seed=707, **kw)
+        p = ctx.plan(0, w.rows, w.n_keep, w.d_h, gather=w.keep_ids is not None,
+                     act_mode=sph.SPH_ACT_BF16 if act == "bf16" else sph.SPH_ACT_FP32)
+        assert p["pair"] == 1 and p["grid"] % 2 == 0 and p["block_rows"] % 32 == 0
+        check_cloud(ctx, w, act_mode=act)
+        # the endpoint ignores the option (its plans never pair)
+        ref = oracle_cloud(w)
+        check_endpoint(ctx, w, torch.from_numpy(ref["codes"]), torch.from_numpy(ref["row_scale"]))
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+
+
+@pytest.mark.parametrize("n_keep", [3000, 20000])
+def test_tensor_core_pairs_split_tiles_without_finisher(ctx, n_keep):
+    # stream-K split tiles finished by the last contributor to count in
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_PAIR, 1)
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 2)
+    ctx.set_option(sph.SPH_OPT_TC_FINISH_WAIT, 0)
+    try:
+        w = small(V=n_keep + 4000, d=2112, d_l=64, rows=130, n_keep=n_keep, seed=708)
+        check_cloud(ctx, w)
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_FINISH_WAIT, 1 << 15)
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+        ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
+
+
+def test_tensor_core_pairs_full_size_sweep(ctx):
+    # the 1024-row sweep point in the pair plan, rows from every row block
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_PAIR, 1)
+    try:
+        w = wl.workload("sweep", device=DEV, rows=1024, keep_frac=1.0)
+        sample = rows_to_check(ctx, w, "fp32")
+        p = ctx.plan(0, 1024, w.n_keep, w.d_h, gather=False)
+        assert p["pair"] == 1
+        assert {r // p["block_rows"] for r in sample} == set(range(p["row_blocks"]))
+        check_cloud(ctx, w, rows=sample)
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
