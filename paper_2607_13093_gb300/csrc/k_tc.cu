@@ -1179,7 +1179,8 @@ namespace {
 // pairs (a multiple of the row-block count, as below).
 TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pairs,
                     int schedule, int max_stages, int block_k, int max_bn_opt) {
-  int cap = 256;
+  // (e4m3 weights: four or two h planes; 128-row blocks keep four stages)
+  int cap = pl.fp8 ? 128 : 256;
   if (max_bn_opt >= 32 && max_bn_opt < cap) cap = max_bn_opt / 32 * 32;
   pl.RB = (rows + cap - 1) / cap;
   pl.BN = ((rows + pl.RB - 1) / pl.RB + 31) / 32 * 32;
@@ -1190,10 +1191,10 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
   // (a pair pays a cross-CTA hand-off per stage, so it prefers fewer,
   // larger stages: measured on 1024 rows x 256000 ids x 4608 with bf16
   // activations, three 128-column stages 1746 us, six 64-column 2005 us)
-  pl.na = block_k == 64 ? 1 : (block_k == 256 ? 4 : 2);
+  pl.na = pl.fp8 ? 1 : (block_k == 64 ? 1 : (block_k == 256 ? 4 : 2));
   const int min_stages = block_k ? 2 : 3;
   while (pl.na > 1 && (int)((kSmemBudget - 2048) / stage_of(pl.na)) < min_stages) pl.na >>= 1;
-  const int bk = pl.na * kAtomK;
+  const int bk = pl.na * (pl.fp8 ? kAtomE8 : kAtomK);
   pl.KB = (K + bk - 1) / bk;
   pl.Kp = pl.KB * bk;
   pl.NT = (n + 255) / 256;
@@ -1212,7 +1213,8 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
   pl.stages = (int)((kSmemBudget - 2048) / stage_of(pl.na));
   if (pl.stages > kMaxStages) pl.stages = kMaxStages;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
-  pl.hs_bytes = align256((size_t)pl.hilo * pl.Rp * pl.Kp * 2);
+  pl.hs_bytes = pl.fp8 ? align256((size_t)pl.hilo * pl.Rp * pl.Kp) + align256((size_t)pl.Rp * 4)
+                       : align256((size_t)pl.hilo * pl.Rp * pl.Kp * 2);
   const bool splits = !pl.whole_tiles && (pl.T % units != 0 || (pl.T / units) % pl.KB != 0);
   pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * 128 * 4) : 0;
   pl.cnt_bytes = align256((size_t)tiles * 4 * kEpiGroups * 2 * sizeof(int));
@@ -1246,11 +1248,11 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   // rows x 12000 x 3840 38.9 vs 37.2; 64 rows x 256000 x 4608 471 vs 433.
   // (an explicitly set tile height keeps single-CTA tiles unless pairs are
   // forced)
-  if (pair_mode > 0 && !fp8 && !endpoint && sm_count >= 2 && (tile_m == 0 || pair_mode == 2)) {
+  if (pair_mode > 0 && !endpoint && sm_count >= 2 && (tile_m == 0 || pair_mode == 2)) {
     pl.pair = 1;
     const TcPlan pp = tc_plan_pair(pl, rows, n, K, sm_count, max_pairs, schedule, max_stages,
                                    block_k, max_bn_opt);
-    if (pair_mode == 2 || pp.BN >= 192 || (pl.hilo == 1 && pp.BN >= 128)) return pp;
+    if (pair_mode == 2 || (!fp8 && (pp.BN >= 192 || (pl.hilo == 1 && pp.BN >= 128)))) return pp;
     pl.pair = 0;
   }
   const int atom = fp8 ? kAtomE8 : kAtomK;   // elements per 128-byte atom
@@ -1420,7 +1422,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                       long long spin_limit, cudaStream_t st) {
   const bool fp8 = g.w_dtype == W_FP8;
   if (!pl.ok || (fp8 != (pl.fp8 != 0)) || (fp8 && g.epilogue != EPI_CLOUD) ||
-      (pl.pair && (fp8 || g.epilogue != EPI_CLOUD || pl.G % 2 || pl.BN % 32)) ||
+      (pl.pair && (g.epilogue != EPI_CLOUD || pl.G % 2 || pl.BN % 32)) ||
       (g.epilogue != EPI_CLOUD && pl.hilo != 2) ||
       (g.epilogue == EPI_FUSED && (!g.yc || !g.rowmax_in || !g.codes_out || !g.scale_out)))
     return cudaErrorNotSupported;
@@ -1497,6 +1499,12 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.status = g.status; prm.spin_limit = spin_limit; prm.finish_wait = g.finish_wait;
 
   const bool hilo2 = pl.hilo == 2;
+  if (pl.pair && fp8) {
+    if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, true, 128, true>(mw, mh, prm, pl, st)
+                             : launch_inst<4, true, EPI_CLOUD, true, 128, true>(mw, mh, prm, pl, st);
+    return hilo2 ? launch_inst<2, false, EPI_CLOUD, true, 128, true>(mw, mh, prm, pl, st)
+                 : launch_inst<4, false, EPI_CLOUD, true, 128, true>(mw, mh, prm, pl, st);
+  }
   if (pl.pair) {
     if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st)
                              : launch_inst<1, true, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st);

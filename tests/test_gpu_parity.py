@@ -799,3 +799,24 @@ def test_tensor_core_pairs_full_size_sweep(ctx):
         check_cloud(ctx, w, rows=sample)
     finally:
         ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
+
+
+@pytest.mark.parametrize("rows,keep", [(40, 1100), (200, 3000), (256, 2500)])
+@pytest.mark.parametrize("schedule", [1, 2])
+@pytest.mark.parametrize("act", ["fp32", "bf16"])
+def test_fp8_tensor_core_pairs(ctx, rows, keep, schedule, act):
+    # e4m3 weights on CTA pairs (kind::f8f6f4, M = 256 over two CTAs);
+    # d_h = 1008: a ragged last k-block
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_PAIR, 1)
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, schedule)
+    try:
+        w = small(V=3000, d=1048, d_l=40, rows=rows, n_keep=keep, w_dtype="fp8", clip=40.0,
+                  seed=331 + rows, with_bias=(rows == 40))
+        p = ctx.plan(0, w.rows, w.n_keep, w.d_h, w_dtype=sph.SPH_DTYPE_FP8_E4M3,
+                     gather=w.keep_ids is not None)
+        assert p["pair"] == 1
+        check_cloud(ctx, w, act_mode=act)
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+        ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
