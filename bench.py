@@ -432,7 +432,7 @@ class Runner:
         self.hs = [w.h] + [w.h.roll(i + 1, dims=0).contiguous() for i in range(ncopy - 1)]
         self.codes = torch.empty(R, n, dtype=torch.int8, device=dev)
         self.scale = torch.empty(R, dtype=torch.float32, device=dev)
-        L = n if (chunk <= 0 or chunk >= n) else chunk
+        L = n if (chunk <= 0 or chunk >= n or not mode.startswith("chunked")) else chunk
         self.nchunk = (n + L - 1) // L
         self.scales = torch.empty(self.nchunk * R, dtype=torch.float32, device=dev)
         self.tokens = torch.empty(R, dtype=torch.int32, device=dev)
