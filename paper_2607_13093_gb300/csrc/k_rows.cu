@@ -41,17 +41,21 @@ __device__ __forceinline__ float seg_weight(float2 st, float M, float inv_tau) {
 }
 
 // ---------------------------------------------------------------------------
-// statistics: a warp takes one 1024-id chunk (32 segments) of one row
+// statistics: a warp takes one 1024-id chunk (32 segments) of one row, a
+// lane one 32-id segment
 // ---------------------------------------------------------------------------
-// Lane pair (2q, 2q + 1) ends with segment h * 16 + q of the chunk for each
-// half h; the chunk statistic combines the 32 segment statistics.
+// Each lane reads its segment's 128 contiguous bytes (eight 16-byte loads
+// where the row allows, the line served from L1 after its first sector),
+// and reduces max and sum of exp in registers as balanced trees: no
+// shuffles per logit (the warp-wide reduce-scatter this replaces spent about
+// eight instructions per logit and left the pass issue-bound at 45 % of
+// HBM).  The chunk statistic then combines the 32 lanes' segments.
 __global__ void __launch_bounds__(kWarps * 32)
 seg_stats_kernel(const float* __restrict__ Z, int rows, int n, int nseg, int nchunk,
                  float inv_tau, float2* __restrict__ stats, float2* __restrict__ cstats) {
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
-  const int kr = (lane >> 1) & 15;
   const float l2t = inv_tau * kLog2e;
   const long long total = (long long)nchunk * rows;
   const long long nwarps = (long long)gridDim.x * kWarps;
@@ -69,35 +73,46 @@ seg_stats_kernel(const float* __restrict__ Z, int rows, int n, int nseg, int nch
       c = (int)(g - r * nchunk);
     }
     const float* z = Z + r * n;
-    float v[2][kGroup];
+    const int sg = c * kSeg + lane;           // this lane's segment
+    const int j0 = sg * kSeg;
+    float v[kSeg];
+    if (sg < nseg && j0 + kSeg <= n && ((reinterpret_cast<uintptr_t>(z + j0) & 15) == 0)) {
+      const float4* zv = reinterpret_cast<const float4*>(z + j0);
 #pragma unroll
-    for (int h = 0; h < 2; ++h)
-#pragma unroll
-      for (int q = 0; q < kGroup; ++q) {
-        const int sg = c * kSeg + h * kGroup + q;
-        const int j = sg * kSeg + lane;
-        v[h][q] = (sg < nseg && j < n) ? __ldcs(z + j) : -INFINITY;
+      for (int q = 0; q < kSeg / 4; ++q) {
+        const float4 t = __ldg(zv + q);
+        v[4 * q] = t.x; v[4 * q + 1] = t.y; v[4 * q + 2] = t.z; v[4 * q + 3] = t.w;
       }
-    float mk[2], sk[2];
+    } else {
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      mk[h] = warp_reduce_scatter16(v[h], MaxOp{}, lane);
-      float e[kGroup];
-#pragma unroll
-      for (int q = 0; q < kGroup; ++q) {
-        const float mq = __shfl_sync(0xFFFFFFFFu, mk[h], 2 * q);
-        e[q] = v[h][q] > -INFINITY ? exp_tau(v[h][q] - mq, l2t) : 0.f;
+      for (int q = 0; q < kSeg; ++q) {
+        const int j = j0 + q;
+        v[q] = (sg < nseg && j < n) ? __ldg(z + j) : -INFINITY;
       }
-      sk[h] = warp_reduce_scatter16(e, SumOp{}, lane);
-      const int sg = c * kSeg + h * kGroup + kr;
-      if (!(lane & 1) && sg < nseg) stats[r * nseg + sg] = make_float2(mk[h], sk[h]);
     }
-    const float Mc = warp_max(fmaxf(mk[0], mk[1]));
-    float Sc = 0.f;
-    if (!(lane & 1))
-      Sc = seg_weight(make_float2(mk[0], sk[0]), Mc, inv_tau) +
-           seg_weight(make_float2(mk[1], sk[1]), Mc, inv_tau);
-    Sc = warp_sum(Sc);
+    float t[kSeg / 2];
+#pragma unroll
+    for (int q = 0; q < kSeg / 2; ++q) t[q] = fmaxf(v[2 * q], v[2 * q + 1]);
+#pragma unroll
+    for (int w = kSeg / 4; w >= 1; w >>= 1)
+#pragma unroll
+      for (int q = 0; q < w; ++q) t[q] = fmaxf(t[2 * q], t[2 * q + 1]);
+    const float m = t[0];
+    float sum = 0.f;
+    if (m > -INFINITY) {
+      // exp of -inf (ids past n) is 0
+#pragma unroll
+      for (int q = 0; q < kSeg / 2; ++q)
+        t[q] = exp_tau(v[2 * q] - m, l2t) + exp_tau(v[2 * q + 1] - m, l2t);
+#pragma unroll
+      for (int w = kSeg / 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int q = 0; q < w; ++q) t[q] = t[2 * q] + t[2 * q + 1];
+      sum = t[0];
+    }
+    if (sg < nseg) stats[r * nseg + sg] = make_float2(m, sum);
+    const float Mc = warp_max(m);
+    const float Sc = warp_sum(seg_weight(make_float2(m, sum), Mc, inv_tau));
     if (lane == 0) cstats[r * nchunk + c] = make_float2(Mc, Sc);
   }
 }
