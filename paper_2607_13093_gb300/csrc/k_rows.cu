@@ -44,18 +44,24 @@ __device__ __forceinline__ float seg_weight(float2 st, float M, float inv_tau) {
 // statistics: a warp takes one 1024-id chunk (32 segments) of one row, a
 // lane one 32-id segment
 // ---------------------------------------------------------------------------
-// Each lane reads its segment's 128 contiguous bytes (eight 16-byte loads
-// where the row allows, the line served from L1 after its first sector),
-// and reduces max and sum of exp in registers as balanced trees: no
-// shuffles per logit (the warp-wide reduce-scatter this replaces spent about
-// eight instructions per logit and left the pass issue-bound at 45 % of
-// HBM).  The chunk statistic then combines the 32 lanes' segments.
+// The warp reads the chunk with coalesced loads (16-byte where the row is so
+// aligned) into its shared-memory tile, segment s at words 36 s .. 36 s + 31
+// (the padding keeps the stores and the lanes' 16-byte reads free of bank
+// conflicts), then each lane reduces its segment's max and sum of exp in
+// registers as balanced trees.  That is a handful of instructions per logit
+// where the warp-wide reduce-scatter it replaces spent about eight (issue-
+// bound at 45 % of HBM); a lane reading its own 128 bytes straight from
+// global memory instead made every load touch 32 lines (47.6 us against
+// 22.5 us on the spec workload's 66 MB).
+constexpr int kSegRow = 36;             // words per segment in the tile
 __global__ void __launch_bounds__(kWarps * 32)
 seg_stats_kernel(const float* __restrict__ Z, int rows, int n, int nseg, int nchunk,
                  float inv_tau, float2* __restrict__ stats, float2* __restrict__ cstats) {
+  __shared__ __align__(16) float tile[kWarps][kSeg * kSegRow];
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
+  float* tb = tile[threadIdx.x >> 5];
   const float l2t = inv_tau * kLog2e;
   const long long total = (long long)nchunk * rows;
   const long long nwarps = (long long)gridDim.x * kWarps;
@@ -72,24 +78,31 @@ seg_stats_kernel(const float* __restrict__ Z, int rows, int n, int nseg, int nch
       r = g / nchunk;
       c = (int)(g - r * nchunk);
     }
-    const float* z = Z + r * n;
-    const int sg = c * kSeg + lane;           // this lane's segment
-    const int j0 = sg * kSeg;
-    float v[kSeg];
-    if (sg < nseg && j0 + kSeg <= n && ((reinterpret_cast<uintptr_t>(z + j0) & 15) == 0)) {
-      const float4* zv = reinterpret_cast<const float4*>(z + j0);
+    const int j0 = c * kSeg * kSeg;             // the chunk's first id
+    const float* z = Z + r * n + j0;
+    const int left = n - j0;                    // ids of the row from j0 on
+    __syncwarp();                               // (the previous item's reads)
+    if (left >= kSeg * kSeg && ((reinterpret_cast<uintptr_t>(z) & 15) == 0)) {
 #pragma unroll
       for (int q = 0; q < kSeg / 4; ++q) {
-        const float4 t = __ldg(zv + q);
-        v[4 * q] = t.x; v[4 * q + 1] = t.y; v[4 * q + 2] = t.z; v[4 * q + 3] = t.w;
+        const float4 t = __ldcs(reinterpret_cast<const float4*>(z) + q * 32 + lane);
+        *reinterpret_cast<float4*>(tb + (q * 4 + (lane >> 3)) * kSegRow + 4 * (lane & 7)) = t;
       }
     } else {
-#pragma unroll
+#pragma unroll 8
       for (int q = 0; q < kSeg; ++q) {
-        const int j = j0 + q;
-        v[q] = (sg < nseg && j < n) ? __ldg(z + j) : -INFINITY;
+        const int e = q * 32 + lane;
+        tb[q * kSegRow + lane] = e < left ? __ldcs(z + e) : -INFINITY;
       }
     }
+    __syncwarp();
+    float v[kSeg];
+#pragma unroll
+    for (int m = 0; m < kSeg / 4; ++m) {
+      const float4 t = *reinterpret_cast<const float4*>(tb + lane * kSegRow + 4 * m);
+      v[4 * m] = t.x; v[4 * m + 1] = t.y; v[4 * m + 2] = t.z; v[4 * m + 3] = t.w;
+    }
+    const int sg = c * kSeg + lane;             // this lane's segment
     float t[kSeg / 2];
 #pragma unroll
     for (int q = 0; q < kSeg / 2; ++q) t[q] = fmaxf(v[2 * q], v[2 * q + 1]);

@@ -70,11 +70,17 @@ constexpr int kMaxBN = 256;
 constexpr int kMaxStages = 12;       // (the barriers, 2 * 12 + 5 words and two more, fit
                                      // the 512-byte area)
 constexpr int kBarrierArea = 512;
+// the endpoint epilogue's transpose tiles: per epilogue warp 8 rows x 32 ids
+// (+4 words of padding per row, so that both the row writes and the 16-byte
+// reads are free of bank conflicts)
+constexpr int kTRow = 36;
+constexpr int kTransposeBytes = 8 /* epilogue warps */ * 8 * kTRow * 4;
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
 constexpr int kMaxDevices = 64;      // per-device launch attribute cache
 
 constexpr int kEpiWarps = 8;         // two per TMEM lane quadrant
+static_assert(kTransposeBytes == kEpiWarps * 8 * kTRow * 4, "transpose tiles per warp");
 constexpr int kEpiGroups = kEpiWarps / 4;
 constexpr int kThreads = 64 + 32 * kEpiWarps;       // producer, MMA, epilogue
 constexpr int kAtomE8 = 128;         // e4m3 elements per 128-byte atom
@@ -112,6 +118,7 @@ struct TcParams {
   int8_t* codes_out;           // fused endpoint: the payload codes [R][n] (out)
   float* scale_out;            // fused endpoint: the row scales [R] (out)
   float2* seg_stats;           // endpoint: [R][nseg] (max, sum exp)
+  int epi_t;                   // endpoint without statistics: transposed epilogue
   int a3d;                     // full vocabulary: A by one 3-D copy per stage
   int single_acc;              // one accumulator (no epilogue overlap): 256-id tiles of > 128 rows
   float* P;                    // split-tile partials [2 * grid][BN][TM]
@@ -267,6 +274,80 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
     const float sk = warp_reduce_scatter16(e, SumOp{}, lane);
     if (!(lane & 1) && row0 + kr < p.R)
       p.seg_stats[(int64_t)(row0 + kr) * p.nseg + seg] = make_float2(mk, sk);
+  }
+}
+
+// Endpoint epilogue without statistics (Eq. 13: z = code * s + local
+// partial), through this warp's shared-memory tile `tb` [8][kTRow]: the
+// 16 rows of a chunk go in two halves of 8; after the transpose lane l holds
+// row (l >> 2) of the half and the 8 consecutive ids 8 (l & 3) .. + 7 of the
+// warp's 32, so its payload is one 8-byte (or two 4-byte) load and its z two
+// 16-byte stores, instead of 16 one-byte loads and 16 strided stores per
+// lane.  Used when rows of codes and z are 4-element aligned (n and the z
+// row stride multiples of 4).  The payload of a chunk does not depend on the
+// accumulator, so it is loaded a chunk ahead (TPay).
+struct TPay {
+  uint2 cw[2];     // the 8 codes of this lane's row and ids, per half
+  float sc[2];     // that row's scale, per half (0 past the rows)
+};
+__device__ __forceinline__ void load_tpay(const TcParams& p, int row0, int j0w, int lane,
+                                          TPay& t) {
+  const int q = lane >> 2, seg = lane & 3;
+#pragma unroll
+  for (int h8 = 0; h8 < 2; ++h8) {
+    t.cw[h8] = make_uint2(0u, 0u);
+    t.sc[h8] = 0.f;
+    const int r = row0 + h8 * 8 + q;
+    const int j = j0w + 8 * seg;
+    if (!p.codes || r >= p.R || j >= p.n) continue;
+    t.sc[h8] = __ldg(p.row_scale + r);
+    const int8_t* cp = p.codes + (int64_t)r * p.n + j;     // 4-byte aligned
+    if (j + 8 <= p.n) {
+      if ((reinterpret_cast<uintptr_t>(cp) & 7) == 0) {
+        t.cw[h8] = __ldg(reinterpret_cast<const uint2*>(cp));
+      } else {
+        t.cw[h8].x = __ldg(reinterpret_cast<const unsigned*>(cp));
+        t.cw[h8].y = __ldg(reinterpret_cast<const unsigned*>(cp) + 1);
+      }
+    } else {                                   // the row's last ids
+      unsigned w[2] = {0u, 0u};
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        if (j + e < p.n) w[e >> 2] |= ((unsigned)(uint8_t)__ldg(cp + e)) << (8 * (e & 3));
+      t.cw[h8] = make_uint2(w[0], w[1]);
+    }
+  }
+}
+__device__ __forceinline__ void finish_chunk_t(const TcParams& p, const float (&v)[16], int row0,
+                                               int j0w, int lane, float* tb, const TPay& pay) {
+  const int q = lane >> 2, seg = lane & 3;
+#pragma unroll
+  for (int h8 = 0; h8 < 2; ++h8) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) tb[k * kTRow + lane] = v[h8 * 8 + k];
+    __syncwarp();
+    const float4 a = *reinterpret_cast<const float4*>(tb + q * kTRow + 8 * seg);
+    const float4 b = *reinterpret_cast<const float4*>(tb + q * kTRow + 8 * seg + 4);
+    __syncwarp();
+    const int r = row0 + h8 * 8 + q;
+    const int j = j0w + 8 * seg;
+    if (r >= p.R || j >= p.n) continue;
+    float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+    const float sc = pay.sc[h8];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      x[e] += (float)(int8_t)((pay.cw[h8].x >> (8 * e)) & 0xFF) * sc;
+      x[4 + e] += (float)(int8_t)((pay.cw[h8].y >> (8 * e)) & 0xFF) * sc;
+    }
+    float* zp = p.Y + (int64_t)r * p.ldy + j;                 // 16-byte aligned
+    if (j + 8 <= p.n) {
+      reinterpret_cast<float4*>(zp)[0] = make_float4(x[0], x[1], x[2], x[3]);
+      reinterpret_cast<float4*>(zp)[1] = make_float4(x[4], x[5], x[6], x[7]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        if (j + e < p.n) zp[e] = x[e];
+    }
   }
 }
 
@@ -692,6 +773,12 @@ tc_kernel(const __grid_constant__ WMaps wm,
       auto J = [&](int hf) { return (kHalves > 1 && hf) ? jh[kHalves - 1] : jh[0]; };
       auto VJ = [&](int hf) { return (kHalves > 1 && hf) ? vjh[kHalves - 1] : vjh[0]; };
       auto ID = [&](int hf) { return (kHalves > 1 && hf) ? idh[kHalves - 1] : idh[0]; };
+      // the endpoint without statistics finishes chunks through this warp's
+      // transpose tile (no per-lane payload registers then)
+      const bool epi_t = EPI == EPI_ENDPOINT && p.epi_t;
+      float* tb = reinterpret_cast<float*>(base + (size_t)S * stage_bytes + kBarrierArea +
+                                           kMaxBoxes * sizeof(int2)) +
+                  (warp - 2) * 8 * kTRow;
       Payload pay;
       if constexpr (EPI != EPI_CLOUD) {
         // the payload does not depend on the accumulator: start on it
@@ -700,9 +787,22 @@ tc_kernel(const __grid_constant__ WMaps wm,
         for (int hf = 0; hf < kHalves; ++hf)
           prefetch_payload<EPI>(p, rb * BN + grp * (BN / 2), BN / 2,
                                 t * kTileStride + half * 128 + hf * 128 + quad * 32, lane);
-        if (whole && grp < nhc)
+        if (whole && grp < nhc && !epi_t)
           load_payload<EPI>(p, rb * BN + (grp % nch) * 16, J(grp / nch), lane, pay);
       }
+      TPay tpay;
+      if (epi_t && whole && grp < nhc)
+        load_tpay(p, rb * BN + (grp % nch) * 16, J(grp / nch) - lane, lane, tpay);
+      // (split tiles load the transposed payload right before finishing)
+      auto finish = [&](const float (&vv)[16], int hf, int ch) {
+        if (epi_t) {
+          if (!whole) load_tpay(p, rb * BN + ch * 16, J(hf) - lane, lane, tpay);
+          finish_chunk_t(p, vv, rb * BN + ch * 16, J(hf) - lane, lane, tb, tpay);
+        } else {
+          finish_chunk<EPI>(p, vv, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
+                            segb + hf * 4 + quad, pay);
+        }
+      };
       // Split tile: contributors c0 .. c0 + C - 1 (CTA order).  All but the
       // last end their ranges inside the tile, so they reach it at the end
       // of their work; the last one reaches it first thing (its range starts
@@ -790,15 +890,18 @@ tc_kernel(const __grid_constant__ WMaps wm,
         if (whole) {
           Payload nxt;
           const int hn = hc + kEpiGroups;
-          if (EPI != EPI_CLOUD && hn < nhc)
+          TPay tnxt;
+          if (EPI != EPI_CLOUD && hn < nhc && !epi_t)
             load_payload<EPI>(p, rb * BN + (hn % nch) * 16, J(hn / nch), lane, nxt);
-          finish_chunk<EPI>(p, v, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
-                            segb + hf * 4 + quad, pay);
+          if (epi_t && hn < nhc)
+            load_tpay(p, rb * BN + (hn % nch) * 16, J(hn / nch) - lane, lane, tnxt);
+          finish(v, hf, ch);
           if constexpr (EPI != EPI_CLOUD) pay = nxt;
+          if (epi_t) tpay = tnxt;
         } else if (known_last) {
           // the partials in CTA order (the same order, and so the same
           // result, as the fix-up below), this CTA's own from registers
-          if constexpr (EPI != EPI_CLOUD) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
+          if (EPI != EPI_CLOUD && !epi_t) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
           const int me = unit - c0;
           const size_t o = (size_t)ch * 16 * TM + i;
           float s[16];
@@ -818,8 +921,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
               }
             }
           }
-          finish_chunk<EPI>(p, s, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
-                            segb + hf * 4 + quad, pay);
+          finish(s, hf, ch);
         } else {
 #pragma unroll
           for (int q = 0; q < 16; ++q) Pt[(size_t)(ch * 16 + q) * TM + i] = v[q];
@@ -850,7 +952,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
             ps[c] = p.P + (size_t)slot_of(c < C ? c : 0) * BN * TM + quad * 32 + lane;
           for (int hc = grp; hc < nhc; hc += kEpiGroups) {
             const int hf = hc / nch, ch = hc - hf * nch;
-            if constexpr (EPI != EPI_CLOUD) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
+            if (EPI != EPI_CLOUD && !epi_t) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
             const size_t o = (size_t)ch * 16 * TM + hf * 128;
             float v[16];
 #pragma unroll
@@ -867,8 +969,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
 #pragma unroll
               for (int q = 0; q < 16; ++q) v[q] += __ldcg(pc + o + (size_t)q * TM);
             }
-            finish_chunk<EPI>(p, v, rb * BN + ch * 16, J(hf), VJ(hf), ID(hf), lane,
-                              segb + hf * 4 + quad, pay);
+            finish(v, hf, ch);
           }
           if (lane == 0) p.counters[cnt] = 0;
         }
@@ -1332,7 +1433,11 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.whole_tiles = schedule == 1 || (schedule == 0 && whole_span <= 1.1 * split_span + 2.0);
   pl.G = pl.whole_tiles ? g_whole : (int)(pl.T < sm_use ? pl.T : sm_use);
   const int stage_bytes = pl.na * (halves * kAtomBytes + pl.hilo * pl.BN * 128);
-  pl.stages = (int)((kSmemBudget - 2048) / stage_bytes);
+  // endpoint without epilogue statistics: the epilogue transposes each
+  // warp's chunk through shared memory (kTransposeBytes beside the stages)
+  pl.epi_stats = endpoint && (pl.BN < 128 || 4 * pl.BN <= K);
+  pl.epi_t = endpoint && !pl.epi_stats;
+  pl.stages = (int)((kSmemBudget - 2048 - (pl.epi_t ? kTransposeBytes : 0)) / stage_bytes);
   if (pl.stages > kMaxStages) pl.stages = kMaxStages;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
   // h planes (bf16 or e4m3), and with e4m3 the per-row scales after them
@@ -1349,9 +1454,9 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   // the hidden dimension is long enough; otherwise a separate pass over z at
   // memory speed is cheaper (measured: 320 rows x 51302 ids x 512 and
   // 1024 rows x 256000 ids x 512 gain; 256 rows x 152064 ids x 1024 loses)
-  pl.epi_stats = endpoint && (pl.BN < 128 || 4 * pl.BN <= K);
   pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
-  pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + kBarrierArea + kMaxBoxes * sizeof(int2);
+  pl.smem_bytes = 1024 + (size_t)pl.stages * stage_bytes + kBarrierArea + kMaxBoxes * sizeof(int2) +
+                  (pl.epi_t ? kTransposeBytes : 0);
   pl.ok = pl.stages >= 2;
   return pl;
 }
@@ -1495,6 +1600,10 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
   prm.single_acc = pl.single_acc;
   prm.inv_tau = g.inv_tau; prm.seg_stats = (pl.epi_stats && !g.no_stats) ? stats : nullptr; prm.a3d = a3d;
+  // (4-element-aligned rows of codes and z: n and the z stride multiples of 4)
+  prm.epi_t = pl.epi_t && g.epilogue == EPI_ENDPOINT && g.n % 4 == 0 && prm.ldy % 4 == 0 &&
+              (reinterpret_cast<uintptr_t>(g.Y) & 15) == 0 &&
+              (reinterpret_cast<uintptr_t>(g.codes) & 3) == 0;
   prm.P = P; prm.counters = counters;
   prm.status = g.status; prm.spin_limit = spin_limit; prm.finish_wait = g.finish_wait;
 

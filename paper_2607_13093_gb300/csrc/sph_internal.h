@@ -122,6 +122,7 @@ struct TcPlan {
   int single_acc;  // one TMEM accumulator (256-id tiles over > 128 rows)
   int nseg;        // endpoint statistics: 32-id segments per row, NT * tm / 32
   int epi_stats;   // endpoint: softmax statistics in the epilogue (else a pass over z)
+  int epi_t;       // endpoint without them: the epilogue transposes through shared memory
   long long T;
   size_t hs_bytes, p_bytes, cnt_bytes, stats_bytes, scratch_bytes, smem_bytes;
   bool ok;

@@ -820,3 +820,25 @@ def test_fp8_tensor_core_pairs(ctx, rows, keep, schedule, act):
     finally:
         ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
         ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
+
+
+@pytest.mark.parametrize("n_keep", [2004, 3000, 3002])
+@pytest.mark.parametrize("payload", [True, False])
+def test_endpoint_transposed_epilogue(ctx, n_keep, payload):
+    # row blocks of >= 128 rows over a short hidden dimension finish the
+    # endpoint through shared memory when rows are 4-element aligned (2004:
+    # 8-byte code loads on every other row, a ragged last window; 3000: all
+    # aligned; 3002: not aligned, the per-lane path)
+    w = small(V=n_keep + 1500, d=1088, d_l=64, rows=160, n_keep=n_keep, seed=909)
+    if payload:
+        ref = oracle_cloud(w)
+        check_endpoint(ctx, w, torch.from_numpy(ref["codes"]), torch.from_numpy(ref["row_scale"]))
+    else:
+        W_full = torch.cat([w.W_l, w.W_h], dim=1).contiguous()
+        z = torch.empty(w.rows, w.n_keep, device=DEV)
+        tok = ctx.fuse_sample(None, None, w.h, W_full, keep_ids=w.keep_ids, temperature=w.tau,
+                              seed=w.seed, fused_logits_out=z)
+        ctx.sync()
+        zref = oracle.local_partial(np_(w.h), bits(W_full), np_(w.keep_ids))
+        assert_close(np_(z), zref, "unsplit fused logits")
+        assert np.isin(np_(tok), np_(w.keep_ids)).all()

@@ -182,6 +182,10 @@ CHUNKED = [
                             clip=40.0), 768),
     ("one-id-chunks", dict(V=40, d=96, d_l=16, rows=5, n_keep=7, run_lo=1, run_hi=3), 1),
     ("greedy", dict(V=4000, d=1024, d_l=256, rows=24, n_keep=2500, tau=0.0), 1024),
+    # 160-row blocks over d_l = 64: the endpoint's transposed epilogue, with
+    # chunk offsets that keep z's rows 16-byte aligned (1000) or not (1002)
+    ("rows160-1000", dict(V=5000, d=1088, d_l=64, rows=160, n_keep=4000), 1000),
+    ("rows160-1002", dict(V=5000, d=1088, d_l=64, rows=160, n_keep=4000), 1002),
 ]
 
 
