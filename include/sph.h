@@ -142,8 +142,9 @@ typedef enum sph_option {
                                returning SPH_ERR_INVALID_ARG for unsorted,
                                repeated or out-of-range ids.  0 (default):
                                the ids are a precondition, not checked.    */
-  SPH_OPT_TC_PAIR = 11,     /* CTA pairs for the cloud contraction with bf16
-                               weights (clusters of two CTAs, tcgen05
+  SPH_OPT_TC_PAIR = 11,     /* CTA pairs for the tensor-core contractions
+                               (the cloud's with bf16 weights, and the
+                               endpoint's; clusters of two CTAs, tcgen05
                                .cta_group::2): each 256-id tile is one M = 256
                                MMA over both CTAs' shared memory, each CTA
                                loading 128 ids of the weights and half of the
@@ -160,6 +161,19 @@ typedef enum sph_option {
                                epilogue, 2 always a separate quantize pass.
                                The payload, z and tokens are bit-identical
                                either way.                                  */
+  SPH_OPT_ENDPOINT_Z = 12,  /* where sph_fuse_sample and sph_split_step are
+                               not asked for z (fused_logits_out NULL) and
+                               run on tensor cores with the inverse-CDF or
+                               greedy draw: 0 automatic (default: stored),
+                               1 store z in the scratch arena, 2 never store
+                               it.  Unstored, the endpoint contraction's
+                               epilogue keeps the softmax statistics of every
+                               32-id segment and the draw recomputes z for
+                               the 32 ids of the segment it lands in (one
+                               fp32 dot product of d_l per id, CUDA cores):
+                               tokens can differ from the stored path's only
+                               where a draw lies within fp32 rounding of a
+                               CDF step (or greedy ties within it).          */
   SPH_OPT_SAMPLER = 8       /* the draw of sph_fuse_sample at temperature > 0:
                                0 inverse CDF (default), 1 Gumbel-max: the
                                first index j of the largest

@@ -241,11 +241,87 @@ struct StatsWeight {                    // chunk or segment weight relative to M
   float M, inv_tau;
   __device__ float operator()(int s) const { return seg_weight(st[s], M, inv_tau); }
 };
-struct ExpWeight {                      // exp((z_j - M) / tau)
+// A row of fused logits as the draws read it (z(j) for j < n): stored, or
+// recomputed id by id from the endpoint's inputs (ZSource).  A draw reads
+// the 32 ids of one segment, one per lane, so a recomputing lane takes one
+// K-long dot product: the z a draw needs cost 32 weight rows per row
+// instead of a store and a reload of all n.
+struct ZRowStored {
   const float* z;
-  float M, inv_tau;
-  __device__ float operator()(int j) const { return expf((z[j] - M) * inv_tau); }
+  __device__ float operator()(int j) const { return z[j]; }
 };
+struct ZRowRecomputed {
+  const float* h;          // the row's hidden state, K values
+  int K;
+  const uint16_t* W;       // bf16 weight rows, ld_w elements apart (16-byte aligned)
+  int64_t ld_w;
+  const int32_t* ids;      // compact index -> weight row (nullptr: identity)
+  const int8_t* c;         // the row's codes, or nullptr (no payload)
+  float s;                 // the row's scale
+  bool h16;                // h is 16-byte aligned
+  __device__ void dot8(const uint4& wv, int k, float (&a)[4]) const {
+    float x[8];
+    if (h16) {
+      const float4 x0 = __ldg(reinterpret_cast<const float4*>(h + k));
+      const float4 x1 = __ldg(reinterpret_cast<const float4*>(h + k) + 1);
+      x[0] = x0.x; x[1] = x0.y; x[2] = x0.z; x[3] = x0.w;
+      x[4] = x1.x; x[5] = x1.y; x[6] = x1.z; x[7] = x1.w;
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) x[e] = __ldg(h + k + e);
+    }
+    const unsigned u[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {     // element 2e in the low half, 2e + 1 in the high
+      a[e] = fmaf(x[2 * e], __uint_as_float(u[e] << 16), a[e]);
+      a[e] = fmaf(x[2 * e + 1], __uint_as_float(u[e] & 0xFFFF0000u), a[e]);
+    }
+  }
+  __device__ float operator()(int j) const {
+    const int id = ids ? __ldg(ids + j) : j;
+    const uint16_t* w = W + (int64_t)id * ld_w;
+    float a[4] = {0.f, 0.f, 0.f, 0.f};
+    int k = 0;
+    // the draw is latency-bound: eight 16-byte loads of the row in flight
+#pragma unroll 1
+    for (; k + 64 <= K; k += 64) {
+      uint4 wv[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) wv[q] = __ldg(reinterpret_cast<const uint4*>(w + k) + q);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) dot8(wv[q], k + 8 * q, a);
+    }
+#pragma unroll 1
+    for (; k + 8 <= K; k += 8) dot8(__ldg(reinterpret_cast<const uint4*>(w + k)), k, a);
+    for (; k < K; ++k) a[0] = fmaf(__ldg(h + k), __uint_as_float((unsigned)w[k] << 16), a[0]);
+    const float z = (a[0] + a[1]) + (a[2] + a[3]);
+    return c ? fmaf((float)__ldg(c + j), s, z) : z;
+  }
+};
+struct ZRowsStored {
+  const float* Z;
+  int n;
+  __device__ ZRowStored row(int64_t r) const { return ZRowStored{Z + r * n}; }
+};
+struct ZRowsRecomputed {
+  ZSource zs;
+  int n;
+  __device__ ZRowRecomputed row(int64_t r) const {
+    const float* hr = zs.h + r * zs.ld_h;
+    return ZRowRecomputed{hr, zs.K, static_cast<const uint16_t*>(zs.W), zs.ld_w,
+                          zs.ids, zs.codes ? zs.codes + r * n : nullptr,
+                          zs.codes ? __ldg(zs.row_scale + r) : 0.f,
+                          (reinterpret_cast<uintptr_t>(hr) & 15) == 0};
+  }
+};
+
+template <class ZR>
+struct ExpWeightOf {                    // exp((z_j - M) / tau)
+  ZR z;
+  float M, inv_tau;
+  __device__ float operator()(int j) const { return expf((z(j) - M) * inv_tau); }
+};
+using ExpWeight = ExpWeightOf<ZRowStored>;
 // Residual weight of the rejected position: max(0, p_j - q_j), or with
 // greedy drafts (q == nullptr) p_j with the draft id xi removed.
 struct ResidualWeight {
@@ -277,8 +353,9 @@ __device__ __forceinline__ float stats_max(const float2* cst, int nchunk, int la
 // ---------------------------------------------------------------------------
 // sampling: one warp per row
 // ---------------------------------------------------------------------------
+template <class ZRows>
 __global__ void __launch_bounds__(kWarps * 32)
-sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
+sample_seg_kernel(const ZRows zr, int rows, int n,
                   const float2* __restrict__ stats, int nseg,
                   const float2* __restrict__ cstats, const int32_t* __restrict__ ids,
                   float inv_tau, uint64_t seed, uint64_t offset,
@@ -293,7 +370,7 @@ sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
   const float M = stats_max(cst, nchunk, lane);
   const StatsWeight cw{cst, M, inv_tau};
   const StatsWeight sw{stats + (int64_t)r * nseg, M, inv_tau};
-  const ExpWeight ew{Z + (int64_t)r * n, M, inv_tau};
+  const ExpWeightOf<decltype(zr.row(0))> ew{zr.row(r), M, inv_tau};
   const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
   int j;
   warp_draw(nchunk, nseg, n, cw, sw, ew, u, lane, j);
@@ -308,8 +385,9 @@ sample_seg_kernel(const float* __restrict__ Z, int rows, int n,
 // path.
 constexpr int kMaxFusedChunks = 4096;   // shared memory: 8 bytes per chunk
 constexpr int kFusedU = 4;              // chunks in flight per warp
+template <class ZRows>
 __global__ void __launch_bounds__(1024)
-sample_rows_kernel(const float* __restrict__ Z, int n, const float2* __restrict__ stats,
+sample_rows_kernel(const ZRows zr, int n, const float2* __restrict__ stats,
                    int nseg, const int32_t* __restrict__ ids, float inv_tau, uint64_t seed,
                    uint64_t offset, int32_t* __restrict__ tokens) {
   extern __shared__ float2 s_cst[];
@@ -342,7 +420,7 @@ sample_rows_kernel(const float* __restrict__ Z, int n, const float2* __restrict_
   const float M = stats_max(s_cst, nchunk, lane);
   const StatsWeight cw{s_cst, M, inv_tau};
   const StatsWeight sw{srow, M, inv_tau};
-  const ExpWeight ew{Z + (int64_t)r * n, M, inv_tau};
+  const ExpWeightOf<decltype(zr.row(0))> ew{zr.row(r), M, inv_tau};
   const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
   int j;
   warp_draw(nchunk, nseg, n, cw, sw, ew, u, lane, j);
@@ -423,8 +501,10 @@ __device__ __forceinline__ int warp_min_int(int v) {
 }
 
 // The lowest segment holding the row maximum (from its statistics), then the
-// lowest id in it whose z equals that maximum; all lanes return it.
-__device__ __forceinline__ int warp_argmax(const float* z, int n, const float2* st, int nseg,
+// lowest id in it whose z equals the segment's largest z (the maximum
+// itself where z is stored); all lanes return it.
+template <class ZR>
+__device__ __forceinline__ int warp_argmax(const ZR& z, int n, const float2* st, int nseg,
                                            int lane) {
   float M = -INFINITY;
   int sb = nseg;
@@ -436,13 +516,16 @@ __device__ __forceinline__ int warp_argmax(const float* z, int n, const float2* 
   if (!(Mw > -INFINITY)) return 0;
   const int seg = warp_min_int(M == Mw ? sb : nseg);
   const int j = seg * kSeg + lane;
-  const unsigned hit = __ballot_sync(0xFFFFFFFFu, j < n && z[j] == Mw);
+  const float zj = j < n ? z(j) : -INFINITY;
+  const float mz = warp_max(zj);
+  const unsigned hit = __ballot_sync(0xFFFFFFFFu, j < n && zj == mz);
   return hit ? seg * kSeg + __ffs(hit) - 1 : min(seg * kSeg, n - 1);
 }
 
 // One warp per row: vocabulary ids into tokens and/or compact indices.
+template <class ZRows>
 __global__ void __launch_bounds__(kWarps * 32)
-greedy_kernel(const float* __restrict__ Z, int rows, int n, const float2* __restrict__ stats,
+greedy_kernel(const ZRows zr, int rows, int n, const float2* __restrict__ stats,
               int nseg, const int32_t* __restrict__ ids, int32_t* __restrict__ tokens,
               int32_t* __restrict__ compact) {
   ptx::griddep_wait();
@@ -450,7 +533,7 @@ greedy_kernel(const float* __restrict__ Z, int rows, int n, const float2* __rest
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (r >= rows) return;
-  const int j = warp_argmax(Z + (int64_t)r * n, n, stats + (int64_t)r * nseg, nseg, lane);
+  const int j = warp_argmax(zr.row(r), n, stats + (int64_t)r * nseg, nseg, lane);
   if (lane == 0) {
     if (tokens) tokens[r] = ids ? ids[j] : j;
     if (compact) compact[r] = j;
@@ -611,7 +694,7 @@ verify_draw_kernel(const float* __restrict__ Z, int n, const float2* __restrict_
   if (!(tot > 0.f)) {
     const StatsWeight cw{cstats + r * nchunk, ms.x, inv_tau};
     const StatsWeight sw{stats + r * nseg, ms.x, inv_tau};
-    const ExpWeight ew{Z + r * n, ms.x, inv_tau};
+    const ExpWeight ew{ZRowStored{Z + r * n}, ms.x, inv_tau};
     warp_draw(nchunk, nseg, n, cw, sw, ew, u, lane, j);
   }
   if (lane == 0) {
@@ -654,16 +737,44 @@ cudaError_t launch_chunk_stats(const float2* stats, int rows, int nseg, float in
                     dim3(kWarps * 32), 0, st, stats, rows, nseg, nchunk, inv_tau, cstats);
 }
 
-cudaError_t launch_sample_segments(const float* Z, int rows, int n, const float2* stats,
+namespace {
+template <class ZRows>
+cudaError_t sample_segments_with(const ZRows& zr, int rows, int n, const float2* stats,
+                                 int nseg, const float2* cstats, const int32_t* ids,
+                                 float inv_tau, uint64_t seed, uint64_t offset,
+                                 int32_t* tokens, cudaStream_t st, int greedy) {
+  if (greedy)
+    return launch_pdl(greedy_kernel<ZRows>, dim3((rows + kWarps - 1) / kWarps),
+                      dim3(kWarps * 32), 0, st, zr, rows, n, stats, nseg, ids, tokens,
+                      (int32_t*)nullptr);
+  return launch_pdl(sample_seg_kernel<ZRows>, dim3((rows + kWarps - 1) / kWarps),
+                    dim3(kWarps * 32), 0, st, zr, rows, n, stats, nseg, cstats, ids, inv_tau,
+                    seed, offset, tokens);
+}
+template <class ZRows>
+cudaError_t sample_rows_with(const ZRows& zr, int rows, int n, const float2* stats, int nseg,
+                             const int32_t* ids, float inv_tau, uint64_t seed, uint64_t offset,
+                             int32_t* tokens, cudaStream_t st) {
+  const int nchunk = chunk_count(nseg);
+  if (rows < 1 || nchunk > kMaxFusedChunks) return cudaErrorNotSupported;
+  int warps = (nchunk + kFusedU - 1) / kFusedU;
+  warps = warps < 4 ? 4 : (warps > 32 ? 32 : warps);
+  return launch_pdl(sample_rows_kernel<ZRows>, dim3(rows), dim3(warps * 32),
+                    (size_t)nchunk * sizeof(float2), st, zr, n, stats, nseg, ids, inv_tau, seed,
+                    offset, tokens);
+}
+}  // namespace
+
+cudaError_t launch_sample_segments(const ZSource& zs, int rows, int n, const float2* stats,
                                    int nseg, const float2* cstats, const int32_t* ids,
                                    float inv_tau, uint64_t seed, uint64_t offset,
                                    int32_t* tokens, cudaStream_t st, int greedy) {
-  if (greedy)
-    return launch_pdl(greedy_kernel, dim3((rows + kWarps - 1) / kWarps), dim3(kWarps * 32), 0,
-                      st, Z, rows, n, stats, nseg, ids, tokens, (int32_t*)nullptr);
-  return launch_pdl(sample_seg_kernel, dim3((rows + kWarps - 1) / kWarps),
-                    dim3(kWarps * 32), 0, st, Z, rows, n, stats, nseg, cstats, ids, inv_tau,
-                    seed, offset, tokens);
+  if (zs.Z)
+    return sample_segments_with(ZRowsStored{zs.Z, n}, rows, n, stats, nseg, cstats, ids,
+                                inv_tau, seed, offset, tokens, st, greedy);
+  if (!zs.h || !zs.W || zs.K < 1 || (zs.codes && !zs.row_scale)) return cudaErrorInvalidValue;
+  return sample_segments_with(ZRowsRecomputed{zs, n}, rows, n, stats, nseg, cstats, ids,
+                              inv_tau, seed, offset, tokens, st, greedy);
 }
 
 cudaError_t launch_gumbel(const float* Z, int rows, int n, const int32_t* ids, float inv_tau,
@@ -673,16 +784,15 @@ cudaError_t launch_gumbel(const float* Z, int rows, int n, const int32_t* ids, f
                     inv_tau, seed, offset, tokens);
 }
 
-cudaError_t launch_sample_rows(const float* Z, int rows, int n, const float2* stats,
+cudaError_t launch_sample_rows(const ZSource& zs, int rows, int n, const float2* stats,
                                int nseg, const int32_t* ids, float inv_tau, uint64_t seed,
                                uint64_t offset, int32_t* tokens, cudaStream_t st) {
-  const int nchunk = chunk_count(nseg);
-  if (rows < 1 || nchunk > kMaxFusedChunks) return cudaErrorNotSupported;
-  int warps = (nchunk + kFusedU - 1) / kFusedU;
-  warps = warps < 4 ? 4 : (warps > 32 ? 32 : warps);
-  return launch_pdl(sample_rows_kernel, dim3(rows), dim3(warps * 32),
-                    (size_t)nchunk * sizeof(float2), st, Z, n, stats, nseg, ids, inv_tau, seed,
-                    offset, tokens);
+  if (zs.Z)
+    return sample_rows_with(ZRowsStored{zs.Z, n}, rows, n, stats, nseg, ids, inv_tau, seed,
+                            offset, tokens, st);
+  if (!zs.h || !zs.W || zs.K < 1 || (zs.codes && !zs.row_scale)) return cudaErrorInvalidValue;
+  return sample_rows_with(ZRowsRecomputed{zs, n}, rows, n, stats, nseg, ids, inv_tau, seed,
+                          offset, tokens, st);
 }
 
 // Scratch: stats [R][nseg] float2 | chunk stats [R][nchunk] float2 | rowMS
@@ -722,8 +832,9 @@ cudaError_t launch_verify(const float* Z, int sessions, int k, int n, const int3
     // area), then one thread per session
     int32_t* amax = reinterpret_cast<int32_t*>(rowMS);
     if (e == cudaSuccess)
-      e = launch_pdl(greedy_kernel, dim3((R + kWarps - 1) / kWarps), dim3(kWarps * 32), 0, st,
-                     Z, R, n, (const float2*)stats, nseg, ids, (int32_t*)nullptr, amax);
+      e = launch_pdl(greedy_kernel<ZRowsStored>, dim3((R + kWarps - 1) / kWarps),
+                     dim3(kWarps * 32), 0, st, ZRowsStored{Z, n}, R, n, (const float2*)stats,
+                     nseg, ids, (int32_t*)nullptr, amax);
     if (e == cudaSuccess)
       e = launch_pdl(greedy_verify_kernel, dim3((sessions + 127) / 128), dim3(128), 0, st,
                      (const int32_t*)amax, sessions, k, n, ids, V, draft, n_acc, next_token);

@@ -74,6 +74,9 @@ constexpr int kBarrierArea = 512;
 // (+4 words of padding per row, so that both the row writes and the 16-byte
 // reads are free of bank conflicts)
 constexpr int kTRow = 36;
+// Kernel instantiations of EPI_ENDPOINT that finish through the per-warp
+// shared-memory transpose (finish_chunk_t) rather than per lane.
+constexpr int EPI_ENDPOINT_T = 3;
 constexpr int kTransposeBytes = 8 /* epilogue warps */ * 8 * kTRow * 4;
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
@@ -118,7 +121,6 @@ struct TcParams {
   int8_t* codes_out;           // fused endpoint: the payload codes [R][n] (out)
   float* scale_out;            // fused endpoint: the row scales [R] (out)
   float2* seg_stats;           // endpoint: [R][nseg] (max, sum exp)
-  int epi_t;                   // endpoint without statistics: transposed epilogue
   int a3d;                     // full vocabulary: A by one 3-D copy per stage
   int single_acc;              // one accumulator (no epilogue overlap): 256-id tiles of > 128 rows
   float* P;                    // split-tile partials [2 * grid][BN][TM]
@@ -259,7 +261,7 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const int r = row0 + q;
-      if (vj && r < p.R) p.Y[(int64_t)r * p.ldy + j] = z[q];
+      if (p.Y && vj && r < p.R) p.Y[(int64_t)r * p.ldy + j] = z[q];
     }
     if (!p.seg_stats) return;          // statistics come from a pass over z
     // softmax statistics of this 32-id segment for each row: the maxima,
@@ -277,15 +279,16 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
   }
 }
 
-// Endpoint epilogue without statistics (Eq. 13: z = code * s + local
-// partial), through this warp's shared-memory tile `tb` [8][kTRow]: the
-// 16 rows of a chunk go in two halves of 8; after the transpose lane l holds
-// row (l >> 2) of the half and the 8 consecutive ids 8 (l & 3) .. + 7 of the
-// warp's 32, so its payload is one 8-byte (or two 4-byte) load and its z two
-// 16-byte stores, instead of 16 one-byte loads and 16 strided stores per
-// lane.  Used when rows of codes and z are 4-element aligned (n and the z
-// row stride multiples of 4).  The payload of a chunk does not depend on the
-// accumulator, so it is loaded a chunk ahead (TPay).
+// Endpoint epilogue through this warp's shared-memory tile `tb` [8][kTRow]
+// (Eq. 13: z = code * s + local partial): the 16 rows of a chunk go in two
+// halves of 8; after the transpose lane l holds row (l >> 2) of the half and
+// the 8 consecutive ids 8 (l & 3) .. + 7 of the warp's 32, so its payload is
+// one 8-byte load and its z two 16-byte stores (narrower where a row is less
+// aligned), instead of 16 one-byte loads and 16 strided stores per lane, and
+// the 32-id segment statistics of a row are a reduction over four lanes.
+// Used when rows of codes (and of z, where z is stored) are 2-element
+// aligned.  The payload of a chunk does not depend on the accumulator, so it
+// is loaded a chunk ahead (TPay).
 struct TPay {
   uint2 cw[2];     // the 8 codes of this lane's row and ids, per half
   float sc[2];     // that row's scale, per half (0 past the rows)
@@ -301,13 +304,18 @@ __device__ __forceinline__ void load_tpay(const TcParams& p, int row0, int j0w, 
     const int j = j0w + 8 * seg;
     if (!p.codes || r >= p.R || j >= p.n) continue;
     t.sc[h8] = __ldg(p.row_scale + r);
-    const int8_t* cp = p.codes + (int64_t)r * p.n + j;     // 4-byte aligned
+    const int8_t* cp = p.codes + (int64_t)r * p.n + j;     // 2-byte aligned
+    const uintptr_t ca = reinterpret_cast<uintptr_t>(cp);
     if (j + 8 <= p.n) {
-      if ((reinterpret_cast<uintptr_t>(cp) & 7) == 0) {
+      if ((ca & 7) == 0) {
         t.cw[h8] = __ldg(reinterpret_cast<const uint2*>(cp));
-      } else {
+      } else if ((ca & 3) == 0) {
         t.cw[h8].x = __ldg(reinterpret_cast<const unsigned*>(cp));
         t.cw[h8].y = __ldg(reinterpret_cast<const unsigned*>(cp) + 1);
+      } else {
+        const unsigned short* hp = reinterpret_cast<const unsigned short*>(cp);
+        t.cw[h8].x = (unsigned)__ldg(hp) | ((unsigned)__ldg(hp + 1) << 16);
+        t.cw[h8].y = (unsigned)__ldg(hp + 2) | ((unsigned)__ldg(hp + 3) << 16);
       }
     } else {                                   // the row's last ids
       unsigned w[2] = {0u, 0u};
@@ -331,7 +339,7 @@ __device__ __forceinline__ void finish_chunk_t(const TcParams& p, const float (&
     __syncwarp();
     const int r = row0 + h8 * 8 + q;
     const int j = j0w + 8 * seg;
-    if (r >= p.R || j >= p.n) continue;
+    const bool rv = r < p.R;
     float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
     const float sc = pay.sc[h8];
 #pragma unroll
@@ -339,14 +347,39 @@ __device__ __forceinline__ void finish_chunk_t(const TcParams& p, const float (&
       x[e] += (float)(int8_t)((pay.cw[h8].x >> (8 * e)) & 0xFF) * sc;
       x[4 + e] += (float)(int8_t)((pay.cw[h8].y >> (8 * e)) & 0xFF) * sc;
     }
-    float* zp = p.Y + (int64_t)r * p.ldy + j;                 // 16-byte aligned
-    if (j + 8 <= p.n) {
-      reinterpret_cast<float4*>(zp)[0] = make_float4(x[0], x[1], x[2], x[3]);
-      reinterpret_cast<float4*>(zp)[1] = make_float4(x[4], x[5], x[6], x[7]);
-    } else {
+    if (p.Y && rv && j < p.n) {
+      float* zp = p.Y + (int64_t)r * p.ldy + j;               // 8-byte aligned
+      if (j + 8 <= p.n && (reinterpret_cast<uintptr_t>(zp) & 15) == 0) {
+        reinterpret_cast<float4*>(zp)[0] = make_float4(x[0], x[1], x[2], x[3]);
+        reinterpret_cast<float4*>(zp)[1] = make_float4(x[4], x[5], x[6], x[7]);
+      } else if (j + 8 <= p.n) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          reinterpret_cast<float2*>(zp)[e] = make_float2(x[2 * e], x[2 * e + 1]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+          if (j + e < p.n) zp[e] = x[e];
+      }
+    }
+    if (p.seg_stats) {
+      // this row's 32-id segment: (max z, sum of exp((z - max) / tau)) over
+      // its ids below n, from the four lanes that hold it
 #pragma unroll
       for (int e = 0; e < 8; ++e)
-        if (j + e < p.n) zp[e] = x[e];
+        if (!rv || j + e >= p.n) x[e] = -INFINITY;
+      float m = fmaxf(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])),
+                      fmaxf(fmaxf(x[4], x[5]), fmaxf(x[6], x[7])));
+      m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, 1));
+      m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, 2));
+      float sum = 0.f;
+      if (m > -INFINITY) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) sum += expf((x[e] - m) * p.inv_tau);   // exp(-inf) = 0
+      }
+      sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 1);
+      sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 2);
+      if (seg == 0 && rv) p.seg_stats[(int64_t)r * p.nseg + (j0w >> 5)] = make_float2(m, sum);
     }
   }
 }
@@ -773,9 +806,10 @@ tc_kernel(const __grid_constant__ WMaps wm,
       auto J = [&](int hf) { return (kHalves > 1 && hf) ? jh[kHalves - 1] : jh[0]; };
       auto VJ = [&](int hf) { return (kHalves > 1 && hf) ? vjh[kHalves - 1] : vjh[0]; };
       auto ID = [&](int hf) { return (kHalves > 1 && hf) ? idh[kHalves - 1] : idh[0]; };
-      // the endpoint without statistics finishes chunks through this warp's
-      // transpose tile (no per-lane payload registers then)
-      const bool epi_t = EPI == EPI_ENDPOINT && p.epi_t;
+      // the endpoint through this warp's transpose tile (no per-lane
+      // payload registers then)
+      constexpr bool epi_t = EPI == EPI_ENDPOINT_T;
+      constexpr bool lane_pay = EPI == EPI_ENDPOINT || EPI == EPI_FUSED;
       float* tb = reinterpret_cast<float*>(base + (size_t)S * stage_bytes + kBarrierArea +
                                            kMaxBoxes * sizeof(int2)) +
                   (warp - 2) * 8 * kTRow;
@@ -787,15 +821,28 @@ tc_kernel(const __grid_constant__ WMaps wm,
         for (int hf = 0; hf < kHalves; ++hf)
           prefetch_payload<EPI>(p, rb * BN + grp * (BN / 2), BN / 2,
                                 t * kTileStride + half * 128 + hf * 128 + quad * 32, lane);
-        if (whole && grp < nhc && !epi_t)
-          load_payload<EPI>(p, rb * BN + (grp % nch) * 16, J(grp / nch), lane, pay);
+        if constexpr (lane_pay)
+          if (whole && grp < nhc)
+            load_payload<EPI>(p, rb * BN + (grp % nch) * 16, J(grp / nch), lane, pay);
       }
-      TPay tpay;
-      if (epi_t && whole && grp < nhc)
-        load_tpay(p, rb * BN + (grp % nch) * 16, J(grp / nch) - lane, lane, tpay);
+      // the transposed payload of whole tiles runs kTAhead chunks ahead of
+      // the one being finished (tq[a]: chunk hc + (a + 1) kEpiGroups): a
+      // chunk's work is shorter than a load's latency under the kernel's
+      // own traffic
+      constexpr int kTAhead = 3;
+      TPay tpay, tq[kTAhead];
+      if (epi_t && whole) {
+#pragma unroll
+        for (int a = 0; a <= kTAhead; ++a) {
+          const int hn = grp + a * kEpiGroups;
+          if (hn < nhc)
+            load_tpay(p, rb * BN + (hn % nch) * 16, J(hn / nch) - lane, lane,
+                      a == 0 ? tpay : tq[a - 1]);
+        }
+      }
       // (split tiles load the transposed payload right before finishing)
       auto finish = [&](const float (&vv)[16], int hf, int ch) {
-        if (epi_t) {
+        if constexpr (epi_t) {
           if (!whole) load_tpay(p, rb * BN + ch * 16, J(hf) - lane, lane, tpay);
           finish_chunk_t(p, vv, rb * BN + ch * 16, J(hf) - lane, lane, tb, tpay);
         } else {
@@ -891,17 +938,23 @@ tc_kernel(const __grid_constant__ WMaps wm,
           Payload nxt;
           const int hn = hc + kEpiGroups;
           TPay tnxt;
-          if (EPI != EPI_CLOUD && hn < nhc && !epi_t)
-            load_payload<EPI>(p, rb * BN + (hn % nch) * 16, J(hn / nch), lane, nxt);
-          if (epi_t && hn < nhc)
-            load_tpay(p, rb * BN + (hn % nch) * 16, J(hn / nch) - lane, lane, tnxt);
+          if constexpr (lane_pay)
+            if (hn < nhc) load_payload<EPI>(p, rb * BN + (hn % nch) * 16, J(hn / nch), lane, nxt);
+          const int ht = hc + (kTAhead + 1) * kEpiGroups;
+          if (epi_t && ht < nhc)
+            load_tpay(p, rb * BN + (ht % nch) * 16, J(ht / nch) - lane, lane, tnxt);
           finish(v, hf, ch);
-          if constexpr (EPI != EPI_CLOUD) pay = nxt;
-          if (epi_t) tpay = tnxt;
+          if constexpr (lane_pay) pay = nxt;
+          if constexpr (epi_t) {
+            tpay = tq[0];
+#pragma unroll
+            for (int a = 0; a + 1 < kTAhead; ++a) tq[a] = tq[a + 1];
+            tq[kTAhead - 1] = tnxt;
+          }
         } else if (known_last) {
           // the partials in CTA order (the same order, and so the same
           // result, as the fix-up below), this CTA's own from registers
-          if (EPI != EPI_CLOUD && !epi_t) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
+          if constexpr (lane_pay) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
           const int me = unit - c0;
           const size_t o = (size_t)ch * 16 * TM + i;
           float s[16];
@@ -952,7 +1005,7 @@ tc_kernel(const __grid_constant__ WMaps wm,
             ps[c] = p.P + (size_t)slot_of(c < C ? c : 0) * BN * TM + quad * 32 + lane;
           for (int hc = grp; hc < nhc; hc += kEpiGroups) {
             const int hf = hc / nch, ch = hc - hf * nch;
-            if (EPI != EPI_CLOUD && !epi_t) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
+            if constexpr (lane_pay) load_payload<EPI>(p, rb * BN + ch * 16, J(hf), lane, pay);
             const size_t o = (size_t)ch * 16 * TM + hf * 128;
             float v[16];
 #pragma unroll
@@ -1279,7 +1332,7 @@ namespace {
 // 32, so that each CTA's half is whole 16-row groups), work split over the
 // pairs (a multiple of the row-block count, as below).
 TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pairs,
-                    int schedule, int max_stages, int block_k, int max_bn_opt) {
+                    int schedule, int max_stages, int block_k, int max_bn_opt, int endpoint) {
   // (e4m3 weights: four or two h planes; 128-row blocks keep four stages)
   int cap = pl.fp8 ? 128 : 256;
   if (max_bn_opt >= 32 && max_bn_opt < cap) cap = max_bn_opt / 32 * 32;
@@ -1311,7 +1364,11 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
   pl.whole_tiles = schedule == 1 || (schedule == 0 && whole_span <= 1.1 * split_span + 2.0);
   units = pl.whole_tiles ? g_whole : (int)(pl.T < units ? pl.T : units);
   pl.G = 2 * units;
-  pl.stages = (int)((kSmemBudget - 2048) / stage_of(pl.na));
+  // the endpoint's epilogue as on single CTAs (each CTA of a pair finishes
+  // its own 128 ids for all BN rows)
+  pl.epi_stats = endpoint == 2 || (endpoint && (pl.BN < 128 || 4 * pl.BN <= K));
+  pl.epi_t = endpoint == 2 || (endpoint && !pl.epi_stats);
+  pl.stages = (int)((kSmemBudget - 2048 - (pl.epi_t ? kTransposeBytes : 0)) / stage_of(pl.na));
   if (pl.stages > kMaxStages) pl.stages = kMaxStages;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
   pl.hs_bytes = pl.fp8 ? align256((size_t)pl.hilo * pl.Rp * pl.Kp) + align256((size_t)pl.Rp * 4)
@@ -1320,11 +1377,10 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
   pl.p_bytes = splits ? align256((size_t)2 * pl.G * pl.BN * 128 * 4) : 0;
   pl.cnt_bytes = align256((size_t)tiles * 4 * kEpiGroups * 2 * sizeof(int));
   pl.nseg = pl.NT * 8;
-  pl.stats_bytes = 0;
-  pl.epi_stats = 0;
-  pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes;
+  pl.stats_bytes = endpoint ? align256((size_t)rows * pl.nseg * sizeof(float2)) : 0;
+  pl.scratch_bytes = pl.hs_bytes + pl.p_bytes + pl.cnt_bytes + pl.stats_bytes;
   pl.smem_bytes = 1024 + (size_t)pl.stages * stage_of(pl.na) + kBarrierArea +
-                  kMaxBoxes * sizeof(int2);
+                  kMaxBoxes * sizeof(int2) + (pl.epi_t ? kTransposeBytes : 0);
   pl.ok = pl.stages >= 2;
   return pl;
 }
@@ -1347,12 +1403,15 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   // stages) 1746 vs 2005; 256 rows x 256000 fp32 737 vs 897; 320 rows x
   // 51302 x 3584 bf16 161 vs 195, fp32 (160-row blocks) 242 vs 223; 32
   // rows x 12000 x 3840 38.9 vs 37.2; 64 rows x 256000 x 4608 471 vs 433.
+  // The endpoint (K = d_l) pairs by the same rule: its B bytes per MMA are
+  // most of its traffic (measured 1024 rows x 256000 ids x 512: 665 vs 721
+  // us; 256 rows: 189 vs 408).
   // (an explicitly set tile height keeps single-CTA tiles unless pairs are
   // forced)
-  if (pair_mode > 0 && !endpoint && sm_count >= 2 && (tile_m == 0 || pair_mode == 2)) {
+  if (pair_mode > 0 && sm_count >= 2 && (tile_m == 0 || pair_mode == 2)) {
     pl.pair = 1;
     const TcPlan pp = tc_plan_pair(pl, rows, n, K, sm_count, max_pairs, schedule, max_stages,
-                                   block_k, max_bn_opt);
+                                   block_k, max_bn_opt, endpoint);
     if (pair_mode == 2 || (!fp8 && (pp.BN >= 192 || (pl.hilo == 1 && pp.BN >= 128)))) return pp;
     pl.pair = 0;
   }
@@ -1433,10 +1492,12 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   pl.whole_tiles = schedule == 1 || (schedule == 0 && whole_span <= 1.1 * split_span + 2.0);
   pl.G = pl.whole_tiles ? g_whole : (int)(pl.T < sm_use ? pl.T : sm_use);
   const int stage_bytes = pl.na * (halves * kAtomBytes + pl.hilo * pl.BN * 128);
-  // endpoint without epilogue statistics: the epilogue transposes each
-  // warp's chunk through shared memory (kTransposeBytes beside the stages)
-  pl.epi_stats = endpoint && (pl.BN < 128 || 4 * pl.BN <= K);
-  pl.epi_t = endpoint && !pl.epi_stats;
+  // endpoint: the epilogue makes the segment statistics where z is not
+  // stored (endpoint == 2) or where the hidden dimension hides them (below);
+  // without them, or without z, it transposes each warp's chunk through
+  // shared memory (kTransposeBytes beside the stages)
+  pl.epi_stats = endpoint == 2 || (endpoint && (pl.BN < 128 || 4 * pl.BN <= K));
+  pl.epi_t = endpoint == 2 || (endpoint && !pl.epi_stats);
   pl.stages = (int)((kSmemBudget - 2048 - (pl.epi_t ? kTransposeBytes : 0)) / stage_bytes);
   if (pl.stages > kMaxStages) pl.stages = kMaxStages;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
@@ -1527,7 +1588,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                       long long spin_limit, cudaStream_t st) {
   const bool fp8 = g.w_dtype == W_FP8;
   if (!pl.ok || (fp8 != (pl.fp8 != 0)) || (fp8 && g.epilogue != EPI_CLOUD) ||
-      (pl.pair && (g.epilogue != EPI_CLOUD || pl.G % 2 || pl.BN % 32)) ||
+      (pl.pair && (pl.G % 2 || pl.BN % 32)) ||
       (g.epilogue != EPI_CLOUD && pl.hilo != 2) ||
       (g.epilogue == EPI_FUSED && (!g.yc || !g.rowmax_in || !g.codes_out || !g.scale_out)))
     return cudaErrorNotSupported;
@@ -1600,10 +1661,11 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   prm.rowmax = g.rowmax; prm.codes = g.codes; prm.row_scale = g.row_scale;
   prm.single_acc = pl.single_acc;
   prm.inv_tau = g.inv_tau; prm.seg_stats = (pl.epi_stats && !g.no_stats) ? stats : nullptr; prm.a3d = a3d;
-  // (4-element-aligned rows of codes and z: n and the z stride multiples of 4)
-  prm.epi_t = pl.epi_t && g.epilogue == EPI_ENDPOINT && g.n % 4 == 0 && prm.ldy % 4 == 0 &&
-              (reinterpret_cast<uintptr_t>(g.Y) & 15) == 0 &&
-              (reinterpret_cast<uintptr_t>(g.codes) & 3) == 0;
+  // (2-element-aligned rows of codes and of a stored z: n and the z stride
+  // even)
+  const bool et = pl.epi_t && g.epilogue == EPI_ENDPOINT && g.n % 2 == 0 &&
+                 (!g.Y || (prm.ldy % 2 == 0 && (reinterpret_cast<uintptr_t>(g.Y) & 7) == 0)) &&
+                 (reinterpret_cast<uintptr_t>(g.codes) & 1) == 0;
   prm.P = P; prm.counters = counters;
   prm.status = g.status; prm.spin_limit = spin_limit; prm.finish_wait = g.finish_wait;
 
@@ -1615,6 +1677,15 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                  : launch_inst<4, false, EPI_CLOUD, true, 128, true>(mw, mh, prm, pl, st);
   }
   if (pl.pair) {
+    if (g.epilogue == EPI_FUSED)
+      return gather ? launch_inst<2, true, EPI_FUSED, false, 128, true>(mw, mh, prm, pl, st)
+                    : launch_inst<2, false, EPI_FUSED, false, 128, true>(mw, mh, prm, pl, st);
+    if (et)
+      return gather ? launch_inst<2, true, EPI_ENDPOINT_T, false, 128, true>(mw, mh, prm, pl, st)
+                    : launch_inst<2, false, EPI_ENDPOINT_T, false, 128, true>(mw, mh, prm, pl, st);
+    if (g.epilogue == EPI_ENDPOINT)
+      return gather ? launch_inst<2, true, EPI_ENDPOINT, false, 128, true>(mw, mh, prm, pl, st)
+                    : launch_inst<2, false, EPI_ENDPOINT, false, 128, true>(mw, mh, prm, pl, st);
     if (gather) return hilo2 ? launch_inst<2, true, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st)
                              : launch_inst<1, true, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st);
     return hilo2 ? launch_inst<2, false, EPI_CLOUD, false, 128, true>(mw, mh, prm, pl, st)
@@ -1637,6 +1708,9 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
     if (g.epilogue == EPI_FUSED)
       return gather ? launch_inst<2, true, EPI_FUSED, false, 256>(mw, mh, prm, pl, st)
                     : launch_inst<2, false, EPI_FUSED, false, 256>(mw, mh, prm, pl, st);
+    if (et)
+      return gather ? launch_inst<2, true, EPI_ENDPOINT_T, false, 256>(mw, mh, prm, pl, st)
+                    : launch_inst<2, false, EPI_ENDPOINT_T, false, 256>(mw, mh, prm, pl, st);
     return gather ? launch_inst<2, true, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st)
                   : launch_inst<2, false, EPI_ENDPOINT, false, 256>(mw, mh, prm, pl, st);
   }
@@ -1655,11 +1729,14 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   if (g.epilogue == EPI_FUSED)
     return gather ? launch_inst<2, true, EPI_FUSED>(mw, mh, prm, pl, st)
                   : launch_inst<2, false, EPI_FUSED>(mw, mh, prm, pl, st);
+  if (et)
+    return gather ? launch_inst<2, true, EPI_ENDPOINT_T>(mw, mh, prm, pl, st)
+                  : launch_inst<2, false, EPI_ENDPOINT_T>(mw, mh, prm, pl, st);
   return gather ? launch_inst<2, true, EPI_ENDPOINT>(mw, mh, prm, pl, st)
                 : launch_inst<2, false, EPI_ENDPOINT>(mw, mh, prm, pl, st);
 }
 
-cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPlan& pl,
+cudaError_t launch_sample_from_stats(const ZSource& zs, int rows, int n, const TcPlan& pl,
                                      const void* scratch, float2* cstats,
                                      const int32_t* ids, float inv_tau, uint64_t seed,
                                      uint64_t offset, int sm_count, int32_t* tokens,
@@ -1668,21 +1745,22 @@ cudaError_t launch_sample_from_stats(const float* Z, int rows, int n, const TcPl
   const float2* stats =
       reinterpret_cast<const float2*>(sc + pl.hs_bytes + pl.p_bytes + pl.cnt_bytes);
   if (!pl.epi_stats) {
+    if (!zs.Z) return cudaErrorInvalidValue;
     float2* sst = const_cast<float2*>(stats);
-    cudaError_t e = launch_seg_stats(Z, rows, n, inv_tau, sst, cstats, sm_count, st);
+    cudaError_t e = launch_seg_stats(zs.Z, rows, n, inv_tau, sst, cstats, sm_count, st);
     if (e != cudaSuccess) return e;
-    return launch_sample_segments(Z, rows, n, sst, seg_count(n), cstats, ids, inv_tau, seed,
+    return launch_sample_segments(zs, rows, n, sst, seg_count(n), cstats, ids, inv_tau, seed,
                                   offset, tokens, st, greedy);
   }
   const int nseg = pl.nseg;
   if (greedy)   // the segment maxima are all greedy decoding needs
-    return launch_sample_segments(Z, rows, n, stats, nseg, nullptr, ids, inv_tau, seed, offset,
+    return launch_sample_segments(zs, rows, n, stats, nseg, nullptr, ids, inv_tau, seed, offset,
                                   tokens, st, 1);
   if (chunk_count(nseg) <= 4096)
-    return launch_sample_rows(Z, rows, n, stats, nseg, ids, inv_tau, seed, offset, tokens, st);
+    return launch_sample_rows(zs, rows, n, stats, nseg, ids, inv_tau, seed, offset, tokens, st);
   cudaError_t e = launch_chunk_stats(stats, rows, nseg, inv_tau, cstats, sm_count, st);
   if (e != cudaSuccess) return e;
-  return launch_sample_segments(Z, rows, n, stats, nseg, cstats, ids, inv_tau, seed, offset,
+  return launch_sample_segments(zs, rows, n, stats, nseg, cstats, ids, inv_tau, seed, offset,
                                 tokens, st);
 }
 

@@ -40,6 +40,7 @@ struct sph_ctx {
   int check_ids = 0;                // SPH_OPT_CHECK_IDS
   int split_quantize = 0;           // SPH_OPT_SPLIT_QUANTIZE
   int tc_pair = 0;                  // SPH_OPT_TC_PAIR: 0 automatic, 1 always, 2 never
+  int endpoint_z = 0;               // SPH_OPT_ENDPOINT_Z: 0 automatic, 1 store, 2 recompute
   int pair_units = 0;               // CTA pairs that fit at once (0: pairs unavailable)
   // chunked split steps: the endpoint's own stream (created on first use
   // when the caller passes none) and the events that order the two streams
@@ -153,16 +154,20 @@ size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_
   // the larger of the two paths, for the plan the call makes (tile height
   // as set, 0 automatic) and, with the automatic height, for both heights
   // (which smaller calls may choose)
+  // (and with and without CTA pairs, which some endpoint calls leave out)
+  const int pms[2] = {0, pair_mode(ctx)};
   for (int gather = 0; gather < 2; ++gather)
-    for (int tm = 0; tm <= 256; tm += 128) {
-      if (ctx->tc_tile_m && tm != ctx->tc_tile_m) continue;
-      const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, sm_count,
-                                    endpoint, ctx->tc_schedule, ctx->tc_stages,
-                                    ctx->tc_block_k, gather, w_dtype == sph::W_FP8,
-                                    ctx->tc_max_bn, tm, pair_mode(ctx), ctx->pair_units)
-                           .scratch_bytes;
-      if (x > b) b = x;
-    }
+    for (int tm = 0; tm <= 256; tm += 128)
+      for (int pi = 0; pi < (pms[1] ? 2 : 1); ++pi) {
+        const int pm = pms[pi];
+        if (ctx->tc_tile_m && tm != ctx->tc_tile_m) continue;
+        const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, sm_count,
+                                      endpoint, ctx->tc_schedule, ctx->tc_stages,
+                                      ctx->tc_block_k, gather, w_dtype == sph::W_FP8,
+                                      ctx->tc_max_bn, tm, pm, ctx->pair_units)
+                             .scratch_bytes;
+        if (x > b) b = x;
+      }
   return b;
 }
 
@@ -321,9 +326,12 @@ sph_status traced_status(sph_ctx* ctx, int cls, F&& launch) {
 // The endpoint half of a step on a prepared GatherGemm (EPI_ENDPOINT or
 // EPI_FUSED, gg.Y = z): the local contraction with its fused epilogue, then
 // the draw (S7-S11), on the context's stream.  `c` carves the rest of the
-// scratch arena.
+// scratch arena.  z_out: the caller asked for z (gg.Y is its buffer);
+// otherwise gg.Y is scratch, and z need not be stored at all
+// (SPH_OPT_ENDPOINT_Z): the epilogue then keeps only the segment
+// statistics and the draw recomputes z for the segment it lands in.
 sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temperature,
-                         uint64_t seed, uint64_t offset, int32_t* tokens) {
+                         uint64_t seed, uint64_t offset, int32_t* tokens, bool z_out) {
   const int rows = gg.rows, n_keep = gg.n;
   const int32_t* keep_ids = gg.ids;
   float* Z = gg.Y;
@@ -334,6 +342,22 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
   // Gumbel-max draws need no softmax statistics: the epilogue skips them
   const bool gumbel = ctx->sampler == 1 && !greedy;
   gg.no_stats = gumbel;
+  // unstored z (SPH_OPT_ENDPOINT_Z = 2; not automatic: measured slower on
+  // 1024 x 256000 ids x d_l 512, 32 x 12000 x 256 and 1024 x 256000 x 5120,
+  // faster on 256 x 152064 x 1024)
+  const bool tc = use_tc(ctx, rows, sph::W_BF16);
+  const bool z_free = tc && !gumbel && !z_out && ctx->endpoint_z == 2;
+  sph::ZSource zs;
+  if (z_free) {
+    gg.Y = nullptr;
+    zs.h = gg.h; zs.ld_h = gg.ld_h; zs.K = gg.K; zs.W = gg.W; zs.ld_w = gg.ld_w;
+    zs.ids = gg.ids;
+    const bool fq = gg.epilogue == sph::EPI_FUSED;
+    zs.codes = fq ? gg.codes_out : gg.codes;
+    zs.row_scale = fq ? gg.scale_out : gg.row_scale;
+  } else {
+    zs.Z = Z;
+  }
   sph_status st;
   auto draw_gumbel = [&] {
     return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
@@ -342,11 +366,13 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
                                                      ctx->stream);
                          }), "sample launch");
   };
-  if (use_tc(ctx, rows, sph::W_BF16)) {
+  if (tc) {
     const sph::TcPlan pl = sph::tc_plan(rows, n_keep, gg.K, 0,
-                                        ctx->sm_count, 1, ctx->tc_schedule, ctx->tc_stages,
+                                        ctx->sm_count, z_free ? 2 : 1, ctx->tc_schedule,
+                                        ctx->tc_stages,
                                         ctx->tc_block_k, keep_ids != nullptr, 0,
-                                        ctx->tc_max_bn, ctx->tc_tile_m);
+                                        ctx->tc_max_bn, ctx->tc_tile_m, pair_mode(ctx),
+                                        ctx->pair_units);
     void* tcs = c.take(pl.scratch_bytes);
     if (!c.fits())
       return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
@@ -358,7 +384,7 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
     if (gumbel) return draw_gumbel();
     return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                            return sph::launch_sample_from_stats(
-                               Z, rows, n_keep, pl, tcs, cstats, keep_ids,
+                               zs, rows, n_keep, pl, tcs, cstats, keep_ids,
                                gg.inv_tau, seed, offset, ctx->sm_count, tokens,
                                ctx->stream, greedy);
                          }), "sample launch");
@@ -651,6 +677,10 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "split_quantize must be 0, 1 or 2");
       ctx->split_quantize = (int)value;
       return SPH_OK;
+    case SPH_OPT_ENDPOINT_Z:
+      if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "endpoint_z must be 0, 1 or 2");
+      ctx->endpoint_z = (int)value;
+      return SPH_OK;
     case SPH_OPT_CHECK_IDS:
       if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "check_ids must be 0 or 1");
       ctx->check_ids = (int)value;
@@ -807,7 +837,7 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
   gg.ids = keep_ids; gg.n = (int)n_keep;
   gg.epilogue = sph::EPI_ENDPOINT;
   gg.Y = Z; gg.codes = codes; gg.row_scale = row_scale;
-  return endpoint_draw(ctx, gg, c, temperature, seed, offset, tokens);
+  return endpoint_draw(ctx, gg, c, temperature, seed, offset, tokens, fused_logits_out != nullptr);
 }
 
 sph_status sph_verify_draft(sph_ctx* ctx, const float* target_logits,
@@ -979,7 +1009,8 @@ sph_status sph_split_step(sph_ctx* ctx, const float* h, int64_t rows, int64_t ld
       gg.epilogue = sph::EPI_ENDPOINT;
       gg.codes = codes; gg.row_scale = scales;
     }
-    return endpoint_draw(ctx, gg, c, temperature, seed, offset, tokens);
+    return endpoint_draw(ctx, gg, c, temperature, seed, offset, tokens,
+                         fused_logits_out != nullptr);
   }
 
   // chunks: the cloud emits chunk q (codes + a scale per row) on the

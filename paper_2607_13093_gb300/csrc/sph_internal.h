@@ -122,7 +122,8 @@ struct TcPlan {
   int single_acc;  // one TMEM accumulator (256-id tiles over > 128 rows)
   int nseg;        // endpoint statistics: 32-id segments per row, NT * tm / 32
   int epi_stats;   // endpoint: softmax statistics in the epilogue (else a pass over z)
-  int epi_t;       // endpoint without them: the epilogue transposes through shared memory
+  int epi_t;       // endpoint: the epilogue may finish through a shared-memory transpose
+                   // (where rows are 2-element aligned; shared memory reserved for it)
   long long T;
   size_t hs_bytes, p_bytes, cnt_bytes, stats_bytes, scratch_bytes, smem_bytes;
   bool ok;
@@ -146,11 +147,29 @@ int tc_pair_max_units(int device);
 // plan.scratch_bytes bytes.  bf16 weights only.
 cudaError_t launch_tc(const GatherGemm& g, const TcPlan& plan, void* scratch,
                       long long spin_limit, cudaStream_t st);
+// Where a draw finds the fused logits of the ids it visits (the 32 ids of
+// the segment it lands in): stored in Z (fp32 [rows, n]), or, with Z null,
+// recomputed for just those ids from the endpoint call's own inputs (Eq. 13),
+//   z[r, j] = codes[r, j] * row_scale[r] + sum_{c < K} h[r, c] * W[ids[j], c]
+// with bf16 W (16-byte aligned rows), fp32 h, fp32 accumulation; codes null:
+// the local part alone.
+struct ZSource {
+  const float* Z = nullptr;
+  const float* h = nullptr;
+  int64_t ld_h = 0;
+  int K = 0;
+  const void* W = nullptr;
+  int64_t ld_w = 0;
+  const int32_t* ids = nullptr;
+  const int8_t* codes = nullptr;
+  const float* row_scale = nullptr;
+};
 // One inverse-CDF draw per row after an endpoint launch_tc: from the segment
 // statistics its epilogue left in `scratch` (plan.epi_stats), else from a
-// statistics pass over Z into the same area; `cstats` receives the chunk
-// statistics on the way (at most rows * (n / 1024 + 2)).
-cudaError_t launch_sample_from_stats(const float* Z, int rows, int n,
+// statistics pass over the stored z into the same area (a z that is not
+// stored needs plan.epi_stats); `cstats` receives the chunk statistics on
+// the way (at most rows * (n / 1024 + 2)).
+cudaError_t launch_sample_from_stats(const ZSource& zs, int rows, int n,
                                      const TcPlan& plan, const void* scratch,
                                      float2* cstats, const int32_t* ids,
                                      float inv_tau, uint64_t seed, uint64_t offset,
@@ -183,16 +202,28 @@ cudaError_t launch_gumbel(const float* Z, int rows, int n, const int32_t* ids, f
 // One inverse-CDF draw per row from segment statistics alone (nseg per row):
 // a block per row makes the chunk statistics in shared memory first.
 // cudaErrorNotSupported (nothing launched) past 4096 chunks per row.
-cudaError_t launch_sample_rows(const float* Z, int rows, int n, const float2* stats,
+cudaError_t launch_sample_rows(const ZSource& zs, int rows, int n, const float2* stats,
                                int nseg, const int32_t* ids, float inv_tau, uint64_t seed,
                                uint64_t offset, int32_t* tokens, cudaStream_t st);
 // One inverse-CDF draw per row from segment and chunk statistics with nseg
-// segments per row (nseg * 32 >= n; segments past n hold zero weight).
-cudaError_t launch_sample_segments(const float* Z, int rows, int n,
+// segments per row (nseg * 32 >= n; segments past n hold zero weight);
+// greedy: the first id of the row maximum (segment maxima, then the ids of
+// the segment that holds it).
+cudaError_t launch_sample_segments(const ZSource& zs, int rows, int n,
                                    const float2* stats, int nseg,
                                    const float2* cstats, const int32_t* ids,
                                    float inv_tau, uint64_t seed, uint64_t offset,
                                    int32_t* tokens, cudaStream_t st, int greedy = 0);
+inline cudaError_t launch_sample_segments(const float* Z, int rows, int n,
+                                          const float2* stats, int nseg,
+                                          const float2* cstats, const int32_t* ids,
+                                          float inv_tau, uint64_t seed, uint64_t offset,
+                                          int32_t* tokens, cudaStream_t st, int greedy = 0) {
+  ZSource zs;
+  zs.Z = Z;
+  return launch_sample_segments(zs, rows, n, stats, nseg, cstats, ids, inv_tau, seed, offset,
+                                tokens, st, greedy);
+}
 int sample_max_n();
 int verify_max_k();
 

@@ -33,6 +33,7 @@ SPH_OPT_SAMPLER = 8
 SPH_OPT_CHECK_IDS = 9
 SPH_OPT_SPLIT_QUANTIZE = 10
 SPH_OPT_TC_PAIR = 11
+SPH_OPT_ENDPOINT_Z = 12
 SPH_SAMPLER_CDF, SPH_SAMPLER_GUMBEL = 0, 1
 
 _c_void_p = ctypes.c_void_p

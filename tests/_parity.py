@@ -77,14 +77,31 @@ def check_cloud(ctx, w, act_mode="fp32", rows=None):
     return codes, scale, part
 
 
-def check_endpoint(ctx, w, codes, scale, rows=None):
+def fuse_sample_unstored(ctx, *a, **kw):
+    """sph_fuse_sample without a z output and with z never stored
+    (SPH_OPT_ENDPOINT_Z = 2: the draw recomputes the z it visits)."""
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, 2)
+    try:
+        return ctx.fuse_sample(*a, **kw)
+    finally:
+        ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, 0)
+
+
+def check_endpoint(ctx, w, codes, scale, rows=None, unstored=True):
     """GPU fuse+sample on a given payload (a host-side input shared with the
-    oracle); compare fused logits and tokens (margin rule)."""
+    oracle); compare fused logits and tokens (margin rule).  unstored: also
+    draw without storing z (the tokens under the same rule)."""
     dev = w.h.device
     z = torch.empty(w.rows, w.n_keep, device=dev)
     tok = ctx.fuse_sample(codes.to(dev), scale.to(dev), w.h_local, w.W_l,
                           keep_ids=w.keep_ids, temperature=w.tau, seed=w.seed,
                           offset=w.offset, fused_logits_out=z)
+    toks = [tok]
+    if unstored:
+        toks.append(fuse_sample_unstored(ctx, codes.to(dev), scale.to(dev), w.h_local, w.W_l,
+                                         keep_ids=w.keep_ids, temperature=w.tau,
+                                         seed=w.seed, offset=w.offset))
     ctx.sync()
     c = np_(codes)
     s = np_(scale)
@@ -105,10 +122,11 @@ def check_endpoint(ctx, w, codes, scale, rows=None):
         ok = margin >= MARGIN
     vocab = np.arange(w.V) if ids is None else ids
     want = vocab[j]
-    got = np_(tok)[sel]
-    bad = (got != want) & ok
-    assert not bad.any(), f"tokens differ at rows {sel[bad]}: {got[bad]} vs {want[bad]}"
-    assert np.isin(np_(tok), vocab).all(), "a masked id was sampled"
+    for t, what in zip(toks, ("z stored", "z recomputed")):
+        got = np_(t)[sel]
+        bad = (got != want) & ok
+        assert not bad.any(), f"tokens ({what}) differ at rows {sel[bad]}: {got[bad]} vs {want[bad]}"
+        assert np.isin(np_(t), vocab).all(), f"a masked id was sampled ({what})"
     return tok, z
 
 

@@ -761,7 +761,9 @@ def test_tensor_core_pairs(ctx, name, kw, schedule, act):
                      act_mode=sph.SPH_ACT_BF16 if act == "bf16" else sph.SPH_ACT_FP32)
         assert p["pair"] == 1 and p["grid"] % 2 == 0 and p["block_rows"] % 32 == 0
         check_cloud(ctx, w, act_mode=act)
-        # the endpoint ignores the option (its plans never pair)
+        # the endpoint on pairs too (z stored and not)
+        pe = ctx.plan(1, w.rows, w.n_keep, w.d_l, gather=w.keep_ids is not None)
+        assert pe["pair"] == 1 and pe["grid"] % 2 == 0
         ref = oracle_cloud(w)
         check_endpoint(ctx, w, torch.from_numpy(ref["codes"]), torch.from_numpy(ref["row_scale"]))
     finally:
@@ -822,13 +824,14 @@ def test_fp8_tensor_core_pairs(ctx, rows, keep, schedule, act):
         ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
 
 
-@pytest.mark.parametrize("n_keep", [2004, 3000, 3002])
+@pytest.mark.parametrize("n_keep", [2004, 3000, 3002, 3001])
 @pytest.mark.parametrize("payload", [True, False])
 def test_endpoint_transposed_epilogue(ctx, n_keep, payload):
     # row blocks of >= 128 rows over a short hidden dimension finish the
-    # endpoint through shared memory when rows are 4-element aligned (2004:
+    # endpoint through shared memory when rows are 2-element aligned (2004:
     # 8-byte code loads on every other row, a ragged last window; 3000: all
-    # aligned; 3002: not aligned, the per-lane path)
+    # 16-byte aligned; 3002: rows alternately 8- and 16-byte aligned, 2-byte
+    # code loads; 3001: odd, the per-lane path)
     w = small(V=n_keep + 1500, d=1088, d_l=64, rows=160, n_keep=n_keep, seed=909)
     if payload:
         ref = oracle_cloud(w)
@@ -842,3 +845,78 @@ def test_endpoint_transposed_epilogue(ctx, n_keep, payload):
         zref = oracle.local_partial(np_(w.h), bits(W_full), np_(w.keep_ids))
         assert_close(np_(z), zref, "unsplit fused logits")
         assert np.isin(np_(tok), np_(w.keep_ids)).all()
+
+
+# ---------------------------------------------------------------------------
+# the endpoint without a stored z: the contraction's epilogue keeps the
+# 32-id segment statistics and the draw recomputes z for the segment it
+# lands in (SPH_OPT_ENDPOINT_Z = 2)
+# ---------------------------------------------------------------------------
+
+UNSTORED = [
+    # name, workload, extra elements per W_l row (a padded row stride)
+    ("aligned", dict(V=6000, d=640, d_l=128, rows=40, n_keep=3000), 0),
+    ("even", dict(V=6000, d=640, d_l=128, rows=40, n_keep=3002), 0),
+    ("odd", dict(V=6000, d=640, d_l=128, rows=40, n_keep=3001), 0),
+    ("short", dict(V=500, d=136, d_l=16, rows=9, n_keep=7, run_lo=1, run_hi=3), 0),
+    ("k-tail", dict(V=3000, d=302, d_l=44, rows=20, n_keep=1111), 4),
+    ("row-blocks", dict(V=30000, d=640, d_l=64, rows=300, n_keep=20000), 0),
+    ("full-vocab", dict(V=3000, d=1280, d_l=264, rows=16, n_keep=3000), 0),
+]
+
+
+@pytest.mark.parametrize("tau", [0.8, 0.0])
+@pytest.mark.parametrize("payload", [True, False])
+@pytest.mark.parametrize("name,kw,pad", UNSTORED, ids=[c[0] for c in UNSTORED])
+def test_endpoint_unstored_z(ctx, name, kw, pad, payload, tau):
+    # tokens of the unstored path and of the stored one against the oracle
+    # (margin rule), on rows whose hidden states are 8- or 16-byte aligned
+    # ("k-tail": d = 302; a hidden dimension of 44 = 5 x 8 + 4 over a padded
+    # weight row stride)
+    from paper_2607_13093_gb300 import sph
+    from _parity import fuse_sample_unstored
+    w = small(seed=1301, tau=tau, **kw)
+    W_l = w.W_l
+    if pad:
+        buf = torch.zeros(w.V, w.d_l + pad, dtype=torch.bfloat16, device=DEV)
+        buf[:, :w.d_l] = w.W_l
+        W_l = buf[:, :w.d_l]
+    pc, ps = wl.make_payload(w.rows, w.n_keep, seed=21, device=DEV) if payload else (None, None)
+    ids = np_(w.keep_ids)
+    vocab = np.arange(w.V) if ids is None else ids
+    zref = oracle.fuse(np_(pc), np_(ps), oracle.local_partial(np_(w.h_local), bits(w.W_l), vocab))
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    try:
+        for off in (0, 5):
+            z = torch.empty(w.rows, w.n_keep, device=DEV)
+            t1 = ctx.fuse_sample(pc, ps, w.h_local, W_l, keep_ids=w.keep_ids, temperature=tau,
+                                 seed=w.seed, offset=off, fused_logits_out=z)
+            t2 = fuse_sample_unstored(ctx, pc, ps, w.h_local, W_l, keep_ids=w.keep_ids,
+                                      temperature=tau, seed=w.seed, offset=off)
+            ctx.sync()
+            assert_close(np_(z), zref, "fused logits")
+            if tau == 0:
+                j, gap = oracle.greedy_rows(zref)
+                ok = gap >= GREEDY_GAP
+            else:
+                u = oracle.philox_uniform(w.seed, np.arange(w.rows), 0, off)
+                j, margin = oracle.sample_rows(zref, tau, u)
+                ok = margin >= MARGIN
+            assert ok.mean() > 0.5
+            for t, what in ((t1, "stored"), (t2, "unstored")):
+                got = np_(t)
+                bad = (got != vocab[j]) & ok
+                assert not bad.any(), f"{what}: rows {np.nonzero(bad)[0]}"
+                assert np.isin(got, vocab).all()
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+
+
+def test_endpoint_z_option_values(ctx):
+    from paper_2607_13093_gb300 import sph
+    for v in (0, 1, 2):
+        ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, v)
+    for v in (-1, 3):
+        with pytest.raises(sph.SphError):
+            ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, v)
+    ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, 0)

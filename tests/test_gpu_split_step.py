@@ -39,13 +39,20 @@ def small(**kw):
     return wl.make_workload(device=DEV, **kw)
 
 
-def run_gpu(ctx, w, chunk, act="fp32"):
+def run_gpu(ctx, w, chunk, act="fp32", store_z=True):
+    """The split step; store_z False: no z output and z never stored
+    (SPH_OPT_ENDPOINT_Z = 2), z returned as None."""
     from paper_2607_13093_gb300 import sph
-    z = torch.empty(w.rows, w.n_keep, device=DEV)
-    codes, scales, tok, pb = ctx.split_step(
-        w.h, w.d_l, w.W_h, w.W_l, keep_ids=w.keep_ids, clip=w.clip, w_row_scale=w.w_scale,
-        bias=w.bias, act_mode=sph.SPH_ACT_BF16 if act == "bf16" else sph.SPH_ACT_FP32,
-        temperature=w.tau, seed=w.seed, offset=w.offset, chunk=chunk, fused_logits_out=z)
+    z = torch.empty(w.rows, w.n_keep, device=DEV) if store_z else None
+    ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, 0 if store_z else 2)
+    try:
+        codes, scales, tok, pb = ctx.split_step(
+            w.h, w.d_l, w.W_h, w.W_l, keep_ids=w.keep_ids, clip=w.clip,
+            w_row_scale=w.w_scale, bias=w.bias,
+            act_mode=sph.SPH_ACT_BF16 if act == "bf16" else sph.SPH_ACT_FP32,
+            temperature=w.tau, seed=w.seed, offset=w.offset, chunk=chunk, fused_logits_out=z)
+    finally:
+        ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, 0)
     ctx.sync()
     R, n = w.rows, w.n_keep
     b = oracle.chunk_bounds(n, chunk)
@@ -54,7 +61,7 @@ def run_gpu(ctx, w, chunk, act="fp32"):
     for q, (j0, j1) in enumerate(b):         # chunk-major -> [R, n]
         c[:, j0:j1] = flat[j0 * R: j0 * R + R * (j1 - j0)].reshape(R, j1 - j0)
     s = np_(scales)[: len(b) * R].reshape(len(b), R)
-    return c, s, np_(tok), np_(z), pb
+    return c, s, np_(tok), (np_(z) if store_z else None), pb
 
 
 def oracle_split(w, chunk, act="fp32", rows=None):
@@ -120,6 +127,14 @@ def check_split(ctx, w, chunk, act="fp32", rows=None):
     assert not bad.any(), f"tokens differ at rows {sel[bad]}"
     assert np.isin(tok, ref["vocab"]).all(), "a masked id was sampled"
     assert check.any()
+    if chunk == 0:
+        # the same step without storing z: the same payload bit for bit, and
+        # tokens under the same rule
+        c2, s2, tok2, _, pb2 = run_gpu(ctx, w, chunk, act, store_z=False)
+        assert pb2 == pb and np.array_equal(c2, c) and np.array_equal(s2, s)
+        bad = check & (tok2[sel] != ref["tokens"])
+        assert not bad.any(), f"tokens (z recomputed) differ at rows {sel[bad]}"
+        assert np.isin(tok2, ref["vocab"]).all(), "a masked id was sampled (z recomputed)"
     return c, s, tok, z
 
 
@@ -137,6 +152,26 @@ ONE_CHUNK = [
 @pytest.mark.parametrize("name,kw", ONE_CHUNK, ids=[c[0] for c in ONE_CHUNK])
 def test_split_step_one_chunk(path_ctx, name, kw):
     check_split(path_ctx, small(**kw), 0)
+
+
+@pytest.mark.parametrize("name,kw", [c for c in ONE_CHUNK if c[0] != "fp8"],
+                         ids=[c[0] for c in ONE_CHUNK if c[0] != "fp8"])
+@pytest.mark.parametrize("quantize", [1, 2])
+def test_split_step_pairs(ctx, name, kw, quantize):
+    # both contractions on CTA pairs, the endpoint quantizing in its epilogue
+    # (1) or after a separate pass (2)
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    ctx.set_option(sph.SPH_OPT_TC_PAIR, 1)
+    ctx.set_option(sph.SPH_OPT_SPLIT_QUANTIZE, quantize)
+    try:
+        w = small(**kw)
+        assert ctx.plan(1, w.rows, w.n_keep, w.d_l, gather=w.keep_ids is not None)["pair"] == 1
+        check_split(ctx, w, 0)
+    finally:
+        ctx.set_option(sph.SPH_OPT_SPLIT_QUANTIZE, 0)
+        ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
 
 
 @pytest.mark.parametrize("rows", [2, 40])
