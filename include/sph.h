@@ -161,19 +161,31 @@ typedef enum sph_option {
                                epilogue, 2 always a separate quantize pass.
                                The payload, z and tokens are bit-identical
                                either way.                                  */
+  SPH_OPT_ENDPOINT_ROWS_M = 13, /* the endpoint contraction on CTA pairs
+                               with the hidden-state rows as the MMA's M
+                               dimension (256 rows over the pair, the tile's
+                               256 ids as N), so that each epilogue thread
+                               finishes one row's consecutive ids and makes
+                               their softmax statistics itself: 0 automatic
+                               (default: where the call pairs and 256-row
+                               blocks pad at most 1/8 of the rows), 1 always
+                               where the call pairs, 2 never.  Whole tiles
+                               only (not with SPH_OPT_TC_SCHEDULE = 2).     */
   SPH_OPT_ENDPOINT_Z = 12,  /* where sph_fuse_sample and sph_split_step are
                                not asked for z (fused_logits_out NULL) and
                                run on tensor cores with the inverse-CDF or
-                               greedy draw: 0 automatic (default: stored),
-                               1 store z in the scratch arena, 2 never store
-                               it.  Unstored, the endpoint contraction's
-                               epilogue keeps the softmax statistics of every
-                               32-id segment and the draw recomputes z for
-                               the 32 ids of the segment it lands in (one
-                               fp32 dot product of d_l per id, CUDA cores):
-                               tokens can differ from the stored path's only
-                               where a draw lies within fp32 rounding of a
-                               CDF step (or greedy ties within it).          */
+                               greedy draw: 0 automatic (default: not stored
+                               where the endpoint runs with rows as M, see
+                               SPH_OPT_ENDPOINT_ROWS_M; else stored), 1 store
+                               z in the scratch arena, 2 never store it.
+                               Unstored, the endpoint contraction's epilogue
+                               keeps the softmax statistics of every 32-id
+                               segment and the draw recomputes z for the 32
+                               ids of the segment it lands in (one fp32 dot
+                               product of d_l per id, CUDA cores): tokens can
+                               differ from the stored path's only where a
+                               draw lies within fp32 rounding of a CDF step
+                               (or greedy ties within it).                 */
   SPH_OPT_SAMPLER = 8       /* the draw of sph_fuse_sample at temperature > 0:
                                0 inverse CDF (default), 1 Gumbel-max: the
                                first index j of the largest
@@ -263,6 +275,12 @@ typedef struct sph_plan {
   int32_t gemv_rows;        /* GEMV: rows per launch (1, 2, 4 or 8)        */
   int32_t pair;             /* 1: CTA pairs (SPH_OPT_TC_PAIR); grid counts
                                CTAs, tile_ids is per CTA (a tile is 256)   */
+  int32_t rows_m;           /* endpoint: 1 = hidden-state rows as the MMA's M
+                               (SPH_OPT_ENDPOINT_ROWS_M; CTA pairs, 256-row
+                               blocks, 256-id tiles)                       */
+  int32_t epilogue_stats;   /* endpoint: 1 = the softmax statistics of each
+                               32-id segment come from the contraction's
+                               epilogue, 0 = from a pass over z            */
 } sph_plan;
 sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep,
                           int64_t K, sph_dtype w_dtype, sph_act_mode act_mode,

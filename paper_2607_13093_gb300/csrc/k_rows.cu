@@ -182,11 +182,14 @@ __device__ __forceinline__ int scan_pick(float w, float target, float& before, i
 // a contiguous run of chunks; the warp then scans the run that holds the
 // target 32 chunks at a time, then that chunk's segments, then the
 // segment's ids.  Returns the total weight (the draw is void if it is 0);
-// all lanes receive the same j.
-template <class CW, class SW, class EW>
-__device__ __forceinline__ float warp_draw(int nchunk, int nseg, int n, const CW& cw,
-                                           const SW& sw, const EW& ew, float u, int lane,
-                                           int& j_out) {
+// all lanes receive the same j.  warp_draw_segment stops after the segment
+// (the target and the weight before the segment in target/before), for
+// callers that make the segment's id weights themselves.
+template <class CW, class SW>
+__device__ __forceinline__ float warp_draw_segment(int nchunk, int nseg, const CW& cw,
+                                                   const SW& sw, float u, int lane,
+                                                   int& seg_out, float& target_out,
+                                                   float& before_out) {
   const int per = (nchunk + 31) / 32;
   const int c0 = min(nchunk, lane * per), c1 = min(nchunk, c0 + per);
   float local = 0.f;
@@ -229,7 +232,18 @@ __device__ __forceinline__ float warp_draw(int nchunk, int nseg, int n, const CW
   if (chunk < 0) { chunk = last_chunk; before = before_last; }
   const int s = chunk * kSeg + lane;
   const int ls = scan_pick(s < nseg ? sw(s) : 0.f, target, before, lane);
-  const int seg = chunk * kSeg + ls;
+  seg_out = chunk * kSeg + ls;
+  target_out = target;
+  before_out = before;
+  return total;
+}
+template <class CW, class SW, class EW>
+__device__ __forceinline__ float warp_draw(int nchunk, int nseg, int n, const CW& cw,
+                                           const SW& sw, const EW& ew, float u, int lane,
+                                           int& j_out) {
+  int seg;
+  float target, before;
+  const float total = warp_draw_segment(nchunk, nseg, cw, sw, u, lane, seg, target, before);
   const int j = seg * kSeg + lane;
   const int lj = scan_pick(j < n ? ew(j) : 0.f, target, before, lane);
   j_out = min(seg * kSeg + lj, n - 1);
@@ -297,13 +311,28 @@ struct ZRowRecomputed {
     const float z = (a[0] + a[1]) + (a[2] + a[3]);
     return c ? fmaf((float)__ldg(c + j), s, z) : z;
   }
+  // The same z by the whole warp (every lane gets it): lane l takes the
+  // 8-element pieces l, l + 32, ... of the row, then a warp sum.
+  __device__ float coop(int j, int lane) const {
+    const int id = ids ? __ldg(ids + j) : j;
+    const uint16_t* w = W + (int64_t)id * ld_w;
+    float a[4] = {0.f, 0.f, 0.f, 0.f};
+    const int K8 = K & ~7;
+    for (int k = 8 * lane; k < K8; k += 256) dot8(__ldg(reinterpret_cast<const uint4*>(w + k)), k, a);
+    for (int k = K8 + lane; k < K; k += 32)
+      a[0] = fmaf(__ldg(h + k), __uint_as_float((unsigned)w[k] << 16), a[0]);
+    const float z = warp_sum((a[0] + a[1]) + (a[2] + a[3]));
+    return c ? fmaf((float)__ldg(c + j), s, z) : z;
+  }
 };
 struct ZRowsStored {
+  static constexpr bool kRecompute = false;
   const float* Z;
   int n;
   __device__ ZRowStored row(int64_t r) const { return ZRowStored{Z + r * n}; }
 };
 struct ZRowsRecomputed {
+  static constexpr bool kRecompute = true;
   ZSource zs;
   int n;
   __device__ ZRowRecomputed row(int64_t r) const {
@@ -416,15 +445,53 @@ sample_rows_kernel(const ZRows zr, int n, const float2* __restrict__ stats,
     }
   }
   __syncthreads();
-  if (warp != 0) return;
-  const float M = stats_max(s_cst, nchunk, lane);
-  const StatsWeight cw{s_cst, M, inv_tau};
-  const StatsWeight sw{srow, M, inv_tau};
-  const ExpWeightOf<decltype(zr.row(0))> ew{zr.row(r), M, inv_tau};
-  const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
-  int j;
-  warp_draw(nchunk, nseg, n, cw, sw, ew, u, lane, j);
-  if (lane == 0) tokens[r] = ids ? ids[j] : j;
+  if constexpr (ZRows::kRecompute) {
+    // warp 0 finds the segment; all warps recompute its 32 logits (a warp
+    // per id, lanes across the hidden dimension); warp 0 draws the id
+    __shared__ int s_seg;
+    __shared__ float s_par[3];
+    __shared__ float s_z[kSeg];
+    if (warp == 0) {
+      const float M = stats_max(s_cst, nchunk, lane);
+      const StatsWeight cw{s_cst, M, inv_tau};
+      const StatsWeight sw{srow, M, inv_tau};
+      const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
+      int seg;
+      float target, before;
+      warp_draw_segment(nchunk, nseg, cw, sw, u, lane, seg, target, before);
+      if (lane == 0) {
+        s_seg = seg;
+        s_par[0] = M; s_par[1] = target; s_par[2] = before;
+      }
+    }
+    __syncthreads();
+    const int seg = s_seg;
+    const auto zrow = zr.row(r);
+    for (int i = warp; i < kSeg; i += nw) {
+      const int j = seg * kSeg + i;
+      const float z = j < n ? zrow.coop(j, lane) : -INFINITY;
+      if (lane == 0) s_z[i] = z;
+    }
+    __syncthreads();
+    if (warp != 0) return;
+    const float M = s_par[0];
+    float before = s_par[2];
+    const int j = seg * kSeg + lane;
+    const float wj = j < n ? expf((s_z[lane] - M) * inv_tau) : 0.f;
+    const int lj = scan_pick(wj, s_par[1], before, lane);
+    const int jj = min(seg * kSeg + lj, n - 1);
+    if (lane == 0) tokens[r] = ids ? ids[jj] : jj;
+  } else {
+    if (warp != 0) return;
+    const float M = stats_max(s_cst, nchunk, lane);
+    const StatsWeight cw{s_cst, M, inv_tau};
+    const StatsWeight sw{srow, M, inv_tau};
+    const ExpWeightOf<decltype(zr.row(0))> ew{zr.row(r), M, inv_tau};
+    const float u = philox_uniform(seed, (uint32_t)r, 0u, offset);
+    int j;
+    warp_draw(nchunk, nseg, n, cw, sw, ew, u, lane, j);
+    if (lane == 0) tokens[r] = ids ? ids[j] : j;
+  }
 }
 
 // ---------------------------------------------------------------------------

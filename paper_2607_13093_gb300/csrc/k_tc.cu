@@ -77,6 +77,14 @@ constexpr int kTRow = 36;
 // Kernel instantiations of EPI_ENDPOINT that finish through the per-warp
 // shared-memory transpose (finish_chunk_t) rather than per lane.
 constexpr int EPI_ENDPOINT_T = 3;
+// Rows-as-M instantiations of EPI_ENDPOINT and EPI_FUSED (CTA pairs only):
+// the MMA's M dimension is the hidden-state rows (A = the h planes, 128 rows
+// per CTA) and N the tile's 256 ids (B = the gathered weight rows, 128 per
+// CTA), so each epilogue lane holds one row and 32 consecutive ids per
+// accumulator load.
+constexpr int EPI_ENDPOINT_RM = 4;
+constexpr int EPI_FUSED_RM = 5;
+constexpr float kLog2eF = 1.4426950408889634f;
 constexpr int kTransposeBytes = 8 /* epilogue warps */ * 8 * kTRow * 4;
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
@@ -384,6 +392,140 @@ __device__ __forceinline__ void finish_chunk_t(const TcParams& p, const float (&
   }
 }
 
+// ---- rows-as-M endpoint epilogue -----------------------------------------
+// This lane's row r and one 32-id segment j0 .. j0 + 31 of the tile.  The
+// codes of the segment (32 bytes of row r), loaded before the tile's
+// accumulator is ready.
+struct RPay {
+  uint4 c[2];
+};
+__device__ __forceinline__ void load_rpay(const TcParams& p, int r, int j0, RPay& q) {
+  q.c[0] = q.c[1] = make_uint4(0u, 0u, 0u, 0u);
+  if (!p.codes || r >= p.R || j0 >= p.n) return;
+  const int8_t* cp = p.codes + (int64_t)r * p.n + j0;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(cp);
+  if (j0 + 32 <= p.n && (a & 15) == 0) {
+    q.c[0] = __ldg(reinterpret_cast<const uint4*>(cp));
+    q.c[1] = __ldg(reinterpret_cast<const uint4*>(cp) + 1);
+    return;
+  }
+  unsigned w[8];
+  if (j0 + 32 <= p.n && (a & 3) == 0) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) w[e] = __ldg(reinterpret_cast<const unsigned*>(cp) + e);
+  } else {
+    const int cnt = min(32, p.n - j0);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) w[e] = 0u;
+#pragma unroll
+    for (int e = 0; e < 32; ++e)
+      if (e < cnt) w[e >> 2] |= ((unsigned)(uint8_t)__ldg(cp + e)) << (8 * (e & 3));
+  }
+  q.c[0] = make_uint4(w[0], w[1], w[2], w[3]);
+  q.c[1] = make_uint4(w[4], w[5], w[6], w[7]);
+}
+__device__ __forceinline__ unsigned rpay_word(const RPay& q, int w) {
+  const uint4 u = q.c[w >> 2];
+  return (w & 3) == 0 ? u.x : (w & 3) == 1 ? u.y : (w & 3) == 2 ? u.z : u.w;
+}
+// Finish the segment (Eq. 13): z = v + code * s, stored where asked; with the
+// fused endpoint the codes are first quantized from the cloud's clipped
+// partials (Eq. 18) and written out; the segment's softmax statistics
+// (max z, sum of exp((z - max) / tau) over its ids below n) where asked.
+template <int EPI>
+__device__ __forceinline__ void finish_rm(const TcParams& p, float (&v)[32], int r, int j0,
+                                          const RPay& q, const RowQuant& rq) {
+  const bool rv = r < p.R;
+  const int cnt = rv ? max(0, min(32, p.n - j0)) : 0;   // this row's ids in the segment
+  const bool full = cnt == 32;
+  if constexpr (EPI == EPI_FUSED_RM) {
+    if (cnt > 0) {
+      const float* yp = p.yc + (int64_t)r * p.n + j0;
+      float y[32];
+      if (full && (reinterpret_cast<uintptr_t>(yp) & 15) == 0) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float4 t = __ldcg(reinterpret_cast<const float4*>(yp) + e);
+          y[4 * e] = t.x; y[4 * e + 1] = t.y; y[4 * e + 2] = t.z; y[4 * e + 3] = t.w;
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 32; ++e) y[e] = e < cnt ? __ldcg(yp + e) : 0.f;
+      }
+      unsigned w[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) w[e] = 0u;
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        const int code = quantize_one(y[e], rq.k, rq.inv);
+        w[e >> 2] |= ((unsigned)code & 0xFFu) << (8 * (e & 3));
+        v[e] = fmaf((float)code, rq.s, v[e]);
+      }
+      int8_t* cp = p.codes_out + (int64_t)r * p.n + j0;
+      if (full && (reinterpret_cast<uintptr_t>(cp) & 15) == 0) {
+        reinterpret_cast<uint4*>(cp)[0] = make_uint4(w[0], w[1], w[2], w[3]);
+        reinterpret_cast<uint4*>(cp)[1] = make_uint4(w[4], w[5], w[6], w[7]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          if (e < cnt) cp[e] = (int8_t)((w[e >> 2] >> (8 * (e & 3))) & 0xFFu);
+      }
+    }
+  } else {
+    if (p.codes) {
+#pragma unroll
+      for (int w = 0; w < 8; ++w) {
+        const unsigned wx = rpay_word(q, w) ^ 0x80808080u;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) v[4 * w + b] = fmaf(code_f32(wx, b), rq.s, v[4 * w + b]);
+      }
+    }
+  }
+  if (p.Y && cnt > 0) {
+    float* zp = p.Y + (int64_t)r * p.ldy + j0;
+    if (full && (reinterpret_cast<uintptr_t>(zp) & 15) == 0) {
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        reinterpret_cast<float4*>(zp)[e] =
+            make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 32; ++e)
+        if (e < cnt) zp[e] = v[e];
+    }
+  }
+  if (p.seg_stats && rv) {
+    // balanced trees (short dependency chains); ids past n count as -inf,
+    // whose exponential is 0
+    if (!full) {
+#pragma unroll
+      for (int e = 0; e < 32; ++e)
+        if (e >= cnt) v[e] = -INFINITY;
+    }
+    float t[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) t[i] = fmaxf(v[2 * i], v[2 * i + 1]);
+#pragma unroll
+    for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+      for (int i = 0; i < w; ++i) t[i] = fmaxf(t[2 * i], t[2 * i + 1]);
+    const float m = t[0];
+    float sum = 0.f;
+    if (m > -INFINITY) {
+      const float l2t = p.inv_tau * kLog2eF;   // exp(d / tau) = 2^(d log2(e) / tau)
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        t[i] = exp2f((v[2 * i] - m) * l2t) + exp2f((v[2 * i + 1] - m) * l2t);
+#pragma unroll
+      for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) t[i] = t[2 * i] + t[2 * i + 1];
+      sum = t[0];
+    }
+    p.seg_stats[(int64_t)r * p.nseg + (j0 >> 5)] = make_float2(m, sum);
+  }
+}
+
 // TM = vocabulary rows per tile: 128, or 256 as two M = 128 MMAs that share
 // each B stage (half the B bytes per A byte; TMEM holds 2 x 2 x BN columns).
 // PAIR: a cluster of two CTAs computes each 256-id tile as one M = 256
@@ -400,6 +542,10 @@ tc_kernel(const __grid_constant__ WMaps wm,
           const __grid_constant__ CUtensorMap tmH, const TcParams p) {
   static_assert(TM == 128 || TM == 256, "tile height");
   static_assert(!PAIR || TM == 128, "a pair tile is two CTAs of 128 ids");
+  // rows as M: the MMA's A operand is the h planes and B the weights (the
+  // same shared-memory stages); pairs of CTAs with 256-row blocks only
+  constexpr bool rm = EPI == EPI_ENDPOINT_RM || EPI == EPI_FUSED_RM;
+  static_assert(!rm || (PAIR && !FP8), "rows as M: bf16 CTA pairs");
   constexpr int kAtomE = FP8 ? kAtomE8 : kAtomK;   // elements per 128-byte atom
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
@@ -709,7 +855,8 @@ tc_kernel(const __grid_constant__ WMaps wm,
       int si = 0, tile, kb0, kb1;
       constexpr int kMmaM = PAIR ? 2 * kTileM : kTileM;
       const uint32_t idesc =
-          FP8 ? ptx::idesc_e4m3_f32(kMmaM, BN) : ptx::idesc_bf16_f32(kMmaM, BN);
+          FP8 ? ptx::idesc_e4m3_f32(kMmaM, BN)
+              : ptx::idesc_bf16_f32(kMmaM, rm ? kTileStride : BN);   // (rows as M: N = ids)
       auto wait_x = [&](uint64_t* bar, uint32_t parity) {
         return ptx::mbar_wait(bar, parity, limit);
       };
@@ -742,9 +889,10 @@ tc_kernel(const __grid_constant__ WMaps wm,
                 for (int hf = 0; hf < kHalves; ++hf)
                 {
                   // 32 bytes of K per MMA: 16 bf16 or 32 e4m3 elements
-                  const uint64_t ad =
+                  const uint64_t wd =
                       ptx::sdesc_k128(a0 + at * atom_bytes + hf * kAtomBytes + kk * 32);
-                  const uint64_t bd = ptx::sdesc_k128(b0 + (h * NA + at) * BNc * 128 + kk * 32);
+                  const uint64_t hd = ptx::sdesc_k128(b0 + (h * NA + at) * BNc * 128 + kk * 32);
+                  const uint64_t ad = rm ? hd : wd, bd = rm ? wd : hd;
                   const uint32_t accum = (kb != kb0 || at != 0 || h != 0 || kk != 0) ? 1u : 0u;
                   if constexpr (PAIR && FP8)
                     ptx::umma_f8_pair(d, ad, bd, idesc, accum);
@@ -814,7 +962,36 @@ tc_kernel(const __grid_constant__ WMaps wm,
                                            kMaxBoxes * sizeof(int2)) +
                   (warp - 2) * 8 * kTRow;
       Payload pay;
-      if constexpr (EPI != EPI_CLOUD) {
+      // rows as M: this lane's row, its constants, and the codes of its
+      // four 32-id segments of the tile (segments grp, grp + 2, ...), all
+      // loaded while the tile's MMAs run
+      constexpr int kRmSeg = 8 / kEpiGroups;
+      const int r_rm = rb * 256 + half * 128 + quad * 32 + lane;
+      RowQuant rq_rm{0.f, 1.f, 0.f};
+      RPay rp[kRmSeg];
+      if constexpr (rm) {
+        if (r_rm < p.R) {
+          if constexpr (EPI == EPI_FUSED_RM) {
+            rq_rm = row_quant(__ldcg(p.rowmax_in + r_rm));
+            if (t == 0 && grp == 0) p.scale_out[r_rm] = rq_rm.s;
+            // (the clipped partials are read when finishing: warm L2 now)
+#pragma unroll
+            for (int a = 0; a < kRmSeg; ++a) {
+              const int j0 = t * 256 + (grp + a * kEpiGroups) * 32;
+              if (j0 < p.n)
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(p.yc + (int64_t)r_rm * p.n + j0));
+            }
+          } else if (p.codes) {
+            rq_rm.s = __ldg(p.row_scale + r_rm);
+          }
+        }
+        if constexpr (EPI == EPI_ENDPOINT_RM) {
+#pragma unroll
+          for (int a = 0; a < kRmSeg; ++a)
+            load_rpay(p, r_rm, t * 256 + (grp + a * kEpiGroups) * 32, rp[a]);
+        }
+      }
+      if constexpr (EPI != EPI_CLOUD && !rm) {
         // the payload does not depend on the accumulator: start on it
         // while the tile's MMAs run
 #pragma unroll
@@ -842,7 +1019,9 @@ tc_kernel(const __grid_constant__ WMaps wm,
       }
       // (split tiles load the transposed payload right before finishing)
       auto finish = [&](const float (&vv)[16], int hf, int ch) {
-        if constexpr (epi_t) {
+        if constexpr (rm) {
+          // (rows as M takes whole tiles only)
+        } else if constexpr (epi_t) {
           if (!whole) load_tpay(p, rb * BN + ch * 16, J(hf) - lane, lane, tpay);
           finish_chunk_t(p, vv, rb * BN + ch * 16, J(hf) - lane, lane, tb, tpay);
         } else {
@@ -929,7 +1108,19 @@ tc_kernel(const __grid_constant__ WMaps wm,
       // a CTA's split tiles can only be its first and its last segment:
       // slot 2c holds the first, 2c+1 the last ([BN][TM] each)
       float* Pt = p.P + (size_t)pslot(2 * unit + (si == 0 ? 0 : 1)) * BN * TM;
-      for (int hc = grp; hc < nhc; hc += kEpiGroups) {
+      if constexpr (rm) {
+        // this lane's row: 32 consecutive columns (ids) per load
+        // (two segments per accumulator wait, finished side by side)
+#pragma unroll
+        for (int a = 0; a < kRmSeg; a += 2) {
+          const int s0 = grp + a * kEpiGroups, s1 = s0 + kEpiGroups;
+          float v0[32], v1[32];
+          ptx::tmem_ld32x2(taddr + (uint32_t)(s0 * 32), taddr + (uint32_t)(s1 * 32), v0, v1);
+          finish_rm<EPI>(p, v0, r_rm, t * 256 + s0 * 32, rp[a], rq_rm);
+          finish_rm<EPI>(p, v1, r_rm, t * 256 + s1 * 32, rp[a + 1], rq_rm);
+        }
+      }
+      for (int hc = grp; hc < (rm ? 0 : nhc); hc += kEpiGroups) {
         const int hf = hc / nch, ch = hc - hf * nch;
         const int i = hf * 128 + quad * 32 + lane;
         float v[16];
@@ -1332,12 +1523,24 @@ namespace {
 // 32, so that each CTA's half is whole 16-row groups), work split over the
 // pairs (a multiple of the row-block count, as below).
 TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pairs,
-                    int schedule, int max_stages, int block_k, int max_bn_opt, int endpoint) {
+                    int schedule, int max_stages, int block_k, int max_bn_opt, int endpoint,
+                    int rm_mode) {
   // (e4m3 weights: four or two h planes; 128-row blocks keep four stages)
   int cap = pl.fp8 ? 128 : 256;
   if (max_bn_opt >= 32 && max_bn_opt < cap) cap = max_bn_opt / 32 * 32;
   pl.RB = (rows + cap - 1) / cap;
   pl.BN = ((rows + pl.RB - 1) / pl.RB + 31) / 32 * 32;
+  // the endpoint with rows as M: 256-row blocks (M = 256 over the pair),
+  // whole tiles; automatic where the row blocks lose at most 1/8 to padding
+  // (measured on 1024 rows x 256000 ids x 512: ... )
+  const int rb256 = (rows + 255) / 256;
+  pl.rm = endpoint && !pl.fp8 && schedule != 2 && rm_mode != 2 &&
+          (rm_mode == 1 || (cap == 256 && 8 * (rb256 * 256 - rows) <= rb256 * 256));
+  if (pl.rm) {
+    pl.RB = rb256;
+    pl.BN = 256;
+    schedule = 1;
+  }
   pl.tm = 128;
   pl.single_acc = 0;
   pl.Rp = pl.RB * pl.BN;
@@ -1365,9 +1568,10 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
   units = pl.whole_tiles ? g_whole : (int)(pl.T < units ? pl.T : units);
   pl.G = 2 * units;
   // the endpoint's epilogue as on single CTAs (each CTA of a pair finishes
-  // its own 128 ids for all BN rows)
-  pl.epi_stats = endpoint == 2 || (endpoint && (pl.BN < 128 || 4 * pl.BN <= K));
-  pl.epi_t = endpoint == 2 || (endpoint && !pl.epi_stats);
+  // its own 128 ids for all BN rows); rows as M: the statistics of a
+  // lane's 32-id segment are its own, always made in the epilogue
+  pl.epi_stats = pl.rm || endpoint == 2 || (endpoint && (pl.BN < 128 || 4 * pl.BN <= K));
+  pl.epi_t = !pl.rm && (endpoint == 2 || (endpoint && !pl.epi_stats));
   pl.stages = (int)((kSmemBudget - 2048 - (pl.epi_t ? kTransposeBytes : 0)) / stage_of(pl.na));
   if (pl.stages > kMaxStages) pl.stages = kMaxStages;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
@@ -1388,7 +1592,7 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
 
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
                int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn_opt,
-               int tile_m, int pair_mode, int max_pairs) {
+               int tile_m, int pair_mode, int max_pairs, int rm_mode) {
   TcPlan pl{};
   // h planes: bf16 weights take one bf16 plane for bf16-rounded
   // activations (exact) and two (hi + lo) for fp32; e4m3 weights take two
@@ -1411,7 +1615,7 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   if (pair_mode > 0 && sm_count >= 2 && (tile_m == 0 || pair_mode == 2)) {
     pl.pair = 1;
     const TcPlan pp = tc_plan_pair(pl, rows, n, K, sm_count, max_pairs, schedule, max_stages,
-                                   block_k, max_bn_opt, endpoint);
+                                   block_k, max_bn_opt, endpoint, rm_mode);
     if (pair_mode == 2 || (!fp8 && (pp.BN >= 192 || (pl.hilo == 1 && pp.BN >= 128)))) return pp;
     pl.pair = 0;
   }
@@ -1589,6 +1793,7 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
   const bool fp8 = g.w_dtype == W_FP8;
   if (!pl.ok || (fp8 != (pl.fp8 != 0)) || (fp8 && g.epilogue != EPI_CLOUD) ||
       (pl.pair && (pl.G % 2 || pl.BN % 32)) ||
+      (pl.rm && (!pl.pair || pl.BN != 256 || !pl.whole_tiles || g.epilogue == EPI_CLOUD)) ||
       (g.epilogue != EPI_CLOUD && pl.hilo != 2) ||
       (g.epilogue == EPI_FUSED && (!g.yc || !g.rowmax_in || !g.codes_out || !g.scale_out)))
     return cudaErrorNotSupported;
@@ -1675,6 +1880,13 @@ cudaError_t launch_tc(const GatherGemm& g, const TcPlan& pl, void* scratch,
                              : launch_inst<4, true, EPI_CLOUD, true, 128, true>(mw, mh, prm, pl, st);
     return hilo2 ? launch_inst<2, false, EPI_CLOUD, true, 128, true>(mw, mh, prm, pl, st)
                  : launch_inst<4, false, EPI_CLOUD, true, 128, true>(mw, mh, prm, pl, st);
+  }
+  if (pl.rm) {
+    if (g.epilogue == EPI_FUSED)
+      return gather ? launch_inst<2, true, EPI_FUSED_RM, false, 128, true>(mw, mh, prm, pl, st)
+                    : launch_inst<2, false, EPI_FUSED_RM, false, 128, true>(mw, mh, prm, pl, st);
+    return gather ? launch_inst<2, true, EPI_ENDPOINT_RM, false, 128, true>(mw, mh, prm, pl, st)
+                  : launch_inst<2, false, EPI_ENDPOINT_RM, false, 128, true>(mw, mh, prm, pl, st);
   }
   if (pl.pair) {
     if (g.epilogue == EPI_FUSED)

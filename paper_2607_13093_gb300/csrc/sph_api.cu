@@ -41,6 +41,7 @@ struct sph_ctx {
   int split_quantize = 0;           // SPH_OPT_SPLIT_QUANTIZE
   int tc_pair = 0;                  // SPH_OPT_TC_PAIR: 0 automatic, 1 always, 2 never
   int endpoint_z = 0;               // SPH_OPT_ENDPOINT_Z: 0 automatic, 1 store, 2 recompute
+  int endpoint_rm = 0;              // SPH_OPT_ENDPOINT_ROWS_M: 0 automatic, 1 always, 2 never
   int pair_units = 0;               // CTA pairs that fit at once (0: pairs unavailable)
   // chunked split steps: the endpoint's own stream (created on first use
   // when the caller passes none) and the events that order the two streams
@@ -164,7 +165,8 @@ size_t tc_bytes(const sph_ctx* ctx, int64_t rows, int64_t n, int64_t K, int act_
         const size_t x = sph::tc_plan((int)rows, (int)n, (int)K, act_bf16, sm_count,
                                       endpoint, ctx->tc_schedule, ctx->tc_stages,
                                       ctx->tc_block_k, gather, w_dtype == sph::W_FP8,
-                                      ctx->tc_max_bn, tm, pm, ctx->pair_units)
+                                      ctx->tc_max_bn, tm, pm, ctx->pair_units,
+                                      ctx->endpoint_rm)
                              .scratch_bytes;
         if (x > b) b = x;
       }
@@ -342,11 +344,27 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
   // Gumbel-max draws need no softmax statistics: the epilogue skips them
   const bool gumbel = ctx->sampler == 1 && !greedy;
   gg.no_stats = gumbel;
-  // unstored z (SPH_OPT_ENDPOINT_Z = 2; not automatic: measured slower on
-  // 1024 x 256000 ids x d_l 512, 32 x 12000 x 256 and 1024 x 256000 x 5120,
-  // faster on 256 x 152064 x 1024)
+  // z unstored (SPH_OPT_ENDPOINT_Z): automatic where the endpoint runs with
+  // rows as M, whose epilogue makes each segment's statistics in its own
+  // lane (measured, steps of 1024 x 256000 ids x d_l 512: 3.18 vs 3.43 ms;
+  // 256 x 152064 x 1024: 0.87 vs 0.90 ms; 256 x 256000 x 512: 0.88 vs
+  // 1.00 ms), not with ids as M (32 x 12000 x 256: 55 vs 49 us)
   const bool tc = use_tc(ctx, rows, sph::W_BF16);
-  const bool z_free = tc && !gumbel && !z_out && ctx->endpoint_z == 2;
+  bool z_free = tc && !gumbel && !z_out && ctx->endpoint_z != 1;
+  auto plan_of = [&](bool zf) {
+    return sph::tc_plan(rows, n_keep, gg.K, 0, ctx->sm_count, zf ? 2 : 1, ctx->tc_schedule,
+                        ctx->tc_stages, ctx->tc_block_k, keep_ids != nullptr, 0,
+                        ctx->tc_max_bn, ctx->tc_tile_m, pair_mode(ctx), ctx->pair_units,
+                        ctx->endpoint_rm);
+  };
+  sph::TcPlan pl{};
+  if (tc) {
+    pl = plan_of(z_free);
+    if (z_free && ctx->endpoint_z == 0 && !pl.rm) {
+      z_free = false;
+      pl = plan_of(false);
+    }
+  }
   sph::ZSource zs;
   if (z_free) {
     gg.Y = nullptr;
@@ -367,12 +385,6 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
                          }), "sample launch");
   };
   if (tc) {
-    const sph::TcPlan pl = sph::tc_plan(rows, n_keep, gg.K, 0,
-                                        ctx->sm_count, z_free ? 2 : 1, ctx->tc_schedule,
-                                        ctx->tc_stages,
-                                        ctx->tc_block_k, keep_ids != nullptr, 0,
-                                        ctx->tc_max_bn, ctx->tc_tile_m, pair_mode(ctx),
-                                        ctx->pair_units);
     void* tcs = c.take(pl.scratch_bytes);
     if (!c.fits())
       return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
@@ -483,7 +495,8 @@ sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep, 
                                       call == 0 && act_mode == SPH_ACT_BF16, ctx->sm_count,
                                       call, ctx->tc_schedule, ctx->tc_stages, ctx->tc_block_k,
                                       gather != 0, wdt == sph::W_FP8, ctx->tc_max_bn,
-                                      ctx->tc_tile_m, pair_mode(ctx), ctx->pair_units);
+                                      ctx->tc_tile_m, pair_mode(ctx), ctx->pair_units,
+                                      ctx->endpoint_rm);
   out->tensor_core = 1;
   out->row_blocks = pl.RB;
   out->block_rows = pl.BN;
@@ -495,6 +508,8 @@ sph_status sph_plan_query(sph_ctx* ctx, int call, int64_t rows, int64_t n_keep, 
   out->whole_tiles = pl.whole_tiles;
   out->planes = pl.hilo;
   out->pair = pl.pair;
+  out->rows_m = pl.rm;
+  out->epilogue_stats = pl.epi_stats;
   return SPH_OK;
 }
 
@@ -676,6 +691,10 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
     case SPH_OPT_SPLIT_QUANTIZE:
       if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "split_quantize must be 0, 1 or 2");
       ctx->split_quantize = (int)value;
+      return SPH_OK;
+    case SPH_OPT_ENDPOINT_ROWS_M:
+      if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "endpoint_rows_m must be 0, 1 or 2");
+      ctx->endpoint_rm = (int)value;
       return SPH_OK;
     case SPH_OPT_ENDPOINT_Z:
       if (value < 0 || value > 2) return fail(ctx, SPH_ERR_INVALID_ARG, "endpoint_z must be 0, 1 or 2");

@@ -160,6 +160,14 @@ __device__ __forceinline__ int quantize_one(float y, float k, float inv_s) {
   return max(-127, min(127, q));
 }
 
+// The int8 code in byte e (0..3) of a word whose bytes were first XORed with
+// 0x80, as an exact float: the byte permute forms the fp32 2^23 + (code +
+// 128), and one exact subtraction leaves the code.  (Integer and ALU pipes
+// instead of an int-to-float conversion.)
+__device__ __forceinline__ float code_f32(unsigned w_x80, int e) {
+  return __uint_as_float(__byte_perm(w_x80, 0x4B000000u, 0x7440u | (unsigned)e)) - 8388736.0f;
+}
+
 // Non-negative floats order like their bit patterns, so a row maximum of
 // |y| can be kept as an unsigned atomicMax.
 __device__ __forceinline__ void atomic_max_nonneg(unsigned int* addr, float v) {

@@ -122,6 +122,7 @@ struct TcPlan {
   int single_acc;  // one TMEM accumulator (256-id tiles over > 128 rows)
   int nseg;        // endpoint statistics: 32-id segments per row, NT * tm / 32
   int epi_stats;   // endpoint: softmax statistics in the epilogue (else a pass over z)
+  int rm;          // endpoint on CTA pairs with rows as M (256-row blocks, whole tiles)
   int epi_t;       // endpoint: the epilogue may finish through a shared-memory transpose
                    // (where rows are 2-element aligned; shared memory reserved for it)
   long long T;
@@ -134,12 +135,13 @@ struct TcPlan {
 // gather = the kept-id subset path (keep_ids given); fp8 = e4m3 weights;
 // max_bn = most hidden-state rows per tile (0 = automatic); tile_m =
 // vocabulary rows per tile (128, 256 = two M = 128 halves, 0 = automatic);
-// pair_mode = CTA pairs on 256-id tiles (cloud epilogue with bf16 weights
-// only; ignored elsewhere): 0 never, 1 where the row blocks are long enough,
-// 2 always; max_pairs caps the pairs (0: no cap).
+// pair_mode = CTA pairs on 256-id tiles: 0 never, 1 where the row blocks are
+// long enough (bf16 weights), 2 always; max_pairs caps the pairs (0: no cap); rm_mode = the endpoint on
+// pairs with rows as M: 0 where the 256-row blocks pad little, 1 always
+// (where the call pairs), 2 never.
 TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
                int schedule, int max_stages, int block_k, int gather, int fp8, int max_bn,
-               int tile_m, int pair_mode = 0, int max_pairs = 0);
+               int tile_m, int pair_mode = 0, int max_pairs = 0, int rm_mode = 0);
 // CTA pairs of the pair kernel that can run at once on `device` (0 when the
 // query fails): tc_plan's max_pairs.
 int tc_pair_max_units(int device);

@@ -34,6 +34,7 @@ SPH_OPT_CHECK_IDS = 9
 SPH_OPT_SPLIT_QUANTIZE = 10
 SPH_OPT_TC_PAIR = 11
 SPH_OPT_ENDPOINT_Z = 12
+SPH_OPT_ENDPOINT_ROWS_M = 13
 SPH_SAMPLER_CDF, SPH_SAMPLER_GUMBEL = 0, 1
 
 _c_void_p = ctypes.c_void_p
@@ -55,7 +56,8 @@ class sph_profile(ctypes.Structure):
 
 
 PLAN_FIELDS = ("tensor_core", "row_blocks", "block_rows", "tile_ids", "tiles",
-               "k_blocks", "stages", "grid", "whole_tiles", "planes", "gemv_rows", "pair")
+               "k_blocks", "stages", "grid", "whole_tiles", "planes", "gemv_rows", "pair",
+               "rows_m", "epilogue_stats")
 
 
 class sph_plan(ctypes.Structure):

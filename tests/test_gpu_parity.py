@@ -920,3 +920,83 @@ def test_endpoint_z_option_values(ctx):
         with pytest.raises(sph.SphError):
             ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, v)
     ctx.set_option(sph.SPH_OPT_ENDPOINT_Z, 0)
+
+
+# ---------------------------------------------------------------------------
+# the endpoint on CTA pairs with the hidden-state rows as the MMA's M
+# (SPH_OPT_ENDPOINT_ROWS_M = 1): 256-row blocks, a lane per row, the
+# segment statistics from the epilogue
+# ---------------------------------------------------------------------------
+
+ROWS_M = [
+    ("few-rows", dict(V=4000, d=1024, d_l=128, rows=40, n_keep=1500, tau=0.8)),
+    ("ragged-n", dict(V=6000, d=640, d_l=64, rows=300, n_keep=3001)),
+    ("even-n", dict(V=6000, d=640, d_l=64, rows=256, n_keep=2002)),
+    ("aligned", dict(V=9000, d=600, d_l=72, rows=520, n_keep=4096)),
+    ("full-vocab", dict(V=3000, d=1280, d_l=256, rows=200, n_keep=3000)),
+    ("short", dict(V=500, d=136, d_l=16, rows=33, n_keep=7, run_lo=1, run_hi=3)),
+    ("greedy", dict(V=5000, d=768, d_l=128, rows=260, n_keep=2500, tau=0.0)),
+]
+
+
+@pytest.mark.parametrize("payload", [True, False])
+@pytest.mark.parametrize("name,kw", ROWS_M, ids=[c[0] for c in ROWS_M])
+def test_endpoint_rows_as_m(ctx, name, kw, payload):
+    from paper_2607_13093_gb300 import sph
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
+    ctx.set_option(sph.SPH_OPT_TC_PAIR, 1)
+    ctx.set_option(sph.SPH_OPT_ENDPOINT_ROWS_M, 1)
+    try:
+        w = small(seed=1401, **kw)
+        pe = ctx.plan(1, w.rows, w.n_keep, w.d_l, gather=w.keep_ids is not None)
+        assert pe["pair"] == 1 and pe["rows_m"] == 1 and pe["block_rows"] == 256
+        assert pe["epilogue_stats"] == 1
+        if payload:
+            pc, ps = wl.make_payload(w.rows, w.n_keep, seed=31)
+        else:
+            pc = ps = None
+        if payload:
+            check_endpoint(ctx, w, pc, ps)
+        else:
+            # no payload: z is the local partial alone
+            from _parity import fuse_sample_unstored
+            z = torch.empty(w.rows, w.n_keep, device=DEV)
+            t1 = ctx.fuse_sample(None, None, w.h_local, w.W_l, keep_ids=w.keep_ids,
+                                 temperature=w.tau, seed=w.seed, fused_logits_out=z)
+            t2 = fuse_sample_unstored(ctx, None, None, w.h_local, w.W_l, keep_ids=w.keep_ids,
+                                      temperature=w.tau, seed=w.seed)
+            ctx.sync()
+            ids = np_(w.keep_ids)
+            vocab = np.arange(w.V) if ids is None else ids
+            zref = oracle.local_partial(np_(w.h_local), bits(w.W_l), vocab)
+            assert_close(np_(z), zref, "local partial logits")
+            if w.tau == 0:
+                j, gap = oracle.greedy_rows(zref)
+                ok = gap >= GREEDY_GAP
+            else:
+                j, margin = oracle.sample_rows(
+                    zref, w.tau, oracle.philox_uniform(w.seed, np.arange(w.rows), 0, 0))
+                ok = margin >= MARGIN
+            for t in (t1, t2):
+                assert not ((np_(t) != vocab[j]) & ok).any()
+    finally:
+        ctx.set_option(sph.SPH_OPT_ENDPOINT_ROWS_M, 0)
+        ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+
+
+def test_endpoint_rows_as_m_option_values(ctx):
+    from paper_2607_13093_gb300 import sph
+    for v in (0, 1, 2):
+        ctx.set_option(sph.SPH_OPT_ENDPOINT_ROWS_M, v)
+    for v in (-1, 3):
+        with pytest.raises(sph.SphError):
+            ctx.set_option(sph.SPH_OPT_ENDPOINT_ROWS_M, v)
+    ctx.set_option(sph.SPH_OPT_ENDPOINT_ROWS_M, 0)
+    # stream-K schedules keep the transposed (ids as M) endpoint
+    ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 2)
+    try:
+        assert ctx.plan(1, 1024, 256000, 512, gather=False)["rows_m"] == 0
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_SCHEDULE, 0)
+    assert ctx.plan(1, 1024, 256000, 512, gather=False)["rows_m"] == 1

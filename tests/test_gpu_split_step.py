@@ -157,18 +157,23 @@ def test_split_step_one_chunk(path_ctx, name, kw):
 @pytest.mark.parametrize("name,kw", [c for c in ONE_CHUNK if c[0] != "fp8"],
                          ids=[c[0] for c in ONE_CHUNK if c[0] != "fp8"])
 @pytest.mark.parametrize("quantize", [1, 2])
-def test_split_step_pairs(ctx, name, kw, quantize):
+@pytest.mark.parametrize("rows_m", [1, 2])
+def test_split_step_pairs(ctx, name, kw, quantize, rows_m):
     # both contractions on CTA pairs, the endpoint quantizing in its epilogue
-    # (1) or after a separate pass (2)
+    # (1) or after a separate pass (2), with the rows as the MMA's M (1) or
+    # the ids (2)
     from paper_2607_13093_gb300 import sph
     ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1)
     ctx.set_option(sph.SPH_OPT_TC_PAIR, 1)
     ctx.set_option(sph.SPH_OPT_SPLIT_QUANTIZE, quantize)
+    ctx.set_option(sph.SPH_OPT_ENDPOINT_ROWS_M, rows_m)
     try:
         w = small(**kw)
-        assert ctx.plan(1, w.rows, w.n_keep, w.d_l, gather=w.keep_ids is not None)["pair"] == 1
+        pe = ctx.plan(1, w.rows, w.n_keep, w.d_l, gather=w.keep_ids is not None)
+        assert pe["pair"] == 1 and pe["rows_m"] == (rows_m == 1)
         check_split(ctx, w, 0)
     finally:
+        ctx.set_option(sph.SPH_OPT_ENDPOINT_ROWS_M, 0)
         ctx.set_option(sph.SPH_OPT_SPLIT_QUANTIZE, 0)
         ctx.set_option(sph.SPH_OPT_TC_PAIR, 0)
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
