@@ -149,8 +149,9 @@ typedef enum sph_option {
                                MMA over both CTAs' shared memory, each CTA
                                loading 128 ids of the weights and half of the
                                hidden-state rows.  0 (default): where the row
-                               blocks are long (>= 192 rows, or >= 128 with
-                               bf16 activations); 1: always (SPH_ERR_
+                               blocks are long (bf16 weights; >= 128 rows
+                               for the cloud, >= 192 for the endpoint);
+                               1: always (SPH_ERR_
                                UNSUPPORTED where pairs cannot be scheduled);
                                2: never.  The results are the fp32 sums of
                                the same products either way.               */

@@ -1532,7 +1532,8 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
   pl.BN = ((rows + pl.RB - 1) / pl.RB + 31) / 32 * 32;
   // the endpoint with rows as M: 256-row blocks (M = 256 over the pair),
   // whole tiles; automatic where the row blocks lose at most 1/8 to padding
-  // (measured on 1024 rows x 256000 ids x 512: ... )
+  // (measured on 1024 rows x 256000 ids x 512: 0.43 ms with z not stored,
+  // against 0.56 ms and a 0.18 ms statistics pass with ids as M)
   const int rb256 = (rows + 255) / 256;
   pl.rm = endpoint && !pl.fp8 && schedule != 2 && rm_mode != 2 &&
           (rm_mode == 1 || (cap == 256 && 8 * (rb256 * 256 - rows) <= rb256 * 256));
@@ -1544,13 +1545,19 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
   pl.tm = 128;
   pl.single_acc = 0;
   pl.Rp = pl.RB * pl.BN;
+  // the endpoint's epilogue as on single CTAs (each CTA of a pair finishes
+  // its own 128 ids for all BN rows); rows as M: the statistics of a
+  // lane's 32-id segment are its own, always made in the epilogue
+  pl.epi_stats = pl.rm || endpoint == 2 || (endpoint && (pl.BN < 128 || 4 * pl.BN <= K));
+  pl.epi_t = !pl.rm && (endpoint == 2 || (endpoint && !pl.epi_stats));
+  const int reserve = 2048 + (pl.epi_t ? kTransposeBytes : 0);
   auto stage_of = [&](int na) { return na * (kAtomBytes + pl.hilo * (pl.BN / 2) * 128); };
   // (a pair pays a cross-CTA hand-off per stage, so it prefers fewer,
   // larger stages: measured on 1024 rows x 256000 ids x 4608 with bf16
   // activations, three 128-column stages 1746 us, six 64-column 2005 us)
   pl.na = pl.fp8 ? 1 : (block_k == 64 ? 1 : (block_k == 256 ? 4 : 2));
   const int min_stages = block_k ? 2 : 3;
-  while (pl.na > 1 && (int)((kSmemBudget - 2048) / stage_of(pl.na)) < min_stages) pl.na >>= 1;
+  while (pl.na > 1 && (int)((kSmemBudget - reserve) / stage_of(pl.na)) < min_stages) pl.na >>= 1;
   const int bk = pl.na * (pl.fp8 ? kAtomE8 : kAtomK);
   pl.KB = (K + bk - 1) / bk;
   pl.Kp = pl.KB * bk;
@@ -1567,12 +1574,7 @@ TcPlan tc_plan_pair(TcPlan pl, int rows, int n, int K, int sm_count, int max_pai
   pl.whole_tiles = schedule == 1 || (schedule == 0 && whole_span <= 1.1 * split_span + 2.0);
   units = pl.whole_tiles ? g_whole : (int)(pl.T < units ? pl.T : units);
   pl.G = 2 * units;
-  // the endpoint's epilogue as on single CTAs (each CTA of a pair finishes
-  // its own 128 ids for all BN rows); rows as M: the statistics of a
-  // lane's 32-id segment are its own, always made in the epilogue
-  pl.epi_stats = pl.rm || endpoint == 2 || (endpoint && (pl.BN < 128 || 4 * pl.BN <= K));
-  pl.epi_t = !pl.rm && (endpoint == 2 || (endpoint && !pl.epi_stats));
-  pl.stages = (int)((kSmemBudget - 2048 - (pl.epi_t ? kTransposeBytes : 0)) / stage_of(pl.na));
+  pl.stages = (int)((kSmemBudget - reserve) / stage_of(pl.na));
   if (pl.stages > kMaxStages) pl.stages = kMaxStages;
   if (max_stages >= 2 && pl.stages > max_stages) pl.stages = max_stages;
   pl.hs_bytes = pl.fp8 ? align256((size_t)pl.hilo * pl.Rp * pl.Kp) + align256((size_t)pl.Rp * 4)
@@ -1602,21 +1604,23 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   (void)gather;
   // CTA pairs: forced (pair_mode 2), or chosen (1) where their row blocks
   // are long enough that halving each SM's B bytes pays for the pair's
-  // hand-offs: >= 192 rows, or >= 128 with one plane.  Measured pair vs
-  // single: 1024 rows x 256000 ids x 4608 fp32 2654 vs 3191 us, bf16 (three
-  // stages) 1746 vs 2005; 256 rows x 256000 fp32 737 vs 897; 320 rows x
-  // 51302 x 3584 bf16 161 vs 195, fp32 (160-row blocks) 242 vs 223; 32
-  // rows x 12000 x 3840 38.9 vs 37.2; 64 rows x 256000 x 4608 471 vs 433.
-  // The endpoint (K = d_l) pairs by the same rule: its B bytes per MMA are
-  // most of its traffic (measured 1024 rows x 256000 ids x 512: 665 vs 721
-  // us; 256 rows: 189 vs 408).
+  // hand-offs: >= 128 rows.  Measured pair vs single: 1024 rows x 256000
+  // ids x 4608 fp32 2654 vs 3191 us, bf16 (three stages) 1746 vs 2005; 256
+  // rows x 256000 fp32 737 vs 897; 320 rows x 51302 x 3584 bf16 161 vs 195,
+  // fp32 (160-row blocks) 182 vs 208 (with the pair hand-offs of today; 242
+  // vs 223 before them); 32 rows x 12000 x 3840 38.9 vs 37.2; 64 rows x
+  // 256000 x 4608 471 vs 433.
+  // The endpoint (K = d_l) pairs from 192-row blocks: its B bytes per MMA
+  // are most of its traffic (measured 1024 rows x 256000 ids x 512: 665 vs
+  // 721 us; 256 rows: 189 vs 408), but 160-row blocks gain nothing (320
+  // rows x 51302 x 512: 75.3 vs 71.6 us).
   // (an explicitly set tile height keeps single-CTA tiles unless pairs are
   // forced)
   if (pair_mode > 0 && sm_count >= 2 && (tile_m == 0 || pair_mode == 2)) {
     pl.pair = 1;
     const TcPlan pp = tc_plan_pair(pl, rows, n, K, sm_count, max_pairs, schedule, max_stages,
                                    block_k, max_bn_opt, endpoint, rm_mode);
-    if (pair_mode == 2 || (!fp8 && (pp.BN >= 192 || (pl.hilo == 1 && pp.BN >= 128)))) return pp;
+    if (pair_mode == 2 || (!fp8 && pp.BN >= (endpoint ? 192 : 128))) return pp;
     pl.pair = 0;
   }
   const int atom = fp8 ? kAtomE8 : kAtomK;   // elements per 128-byte atom
