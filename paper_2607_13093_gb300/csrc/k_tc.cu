@@ -74,6 +74,7 @@ constexpr int kBarrierArea = 512;
 // (+4 words of padding per row, so that both the row writes and the 16-byte
 // reads are free of bank conflicts)
 constexpr int kTRow = 36;
+constexpr float kLog2eF = 1.4426950408889634f;   // exp(d / tau) = 2^(d log2(e) / tau)
 // Kernel instantiations of EPI_ENDPOINT that finish through the per-warp
 // shared-memory transpose (finish_chunk_t) rather than per lane.
 constexpr int EPI_ENDPOINT_T = 3;
@@ -84,7 +85,6 @@ constexpr int EPI_ENDPOINT_T = 3;
 // accumulator load.
 constexpr int EPI_ENDPOINT_RM = 4;
 constexpr int EPI_FUSED_RM = 5;
-constexpr float kLog2eF = 1.4426950408889634f;
 constexpr int kTransposeBytes = 8 /* epilogue warps */ * 8 * kTRow * 4;
 constexpr size_t kSmemBudget = 220 * 1024;
 constexpr long long kDrainLimit = 1ll << 31;   // cycles, for in-flight copies
@@ -279,7 +279,7 @@ __device__ __forceinline__ void finish_chunk(const TcParams& p, const float (&v)
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const float mq = __shfl_sync(0xFFFFFFFFu, mk, 2 * q);
-      e[q] = (vj && row0 + q < p.R) ? expf((z[q] - mq) * p.inv_tau) : 0.f;
+      e[q] = (vj && row0 + q < p.R) ? ex2_approx((z[q] - mq) * (p.inv_tau * kLog2eF)) : 0.f;
     }
     const float sk = warp_reduce_scatter16(e, SumOp{}, lane);
     if (!(lane & 1) && row0 + kr < p.R)
@@ -383,7 +383,7 @@ __device__ __forceinline__ void finish_chunk_t(const TcParams& p, const float (&
       float sum = 0.f;
       if (m > -INFINITY) {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) sum += expf((x[e] - m) * p.inv_tau);   // exp(-inf) = 0
+        for (int e = 0; e < 8; ++e) sum += ex2_approx((x[e] - m) * (p.inv_tau * kLog2eF));  // 2^-inf = 0
       }
       sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 1);
       sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 2);
@@ -515,7 +515,7 @@ __device__ __forceinline__ void finish_rm(const TcParams& p, float (&v)[32], int
       const float l2t = p.inv_tau * kLog2eF;   // exp(d / tau) = 2^(d log2(e) / tau)
 #pragma unroll
       for (int i = 0; i < 16; ++i)
-        t[i] = exp2f((v[2 * i] - m) * l2t) + exp2f((v[2 * i + 1] - m) * l2t);
+        t[i] = ex2_approx((v[2 * i] - m) * l2t) + ex2_approx((v[2 * i + 1] - m) * l2t);
 #pragma unroll
       for (int w = 8; w >= 1; w >>= 1)
 #pragma unroll

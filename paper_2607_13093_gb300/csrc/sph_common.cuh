@@ -160,6 +160,17 @@ __device__ __forceinline__ int quantize_one(float y, float k, float inv_s) {
   return max(-127, min(127, q));
 }
 
+// 2^x by the special-function unit's approximation (`ex2.approx.ftz`: a
+// relative error of a few ulp; results below 2^-126 flush to 0, which for
+// softmax weights relative to the row maximum is below any weight that can
+// move a draw).  One instruction, where exp2f adds a scaling path for
+// subnormal results.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // The int8 code in byte e (0..3) of a word whose bytes were first XORed with
 // 0x80, as an exact float: the byte permute forms the fp32 2^23 + (code +
 // 128), and one exact subtraction leaves the code.  (Integer and ALU pipes
