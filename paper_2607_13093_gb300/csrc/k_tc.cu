@@ -1328,8 +1328,28 @@ split_h_e4m3_kernel(const float* __restrict__ h, int64_t ld_h, int R, int K, int
     if (act_bf16) x = __bfloat162float(__float2bfloat16_rn(x));
     return x;
   };
+  // each thread takes 4 consecutive columns at a time: one 16-byte load
+  // where the row is so aligned, one 4-byte store per plane
+  const bool v16 = (reinterpret_cast<uintptr_t>(hr) & 15) == 0;
+  auto value4 = [&](int c, float (&x)[4]) {
+    if (v16 && r < R && c + 4 <= K) {
+      const float4 t = __ldg(reinterpret_cast<const float4*>(hr + c));
+      x[0] = t.x; x[1] = t.y; x[2] = t.z; x[3] = t.w;
+      if (act_bf16) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) x[e] = __bfloat162float(__float2bfloat16_rn(x[e]));
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) x[e] = value(c + e);
+    }
+  };
   float m = 0.f;
-  for (int c = threadIdx.x; c < K; c += blockDim.x) m = fmaxf(m, fabsf(value(c)));
+  for (int c = 4 * threadIdx.x; c < K; c += 4 * blockDim.x) {
+    float x[4];
+    value4(c, x);
+    m = fmaxf(m, fmaxf(fmaxf(fabsf(x[0]), fabsf(x[1])), fmaxf(fabsf(x[2]), fabsf(x[3]))));
+  }
 #pragma unroll
   for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
   if ((threadIdx.x & 31) == 0) s_max[threadIdx.x >> 5] = m;
@@ -1344,12 +1364,21 @@ split_h_e4m3_kernel(const float* __restrict__ h, int64_t ld_h, int R, int K, int
                                            : 1.0f;
   if (threadIdx.x == 0) h_scale[r] = scale;
   const int64_t plane = (int64_t)Rp * Kp;
-  for (int c = threadIdx.x; c < Kp; c += blockDim.x) {
-    float x = value(c) * inv;            // exact: a power of two
+  // (Kp is a multiple of 128, so every 4-column group is 4-byte aligned)
+  for (int c = 4 * threadIdx.x; c < Kp; c += 4 * blockDim.x) {
+    float x[4];
+    value4(c, x);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) x[e] *= inv;              // exact: a power of two
     for (int q = 0; q < planes; ++q) {
-      const __nv_fp8_e4m3 e(x);          // round to nearest, saturating
-      Hs[q * plane + (int64_t)r * Kp + c] = e.__x;
-      x -= static_cast<float>(e);
+      uint32_t word = 0;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const __nv_fp8_e4m3 f(x[e]);                      // round to nearest, saturating
+        word |= (uint32_t)f.__x << (8 * e);
+        x[e] -= static_cast<float>(f);
+      }
+      *reinterpret_cast<uint32_t*>(Hs + q * plane + (int64_t)r * Kp + c) = word;
     }
   }
 }
