@@ -1,6 +1,7 @@
 // Thin inline-PTX wrappers for the Blackwell (sm_100 family) features the
-// tensor-core kernels use: mbarriers, TMA tensor copies (tiled and
-// tile::gather4), Tensor Memory allocation, tcgen05.mma / commit / ld.
+// tensor-core kernels use: mbarriers, tiled TMA tensor copies, Tensor Memory
+// allocation, tcgen05.mma / commit / ld, CTA-pair (cluster) forms and
+// programmatic dependent launch.
 #pragma once
 
 #include <cuda.h>
