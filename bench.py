@@ -440,6 +440,12 @@ class Runner:
         self.z = torch.empty(R, n, device=dev) if w.sessions else None
         self.n_acc = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
         self.nxt = torch.empty(max(1, w.sessions), dtype=torch.int32, device=dev)
+        # drafted workloads: the endpoint fuses the target rows (z) and the
+        # verification makes their softmax statistics and draws the next
+        # tokens; other workloads draw one token per row at the endpoint
+        self.draw_kw = {"draw": False} if w.sessions else {"tokens": self.tokens}
+        # what a step hands back to the host
+        self.results = [self.n_acc, self.nxt] if w.sessions else [self.tokens]
         self.gsteps = ncopy * max(1, math.ceil(16 / ncopy))
 
     def step(self, i, h=None, events=None):
@@ -463,8 +469,8 @@ class Runner:
                 events[1].record()
         elif self.nosplit:               # one endpoint call over the whole head
             ctx.fuse_sample(None, None, hh, self.Wfs[c], keep_ids=w.keep_ids,
-                            temperature=w.tau, seed=w.seed, offset=i, tokens=self.tokens,
-                            fused_logits_out=self.z)
+                            temperature=w.tau, seed=w.seed, offset=i,
+                            fused_logits_out=self.z, **self.draw_kw)
         else:
             ctx.partial_logits(hh[:, w.d_l:], self.Whs[c], keep_ids=w.keep_ids, clip=w.clip,
                                w_row_scale=w.w_scale, bias=w.bias, codes=self.codes,
@@ -474,7 +480,7 @@ class Runner:
         if self.mode == "split":
             ctx.fuse_sample(self.codes, self.scale, hh[:, :w.d_l], self.Wls[c],
                             keep_ids=w.keep_ids, temperature=w.tau, seed=w.seed, offset=i,
-                            tokens=self.tokens, fused_logits_out=self.z)
+                            fused_logits_out=self.z, **self.draw_kw)
         if w.sessions:
             ctx.verify_draft(self.z, w.sessions, w.k, w.draft_tokens, keep_ids=w.keep_ids,
                              draft_probs=w.draft_probs, temperature=w.tau,
@@ -584,12 +590,17 @@ def e2e_run(r, steps, world=1):
     import torch.distributed as dist
     dev, w = r.dev, r.w
     h_host = [x.cpu().pin_memory() for x in r.hs]
-    tok_host = torch.empty(w.rows, dtype=torch.int32).pin_memory()
+    res_host = [torch.empty_like(t, device="cpu").pin_memory() for t in r.results]
     h_dev = torch.empty_like(w.h)
+
+    def read_back():
+        for hst, t in zip(res_host, r.results):
+            hst.copy_(t, non_blocking=True)
+
     for i in range(3):
         h_dev.copy_(h_host[i % r.ncopy], non_blocking=True)
         r.step(i, h_dev)
-        tok_host.copy_(r.tokens, non_blocking=True)
+        read_back()
         torch.cuda.synchronize(dev)
     if world > 1:
         dist.barrier()
@@ -597,14 +608,16 @@ def e2e_run(r, steps, world=1):
     for i in range(steps):
         h_dev.copy_(h_host[i % r.ncopy], non_blocking=True)
         r.step(i, h_dev)
-        tok_host.copy_(r.tokens, non_blocking=True)
+        read_back()
         torch.cuda.synchronize(dev)
     dt = max_over_ranks(time.perf_counter() - t0, dev)
     return {"value": round(w.rows * world * steps / dt, 1), "unit": UNIT,
-            "h2d_bytes_per_step": w.rows * w.d * 4, "d2h_bytes_per_step": w.rows * 4,
+            "h2d_bytes_per_step": w.rows * w.d * 4,
+            "d2h_bytes_per_step": sum(t.numel() * t.element_size() for t in r.results),
             "steps": steps,
             "note": ("pinned host h -> device, direct C-ABI calls (no graph), "
-                     "tokens -> host, sync per step")}
+                     + ("accept counts and next tokens" if w.sessions else "tokens")
+                     + " -> host, sync per step")}
 
 
 def unit_stats(unit):

@@ -400,7 +400,10 @@ sph_status sph_partial_logits_noalloc(int device, void* cuda_stream,
  *   W_l bf16 [V, d_l] row-major with row stride ld_wl; the base address
  *   and ld_wl*2 must be multiples of 16 bytes.
  *   keep_ids as for sph_partial_logits.  temperature >= 0 and finite.
- *   tokens int32 [rows] (out, vocabulary ids).
+ *   tokens int32 [rows] (out, vocabulary ids), or NULL: z alone (fuse,
+ *   Eq. 13, and mask), no softmax statistics and no draw -- the form for
+ *   target rows that go to sph_verify_draft, which makes the statistics
+ *   and draws the next tokens itself; fused_logits_out is then required.
  *   fused_logits_out fp32 [rows, n_keep] z before the division by
  *   temperature (out), or NULL.
  * Errors: INVALID_ARG, UNSUPPORTED, CUDA, OOM. */

@@ -1701,9 +1701,14 @@ TcPlan tc_plan(int rows, int n, int K, int act_bf16, int sm_count, int endpoint,
   }
   pl.Rp = pl.RB * pl.BN;
   // k-block width: as asked (automatic: 128), narrowed until the shared
-  // memory holds at least min_stages pipeline stages
+  // memory holds at least min_stages pipeline stages.  The full vocabulary
+  // with row blocks of at most 16 rows keeps 128 columns down to three
+  // stages: one 3-D copy per stage then moves twice the bytes (measured, 8
+  // rows x 256000 ids x 4608 on 256-id tiles: 383 us in three 72 KB stages
+  // against 404 us in six 36 KB ones; with kept-id subsets, or 32 and 64
+  // rows, the narrower stages are as fast or faster)
   pl.na = fp8 ? 1 : (block_k == 64 ? 1 : (block_k == 256 ? 4 : 2));
-  const int min_stages = block_k ? 2 : 4;
+  const int min_stages = block_k ? 2 : ((!gather && pl.BN <= 16) ? 3 : 4);
   while (pl.na > 1 &&
          (int)((kSmemBudget - 2048) / (pl.na * (halves * kAtomBytes + pl.hilo * pl.BN * 128))) <
              min_stages)

@@ -341,9 +341,13 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
   gg.status = ctx->status; gg.finish_wait = ctx->tc_finish_wait;
   gg.inv_tau = stats_inv_tau(temperature);
   const int greedy = temperature == 0.f;
-  // Gumbel-max draws need no softmax statistics: the epilogue skips them
+  // Gumbel-max draws need no softmax statistics: the epilogue skips them;
+  // nor does a call without tokens (z alone, for the verification)
   const bool gumbel = ctx->sampler == 1 && !greedy;
-  gg.no_stats = gumbel;
+  const bool fuse_only = tokens == nullptr;
+  if (fuse_only && !z_out)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "a call without tokens needs fused_logits_out");
+  gg.no_stats = gumbel || fuse_only;
   // z unstored (SPH_OPT_ENDPOINT_Z): automatic where the endpoint runs with
   // rows as M, whose epilogue makes each segment's statistics in its own
   // lane (measured, steps of 1024 x 256000 ids x d_l 512: 3.18 vs 3.43 ms;
@@ -392,7 +396,7 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
     st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
                        }), "tensor-core launch");
-    if (st) return st;
+    if (st || fuse_only) return st;
     if (gumbel) return draw_gumbel();
     return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                            return sph::launch_sample_from_stats(
@@ -408,7 +412,7 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
   st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                        return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
                      }), "gemv launch");
-  if (st) return st;
+  if (st || fuse_only) return st;
   if (gumbel) return draw_gumbel();
   return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                          cudaError_t e = sph::launch_seg_stats(Z, rows, n_keep,
@@ -826,8 +830,10 @@ sph_status sph_fuse_sample(sph_ctx* ctx, const int8_t* codes,
                            uint64_t offset, int32_t* tokens,
                            float* fused_logits_out) {
   if (!ctx) return SPH_ERR_INVALID_ARG;
-  if (!h_local || !W_l || !tokens)
-    return fail(ctx, SPH_ERR_INVALID_ARG, "h_local, W_l and tokens must be non-NULL");
+  if (!h_local || !W_l)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "h_local and W_l must be non-NULL");
+  if (!tokens && !fused_logits_out)
+    return fail(ctx, SPH_ERR_INVALID_ARG, "tokens and fused_logits_out must not both be NULL");
   if (!codes != !row_scale)
     return fail(ctx, SPH_ERR_INVALID_ARG, "codes and row_scale must both be given or both be NULL");
   if (rows < 1 || rows > (1 << 20)) return fail(ctx, SPH_ERR_INVALID_ARG, "rows=%lld out of [1, 2^20]", (long long)rows);

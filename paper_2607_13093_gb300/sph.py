@@ -342,8 +342,10 @@ def sph_partial_logits_noalloc(h_cloud, W_h, *, codes, row_scale,
 
 def sph_fuse_sample(ctx, codes, row_scale, h_local, W_l, *, keep_ids=None,
                     temperature=1.0, seed=0, offset=0, tokens=None,
-                    fused_logits_out=None):
-    """Endpoint call.  Returns tokens int32 [R] (vocabulary ids)."""
+                    fused_logits_out=None, draw=True):
+    """Endpoint call.  Returns tokens int32 [R] (vocabulary ids); with
+    draw=False only z is computed (into fused_logits_out, required) and the
+    call returns None."""
     _need(codes, torch.int8, "codes")
     _need(row_scale, torch.float32, "row_scale")
     _need(h_local, torch.float32, "h_local")
@@ -353,7 +355,10 @@ def sph_fuse_sample(ctx, codes, row_scale, h_local, W_l, *, keep_ids=None,
     R, d_l = h_local.shape
     V = W_l.shape[0]
     n = V if keep_ids is None else keep_ids.numel()
-    if tokens is None:
+    if not draw:
+        if fused_logits_out is None or tokens is not None:
+            raise ValueError("draw=False needs fused_logits_out and no tokens")
+    elif tokens is None:
         tokens = torch.empty(R, dtype=torch.int32, device=h_local.device)
     _need(tokens, torch.int32, "tokens")
     _check(ctx, lib.sph_fuse_sample(

@@ -199,6 +199,54 @@ def test_endpoint_parity(path_ctx, name, kw):
         check_endpoint(ctx, w, codes, scale)
 
 
+FUSE_ONLY = [
+    ("decode-small", dict(V=4000, d=1024, d_l=256, rows=32, n_keep=1500, tau=0.8)),
+    ("spec-like", dict(V=6000, d=640, d_l=128, rows=160, n_keep=2400, sessions=32, k=4)),
+    ("full-vocab", dict(V=3000, d=1280, d_l=264, rows=16, n_keep=3000)),
+    ("rows3", dict(V=2000, d=300, d_l=40, rows=3, n_keep=700)),
+]
+
+
+@pytest.mark.parametrize("name,kw", FUSE_ONLY, ids=[c[0] for c in FUSE_ONLY])
+def test_endpoint_fuse_only(path_ctx, name, kw):
+    # no tokens: z alone (no statistics, no draw), bit-identical to the z of
+    # the drawing call and within tolerance of the oracle; the verification
+    # of drafted rows on it matches the oracle
+    ctx = path_ctx
+    w = small(**kw)
+    ref = oracle_cloud(w)
+    codes = torch.from_numpy(ref["codes"]).to(DEV)
+    scale = torch.from_numpy(ref["row_scale"]).to(DEV)
+    z_draw = torch.empty(w.rows, w.n_keep, device=DEV)
+    z_only = torch.full((w.rows, w.n_keep), float("nan"), device=DEV)
+    ctx.fuse_sample(codes, scale, w.h_local, w.W_l, keep_ids=w.keep_ids, temperature=w.tau,
+                    seed=w.seed, fused_logits_out=z_draw)
+    assert ctx.fuse_sample(codes, scale, w.h_local, w.W_l, keep_ids=w.keep_ids,
+                           temperature=w.tau, seed=w.seed, fused_logits_out=z_only,
+                           draw=False) is None
+    ctx.sync()
+    assert torch.equal(z_draw.view(torch.int32), z_only.view(torch.int32))
+    zl = oracle.local_partial(np_(w.h_local), bits(w.W_l), np_(w.keep_ids))
+    assert_close(np_(z_only), oracle.fuse(ref["codes"], ref["row_scale"], zl), "fused logits")
+    if w.sessions:
+        check_verify(ctx, w, z_only.cpu())
+
+
+def test_endpoint_fuse_only_needs_z(ctx):
+    from paper_2607_13093_gb300 import sph
+    w = small(V=600, d=136, d_l=8, rows=4, n_keep=300)
+    codes, scale = (t.to(DEV) for t in wl.make_payload(4, 300, seed=3))
+    with pytest.raises(ValueError):
+        ctx.fuse_sample(codes, scale, w.h_local, w.W_l, keep_ids=w.keep_ids, draw=False)
+    # through the C ABI: neither tokens nor z is INVALID_ARG, before any launch
+    st = sph.lib.sph_fuse_sample(ctx.handle, codes.data_ptr(), scale.data_ptr(), 4,
+                                 w.h_local.data_ptr(), w.h_local.stride(0),
+                                 w.W_l.data_ptr(), w.V, w.d_l, w.W_l.stride(0),
+                                 w.keep_ids.data_ptr(), 300, 1.0, 0, 0, None, None)
+    assert st == 1
+    ctx.sync()
+
+
 @pytest.mark.parametrize("tau", [0.05, 0.8, 3.0])
 def test_endpoint_temperatures(ctx, tau):
     w = small(V=2000, d=300, d_l=64, rows=24, n_keep=800, tau=tau)
