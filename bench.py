@@ -584,40 +584,67 @@ def timed_run(r, steps, warmup, *, bracket, min_pairs=64, world=1, rank=0, sampl
 
 
 def e2e_run(r, steps, world=1):
-    """The step through the public API with host buffers: pinned h in,
-    tokens out, synchronised every step."""
+    """The step through the public API with host buffers: each step copies
+    its h in from pinned host memory, runs the calls, and reads its results
+    back to pinned host memory, synchronised every step.
+
+    Two ways of driving the same calls: `direct` issues them from the host
+    every step (each launch costs host time); `graph` captures the copy in,
+    the public calls and the copy out into a CUDA graph once per pinned
+    input buffer (the library supports capture after sph_reserve) and
+    replays one per step, as a serving loop would.  A captured step keeps
+    the draws' random-stream offset it was captured with."""
     import torch
     import torch.distributed as dist
     dev, w = r.dev, r.w
     h_host = [x.cpu().pin_memory() for x in r.hs]
-    res_host = [torch.empty_like(t, device="cpu").pin_memory() for t in r.results]
+    res_host = [[torch.empty_like(t, device="cpu").pin_memory() for t in r.results]
+                for _ in range(r.ncopy)]
     h_dev = torch.empty_like(w.h)
 
-    def read_back():
-        for hst, t in zip(res_host, r.results):
+    def one_step(i):
+        c = i % r.ncopy
+        h_dev.copy_(h_host[c], non_blocking=True)
+        r.step(i, h_dev)
+        for hst, t in zip(res_host[c], r.results):
             hst.copy_(t, non_blocking=True)
 
-    for i in range(3):
-        h_dev.copy_(h_host[i % r.ncopy], non_blocking=True)
-        r.step(i, h_dev)
-        read_back()
-        torch.cuda.synchronize(dev)
-    if world > 1:
-        dist.barrier()
-    t0 = time.perf_counter()
-    for i in range(steps):
-        h_dev.copy_(h_host[i % r.ncopy], non_blocking=True)
-        r.step(i, h_dev)
-        read_back()
-        torch.cuda.synchronize(dev)
-    dt = max_over_ranks(time.perf_counter() - t0, dev)
-    return {"value": round(w.rows * world * steps / dt, 1), "unit": UNIT,
+    def timed(run):
+        for i in range(3):
+            run(i)
+            torch.cuda.synchronize(dev)
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for i in range(steps):
+            run(i)
+            torch.cuda.synchronize(dev)
+        return max_over_ranks(time.perf_counter() - t0, dev)
+
+    dt_direct = timed(one_step)
+    # one graph per pinned input buffer, captured on a side stream
+    graphs = []
+    cs = torch.cuda.Stream(device=dev)
+    cs.wait_stream(torch.cuda.current_stream(dev))
+    for c in range(r.ncopy):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cs):
+            one_step(c)
+        graphs.append(g)
+    torch.cuda.synchronize(dev)
+    dt_graph = timed(lambda i: graphs[i % r.ncopy].replay())
+    del graphs
+    rows = w.rows * world * steps
+    return {"value": round(rows / dt_graph, 1), "unit": UNIT,
             "h2d_bytes_per_step": w.rows * w.d * 4,
             "d2h_bytes_per_step": sum(t.numel() * t.element_size() for t in r.results),
             "steps": steps,
-            "note": ("pinned host h -> device, direct C-ABI calls (no graph), "
+            "direct_calls": {"value": round(rows / dt_direct, 1), "unit": UNIT},
+            "note": ("pinned host h -> device, the public C-ABI calls, "
                      + ("accept counts and next tokens" if w.sessions else "tokens")
-                     + " -> host, sync per step")}
+                     + " -> pinned host, sync per step; value: the step captured in a CUDA "
+                       "graph per input buffer and replayed; direct_calls: the same calls "
+                       "issued from the host every step")}
 
 
 def unit_stats(unit):
@@ -689,9 +716,11 @@ def config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks, cpu_seconds,
                  "ms_per_step": round(res["ms"] / steps, 5), "steps": steps,
                  ("step_call_us" if one_call else "cloud_us"): round(unit["mean_ms"] * 1e3, 2),
                  "roofline": roof,
-                 "e2e_rows_per_s": e2e_run(r, e2e_steps)["value"],
                  "payload_bytes_per_step": (w.rows * w.n_keep + 4 * w.rows * r.nchunk),
                  "gpu_launches_per_step": round(res["launches_per_step"], 2)}
+        e2e = e2e_run(r, e2e_steps)
+        entry["e2e_rows_per_s"] = e2e["value"]
+        entry["e2e_direct_rows_per_s"] = e2e["direct_calls"]["value"]
         if with_cpu:
             entry["cpu_baseline"] = cpu_baseline(w, cpu_seconds, act, mode == "nosplit")
         return entry
