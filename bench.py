@@ -109,6 +109,9 @@ def parse():
                     help="skip the per-configuration block")
     ap.add_argument("--dend-grid", action="store_true",
                     help="add the split-dimension study's grid (d_l x keep) to the block")
+    ap.add_argument("--sweep-grid", action="store_true",
+                    help="add the sweep's kept fractions 10 %% and 50 %% for every row count "
+                         "to the block (100 %% is in it already)")
     ap.add_argument("--ref-seconds", type=float, default=150.0,
                     help="--impl reference: host seconds of oracle work over all steps")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -681,6 +684,8 @@ CONFIG_BLOCK = [("tiny", None, None, None, "fp32", "split", 0),
                 # the unsplit head (the no-split ablation)
                 ("decode", None, None, None, "fp32", "nosplit", 0)]
 DEND_GRID = [(k, d) for k in (0.4, 0.3) for d in (48, 96, 128, 256, 512)]
+# the sweep's other kept fractions (rows x keep; fp32 activations)
+SWEEP_GRID = [(r, k) for k in (0.1, 0.5) for r in (1, 8, 64, 256, 1024)]
 
 
 def config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks, cpu_seconds,
@@ -874,6 +879,8 @@ def run_ours(args):
             args.vocab is None:
         block = list(CONFIG_BLOCK) + ([("dend", None, k, d, "fp32", "split", 0)
                                        for k, d in DEND_GRID] if args.dend_grid else [])
+        block += ([("sweep", r, k, None, "fp32", "split", 0) for r, k in SWEEP_GRID]
+                  if args.sweep_grid else [])
         entries = []
         seen_cpu = set()
         for (name, rows, keep, d_l, act, mode, chunk) in block:
