@@ -4,8 +4,10 @@
 A step is one pass of the whole hot path over one batch of R hidden-state
 rows: the cloud call (gathered partial logits over the kept vocabulary ids,
 clip, per-row int8) followed by the endpoint call (local partial, fuse,
-mask, softmax, sample); workloads with drafts add the speculative
-verification.  Inputs are seeded synthetic data of the paper's shapes and
+mask, softmax, sample).  Workloads with drafts take the speculative step
+instead: the endpoint call fuses the target rows (z alone) and the
+verification makes their softmax statistics, accepts or rejects each draft
+and draws every session's next token.  Inputs are seeded synthetic data of the paper's shapes and
 stay resident in HBM; weight copies rotate so that the bytes touched
 between two uses of the same copy exceed twice the L2 size.
 
