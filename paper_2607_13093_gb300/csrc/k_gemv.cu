@@ -189,6 +189,49 @@ gemv_kernel(const GatherGemm g, const int row0) {
     if (lane < kVPW * RT) atomicMax(&smax[lane % RT], __float_as_uint(lmax));
     __syncthreads();
     if (threadIdx.x < rt) atomicMax(&g.rowmax[row0 + threadIdx.x], smax[threadIdx.x]);
+    if (g.q_ticket) {
+      // every block's partials and maxima are visible to the last block to
+      // arrive, which quantizes them exactly as the quantize pass does
+      // (row_quant, quantize_one) and leaves the maxima and its ticket at
+      // zero for the next call
+      __shared__ int s_last;
+      __threadfence();
+      __syncthreads();
+      if (threadIdx.x == 0) s_last = atomicAdd(g.q_ticket, 1u) == gridDim.x - 1;
+      __syncthreads();
+      if (s_last) {
+        __threadfence();
+        __shared__ RowQuant s_rq[RT];
+        if (threadIdx.x < rt) {
+          const RowQuant rq = row_quant(__ldcg(g.rowmax + row0 + threadIdx.x));
+          s_rq[threadIdx.x] = rq;
+          g.q_scale[row0 + threadIdx.x] = rq.s;
+        }
+        __syncthreads();
+        // eight independent loads a thread before their codes (one L2
+        // round trip per batch, not per entry)
+        const int total = rt * g.n;
+        const int64_t o0 = (int64_t)row0 * g.n;
+        for (int b = 0; b < total; b += 8 * kThreads) {
+          float y[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int i = b + u * kThreads + threadIdx.x;
+            y[u] = i < total ? __ldcg(g.Y + o0 + i) : 0.f;
+          }
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int i = b + u * kThreads + threadIdx.x;
+            if (i < total) {
+              const int r = i / g.n;
+              g.q_codes[o0 + i] = (int8_t)quantize_one(y[u], s_rq[r].k, s_rq[r].inv);
+            }
+          }
+        }
+        if (threadIdx.x < rt) g.rowmax[row0 + threadIdx.x] = 0u;
+        if (threadIdx.x == 0) *g.q_ticket = 0u;
+      }
+    }
   }
 }
 
@@ -264,6 +307,11 @@ int gemv_rows_per_launch(int rows, int K) { return rows_per_launch(rows, K); }
 cudaError_t launch_gemv(const GatherGemm& g_in, int sm_count, cudaStream_t st) {
   GatherGemm g = g_in;
   if (!g.ldy) g.ldy = g.n;
+  // the last-block quantization needs every row in one launch
+  if (g.q_ticket && (g.epilogue != EPI_CLOUD || !g.q_codes || !g.q_scale ||
+                     rows_per_launch(g.rows, g.K) < g.rows ||
+                     (int64_t)g.rows * g.n > kGemvQuantizeMax))
+    return cudaErrorNotSupported;
   if (g.epilogue == EPI_FUSED) {
     if (g.w_dtype != W_BF16 || !g.yc || !g.rowmax_in || !g.codes_out || !g.scale_out)
       return cudaErrorNotSupported;

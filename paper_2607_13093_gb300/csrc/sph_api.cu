@@ -42,6 +42,10 @@ struct sph_ctx {
   int tc_pair = 0;                  // SPH_OPT_TC_PAIR: 0 automatic, 1 always, 2 never
   int endpoint_z = 0;               // SPH_OPT_ENDPOINT_Z: 0 automatic, 1 store, 2 recompute
   int endpoint_rm = 0;              // SPH_OPT_ENDPOINT_ROWS_M: 0 automatic, 1 always, 2 never
+  int gemv_quantize = 0;            // SPH_OPT_GEMV_QUANTIZE: 0 automatic, 1 never
+  // the cloud GEMV's last-block quantization: row maxima [8] and the
+  // arrival ticket, zero between calls (the last block resets them)
+  unsigned* gemv_q = nullptr;
   int pair_units = 0;               // CTA pairs that fit at once (0: pairs unavailable)
   // chunked split steps: the endpoint's own stream (created on first use
   // when the caller passes none) and the events that order the two streams
@@ -549,6 +553,14 @@ sph_status sph_create(int device, void* cuda_stream, sph_ctx** out) {
     delete ctx;
     return SPH_ERR_CUDA;
   }
+  if (cudaMalloc(&ctx->gemv_q, 16 * sizeof(unsigned)) != cudaSuccess ||
+      cudaMemset(ctx->gemv_q, 0, 16 * sizeof(unsigned)) != cudaSuccess) {
+    cudaGetLastError();
+    if (ctx->gemv_q) cudaFree(ctx->gemv_q);
+    cudaFree(ctx->status);
+    delete ctx;
+    return SPH_ERR_OOM;
+  }
   *out = ctx;
   return SPH_OK;
 }
@@ -559,6 +571,7 @@ sph_status sph_destroy(sph_ctx* ctx) {
   cudaStreamSynchronize(ctx->stream);
   if (ctx->scratch) cudaFree(ctx->scratch);
   if (ctx->status) cudaFree(ctx->status);
+  if (ctx->gemv_q) cudaFree(ctx->gemv_q);
   if (ctx->aux_stream) cudaStreamDestroy(ctx->aux_stream);
   for (auto ev : ctx->step_events) cudaEventDestroy(ev);
   for (auto& p : ctx->pending) { cudaEventDestroy(p.start); cudaEventDestroy(p.stop); }
@@ -708,6 +721,10 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "check_ids must be 0 or 1");
       ctx->check_ids = (int)value;
       return SPH_OK;
+    case SPH_OPT_GEMV_QUANTIZE:
+      if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "gemv_quantize must be 0 or 1");
+      ctx->gemv_quantize = (int)value;
+      return SPH_OK;
   }
   return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
 }
@@ -781,7 +798,11 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
   Carve c(ctx->scratch, ctx->scratch_cap);
   float* Y = static_cast<float*>(c.take((size_t)rows * n_keep * 4));
   unsigned* rowmax = static_cast<unsigned*>(c.take((size_t)rows * 4));
-  if (!use_tc(ctx, rows, wdt)) {     // the tensor-core path clears them itself
+  // few rows and a small payload: the GEMV's last block quantizes (no
+  // separate pass, and its row maxima need no clearing)
+  const bool gemv_q = !use_tc(ctx, rows, wdt) && ctx->gemv_quantize == 0 && ctx->gemv_q &&
+                      sph::gemv_can_quantize(rows, n_keep, (int)d_h);
+  if (!use_tc(ctx, rows, wdt) && !gemv_q) {   // the tensor-core path clears them itself
     cudaError_t e = cudaMemsetAsync(rowmax, 0, (size_t)rows * 4, ctx->stream);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMemsetAsync");
   }
@@ -810,9 +831,16 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
                          return sph::launch_tc(gg, pl, tcs, ctx->spin_limit, ctx->stream);
                        }), "tensor-core launch");
   } else {
+    if (gemv_q) {
+      gg.rowmax = ctx->gemv_q;
+      gg.q_ticket = ctx->gemv_q + 8;
+      gg.q_codes = codes;
+      gg.q_scale = row_scale;
+    }
     st = launch_status(ctx, traced(ctx, SPH_PROF_CLOUD_GEMM, [&] {
                          return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
                        }), "gemv launch");
+    if (st || gemv_q) return st;
   }
   if (st) return st;
   return launch_status(ctx, traced(ctx, SPH_PROF_QUANTIZE, [&] {

@@ -105,6 +105,12 @@ struct GatherGemm {
   unsigned* status;        // device error word
   long long finish_wait = 1ll << 15;   // split-tile finisher poll (cycles; 0: none)
   bool no_stats = false;   // endpoint: skip the softmax statistics (Gumbel-max draw)
+  // cloud GEMV in one launch: the last block to arrive (q_ticket, which it
+  // resets) quantizes every row (Eq. 18) into q_codes / q_scale and clears
+  // the row maxima for the next call; nullptr: the quantize pass does it
+  unsigned* q_ticket = nullptr;
+  int8_t* q_codes = nullptr;
+  float* q_scale = nullptr;
 };
 
 // CUDA-core gathered GEMV (few rows); returns a cudaError_t.
@@ -113,6 +119,15 @@ cudaError_t launch_gemv(const GatherGemm& g, int sm_count, cudaStream_t st);
 int gemv_max_k();
 // Hidden-state rows one GEMV launch covers (1, 2, 4 or 8).
 int gemv_rows_per_launch(int rows, int K);
+// Most rows x kept ids the cloud GEMV quantizes in its last block (two
+// batches of eight loads a thread; measured: at 25,600 entries the one
+// block took longer than a separate quantize pass over the whole grid)
+constexpr int64_t kGemvQuantizeMax = 1 << 12;
+// Whether the cloud GEMV can quantize in its last block (one launch covers
+// the rows, at most kGemvQuantizeMax entries).
+inline bool gemv_can_quantize(int64_t rows, int64_t n, int K) {
+  return gemv_rows_per_launch((int)rows, K) >= rows && rows * n <= kGemvQuantizeMax;
+}
 
 // Tensor-core path (k_tc.cu): sizes, work split and scratch of one call.
 struct TcPlan {

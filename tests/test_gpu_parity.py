@@ -164,6 +164,44 @@ def test_outputs_stay_inside_their_buffers(path_ctx, w_dtype, n_keep):
         assert guards_intact(buf), name
 
 
+GEMV_Q = [
+    # rows, n_keep, d, w_dtype, act, bias
+    (1, 2048, 512, "bf16", "fp32", False),     # the tiny workload's shape
+    (2, 2000, 1032, "bf16", "bf16", True),
+    (4, 700, 296, "fp8", "fp32", False),
+    (8, 512, 776, "bf16", "fp32", False),      # 2^12 entries, the most it takes
+    (1, 4001, 520, "bf16", "fp32", False),     # a ragged last batch
+]
+
+
+@pytest.mark.parametrize("rows,n_keep,d,w_dtype,act,bias", GEMV_Q,
+                         ids=[f"{c[0]}x{c[1]}-{c[3]}-{c[4]}" for c in GEMV_Q])
+def test_gemv_last_block_quantize(ctx, rows, n_keep, d, w_dtype, act, bias):
+    """The cloud GEMV whose last block quantizes the payload itself: codes,
+    scales and partials bit-identical to the separate quantize pass and
+    within the parity bar of the oracle; calls in a row (different inputs,
+    then the first again) find the row maxima and the arrival count cleared."""
+    from paper_2607_13093_gb300 import sph
+    ws = [small(V=5 * n_keep, d=d, d_l=8, rows=rows, n_keep=n_keep, w_dtype=w_dtype,
+                clip=40.0 if w_dtype == "fp8" else 30.0, with_bias=bias, seed=s)
+          for s in (701, 702)]
+    ws[1].h[rows - 1].zero_()                    # an all-zero row (scale 0)
+    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1 << 40)
+    try:
+        got = {}
+        for mode in (1, 0):                       # separate pass, then the last block
+            ctx.set_option(sph.SPH_OPT_GEMV_QUANTIZE, mode)
+            for i in (0, 1, 0):
+                codes, scale, part = check_cloud(ctx, ws[i], act_mode=act)
+                got.setdefault((mode, i), (np_(codes), np_(scale), np_(part)))
+        for i in (0, 1):
+            for a, b in zip(got[(0, i)], got[(1, i)]):
+                assert np.array_equal(a.view(np.uint8), b.view(np.uint8))
+    finally:
+        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
+        ctx.set_option(sph.SPH_OPT_GEMV_QUANTIZE, 0)
+
+
 def test_cloud_odd_hidden_width_and_strides(path_ctx):
     ctx = path_ctx
     # d_h = 37 (not a multiple of anything) inside a padded weight stride
