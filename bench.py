@@ -311,12 +311,13 @@ KERNEL_FILES = ["paper_2607_13093_gb300/csrc/k_tc.cu", "paper_2607_13093_gb300/c
 
 def traffic_for(kernel_key, files=KERNEL_FILES):
     """DRAM bytes per launch from a committed ncu summary, if it was taken
-    on the current source of that kernel."""
+    on the current source of the kernels that call launches (the record's
+    own list of source files, else `files`)."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(p) as f:
             d = json.load(f).get(kernel_key)
-        if d and d.get("source_hash") == source_hash(files):
+        if d and d.get("source_hash") == source_hash(d.get("source_files") or files):
             return d.get("bytes_per_launch")
     except Exception:
         pass
