@@ -84,3 +84,33 @@ def test_reference_arm_under_torchrun_prints_once_from_rank_zero():
     for key in ("metric", "unit", "steps", "warmup", "ms_per_step", "higher_is_better",
                 "config", "dtype"):
         assert key in out
+
+
+def test_traffic_record_follows_its_own_sources(tmp_path, monkeypatch):
+    # a committed DRAM-traffic record counts while the kernel sources it
+    # lists hash as they did when it was taken, and is dropped once one of
+    # them changes (a file the call does not launch does not matter)
+    import json
+    import bench
+    src = tmp_path / "k.cu"
+    other = tmp_path / "other.cu"
+    src.write_text("kernel v1\n")
+    other.write_text("unrelated v1\n")
+    (tmp_path / "profiles").mkdir()
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    rec = {"call": {"bytes_per_launch": 1234, "source_files": ["k.cu"],
+                    "source_hash": bench.source_hash(["k.cu"])}}
+    (tmp_path / "profiles" / "traffic.json").write_text(json.dumps(rec))
+    assert bench.traffic_for("call", files=["k.cu", "other.cu"]) == 1234
+    other.write_text("unrelated v2\n")
+    assert bench.traffic_for("call", files=["k.cu", "other.cu"]) == 1234
+    src.write_text("kernel v2\n")
+    assert bench.traffic_for("call") is None
+    assert bench.traffic_for("absent") is None
+
+
+def test_block_grids_extend_the_configuration_block():
+    import bench
+    assert len(bench.DEND_GRID) == 10 and len(bench.SWEEP_GRID) == 10
+    assert {k for _, k in bench.SWEEP_GRID} == {0.1, 0.5}
+    assert {r for r, _ in bench.SWEEP_GRID} == {1, 8, 64, 256, 1024}
