@@ -394,7 +394,7 @@ OPTION_NAMES = {"tc_min_rows": "SPH_OPT_TC_MIN_ROWS", "schedule": "SPH_OPT_TC_SC
                 "max_bn": "SPH_OPT_TC_MAX_BN", "tile_m": "SPH_OPT_TC_TILE_M",
                 "finish_wait": "SPH_OPT_TC_FINISH_WAIT", "split_quantize": "SPH_OPT_SPLIT_QUANTIZE",
                 "pair": "SPH_OPT_TC_PAIR", "endpoint_z": "SPH_OPT_ENDPOINT_Z",
-                "rows_m": "SPH_OPT_ENDPOINT_ROWS_M", "gemv_last_block": "SPH_OPT_GEMV_LAST_BLOCK"}
+                "rows_m": "SPH_OPT_ENDPOINT_ROWS_M", "gemv_quantize": "SPH_OPT_GEMV_QUANTIZE"}
 
 
 class Runner:

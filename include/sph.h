@@ -187,17 +187,15 @@ typedef enum sph_option {
                                differ from the stored path's only where a
                                draw lies within fp32 rounding of a CDF step
                                (or greedy ties within it).                 */
-  SPH_OPT_GEMV_LAST_BLOCK = 14, /* the CUDA-core GEMV (fewer rows than
-                               SPH_OPT_TC_MIN_ROWS) where one launch covers
-                               every row and rows x n_keep is at most 2^12:
-                               0 (default) its last block to finish finishes
-                               the call -- sph_partial_logits: it quantizes
-                               the payload (the row maxima live in a small
-                               buffer of the context that the call leaves
-                               cleared); sph_fuse_sample: it makes the
-                               segment softmax statistics -- so that no
-                               separate pass runs; 1 always the separate
-                               passes.  Bit-identical results.             */
+  SPH_OPT_GEMV_QUANTIZE = 14, /* sph_partial_logits on the CUDA-core GEMV
+                               (fewer rows than SPH_OPT_TC_MIN_ROWS) where
+                               one launch covers every row and rows x n_keep
+                               is at most 2^12: 0 (default) the GEMV's last
+                               block to finish quantizes the payload itself
+                               (no separate pass; the row maxima live in a
+                               small buffer of the context that the call
+                               leaves cleared); 1 always a separate quantize
+                               pass.  Bit-identical codes and scales.      */
   SPH_OPT_SAMPLER = 8       /* the draw of sph_fuse_sample at temperature > 0:
                                0 inverse CDF (default), 1 Gumbel-max: the
                                first index j of the largest

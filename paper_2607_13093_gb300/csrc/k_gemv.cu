@@ -233,31 +233,6 @@ gemv_kernel(const GatherGemm g, const int row0) {
       }
     }
   }
-  if constexpr (EPI == EPI_ENDPOINT) {
-    if (g.q_ticket) {
-      // the last block to arrive makes every row's segment statistics from
-      // the stored z (seg_stat32, as the statistics pass) and leaves its
-      // ticket at zero
-      __shared__ int s_last_e;
-      __threadfence();
-      __syncthreads();
-      if (threadIdx.x == 0) s_last_e = atomicAdd(g.q_ticket, 1u) == gridDim.x - 1;
-      __syncthreads();
-      if (s_last_e) {
-        __threadfence();
-        const int nseg = g.q_nseg, total = rt * nseg;
-        for (int i = threadIdx.x; i < total; i += kThreads) {
-          const int r = i / nseg, sg = i - r * nseg, j0 = sg * 32;
-          const float* z = g.Y + (int64_t)(row0 + r) * g.ldy + j0;
-          float v[32];
-#pragma unroll
-          for (int e = 0; e < 32; ++e) v[e] = j0 + e < g.n ? __ldcg(z + e) : -INFINITY;
-          g.q_stats[(int64_t)(row0 + r) * nseg + sg] = seg_stat32(v, g.q_l2t);
-        }
-        if (threadIdx.x == 0) *g.q_ticket = 0u;
-      }
-    }
-  }
 }
 
 template <int RT, int WDT, int EPI>
@@ -332,12 +307,10 @@ int gemv_rows_per_launch(int rows, int K) { return rows_per_launch(rows, K); }
 cudaError_t launch_gemv(const GatherGemm& g_in, int sm_count, cudaStream_t st) {
   GatherGemm g = g_in;
   if (!g.ldy) g.ldy = g.n;
-  // the last block's work needs every row in one launch
-  if (g.q_ticket && (rows_per_launch(g.rows, g.K) < g.rows ||
-                     (int64_t)g.rows * g.n > kGemvQuantizeMax ||
-                     (g.epilogue == EPI_CLOUD && (!g.q_codes || !g.q_scale)) ||
-                     (g.epilogue == EPI_ENDPOINT && (!g.q_stats || g.q_nseg * 32 < g.n)) ||
-                     (g.epilogue != EPI_CLOUD && g.epilogue != EPI_ENDPOINT)))
+  // the last-block quantization needs every row in one launch
+  if (g.q_ticket && (g.epilogue != EPI_CLOUD || !g.q_codes || !g.q_scale ||
+                     rows_per_launch(g.rows, g.K) < g.rows ||
+                     (int64_t)g.rows * g.n > kGemvQuantizeMax))
     return cudaErrorNotSupported;
   if (g.epilogue == EPI_FUSED) {
     if (g.w_dtype != W_BF16 || !g.yc || !g.rowmax_in || !g.codes_out || !g.scale_out)

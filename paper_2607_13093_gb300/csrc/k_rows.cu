@@ -103,10 +103,27 @@ seg_stats_kernel(const float* __restrict__ Z, int rows, int n, int nseg, int nch
       v[4 * m] = t.x; v[4 * m + 1] = t.y; v[4 * m + 2] = t.z; v[4 * m + 3] = t.w;
     }
     const int sg = c * kSeg + lane;             // this lane's segment
-    static_assert(kSeg == 32, "a segment is 32 ids");
-    const float2 st = seg_stat32(v, l2t);       // (exp of -inf, ids past n, is 0)
-    const float m = st.x, sum = st.y;
-    if (sg < nseg) stats[r * nseg + sg] = st;
+    float t[kSeg / 2];
+#pragma unroll
+    for (int q = 0; q < kSeg / 2; ++q) t[q] = fmaxf(v[2 * q], v[2 * q + 1]);
+#pragma unroll
+    for (int w = kSeg / 4; w >= 1; w >>= 1)
+#pragma unroll
+      for (int q = 0; q < w; ++q) t[q] = fmaxf(t[2 * q], t[2 * q + 1]);
+    const float m = t[0];
+    float sum = 0.f;
+    if (m > -INFINITY) {
+      // exp of -inf (ids past n) is 0
+#pragma unroll
+      for (int q = 0; q < kSeg / 2; ++q)
+        t[q] = exp_tau(v[2 * q] - m, l2t) + exp_tau(v[2 * q + 1] - m, l2t);
+#pragma unroll
+      for (int w = kSeg / 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int q = 0; q < w; ++q) t[q] = t[2 * q] + t[2 * q + 1];
+      sum = t[0];
+    }
+    if (sg < nseg) stats[r * nseg + sg] = make_float2(m, sum);
     const float Mc = warp_max(m);
     const float Sc = warp_sum(seg_weight(make_float2(m, sum), Mc, inv_tau));
     if (lane == 0) cstats[r * nchunk + c] = make_float2(Mc, Sc);

@@ -42,10 +42,9 @@ struct sph_ctx {
   int tc_pair = 0;                  // SPH_OPT_TC_PAIR: 0 automatic, 1 always, 2 never
   int endpoint_z = 0;               // SPH_OPT_ENDPOINT_Z: 0 automatic, 1 store, 2 recompute
   int endpoint_rm = 0;              // SPH_OPT_ENDPOINT_ROWS_M: 0 automatic, 1 always, 2 never
-  int gemv_last_block = 0;          // SPH_OPT_GEMV_LAST_BLOCK: 0 automatic, 1 never
-  // the GEMVs' last-block work: the cloud's row maxima [8] and arrival
-  // ticket [8], the endpoint's ticket [9]; zero between calls (the last
-  // block resets them)
+  int gemv_quantize = 0;            // SPH_OPT_GEMV_QUANTIZE: 0 automatic, 1 never
+  // the cloud GEMV's last-block quantization: row maxima [8] and the
+  // arrival ticket, zero between calls (the last block resets them)
   unsigned* gemv_q = nullptr;
   int pair_units = 0;               // CTA pairs that fit at once (0: pairs unavailable)
   // chunked split steps: the endpoint's own stream (created on first use
@@ -414,35 +413,11 @@ sph_status endpoint_draw(sph_ctx* ctx, sph::GatherGemm& gg, Carve& c, float temp
   if (!c.fits())
     return fail(ctx, SPH_ERR_UNSUPPORTED, "internal: scratch plan of %zu bytes exceeds the arena of %zu",
                 c.off, ctx->scratch_cap);
-  // few rows and ids: the GEMV's last block makes the segment statistics
-  // (no statistics pass; the draw makes the chunk statistics itself)
-  const bool gemv_stats = !fuse_only && !gumbel && gg.epilogue == sph::EPI_ENDPOINT &&
-                          ctx->gemv_last_block == 0 && ctx->gemv_q &&
-                          sph::gemv_can_quantize(rows, n_keep, gg.K);
-  if (gemv_stats) {
-    gg.q_ticket = ctx->gemv_q + 9;
-    gg.q_stats = stats;
-    gg.q_nseg = sph::seg_count(n_keep);
-    gg.q_l2t = gg.inv_tau * 1.4426950408889634f;
-  }
   st = launch_status(ctx, traced(ctx, SPH_PROF_LOCAL_GEMM, [&] {
                        return sph::launch_gemv(gg, ctx->sm_count, ctx->stream);
                      }), "gemv launch");
   if (st || fuse_only) return st;
   if (gumbel) return draw_gumbel();
-  if (gemv_stats)
-    return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
-                           sph::ZSource zsg;
-                           zsg.Z = Z;
-                           const int nseg = sph::seg_count(n_keep);
-                           if (greedy)
-                             return sph::launch_sample_segments(zsg, rows, n_keep, stats, nseg,
-                                                                nullptr, keep_ids, gg.inv_tau,
-                                                                seed, offset, tokens, ctx->stream, 1);
-                           return sph::launch_sample_rows(zsg, rows, n_keep, stats, nseg, keep_ids,
-                                                          gg.inv_tau, seed, offset, tokens,
-                                                          ctx->stream);
-                         }), "sample launch");
   return launch_status(ctx, traced(ctx, SPH_PROF_SAMPLE, [&] {
                          cudaError_t e = sph::launch_seg_stats(Z, rows, n_keep,
                                                                gg.inv_tau, stats,
@@ -746,9 +721,9 @@ sph_status sph_set_option(sph_ctx* ctx, sph_option option, int64_t value) {
       if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "check_ids must be 0 or 1");
       ctx->check_ids = (int)value;
       return SPH_OK;
-    case SPH_OPT_GEMV_LAST_BLOCK:
-      if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "gemv_last_block must be 0 or 1");
-      ctx->gemv_last_block = (int)value;
+    case SPH_OPT_GEMV_QUANTIZE:
+      if (value != 0 && value != 1) return fail(ctx, SPH_ERR_INVALID_ARG, "gemv_quantize must be 0 or 1");
+      ctx->gemv_quantize = (int)value;
       return SPH_OK;
   }
   return fail(ctx, SPH_ERR_INVALID_ARG, "unknown option %d", (int)option);
@@ -825,7 +800,7 @@ sph_status sph_partial_logits(sph_ctx* ctx, const float* h_cloud, int64_t rows,
   unsigned* rowmax = static_cast<unsigned*>(c.take((size_t)rows * 4));
   // few rows and a small payload: the GEMV's last block quantizes (no
   // separate pass, and its row maxima need no clearing)
-  const bool gemv_q = !use_tc(ctx, rows, wdt) && ctx->gemv_last_block == 0 && ctx->gemv_q &&
+  const bool gemv_q = !use_tc(ctx, rows, wdt) && ctx->gemv_quantize == 0 && ctx->gemv_q &&
                       sph::gemv_can_quantize(rows, n_keep, (int)d_h);
   if (!use_tc(ctx, rows, wdt) && !gemv_q) {   // the tensor-core path clears them itself
     cudaError_t e = cudaMemsetAsync(rowmax, 0, (size_t)rows * 4, ctx->stream);

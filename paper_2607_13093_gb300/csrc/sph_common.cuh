@@ -171,34 +171,6 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
-// Softmax statistics of one 32-id segment: (max of v, sum of 2^((v - max) *
-// l2t)) with l2t = fl32(log2(e) / tau), both as balanced trees over the
-// segment's ids in order; ids past the row's end hold -inf (weight 0).  The
-// statistics pass and the GEMV's last block both use it, so they agree bit
-// for bit.
-__device__ __forceinline__ float2 seg_stat32(const float (&v)[32], float l2t) {
-  float t[16];
-#pragma unroll
-  for (int q = 0; q < 16; ++q) t[q] = fmaxf(v[2 * q], v[2 * q + 1]);
-#pragma unroll
-  for (int w = 8; w >= 1; w >>= 1)
-#pragma unroll
-    for (int q = 0; q < w; ++q) t[q] = fmaxf(t[2 * q], t[2 * q + 1]);
-  const float m = t[0];
-  float sum = 0.f;
-  if (m > -INFINITY) {
-#pragma unroll
-    for (int q = 0; q < 16; ++q)
-      t[q] = ex2_approx((v[2 * q] - m) * l2t) + ex2_approx((v[2 * q + 1] - m) * l2t);
-#pragma unroll
-    for (int w = 8; w >= 1; w >>= 1)
-#pragma unroll
-      for (int q = 0; q < w; ++q) t[q] = t[2 * q] + t[2 * q + 1];
-    sum = t[0];
-  }
-  return make_float2(m, sum);
-}
-
 // The int8 code in byte e (0..3) of a word whose bytes were first XORed with
 // 0x80, as an exact float: the byte permute forms the fp32 2^23 + (code +
 // 128), and one exact subtraction leaves the code.  (Integer and ALU pipes

@@ -111,12 +111,6 @@ struct GatherGemm {
   unsigned* q_ticket = nullptr;
   int8_t* q_codes = nullptr;
   float* q_scale = nullptr;
-  // endpoint GEMV in one launch: the last block to arrive (q_ticket) makes
-  // the 32-id segment statistics of every row into q_stats [rows][q_nseg]
-  // with q_l2t = fl32(log2(e) / tau), as the statistics pass would
-  float2* q_stats = nullptr;
-  int q_nseg = 0;
-  float q_l2t = 0.f;
 };
 
 // CUDA-core gathered GEMV (few rows); returns a cudaError_t.
@@ -129,9 +123,8 @@ int gemv_rows_per_launch(int rows, int K);
 // batches of eight loads a thread; measured: at 25,600 entries the one
 // block took longer than a separate quantize pass over the whole grid)
 constexpr int64_t kGemvQuantizeMax = 1 << 12;
-// Whether a GEMV's last block can finish the call (quantize the cloud's
-// payload, or make the endpoint's segment statistics): one launch covers the
-// rows, at most kGemvQuantizeMax entries.
+// Whether the cloud GEMV can quantize in its last block (one launch covers
+// the rows, at most kGemvQuantizeMax entries).
 inline bool gemv_can_quantize(int64_t rows, int64_t n, int K) {
   return gemv_rows_per_launch((int)rows, K) >= rows && rows * n <= kGemvQuantizeMax;
 }

@@ -35,7 +35,7 @@ SPH_OPT_SPLIT_QUANTIZE = 10
 SPH_OPT_TC_PAIR = 11
 SPH_OPT_ENDPOINT_Z = 12
 SPH_OPT_ENDPOINT_ROWS_M = 13
-SPH_OPT_GEMV_LAST_BLOCK = 14
+SPH_OPT_GEMV_QUANTIZE = 14
 SPH_SAMPLER_CDF, SPH_SAMPLER_GUMBEL = 0, 1
 
 _c_void_p = ctypes.c_void_p

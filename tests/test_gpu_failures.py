@@ -118,7 +118,7 @@ def test_bad_arguments_are_rejected_before_any_launch(ctx):
         "sampler 2": lambda: ctx.set_option(sph.SPH_OPT_SAMPLER, 2),
         "spin limit 0": lambda: ctx.set_option(sph.SPH_OPT_SPIN_LIMIT, 0),
         "unknown option": lambda: ctx.set_option(99, 0),
-        "gemv_last_block 2": lambda: ctx.set_option(sph.SPH_OPT_GEMV_LAST_BLOCK, 2),
+        "gemv_quantize 2": lambda: ctx.set_option(sph.SPH_OPT_GEMV_QUANTIZE, 2),
     }
     for name, call in cases.items():
         with pytest.raises(sph.SphError) as err:

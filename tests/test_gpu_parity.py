@@ -190,7 +190,7 @@ def test_gemv_last_block_quantize(ctx, rows, n_keep, d, w_dtype, act, bias):
     try:
         got = {}
         for mode in (1, 0):                       # separate pass, then the last block
-            ctx.set_option(sph.SPH_OPT_GEMV_LAST_BLOCK, mode)
+            ctx.set_option(sph.SPH_OPT_GEMV_QUANTIZE, mode)
             for i in (0, 1, 0):
                 codes, scale, part = check_cloud(ctx, ws[i], act_mode=act)
                 got.setdefault((mode, i), (np_(codes), np_(scale), np_(part)))
@@ -199,45 +199,7 @@ def test_gemv_last_block_quantize(ctx, rows, n_keep, d, w_dtype, act, bias):
                 assert np.array_equal(a.view(np.uint8), b.view(np.uint8))
     finally:
         ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
-        ctx.set_option(sph.SPH_OPT_GEMV_LAST_BLOCK, 0)
-
-
-GEMV_STATS = [
-    # rows, n_keep, d_l, tau
-    (1, 2048, 64, 1.0),          # the tiny workload's endpoint
-    (2, 2000, 200, 0.8),
-    (4, 1000, 72, 0.0),          # greedy: the segment maxima alone
-    (8, 512, 40, 3.0),           # 2^12 entries
-    (3, 900, 64, 1.0),           # two launches: the statistics pass runs
-]
-
-
-@pytest.mark.parametrize("rows,n_keep,d_l,tau", GEMV_STATS,
-                         ids=[f"{c[0]}x{c[1]}-tau{c[3]}" for c in GEMV_STATS])
-def test_gemv_last_block_statistics(ctx, rows, n_keep, d_l, tau):
-    """The endpoint GEMV whose last block makes the segment statistics: z bit-
-    identical to the form with the statistics pass, tokens of both forms
-    against the oracle (margin rule), calls in a row with other inputs."""
-    from paper_2607_13093_gb300 import sph
-    ws = [small(V=4 * n_keep, d=d_l + 64, d_l=d_l, rows=rows, n_keep=n_keep, tau=tau, seed=s)
-          for s in (811, 812)]
-    ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 1 << 40)
-    try:
-        zs = {}
-        for mode in (1, 0):
-            ctx.set_option(sph.SPH_OPT_GEMV_LAST_BLOCK, mode)
-            for i in (0, 1, 0):
-                w = ws[i]
-                ref = oracle_cloud(w)
-                w.offset = 3 + i
-                _, z = check_endpoint(ctx, w, torch.from_numpy(ref["codes"]),
-                                      torch.from_numpy(ref["row_scale"]), unstored=False)
-                zs.setdefault((mode, i), z.clone())
-        for i in (0, 1):
-            assert torch.equal(zs[(0, i)].view(torch.int32), zs[(1, i)].view(torch.int32))
-    finally:
-        ctx.set_option(sph.SPH_OPT_TC_MIN_ROWS, 4)
-        ctx.set_option(sph.SPH_OPT_GEMV_LAST_BLOCK, 0)
+        ctx.set_option(sph.SPH_OPT_GEMV_QUANTIZE, 0)
 
 
 def test_cloud_odd_hidden_width_and_strides(path_ctx):
