@@ -411,7 +411,11 @@ FULL = [("tiny", None, None, "fp32"), ("decode", None, None, "fp32"),
         ("fp8", None, None, "bf16"), ("sweep", 1, 0.1, "fp32"),
         ("sweep", 8, 1.0, "fp32"), ("sweep", 64, 0.5, "fp32"),
         ("sweep", 256, 1.0, "fp32"), ("sweep", 1024, 1.0, "fp32"),
-        ("sweep", 1024, 1.0, "bf16")]
+        ("sweep", 1024, 1.0, "bf16"),
+        # the kept-fraction grid of the benchmark (--sweep-grid)
+        ("sweep", 8, 0.1, "fp32"), ("sweep", 64, 0.1, "fp32"),
+        ("sweep", 256, 0.5, "fp32"), ("sweep", 1024, 0.1, "fp32"),
+        ("sweep", 1024, 0.5, "fp32")]
 
 
 def rows_to_check(ctx, w, act, want=16):
