@@ -77,7 +77,11 @@ sph_status sph_create(int device, void* cuda_stream, sph_ctx** out);
 /* Release the context and its scratch (waits for its stream first). */
 sph_status sph_destroy(sph_ctx* ctx);
 
-/* Issue subsequent calls on another stream of the same device. */
+/* Issue subsequent calls on another stream of the same device.  The new
+ * stream is made to wait (an event, no host synchronization) for the work
+ * already issued on the old one, since the next call reuses the context's
+ * scratch.  While either stream is being captured into a CUDA graph no
+ * ordering is added: the caller orders the two streams itself. */
 sph_status sph_set_stream(sph_ctx* ctx, void* cuda_stream);
 
 /* Wait for all work of the context's stream; report device-side errors

@@ -51,6 +51,8 @@ struct sph_ctx {
   // when the caller passes none) and the events that order the two streams
   cudaStream_t aux_stream = nullptr;
   std::vector<cudaEvent_t> step_events;
+  // sph_set_stream: orders the new stream after the old one's work
+  cudaEvent_t switch_event = nullptr;
   // tracing
   bool prof = false;
   long long prof_launch0 = 0;
@@ -574,6 +576,7 @@ sph_status sph_destroy(sph_ctx* ctx) {
   if (ctx->gemv_q) cudaFree(ctx->gemv_q);
   if (ctx->aux_stream) cudaStreamDestroy(ctx->aux_stream);
   for (auto ev : ctx->step_events) cudaEventDestroy(ev);
+  if (ctx->switch_event) cudaEventDestroy(ctx->switch_event);
   for (auto& p : ctx->pending) { cudaEventDestroy(p.start); cudaEventDestroy(p.stop); }
   for (auto ev : ctx->pool) cudaEventDestroy(ev);
   delete ctx;
@@ -615,7 +618,31 @@ sph_status sph_profile_read(sph_ctx* ctx, sph_profile* out) {
 
 sph_status sph_set_stream(sph_ctx* ctx, void* cuda_stream) {
   if (!ctx) return SPH_ERR_INVALID_ARG;
-  ctx->stream = static_cast<cudaStream_t>(cuda_stream);
+  cudaStream_t next = static_cast<cudaStream_t>(cuda_stream);
+  if (next == ctx->stream) return SPH_OK;
+  DeviceGuard g(ctx->device);
+  // Calls already issued on the old stream may still be using the scratch
+  // (partials, row maxima, arrival counters) that the next call reuses, so
+  // the new stream waits for them.  Not while either stream is being
+  // captured: a capturing stream cannot wait on uncaptured work, and
+  // recording on a stream outside a capture can invalidate it.  The new
+  // stream is asked first, so that during a capture the old (possibly the
+  // legacy default) stream is not touched at all.
+  cudaStreamCaptureStatus cn = cudaStreamCaptureStatusNone, co = cudaStreamCaptureStatusNone;
+  cudaError_t q = cudaStreamIsCapturing(next, &cn);
+  if (q == cudaSuccess && cn == cudaStreamCaptureStatusNone)
+    q = cudaStreamIsCapturing(ctx->stream, &co);
+  if (q != cudaSuccess) cudaGetLastError();   // a refused query is not the caller's error
+  if (q == cudaSuccess && cn == cudaStreamCaptureStatusNone &&
+      co == cudaStreamCaptureStatusNone) {
+    cudaError_t e = cudaSuccess;
+    if (!ctx->switch_event)
+      e = cudaEventCreateWithFlags(&ctx->switch_event, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventRecord(ctx->switch_event, ctx->stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(next, ctx->switch_event, 0);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "ordering the new stream after the old one");
+  }
+  ctx->stream = next;
   return SPH_OK;
 }
 
