@@ -309,6 +309,12 @@ KERNEL_FILES = ["paper_2607_13093_gb300/csrc/k_tc.cu", "paper_2607_13093_gb300/c
                 "paper_2607_13093_gb300/csrc/k_finish.cu"]
 
 
+def traffic_key(name, rows, n_keep, act):
+    """Key of a cloud call's record in profiles/traffic.json: the workload,
+    its rows and kept ids, and the activation mode."""
+    return f"cloud_{name}_{rows}_{n_keep}_{act}"
+
+
 def traffic_for(kernel_key, files=KERNEL_FILES):
     """DRAM bytes per launch from a committed ncu summary, if it was taken
     on the current source of the kernels that call launches (the record's
@@ -717,6 +723,8 @@ def config_entry(sph, wl, dev, name, rows, keep, d_l, act, peaks, cpu_seconds,
         res = timed_run(r, steps, 3, bracket=False, min_pairs=64)
         unit = unit_stats(res["unit"])
         roof = roofline(w, act, unit["mean_ms"], peaks, mode)
+        roof["traffic"] = (traffic_for(traffic_key(name, w.rows, w.n_keep, act))
+                           if mode == "split" else None)
         roof["timing"] = res["timing"]
         roof["spread"] = unit
         one_call = mode in ("fused", "chunked", "chunked_serial")
@@ -823,7 +831,7 @@ def run_ours(args):
               "chunked": f"the one-call split step, {r.nchunk} payload chunks on two streams",
               "chunked_serial": (f"the one-call split step, {r.nchunk} payload chunks one "
                                  "after another on one stream")}
-    roof.update({"traffic": traffic_for(f"cloud_{args.workload}_{R}_{n}_{args.act}")
+    roof.update({"traffic": traffic_for(traffic_key(args.workload, R, n, args.act))
                  if args.step == "split" else None,
                  "kernel": kernel[args.step],
                  "timing": res["timing"], "spread": unit,

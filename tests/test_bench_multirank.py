@@ -109,6 +109,31 @@ def test_traffic_record_follows_its_own_sources(tmp_path, monkeypatch):
     assert bench.traffic_for("absent") is None
 
 
+def test_every_traffic_record_is_one_the_bench_looks_up():
+    # a record in profiles/traffic.json counts only under the key that the
+    # default line (the sweep at 1024 rows over the full vocabulary) or a
+    # two-call entry of its configuration block builds for its own call
+    import json
+    import os
+    import bench
+    from paper_2607_13093_gb300 import workloads as wl
+
+    def key(name, rows, keep, act):
+        cfg = wl.WORKLOADS[name]
+        n = cfg["n_keep"] if keep is None else round(keep * cfg["V"])
+        return bench.traffic_key(name, rows or cfg["rows"], n, act)
+
+    built = {key("sweep", 1024, 1.0, "fp32")}
+    built |= {key(name, rows, keep, act)
+              for name, rows, keep, d_l, act, mode, chunk in bench.CONFIG_BLOCK
+              if mode == "split" and d_l is None}
+    with open(os.path.join(bench.ROOT, "profiles", "traffic.json")) as f:
+        records = json.load(f)
+    assert records and set(records) <= built, set(records) - built
+    assert "cloud_decode_32_12000_fp32" in records
+    assert "cloud_sweep_1024_256000_fp32" in records
+
+
 def test_block_grids_extend_the_configuration_block():
     import bench
     assert len(bench.DEND_GRID) == 10 and len(bench.SWEEP_GRID) == 10

@@ -2,9 +2,11 @@
 flops it credits per launch, which roof bounds each workload, which peak a
 fraction is taken against (the measured copy bandwidth, the measured bf16
 burst rate, twice that for e4m3 x e4m3 on the f8f6f4 pipe) and the issued
-fraction beside the algorithmic one (hi/lo planes for fp32 activations).
-The expected figures are built from their physical terms, not from the
-benchmark's own expressions."""
+fraction beside the algorithmic one (hi/lo planes for fp32 activations);
+and one entry of the configuration block assembled around fake timings,
+with the committed DRAM traffic of its call.  The expected figures are
+built from their physical terms, not from the benchmark's own
+expressions."""
 from types import SimpleNamespace
 
 import pytest
@@ -97,3 +99,44 @@ def test_unsplit_head_reads_the_whole_hidden_state():
     assert r["algorithmic_bytes"] == 12000 * 4096 * 2 + 32 * 4096 * 4 + 12000 * 4 + 32 * 4
     assert r["algorithmic_flops"] == 2 * 32 * 12000 * 4096
     assert r["tensor"]["planes"] == 1 and r["tensor"]["issued_frac"] is None
+
+
+class _FakeRunner:
+    """Stands in for the GPU step: config_entry's host logic only."""
+    gsteps = 16
+
+    def __init__(self, sph, wl, w, dev, act="fp32", mode="split", chunk=0, **kw):
+        self.nchunk = 1 if not chunk else -(-w.n_keep // chunk)
+
+    def step(self, i, events=None):
+        pass
+
+    def close(self):
+        pass
+
+
+@pytest.mark.parametrize("mode,has_traffic", [("split", True), ("fused", False)])
+def test_configuration_entry_carries_the_committed_traffic(monkeypatch, mode, has_traffic):
+    # the decode entry of the block reports the DRAM bytes of its cloud call
+    # from the committed record (the two-call step only); the GPU pieces are
+    # replaced by fakes that return fixed timings
+    import torch
+    from paper_2607_13093_gb300 import workloads as wl
+    monkeypatch.setattr(bench, "Runner", _FakeRunner)
+    monkeypatch.setattr(bench, "timed_run", lambda r, steps, warmup, **kw: dict(
+        ms=steps * 0.05, unit=[0.03938] * 64, timing="fake", launches_per_step=6.0))
+    monkeypatch.setattr(bench, "e2e_run", lambda r, steps: {
+        "value": 1.0, "direct_calls": {"value": 0.5}})
+    monkeypatch.setattr(torch.cuda, "synchronize", lambda *a, **k: None)
+    monkeypatch.setattr(torch.cuda, "empty_cache", lambda: None)
+    e = bench.config_entry(None, wl, torch.device("cpu"), "decode", None, None, None, "fp32",
+                           PEAKS, 0.0, with_cpu=False, mode=mode)
+    assert e["workload"].startswith("decode: d=4096 (d_l=256, d_h=3840), V=32000, R=32")
+    assert e["payload_bytes_per_step"] == 32 * 12000 + 4 * 32
+    if has_traffic:
+        assert e["roofline"]["traffic"] == 95_321_216
+        assert e["roofline"]["frac"] == pytest.approx(0.3533, abs=1e-4)
+        assert e["cloud_us"] == pytest.approx(39.38)
+    else:
+        assert e["roofline"]["traffic"] is None and "step_call_us" in e
+    assert e["e2e_rows_per_s"] == 1.0 and e["e2e_direct_rows_per_s"] == 0.5
