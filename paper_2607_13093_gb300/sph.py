@@ -158,6 +158,24 @@ def _need(t, dtype, name):
         raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
 
 
+def _dense(dev, *specs):
+    """Buffers the kernels index densely, (tensor, name, elements) each:
+    every one given must be on `dev`, contiguous, and hold at least that
+    many elements, so that no read or write of the call leaves it.  A count
+    of None checks the device alone (operands with a row stride)."""
+    for t, name, count in specs:
+        if t is None:
+            continue
+        if t.device != dev:
+            raise ValueError(f"{name} is on {t.device}, not on {dev}")
+        if count is None:
+            continue
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous")
+        if t.numel() < count:
+            raise ValueError(f"{name} holds {t.numel()} elements; the call needs {count}")
+
+
 # ---------------------------------------------------------------------------
 # C functions with torch arguments
 # ---------------------------------------------------------------------------
@@ -274,6 +292,9 @@ def sph_partial_logits(ctx, h_cloud, W_h, *, keep_ids=None, clip=30.0,
     _need(codes, torch.int8, "codes")
     _need(row_scale, torch.float32, "row_scale")
     _need(partial_out, torch.float32, "partial_out")
+    _dense(dev, (W_h, "W_h", None), (keep_ids, "keep_ids", n), (w_row_scale, "w_row_scale", V),
+           (bias, "bias", V), (codes, "codes", R * n), (row_scale, "row_scale", R),
+           (partial_out, "partial_out", R * n))
     pb = _sz(0)
     _check(ctx, lib.sph_partial_logits(
         ctx, _ptr(h_cloud), R, _ld(h_cloud), _ptr(W_h), wdt, V, d_h, _ld(W_h),
@@ -362,6 +383,9 @@ def sph_fuse_sample(ctx, codes, row_scale, h_local, W_l, *, keep_ids=None,
     elif tokens is None:
         tokens = torch.empty(R, dtype=torch.int32, device=h_local.device)
     _need(tokens, torch.int32, "tokens")
+    _dense(h_local.device, (W_l, "W_l", None), (keep_ids, "keep_ids", n),
+           (codes, "codes", R * n), (row_scale, "row_scale", R), (tokens, "tokens", R),
+           (fused_logits_out, "fused_logits_out", R * n))
     _check(ctx, lib.sph_fuse_sample(
         ctx, _ptr(codes), _ptr(row_scale), R, _ptr(h_local), _ld(h_local),
         _ptr(W_l), V, d_l, _ld(W_l), _ptr(keep_ids), n, float(temperature),
@@ -406,11 +430,13 @@ def sph_split_step(ctx, h, d_l: int, W_h, W_l, *, keep_ids=None, clip=30.0,
     _need(scales, torch.float32, "scales")
     _need(tokens, torch.int32, "tokens")
     _need(fused_logits_out, torch.float32, "fused_logits_out")
-    if codes.numel() < R * n or scales.numel() < nchunk * R or tokens.numel() < R:
-        raise ValueError("codes, scales or tokens too small")
+    _dense(dev, (W_h, "W_h", None), (W_l, "W_l", None), (keep_ids, "keep_ids", n),
+           (w_row_scale, "w_row_scale", V), (bias, "bias", V), (codes, "codes", R * n),
+           (scales, "scales", nchunk * R), (tokens, "tokens", R))
     if fused_logits_out is not None and (tuple(fused_logits_out.shape) != (R, n)
                                          or not fused_logits_out.is_contiguous()):
         raise ValueError("fused_logits_out must be a contiguous (R, n) tensor")
+    _dense(dev, (fused_logits_out, "fused_logits_out", R * n))
     pb = _sz(0)
     _check(ctx, lib.sph_split_step(
         ctx, _ptr(h), R, _ld(h), int(d_l), d_h, _ptr(W_h), wdt, _ptr(w_row_scale),
@@ -436,6 +462,13 @@ def sph_verify_draft(ctx, target_logits, sessions: int, k: int, draft_tokens,
         n_accepted = torch.empty(sessions, dtype=torch.int32, device=dev)
     if next_token is None:
         next_token = torch.empty(sessions, dtype=torch.int32, device=dev)
+    _need(n_accepted, torch.int32, "n_accepted")
+    _need(next_token, torch.int32, "next_token")
+    S, K = max(int(sessions), 0), max(int(k), 0)
+    _dense(dev, (target_logits, "target_logits", S * (K + 1) * n),
+           (draft_tokens, "draft_tokens", S * K), (draft_probs, "draft_probs", S * K * n),
+           (keep_ids, "keep_ids", n), (n_accepted, "n_accepted", S),
+           (next_token, "next_token", S))
     _check(ctx, lib.sph_verify_draft(
         ctx, _ptr(target_logits), sessions, k, _ptr(keep_ids), n,
         float(temperature), _ptr(draft_tokens), _ptr(draft_probs),

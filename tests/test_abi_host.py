@@ -142,3 +142,25 @@ def test_check_keep_ids_against_the_conventions(sph):
         bad[j] = V + int(rng.integers(0, 3))
         good, at = sph.sph_check_keep_ids(bad, V)
         assert not good and at <= j
+
+
+def test_binding_refuses_buffers_the_kernels_would_leave(sph):
+    # the kernels index codes, scales, tokens, fused logits, id lists and
+    # the verification's inputs densely: the binding refuses a buffer that
+    # is on another device, strided, or smaller than the call needs, before
+    # anything reaches the library; operands with a row stride are checked
+    # for their device only
+    import torch
+    cpu = torch.device("cpu")
+    ok = torch.empty(4, 300)
+    sph._dense(cpu, (ok, "z", 4 * 300), (torch.empty(5, 300), "bigger", 4 * 300),
+               (None, "absent", 10), (torch.empty(4, 600)[:, :300], "W", None),
+               (torch.empty(2, 0), "empty", 0))
+    bad = [(torch.empty(4, 300, device="meta"), 4 * 300, "not on"),
+           (torch.empty(4, 8, device="meta")[:, :4], None, "not on"),
+           (torch.empty(300, 4).t(), 4 * 300, "contiguous"),
+           (torch.empty(8)[::2], 4, "contiguous"),
+           (torch.empty(3, 300), 4 * 300, "elements")]
+    for t, count, what in bad:
+        with pytest.raises(ValueError, match=what):
+            sph._dense(cpu, (t, "x", count))
