@@ -81,7 +81,9 @@ sph_status sph_destroy(sph_ctx* ctx);
  * stream is made to wait (an event, no host synchronization) for the work
  * already issued on the old one, since the next call reuses the context's
  * scratch.  While either stream is being captured into a CUDA graph no
- * ordering is added: the caller orders the two streams itself. */
+ * ordering is added: the caller orders the two streams itself.  The old
+ * stream must not have been destroyed (as for sph_destroy and sph_sync,
+ * which wait on the context's stream). */
 sph_status sph_set_stream(sph_ctx* ctx, void* cuda_stream);
 
 /* Wait for all work of the context's stream; report device-side errors
