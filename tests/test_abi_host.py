@@ -164,3 +164,21 @@ def test_binding_refuses_buffers_the_kernels_would_leave(sph):
     for t, count, what in bad:
         with pytest.raises(ValueError, match=what):
             sph._dense(cpu, (t, "x", count))
+
+
+def test_binding_constants_match_the_header(sph):
+    # every option, activation mode and weight type the binding mirrors has
+    # the header's value, every option of the header is mirrored, and every
+    # option name bench.py accepts (--opt NAME=VALUE) resolves to one of them
+    import bench
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    header = {m.group(1): int(m.group(2))
+              for m in re.finditer(r"\b(SPH_[A-Z0-9_]+)\s*=\s*(\d+)", text)}
+    mirrored = {k: v for k, v in vars(sph).items()
+                if k.startswith(("SPH_OPT_", "SPH_ACT_", "SPH_DTYPE_")) and isinstance(v, int)}
+    assert mirrored
+    for name, value in mirrored.items():
+        assert header.get(name) == value, (name, value, header.get(name))
+    options = {k for k in header if k.startswith("SPH_OPT_")}
+    assert options == {k for k in mirrored if k.startswith("SPH_OPT_")}
+    assert set(bench.OPTION_NAMES.values()) <= options
