@@ -182,3 +182,32 @@ def test_binding_constants_match_the_header(sph):
     options = {k for k in header if k.startswith("SPH_OPT_")}
     assert options == {k for k in mirrored if k.startswith("SPH_OPT_")}
     assert set(bench.OPTION_NAMES.values()) <= options
+
+
+def test_binding_structs_and_signatures_follow_the_header(sph):
+    # the ctypes mirrors of sph_plan and sph_profile have the header's
+    # fields in its order and types, and every bound function takes as many
+    # arguments as the header declares
+    import ctypes
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+
+    def struct_fields(name):
+        body = re.search(r"typedef struct %s \{(.*?)\}" % name, text, flags=re.S).group(1)
+        return re.findall(r"(\w+)\s+(\w+)(?:\[(\w+)\])?\s*;", body)
+
+    assert [(t, f) for t, f, _ in struct_fields("sph_plan")] == \
+        [("int32_t", f) for f in sph.PLAN_FIELDS]
+    assert [f for f, _ in sph.sph_plan._fields_] == list(sph.PLAN_FIELDS)
+    n_classes = int(re.search(r"\bSPH_PROF_CLASSES\s*=\s*(\d+)", text).group(1))
+    assert sph.PROF_CLASSES == n_classes
+    assert struct_fields("sph_profile") == [("double", "ms", "SPH_PROF_CLASSES"),
+                                            ("int64_t", "calls", "SPH_PROF_CLASSES"),
+                                            ("int64_t", "launches", "")]
+    assert [(f, t) for f, t in sph.sph_profile._fields_] == [
+        ("ms", ctypes.c_double * n_classes), ("calls", ctypes.c_int64 * n_classes),
+        ("launches", ctypes.c_int64)]
+    for fn, (_, argtypes) in sph._SIGNATURES.items():
+        m = re.search(r"\b%s\s*\(([^)]*)\)\s*;" % fn, text)
+        assert m, fn
+        params = [p for p in m.group(1).split(",") if p.strip() and p.strip() != "void"]
+        assert len(params) == len(argtypes), (fn, len(params), len(argtypes))
